@@ -1,0 +1,181 @@
+/*
+ * rfq.h -- C ABI of the GB300 (sm_103a) Residual Fallback Quantization
+ * (RFQ) linear layer: "Activation Outliers Matter: Robust Recovery for
+ * Quantized Multimodal LLMs", Sec. 3.2-3.3 (formats), Sec. 4.3 and
+ * Algorithm 1 (method).
+ *
+ * The layer computes Y = X W for an activation X [M x K] (bf16) and a weight
+ * W [K x N] (bf16) as
+ *
+ *     Y = Q(X) Q(W) + phi * Q(X - Q(X)) Q(W)                  (Eq. rfq)
+ *
+ * where Q is a block quantizer to a 4-bit format (MXFP4 or HiF4) along K.
+ * The paper writes Z = X Y with X [P x R], Y [R x Q]; here P = M, R = K,
+ * Q = N and the paper's Y is W.
+ *
+ * Conventions shared by every entry point:
+ *   - Every pointer named "device" is CUDA device memory on the current
+ *     device, allocated and owned by the caller; the library never allocates
+ *     device memory and never frees a caller's buffer.
+ *   - Every device pointer must be 16-byte aligned (RFQ_ERR_ALIGNMENT).
+ *   - Calls are asynchronous: they validate the arguments on the host,
+ *     enqueue kernels on `stream` (a cudaStream_t; NULL = legacy default
+ *     stream) and return.  On any argument error nothing is launched.
+ *   - bf16 inputs must be finite; non-finite inputs give unspecified codes
+ *     but never a fault.
+ *   - The library needs an sm_103 device (GB300); otherwise RFQ_ERR_DEVICE.
+ *
+ * Storage of a quantized matrix (rfq_qtensor), rows x k, quantized along k:
+ *   codes   [rows][k/2] bytes; element 2j of a row in the low nibble of byte
+ *           j, element 2j+1 in the high nibble.
+ *   MXFP4   E2M1 codes (sign, 2 exponent bits, 1 mantissa bit, Sec. 3.2.2)
+ *           with one E8M0 scale byte 2^(byte-127) per 32 elements
+ *           (Sec. 3.2 Eq. 3-4).  Scale layouts:
+ *             RFQ_SCALE_ROWMAJOR  [rows][k/32] bytes (k % 32 == 0)
+ *             RFQ_SCALE_MMA       the tensor-core layout consumed by
+ *               rfq_linear (k % 128 == 0): rows padded to a multiple of 128
+ *               and split into 512-byte atoms of 128 rows x 4 k-blocks; the
+ *               byte for (row m, k-block b) lives at
+ *                 ((m/128) * (k/128) + b/4) * 512 + (m%32)*16 + ((m/32)%4)*4 + b%4
+ *               Bytes of padding rows (m >= rows) are 0.
+ *   HiF4    S1P2 codes (sign, 1 integer bit, 2 fraction bits) with one
+ *           32-bit metadata word per 64 elements (Sec. 3.3):
+ *           bits [7:0] UE6M2 macro scale (E in [7:2], bias 48; M in [1:0]),
+ *           bits [15:8] E1_8 (bit g: group of 8 elements g),
+ *           bits [31:16] E1_16 (bit j: sub-group of 4 elements j).
+ *           Scale array: [rows][k/64] uint32 (k % 64 == 0).
+ */
+#ifndef RFQ_H
+#define RFQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define RFQ_API __attribute__((visibility("default")))
+#else
+#define RFQ_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    RFQ_OK = 0,
+    RFQ_ERR_INVALID_ARG = 1, /* NULL pointer or an enum value out of range */
+    RFQ_ERR_SHAPE = 2,       /* sizes violate the call's constraints */
+    RFQ_ERR_ALIGNMENT = 3,   /* a device pointer is not 16-byte aligned */
+    RFQ_ERR_UNSUPPORTED = 4, /* valid but unimplemented combination */
+    RFQ_ERR_CUDA = 5,        /* a CUDA runtime call or a launch failed */
+    RFQ_ERR_TIMEOUT = 6,     /* a kernel's bounded wait expired (device status) */
+    RFQ_ERR_DEVICE = 7       /* the current device is not an sm_103 GPU */
+} rfq_status;
+
+typedef enum { RFQ_FMT_MXFP4 = 0, RFQ_FMT_HIF4 = 1 } rfq_format;
+
+typedef enum { RFQ_SCALE_ROWMAJOR = 0, RFQ_SCALE_MMA = 1 } rfq_scale_layout;
+
+/* Fallback indicator phi(p, r) of Sec. 4.3 over tiles of p_s rows x r_s
+ * columns of X.  The paper gives no formula for it:
+ *   RFQ_FALLBACK_NONE  phi = 0: plain W4A4, no residual pathway
+ *   RFQ_FALLBACK_ALL   phi = 1 on every tile (the default; Sec. 1 describes
+ *                      RFQ as working without threshold-based selection)
+ *   RFQ_FALLBACK_AMAX  phi(p, r) = 1 iff max |x| over the tile > tau */
+typedef enum {
+    RFQ_FALLBACK_NONE = 0,
+    RFQ_FALLBACK_ALL = 1,
+    RFQ_FALLBACK_AMAX = 2
+} rfq_fallback_mode;
+
+typedef enum { RFQ_OUT_F32 = 0, RFQ_OUT_BF16 = 1 } rfq_out_dtype;
+
+typedef struct {
+    int32_t fmt;          /* rfq_format */
+    int32_t scale_layout; /* rfq_scale_layout; HiF4 uses RFQ_SCALE_ROWMAJOR */
+    int64_t rows;         /* M for an activation, N for a weight */
+    int64_t k;            /* length of the quantized (reduction) axis */
+    void *codes;          /* device, see "Storage" above */
+    void *scales;         /* device, see "Storage" above */
+} rfq_qtensor;
+
+typedef struct {
+    int32_t mode; /* rfq_fallback_mode */
+    float tau;    /* threshold for RFQ_FALLBACK_AMAX */
+    int32_t p_s;  /* tile rows (>= 1); rfq_linear reads phi tiles of 128 rows */
+    int32_t r_s;  /* tile columns, a multiple of 32; rfq_linear needs a multiple of 128 */
+} rfq_fallback;
+
+/* Human-readable name of a status code (static string, never NULL). */
+RFQ_API const char *rfq_status_string(rfq_status s);
+
+/* Byte sizes of the code and scale arrays of a rows x k quantized matrix in
+ * the given format and scale layout (host only, no device work).
+ * Errors: RFQ_ERR_INVALID_ARG (NULL outputs, bad enums), RFQ_ERR_SHAPE
+ * (rows < 0, k not a multiple of the layout's granule). */
+RFQ_API rfq_status rfq_qtensor_bytes(int32_t fmt, int32_t scale_layout, int64_t rows, int64_t k,
+                             size_t *codes_bytes, size_t *scale_bytes);
+
+/* Weight quantization W~ = Q(W) (Sec. 4.3; Algorithm 1 quantizes every
+ * weight block).  W: device bf16 [K][N] row-major.  out->fmt,
+ * out->scale_layout, out->codes and out->scales are set by the caller and
+ * out->rows must equal N, out->k must equal K; codes are written K-major
+ * ([N][K/2]).  Meant to run once per weight, off the hot path.
+ * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
+ * RFQ_ERR_UNSUPPORTED, RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */
+RFQ_API rfq_status rfq_quantize_weight(const void *w_bf16, int64_t K, int64_t N, rfq_qtensor *out,
+                               void *stream);
+
+/* RFQ activation decomposition in one pass over X (Sec. 4.3, Algorithm 1):
+ *   X~ = Q(X), dX = X - X~, X^ = Q(dX) where phi = 1 (same format, Sec. 4.3),
+ * with the E8M0 scale floor(log2 amax) - 2 clamped to [-127, 127] and
+ * round-to-nearest-even, saturating element rounding (MXFP4); HiF4 per its
+ * encoder.  X: device bf16 [M][K] row-major.  xq: main pathway output,
+ * xr: residual pathway output (both with rows = M, k = K and the same fmt
+ * and layout); xr may be NULL only when fb->mode == RFQ_FALLBACK_NONE.
+ * Residual codes and scales of tiles with phi = 0 are written as zero.
+ * phi: device bytes [ceil(M/p_s)][ceil(K/r_s)], may be NULL; fb may be
+ * NULL (= RFQ_FALLBACK_ALL).  M may be 0 (nothing is launched).
+ * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
+ * RFQ_ERR_UNSUPPORTED, RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */
+RFQ_API rfq_status rfq_quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_fallback *fb,
+                            rfq_qtensor *xq, rfq_qtensor *xr, uint8_t *phi, void *stream);
+
+/* Bytes of device workspace rfq_linear needs (a status word, padded). */
+RFQ_API size_t rfq_linear_workspace_bytes(void);
+
+/* RFQ GEMM (Algorithm 1, Eq. rfq): Y = X~ W~ + phi X^ W~ with both products
+ * accumulated into one fp32 accumulator per output tile, the weight tile read
+ * once for both.  xq: [M x K] main codes; xr: [M x K] residual codes or NULL
+ * (plain W4A4); phi: device bytes [ceil(M/128)][K/r_s] selecting the
+ * residual k-tiles per 128-row tile, or NULL (= all ones); phi_r_s: the
+ * column tile r_s of phi (a multiple of 128; ignored when phi is NULL).
+ * wq: [N x K] weight codes.  MXFP4 operands must use RFQ_SCALE_MMA;
+ * requirements: K % 128 == 0 (MXFP4) or K % 64 == 0 (HiF4), N % 16 == 0,
+ * M >= 0.  y: device [M][N] row-major fp32 or bf16 (round-to-nearest-even
+ * of the fp32 accumulator).  workspace: device, rfq_linear_workspace_bytes()
+ * bytes, zeroed by the caller once; a kernel that gives up a bounded wait
+ * records a timeout there (read it with rfq_workspace_status).  The record
+ * is sticky: later calls with that workspace return without computing until
+ * it is cleared.
+ * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
+ * RFQ_ERR_UNSUPPORTED, RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */
+RFQ_API rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_t *phi,
+                      int32_t phi_r_s, const rfq_qtensor *wq, void *y, int32_t out_dtype,
+                      void *workspace, void *stream);
+
+/* Synchronizes `stream` and returns the device status left in a workspace by
+ * earlier calls (RFQ_OK or RFQ_ERR_TIMEOUT); clears it when `clear` != 0. */
+RFQ_API rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *stream);
+
+/* Dequantization x = code value * scale (Sec. 3.2 Eq. 4; Sec. 3.3 V_i) of a
+ * quantized matrix into device fp32 out[rows][k].
+ * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
+ * RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */
+RFQ_API rfq_status rfq_dequant(const rfq_qtensor *q, float *out, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RFQ_H */

@@ -13,6 +13,7 @@ from __future__ import annotations
 
 import ctypes
 import os
+import platform
 import subprocess
 
 import numpy as np
@@ -25,7 +26,7 @@ PHI_AMAX = 2
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "rfq_oracle.c")
-_LIB = os.path.join(_HERE, "librfq_oracle.so")
+_LIB = os.path.join(_HERE, f"librfq_oracle.{platform.machine()}.so")
 _lib = None
 
 

@@ -1,0 +1,301 @@
+// api.cu -- the C ABI declared in include/rfq.h: argument validation,
+// tensor-map encoding and kernel dispatch.  No entry point allocates device
+// memory; every buffer belongs to the caller.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+#include <mutex>
+
+#include "internal.h"
+
+namespace rfq {
+namespace {
+
+typedef CUresult (*PFN_encodeTiled)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                    const cuuint64_t *, const cuuint32_t *, const cuuint32_t *,
+                                    CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                    CUtensorMapFloatOOBfill);
+
+PFN_encodeTiled get_encode()
+{
+    static PFN_encodeTiled fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_encodeTiled>(p);
+    });
+    return fn;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+rfq_status check_device()
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess)
+        return RFQ_ERR_DEVICE;
+    static int cache[64];   // 0 unknown, 1 ok, 2 not sm_103
+    if (dev < 0 || dev >= 64)
+        return RFQ_ERR_DEVICE;
+    if (cache[dev] == 0) {
+        int major = 0, minor = 0;
+        if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+            return RFQ_ERR_DEVICE;
+        cache[dev] = (major == 10 && minor == 3) ? 1 : 2;
+    }
+    return cache[dev] == 1 ? RFQ_OK : RFQ_ERR_DEVICE;
+}
+
+rfq_status from_cuda(cudaError_t e) { return e == cudaSuccess ? RFQ_OK : RFQ_ERR_CUDA; }
+
+bool fmt_ok(int32_t f) { return f == RFQ_FMT_MXFP4 || f == RFQ_FMT_HIF4; }
+bool layout_ok(int32_t l) { return l == RFQ_SCALE_ROWMAJOR || l == RFQ_SCALE_MMA; }
+
+// Granule of the k axis for a format / scale layout.
+int64_t k_granule(int32_t fmt, int32_t layout)
+{
+    if (fmt == RFQ_FMT_HIF4)
+        return 64;
+    return layout == RFQ_SCALE_MMA ? 128 : 32;
+}
+
+rfq_status check_qtensor(const rfq_qtensor *q, int64_t rows, int64_t k)
+{
+    if (!q || !fmt_ok(q->fmt) || !layout_ok(q->scale_layout))
+        return RFQ_ERR_INVALID_ARG;
+    if (q->fmt == RFQ_FMT_HIF4 && q->scale_layout != RFQ_SCALE_ROWMAJOR)
+        return RFQ_ERR_INVALID_ARG;
+    if (q->rows != rows || q->k != k || rows < 0 || k <= 0 || k % k_granule(q->fmt, q->scale_layout) != 0)
+        return RFQ_ERR_SHAPE;
+    if (rows > 0 && (!q->codes || !q->scales))
+        return RFQ_ERR_INVALID_ARG;
+    if (!aligned16(q->codes) || !aligned16(q->scales))
+        return RFQ_ERR_ALIGNMENT;
+    return RFQ_OK;
+}
+
+} // namespace
+
+bool encode_tmap_2d_u8(CUtensorMap *map, const void *base, uint64_t inner_bytes, uint64_t rows,
+                       uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows, bool swizzle128)
+{
+    PFN_encodeTiled enc = get_encode();
+    if (!enc)
+        return false;
+    cuuint64_t dims[2] = {inner_bytes, rows};
+    cuuint64_t strides[1] = {row_stride_bytes};
+    cuuint32_t box[2] = {box_inner, box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE,
+                     swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+} // namespace rfq
+
+using namespace rfq;
+
+extern "C" {
+
+const char *rfq_status_string(rfq_status s)
+{
+    switch (s) {
+    case RFQ_OK: return "RFQ_OK";
+    case RFQ_ERR_INVALID_ARG: return "RFQ_ERR_INVALID_ARG: null pointer or enum out of range";
+    case RFQ_ERR_SHAPE: return "RFQ_ERR_SHAPE: sizes violate the call's constraints";
+    case RFQ_ERR_ALIGNMENT: return "RFQ_ERR_ALIGNMENT: device pointer not 16-byte aligned";
+    case RFQ_ERR_UNSUPPORTED: return "RFQ_ERR_UNSUPPORTED: combination not implemented";
+    case RFQ_ERR_CUDA: return "RFQ_ERR_CUDA: CUDA runtime call or launch failed";
+    case RFQ_ERR_TIMEOUT: return "RFQ_ERR_TIMEOUT: a kernel's bounded wait expired";
+    case RFQ_ERR_DEVICE: return "RFQ_ERR_DEVICE: current device is not an sm_103 GPU";
+    }
+    return "RFQ_ERR_UNKNOWN";
+}
+
+rfq_status rfq_qtensor_bytes(int32_t fmt, int32_t scale_layout, int64_t rows, int64_t k, size_t *codes_bytes,
+                             size_t *scale_bytes)
+{
+    if (!codes_bytes || !scale_bytes || !fmt_ok(fmt) || !layout_ok(scale_layout))
+        return RFQ_ERR_INVALID_ARG;
+    if (fmt == RFQ_FMT_HIF4 && scale_layout != RFQ_SCALE_ROWMAJOR)
+        return RFQ_ERR_INVALID_ARG;
+    if (rows < 0 || k <= 0 || k % k_granule(fmt, scale_layout) != 0)
+        return RFQ_ERR_SHAPE;
+    *codes_bytes = (size_t)rows * (size_t)(k / 2);
+    if (fmt == RFQ_FMT_HIF4)
+        *scale_bytes = (size_t)rows * (size_t)(k / 64) * 4;
+    else if (scale_layout == RFQ_SCALE_MMA)
+        *scale_bytes = (size_t)((rows + 127) / 128) * 128 * (size_t)(k / 32);
+    else
+        *scale_bytes = (size_t)rows * (size_t)(k / 32);
+    return RFQ_OK;
+}
+
+rfq_status rfq_quantize_weight(const void *w_bf16, int64_t K, int64_t N, rfq_qtensor *out, void *stream)
+{
+    if (!w_bf16 || !out)
+        return RFQ_ERR_INVALID_ARG;
+    if (K <= 0 || N < 0)
+        return RFQ_ERR_SHAPE;
+    rfq_status s = check_qtensor(out, N, K);
+    if (s != RFQ_OK)
+        return s;
+    if (!aligned16(w_bf16))
+        return RFQ_ERR_ALIGNMENT;
+    if ((s = check_device()) != RFQ_OK)
+        return s;
+    if (N == 0)
+        return RFQ_OK;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (out->fmt == RFQ_FMT_MXFP4)
+        return from_cuda(launch_weight_quant_mxfp4(w_bf16, K, N, out->codes, out->scales, out->scale_layout, st));
+    return RFQ_ERR_UNSUPPORTED;
+}
+
+rfq_status rfq_quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_fallback *fb, rfq_qtensor *xq,
+                            rfq_qtensor *xr, uint8_t *phi, void *stream)
+{
+    rfq_fallback def = {RFQ_FALLBACK_ALL, 0.f, 128, 256};
+    const rfq_fallback &f = fb ? *fb : def;
+    if (!x_bf16 || !xq)
+        return RFQ_ERR_INVALID_ARG;
+    if (f.mode < RFQ_FALLBACK_NONE || f.mode > RFQ_FALLBACK_AMAX)
+        return RFQ_ERR_INVALID_ARG;
+    if (M < 0 || K <= 0)
+        return RFQ_ERR_SHAPE;
+    rfq_status s = check_qtensor(xq, M, K);
+    if (s != RFQ_OK)
+        return s;
+    const bool res = f.mode != RFQ_FALLBACK_NONE;
+    if (res) {
+        if (!xr)
+            return RFQ_ERR_INVALID_ARG;
+        if ((s = check_qtensor(xr, M, K)) != RFQ_OK)
+            return s;
+        if (xr->fmt != xq->fmt || xr->scale_layout != xq->scale_layout)
+            return RFQ_ERR_INVALID_ARG;
+    }
+    if (f.p_s < 1 || f.r_s < 32 || f.r_s % 32 != 0)
+        return RFQ_ERR_SHAPE;
+    if (f.mode == RFQ_FALLBACK_AMAX && !phi)
+        return RFQ_ERR_INVALID_ARG;
+    if (!aligned16(x_bf16))
+        return RFQ_ERR_ALIGNMENT;
+    if ((s = check_device()) != RFQ_OK)
+        return s;
+    if (M == 0)
+        return RFQ_OK;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (xq->fmt == RFQ_FMT_MXFP4)
+        return from_cuda(launch_act_quant_mxfp4(x_bf16, M, K, f.mode, f.tau, f.p_s, f.r_s, xq->codes, xq->scales,
+                                                res ? xr->codes : nullptr, res ? xr->scales : nullptr, phi,
+                                                xq->scale_layout, st));
+    return RFQ_ERR_UNSUPPORTED;
+}
+
+size_t rfq_linear_workspace_bytes(void) { return 256; }
+
+rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_t *phi, int32_t phi_r_s,
+                      const rfq_qtensor *wq, void *y, int32_t out_dtype, void *workspace, void *stream)
+{
+    if (!xq || !wq || !y || !workspace)
+        return RFQ_ERR_INVALID_ARG;
+    if (out_dtype != RFQ_OUT_F32 && out_dtype != RFQ_OUT_BF16)
+        return RFQ_ERR_INVALID_ARG;
+    const int64_t M = xq->rows, K = xq->k, N = wq->rows;
+    if (M < 0 || N < 0 || K <= 0 || wq->k != K)
+        return RFQ_ERR_SHAPE;
+    rfq_status s = check_qtensor(xq, M, K);
+    if (s != RFQ_OK)
+        return s;
+    if ((s = check_qtensor(wq, N, K)) != RFQ_OK)
+        return s;
+    if (xr) {
+        if ((s = check_qtensor(xr, M, K)) != RFQ_OK)
+            return s;
+        if (xr->fmt != xq->fmt || xr->scale_layout != xq->scale_layout)
+            return RFQ_ERR_INVALID_ARG;
+    }
+    if (wq->fmt != xq->fmt)
+        return RFQ_ERR_INVALID_ARG;
+    if (N % 16 != 0)
+        return RFQ_ERR_SHAPE;
+    if (M > (int64_t)INT32_MAX || N > (int64_t)INT32_MAX || K > (int64_t)INT32_MAX)
+        return RFQ_ERR_SHAPE;
+    if (phi && xr && (phi_r_s < 128 || phi_r_s % 128 != 0))
+        return RFQ_ERR_SHAPE;
+    if (!aligned16(y) || !aligned16(workspace))
+        return RFQ_ERR_ALIGNMENT;
+    if ((s = check_device()) != RFQ_OK)
+        return s;
+    if (M == 0 || N == 0)
+        return RFQ_OK;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (xq->fmt == RFQ_FMT_MXFP4) {
+        if (xq->scale_layout != RFQ_SCALE_MMA || wq->scale_layout != RFQ_SCALE_MMA)
+            return RFQ_ERR_UNSUPPORTED;
+        GemmMxf4Args a;
+        a.a_codes = xq->codes;
+        a.a_sf = xq->scales;
+        a.r_codes = xr ? xr->codes : nullptr;
+        a.r_sf = xr ? xr->scales : nullptr;
+        a.b_codes = wq->codes;
+        a.b_sf = wq->scales;
+        a.phi = xr ? phi : nullptr;
+        a.phi_r_s = phi_r_s;
+        a.y = y;
+        a.out_bf16 = out_dtype == RFQ_OUT_BF16;
+        a.M = M;
+        a.N = N;
+        a.K = K;
+        a.status = static_cast<int32_t *>(workspace);
+        return from_cuda(launch_gemm_mxf4(a, st));
+    }
+    return RFQ_ERR_UNSUPPORTED;
+}
+
+rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *stream)
+{
+    if (!workspace)
+        return RFQ_ERR_INVALID_ARG;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int32_t v = 0;
+    if (cudaMemcpyAsync(&v, workspace, sizeof v, cudaMemcpyDeviceToHost, st) != cudaSuccess)
+        return RFQ_ERR_CUDA;
+    if (cudaStreamSynchronize(st) != cudaSuccess)
+        return RFQ_ERR_CUDA;
+    if (clear && v != kDevOk) {
+        if (cudaMemsetAsync(workspace, 0, sizeof(int32_t), st) != cudaSuccess)
+            return RFQ_ERR_CUDA;
+    }
+    return v == kDevOk ? RFQ_OK : RFQ_ERR_TIMEOUT;
+}
+
+rfq_status rfq_dequant(const rfq_qtensor *q, float *out, void *stream)
+{
+    if (!q || !out)
+        return RFQ_ERR_INVALID_ARG;
+    rfq_status s = check_qtensor(q, q->rows, q->k);
+    if (s != RFQ_OK)
+        return s;
+    if (!aligned16(out))
+        return RFQ_ERR_ALIGNMENT;
+    if ((s = check_device()) != RFQ_OK)
+        return s;
+    if (q->rows == 0)
+        return RFQ_OK;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (q->fmt == RFQ_FMT_MXFP4)
+        return from_cuda(launch_dequant_mxfp4(q->codes, q->scales, q->rows, q->k, q->scale_layout, out, st));
+    return RFQ_ERR_UNSUPPORTED;
+}
+
+} // extern "C"

@@ -1,0 +1,53 @@
+// internal.h -- launchers shared between the C-ABI layer and the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "../../include/rfq.h"
+
+namespace rfq {
+
+// Device status word values written into a workspace by kernels.
+constexpr int32_t kDevOk = 0;
+constexpr int32_t kDevTimeout = 1;
+
+// Bounded waits in the GEMM give up after this many nanoseconds.
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+
+// Byte offset of E8M0 scale (row m, 32-element block b) in the MMA layout
+// (512-byte atoms of 128 rows x 4 blocks; kc = K / 128 atoms per row band).
+__host__ __device__ inline int64_t sf_mma_offset(int64_t m, int64_t b, int64_t kc)
+{
+    return (((m >> 7) * kc + (b >> 2)) << 9) + ((m & 31) << 4) + (((m >> 5) & 3) << 2) + (b & 3);
+}
+
+// ---- MXFP4 quantization (quant_mxfp4.cu)
+// Activation: main (+ residual) codes and scales in one pass over X.
+cudaError_t launch_act_quant_mxfp4(const void *x, int64_t M, int64_t K, int mode, float tau, int p_s, int r_s,
+                                   void *mcodes, void *mscales, void *rcodes, void *rscales, uint8_t *phi,
+                                   int layout, cudaStream_t st);
+cudaError_t launch_weight_quant_mxfp4(const void *w, int64_t K, int64_t N, void *codes, void *scales, int layout,
+                                      cudaStream_t st);
+cudaError_t launch_dequant_mxfp4(const void *codes, const void *scales, int64_t rows, int64_t k, int layout,
+                                 float *out, cudaStream_t st);
+
+// ---- MXFP4 RFQ GEMM (gemm_mxf4.cu)
+struct GemmMxf4Args {
+    const void *a_codes, *r_codes, *b_codes;   // [M][K/2], [M][K/2] or null, [N][K/2]
+    const void *a_sf, *r_sf, *b_sf;            // MMA-layout scales
+    const uint8_t *phi;                        // [ceil(M/128)][K/phi_r_s] or null
+    int phi_r_s;
+    void *y;
+    int out_bf16;
+    int64_t M, N, K;
+    int32_t *status;
+};
+cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st);
+
+// ---- tensor maps (api.cu)
+bool encode_tmap_2d_u8(CUtensorMap *map, const void *base, uint64_t inner_bytes, uint64_t rows,
+                       uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows, bool swizzle128);
+
+} // namespace rfq

@@ -1,0 +1,165 @@
+"""ctypes binding of ``librfq.so`` (declared in ``include/rfq.h``).
+
+Argument marshalling only: every step of the RFQ path runs in the library's
+CUDA kernels.  PyTorch provides device memory and streams.  There is no CPU
+fallback: if the library is missing or fails to load, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "librfq.so")
+
+RFQ_OK = 0
+RFQ_FMT_MXFP4, RFQ_FMT_HIF4 = 0, 1
+RFQ_SCALE_ROWMAJOR, RFQ_SCALE_MMA = 0, 1
+RFQ_FALLBACK_NONE, RFQ_FALLBACK_ALL, RFQ_FALLBACK_AMAX = 0, 1, 2
+RFQ_OUT_F32, RFQ_OUT_BF16 = 0, 1
+STATUS_NAMES = {0: "RFQ_OK", 1: "RFQ_ERR_INVALID_ARG", 2: "RFQ_ERR_SHAPE", 3: "RFQ_ERR_ALIGNMENT",
+                4: "RFQ_ERR_UNSUPPORTED", 5: "RFQ_ERR_CUDA", 6: "RFQ_ERR_TIMEOUT", 7: "RFQ_ERR_DEVICE"}
+
+EXPORTED = ("rfq_status_string", "rfq_qtensor_bytes", "rfq_quantize_weight", "rfq_quantize_act",
+            "rfq_linear_workspace_bytes", "rfq_linear", "rfq_workspace_status", "rfq_dequant")
+
+
+class RFQError(RuntimeError):
+    def __init__(self, status: int, call: str):
+        self.status = status
+        super().__init__(f"{call}: {STATUS_NAMES.get(status, status)}")
+
+
+class _QT(ctypes.Structure):
+    _fields_ = [("fmt", ctypes.c_int32), ("scale_layout", ctypes.c_int32), ("rows", ctypes.c_int64),
+                ("k", ctypes.c_int64), ("codes", ctypes.c_void_p), ("scales", ctypes.c_void_p)]
+
+
+class _FB(ctypes.Structure):
+    _fields_ = [("mode", ctypes.c_int32), ("tau", ctypes.c_float), ("p_s", ctypes.c_int32),
+                ("r_s", ctypes.c_int32)]
+
+
+_lib = None
+
+
+def load_library(path: str = LIB_PATH):
+    """Load librfq.so; raises if it has not been built (no fallback)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(path):
+            raise RuntimeError(f"{path} is missing: build it with paper_2608_26581_gb300._build.build()")
+        lib = ctypes.CDLL(path)
+        P, I32, I64, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
+        QTP = ctypes.POINTER(_QT)
+        lib.rfq_status_string.restype = ctypes.c_char_p
+        lib.rfq_status_string.argtypes = [I32]
+        lib.rfq_qtensor_bytes.restype = I32
+        lib.rfq_qtensor_bytes.argtypes = [I32, I32, I64, I64, ctypes.POINTER(SZ), ctypes.POINTER(SZ)]
+        lib.rfq_quantize_weight.restype = I32
+        lib.rfq_quantize_weight.argtypes = [P, I64, I64, QTP, P]
+        lib.rfq_quantize_act.restype = I32
+        lib.rfq_quantize_act.argtypes = [P, I64, I64, ctypes.POINTER(_FB), QTP, QTP, P, P]
+        lib.rfq_linear_workspace_bytes.restype = SZ
+        lib.rfq_linear_workspace_bytes.argtypes = []
+        lib.rfq_linear.restype = I32
+        lib.rfq_linear.argtypes = [QTP, QTP, P, I32, QTP, P, I32, P, P]
+        lib.rfq_workspace_status.restype = I32
+        lib.rfq_workspace_status.argtypes = [P, I32, P]
+        lib.rfq_dequant.restype = I32
+        lib.rfq_dequant.argtypes = [QTP, P, P]
+        _lib = lib
+    return _lib
+
+
+def _check(status: int, call: str):
+    if status != RFQ_OK:
+        raise RFQError(status, call)
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+@dataclass
+class QTensor:
+    """A quantized rows x k matrix: device ``codes`` and ``scales`` tensors."""
+    fmt: int
+    scale_layout: int
+    rows: int
+    k: int
+    codes: torch.Tensor
+    scales: torch.Tensor
+
+    def c(self) -> _QT:
+        return _QT(self.fmt, self.scale_layout, self.rows, self.k,
+                   self.codes.data_ptr(), self.scales.data_ptr())
+
+
+def rfq_status_string(status: int) -> str:
+    return load_library().rfq_status_string(status).decode()
+
+
+def rfq_qtensor_bytes(fmt: int, scale_layout: int, rows: int, k: int):
+    cb, sb = ctypes.c_size_t(), ctypes.c_size_t()
+    _check(load_library().rfq_qtensor_bytes(fmt, scale_layout, rows, k, ctypes.byref(cb), ctypes.byref(sb)),
+           "rfq_qtensor_bytes")
+    return cb.value, sb.value
+
+
+def empty_qtensor(fmt: int, scale_layout: int, rows: int, k: int, device="cuda") -> QTensor:
+    """Allocate (with torch) the buffers of a quantized matrix."""
+    cb, sb = rfq_qtensor_bytes(fmt, scale_layout, rows, k)
+    return QTensor(fmt, scale_layout, rows, k,
+                   torch.empty(max(cb, 16), dtype=torch.uint8, device=device),
+                   torch.empty(max(sb, 16), dtype=torch.uint8, device=device))
+
+
+def rfq_quantize_weight(w: torch.Tensor, out: QTensor, stream=None):
+    K, N = w.shape
+    qt = out.c()
+    _check(load_library().rfq_quantize_weight(_ptr(w), K, N, ctypes.byref(qt), _stream(stream)),
+           "rfq_quantize_weight")
+
+
+def rfq_quantize_act(x: torch.Tensor, xq: QTensor, xr: QTensor | None, phi: torch.Tensor | None = None,
+                     mode: int = RFQ_FALLBACK_ALL, tau: float = 0.0, p_s: int = 128, r_s: int = 256,
+                     stream=None):
+    M, K = x.shape
+    fb = _FB(mode, tau, p_s, r_s)
+    q = xq.c()
+    r = xr.c() if xr is not None else None
+    _check(load_library().rfq_quantize_act(_ptr(x), M, K, ctypes.byref(fb), ctypes.byref(q),
+                                           ctypes.byref(r) if r is not None else None, _ptr(phi),
+                                           _stream(stream)), "rfq_quantize_act")
+
+
+def rfq_linear_workspace_bytes() -> int:
+    return load_library().rfq_linear_workspace_bytes()
+
+
+def rfq_linear(xq: QTensor, xr: QTensor | None, phi: torch.Tensor | None, phi_r_s: int, wq: QTensor,
+               y: torch.Tensor, out_dtype: int, workspace: torch.Tensor, stream=None):
+    q, w = xq.c(), wq.c()
+    r = xr.c() if xr is not None else None
+    _check(load_library().rfq_linear(ctypes.byref(q), ctypes.byref(r) if r is not None else None, _ptr(phi),
+                                     phi_r_s, ctypes.byref(w), _ptr(y), out_dtype, _ptr(workspace),
+                                     _stream(stream)), "rfq_linear")
+
+
+def rfq_workspace_status(workspace: torch.Tensor, clear: bool = False, stream=None) -> int:
+    return load_library().rfq_workspace_status(_ptr(workspace), 1 if clear else 0, _stream(stream))
+
+
+def rfq_dequant(q: QTensor, out: torch.Tensor, stream=None):
+    qt = q.c()
+    _check(load_library().rfq_dequant(ctypes.byref(qt), _ptr(out), _stream(stream)), "rfq_dequant")

@@ -1,0 +1,57 @@
+"""Helpers shared by the GPU parity tests: device buffers, layout permutations
+of the library's scale arrays, and the tolerance checks."""
+import numpy as np
+import torch
+
+from paper_2608_26581_gb300 import rfq
+
+DEV = "cuda"
+
+
+def to_dev_bf16(bits: np.ndarray) -> torch.Tensor:
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).to(DEV).view(torch.bfloat16)
+
+
+def mma_scale_to_rowmajor(sf_bytes: np.ndarray, rows: int, k: int) -> np.ndarray:
+    """Undo the tensor-core scale layout: byte (m, b) sits at
+    ((m/128)*(k/128) + b/4)*512 + (m%32)*16 + ((m/32)%4)*4 + b%4."""
+    kb = k // 32
+    m = np.arange(rows)[:, None]
+    b = np.arange(kb)[None, :]
+    off = ((m // 128) * (k // 128) + b // 4) * 512 + (m % 32) * 16 + ((m // 32) % 4) * 4 + (b % 4)
+    return np.asarray(sf_bytes)[off]
+
+
+def qtensor_host(q: rfq.QTensor):
+    """(codes [rows, k/2] uint8, scales in the oracle's row-major form)."""
+    rows, k = q.rows, q.k
+    codes = q.codes[: rows * k // 2].cpu().numpy().reshape(rows, k // 2)
+    sf = q.scales.cpu().numpy()
+    if q.fmt == rfq.RFQ_FMT_HIF4:
+        scales = sf[: rows * (k // 64) * 4].view(np.uint32).reshape(rows, k // 64)
+    elif q.scale_layout == rfq.RFQ_SCALE_MMA:
+        scales = mma_scale_to_rowmajor(sf, rows, k)
+    else:
+        scales = sf[: rows * (k // 32)].reshape(rows, k // 32)
+    return codes, scales
+
+
+def check_y(y_gpu: np.ndarray, y_ref: np.ndarray, bf16: bool = False):
+    """Y tolerance.  fp32 output: relative Frobenius error <= 1e-5 and max abs
+    error <= 1e-3 max|Y|.  bf16 output adds the final rounding to bf16
+    (relative 2^-9 per element): relative Frobenius <= 2^-8 and max abs
+    <= 1e-3 max|Y| + 2^-8 |Y_ref|."""
+    y_gpu = np.asarray(y_gpu, np.float64)
+    ref = np.asarray(y_ref, np.float64)
+    nrm = np.linalg.norm(ref)
+    rel = np.linalg.norm(y_gpu - ref) / max(nrm, 1e-300)
+    amax = np.abs(ref).max()
+    err = np.abs(y_gpu - ref)
+    if bf16:
+        ok_abs = np.all(err <= 1e-3 * amax + 2.0 ** -8 * np.abs(ref))
+        assert rel <= 2.0 ** -8, f"bf16 rel Frobenius {rel:.3e}"
+    else:
+        ok_abs = np.all(err <= 1e-3 * amax)
+        assert rel <= 1e-5, f"rel Frobenius {rel:.3e}"
+    assert ok_abs, f"max abs err {err.max():.3e} vs max|Y| {amax:.3e}"
+    return rel

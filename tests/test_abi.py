@@ -1,0 +1,75 @@
+"""The C ABI library builds, loads and exports every entry point that
+include/rfq.h declares; host-side validation works without a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from conftest import ROOT
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_26581_gb300 import _build, rfq
+    _build.build()
+    return rfq.load_library()
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "rfq.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(rfq_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for n in ("rfq_quantize_weight", "rfq_quantize_act", "rfq_linear", "rfq_dequant"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    from paper_2608_26581_gb300 import rfq
+    for n in _declared():
+        assert hasattr(lib, n), n
+        assert n in rfq.EXPORTED, n
+
+
+def test_status_strings(lib):
+    from paper_2608_26581_gb300 import rfq
+    for code, name in rfq.STATUS_NAMES.items():
+        assert rfq.rfq_status_string(code).startswith(name)
+
+
+def test_qtensor_bytes(lib):
+    from paper_2608_26581_gb300 import rfq
+    assert rfq.rfq_qtensor_bytes(0, 0, 128, 512) == (128 * 256, 128 * 16)
+    assert rfq.rfq_qtensor_bytes(0, 1, 130, 512) == (130 * 256, 256 * 16)
+    assert rfq.rfq_qtensor_bytes(1, 0, 10, 640) == (10 * 320, 10 * 10 * 4)
+    # HiF4: 36 bytes per 64 elements (4.5 bits each)
+    cb, sb = rfq.rfq_qtensor_bytes(1, 0, 1, 64)
+    assert cb + sb == 36
+    with pytest.raises(rfq.RFQError) as e:
+        rfq.rfq_qtensor_bytes(0, 1, 128, 96)          # MMA layout needs k % 128
+    assert e.value.status == 2
+    with pytest.raises(rfq.RFQError) as e:
+        rfq.rfq_qtensor_bytes(1, 1, 128, 128)         # HiF4 has one layout
+    assert e.value.status == 1
+
+
+def test_workspace_bytes(lib):
+    from paper_2608_26581_gb300 import rfq
+    assert rfq.rfq_linear_workspace_bytes() >= 4
+
+
+def test_null_arguments_rejected_before_any_device_work(lib):
+    from paper_2608_26581_gb300 import rfq
+    assert lib.rfq_quantize_act(None, 1, 32, None, None, None, None, None) == 1
+    assert lib.rfq_quantize_weight(None, 32, 16, None, None) == 1
+    assert lib.rfq_linear(None, None, None, 0, None, None, 0, None, None) == 1
+    assert lib.rfq_dequant(None, None, None) == 1
+    qt = rfq._QT(0, 1, 128, 96, 16, 16)           # k not a multiple of 128 for the MMA layout
+    assert lib.rfq_quantize_act(ctypes.c_void_p(16), 128, 96, None, ctypes.byref(qt), ctypes.byref(qt),
+                                None, None) == 2
+    qt = rfq._QT(0, 0, 4, 64, 8, 16)              # misaligned codes pointer
+    assert lib.rfq_dequant(ctypes.byref(qt), ctypes.c_void_p(16), None) == 3
