@@ -129,9 +129,16 @@ def _dist():
     return ws, rank, local
 
 
-def _workload():
+def _workload(rows: int = 0):
+    """The benchmark workload; rows > 0 keeps only the first `rows` token
+    rows (a smaller case of the same kernels, for profiler captures)."""
+    import dataclasses
     from paper_2608_26581_gb300.synth import WORKLOADS
-    return WORKLOADS[WORKLOAD]
+    spec = WORKLOADS[WORKLOAD]
+    if rows and rows < spec.act.M:
+        spec = dataclasses.replace(spec, name=f"{spec.name}_first{rows}rows",
+                                   act=dataclasses.replace(spec.act, M=rows))
+    return spec
 
 
 def _config(spec, extra=None):
@@ -206,7 +213,7 @@ def run_rfq(args):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    spec = _workload()
+    spec = _workload(args.rows)
     M, K, N = spec.act.M, spec.act.K, spec.N
     F, L = rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA
 
@@ -267,7 +274,7 @@ def run_rfq(args):
 
     # end to end through the public API with host buffers
     e2e_ms = None
-    for i in range(args.warmup + args.steps):
+    for i in range(0 if args.no_e2e else args.warmup + args.steps):
         if i == args.warmup:
             barrier()
             torch.cuda.synchronize()
@@ -276,11 +283,12 @@ def run_rfq(args):
         x.copy_(x_host, non_blocking=True)
         step()
         y_host.copy_(y, non_blocking=True)
-    e1.record(stream)
-    torch.cuda.synchronize()
-    barrier()
-    e2e_ms = e0.elapsed_time(e1) / args.steps
-    if ws > 1:
+    if not args.no_e2e:
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        e2e_ms = e0.elapsed_time(e1) / args.steps
+    if ws > 1 and e2e_ms is not None:
         t = torch.tensor([e2e_ms], device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         e2e_ms = float(t.item())
@@ -318,8 +326,9 @@ def run_rfq(args):
                           "peak": pk["hbm"], "unit": "GB/s", "frac": aq_gbs / pk["hbm"],
                           "bytes_per_launch": aq_bytes, "ms_per_launch": q_ms,
                           "traffic": _kernel_traffic("act_quant_mxfp4_kernel", spec.name)},
-            "e2e": {"value": ws * flop / (e2e_ms * 1e-3) / 1e12, "unit": UNIT, "ms_per_step": e2e_ms,
-                    "h2d_bytes_per_step": M * K * 2, "d2h_bytes_per_step": M * N * 2},
+            "e2e": None if e2e_ms is None else {
+                "value": ws * flop / (e2e_ms * 1e-3) / 1e12, "unit": UNIT, "ms_per_step": e2e_ms,
+                "h2d_bytes_per_step": M * K * 2, "d2h_bytes_per_step": M * N * 2},
             "gpu_launches": 2 * args.steps,
             "clocks": clocks,
             "cpu_baseline": cpu,
@@ -336,6 +345,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="rfq", choices=["rfq", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffer) timing")
+    ap.add_argument("--rows", type=int, default=0, help="profile a smaller case: the first ROWS token rows")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
