@@ -168,6 +168,32 @@ RFQ_API rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, cons
  * earlier calls (RFQ_OK or RFQ_ERR_TIMEOUT); clears it when `clear` != 0. */
 RFQ_API rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *stream);
 
+/* Allocation-free variant of rfq_linear.  The paper has no counterpart: this
+ * entry point exists for callers that cannot allocate device memory, such as
+ * a serving loop that must not stall the device on cudaMalloc, a plug-in
+ * whose host program owns every device buffer, or a runtime with no device
+ * allocator of its own.  It takes the same arguments as rfq_linear except
+ * the workspace and allocates nothing: no cudaMalloc, no cudaFree, no
+ * allocating library routine.
+ *
+ * The GEMM's workspace (its status word) lives instead in a fixed 256-byte
+ * __device__ array inside the library; every GPU that loads the library
+ * holds it until the process exits.  If the GEMM ever needed more workspace
+ * than 256 bytes the call would return RFQ_ERR_SHAPE; every size rfq_linear
+ * accepts fits today.
+ *
+ * The first call on each device looks up the array's device address with
+ * that device current; make that first call before any stream capture.
+ * Every call clears the array on `stream` before the GEMM runs, because all
+ * calls share it and it keeps what the last call left.  Calls that overlap
+ * on the GPU (other streams, other host threads) race on the array.  A
+ * timeout of a bounded wait is not reported by this variant (use rfq_linear
+ * with a workspace to read it); Y is then left unwritten.
+ * Errors: those of rfq_linear, and RFQ_ERR_SHAPE as above. */
+RFQ_API rfq_status rfq_linear_noalloc(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_t *phi,
+                                      int32_t phi_r_s, const rfq_qtensor *wq, void *y, int32_t out_dtype,
+                                      void *stream);
+
 /* Dequantization x = code value * scale (Sec. 3.2 Eq. 4; Sec. 3.3 V_i) of a
  * quantized matrix into device fp32 out[rows][k].
  * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,

@@ -24,7 +24,8 @@ STATUS_NAMES = {0: "RFQ_OK", 1: "RFQ_ERR_INVALID_ARG", 2: "RFQ_ERR_SHAPE", 3: "R
                 4: "RFQ_ERR_UNSUPPORTED", 5: "RFQ_ERR_CUDA", 6: "RFQ_ERR_TIMEOUT", 7: "RFQ_ERR_DEVICE"}
 
 EXPORTED = ("rfq_status_string", "rfq_qtensor_bytes", "rfq_quantize_weight", "rfq_quantize_act",
-            "rfq_linear_workspace_bytes", "rfq_linear", "rfq_workspace_status", "rfq_dequant")
+            "rfq_linear_workspace_bytes", "rfq_linear", "rfq_workspace_status", "rfq_dequant",
+            "rfq_linear_noalloc")
 
 
 class RFQError(RuntimeError):
@@ -71,6 +72,8 @@ def load_library(path: str = LIB_PATH):
         lib.rfq_workspace_status.argtypes = [P, I32, P]
         lib.rfq_dequant.restype = I32
         lib.rfq_dequant.argtypes = [QTP, P, P]
+        lib.rfq_linear_noalloc.restype = I32
+        lib.rfq_linear_noalloc.argtypes = [QTP, QTP, P, I32, QTP, P, I32, P]
         _lib = lib
     return _lib
 
@@ -163,3 +166,14 @@ def rfq_workspace_status(workspace: torch.Tensor, clear: bool = False, stream=No
 def rfq_dequant(q: QTensor, out: torch.Tensor, stream=None):
     qt = q.c()
     _check(load_library().rfq_dequant(ctypes.byref(qt), _ptr(out), _stream(stream)), "rfq_dequant")
+
+
+def rfq_linear_noalloc(xq: QTensor, xr: QTensor | None, phi: torch.Tensor | None, phi_r_s: int, wq: QTensor,
+                       y: torch.Tensor, out_dtype: int, stream=None):
+    """rfq_linear for callers that cannot allocate device memory: the GEMM's
+    workspace is a fixed array inside the library (see include/rfq.h)."""
+    q, w = xq.c(), wq.c()
+    r = xr.c() if xr is not None else None
+    _check(load_library().rfq_linear_noalloc(ctypes.byref(q), ctypes.byref(r) if r is not None else None,
+                                             _ptr(phi), phi_r_s, ctypes.byref(w), _ptr(y), out_dtype,
+                                             _stream(stream)), "rfq_linear_noalloc")
