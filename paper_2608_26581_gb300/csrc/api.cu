@@ -82,8 +82,23 @@ rfq_status check_qtensor(const rfq_qtensor *q, int64_t rows, int64_t k)
 
 } // namespace
 
+int num_sms()
+{
+    static int cache[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64)
+        return 148;
+    if (cache[dev] == 0) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+            n = 148;
+        cache[dev] = n;
+    }
+    return cache[dev];
+}
+
 bool encode_tmap_2d_u8(CUtensorMap *map, const void *base, uint64_t inner_bytes, uint64_t rows,
-                       uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows, bool swizzle128)
+                       uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows, int swizzle)
 {
     PFN_encodeTiled enc = get_encode();
     if (!enc)
@@ -94,7 +109,9 @@ bool encode_tmap_2d_u8(CUtensorMap *map, const void *base, uint64_t inner_bytes,
     cuuint32_t estr[2] = {1, 1};
     CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box, estr,
                      CU_TENSOR_MAP_INTERLEAVE_NONE,
-                     swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                     swizzle == 128  ? CU_TENSOR_MAP_SWIZZLE_128B
+                     : swizzle == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                     : CU_TENSOR_MAP_SWIZZLE_NONE,
                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }

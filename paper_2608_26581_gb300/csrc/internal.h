@@ -47,7 +47,11 @@ struct GemmMxf4Args {
 cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st);
 
 // ---- tensor maps (api.cu)
+// swizzle: 0 none, 64 or 128 (bytes)
 bool encode_tmap_2d_u8(CUtensorMap *map, const void *base, uint64_t inner_bytes, uint64_t rows,
-                       uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows, bool swizzle128);
+                       uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows, int swizzle);
+
+// Number of SMs of the current device (cached).
+int num_sms();
 
 } // namespace rfq

@@ -214,6 +214,19 @@ __device__ __forceinline__ uint64_t sdesc_k_sw128(uint32_t saddr)
     return d;
 }
 
+// The same for the 64-byte swizzle (rows of 64 bytes, 8-row atoms of 512
+// bytes, tile base 512-byte aligned).
+__device__ __forceinline__ uint64_t sdesc_k_sw64(uint32_t saddr)
+{
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)1 << 16;
+    d |= (uint64_t)(512 >> 4) << 32;             // stride byte offset: 8 rows x 64 B
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)4 << 61;                      // 64-byte swizzle
+    return d;
+}
+
 // Descriptor of an unswizzled block of 16-byte rows (8-row core matrices,
 // 128 bytes apart), as read by tcgen05.cp 32x128b.
 __device__ __forceinline__ uint64_t sdesc_rows16(uint32_t saddr)

@@ -93,6 +93,49 @@ __device__ __forceinline__ int64_t scale_index(int64_t m, int64_t b, int64_t kbl
     return m * kblocks + b;
 }
 
+// Packed fp32 pairs (Blackwell f32x2 arithmetic): one instruction for two
+// multiplies or fused multiply-adds, both rounded to nearest even.
+__device__ __forceinline__ uint64_t f2pack(float a, float b)
+{
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+    return r;
+}
+
+__device__ __forceinline__ void f2unpack(uint64_t v, float &a, float &b)
+{
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
+}
+
+__device__ __forceinline__ uint64_t fmul2(uint64_t a, uint64_t b)
+{
+    uint64_t r;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c)
+{
+    uint64_t r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+
+__device__ __forceinline__ float fmax3(float a, float b, float c)
+{
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
+// max |v_i| over eight values
+__device__ __forceinline__ float absmax8(const float (&v)[8])
+{
+    const float m0 = fmax3(fabsf(v[0]), fabsf(v[1]), fabsf(v[2]));
+    const float m1 = fmax3(fabsf(v[3]), fabsf(v[4]), fabsf(v[5]));
+    return fmax3(m0, m1, fmaxf(fabsf(v[6]), fabsf(v[7])));
+}
+
 // Items are (row, 1024-element segment); a warp handles one item with four
 // 16-byte loads per lane in flight; four consecutive lanes form one
 // 32-element block.
@@ -109,9 +152,9 @@ __global__ void __launch_bounds__(256) act_quant_mxfp4_kernel(const uint4 *__res
                                                              int64_t pad_rows)
 {
     const int lane = threadIdx.x & 31;
-    const int64_t kchunks = K >> 3; // 8-element chunks per row
-    const int64_t kblocks = K >> 5;
-    const int64_t segs = (K + kSeg - 1) / kSeg;
+    const int kchunks = (int)(K >> 3); // 8-element chunks per row
+    const int kblocks = (int)(K >> 5);
+    const int segs = (kchunks + kSeg / 8 - 1) / (kSeg / 8);
     const int64_t items = M * segs;
     const int64_t gwarp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -129,63 +172,72 @@ __global__ void __launch_bounds__(256) act_quant_mxfp4_kernel(const uint4 *__res
 
     for (int64_t it = gwarp; it < items; it += nwarps) {
         const int64_t m = it / segs;
-        const int64_t c0 = (it - m * segs) * (kSeg / 8);
+        const int c0 = (int)(it - m * segs) * (kSeg / 8);
         const uint4 *xr = x + m * kchunks;
         uint4 v[kU];
 #pragma unroll
         for (int j = 0; j < kU; ++j) {
-            const int64_t c = c0 + j * 32 + lane;
+            const int c = c0 + j * 32 + lane;
             v[j] = c < kchunks ? __ldcs(xr + c) : make_uint4(0, 0, 0, 0);
         }
+        uint32_t *mrow = mcodes + m * kchunks;
+        uint32_t *rrow = RES ? rcodes + m * kchunks : nullptr;
+        // scale byte offset of (m, block 0) and the per-block step
+        int64_t srow;
+        if (LAYOUT == RFQ_SCALE_MMA)
+            srow = ((m >> 7) * (int64_t)(kblocks >> 2) << 9) + ((m & 31) << 4) + (((m >> 5) & 3) << 2);
+        else
+            srow = m * kblocks;
+        const uint8_t *prow = PHI ? phi + (m / p_s) * ((K + r_s - 1) / r_s) : nullptr;
 #pragma unroll
         for (int j = 0; j < kU; ++j) {
-            const int64_t c = c0 + j * 32 + lane;
+            const int c = c0 + j * 32 + lane;
             const bool ok = c < kchunks; // uniform over each group of 4 lanes
-            // amax of the 8 magnitudes as 15-bit integers (bf16 bits without sign)
-            uint32_t m2 = __vmaxu2(__vmaxu2(v[j].x & 0x7FFF7FFFu, v[j].y & 0x7FFF7FFFu),
-                                   __vmaxu2(v[j].z & 0x7FFF7FFFu, v[j].w & 0x7FFF7FFFu));
-            uint32_t am = max(m2 & 0xFFFFu, m2 >> 16);
-            am = max(am, __shfl_xor_sync(0xFFFFFFFFu, am, 1));
-            am = max(am, __shfl_xor_sync(0xFFFFFFFFu, am, 2));
-            const int sb = scale_byte_from_f32_bits(am << 16);
-            const float inv = pow2_neg_e(sb);
-            float xf[8], y[8];
+            const int b = c >> 2;
+            const int64_t soff = LAYOUT == RFQ_SCALE_MMA ? srow + ((b >> 2) << 9) + (b & 3) : srow + b;
+            float xf[8];
             bf16x8_to_f32(v[j], xf);
+            // block amax -> E8M0 byte from the exponent field (Sec. 3.2 Eq. 3, OCP rule)
+            float am = absmax8(xf);
+            am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 1));
+            am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 2));
+            const int sb = scale_byte_from_f32_bits(__float_as_uint(am));
+            const float inv = pow2_neg_e(sb);
+            const uint64_t inv2 = f2pack(inv, inv);
+            float y[8];
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
-                y[i] = xf[i] * inv;
+            for (int i = 0; i < 4; ++i)
+                f2unpack(fmul2(f2pack(xf[2 * i], xf[2 * i + 1]), inv2), y[2 * i], y[2 * i + 1]);
             const uint32_t qc = e2m1x8(y);
-            const int64_t b = c >> 2;
             if (ok) {
-                mcodes[m * kchunks + c] = qc;
+                mrow[c] = qc;
                 if ((lane & 3) == 0)
-                    mscales[scale_index<LAYOUT>(m, b, kblocks)] = (uint8_t)sb;
+                    mscales[soff] = (uint8_t)sb;
             }
             if (RES) {
-                bool on = true;
-                if (PHI)
-                    on = ok && phi[(m / p_s) * ((K + r_s - 1) / r_s) + (c * 8) / r_s] != 0;
+                const bool on = !PHI || (ok && prow[(c * 8) / r_s] != 0);
                 float q[8], r[8];
                 e2m1x8_decode(qc, q);
-                const float sc = pow2_e(sb);
-                float ra = 0.f;
+                const float nsc = -pow2_e(sb);
+                const uint64_t nsc2 = f2pack(nsc, nsc);
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    r[i] = fmaf(-q[i], sc, xf[i]); // x - x~, exact
-                    ra = fmaxf(ra, fabsf(r[i]));
-                }
+                for (int i = 0; i < 4; ++i) // x - x~ (exact)
+                    f2unpack(ffma2(f2pack(q[2 * i], q[2 * i + 1]), nsc2, f2pack(xf[2 * i], xf[2 * i + 1])),
+                             r[2 * i], r[2 * i + 1]);
+                float ra = absmax8(r);
                 ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, 1));
                 ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, 2));
                 const int rb = scale_byte_from_f32_bits(__float_as_uint(ra));
                 const float rinv = pow2_neg_e(rb);
+                const uint64_t rinv2 = f2pack(rinv, rinv);
 #pragma unroll
-                for (int i = 0; i < 8; ++i)
-                    r[i] *= rinv;
+                for (int i = 0; i < 4; ++i)
+                    f2unpack(fmul2(f2pack(r[2 * i], r[2 * i + 1]), rinv2), r[2 * i], r[2 * i + 1]);
                 const uint32_t rc = e2m1x8(r);
                 if (ok) {
-                    rcodes[m * kchunks + c] = on ? rc : 0u;
+                    rrow[c] = on ? rc : 0u;
                     if ((lane & 3) == 0)
-                        rscales[scale_index<LAYOUT>(m, b, kblocks)] = on ? (uint8_t)rb : 0;
+                        rscales[soff] = on ? (uint8_t)rb : 0;
                 }
             }
         }
