@@ -4,9 +4,11 @@
 // Persistent kernel: one CTA per SM walks output tiles of 128 x 256.  Per
 // 128-element k-stage the TMA producer stages the main A tile (X~ codes), the
 // residual A tile (X^ codes), the W~ tile and their E8M0 scale atoms in
-// shared memory (six stages in flight).  The MMA thread copies the scales into
-// TMEM (tcgen05.cp) and issues, per K=64 step, the main MMA and the residual
-// MMA against the SAME shared-memory W~ tile into the SAME TMEM accumulator:
+// shared memory (six stages in flight).  Four scale-writer warps (one per TMEM
+// lane quarter) move each stage's scale atoms from shared memory into TMEM
+// with tcgen05.st, which keeps the scale traffic off the MMA issue path; the
+// MMA thread then issues, per K=64 step, the main MMA and the residual MMA
+// against the SAME shared-memory W~ tile into the SAME TMEM accumulator:
 // W~ is read once for both products and the correction costs only MMA issue
 // (the on-the-fly residual accumulation of Sec. 4.3).  Residual MMAs of
 // k-tiles with phi = 0 are not issued and their A tiles are not loaded.
@@ -15,8 +17,12 @@
 // MMA thread starts it as soon as the accumulator has been read.
 //
 // Scale layout in TMEM (per 128-element k-chunk): 4 columns per 128 rows,
-// column j of lane i holding the four scales of row 32 j + i (written by
-// tcgen05.cp 32x128b.warpx4 from one 512-byte MMA-layout atom).
+// column j of lane i (of every lane quarter) holding the four scales of row
+// 32 j + i, i.e. lane i of a quarter takes bytes [16 i, 16 i + 16) of the
+// 512-byte MMA-layout atom.  Eight scale slots of 16 columns (A, R, B rows
+// 0-127, B rows 128-255) rotate per stage; with 8 slots >= 6 stages, a slot is
+// rewritten only after the stage that used it has had its MMAs complete (its
+// shared-memory slot was refilled, which waits for that).
 //
 // Every mbarrier wait is bounded (kWaitLimitNs) and also gives up as soon as
 // any CTA has recorded a timeout in the caller's status word; the CTA then
@@ -32,47 +38,70 @@ namespace {
 
 constexpr int BM = 128;
 constexpr int BN = 256;
-constexpr int BK = 128; // elements per k-stage: 64 bytes of codes per row
-constexpr int STAGES = 6;
-constexpr int A_BYTES = BM * BK / 2;
-constexpr int B_BYTES = BN * BK / 2;
 constexpr int ATOM = 512;              // scale bytes of 128 rows x one 128-element chunk
 constexpr int TMEM_COLS = 512;
-constexpr int SF_COL0 = 256;           // TMEM columns [256, 320): four scale slots of 16 columns
+constexpr int SF_COL0 = 256;           // TMEM columns [256, 384): scale slots
 constexpr int EPI_WARPS = 8;
-constexpr int THREADS = 64 + 32 * EPI_WARPS;
+constexpr int SF_WARPS = 4;
+constexpr int THREADS = 64 + 32 * EPI_WARPS + 32 * SF_WARPS;
 
-struct alignas(1024) Stage {
-    uint8_t a[A_BYTES];
-    uint8_t r[A_BYTES];
-    uint8_t b[B_BYTES];
-    uint8_t sfa[ATOM];
-    uint8_t sfr[ATOM];
-    uint8_t sfb[2 * ATOM];
+// Pipeline shape for a k-stage of KC 128-element chunks (BK = 128 KC
+// elements, 64 KC bytes of codes per row, swizzle = that row length).
+template <int KC>
+struct Cfg {
+    static constexpr int BK = 128 * KC;
+    static constexpr int ROW = BK / 2;                  // bytes per row per stage
+    static constexpr int A_BYTES = BM * ROW;
+    static constexpr int B_BYTES = BN * ROW;
+    static constexpr int STAGES = KC == 1 ? 6 : 3;
+    static constexpr int SF_STRIDE = 16 * KC;           // TMEM columns per scale slot
+    static constexpr int SF_SLOTS = KC == 1 ? 8 : 4;    // slots of SF_STRIDE columns
+    static_assert(SF_SLOTS >= STAGES, "a scale slot is rewritten only after its stage's MMAs completed");
+    static_assert(SF_SLOTS * SF_STRIDE <= 128, "scale slots fit in TMEM columns [256, 384)");
 };
 
+template <int KC>
+struct alignas(1024) Stage {
+    uint8_t a[Cfg<KC>::A_BYTES];
+    uint8_t r[Cfg<KC>::A_BYTES];
+    uint8_t b[Cfg<KC>::B_BYTES];
+    uint8_t sfa[KC * ATOM];            // chunk c at c * ATOM
+    uint8_t sfr[KC * ATOM];
+    uint8_t sfb[2 * KC * ATOM];        // W~ rows 128 h..128 h + 127: chunk c at (h * KC + c) * ATOM
+};
+
+template <int KC>
 struct Smem {
-    Stage st[STAGES];
-    uint64_t full[STAGES];
-    uint64_t empty[STAGES];
+    Stage<KC> st[Cfg<KC>::STAGES];
+    uint64_t full[Cfg<KC>::STAGES];
+    uint64_t empty[Cfg<KC>::STAGES];
     uint64_t acc_full;
     uint64_t acc_empty;
     uint64_t drain;
+    uint64_t sf_ready[Cfg<KC>::SF_SLOTS];
     uint32_t tmem_base;
     int32_t abort_flag;
     int32_t issued;
 };
 
-constexpr size_t kSmemBytes = sizeof(Smem) + 1024;
-static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+template <int KC>
+constexpr size_t smem_bytes() { return sizeof(Smem<KC>) + 1024; }
+static_assert(smem_bytes<1>() <= 227 * 1024 && smem_bytes<2>() <= 227 * 1024, "shared memory budget");
 
-__device__ __forceinline__ void flag_timeout(Smem &S, int32_t *status)
+template <int KC>
+__device__ __forceinline__ uint64_t sdesc_k(uint32_t saddr)
+{
+    return KC == 1 ? sdesc_k_sw64(saddr) : sdesc_k_sw128(saddr);
+}
+
+template <class SM>
+__device__ __forceinline__ void flag_timeout(SM &S, int32_t *status)
 {
     S.abort_flag = 1;
     atomicExch(status, kDevTimeout);
 }
 
-template <bool RES, bool PHI, bool OUT_BF16>
+template <int KC, bool RES, bool PHI, bool OUT_BF16>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_mxf4_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmR,
                      const __grid_constant__ CUtensorMap tmB, const uint8_t *__restrict__ sfa,
@@ -81,7 +110,9 @@ __global__ void __launch_bounds__(THREADS, 1)
                      int N, int K, int32_t *status)
 {
     extern __shared__ uint8_t smem_raw[];
-    Smem &S = *reinterpret_cast<Smem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    using C = Cfg<KC>;
+    constexpr int STAGES = C::STAGES, SF_SLOTS = C::SF_SLOTS, BK = C::BK;
+    Smem<KC> &S = *reinterpret_cast<Smem<KC> *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const volatile int32_t *gstat = status;
 
@@ -93,7 +124,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         return;
     __syncthreads();
 
-    const int kc = K >> 7;                 // k-stages (128-element chunks)
+    const int kc = K >> 7;                 // 128-element chunks
+    const int nks = (kc + KC - 1) / KC;    // k-stages (the last may hold fewer chunks)
     const int n_tiles = (N + BN - 1) / BN;
     const int m_tiles = (M + BM - 1) / BM;
     const int tiles = n_tiles * m_tiles;
@@ -107,6 +139,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         mbar_init(&S.acc_full, 1);
         mbar_init(&S.acc_empty, EPI_WARPS);
         mbar_init(&S.drain, 1);
+        for (int i = 0; i < SF_SLOTS; ++i)
+            mbar_init(&S.sf_ready[i], SF_WARPS);
         S.issued = 0;
         fence_mbar_init();
     }
@@ -132,33 +166,38 @@ __global__ void __launch_bounds__(THREADS, 1)
             bool stop = false;
             for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x) {
                 const int m_tile = tile / n_tiles, n_tile = tile - m_tile * n_tiles;
-                for (int ks = 0; ks < kc; ++ks, ++p) {
+                for (int ks = 0; ks < nks; ++ks, ++p) {
                     const int slot = p % STAGES;
                     if (!mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, kWaitLimitNs, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
                         break;
                     }
-                    const bool res_on =
-                        RES && (!PHI || phi[(int64_t)m_tile * phi_cols + ks / phi_chunks] != 0);
-                    uint32_t bytes = A_BYTES + B_BYTES + ATOM;
-                    if (res_on)
-                        bytes += A_BYTES + ATOM;
+                    const int c0 = ks * KC, nch = min(KC, kc - c0);
+                    bool res_on = RES;
+                    if (RES && PHI) {
+                        res_on = false;
+                        for (int c = 0; c < nch; ++c)
+                            res_on |= phi[(int64_t)m_tile * phi_cols + (c0 + c) / phi_chunks] != 0;
+                    }
                     const int atom0 = n_tile * 2;
-                    bytes += (atom0 + 1 < n_atoms ? 2 : 1) * ATOM;
-                    Stage &st = S.st[slot];
+                    const int nb = atom0 + 1 < n_atoms ? 2 : 1;
+                    uint32_t bytes = C::A_BYTES + C::B_BYTES + (1 + nb) * nch * ATOM;
+                    if (res_on)
+                        bytes += C::A_BYTES + nch * ATOM;
+                    Stage<KC> &st = S.st[slot];
                     uint64_t *bar = &S.full[slot];
                     mbar_arrive_expect_tx(bar, bytes);
-                    tma_load_2d(st.a, &tmA, bar, ks * (BK / 2), m_tile * BM);
+                    tma_load_2d(st.a, &tmA, bar, c0 * 64, m_tile * BM);
                     if (res_on)
-                        tma_load_2d(st.r, &tmR, bar, ks * (BK / 2), m_tile * BM);
-                    tma_load_2d(st.b, &tmB, bar, ks * (BK / 2), n_tile * BN);
-                    bulk_load(st.sfa, sfa + ((int64_t)m_tile * kc + ks) * ATOM, ATOM, bar);
+                        tma_load_2d(st.r, &tmR, bar, c0 * 64, m_tile * BM);
+                    tma_load_2d(st.b, &tmB, bar, c0 * 64, n_tile * BN);
+                    bulk_load(st.sfa, sfa + ((int64_t)m_tile * kc + c0) * ATOM, nch * ATOM, bar);
                     if (res_on)
-                        bulk_load(st.sfr, sfr + ((int64_t)m_tile * kc + ks) * ATOM, ATOM, bar);
-                    bulk_load(st.sfb, sfb + ((int64_t)atom0 * kc + ks) * ATOM, ATOM, bar);
-                    if (atom0 + 1 < n_atoms)
-                        bulk_load(st.sfb + ATOM, sfb + ((int64_t)(atom0 + 1) * kc + ks) * ATOM, ATOM, bar);
+                        bulk_load(st.sfr, sfr + ((int64_t)m_tile * kc + c0) * ATOM, nch * ATOM, bar);
+                    for (int h = 0; h < nb; ++h)
+                        bulk_load(st.sfb + h * KC * ATOM, sfb + ((int64_t)(atom0 + h) * kc + c0) * ATOM, nch * ATOM,
+                                  bar);
                 }
             }
             S.issued = p;
@@ -175,31 +214,31 @@ __global__ void __launch_bounds__(THREADS, 1)
                     break;
                 }
                 tc_fence_after();
-                for (int ks = 0; ks < kc; ++ks, ++p) {
+                for (int ks = 0; ks < nks; ++ks, ++p) {
                     const int slot = p % STAGES;
-                    if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat)) {
+                    if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat) ||
+                        !mbar_wait(&S.sf_ready[p % SF_SLOTS], (p / SF_SLOTS) & 1, kWaitLimitNs, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
                         break;
                     }
                     tc_fence_after();
-                    const bool res_on =
-                        RES && (!PHI || phi[(int64_t)m_tile * phi_cols + ks / phi_chunks] != 0);
-                    const Stage &st = S.st[slot];
-                    const uint32_t sf = tmem + SF_COL0 + 16 * (p & 3); // [0,4) A, [4,8) R, [8,16) B
-                    tc_cp_32x128b_warpx4(sf, sdesc_rows16(smem_u32(st.sfa)));
-                    if (res_on)
-                        tc_cp_32x128b_warpx4(sf + 4, sdesc_rows16(smem_u32(st.sfr)));
-                    tc_cp_32x128b_warpx4(sf + 8, sdesc_rows16(smem_u32(st.sfb)));
-                    tc_cp_32x128b_warpx4(sf + 12, sdesc_rows16(smem_u32(st.sfb + ATOM)));
+                    const int c0 = ks * KC, nch = min(KC, kc - c0);
+                    // scale slot columns: A chunk c at 4c, R at 4 KC + 4c, W~ at 8 KC + 8c (+4: rows 128-255)
+                    const uint32_t sf = tmem + SF_COL0 + C::SF_STRIDE * (p % SF_SLOTS);
+                    const Stage<KC> &st = S.st[slot];
                     const uint32_t a0 = smem_u32(st.a), r0 = smem_u32(st.r), b0 = smem_u32(st.b);
 #pragma unroll
-                    for (int j = 0; j < 2; ++j) {
-                        const uint32_t id = idesc_mxf4(BM, BN, 2 * j, 2 * j);
-                        const uint64_t bd = sdesc_k_sw64(b0 + 32 * j);
-                        tc_mma_mxf4(tmem, sdesc_k_sw64(a0 + 32 * j), bd, id, sf, sf + 8, (ks | j) != 0);
-                        if (res_on)
-                            tc_mma_mxf4(tmem, sdesc_k_sw64(r0 + 32 * j), bd, id, sf + 4, sf + 8, 1);
+                    for (int j = 0; j < 2 * KC; ++j) {
+                        const int c = j >> 1;
+                        if (c >= nch)
+                            break;
+                        const uint32_t id = idesc_mxf4(BM, BN, 2 * (j & 1), 2 * (j & 1));
+                        const uint64_t bd = sdesc_k<KC>(b0 + 32 * j);
+                        const uint32_t sfb_t = sf + 8 * KC + 8 * c;
+                        tc_mma_mxf4(tmem, sdesc_k<KC>(a0 + 32 * j), bd, id, sf + 4 * c, sfb_t, (ks | j) != 0);
+                        if (RES && (!PHI || phi[(int64_t)m_tile * phi_cols + (c0 + c) / phi_chunks] != 0))
+                            tc_mma_mxf4(tmem, sdesc_k<KC>(r0 + 32 * j), bd, id, sf + 4 * KC + 4 * c, sfb_t, 1);
                     }
                     tc_commit(&S.empty[slot]);
                 }
@@ -212,7 +251,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 (void)mbar_wait(&S.drain, 0, kWaitLimitNs);
             }
         }
-    } else {
+    } else if (warp < 2 + EPI_WARPS) {
         // ------------------------------------------------ epilogue (warps 2..9)
         const int q = warp & 3;          // TMEM lane quarter this warp may access
         const int h = (warp - 2) >> 2;   // column half of the tile
@@ -227,47 +266,97 @@ __global__ void __launch_bounds__(THREADS, 1)
             tc_fence_after();
             const int row = m_tile * BM + q * 32 + lane;
             const bool store = row < M;
-#pragma unroll 1
-            for (int c = 0; c < BN / 64; ++c) {
-                const int col0 = h * (BN / 2) + c * 32;
-                uint32_t v[32];
-                tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + col0, v);
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                // two 32-column chunks in flight, then the stores; the
+                // accumulator goes back to the MMA thread after the last load
+                uint32_t v[2][32];
+#pragma unroll
+                for (int c = 0; c < 2; ++c)
+                    tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + h * (BN / 2) + (2 * half + c) * 32,
+                                       v[c]);
                 tmem_ld_wait();
-                if (c == BN / 64 - 1) {
-                    // the accumulator is in registers: hand it back to the MMA thread
+                if (half == 1) {
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0)
                         mbar_arrive(&S.acc_empty);
                 }
-                const int col = n_tile * BN + col0;
-                if (!store || col >= N)
-                    continue;
-                const int nvalid = min(32, N - col); // 16 or 32 (N % 16 == 0)
-                if (OUT_BF16) {
-                    uint4 *dst =
-                        reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(Y) + (int64_t)row * N + col);
-                    uint32_t pk[16];
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        __nv_bfloat162 b2 =
-                            __floats2bfloat162_rn(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
-                        pk[i] = *reinterpret_cast<uint32_t *>(&b2);
+                for (int c = 0; c < 2; ++c) {
+                    const int col = n_tile * BN + h * (BN / 2) + (2 * half + c) * 32;
+                    if (!store || col >= N)
+                        continue;
+                    const int nvalid = min(32, N - col); // 16 or 32 (N % 16 == 0)
+                    if (OUT_BF16) {
+                        uint4 *dst =
+                            reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(Y) + (int64_t)row * N + col);
+                        uint32_t pk[16];
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            __nv_bfloat162 b2 = __floats2bfloat162_rn(__uint_as_float(v[c][2 * i]),
+                                                                      __uint_as_float(v[c][2 * i + 1]));
+                            pk[i] = *reinterpret_cast<uint32_t *>(&b2);
+                        }
+#pragma unroll
+                        for (int i = 0; i < 4; ++i)
+                            if (i * 8 < nvalid)
+                                dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+                    } else {
+                        uint4 *dst = reinterpret_cast<uint4 *>(static_cast<float *>(Y) + (int64_t)row * N + col);
+#pragma unroll
+                        for (int i = 0; i < 8; ++i)
+                            if (i * 4 < nvalid)
+                                dst[i] = make_uint4(v[c][4 * i], v[c][4 * i + 1], v[c][4 * i + 2], v[c][4 * i + 3]);
                     }
-#pragma unroll
-                    for (int i = 0; i < 4; ++i)
-                        if (i * 8 < nvalid)
-                            dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-                } else {
-                    uint4 *dst = reinterpret_cast<uint4 *>(static_cast<float *>(Y) + (int64_t)row * N + col);
-#pragma unroll
-                    for (int i = 0; i < 8; ++i)
-                        if (i * 4 < nvalid)
-                            dst[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
                 }
             }
             if (S.abort_flag)
                 break;
+        }
+    } else {
+        // ------------------------------------------------ scale writers (warps 10..13)
+        // Warp quarter q writes TMEM lanes 32q..32q+31; every quarter holds
+        // the same scale words (the MMA reads row 32 j + i from column j of
+        // lane i of the quarter that computes it).
+        const int q = warp & 3;
+        int p = 0;
+        bool stop = false;
+        for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x) {
+            const int m_tile = tile / n_tiles;
+            for (int ks = 0; ks < nks; ++ks, ++p) {
+                const int slot = p % STAGES;
+                if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat)) {
+                    if (lane == 0)
+                        flag_timeout(S, status);
+                    stop = true;
+                    break;
+                }
+                tc_fence_after();
+                const int c0 = ks * KC, nch = min(KC, kc - c0);
+                const Stage<KC> &st = S.st[slot];
+                const uint32_t tb = tmem + ((uint32_t)(q * 32) << 16) + SF_COL0 + C::SF_STRIDE * (p % SF_SLOTS);
+#pragma unroll
+                for (int c = 0; c < KC; ++c) {
+                    if (c >= nch)
+                        break;
+                    const uint4 va = *reinterpret_cast<const uint4 *>(st.sfa + c * ATOM + lane * 16);
+                    const uint4 vb0 = *reinterpret_cast<const uint4 *>(st.sfb + c * ATOM + lane * 16);
+                    const uint4 vb1 = *reinterpret_cast<const uint4 *>(st.sfb + (KC + c) * ATOM + lane * 16);
+                    tmem_st_32x32b_x4(tb + 4 * c, va.x, va.y, va.z, va.w);
+                    if (RES && (!PHI || phi[(int64_t)m_tile * phi_cols + (c0 + c) / phi_chunks] != 0)) {
+                        const uint4 vr = *reinterpret_cast<const uint4 *>(st.sfr + c * ATOM + lane * 16);
+                        tmem_st_32x32b_x4(tb + 4 * KC + 4 * c, vr.x, vr.y, vr.z, vr.w);
+                    }
+                    tmem_st_32x32b_x4(tb + 8 * KC + 8 * c, vb0.x, vb0.y, vb0.z, vb0.w);
+                    tmem_st_32x32b_x4(tb + 8 * KC + 8 * c + 4, vb1.x, vb1.y, vb1.z, vb1.w);
+                }
+                tmem_st_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(&S.sf_ready[p % SF_SLOTS]);
+            }
         }
     }
 
@@ -287,42 +376,44 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
 }
 
-template <bool RES, bool PHI, bool OUT>
+template <int KC, bool RES, bool PHI, bool OUT>
 cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const CUtensorMap &tb,
                            const GemmMxf4Args &a, cudaStream_t st)
 {
-    auto kern = gemm_mxf4_kernel<RES, PHI, OUT>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+    auto kern = gemm_mxf4_kernel<KC, RES, PHI, OUT>;
+    constexpr size_t smem = smem_bytes<KC>();
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess)
         return e;
     const int64_t tiles = ((a.N + BN - 1) / BN) * ((a.M + BM - 1) / BM);
     const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
     const int phi_chunks = a.phi_r_s / 128;
     const int phi_cols = a.phi ? (int)((a.K + a.phi_r_s - 1) / a.phi_r_s) : 0;
-    kern<<<grid, THREADS, kSmemBytes, st>>>(ta, tr, tb, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf,
-                                            (const uint8_t *)a.b_sf, a.phi, phi_chunks, phi_cols, a.y, (int)a.M,
-                                            (int)a.N, (int)a.K, a.status);
+    kern<<<grid, THREADS, smem, st>>>(ta, tr, tb, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf,
+                                      (const uint8_t *)a.b_sf, a.phi, phi_chunks, phi_cols, a.y, (int)a.M, (int)a.N,
+                                      (int)a.K, a.status);
     return cudaGetLastError();
 }
 
-} // namespace
-
-cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st)
+template <int KC>
+cudaError_t launch_kc(const GemmMxf4Args &a, cudaStream_t st)
 {
     CUtensorMap ta, tr, tb;
     const uint64_t kb = (uint64_t)a.K / 2;
-    if (!encode_tmap_2d_u8(&ta, a.a_codes, kb, (uint64_t)a.M, kb, BK / 2, BM, 64))
+    constexpr uint32_t row = Cfg<KC>::ROW;
+    constexpr int swz = KC == 1 ? 64 : 128;
+    if (!encode_tmap_2d_u8(&ta, a.a_codes, kb, (uint64_t)a.M, kb, row, BM, swz))
         return cudaErrorInvalidValue;
-    if (!encode_tmap_2d_u8(&tb, a.b_codes, kb, (uint64_t)a.N, kb, BK / 2, BN, 64))
+    if (!encode_tmap_2d_u8(&tb, a.b_codes, kb, (uint64_t)a.N, kb, row, BN, swz))
         return cudaErrorInvalidValue;
     if (a.r_codes) {
-        if (!encode_tmap_2d_u8(&tr, a.r_codes, kb, (uint64_t)a.M, kb, BK / 2, BM, 64))
+        if (!encode_tmap_2d_u8(&tr, a.r_codes, kb, (uint64_t)a.M, kb, row, BM, swz))
             return cudaErrorInvalidValue;
     } else {
         tr = ta;
     }
     const bool res = a.r_codes != nullptr, phi = res && a.phi != nullptr;
-#define RFQ_GV(R, P, O) return launch_variant<R, P, O>(ta, tr, tb, a, st)
+#define RFQ_GV(R, P, O) return launch_variant<KC, R, P, O>(ta, tr, tb, a, st)
     if (!res) {
         if (a.out_bf16) RFQ_GV(false, false, true);
         RFQ_GV(false, false, false);
@@ -334,6 +425,17 @@ cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st)
     if (a.out_bf16) RFQ_GV(true, false, true);
     RFQ_GV(true, false, false);
 #undef RFQ_GV
+}
+
+} // namespace
+
+cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st)
+{
+#ifdef RFQ_GEMM_KC
+    return launch_kc<RFQ_GEMM_KC>(a, st);
+#else
+    return launch_kc<2>(a, st);
+#endif
 }
 
 } // namespace rfq
