@@ -43,7 +43,13 @@
  *           bits [7:0] UE6M2 macro scale (E in [7:2], bias 48; M in [1:0]),
  *           bits [15:8] E1_8 (bit g: group of 8 elements g),
  *           bits [31:16] E1_16 (bit j: sub-group of 4 elements j).
- *           Scale array: [rows][k/64] uint32 (k % 64 == 0).
+ *           Metadata layouts (k % 64 == 0):
+ *             RFQ_SCALE_ROWMAJOR  [rows][k/64] uint32
+ *             RFQ_SCALE_MMA       block-major [k/64][rows rounded up to 128]
+ *                                 uint32, the layout rfq_linear consumes
+ *   BF16    an exact bf16 expansion of a quantized matrix, [rows][k]
+ *           (codes = the bf16 data, scales unused): rfq_dequant writes it,
+ *           and rfq_linear takes the HiF4 weight in this form.
  */
 #ifndef RFQ_H
 #define RFQ_H
@@ -72,7 +78,7 @@ typedef enum {
     RFQ_ERR_DEVICE = 7       /* the current device is not an sm_103 GPU */
 } rfq_status;
 
-typedef enum { RFQ_FMT_MXFP4 = 0, RFQ_FMT_HIF4 = 1 } rfq_format;
+typedef enum { RFQ_FMT_MXFP4 = 0, RFQ_FMT_HIF4 = 1, RFQ_FMT_BF16 = 2 } rfq_format;
 
 typedef enum { RFQ_SCALE_ROWMAJOR = 0, RFQ_SCALE_MMA = 1 } rfq_scale_layout;
 
@@ -92,7 +98,7 @@ typedef enum { RFQ_OUT_F32 = 0, RFQ_OUT_BF16 = 1 } rfq_out_dtype;
 
 typedef struct {
     int32_t fmt;          /* rfq_format */
-    int32_t scale_layout; /* rfq_scale_layout; HiF4 uses RFQ_SCALE_ROWMAJOR */
+    int32_t scale_layout; /* rfq_scale_layout (ignored for RFQ_FMT_BF16) */
     int64_t rows;         /* M for an activation, N for a weight */
     int64_t k;            /* length of the quantized (reduction) axis */
     void *codes;          /* device, see "Storage" above */
@@ -150,9 +156,12 @@ RFQ_API size_t rfq_linear_workspace_bytes(void);
  * (plain W4A4); phi: device bytes [ceil(M/128)][K/r_s] selecting the
  * residual k-tiles per 128-row tile, or NULL (= all ones); phi_r_s: the
  * column tile r_s of phi (a multiple of 128; ignored when phi is NULL).
- * wq: [N x K] weight codes.  MXFP4 operands must use RFQ_SCALE_MMA;
- * requirements: K % 128 == 0 (MXFP4) or K % 64 == 0 (HiF4), N % 16 == 0,
- * M >= 0.  y: device [M][N] row-major fp32 or bf16 (round-to-nearest-even
+ * wq: [N x K] weight.  MXFP4: every operand MXFP4 with RFQ_SCALE_MMA,
+ * K % 128 == 0.  HiF4 (Sec. 3.3): xq/xr HiF4 with RFQ_SCALE_MMA metadata and
+ * wq the exact bf16 expansion of the HiF4 weight (RFQ_FMT_BF16, from
+ * rfq_dequant), K % 64 == 0, phi_r_s a multiple of 64; the HiF4 tiles are
+ * expanded exactly to bf16 in shared memory and multiplied on the bf16 tensor
+ * path.  N % 16 == 0, M >= 0.  y: device [M][N] row-major fp32 or bf16 (round-to-nearest-even
  * of the fp32 accumulator).  workspace: device, rfq_linear_workspace_bytes()
  * bytes, zeroed by the caller once; a kernel that gives up a bounded wait
  * records a timeout there (read it with rfq_workspace_status).  The record
@@ -195,10 +204,12 @@ RFQ_API rfq_status rfq_linear_noalloc(const rfq_qtensor *xq, const rfq_qtensor *
                                       void *stream);
 
 /* Dequantization x = code value * scale (Sec. 3.2 Eq. 4; Sec. 3.3 V_i) of a
- * quantized matrix into device fp32 out[rows][k].
+ * quantized matrix (MXFP4 or HiF4) into device out[rows][k], fp32
+ * (RFQ_OUT_F32) or bf16 (RFQ_OUT_BF16).  Every HiF4 value is exact in bf16;
+ * MXFP4 values are exact in bf16 except below bf16's normal range.
  * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
  * RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */
-RFQ_API rfq_status rfq_dequant(const rfq_qtensor *q, float *out, void *stream);
+RFQ_API rfq_status rfq_dequant(const rfq_qtensor *q, void *out, int32_t out_dtype, void *stream);
 
 #ifdef __cplusplus
 }

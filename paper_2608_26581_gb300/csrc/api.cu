@@ -54,7 +54,7 @@ rfq_status check_device()
 
 rfq_status from_cuda(cudaError_t e) { return e == cudaSuccess ? RFQ_OK : RFQ_ERR_CUDA; }
 
-bool fmt_ok(int32_t f) { return f == RFQ_FMT_MXFP4 || f == RFQ_FMT_HIF4; }
+bool fmt_ok(int32_t f) { return f == RFQ_FMT_MXFP4 || f == RFQ_FMT_HIF4 || f == RFQ_FMT_BF16; }
 bool layout_ok(int32_t l) { return l == RFQ_SCALE_ROWMAJOR || l == RFQ_SCALE_MMA; }
 
 // Granule of the k axis for a format / scale layout.
@@ -62,6 +62,8 @@ int64_t k_granule(int32_t fmt, int32_t layout)
 {
     if (fmt == RFQ_FMT_HIF4)
         return 64;
+    if (fmt == RFQ_FMT_BF16)
+        return 8;
     return layout == RFQ_SCALE_MMA ? 128 : 32;
 }
 
@@ -69,13 +71,12 @@ rfq_status check_qtensor(const rfq_qtensor *q, int64_t rows, int64_t k)
 {
     if (!q || !fmt_ok(q->fmt) || !layout_ok(q->scale_layout))
         return RFQ_ERR_INVALID_ARG;
-    if (q->fmt == RFQ_FMT_HIF4 && q->scale_layout != RFQ_SCALE_ROWMAJOR)
-        return RFQ_ERR_INVALID_ARG;
     if (q->rows != rows || q->k != k || rows < 0 || k <= 0 || k % k_granule(q->fmt, q->scale_layout) != 0)
         return RFQ_ERR_SHAPE;
-    if (rows > 0 && (!q->codes || !q->scales))
+    const bool need_scales = q->fmt != RFQ_FMT_BF16;
+    if (rows > 0 && (!q->codes || (need_scales && !q->scales)))
         return RFQ_ERR_INVALID_ARG;
-    if (!aligned16(q->codes) || !aligned16(q->scales))
+    if (!aligned16(q->codes) || (need_scales && !aligned16(q->scales)))
         return RFQ_ERR_ALIGNMENT;
     return RFQ_OK;
 }
@@ -142,12 +143,15 @@ rfq_status rfq_qtensor_bytes(int32_t fmt, int32_t scale_layout, int64_t rows, in
 {
     if (!codes_bytes || !scale_bytes || !fmt_ok(fmt) || !layout_ok(scale_layout))
         return RFQ_ERR_INVALID_ARG;
-    if (fmt == RFQ_FMT_HIF4 && scale_layout != RFQ_SCALE_ROWMAJOR)
-        return RFQ_ERR_INVALID_ARG;
     if (rows < 0 || k <= 0 || k % k_granule(fmt, scale_layout) != 0)
         return RFQ_ERR_SHAPE;
     *codes_bytes = (size_t)rows * (size_t)(k / 2);
-    if (fmt == RFQ_FMT_HIF4)
+    if (fmt == RFQ_FMT_BF16) {
+        *codes_bytes = (size_t)rows * (size_t)k * 2;
+        *scale_bytes = 0;
+    } else if (fmt == RFQ_FMT_HIF4 && scale_layout == RFQ_SCALE_MMA)
+        *scale_bytes = (size_t)((rows + 127) / 128) * 128 * (size_t)(k / 64) * 4;
+    else if (fmt == RFQ_FMT_HIF4)
         *scale_bytes = (size_t)rows * (size_t)(k / 64) * 4;
     else if (scale_layout == RFQ_SCALE_MMA)
         *scale_bytes = (size_t)((rows + 127) / 128) * 128 * (size_t)(k / 32);
@@ -174,7 +178,9 @@ rfq_status rfq_quantize_weight(const void *w_bf16, int64_t K, int64_t N, rfq_qte
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (out->fmt == RFQ_FMT_MXFP4)
         return from_cuda(launch_weight_quant_mxfp4(w_bf16, K, N, out->codes, out->scales, out->scale_layout, st));
-    return RFQ_ERR_UNSUPPORTED;
+    if (out->fmt == RFQ_FMT_HIF4)
+        return from_cuda(launch_weight_quant_hif4(w_bf16, K, N, out->codes, out->scales, out->scale_layout, st));
+    return RFQ_ERR_INVALID_ARG;
 }
 
 rfq_status rfq_quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_fallback *fb, rfq_qtensor *xq,
@@ -200,8 +206,10 @@ rfq_status rfq_quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_
         if (xr->fmt != xq->fmt || xr->scale_layout != xq->scale_layout)
             return RFQ_ERR_INVALID_ARG;
     }
-    if (f.p_s < 1 || f.r_s < 32 || f.r_s % 32 != 0)
+    if (f.p_s < 1 || f.r_s < 32 || f.r_s % 32 != 0 || (xq->fmt == RFQ_FMT_HIF4 && f.r_s % 64 != 0))
         return RFQ_ERR_SHAPE;
+    if (xq->fmt == RFQ_FMT_BF16)
+        return RFQ_ERR_INVALID_ARG;
     if (f.mode == RFQ_FALLBACK_AMAX && !phi)
         return RFQ_ERR_INVALID_ARG;
     if (!aligned16(x_bf16))
@@ -215,7 +223,23 @@ rfq_status rfq_quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_
         return from_cuda(launch_act_quant_mxfp4(x_bf16, M, K, f.mode, f.tau, f.p_s, f.r_s, xq->codes, xq->scales,
                                                 res ? xr->codes : nullptr, res ? xr->scales : nullptr, phi,
                                                 xq->scale_layout, st));
-    return RFQ_ERR_UNSUPPORTED;
+    if (xq->fmt == RFQ_FMT_HIF4) {
+        if (f.mode == RFQ_FALLBACK_AMAX) {
+            // the indicator tiles are computed by the MXFP4 path's phi kernel
+            cudaError_t e = launch_phi_amax(x_bf16, M, K, f.p_s, f.r_s, f.tau, phi, st);
+            if (e != cudaSuccess)
+                return RFQ_ERR_CUDA;
+        } else if (phi) {
+            cudaError_t e = launch_phi_fill(phi, (M + f.p_s - 1) / f.p_s * ((K + f.r_s - 1) / f.r_s),
+                                            f.mode == RFQ_FALLBACK_ALL ? 1 : 0, st);
+            if (e != cudaSuccess)
+                return RFQ_ERR_CUDA;
+        }
+        return from_cuda(launch_act_quant_hif4(x_bf16, M, K, f.mode, f.p_s, f.r_s, xq->codes, xq->scales,
+                                               res ? xr->codes : nullptr, res ? xr->scales : nullptr, phi,
+                                               xq->scale_layout, st));
+    }
+    return RFQ_ERR_INVALID_ARG;
 }
 
 size_t rfq_linear_workspace_bytes(void) { return 256; }
@@ -241,13 +265,14 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
         if (xr->fmt != xq->fmt || xr->scale_layout != xq->scale_layout)
             return RFQ_ERR_INVALID_ARG;
     }
-    if (wq->fmt != xq->fmt)
+    const bool hif4 = xq->fmt == RFQ_FMT_HIF4;
+    if (xq->fmt == RFQ_FMT_BF16 || (hif4 ? wq->fmt != RFQ_FMT_BF16 : wq->fmt != RFQ_FMT_MXFP4))
         return RFQ_ERR_INVALID_ARG;
     if (N % 16 != 0)
         return RFQ_ERR_SHAPE;
     if (M > (int64_t)INT32_MAX || N > (int64_t)INT32_MAX || K > (int64_t)INT32_MAX)
         return RFQ_ERR_SHAPE;
-    if (phi && xr && (phi_r_s < 128 || phi_r_s % 128 != 0))
+    if (phi && xr && (hif4 ? (phi_r_s < 64 || phi_r_s % 64 != 0) : (phi_r_s < 128 || phi_r_s % 128 != 0)))
         return RFQ_ERR_SHAPE;
     if (!aligned16(y) || !aligned16(workspace))
         return RFQ_ERR_ALIGNMENT;
@@ -255,17 +280,16 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
         return s;
     if (M == 0 || N == 0)
         return RFQ_OK;
+    if (xq->scale_layout != RFQ_SCALE_MMA)
+        return RFQ_ERR_UNSUPPORTED;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    if (xq->fmt == RFQ_FMT_MXFP4) {
-        if (xq->scale_layout != RFQ_SCALE_MMA || wq->scale_layout != RFQ_SCALE_MMA)
-            return RFQ_ERR_UNSUPPORTED;
-        GemmMxf4Args a;
+    if (hif4) {
+        GemmHif4Args a;
         a.a_codes = xq->codes;
-        a.a_sf = xq->scales;
+        a.a_meta = xq->scales;
         a.r_codes = xr ? xr->codes : nullptr;
-        a.r_sf = xr ? xr->scales : nullptr;
-        a.b_codes = wq->codes;
-        a.b_sf = wq->scales;
+        a.r_meta = xr ? xr->scales : nullptr;
+        a.b_bf16 = wq->codes;
         a.phi = xr ? phi : nullptr;
         a.phi_r_s = phi_r_s;
         a.y = y;
@@ -274,9 +298,26 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
         a.N = N;
         a.K = K;
         a.status = static_cast<int32_t *>(workspace);
-        return from_cuda(launch_gemm_mxf4(a, st));
+        return from_cuda(launch_gemm_hif4(a, st));
     }
-    return RFQ_ERR_UNSUPPORTED;
+    if (wq->scale_layout != RFQ_SCALE_MMA)
+        return RFQ_ERR_UNSUPPORTED;
+    GemmMxf4Args a;
+    a.a_codes = xq->codes;
+    a.a_sf = xq->scales;
+    a.r_codes = xr ? xr->codes : nullptr;
+    a.r_sf = xr ? xr->scales : nullptr;
+    a.b_codes = wq->codes;
+    a.b_sf = wq->scales;
+    a.phi = xr ? phi : nullptr;
+    a.phi_r_s = phi_r_s;
+    a.y = y;
+    a.out_bf16 = out_dtype == RFQ_OUT_BF16;
+    a.M = M;
+    a.N = N;
+    a.K = K;
+    a.status = static_cast<int32_t *>(workspace);
+    return from_cuda(launch_gemm_mxf4(a, st));
 }
 
 rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *stream)
@@ -296,13 +337,15 @@ rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *stream)
     return v == kDevOk ? RFQ_OK : RFQ_ERR_TIMEOUT;
 }
 
-rfq_status rfq_dequant(const rfq_qtensor *q, float *out, void *stream)
+rfq_status rfq_dequant(const rfq_qtensor *q, void *out, int32_t out_dtype, void *stream)
 {
-    if (!q || !out)
+    if (!q || !out || (out_dtype != RFQ_OUT_F32 && out_dtype != RFQ_OUT_BF16))
         return RFQ_ERR_INVALID_ARG;
     rfq_status s = check_qtensor(q, q->rows, q->k);
     if (s != RFQ_OK)
         return s;
+    if (q->fmt == RFQ_FMT_BF16)
+        return RFQ_ERR_INVALID_ARG;
     if (!aligned16(out))
         return RFQ_ERR_ALIGNMENT;
     if ((s = check_device()) != RFQ_OK)
@@ -310,9 +353,13 @@ rfq_status rfq_dequant(const rfq_qtensor *q, float *out, void *stream)
     if (q->rows == 0)
         return RFQ_OK;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    if (q->fmt == RFQ_FMT_MXFP4)
-        return from_cuda(launch_dequant_mxfp4(q->codes, q->scales, q->rows, q->k, q->scale_layout, out, st));
-    return RFQ_ERR_UNSUPPORTED;
+    const bool bf16 = out_dtype == RFQ_OUT_BF16;
+    if (q->fmt == RFQ_FMT_HIF4)
+        return from_cuda(launch_dequant_hif4(q->codes, q->scales, q->rows, q->k, q->scale_layout, out, bf16, st));
+    if (bf16)
+        return from_cuda(launch_dequant_mxfp4_bf16(q->codes, q->scales, q->rows, q->k, q->scale_layout, out, st));
+    return from_cuda(
+        launch_dequant_mxfp4(q->codes, q->scales, q->rows, q->k, q->scale_layout, static_cast<float *>(out), st));
 }
 
 } // extern "C"

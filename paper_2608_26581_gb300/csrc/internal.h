@@ -28,6 +28,10 @@ __host__ __device__ inline int64_t sf_mma_offset(int64_t m, int64_t b, int64_t k
 cudaError_t launch_act_quant_mxfp4(const void *x, int64_t M, int64_t K, int mode, float tau, int p_s, int r_s,
                                    void *mcodes, void *mscales, void *rcodes, void *rscales, uint8_t *phi,
                                    int layout, cudaStream_t st);
+// phi(p, r) tiles: amax > tau, or a constant (0 / 1)
+cudaError_t launch_phi_amax(const void *x, int64_t M, int64_t K, int p_s, int r_s, float tau, uint8_t *phi,
+                            cudaStream_t st);
+cudaError_t launch_phi_fill(uint8_t *phi, int64_t n, int value, cudaStream_t st);
 cudaError_t launch_weight_quant_mxfp4(const void *w, int64_t K, int64_t N, void *codes, void *scales, int layout,
                                       cudaStream_t st);
 cudaError_t launch_dequant_mxfp4(const void *codes, const void *scales, int64_t rows, int64_t k, int layout,
@@ -45,6 +49,32 @@ struct GemmMxf4Args {
     int32_t *status;
 };
 cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st);
+
+// ---- HiF4 quantization (quant_hif4.cu); metadata layout RFQ_SCALE_MMA is
+// block-major [K/64][rows rounded up to 128]
+cudaError_t launch_act_quant_hif4(const void *x, int64_t M, int64_t K, int mode, int p_s, int r_s, void *mcodes,
+                                  void *mmeta, void *rcodes, void *rmeta, const uint8_t *phi, int layout,
+                                  cudaStream_t st);
+cudaError_t launch_weight_quant_hif4(const void *w, int64_t K, int64_t N, void *codes, void *meta, int layout,
+                                     cudaStream_t st);
+cudaError_t launch_dequant_hif4(const void *codes, const void *meta, int64_t rows, int64_t k, int layout,
+                                void *out, bool bf16, cudaStream_t st);
+cudaError_t launch_dequant_mxfp4_bf16(const void *codes, const void *scales, int64_t rows, int64_t k, int layout,
+                                      void *out, cudaStream_t st);
+
+// ---- HiF4 RFQ GEMM (gemm_hif4.cu)
+struct GemmHif4Args {
+    const void *a_codes, *r_codes;   // [M][K/2] HiF4 codes; r_codes may be null
+    const void *a_meta, *r_meta;     // block-major [K/64][Mpad] metadata words
+    const void *b_bf16;              // exact bf16 expansion of W~, [N][K]
+    const uint8_t *phi;
+    int phi_r_s;
+    void *y;
+    int out_bf16;
+    int64_t M, N, K;
+    int32_t *status;
+};
+cudaError_t launch_gemm_hif4(const GemmHif4Args &a, cudaStream_t st);
 
 // ---- tensor maps (api.cu)
 // swizzle: 0 none, 64 or 128 (bytes)

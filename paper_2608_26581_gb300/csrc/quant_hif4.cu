@@ -1,0 +1,334 @@
+// quant_hif4.cu -- HiF4 quantization kernels for sm_103a (Sec. 3.3).
+//
+// A HiF4 block is 64 elements along K with one 32-bit metadata word:
+//   bits [7:0]   UE6M2 macro scale S = 2^(E-48) (1 + M/4)   (E in [7:2], M in [1:0])
+//   bits [15:8]  E1_8:  one exponent bit per group of 8 elements
+//   bits [31:16] E1_16: one exponent bit per sub-group of 4 elements
+// and 4-bit S1P2 codes (sign, magnitude k/4 with k = 0..7):
+//   V_i = S 2^(E1_8[i/8] + E1_16[i/4]) (k_i / 4).
+// The encoder is this library's reading of the paper, which gives only the
+// decoder: S is the smallest UE6M2 value with 7 S >= amax; a sub-group takes
+// the smallest exponent t in {0,1,2} with amax_sub <= 1.75 2^t S; E1_8 is set
+// when a sub-group of its group needs t = 2 and E1_16 = max(t - E1_8, 0);
+// elements round to the nearest k/4 step, ties to even k, saturating at 7.
+// Every comparison is exact in fp32 (all products carry a few significant
+// bits), so the kernels reproduce the fp64 definition bit for bit.
+//
+//   act_quant_hif4     main (+ residual, Sec. 4.3) codes and metadata of X
+//   weight_quant_hif4  W [K x N] -> K-major HiF4
+//   dequant_hif4       -> fp32 or bf16 values
+//
+// Metadata layouts: row-major [rows][K/64] words, or block-major
+// [K/64][rows] words (RFQ_SCALE_MMA: one k-block of every row contiguous, as
+// the HiF4 GEMM stages it).
+#include <cuda_bf16.h>
+#include <cstdint>
+
+#include "internal.h"
+
+namespace rfq {
+namespace {
+
+__device__ __forceinline__ float ue6m2_value(int E, int M) // 2^(E-48) (1 + M/4), E in [0, 63]
+{
+    return __uint_as_float(((uint32_t)(E - 48 + 127) << 23) | ((uint32_t)M << 21));
+}
+
+// Smallest UE6M2 byte with 7 * value >= amax (amax > 0), clamped to [0, 255].
+__device__ __forceinline__ int hif4_scale_byte(float amax)
+{
+    // floor(log2 amax) for a normal amax; a subnormal amax is below every
+    // 7 S, so byte 0 is the answer for it
+    if (__float_as_uint(amax) < 0x00800000u)
+        return 0;
+    const int ea = (int)((__float_as_uint(amax) >> 23) & 0xFF) - 127;
+    // 7 (1 + M/4) 2^(E-48) spans [7, 12.25] 2^(E-48), so the smallest valid
+    // (E, M) has E - 48 in {ea - 3, ea - 2}; scan those eight candidates in
+    // increasing order, skipping exponents below the format's range.
+    const int e_lo = ea - 3 + 48;
+    for (int d = 0; d < 2; ++d) {
+        const int E = e_lo + d;
+        if (E < 0)
+            continue;
+        if (E > 63)
+            return 255; // above the largest macro scale: saturate
+        for (int M = 0; M < 4; ++M)
+            if (7.0f * ue6m2_value(E, M) >= amax)
+                return (E << 2) | M;
+    }
+    return e_lo + 1 < 0 ? 0 : 255;
+}
+
+// Quantizes the eight elements x[0..7] of group g (sub-groups 2g, 2g+1) of a
+// 64-element block whose macro scale S is given.  Returns the codes (element
+// i in nibble i) and this group's E1_8 / E1_16 bits (placed at their final
+// metadata positions); `deq` receives the dequantized values.
+__device__ __forceinline__ uint32_t hif4_group(const float (&x)[8], float S, int g, uint32_t &meta_bits,
+                                               float (&deq)[8])
+{
+    int t[2];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        float a = 0.f;
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            a = fmaxf(a, fabsf(x[4 * h + i]));
+        t[h] = a <= 1.75f * S ? 0 : (a <= 3.5f * S ? 1 : 2);
+    }
+    const int e18 = (t[0] == 2 || t[1] == 2) ? 1 : 0;
+    const int e116_0 = max(t[0] - e18, 0), e116_1 = max(t[1] - e18, 0);
+    meta_bits = ((uint32_t)e18 << (8 + g)) | ((uint32_t)e116_0 << (16 + 2 * g)) | ((uint32_t)e116_1 << (17 + 2 * g));
+    uint32_t codes = 0;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int ex = e18 + (h ? e116_1 : e116_0);
+        const float step = 0.25f * S * (float)(1 << ex); // exact: S has 3 significant bits
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float v = x[4 * h + i];
+            const float a = fabsf(v);
+            // nearest k from the rounded quotient, then fixed up with exact
+            // comparisons against the midpoints (k +- 1/2) step
+            int k = (int)rintf(__fdiv_rn(a, step));
+            k = min(max(k, 0), 8);
+            const float hi = (float)(2 * k + 1) * 0.5f * step, lo = (float)(2 * k - 1) * 0.5f * step;
+            if (a > hi || (a == hi && (k & 1)))
+                ++k;
+            else if (k > 0 && (a < lo || (a == lo && (k & 1))))
+                --k;
+            k = min(k, 7);
+            const uint32_t s = __float_as_uint(v) >> 31;
+            codes |= (uint32_t)((s << 3) | k) << (4 * (4 * h + i));
+            const float q = (float)k * step;
+            deq[4 * h + i] = s ? -q : q;
+        }
+    }
+    return codes;
+}
+
+// rows: the matrix's row count; the block-major layout pads it to 128.
+template <int LAYOUT>
+__device__ __forceinline__ int64_t meta_index(int64_t m, int64_t blk, int64_t rows, int64_t kblocks)
+{
+    return LAYOUT == RFQ_SCALE_MMA ? blk * (((rows + 127) >> 7) << 7) + m : m * kblocks + blk;
+}
+
+// Eight consecutive lanes hold one 64-element block (lane l: group l % 8).
+// Quantizes x (main), and with RES its residual x - x~ (Sec. 4.3).
+template <bool RES, bool PHI, int LAYOUT>
+__global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__restrict__ x, int64_t M, int64_t K,
+                                                            uint32_t *__restrict__ mcodes,
+                                                            uint32_t *__restrict__ mmeta,
+                                                            uint32_t *__restrict__ rcodes,
+                                                            uint32_t *__restrict__ rmeta,
+                                                            const uint8_t *__restrict__ phi, int p_s, int r_s)
+{
+    const int lane = threadIdx.x & 31;
+    const int g = lane & 7;
+    const int64_t kchunks = K >> 3;
+    const int64_t kblocks = K >> 6;
+    const int64_t total = M * kchunks;
+    for (int64_t base = ((int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31)) * 1;; base += (int64_t)gridDim.x * blockDim.x) {
+        if (base >= total)
+            break;
+        const int64_t c = base + lane;            // chunk of 8 elements; a block never straddles rows
+        const bool ok = c < total;
+        const uint4 v = ok ? __ldcs(x + c) : make_uint4(0, 0, 0, 0);
+        float xf[8];
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            xf[2 * i] = __uint_as_float(w[i] << 16);
+            xf[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+        }
+        const int64_t m = c / kchunks, blk = (c % kchunks) >> 3;
+        float am = 0.f;
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            am = fmaxf(am, fabsf(xf[i]));
+#pragma unroll
+        for (int o = 1; o < 8; o <<= 1)
+            am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, o));
+        const int sb = am > 0.f ? hif4_scale_byte(am) : 0;
+        const float S = ue6m2_value(sb >> 2, sb & 3);
+        uint32_t bits;
+        float deq[8];
+        uint32_t code = hif4_group(xf, S, g, bits, deq);
+        if (am == 0.f) {
+            bits = 0;   // all-zero block: metadata 0, codes keep the sign of zero
+        }
+#pragma unroll
+        for (int o = 1; o < 8; o <<= 1)
+            bits |= __shfl_xor_sync(0xFFFFFFFFu, bits, o);
+        if (ok) {
+            mcodes[c] = code;
+            if (g == 0)
+                mmeta[meta_index<LAYOUT>(m, blk, M, kblocks)] = am == 0.f ? 0u : (bits | (uint32_t)sb);
+        }
+        if (RES) {
+            const bool on = !PHI || (ok && phi[(m / p_s) * ((K + r_s - 1) / r_s) + (blk * 64) / r_s] != 0);
+            float r[8];
+            float ra = 0.f;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                r[i] = xf[i] - deq[i]; // exact
+                ra = fmaxf(ra, fabsf(r[i]));
+            }
+#pragma unroll
+            for (int o = 1; o < 8; o <<= 1)
+                ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, o));
+            const int rsb = ra > 0.f ? hif4_scale_byte(ra) : 0;
+            const float RS = ue6m2_value(rsb >> 2, rsb & 3);
+            uint32_t rbits;
+            float rdeq[8];
+            const uint32_t rcode = hif4_group(r, RS, g, rbits, rdeq);
+#pragma unroll
+            for (int o = 1; o < 8; o <<= 1)
+                rbits |= __shfl_xor_sync(0xFFFFFFFFu, rbits, o);
+            if (ok) {
+                rcodes[c] = on ? rcode : 0u;
+                if (g == 0)
+                    rmeta[meta_index<LAYOUT>(m, blk, M, kblocks)] = (on && ra > 0.f) ? (rbits | (uint32_t)rsb) : 0u;
+            }
+        }
+    }
+}
+
+// One thread per (column n, 64-block) of W [K x N]: a warp reads 32
+// consecutive columns of one K row at a time.
+template <int LAYOUT>
+__global__ void __launch_bounds__(256) weight_quant_hif4_kernel(const __nv_bfloat16 *__restrict__ w, int64_t K,
+                                                               int64_t N, uint8_t *__restrict__ codes,
+                                                               uint32_t *__restrict__ meta)
+{
+    const int64_t kblocks = K >> 6;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t n = t % N, blk = t / N;
+    if (blk >= kblocks)
+        return;
+    float am = 0.f;
+    for (int i = 0; i < 64; ++i)
+        am = fmaxf(am, fabsf(__bfloat162float(w[(blk * 64 + i) * N + n])));
+    const int sb = am > 0.f ? hif4_scale_byte(am) : 0;
+    const float S = ue6m2_value(sb >> 2, sb & 3);
+    uint32_t bits = 0, out[8];
+    for (int g = 0; g < 8; ++g) {
+        float xf[8], deq[8];
+        for (int i = 0; i < 8; ++i)
+            xf[i] = __bfloat162float(w[(blk * 64 + 8 * g + i) * N + n]);
+        uint32_t gb;
+        out[g] = hif4_group(xf, S, g, gb, deq);
+        bits |= gb;
+    }
+    uint4 *dst = reinterpret_cast<uint4 *>(codes + n * (K >> 1) + blk * 32);
+    dst[0] = make_uint4(out[0], out[1], out[2], out[3]);
+    dst[1] = make_uint4(out[4], out[5], out[6], out[7]);
+    meta[meta_index<LAYOUT>(n, blk, N, kblocks)] = am == 0.f ? 0u : (bits | (uint32_t)sb);
+}
+
+// x = S 2^(E1_8 + E1_16) k / 4 with the code's sign; 8 elements per thread.
+template <int LAYOUT, bool BF16>
+__global__ void dequant_hif4_kernel(const uint32_t *__restrict__ codes, const uint32_t *__restrict__ meta,
+                                    int64_t rows, int64_t k, void *__restrict__ out)
+{
+    const int64_t kchunks = k >> 3;
+    for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < rows * kchunks;
+         c += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t m = c / kchunks, cc = c % kchunks;
+        const int64_t blk = cc >> 3;
+        const int g = (int)(cc & 7);
+        const uint32_t md = meta[meta_index<LAYOUT>(m, blk, rows, k >> 6)];
+        const float S = ue6m2_value((int)((md >> 2) & 63), (int)(md & 3));
+        const uint32_t cw = codes[c];
+        float v[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const int j = 2 * g + (i >> 2); // sub-group
+            const int ex = (int)((md >> (8 + g)) & 1) + (int)((md >> (16 + j)) & 1);
+            const uint32_t code = (cw >> (4 * i)) & 0xF;
+            const float q = (float)(code & 7) * 0.25f * S * (float)(1 << ex);
+            v[i] = (code & 8) ? -q : q;
+        }
+        if (BF16) {
+            uint32_t p[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                __nv_bfloat162 b = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]); // exact
+                p[i] = *reinterpret_cast<uint32_t *>(&b);
+            }
+            reinterpret_cast<uint4 *>(out)[c] = make_uint4(p[0], p[1], p[2], p[3]);
+        } else {
+            float4 *o = reinterpret_cast<float4 *>(static_cast<float *>(out) + c * 8);
+            o[0] = make_float4(v[0], v[1], v[2], v[3]);
+            o[1] = make_float4(v[4], v[5], v[6], v[7]);
+        }
+    }
+}
+
+int grid_for(int64_t work, int threads, int max_blocks)
+{
+    int64_t b = (work + threads - 1) / threads;
+    if (b > max_blocks)
+        b = max_blocks;
+    return (int)(b < 1 ? 1 : b);
+}
+
+} // namespace
+
+cudaError_t launch_act_quant_hif4(const void *x, int64_t M, int64_t K, int mode, int p_s, int r_s, void *mcodes,
+                                  void *mmeta, void *rcodes, void *rmeta, const uint8_t *phi, int layout,
+                                  cudaStream_t st)
+{
+    const int blocks = grid_for(M * (K / 8), 256, 152 * 8);
+    auto *xi = static_cast<const uint4 *>(x);
+    auto *mc = static_cast<uint32_t *>(mcodes);
+    auto *mm = static_cast<uint32_t *>(mmeta);
+    auto *rc = static_cast<uint32_t *>(rcodes);
+    auto *rm = static_cast<uint32_t *>(rmeta);
+#define RFQ_HQ(RES, PHI, LAY)                                                                                     \
+    act_quant_hif4_kernel<RES, PHI, LAY><<<blocks, 256, 0, st>>>(xi, M, K, mc, mm, rc, rm, phi, p_s, r_s)
+    if (mode == RFQ_FALLBACK_NONE) {
+        if (layout == RFQ_SCALE_MMA) RFQ_HQ(false, false, RFQ_SCALE_MMA);
+        else RFQ_HQ(false, false, RFQ_SCALE_ROWMAJOR);
+    } else if (mode == RFQ_FALLBACK_ALL) {
+        if (layout == RFQ_SCALE_MMA) RFQ_HQ(true, false, RFQ_SCALE_MMA);
+        else RFQ_HQ(true, false, RFQ_SCALE_ROWMAJOR);
+    } else {
+        if (layout == RFQ_SCALE_MMA) RFQ_HQ(true, true, RFQ_SCALE_MMA);
+        else RFQ_HQ(true, true, RFQ_SCALE_ROWMAJOR);
+    }
+#undef RFQ_HQ
+    return cudaGetLastError();
+}
+
+cudaError_t launch_weight_quant_hif4(const void *w, int64_t K, int64_t N, void *codes, void *meta, int layout,
+                                     cudaStream_t st)
+{
+    const int64_t work = N * (K / 64);
+    const unsigned blocks = (unsigned)((work + 255) / 256);
+    if (layout == RFQ_SCALE_MMA)
+        weight_quant_hif4_kernel<RFQ_SCALE_MMA><<<blocks, 256, 0, st>>>((const __nv_bfloat16 *)w, K, N,
+                                                                         (uint8_t *)codes, (uint32_t *)meta);
+    else
+        weight_quant_hif4_kernel<RFQ_SCALE_ROWMAJOR><<<blocks, 256, 0, st>>>((const __nv_bfloat16 *)w, K, N,
+                                                                              (uint8_t *)codes, (uint32_t *)meta);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_dequant_hif4(const void *codes, const void *meta, int64_t rows, int64_t k, int layout,
+                                void *out, bool bf16, cudaStream_t st)
+{
+    const int blocks = grid_for(rows * (k / 8), 256, 152 * 32);
+    auto *c = static_cast<const uint32_t *>(codes);
+    auto *m = static_cast<const uint32_t *>(meta);
+    if (layout == RFQ_SCALE_MMA) {
+        if (bf16) dequant_hif4_kernel<RFQ_SCALE_MMA, true><<<blocks, 256, 0, st>>>(c, m, rows, k, out);
+        else dequant_hif4_kernel<RFQ_SCALE_MMA, false><<<blocks, 256, 0, st>>>(c, m, rows, k, out);
+    } else {
+        if (bf16) dequant_hif4_kernel<RFQ_SCALE_ROWMAJOR, true><<<blocks, 256, 0, st>>>(c, m, rows, k, out);
+        else dequant_hif4_kernel<RFQ_SCALE_ROWMAJOR, false><<<blocks, 256, 0, st>>>(c, m, rows, k, out);
+    }
+    return cudaGetLastError();
+}
+
+} // namespace rfq

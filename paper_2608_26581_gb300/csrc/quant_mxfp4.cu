@@ -334,6 +334,30 @@ __global__ void dequant_mxfp4_kernel(const uint32_t *__restrict__ codes, const u
     }
 }
 
+template <int LAYOUT>
+__global__ void dequant_mxfp4_bf16_kernel(const uint32_t *__restrict__ codes, const uint8_t *__restrict__ scales,
+                                          int64_t rows, int64_t k, uint4 *__restrict__ out)
+{
+    const int64_t kchunks = k >> 3;
+    for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < rows * kchunks;
+         c += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t m = c / kchunks, cc = c % kchunks;
+        const int sb = scales[scale_index<LAYOUT>(m, cc >> 2, k >> 5)];
+        float q[8];
+        e2m1x8_decode(codes[c], q);
+        const float s = pow2_e(sb);
+        uint32_t p[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            // code value times a power of two: exact in bf16 except below its
+            // normal range, where round-to-nearest-even applies
+            __nv_bfloat162 b = __floats2bfloat162_rn(q[2 * i] * s, q[2 * i + 1] * s);
+            p[i] = *reinterpret_cast<uint32_t *>(&b);
+        }
+        out[c] = make_uint4(p[0], p[1], p[2], p[3]);
+    }
+}
+
 int grid_for(int64_t work, int threads, int max_blocks)
 {
     int64_t b = (work + threads - 1) / threads;
@@ -343,6 +367,20 @@ int grid_for(int64_t work, int threads, int max_blocks)
 }
 
 } // namespace
+
+cudaError_t launch_phi_amax(const void *x, int64_t M, int64_t K, int p_s, int r_s, float tau, uint8_t *phi,
+                            cudaStream_t st)
+{
+    const int64_t np = (M + p_s - 1) / p_s, nr = (K + r_s - 1) / r_s;
+    phi_amax_kernel<<<(unsigned)(np * nr), 256, 0, st>>>((const __nv_bfloat16 *)x, M, K, p_s, r_s, tau, phi);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_phi_fill(uint8_t *phi, int64_t n, int value, cudaStream_t st)
+{
+    fill_u8_kernel<<<grid_for(n, 256, 1024), 256, 0, st>>>(phi, n, (uint8_t)value);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_act_quant_mxfp4(const void *x, int64_t M, int64_t K, int mode, float tau, int p_s, int r_s,
                                    void *mcodes, void *mscales, void *rcodes, void *rscales, uint8_t *phi,
@@ -403,6 +441,19 @@ cudaError_t launch_dequant_mxfp4(const void *codes, const void *scales, int64_t 
     else
         dequant_mxfp4_kernel<RFQ_SCALE_ROWMAJOR><<<blocks, 256, 0, st>>>((const uint32_t *)codes,
                                                                           (const uint8_t *)scales, rows, k, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_dequant_mxfp4_bf16(const void *codes, const void *scales, int64_t rows, int64_t k, int layout,
+                                      void *out, cudaStream_t st)
+{
+    const int blocks = grid_for(rows * (k / 8), 256, 152 * 32);
+    if (layout == RFQ_SCALE_MMA)
+        dequant_mxfp4_bf16_kernel<RFQ_SCALE_MMA><<<blocks, 256, 0, st>>>(
+            (const uint32_t *)codes, (const uint8_t *)scales, rows, k, (uint4 *)out);
+    else
+        dequant_mxfp4_bf16_kernel<RFQ_SCALE_ROWMAJOR><<<blocks, 256, 0, st>>>(
+            (const uint32_t *)codes, (const uint8_t *)scales, rows, k, (uint4 *)out);
     return cudaGetLastError();
 }
 

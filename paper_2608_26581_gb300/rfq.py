@@ -16,7 +16,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "librfq.so")
 
 RFQ_OK = 0
-RFQ_FMT_MXFP4, RFQ_FMT_HIF4 = 0, 1
+RFQ_FMT_MXFP4, RFQ_FMT_HIF4, RFQ_FMT_BF16 = 0, 1, 2
 RFQ_SCALE_ROWMAJOR, RFQ_SCALE_MMA = 0, 1
 RFQ_FALLBACK_NONE, RFQ_FALLBACK_ALL, RFQ_FALLBACK_AMAX = 0, 1, 2
 RFQ_OUT_F32, RFQ_OUT_BF16 = 0, 1
@@ -71,7 +71,7 @@ def load_library(path: str = LIB_PATH):
         lib.rfq_workspace_status.restype = I32
         lib.rfq_workspace_status.argtypes = [P, I32, P]
         lib.rfq_dequant.restype = I32
-        lib.rfq_dequant.argtypes = [QTP, P, P]
+        lib.rfq_dequant.argtypes = [QTP, P, I32, P]
         lib.rfq_linear_noalloc.restype = I32
         lib.rfq_linear_noalloc.argtypes = [QTP, QTP, P, I32, QTP, P, I32, P]
         _lib = lib
@@ -105,7 +105,7 @@ class QTensor:
 
     def c(self) -> _QT:
         return _QT(self.fmt, self.scale_layout, self.rows, self.k,
-                   self.codes.data_ptr(), self.scales.data_ptr())
+                   self.codes.data_ptr(), None if self.scales is None else self.scales.data_ptr())
 
 
 def rfq_status_string(status: int) -> str:
@@ -125,6 +125,10 @@ def empty_qtensor(fmt: int, scale_layout: int, rows: int, k: int, device="cuda")
     return QTensor(fmt, scale_layout, rows, k,
                    torch.empty(max(cb, 16), dtype=torch.uint8, device=device),
                    torch.empty(max(sb, 16), dtype=torch.uint8, device=device))
+
+
+def empty_bf16_operand(rows: int, k: int, device="cuda") -> QTensor:
+    return bf16_operand(torch.empty(rows, k, dtype=torch.bfloat16, device=device))
 
 
 def rfq_quantize_weight(w: torch.Tensor, out: QTensor, stream=None):
@@ -163,9 +167,18 @@ def rfq_workspace_status(workspace: torch.Tensor, clear: bool = False, stream=No
     return load_library().rfq_workspace_status(_ptr(workspace), 1 if clear else 0, _stream(stream))
 
 
-def rfq_dequant(q: QTensor, out: torch.Tensor, stream=None):
+def rfq_dequant(q: QTensor, out: torch.Tensor, out_dtype: int | None = None, stream=None):
+    if out_dtype is None:
+        out_dtype = RFQ_OUT_BF16 if out.dtype == torch.bfloat16 else RFQ_OUT_F32
     qt = q.c()
-    _check(load_library().rfq_dequant(ctypes.byref(qt), _ptr(out), _stream(stream)), "rfq_dequant")
+    _check(load_library().rfq_dequant(ctypes.byref(qt), _ptr(out), out_dtype, _stream(stream)), "rfq_dequant")
+
+
+def bf16_operand(t: torch.Tensor) -> QTensor:
+    """A bf16 [rows, k] tensor as an RFQ_FMT_BF16 operand (e.g. the exact
+    expansion of a HiF4 weight written by rfq_dequant)."""
+    rows, k = t.shape
+    return QTensor(RFQ_FMT_BF16, RFQ_SCALE_ROWMAJOR, rows, k, t, t)
 
 
 def rfq_linear_noalloc(xq: QTensor, xr: QTensor | None, phi: torch.Tensor | None, phi_r_s: int, wq: QTensor,

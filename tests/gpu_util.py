@@ -27,7 +27,11 @@ def qtensor_host(q: rfq.QTensor):
     rows, k = q.rows, q.k
     codes = q.codes[: rows * k // 2].cpu().numpy().reshape(rows, k // 2)
     sf = q.scales.cpu().numpy()
-    if q.fmt == rfq.RFQ_FMT_HIF4:
+    if q.fmt == rfq.RFQ_FMT_HIF4 and q.scale_layout == rfq.RFQ_SCALE_MMA:
+        # block-major [k/64][rows rounded up to 128]
+        rp = -(-rows // 128) * 128
+        scales = sf[: rp * (k // 64) * 4].view(np.uint32).reshape(k // 64, rp)[:, :rows].T.copy()
+    elif q.fmt == rfq.RFQ_FMT_HIF4:
         scales = sf[: rows * (k // 64) * 4].view(np.uint32).reshape(rows, k // 64)
     elif q.scale_layout == rfq.RFQ_SCALE_MMA:
         scales = mma_scale_to_rowmajor(sf, rows, k)

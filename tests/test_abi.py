@@ -46,6 +46,8 @@ def test_qtensor_bytes(lib):
     assert rfq.rfq_qtensor_bytes(0, 0, 128, 512) == (128 * 256, 128 * 16)
     assert rfq.rfq_qtensor_bytes(0, 1, 130, 512) == (130 * 256, 256 * 16)
     assert rfq.rfq_qtensor_bytes(1, 0, 10, 640) == (10 * 320, 10 * 10 * 4)
+    assert rfq.rfq_qtensor_bytes(1, 1, 10, 640) == (10 * 320, 128 * 10 * 4)   # block-major, rows padded
+    assert rfq.rfq_qtensor_bytes(2, 0, 10, 640) == (10 * 640 * 2, 0)         # bf16 expansion
     # HiF4: 36 bytes per 64 elements (4.5 bits each)
     cb, sb = rfq.rfq_qtensor_bytes(1, 0, 1, 64)
     assert cb + sb == 36
@@ -53,8 +55,8 @@ def test_qtensor_bytes(lib):
         rfq.rfq_qtensor_bytes(0, 1, 128, 96)          # MMA layout needs k % 128
     assert e.value.status == 2
     with pytest.raises(rfq.RFQError) as e:
-        rfq.rfq_qtensor_bytes(1, 1, 128, 128)         # HiF4 has one layout
-    assert e.value.status == 1
+        rfq.rfq_qtensor_bytes(1, 1, 128, 96)          # HiF4 needs k % 64
+    assert e.value.status == 2
 
 
 def test_workspace_bytes(lib):
@@ -67,9 +69,9 @@ def test_null_arguments_rejected_before_any_device_work(lib):
     assert lib.rfq_quantize_act(None, 1, 32, None, None, None, None, None) == 1
     assert lib.rfq_quantize_weight(None, 32, 16, None, None) == 1
     assert lib.rfq_linear(None, None, None, 0, None, None, 0, None, None) == 1
-    assert lib.rfq_dequant(None, None, None) == 1
+    assert lib.rfq_dequant(None, None, 0, None) == 1
     qt = rfq._QT(0, 1, 128, 96, 16, 16)           # k not a multiple of 128 for the MMA layout
     assert lib.rfq_quantize_act(ctypes.c_void_p(16), 128, 96, None, ctypes.byref(qt), ctypes.byref(qt),
                                 None, None) == 2
     qt = rfq._QT(0, 0, 4, 64, 8, 16)              # misaligned codes pointer
-    assert lib.rfq_dequant(ctypes.byref(qt), ctypes.c_void_p(16), None) == 3
+    assert lib.rfq_dequant(ctypes.byref(qt), ctypes.c_void_p(16), 0, None) == 3

@@ -166,3 +166,7 @@ def test_dequant_matches_oracle(orc):
             c, s = qtensor_host(q)
             ref = orc.dequant(orc.FMT_MXFP4, c, s, 200, 512)
             assert np.array_equal(out.cpu().numpy().astype(np.float64), ref)
+            out16 = torch.empty(200, 512, dtype=torch.bfloat16, device=DEV)
+            rfq.rfq_dequant(q, out16)
+            torch.cuda.synchronize()
+            assert np.array_equal(out16.double().cpu().numpy(), ref)   # in bf16's normal range: exact
