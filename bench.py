@@ -33,7 +33,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 if HERE not in sys.path:
     sys.path.insert(0, HERE)
 
-WORKLOAD = "wan_ffn_up"
+WORKLOAD = "wan_ffn_up"   # default; --workload picks another of synth.WORKLOADS
 METRIC = "RFQ W4A4 linear TFLOP/s & % FP4 MMA peak; act-quant HBM GB/s (1xGB300)"
 UNIT = "TFLOP/s"
 FP4_OVER_BF16 = 13.5 / 2.25   # nominal dense FP4 : BF16 tensor rate of GB300
@@ -129,23 +129,36 @@ def _dist():
     return ws, rank, local
 
 
-def _workload(rows: int = 0):
+def _workload(rows: int = 0, name: str = WORKLOAD):
     """The benchmark workload; rows > 0 keeps only the first `rows` token
     rows (a smaller case of the same kernels, for profiler captures)."""
     import dataclasses
     from paper_2608_26581_gb300.synth import WORKLOADS
-    spec = WORKLOADS[WORKLOAD]
+    spec = WORKLOADS[name]
     if rows and rows < spec.act.M:
         spec = dataclasses.replace(spec, name=f"{spec.name}_first{rows}rows",
                                    act=dataclasses.replace(spec.act, M=rows))
     return spec
 
 
+def _inputs_desc(a):
+    body = {"normal": "N(0,1)", "student_t3": "Student-t(3)", "laplace": f"Laplace(0,{a.body_scale:g})"}[a.body]
+    d = f"synthetic: X {body}"
+    if a.chan_count or a.chan_frac:
+        d += f", {a.chan_count if a.chan_count is not None else f'{100 * a.chan_frac:g}%'} outlier channels x{a.chan_scale:g}"
+    if a.tok_count or a.tok_frac:
+        d += f", {a.tok_count if a.tok_count is not None else f'{100 * a.tok_frac:g}%'} tokens x{a.tok_scale:g}"
+    return d + "; W N(0,0.02)"
+
+
 def _config(spec, extra=None):
-    c = {"workload": spec.name, "M": spec.act.M, "K": spec.act.K, "N": spec.N, "main_format": "mxfp4",
-         "residual_format": "mxfp4", "phi": "all tiles (phi = 1)", "y_dtype": "bf16",
-         "inputs": "synthetic: X N(0,1), 1% outlier channels x64, 0.1% tokens x200; W N(0,0.02)",
-         "l2": "inputs larger than L2 (X 335 MB, Y 906 MB per step), no flush"}
+    M, K, N = spec.act.M, spec.act.K, spec.N
+    x_mb, y_mb = M * K * 2 / 1e6, M * N * 2 / 1e6
+    c = {"workload": spec.name, "M": M, "K": K, "N": N, "main_format": spec.fmt,
+         "residual_format": spec.fmt, "phi": "all tiles (phi = 1)", "y_dtype": "bf16",
+         "inputs": _inputs_desc(spec.act),
+         "l2": (f"inputs larger than L2 (X {x_mb:.0f} MB, Y {y_mb:.0f} MB per step), no flush"
+                if x_mb + y_mb > 129 else "working set below L2 size")}
     if extra:
         c.update(extra)
     return c
@@ -213,23 +226,38 @@ def run_rfq(args):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    spec = _workload(args.rows)
+    spec = _workload(args.rows, args.workload)
     M, K, N = spec.act.M, spec.act.K, spec.N
-    F, L = rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA
+    hif4 = spec.fmt == "hif4"
+    quant_only = N == 0
+    F = rfq.RFQ_FMT_HIF4 if hif4 else rfq.RFQ_FMT_MXFP4
+    L = rfq.RFQ_SCALE_MMA
 
     xb = make_activation(spec.act)
-    wb = make_weight(K, N, seed=spec.act.seed)
     x_host = torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16).pin_memory()
-    w = torch.from_numpy(wb.view(np.int16)).to(dev).view(torch.bfloat16)
     x = x_host.to(dev)
-    wq = rfq.empty_qtensor(F, L, N, K, device=dev)
-    rfq.rfq_quantize_weight(w, wq)                         # offline weight step, untimed
+    wop = None
+    if not quant_only:
+        wb = make_weight(K, N, seed=spec.act.seed)
+        w = torch.from_numpy(wb.view(np.int16)).to(dev).view(torch.bfloat16)
+        wq = rfq.empty_qtensor(F, L, N, K, device=dev)
+        rfq.rfq_quantize_weight(w, wq)                     # offline weight step, untimed
+        if hif4:
+            wop = rfq.empty_bf16_operand(N, K, device=dev)  # exact bf16 expansion of W~ (offline)
+            rfq.rfq_dequant(wq, wop.codes)
+        else:
+            wop = wq
+        del w
     xq = rfq.empty_qtensor(F, L, M, K, device=dev)
     xr = rfq.empty_qtensor(F, L, M, K, device=dev)
-    y = torch.empty(M, N, dtype=torch.bfloat16, device=dev)
-    y_host = torch.empty(M, N, dtype=torch.bfloat16).pin_memory()
+    y = torch.empty(M, max(N, 16), dtype=torch.bfloat16, device=dev)
+    y_host = torch.empty(M, max(N, 16), dtype=torch.bfloat16).pin_memory()
     wsp = torch.zeros(rfq.rfq_linear_workspace_bytes() // 4, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream(dev)
+    # quantizer-only workload: its result (both pathways' codes and scales) is read back
+    host_q = [(torch.empty_like(t, device="cpu").pin_memory(), t)
+              for t in (xq.codes, xq.scales, xr.codes, xr.scales)] if quant_only else []
+    q_bytes = sum(t.numel() for _, t in host_q)
 
     ev = lambda: torch.cuda.Event(enable_timing=True)
     per_step = [(ev(), ev(), ev()) for _ in range(args.steps)]
@@ -240,7 +268,8 @@ def run_rfq(args):
         rfq.rfq_quantize_act(x, xq, xr, None, stream=stream)
         if i is not None:
             per_step[i][1].record(stream)
-        rfq.rfq_linear(xq, xr, None, 256, wq, y, rfq.RFQ_OUT_BF16, wsp, stream=stream)
+        if not quant_only:
+            rfq.rfq_linear(xq, xr, None, 256, wop, y, rfq.RFQ_OUT_BF16, wsp, stream=stream)
         if i is not None:
             per_step[i][2].record(stream)
 
@@ -282,7 +311,11 @@ def run_rfq(args):
             e0.record(stream)
         x.copy_(x_host, non_blocking=True)
         step()
-        y_host.copy_(y, non_blocking=True)
+        if quant_only:
+            for dst, src in host_q:
+                dst.copy_(src, non_blocking=True)
+        else:
+            y_host.copy_(y, non_blocking=True)
     if not args.no_e2e:
         e1.record(stream)
         torch.cuda.synchronize()
@@ -296,43 +329,68 @@ def run_rfq(args):
         raise RuntimeError("rfq_linear reported a device timeout")
 
     flop = 2.0 * 2.0 * M * N * K                 # main + residual product, phi = 1 everywhere
-    value = ws * flop / (ms * 1e-3) / 1e12
     pk = _peaks()
-    fp4_peak = pk["bf16_sust"] * FP4_OVER_BF16
-    gemm_tflops = flop / (g_ms * 1e-3) / 1e12
-    aq_bytes = M * K * 2 + 2 * (M * K // 2) + 2 * (((M + 127) // 128) * 128 * K // 32)
+    if hif4:
+        # HiF4 runs on the bf16 tensor path (exact bf16 expansion)
+        t_peak, t_src = pk["bf16_sust"], f"{pk['src']} bf16 sustained {pk['bf16_sust']} TFLOP/s, of {pk['src']}"
+        t_kernel = "gemm_hif4_kernel"
+    else:
+        t_peak = pk["bf16_sust"] * FP4_OVER_BF16
+        t_src = (f"{pk['src']} bf16 sustained {pk['bf16_sust']} TFLOP/s x {FP4_OVER_BF16:g} "
+                 f"(nominal dense FP4/BF16 ratio), of {pk['src']}")
+        t_kernel = "gemm_mxf4_kernel"
+    if hif4:
+        aq_bytes = M * K * 2 + 2 * (M * K // 2) + 2 * (((M + 127) // 128) * 128 * (K // 64) * 4)
+        aq_kernel = "act_quant_hif4_kernel"
+    else:
+        aq_bytes = M * K * 2 + 2 * (M * K // 2) + 2 * (((M + 127) // 128) * 128 * K // 32)
+        aq_kernel = "act_quant_mxfp4_kernel"
     aq_gbs = aq_bytes / (q_ms * 1e-3) / 1e9
+    act_quant = {"bound": "hbm", "kernel": aq_kernel, "achieved": aq_gbs, "peak": pk["hbm"], "unit": "GB/s",
+                 "frac": aq_gbs / pk["hbm"], "bytes_per_launch": aq_bytes, "ms_per_launch": q_ms,
+                 "traffic": _kernel_traffic(aq_kernel, spec.name)}
+    if quant_only:
+        value = ws * aq_bytes / (ms * 1e-3) / 1e9
+        unit = "GB/s"
+        roofline = dict(act_quant)
+    else:
+        value = ws * flop / (ms * 1e-3) / 1e12
+        unit = UNIT
+        gemm_tflops = flop / (g_ms * 1e-3) / 1e12
+        roofline = {"bound": "tensor", "kernel": t_kernel, "achieved": gemm_tflops, "peak": t_peak,
+                    "unit": "TFLOP/s", "frac": gemm_tflops / t_peak,
+                    "traffic": _kernel_traffic(t_kernel, spec.name), "flop_per_launch": flop, "ms_per_launch": g_ms,
+                    "peak_source": t_src}
     clocks = clk.summary()
+    if e2e_ms is not None:
+        e2e = {"value": ws * (aq_bytes / 1e9 if quant_only else flop / 1e12) / (e2e_ms * 1e-3), "unit": unit,
+               "ms_per_step": e2e_ms, "h2d_bytes_per_step": M * K * 2,
+               "d2h_bytes_per_step": q_bytes if quant_only else M * N * 2}
+    else:
+        e2e = None
 
     if rank == 0:
         cpu = None
-        if ws == 1 and not args.no_cpu_baseline:
+        if ws == 1 and not args.no_cpu_baseline and args.workload == WORKLOAD:
             v, dt, sample = cpu_oracle_sample()
             cpu = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample,
                    "seconds": round(dt, 2)}
         line = {
-            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+            "metric": METRIC, "value": value, "unit": unit, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "mxfp4 (e2m1 x e2m1, fp32 accumulate)", "data": "synthetic",
+            "vs_baseline": None,
+            "dtype": "hif4 (exact bf16 x bf16, fp32 accumulate)" if hif4 else "mxfp4 (e2m1 x e2m1, fp32 accumulate)",
+            "data": "synthetic",
             "config": _config(spec, {"parallelism": f"dp{ws} over token rows" if ws > 1 else "single GPU"}),
-            "effective_tflops_2mnk": ws * flop / 2 / (ms * 1e-3) / 1e12,
-            "roofline": {"bound": "tensor", "kernel": "gemm_mxf4_kernel", "achieved": gemm_tflops,
-                         "peak": fp4_peak, "unit": "TFLOP/s", "frac": gemm_tflops / fp4_peak,
-                         "traffic": _kernel_traffic("gemm_mxf4_kernel", spec.name),
-                         "flop_per_launch": flop, "ms_per_launch": g_ms,
-                         "peak_source": f"{pk['src']} bf16 sustained {pk['bf16_sust']} TFLOP/s x "
-                                        f"{FP4_OVER_BF16:g} (nominal dense FP4/BF16 ratio), of {pk['src']}"},
-            "act_quant": {"bound": "hbm", "kernel": "act_quant_mxfp4_kernel", "achieved": aq_gbs,
-                          "peak": pk["hbm"], "unit": "GB/s", "frac": aq_gbs / pk["hbm"],
-                          "bytes_per_launch": aq_bytes, "ms_per_launch": q_ms,
-                          "traffic": _kernel_traffic("act_quant_mxfp4_kernel", spec.name)},
-            "e2e": None if e2e_ms is None else {
-                "value": ws * flop / (e2e_ms * 1e-3) / 1e12, "unit": UNIT, "ms_per_step": e2e_ms,
-                "h2d_bytes_per_step": M * K * 2, "d2h_bytes_per_step": M * N * 2},
-            "gpu_launches": 2 * args.steps,
+            "roofline": roofline,
+            "act_quant": act_quant,
+            "e2e": e2e,
+            "gpu_launches": (1 if quant_only else 2) * args.steps,
             "clocks": clocks,
             "cpu_baseline": cpu,
         }
+        if not quant_only:
+            line["effective_tflops_2mnk"] = ws * flop / 2 / (ms * 1e-3) / 1e12
         print(json.dumps(line), flush=True)
     if ws > 1:
         dist.destroy_process_group()
@@ -347,6 +405,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffer) timing")
     ap.add_argument("--rows", type=int, default=0, help="profile a smaller case: the first ROWS token rows")
+    ap.add_argument("--workload", default=WORKLOAD,
+                    choices=["wan_ffn_up", "qwen_gate_up", "qwen_down_hif4", "act_quant", "tiny"])
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
