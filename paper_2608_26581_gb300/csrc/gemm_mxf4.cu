@@ -70,9 +70,12 @@ struct alignas(1024) Stage {
     uint8_t sfb[2 * KC * ATOM];        // W~ rows 128 h..128 h + 127: chunk c at (h * KC + c) * ATOM
 };
 
+constexpr int YSTAGE = 2048;          // per epilogue warp: 32 rows x 64 bytes of Y
+
 template <int KC>
 struct Smem {
     Stage<KC> st[Cfg<KC>::STAGES];
+    alignas(1024) uint8_t ystage[EPI_WARPS * YSTAGE]; // 64B-swizzled staging for the TMA stores of Y
     uint64_t full[Cfg<KC>::STAGES];
     uint64_t empty[Cfg<KC>::STAGES];
     uint64_t acc_full;
@@ -104,7 +107,8 @@ __device__ __forceinline__ void flag_timeout(SM &S, int32_t *status)
 template <int KC, bool RES, bool PHI, bool OUT_BF16>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_mxf4_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmR,
-                     const __grid_constant__ CUtensorMap tmB, const uint8_t *__restrict__ sfa,
+                     const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmY,
+                     const uint8_t *__restrict__ sfa,
                      const uint8_t *__restrict__ sfr, const uint8_t *__restrict__ sfb,
                      const uint8_t *__restrict__ phi, int phi_chunks, int phi_cols, void *__restrict__ Y, int M,
                      int N, int K, int32_t *status)
@@ -149,6 +153,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (RES)
             prefetch_tmap(&tmR);
         prefetch_tmap(&tmB);
+        prefetch_tmap(&tmY);
     }
     if (warp == 1) {
         tmem_alloc(&S.tmem_base, TMEM_COLS);
@@ -264,12 +269,14 @@ __global__ void __launch_bounds__(THREADS, 1)
                 break;
             }
             tc_fence_after();
-            const int row = m_tile * BM + q * 32 + lane;
-            const bool store = row < M;
+            // Y goes out through a per-warp shared-memory stage and TMA
+            // stores: full-line writes, clipped by the hardware at M and N.
+            uint8_t *stg = S.ystage + (warp - 2) * YSTAGE;
+            const int row0 = m_tile * BM + q * 32;
 #pragma unroll
             for (int half = 0; half < 2; ++half) {
-                // two 32-column chunks in flight, then the stores; the
-                // accumulator goes back to the MMA thread after the last load
+                // two 32-column chunks in flight; the accumulator goes back to
+                // the MMA thread after the last load of the tile
                 uint32_t v[2][32];
 #pragma unroll
                 for (int c = 0; c < 2; ++c)
@@ -285,12 +292,14 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
                 for (int c = 0; c < 2; ++c) {
                     const int col = n_tile * BN + h * (BN / 2) + (2 * half + c) * 32;
-                    if (!store || col >= N)
+                    if (col >= N)
                         continue;
-                    const int nvalid = min(32, N - col); // 16 or 32 (N % 16 == 0)
+                    // 64-byte rows, 16-byte chunk j of row r at r*64 + ((j ^ ((r >> 1) & 3)) << 4)
+                    const uint32_t sw = (uint32_t)((lane >> 1) & 3);
                     if (OUT_BF16) {
-                        uint4 *dst =
-                            reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(Y) + (int64_t)row * N + col);
+                        if (lane == 0)
+                            bulk_wait_group_read<0>();
+                        __syncwarp();
                         uint32_t pk[16];
 #pragma unroll
                         for (int i = 0; i < 16; ++i) {
@@ -299,21 +308,43 @@ __global__ void __launch_bounds__(THREADS, 1)
                             pk[i] = *reinterpret_cast<uint32_t *>(&b2);
                         }
 #pragma unroll
-                        for (int i = 0; i < 4; ++i)
-                            if (i * 8 < nvalid)
-                                dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+                        for (int j = 0; j < 4; ++j)
+                            *reinterpret_cast<uint4 *>(stg + lane * 64 + ((j ^ sw) << 4)) =
+                                make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
+                        fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) {
+                            tma_store_2d(&tmY, stg, col * 2, row0);
+                            bulk_commit_group();
+                        }
                     } else {
-                        uint4 *dst = reinterpret_cast<uint4 *>(static_cast<float *>(Y) + (int64_t)row * N + col);
 #pragma unroll
-                        for (int i = 0; i < 8; ++i)
-                            if (i * 4 < nvalid)
-                                dst[i] = make_uint4(v[c][4 * i], v[c][4 * i + 1], v[c][4 * i + 2], v[c][4 * i + 3]);
+                        for (int hb = 0; hb < 2; ++hb) { // 16 fp32 columns (64 bytes) per store
+                            if (col + 16 * hb >= N)
+                                break;
+                            if (lane == 0)
+                                bulk_wait_group_read<0>();
+                            __syncwarp();
+#pragma unroll
+                            for (int j = 0; j < 4; ++j)
+                                *reinterpret_cast<uint4 *>(stg + lane * 64 + ((j ^ sw) << 4)) =
+                                    make_uint4(v[c][16 * hb + 4 * j], v[c][16 * hb + 4 * j + 1],
+                                               v[c][16 * hb + 4 * j + 2], v[c][16 * hb + 4 * j + 3]);
+                            fence_proxy_async_smem();
+                            __syncwarp();
+                            if (lane == 0) {
+                                tma_store_2d(&tmY, stg, (col + 16 * hb) * 4, row0);
+                                bulk_commit_group();
+                            }
+                        }
                     }
                 }
             }
             if (S.abort_flag)
                 break;
         }
+        if (lane == 0)
+            bulk_wait_group<0>(); // every TMA store of this warp has completed
     } else {
         // ------------------------------------------------ scale writers (warps 10..13)
         // Warp quarter q writes TMEM lanes 32q..32q+31; every quarter holds
@@ -378,7 +409,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 
 template <int KC, bool RES, bool PHI, bool OUT>
 cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const CUtensorMap &tb,
-                           const GemmMxf4Args &a, cudaStream_t st)
+                           const CUtensorMap &ty, const GemmMxf4Args &a, cudaStream_t st)
 {
     auto kern = gemm_mxf4_kernel<KC, RES, PHI, OUT>;
     constexpr size_t smem = smem_bytes<KC>();
@@ -389,7 +420,7 @@ cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const C
     const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
     const int phi_chunks = a.phi_r_s / 128;
     const int phi_cols = a.phi ? (int)((a.K + a.phi_r_s - 1) / a.phi_r_s) : 0;
-    kern<<<grid, THREADS, smem, st>>>(ta, tr, tb, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf,
+    kern<<<grid, THREADS, smem, st>>>(ta, tr, tb, ty, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf,
                                       (const uint8_t *)a.b_sf, a.phi, phi_chunks, phi_cols, a.y, (int)a.M, (int)a.N,
                                       (int)a.K, a.status);
     return cudaGetLastError();
@@ -412,8 +443,13 @@ cudaError_t launch_kc(const GemmMxf4Args &a, cudaStream_t st)
     } else {
         tr = ta;
     }
+    // Y [M][N] (bf16 or fp32) as bytes; boxes of 64 bytes x 32 rows, 64B swizzle
+    CUtensorMap ty;
+    const uint64_t yrow = (uint64_t)a.N * (a.out_bf16 ? 2 : 4);
+    if (!encode_tmap_2d_u8(&ty, a.y, yrow, (uint64_t)a.M, yrow, 64, 32, 64))
+        return cudaErrorInvalidValue;
     const bool res = a.r_codes != nullptr, phi = res && a.phi != nullptr;
-#define RFQ_GV(R, P, O) return launch_variant<KC, R, P, O>(ta, tr, tb, a, st)
+#define RFQ_GV(R, P, O) return launch_variant<KC, R, P, O>(ta, tr, tb, ty, a, st)
     if (!res) {
         if (a.out_bf16) RFQ_GV(false, false, true);
         RFQ_GV(false, false, false);

@@ -394,7 +394,7 @@ cudaError_t launch_act_quant_mxfp4(const void *x, int64_t M, int64_t K, int mode
     }
     const int64_t pad = layout == RFQ_SCALE_MMA ? ((M + 127) / 128) * 128 - M : 0;
     const int64_t warps = M * ((K + kSeg - 1) / kSeg);
-    const int blocks = grid_for(warps * 32 > pad * (K / 32) ? warps * 32 : pad * (K / 32), 256, 152 * 16);
+    const int blocks = grid_for(warps * 32 > pad * (K / 32) ? warps * 32 : pad * (K / 32), 256, 152 * 24);
     auto *xi = static_cast<const uint4 *>(x);
     auto *mc = static_cast<uint32_t *>(mcodes);
     auto *ms = static_cast<uint8_t *>(mscales);
