@@ -250,6 +250,10 @@ def run_rfq(args):
         del w
     xq = rfq.empty_qtensor(F, L, M, K, device=dev)
     xr = rfq.empty_qtensor(F, L, M, K, device=dev)
+    # HiF4: the GEMM takes the exact bf16 expansions of X~ and X^ (expanding
+    # once per activation, not once per output tile inside the GEMM)
+    xq16 = rfq.empty_bf16_operand(M, K, device=dev) if hif4 and not quant_only else None
+    xr16 = rfq.empty_bf16_operand(M, K, device=dev) if hif4 and not quant_only else None
     y = torch.empty(M, max(N, 16), dtype=torch.bfloat16, device=dev)
     y_host = torch.empty(M, max(N, 16), dtype=torch.bfloat16).pin_memory()
     wsp = torch.zeros(rfq.rfq_linear_workspace_bytes() // 4, dtype=torch.int32, device=dev)
@@ -260,7 +264,7 @@ def run_rfq(args):
     q_bytes = sum(t.numel() for _, t in host_q)
 
     ev = lambda: torch.cuda.Event(enable_timing=True)
-    per_step = [(ev(), ev(), ev()) for _ in range(args.steps)]
+    per_step = [(ev(), ev(), ev(), ev()) for _ in range(args.steps)]
 
     def step(i=None):
         if i is not None:
@@ -268,10 +272,17 @@ def run_rfq(args):
         rfq.rfq_quantize_act(x, xq, xr, None, stream=stream)
         if i is not None:
             per_step[i][1].record(stream)
-        if not quant_only:
-            rfq.rfq_linear(xq, xr, None, 256, wop, y, rfq.RFQ_OUT_BF16, wsp, stream=stream)
+        if hif4 and not quant_only:
+            rfq.rfq_dequant(xq, xq16.codes, stream=stream)
+            rfq.rfq_dequant(xr, xr16.codes, stream=stream)
         if i is not None:
             per_step[i][2].record(stream)
+        if hif4 and not quant_only:
+            rfq.rfq_linear(xq16, xr16, None, 256, wop, y, rfq.RFQ_OUT_BF16, wsp, stream=stream)
+        elif not quant_only:
+            rfq.rfq_linear(xq, xr, None, 256, wop, y, rfq.RFQ_OUT_BF16, wsp, stream=stream)
+        if i is not None:
+            per_step[i][3].record(stream)
 
     for _ in range(args.warmup):
         step()
@@ -294,8 +305,9 @@ def run_rfq(args):
         torch.cuda.synchronize()
         barrier()
     ms = t_start.elapsed_time(t_end) / args.steps
-    q_ms = statistics.mean(a.elapsed_time(b) for a, b, _ in per_step)
-    g_ms = statistics.mean(b.elapsed_time(c) for _, b, c in per_step)
+    q_ms = statistics.mean(a.elapsed_time(b) for a, b, _, _ in per_step)
+    x_ms = statistics.mean(b.elapsed_time(c) for _, b, c, _ in per_step)   # HiF4 expansions (0 otherwise)
+    g_ms = statistics.mean(c.elapsed_time(d) for _, _, c, d in per_step)
     if ws > 1:
         t = torch.tensor([ms], device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
@@ -384,8 +396,9 @@ def run_rfq(args):
             "config": _config(spec, {"parallelism": f"dp{ws} over token rows" if ws > 1 else "single GPU"}),
             "roofline": roofline,
             "act_quant": act_quant,
+            "expand_ms_per_step": x_ms if hif4 else None,
             "e2e": e2e,
-            "gpu_launches": (1 if quant_only else 2) * args.steps,
+            "gpu_launches": (1 if quant_only else (4 if hif4 else 2)) * args.steps,
             "clocks": clocks,
             "cpu_baseline": cpu,
         }

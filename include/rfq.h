@@ -157,11 +157,13 @@ RFQ_API size_t rfq_linear_workspace_bytes(void);
  * residual k-tiles per 128-row tile, or NULL (= all ones); phi_r_s: the
  * column tile r_s of phi (a multiple of 128; ignored when phi is NULL).
  * wq: [N x K] weight.  MXFP4: every operand MXFP4 with RFQ_SCALE_MMA,
- * K % 128 == 0.  HiF4 (Sec. 3.3): xq/xr HiF4 with RFQ_SCALE_MMA metadata and
- * wq the exact bf16 expansion of the HiF4 weight (RFQ_FMT_BF16, from
- * rfq_dequant), K % 64 == 0, phi_r_s a multiple of 64; the HiF4 tiles are
- * expanded exactly to bf16 in shared memory and multiplied on the bf16 tensor
- * path.  N % 16 == 0, M >= 0.  y: device [M][N] row-major fp32 or bf16 (round-to-nearest-even
+ * K % 128 == 0.  HiF4 (Sec. 3.3): wq is the exact bf16 expansion of the HiF4
+ * weight (RFQ_FMT_BF16, from rfq_dequant), K % 64 == 0, phi_r_s a multiple
+ * of 64, and xq/xr are either HiF4 with RFQ_SCALE_MMA metadata (expanded
+ * exactly to bf16 in shared memory inside the GEMM) or their exact bf16
+ * expansions (RFQ_FMT_BF16, from rfq_dequant; faster when N spans several
+ * tiles, since each activation tile is then expanded once instead of once
+ * per output tile).  Both run on the bf16 tensor path.  N % 16 == 0, M >= 0.  y: device [M][N] row-major fp32 or bf16 (round-to-nearest-even
  * of the fp32 accumulator).  workspace: device, rfq_linear_workspace_bytes()
  * bytes, zeroed by the caller once; a kernel that gives up a bounded wait
  * records a timeout there (read it with rfq_workspace_status).  The record

@@ -265,9 +265,14 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
         if (xr->fmt != xq->fmt || xr->scale_layout != xq->scale_layout)
             return RFQ_ERR_INVALID_ARG;
     }
-    const bool hif4 = xq->fmt == RFQ_FMT_HIF4;
-    if (xq->fmt == RFQ_FMT_BF16 || (hif4 ? wq->fmt != RFQ_FMT_BF16 : wq->fmt != RFQ_FMT_MXFP4))
+    // operand formats: MXFP4 x MXFP4, or HiF4 (codes, or their exact bf16
+    // expansion) x the bf16 expansion of W~
+    const bool bf16_act = xq->fmt == RFQ_FMT_BF16;
+    const bool hif4 = xq->fmt == RFQ_FMT_HIF4 || bf16_act;
+    if (hif4 ? wq->fmt != RFQ_FMT_BF16 : wq->fmt != RFQ_FMT_MXFP4)
         return RFQ_ERR_INVALID_ARG;
+    if (bf16_act && K % 64 != 0)
+        return RFQ_ERR_SHAPE;
     if (N % 16 != 0)
         return RFQ_ERR_SHAPE;
     if (M > (int64_t)INT32_MAX || N > (int64_t)INT32_MAX || K > (int64_t)INT32_MAX)
@@ -280,11 +285,12 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
         return s;
     if (M == 0 || N == 0)
         return RFQ_OK;
-    if (xq->scale_layout != RFQ_SCALE_MMA)
+    if (!bf16_act && xq->scale_layout != RFQ_SCALE_MMA)
         return RFQ_ERR_UNSUPPORTED;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (hif4) {
         GemmHif4Args a;
+        a.a_bf16 = bf16_act;
         a.a_codes = xq->codes;
         a.a_meta = xq->scales;
         a.r_codes = xr ? xr->codes : nullptr;

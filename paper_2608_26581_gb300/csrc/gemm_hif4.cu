@@ -18,6 +18,7 @@
 // MMAs of tile t+1 run.  Waits are bounded as in the MXFP4 GEMM.
 #include <cuda_bf16.h>
 #include <cstdint>
+#include <type_traits>
 
 #include "internal.h"
 #include "ptx.cuh"
@@ -48,8 +49,19 @@ struct alignas(1024) Stage {
     uint32_t rmeta[BM];
 };
 
+// Operands already expanded to bf16 (X~, X^ and W~ all loaded by TMA).
+struct alignas(1024) Stage16 {
+    uint8_t b[B16_BYTES];
+    uint8_t a16[A16_BYTES];
+    uint8_t r16[A16_BYTES];
+};
+
+constexpr int YSTAGE = 2048; // per epilogue warp: 32 rows x 64 bytes of Y
+
+template <bool CONV>
 struct Smem {
-    Stage st[STAGES];
+    typename std::conditional<CONV, Stage, Stage16>::type st[STAGES];
+    alignas(1024) uint8_t ystage[CONV ? 16 : EPI_WARPS * YSTAGE];
     uint64_t full[STAGES];
     uint64_t conv[STAGES];
     uint64_t empty[STAGES];
@@ -61,10 +73,12 @@ struct Smem {
     int32_t issued;
 };
 
-constexpr size_t kSmemBytes = sizeof(Smem) + 1024;
-static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+template <bool CONV>
+constexpr size_t smem_bytes() { return sizeof(Smem<CONV>) + 1024; }
+static_assert(smem_bytes<true>() <= 227 * 1024 && smem_bytes<false>() <= 227 * 1024, "shared memory budget");
 
-__device__ __forceinline__ void flag_timeout(Smem &S, int32_t *status)
+template <class SM>
+__device__ __forceinline__ void flag_timeout(SM &S, int32_t *status)
 {
     S.abort_flag = 1;
     atomicExch(status, kDevTimeout);
@@ -93,15 +107,19 @@ __device__ __forceinline__ uint4 hif4_group_to_bf16(uint32_t cw, uint32_t meta, 
     return make_uint4(out[0], out[1], out[2], out[3]);
 }
 
-template <bool RES, bool PHI, bool OUT_BF16>
+// CONV: the activation operands are HiF4 codes + metadata expanded in the
+// kernel; otherwise they are bf16 expansions loaded by TMA like W~.
+template <bool CONV, bool RES, bool PHI, bool OUT_BF16>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_hif4_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmR,
-                     const __grid_constant__ CUtensorMap tmB, const uint32_t *__restrict__ ameta,
+                     const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmY,
+                     const uint32_t *__restrict__ ameta,
                      const uint32_t *__restrict__ rmeta, const uint8_t *__restrict__ phi, int phi_blocks,
                      int phi_cols, void *__restrict__ Y, int M, int N, int K, int32_t *status)
 {
     extern __shared__ uint8_t smem_raw[];
-    Smem &S = *reinterpret_cast<Smem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    Smem<CONV> &S =
+        *reinterpret_cast<Smem<CONV> *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const volatile int32_t *gstat = status;
 
@@ -121,7 +139,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&S.full[s], 1);
-            mbar_init(&S.conv[s], CONV_WARPS);
+            mbar_init(&S.conv[s], CONV ? CONV_WARPS : 1);
             mbar_init(&S.empty[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -137,6 +155,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (RES)
             prefetch_tmap(&tmR);
         prefetch_tmap(&tmB);
+        if (!CONV)
+            prefetch_tmap(&tmY);
     }
     if (warp == 1) {
         tmem_alloc(&S.tmem_base, TMEM_COLS);
@@ -166,18 +186,28 @@ __global__ void __launch_bounds__(THREADS, 1)
                         break;
                     }
                     const bool ron = res_on(m_tile, ks);
-                    uint32_t bytes = B16_BYTES + CODE_BYTES + META_BYTES;
-                    if (ron)
-                        bytes += CODE_BYTES + META_BYTES;
-                    Stage &st = S.st[slot];
+                    auto &st = S.st[slot];
                     uint64_t *bar = &S.full[slot];
-                    mbar_arrive_expect_tx(bar, bytes);
-                    tma_load_2d(st.b, &tmB, bar, ks * BK * 2, n_tile * BN);
-                    tma_load_2d(st.acode, &tmA, bar, ks * BK / 2, m_tile * BM);
-                    bulk_load(st.ameta, ameta + ks * mpad + (int64_t)m_tile * BM, META_BYTES, bar);
-                    if (ron) {
-                        tma_load_2d(st.rcode, &tmR, bar, ks * BK / 2, m_tile * BM);
-                        bulk_load(st.rmeta, rmeta + ks * mpad + (int64_t)m_tile * BM, META_BYTES, bar);
+                    if (CONV) {
+                        uint32_t bytes = B16_BYTES + CODE_BYTES + META_BYTES;
+                        if (ron)
+                            bytes += CODE_BYTES + META_BYTES;
+                        mbar_arrive_expect_tx(bar, bytes);
+                        tma_load_2d(st.b, &tmB, bar, ks * BK * 2, n_tile * BN);
+                        if constexpr (CONV) {
+                            tma_load_2d(st.acode, &tmA, bar, ks * BK / 2, m_tile * BM);
+                            bulk_load(st.ameta, ameta + ks * mpad + (int64_t)m_tile * BM, META_BYTES, bar);
+                            if (ron) {
+                                tma_load_2d(st.rcode, &tmR, bar, ks * BK / 2, m_tile * BM);
+                                bulk_load(st.rmeta, rmeta + ks * mpad + (int64_t)m_tile * BM, META_BYTES, bar);
+                            }
+                        }
+                    } else {
+                        mbar_arrive_expect_tx(bar, B16_BYTES + A16_BYTES + (ron ? A16_BYTES : 0));
+                        tma_load_2d(st.b, &tmB, bar, ks * BK * 2, n_tile * BN);
+                        tma_load_2d(st.a16, &tmA, bar, ks * BK * 2, m_tile * BM);
+                        if (ron)
+                            tma_load_2d(st.r16, &tmR, bar, ks * BK * 2, m_tile * BM);
                     }
                 }
             }
@@ -201,13 +231,13 @@ __global__ void __launch_bounds__(THREADS, 1)
                 for (int ks = 0; ks < nks; ++ks, ++p) {
                     const int slot = p % STAGES;
                     if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat) ||
-                        !mbar_wait(&S.conv[slot], (p / STAGES) & 1, kWaitLimitNs, gstat)) {
+                        (CONV && !mbar_wait(&S.conv[slot], (p / STAGES) & 1, kWaitLimitNs, gstat))) {
                         flag_timeout(S, status);
                         stop = true;
                         break;
                     }
                     tc_fence_after();
-                    const Stage &st = S.st[slot];
+                    const auto &st = S.st[slot];
                     const uint32_t a0 = smem_u32(st.a16), r0 = smem_u32(st.r16), b0 = smem_u32(st.b);
                     const bool ron = res_on(m_tile, ks);
 #pragma unroll
@@ -243,6 +273,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             const int row = m_tile * BM + q * 32 + lane;
             const bool store = row < M;
             const uint32_t acc = tmem + 256 * buf + ((uint32_t)(q * 32) << 16);
+            uint8_t *stg = S.ystage + (CONV ? 0 : (warp - 2) * YSTAGE);
 #pragma unroll 1
             for (int c = 0; c < BN / 32; ++c) {
                 uint32_t v[32];
@@ -255,7 +286,43 @@ __global__ void __launch_bounds__(THREADS, 1)
                         mbar_arrive(&S.acc_empty[buf]);
                 }
                 const int col = n_tile * BN + c * 32;
-                if (!store || col >= N)
+                if (col >= N)
+                    continue;
+                if (!CONV) {
+                    // shared-memory stage (64B swizzle) + TMA store, clipped at M and N
+                    const uint32_t sw = (uint32_t)((lane >> 1) & 3);
+#pragma unroll
+                    for (int hb = 0; hb < (OUT_BF16 ? 1 : 2); ++hb) {
+                        if (col + 16 * hb >= N)
+                            break;
+                        if (lane == 0)
+                            bulk_wait_group_read<0>();
+                        __syncwarp();
+                        uint32_t pk[16];
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            if (OUT_BF16) {
+                                __nv_bfloat162 b2 = __floats2bfloat162_rn(__uint_as_float(v[2 * i]),
+                                                                          __uint_as_float(v[2 * i + 1]));
+                                pk[i] = *reinterpret_cast<uint32_t *>(&b2);
+                            } else {
+                                pk[i] = v[16 * hb + i];
+                            }
+                        }
+#pragma unroll
+                        for (int j = 0; j < 4; ++j)
+                            *reinterpret_cast<uint4 *>(stg + lane * 64 + ((j ^ sw) << 4)) =
+                                make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
+                        fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) {
+                            tma_store_2d(&tmY, stg, OUT_BF16 ? col * 2 : (col + 16 * hb) * 4, m_tile * BM + q * 32);
+                            bulk_commit_group();
+                        }
+                    }
+                    continue;
+                }
+                if (!store)
                     continue;
                 const int nvalid = min(32, N - col);
                 if (OUT_BF16) {
@@ -283,7 +350,10 @@ __global__ void __launch_bounds__(THREADS, 1)
             if (S.abort_flag)
                 break;
         }
+        if (!CONV && lane == 0)
+            bulk_wait_group<0>(); // every TMA store of this warp has completed
     } else {
+        if constexpr (CONV) {
         // ------------------------------------------------ converters (warps 6..13)
         // 2 x 128 rows x 8 groups of 8 elements per stage; thread u handles
         // chunks u, u + 256, ... (row = chunk / 8, group = chunk % 8).
@@ -300,7 +370,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     stop = true;
                     break;
                 }
-                Stage &st = S.st[slot];
+                auto &st = S.st[slot];
                 const bool ron = res_on(m_tile, ks);
 #pragma unroll 2
                 for (int ch = u; ch < 2 * BM * 8; ch += 32 * CONV_WARPS) {
@@ -322,6 +392,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     mbar_arrive(&S.conv[slot]);
             }
         }
+        }
     }
 
     // ---------------------------------------------------- teardown
@@ -339,42 +410,46 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
 }
 
-template <bool RES, bool PHI, bool OUT>
+template <bool CONV, bool RES, bool PHI, bool OUT>
 cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const CUtensorMap &tb,
-                           const GemmHif4Args &a, cudaStream_t st)
+                           const CUtensorMap &ty, const GemmHif4Args &a, cudaStream_t st)
 {
-    auto kern = gemm_hif4_kernel<RES, PHI, OUT>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+    auto kern = gemm_hif4_kernel<CONV, RES, PHI, OUT>;
+    constexpr size_t smem = smem_bytes<CONV>();
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess)
         return e;
     const int64_t tiles = ((a.N + BN - 1) / BN) * ((a.M + BM - 1) / BM);
     const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
     const int phi_blocks = a.phi_r_s / BK;
     const int phi_cols = a.phi ? (int)((a.K + a.phi_r_s - 1) / a.phi_r_s) : 0;
-    kern<<<grid, THREADS, kSmemBytes, st>>>(ta, tr, tb, (const uint32_t *)a.a_meta, (const uint32_t *)a.r_meta,
-                                            a.phi, phi_blocks, phi_cols, a.y, (int)a.M, (int)a.N, (int)a.K,
-                                            a.status);
+    kern<<<grid, THREADS, smem, st>>>(ta, tr, tb, ty, (const uint32_t *)a.a_meta, (const uint32_t *)a.r_meta, a.phi,
+                                      phi_blocks, phi_cols, a.y, (int)a.M, (int)a.N, (int)a.K, a.status);
     return cudaGetLastError();
 }
 
-} // namespace
-
-cudaError_t launch_gemm_hif4(const GemmHif4Args &a, cudaStream_t st)
+template <bool CONV>
+cudaError_t launch_conv(const GemmHif4Args &a, cudaStream_t st)
 {
-    CUtensorMap ta, tr, tb;
-    const uint64_t kb = (uint64_t)a.K / 2;
-    if (!encode_tmap_2d_u8(&ta, a.a_codes, kb, (uint64_t)a.M, kb, BK / 2, BM, 0))
+    CUtensorMap ta, tr, tb, ty;
+    const uint64_t kb = CONV ? (uint64_t)a.K / 2 : (uint64_t)a.K * 2; // bytes per activation row
+    const uint32_t box = CONV ? BK / 2 : BK * 2;
+    const int swz = CONV ? 0 : 128;
+    if (!encode_tmap_2d_u8(&ta, a.a_codes, kb, (uint64_t)a.M, kb, box, BM, swz))
         return cudaErrorInvalidValue;
     if (!encode_tmap_2d_u8(&tb, a.b_bf16, (uint64_t)a.K * 2, (uint64_t)a.N, (uint64_t)a.K * 2, BK * 2, BN, 128))
         return cudaErrorInvalidValue;
     if (a.r_codes) {
-        if (!encode_tmap_2d_u8(&tr, a.r_codes, kb, (uint64_t)a.M, kb, BK / 2, BM, 0))
+        if (!encode_tmap_2d_u8(&tr, a.r_codes, kb, (uint64_t)a.M, kb, box, BM, swz))
             return cudaErrorInvalidValue;
     } else {
         tr = ta;
     }
+    const uint64_t yrow = (uint64_t)a.N * (a.out_bf16 ? 2 : 4);
+    if (!encode_tmap_2d_u8(&ty, a.y, yrow, (uint64_t)a.M, yrow, 64, 32, 64))
+        return cudaErrorInvalidValue;
     const bool res = a.r_codes != nullptr, phi = res && a.phi != nullptr;
-#define RFQ_GV(R, P, O) return launch_variant<R, P, O>(ta, tr, tb, a, st)
+#define RFQ_GV(R, P, O) return launch_variant<CONV, R, P, O>(ta, tr, tb, ty, a, st)
     if (!res) {
         if (a.out_bf16) RFQ_GV(false, false, true);
         RFQ_GV(false, false, false);
@@ -386,6 +461,13 @@ cudaError_t launch_gemm_hif4(const GemmHif4Args &a, cudaStream_t st)
     if (a.out_bf16) RFQ_GV(true, false, true);
     RFQ_GV(true, false, false);
 #undef RFQ_GV
+}
+
+} // namespace
+
+cudaError_t launch_gemm_hif4(const GemmHif4Args &a, cudaStream_t st)
+{
+    return a.a_bf16 ? launch_conv<false>(a, st) : launch_conv<true>(a, st);
 }
 
 } // namespace rfq

@@ -64,7 +64,8 @@ cudaError_t launch_dequant_mxfp4_bf16(const void *codes, const void *scales, int
 
 // ---- HiF4 RFQ GEMM (gemm_hif4.cu)
 struct GemmHif4Args {
-    const void *a_codes, *r_codes;   // [M][K/2] HiF4 codes; r_codes may be null
+    bool a_bf16;                     // activations given as exact bf16 expansions [M][K]
+    const void *a_codes, *r_codes;   // [M][K/2] HiF4 codes (or bf16 [M][K]); r_codes may be null
     const void *a_meta, *r_meta;     // block-major [K/64][Mpad] metadata words
     const void *b_bf16;              // exact bf16 expansion of W~, [N][K]
     const uint8_t *phi;

@@ -83,24 +83,28 @@ __device__ __forceinline__ uint32_t hif4_group(const float (&x)[8], float S, int
     for (int h = 0; h < 2; ++h) {
         const int ex = e18 + (h ? e116_1 : e116_0);
         const float step = 0.25f * S * (float)(1 << ex); // exact: S has 3 significant bits
+        const float inv = __frcp_rn(step);
+        const float hstep = 0.5f * step;
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             const float v = x[4 * h + i];
             const float a = fabsf(v);
-            // nearest k from the rounded quotient, then fixed up with exact
-            // comparisons against the midpoints (k +- 1/2) step
-            int k = (int)rintf(__fdiv_rn(a, step));
-            k = min(max(k, 0), 8);
-            const float hi = (float)(2 * k + 1) * 0.5f * step, lo = (float)(2 * k - 1) * 0.5f * step;
-            if (a > hi || (a == hi && (k & 1)))
-                ++k;
-            else if (k > 0 && (a < lo || (a == lo && (k & 1))))
-                --k;
-            k = min(k, 7);
-            const uint32_t s = __float_as_uint(v) >> 31;
-            codes |= (uint32_t)((s << 3) | k) << (4 * (4 * h + i));
-            const float q = (float)k * step;
-            deq[4 * h + i] = s ? -q : q;
+            // nearest k from the (approximate) quotient, kept in fp32, then
+            // fixed up with exact comparisons against the midpoints
+            // (k +- 1/2) step; ties go to even k
+            float k = rintf(fminf(a * inv, 8.0f));
+            const float hi = fmaf(k, step, hstep), lo = fmaf(k, step, -hstep);   // exact
+            const bool odd = (__float_as_uint(k + 8388608.0f) & 1u) != 0;
+            if (a > hi || (a == hi && odd))
+                k += 1.0f;
+            else if (k > 0.0f && (a < lo || (a == lo && odd)))
+                k -= 1.0f;
+            k = fminf(k, 7.0f);
+            const uint32_t ki = __float_as_uint(k + 8388608.0f) & 7u;   // k as an integer, exactly
+            const uint32_t sgn = __float_as_uint(v) >> 31;
+            codes |= ((sgn << 3) | ki) << (4 * (4 * h + i));
+            const float q = k * step;
+            deq[4 * h + i] = sgn ? -q : q;
         }
     }
     return codes;

@@ -128,7 +128,14 @@ def test_dequant_fp32_and_bf16_exact(orc):
                 assert np.array_equal(out.double().cpu().numpy(), ref)
 
 
-def _linear(xb, wb, out=rfq.RFQ_OUT_F32, mode=rfq.RFQ_FALLBACK_ALL, tau=0.0, r_s=256, use_phi=False):
+def _expand(q):
+    t = rfq.empty_bf16_operand(q.rows, q.k)
+    rfq.rfq_dequant(q, t.codes)
+    return t
+
+
+def _linear(xb, wb, out=rfq.RFQ_OUT_F32, mode=rfq.RFQ_FALLBACK_ALL, tau=0.0, r_s=256, use_phi=False,
+            expand=False):
     M, K = xb.shape
     N = wb.shape[1]
     wq = rfq.empty_qtensor(H, rfq.RFQ_SCALE_ROWMAJOR, N, K)
@@ -139,7 +146,8 @@ def _linear(xb, wb, out=rfq.RFQ_OUT_F32, mode=rfq.RFQ_FALLBACK_ALL, tau=0.0, r_s
     y = torch.full((M, N), float("nan"), dtype=torch.float32 if out == rfq.RFQ_OUT_F32 else torch.bfloat16,
                    device=DEV)
     ws = torch.zeros(64, dtype=torch.int32, device=DEV)
-    rfq.rfq_linear(xq, xr, phi if use_phi else None, r_s, w16, y, out, ws)
+    a, r = (_expand(xq), _expand(xr) if xr is not None else None) if expand else (xq, xr)
+    rfq.rfq_linear(a, r, phi if use_phi else None, r_s, w16, y, out, ws)
     assert rfq.rfq_workspace_status(ws) == rfq.RFQ_OK
     return xq, xr, wq, y.double().cpu().numpy()
 
@@ -151,31 +159,33 @@ def _ref(orc, xq, xr, wq, M, K, N):
     return orc.linear(orc.FMT_HIF4, mc, mm, rc, rm, wc, wm, M, K, N)
 
 
+@pytest.mark.parametrize("expand", [False, True])
 @pytest.mark.parametrize("M,K,N", [(1, 64, 16), (128, 512, 256), (129, 640, 272), (300, 1024, 528)])
-def test_linear_shapes(orc, M, K, N):
+def test_linear_shapes(orc, M, K, N, expand):
     xb = make_activation(ActSpec(M, K, "laplace", body_scale=0.3, chan_count=2, chan_scale=50.0, seed=M + N))
     wb = make_weight(K, N, seed=K)
-    xq, xr, wq, y = _linear(xb, wb)
+    xq, xr, wq, y = _linear(xb, wb, expand=expand)
     check_y(y, _ref(orc, xq, xr, wq, M, K, N))
 
 
-def test_linear_no_residual_and_phi(orc):
+@pytest.mark.parametrize("expand", [False, True])
+def test_linear_no_residual_and_phi(orc, expand):
     M, K, N = 256, 1024, 256
     xb = make_activation(ActSpec(M, K, "laplace", body_scale=0.3, chan_count=3, chan_scale=50.0, seed=5))
     wb = make_weight(K, N, seed=5)
-    xq, xr, wq, y = _linear(xb, wb, mode=rfq.RFQ_FALLBACK_NONE)
+    xq, xr, wq, y = _linear(xb, wb, mode=rfq.RFQ_FALLBACK_NONE, expand=expand)
     check_y(y, _ref(orc, xq, None, wq, M, K, N))
-    xq, xr, wq, y = _linear(xb, wb, mode=rfq.RFQ_FALLBACK_AMAX, tau=10.0, r_s=128, use_phi=True)
+    xq, xr, wq, y = _linear(xb, wb, mode=rfq.RFQ_FALLBACK_AMAX, tau=10.0, r_s=128, use_phi=True, expand=expand)
     check_y(y, _ref(orc, xq, xr, wq, M, K, N))
 
 
-@pytest.mark.parametrize("out", [rfq.RFQ_OUT_BF16, rfq.RFQ_OUT_F32])
-def test_full_size_qwen_down_hif4(orc, out):
+@pytest.mark.parametrize("out,expand", [(rfq.RFQ_OUT_BF16, True), (rfq.RFQ_OUT_F32, True), (rfq.RFQ_OUT_BF16, False)])
+def test_full_size_qwen_down_hif4(orc, out, expand):
     spec = WORKLOADS["qwen_down_hif4"]
     M, K, N = spec.act.M, spec.act.K, spec.N
     xb = make_activation(spec.act)
     wb = make_weight(K, N, seed=spec.act.seed)
-    xq, xr, wq, y = _linear(xb, wb, out=out)
+    xq, xr, wq, y = _linear(xb, wb, out=out, expand=expand)
     wc, wm = qtensor_host(wq)
     rwc, rwm = orc.quantize_weight(wb, orc.FMT_HIF4)
     assert np.array_equal(wc, rwc) and np.array_equal(wm, rwm)
