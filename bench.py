@@ -342,13 +342,16 @@ def run_rfq(args):
 
     flop = 2.0 * 2.0 * M * N * K                 # main + residual product, phi = 1 everywhere
     pk = _peaks()
+    # The timed loop is short (tens of ms at full clocks), so the kernels are
+    # held against the burst figure; the sustained one is reported beside it.
     if hif4:
         # HiF4 runs on the bf16 tensor path (exact bf16 expansion)
-        t_peak, t_src = pk["bf16_sust"], f"{pk['src']} bf16 sustained {pk['bf16_sust']} TFLOP/s, of {pk['src']}"
+        t_peak, t_peak_sust = pk["bf16_burst"], pk["bf16_sust"]
+        t_src = f"{pk['src']} bf16 burst {pk['bf16_burst']} TFLOP/s, of {pk['src']}"
         t_kernel = "gemm_hif4_kernel"
     else:
-        t_peak = pk["bf16_sust"] * FP4_OVER_BF16
-        t_src = (f"{pk['src']} bf16 sustained {pk['bf16_sust']} TFLOP/s x {FP4_OVER_BF16:g} "
+        t_peak, t_peak_sust = pk["bf16_burst"] * FP4_OVER_BF16, pk["bf16_sust"] * FP4_OVER_BF16
+        t_src = (f"{pk['src']} bf16 burst {pk['bf16_burst']} TFLOP/s x {FP4_OVER_BF16:g} "
                  f"(nominal dense FP4/BF16 ratio), of {pk['src']}")
         t_kernel = "gemm_mxf4_kernel"
     if hif4:
@@ -372,7 +375,7 @@ def run_rfq(args):
         roofline = {"bound": "tensor", "kernel": t_kernel, "achieved": gemm_tflops, "peak": t_peak,
                     "unit": "TFLOP/s", "frac": gemm_tflops / t_peak,
                     "traffic": _kernel_traffic(t_kernel, spec.name), "flop_per_launch": flop, "ms_per_launch": g_ms,
-                    "peak_source": t_src}
+                    "peak_source": t_src, "frac_of_sustained_peak": gemm_tflops / t_peak_sust}
     clocks = clk.summary()
     if e2e_ms is not None:
         e2e = {"value": ws * (aq_bytes / 1e9 if quant_only else flop / 1e12) / (e2e_ms * 1e-3), "unit": unit,
