@@ -48,13 +48,20 @@ def _peaks():
     return dict(hbm=6800.0, bf16_burst=1900.0, bf16_sust=1700.0, src="fallback")
 
 
+# source file of each timed kernel: its DRAM counters hold only for the
+# sources they were taken on (the kernel's file plus the shared headers)
+_KERNEL_SRC = {"gemm_mxf4_kernel": "gemm_mxf4.cu", "act_quant_mxfp4_kernel": "quant_mxfp4.cu",
+               "gemm_hif4_kernel": "gemm_hif4.cu", "act_quant_hif4_kernel": "quant_hif4.cu"}
+
+
 def _kernel_traffic(kernel: str, workload: str):
-    """DRAM bytes per launch from a committed ncu summary, if it was taken on
-    the current kernel sources (matching hash); else None."""
+    """DRAM bytes per launch from profiles/dram_traffic.txt (an ncu capture of
+    that kernel on that workload), if the kernel's sources still hash to the
+    value recorded there; else None."""
     path = os.path.join(HERE, "profiles", "dram_traffic.txt")
-    if not os.path.exists(path):
+    if not os.path.exists(path) or kernel not in _KERNEL_SRC:
         return None
-    h = _src_hash()
+    h = _src_hash(kernel)
     for line in open(path):
         f = line.split()
         if len(f) >= 4 and not line.startswith("#") and f[0] == kernel and f[1] == workload and f[2] == h:
@@ -62,10 +69,10 @@ def _kernel_traffic(kernel: str, workload: str):
     return None
 
 
-def _src_hash():
+def _src_hash(kernel: str):
     d = os.path.join(HERE, "paper_2608_26581_gb300", "csrc")
     m = hashlib.sha256()
-    for n in sorted(os.listdir(d)):
+    for n in (_KERNEL_SRC[kernel], "ptx.cuh", "internal.h"):
         m.update(open(os.path.join(d, n), "rb").read())
     return m.hexdigest()[:16]
 

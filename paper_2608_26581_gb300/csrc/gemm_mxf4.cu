@@ -2,27 +2,31 @@
 // Eq. rfq):  Y = X~ W~ + phi X^ W~.
 //
 // Persistent kernel: one CTA per SM walks output tiles of 128 x 256.  Per
-// 128-element k-stage the TMA producer stages the main A tile (X~ codes), the
-// residual A tile (X^ codes), the W~ tile and their E8M0 scale atoms in
-// shared memory (six stages in flight).  Four scale-writer warps (one per TMEM
-// lane quarter) move each stage's scale atoms from shared memory into TMEM
-// with tcgen05.st, which keeps the scale traffic off the MMA issue path; the
-// MMA thread then issues, per K=64 step, the main MMA and the residual MMA
-// against the SAME shared-memory W~ tile into the SAME TMEM accumulator:
-// W~ is read once for both products and the correction costs only MMA issue
-// (the on-the-fly residual accumulation of Sec. 4.3).  Residual MMAs of
-// k-tiles with phi = 0 are not issued and their A tiles are not loaded.
-// Eight epilogue warps drain the fp32 accumulator (TMEM -> registers ->
-// fp32 or bf16 Y); the producer keeps loading the next tile meanwhile, and the
-// MMA thread starts it as soon as the accumulator has been read.
+// 256-element k-stage the TMA producer stages the main A tile (X~ codes), the
+// residual A tile (X^ codes), the W~ tile (128-byte rows, 128-byte swizzle)
+// and their E8M0 scale atoms (bulk copies) in shared memory, three 68 KB
+// stages in flight.  Four scale-writer warps (one per TMEM lane quarter) move
+// each stage's scale words from shared memory into a ring of four TMEM scale
+// slots with tcgen05.st (a scale copy issued by the MMA thread would wait for
+// its earlier MMAs).  With four slots and three stages, a slot is rewritten
+// only after its previous stage's MMAs completed: the writers wait for the
+// stage's copies, which the producer issued after those MMAs released the
+// shared-memory stage.  The MMA
+// thread issues, per K=64 step, the main MMA and the residual MMA against the
+// SAME shared-memory W~ tile into the SAME TMEM accumulator: W~ is read once
+// for both products and the correction costs only MMA issue (the on-the-fly
+// residual accumulation of Sec. 4.3).  Residual MMAs of k-chunks with
+// phi = 0 are not issued and their A tiles are not loaded.  Eight epilogue
+// warps drain the fp32 accumulator; with bf16 Y each warp first loads and
+// packs all 128 of its columns, hands the accumulator back to the MMA thread,
+// then stages and stores them (shared memory + TMA stores), so the next
+// tile's MMAs start after the loads only.
 //
 // Scale layout in TMEM (per 128-element k-chunk): 4 columns per 128 rows,
 // column j of lane i (of every lane quarter) holding the four scales of row
 // 32 j + i, i.e. lane i of a quarter takes bytes [16 i, 16 i + 16) of the
-// 512-byte MMA-layout atom.  Eight scale slots of 16 columns (A, R, B rows
-// 0-127, B rows 128-255) rotate per stage; with 8 slots >= 6 stages, a slot is
-// rewritten only after the stage that used it has had its MMAs complete (its
-// shared-memory slot was refilled, which waits for that).
+// 512-byte MMA-layout atom.  A slot holds one stage: A chunk c at 4c, R at
+// 8 + 4c, W~ rows 0-127 at 16 + 8c and rows 128-255 at 20 + 8c.
 //
 // Every mbarrier wait is bounded (kWaitLimitNs) and also gives up as soon as
 // any CTA has recorded a timeout in the caller's status word; the CTA then
@@ -38,85 +42,72 @@ namespace {
 
 constexpr int BM = 128;
 constexpr int BN = 256;
+constexpr int BK = 256;                // k-elements per stage (two 128-element chunks)
+constexpr int ROW = BK / 2;            // bytes of codes per row per stage
+constexpr int A_BYTES = BM * ROW;
+constexpr int B_BYTES = BN * ROW;
+constexpr int STAGES = 3;
 constexpr int ATOM = 512;              // scale bytes of 128 rows x one 128-element chunk
 constexpr int TMEM_COLS = 512;
 constexpr int SF_COL0 = 256;           // TMEM columns [256, 384): scale slots
+constexpr int SF_SLOT_COLS = 32;
+constexpr int SF_SLOTS = 4;
 constexpr int EPI_WARPS = 8;
 constexpr int SF_WARPS = 4;
 constexpr int THREADS = 64 + 32 * EPI_WARPS + 32 * SF_WARPS;
+static_assert(SF_COL0 + SF_SLOTS * SF_SLOT_COLS <= TMEM_COLS, "TMEM budget");
+static_assert(SF_SLOTS >= STAGES, "a scale slot is rewritten only after its stage's MMAs completed");
 
-// Pipeline shape for a k-stage of KC 128-element chunks (BK = 128 KC
-// elements, 64 KC bytes of codes per row, swizzle = that row length).
-template <int KC>
-struct Cfg {
-    static constexpr int BK = 128 * KC;
-    static constexpr int ROW = BK / 2;                  // bytes per row per stage
-    static constexpr int A_BYTES = BM * ROW;
-    static constexpr int B_BYTES = BN * ROW;
-    static constexpr int STAGES = KC == 1 ? 6 : 3;
-    static constexpr int SF_STRIDE = 16 * KC;           // TMEM columns per scale slot
-    static constexpr int SF_SLOTS = KC == 1 ? 8 : 4;    // slots of SF_STRIDE columns
-    static_assert(SF_SLOTS >= STAGES, "a scale slot is rewritten only after its stage's MMAs completed");
-    static_assert(SF_SLOTS * SF_STRIDE <= 128, "scale slots fit in TMEM columns [256, 384)");
-};
-
-template <int KC>
 struct alignas(1024) Stage {
-    uint8_t a[Cfg<KC>::A_BYTES];
-    uint8_t r[Cfg<KC>::A_BYTES];
-    uint8_t b[Cfg<KC>::B_BYTES];
-    uint8_t sfa[KC * ATOM];            // chunk c at c * ATOM
-    uint8_t sfr[KC * ATOM];
-    uint8_t sfb[2 * KC * ATOM];        // W~ rows 128 h..128 h + 127: chunk c at (h * KC + c) * ATOM
+    uint8_t a[A_BYTES];
+    uint8_t r[A_BYTES];
+    uint8_t b[B_BYTES];
+    uint8_t sfa[2 * ATOM];             // chunk c at c * ATOM
+    uint8_t sfr[2 * ATOM];
+    uint8_t sfb[4 * ATOM];             // W~ rows 128 h..128 h + 127: chunk c at (2 h + c) * ATOM
 };
 
 constexpr int YSTAGE = 2048;          // per epilogue warp: 32 rows x 64 bytes of Y
 
-template <int KC>
 struct Smem {
-    Stage<KC> st[Cfg<KC>::STAGES];
+    Stage st[STAGES];
     alignas(1024) uint8_t ystage[EPI_WARPS * YSTAGE]; // 64B-swizzled staging for the TMA stores of Y
-    uint64_t full[Cfg<KC>::STAGES];
-    uint64_t empty[Cfg<KC>::STAGES];
+    uint64_t full[STAGES];
+    uint64_t empty[STAGES];
     uint64_t acc_full;
     uint64_t acc_empty;
     uint64_t drain;
-    uint64_t sf_ready[Cfg<KC>::SF_SLOTS];
+    uint64_t sf_ready[SF_SLOTS];      // the scale writers filled the slot
     uint32_t tmem_base;
     int32_t abort_flag;
     int32_t issued;
 };
 
-template <int KC>
-constexpr size_t smem_bytes() { return sizeof(Smem<KC>) + 1024; }
-static_assert(smem_bytes<1>() <= 227 * 1024 && smem_bytes<2>() <= 227 * 1024, "shared memory budget");
+constexpr size_t kSmemBytes = sizeof(Smem) + 1024;
+static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 
-template <int KC>
-__device__ __forceinline__ uint64_t sdesc_k(uint32_t saddr)
-{
-    return KC == 1 ? sdesc_k_sw64(saddr) : sdesc_k_sw128(saddr);
-}
-
-template <class SM>
-__device__ __forceinline__ void flag_timeout(SM &S, int32_t *status)
+__device__ __forceinline__ void flag_timeout(Smem &S, int32_t *status)
 {
     S.abort_flag = 1;
     atomicExch(status, kDevTimeout);
 }
 
-template <int KC, bool RES, bool PHI, bool OUT_BF16>
+template <bool PHI>
+__device__ __forceinline__ bool res_chunk(const uint8_t *phi, int m_tile, int phi_cols, int phi_chunks, int chunk)
+{
+    return !PHI || phi[(int64_t)m_tile * phi_cols + chunk / phi_chunks] != 0;
+}
+
+template <bool RES, bool PHI, bool OUT_BF16>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_mxf4_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmR,
                      const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmY,
-                     const uint8_t *__restrict__ sfa,
-                     const uint8_t *__restrict__ sfr, const uint8_t *__restrict__ sfb,
-                     const uint8_t *__restrict__ phi, int phi_chunks, int phi_cols, void *__restrict__ Y, int M,
-                     int N, int K, int32_t *status)
+                     const uint8_t *__restrict__ sfa, const uint8_t *__restrict__ sfr,
+                     const uint8_t *__restrict__ sfb, const uint8_t *__restrict__ phi, int phi_chunks,
+                     int phi_cols, int M, int N, int K, int32_t *status)
 {
     extern __shared__ uint8_t smem_raw[];
-    using C = Cfg<KC>;
-    constexpr int STAGES = C::STAGES, SF_SLOTS = C::SF_SLOTS, BK = C::BK;
-    Smem<KC> &S = *reinterpret_cast<Smem<KC> *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    Smem &S = *reinterpret_cast<Smem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const volatile int32_t *gstat = status;
 
@@ -129,7 +120,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     __syncthreads();
 
     const int kc = K >> 7;                 // 128-element chunks
-    const int nks = (kc + KC - 1) / KC;    // k-stages (the last may hold fewer chunks)
+    const int nks = (kc + 1) >> 1;         // k-stages (the last may hold one chunk)
     const int n_tiles = (N + BN - 1) / BN;
     const int m_tiles = (M + BM - 1) / BM;
     const int tiles = n_tiles * m_tiles;
@@ -178,31 +169,27 @@ __global__ void __launch_bounds__(THREADS, 1)
                         stop = true;
                         break;
                     }
-                    const int c0 = ks * KC, nch = min(KC, kc - c0);
-                    bool res_on = RES;
-                    if (RES && PHI) {
-                        res_on = false;
+                    const int c0 = 2 * ks, nch = min(2, kc - c0);
+                    bool res_on = false;
+                    if (RES)
                         for (int c = 0; c < nch; ++c)
-                            res_on |= phi[(int64_t)m_tile * phi_cols + (c0 + c) / phi_chunks] != 0;
-                    }
+                            res_on |= res_chunk<PHI>(phi, m_tile, phi_cols, phi_chunks, c0 + c);
                     const int atom0 = n_tile * 2;
                     const int nb = atom0 + 1 < n_atoms ? 2 : 1;
-                    uint32_t bytes = C::A_BYTES + C::B_BYTES + (1 + nb) * nch * ATOM;
-                    if (res_on)
-                        bytes += C::A_BYTES + nch * ATOM;
-                    Stage<KC> &st = S.st[slot];
+                    const uint32_t sfbytes = (uint32_t)nch * ATOM;
+                    Stage &st = S.st[slot];
                     uint64_t *bar = &S.full[slot];
-                    mbar_arrive_expect_tx(bar, bytes);
+                    mbar_arrive_expect_tx(bar, A_BYTES + B_BYTES + (1 + nb) * sfbytes +
+                                                   (res_on ? A_BYTES + sfbytes : 0));
                     tma_load_2d(st.a, &tmA, bar, c0 * 64, m_tile * BM);
                     if (res_on)
                         tma_load_2d(st.r, &tmR, bar, c0 * 64, m_tile * BM);
                     tma_load_2d(st.b, &tmB, bar, c0 * 64, n_tile * BN);
-                    bulk_load(st.sfa, sfa + ((int64_t)m_tile * kc + c0) * ATOM, nch * ATOM, bar);
+                    bulk_load(st.sfa, sfa + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, bar);
                     if (res_on)
-                        bulk_load(st.sfr, sfr + ((int64_t)m_tile * kc + c0) * ATOM, nch * ATOM, bar);
+                        bulk_load(st.sfr, sfr + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, bar);
                     for (int h = 0; h < nb; ++h)
-                        bulk_load(st.sfb + h * KC * ATOM, sfb + ((int64_t)(atom0 + h) * kc + c0) * ATOM, nch * ATOM,
-                                  bar);
+                        bulk_load(st.sfb + h * 2 * ATOM, sfb + ((int64_t)(atom0 + h) * kc + c0) * ATOM, sfbytes, bar);
                 }
             }
             S.issued = p;
@@ -220,30 +207,29 @@ __global__ void __launch_bounds__(THREADS, 1)
                 }
                 tc_fence_after();
                 for (int ks = 0; ks < nks; ++ks, ++p) {
-                    const int slot = p % STAGES;
+                    const int slot = p % STAGES, sfs = p % SF_SLOTS;
                     if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat) ||
-                        !mbar_wait(&S.sf_ready[p % SF_SLOTS], (p / SF_SLOTS) & 1, kWaitLimitNs, gstat)) {
+                        !mbar_wait(&S.sf_ready[sfs], (p / SF_SLOTS) & 1, kWaitLimitNs, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
                         break;
                     }
                     tc_fence_after();
-                    const int c0 = ks * KC, nch = min(KC, kc - c0);
-                    // scale slot columns: A chunk c at 4c, R at 4 KC + 4c, W~ at 8 KC + 8c (+4: rows 128-255)
-                    const uint32_t sf = tmem + SF_COL0 + C::SF_STRIDE * (p % SF_SLOTS);
-                    const Stage<KC> &st = S.st[slot];
+                    const int c0 = 2 * ks, nch = min(2, kc - c0);
+                    const uint32_t sf = tmem + SF_COL0 + SF_SLOT_COLS * sfs;
+                    const Stage &st = S.st[slot];
                     const uint32_t a0 = smem_u32(st.a), r0 = smem_u32(st.r), b0 = smem_u32(st.b);
 #pragma unroll
-                    for (int j = 0; j < 2 * KC; ++j) {
+                    for (int j = 0; j < 4; ++j) {
                         const int c = j >> 1;
                         if (c >= nch)
                             break;
                         const uint32_t id = idesc_mxf4(BM, BN, 2 * (j & 1), 2 * (j & 1));
-                        const uint64_t bd = sdesc_k<KC>(b0 + 32 * j);
-                        const uint32_t sfb_t = sf + 8 * KC + 8 * c;
-                        tc_mma_mxf4(tmem, sdesc_k<KC>(a0 + 32 * j), bd, id, sf + 4 * c, sfb_t, (ks | j) != 0);
-                        if (RES && (!PHI || phi[(int64_t)m_tile * phi_cols + (c0 + c) / phi_chunks] != 0))
-                            tc_mma_mxf4(tmem, sdesc_k<KC>(r0 + 32 * j), bd, id, sf + 4 * KC + 4 * c, sfb_t, 1);
+                        const uint64_t bd = sdesc_k_sw128(b0 + 32 * j);
+                        const uint32_t sfb_t = sf + 16 + 8 * c;
+                        tc_mma_mxf4(tmem, sdesc_k_sw128(a0 + 32 * j), bd, id, sf + 4 * c, sfb_t, (ks | j) != 0);
+                        if (RES && res_chunk<PHI>(phi, m_tile, phi_cols, phi_chunks, c0 + c))
+                            tc_mma_mxf4(tmem, sdesc_k_sw128(r0 + 32 * j), bd, id, sf + 8 + 4 * c, sfb_t, 1);
                     }
                     tc_commit(&S.empty[slot]);
                 }
@@ -260,64 +246,84 @@ __global__ void __launch_bounds__(THREADS, 1)
         // ------------------------------------------------ epilogue (warps 2..9)
         const int q = warp & 3;          // TMEM lane quarter this warp may access
         const int h = (warp - 2) >> 2;   // column half of the tile
+        uint8_t *stg = S.ystage + (warp - 2) * YSTAGE;
+        const uint32_t sw = (uint32_t)((lane >> 1) & 3);   // 64B swizzle: chunk j of row r at (j ^ ((r >> 1) & 3))
         int it = 0;
         for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++it) {
             const int m_tile = tile / n_tiles, n_tile = tile - m_tile * n_tiles;
-            if (!mbar_wait(&S.acc_full, it & 1, kWaitLimitNs, gstat)) {
+            // warp-uniform outcome: the tcgen05 loads below need the whole warp
+            if (!__all_sync(0xffffffffu, mbar_wait(&S.acc_full, it & 1, kWaitLimitNs, gstat))) {
                 if (lane == 0)
                     flag_timeout(S, status);
                 break;
             }
             tc_fence_after();
-            // Y goes out through a per-warp shared-memory stage and TMA
-            // stores: full-line writes, clipped by the hardware at M and N.
-            uint8_t *stg = S.ystage + (warp - 2) * YSTAGE;
             const int row0 = m_tile * BM + q * 32;
+            const uint32_t tcol = tmem + ((uint32_t)(q * 32) << 16) + h * (BN / 2);
+            if (OUT_BF16) {
+                // all 128 columns of this warp into registers as packed bf16,
+                // then the accumulator goes back to the MMA thread
+                uint32_t pk[64];
 #pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                // two 32-column chunks in flight; the accumulator goes back to
-                // the MMA thread after the last load of the tile
-                uint32_t v[2][32];
+                for (int g = 0; g < 2; ++g) {
+                    uint32_t v[2][32];
+                    tmem_ld_32x32b_x32(tcol + 64 * g, v[0]);
+                    tmem_ld_32x32b_x32(tcol + 64 * g + 32, v[1]);
+                    tmem_ld_wait();
 #pragma unroll
-                for (int c = 0; c < 2; ++c)
-                    tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + h * (BN / 2) + (2 * half + c) * 32,
-                                       v[c]);
-                tmem_ld_wait();
-                if (half == 1) {
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0)
-                        mbar_arrive(&S.acc_empty);
-                }
-#pragma unroll
-                for (int c = 0; c < 2; ++c) {
-                    const int col = n_tile * BN + h * (BN / 2) + (2 * half + c) * 32;
-                    if (col >= N)
-                        continue;
-                    // 64-byte rows, 16-byte chunk j of row r at r*64 + ((j ^ ((r >> 1) & 3)) << 4)
-                    const uint32_t sw = (uint32_t)((lane >> 1) & 3);
-                    if (OUT_BF16) {
-                        if (lane == 0)
-                            bulk_wait_group_read<0>();
-                        __syncwarp();
-                        uint32_t pk[16];
+                    for (int c = 0; c < 2; ++c)
 #pragma unroll
                         for (int i = 0; i < 16; ++i) {
                             __nv_bfloat162 b2 = __floats2bfloat162_rn(__uint_as_float(v[c][2 * i]),
                                                                       __uint_as_float(v[c][2 * i + 1]));
-                            pk[i] = *reinterpret_cast<uint32_t *>(&b2);
+                            pk[32 * g + 16 * c + i] = *reinterpret_cast<uint32_t *>(&b2);
                         }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(&S.acc_empty);
 #pragma unroll
-                        for (int j = 0; j < 4; ++j)
-                            *reinterpret_cast<uint4 *>(stg + lane * 64 + ((j ^ sw) << 4)) =
-                                make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
-                        fence_proxy_async_smem();
+                for (int c = 0; c < 4; ++c) {   // 32-column chunks: one 64-byte TMA box row per lane
+                    const int col = n_tile * BN + h * (BN / 2) + 32 * c;
+                    if (col >= N)
+                        break;
+                    if (lane == 0)
+                        bulk_wait_group_read<0>();
+                    __syncwarp();
+#pragma unroll
+                    for (int j = 0; j < 4; ++j)
+                        *reinterpret_cast<uint4 *>(stg + lane * 64 + ((j ^ sw) << 4)) =
+                            make_uint4(pk[16 * c + 4 * j], pk[16 * c + 4 * j + 1], pk[16 * c + 4 * j + 2],
+                                       pk[16 * c + 4 * j + 3]);
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tma_store_2d(&tmY, stg, col * 2, row0);
+                        bulk_commit_group();
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int half = 0; half < 2; ++half) {
+                    // two 32-column chunks in flight; the accumulator goes back
+                    // to the MMA thread after the last load of the tile
+                    uint32_t v[2][32];
+#pragma unroll
+                    for (int c = 0; c < 2; ++c)
+                        tmem_ld_32x32b_x32(tcol + (2 * half + c) * 32, v[c]);
+                    tmem_ld_wait();
+                    if (half == 1) {
+                        tc_fence_before();
                         __syncwarp();
-                        if (lane == 0) {
-                            tma_store_2d(&tmY, stg, col * 2, row0);
-                            bulk_commit_group();
-                        }
-                    } else {
+                        if (lane == 0)
+                            mbar_arrive(&S.acc_empty);
+                    }
+#pragma unroll
+                    for (int c = 0; c < 2; ++c) {
+                        const int col = n_tile * BN + h * (BN / 2) + (2 * half + c) * 32;
+                        if (col >= N)
+                            continue;
 #pragma unroll
                         for (int hb = 0; hb < 2; ++hb) { // 16 fp32 columns (64 bytes) per store
                             if (col + 16 * hb >= N)
@@ -356,37 +362,38 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x) {
             const int m_tile = tile / n_tiles;
             for (int ks = 0; ks < nks; ++ks, ++p) {
-                const int slot = p % STAGES;
-                if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat)) {
+                const int slot = p % STAGES, sfs = p % SF_SLOTS;
+                // warp-uniform outcome: the tcgen05 stores below need the whole warp
+                if (!__all_sync(0xffffffffu, mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat))) {
                     if (lane == 0)
                         flag_timeout(S, status);
                     stop = true;
                     break;
                 }
                 tc_fence_after();
-                const int c0 = ks * KC, nch = min(KC, kc - c0);
-                const Stage<KC> &st = S.st[slot];
-                const uint32_t tb = tmem + ((uint32_t)(q * 32) << 16) + SF_COL0 + C::SF_STRIDE * (p % SF_SLOTS);
+                const int c0 = 2 * ks, nch = min(2, kc - c0);
+                const Stage &st = S.st[slot];
+                const uint32_t tb = tmem + ((uint32_t)(q * 32) << 16) + SF_COL0 + SF_SLOT_COLS * sfs;
 #pragma unroll
-                for (int c = 0; c < KC; ++c) {
+                for (int c = 0; c < 2; ++c) {
                     if (c >= nch)
                         break;
                     const uint4 va = *reinterpret_cast<const uint4 *>(st.sfa + c * ATOM + lane * 16);
                     const uint4 vb0 = *reinterpret_cast<const uint4 *>(st.sfb + c * ATOM + lane * 16);
-                    const uint4 vb1 = *reinterpret_cast<const uint4 *>(st.sfb + (KC + c) * ATOM + lane * 16);
+                    const uint4 vb1 = *reinterpret_cast<const uint4 *>(st.sfb + (2 + c) * ATOM + lane * 16);
                     tmem_st_32x32b_x4(tb + 4 * c, va.x, va.y, va.z, va.w);
-                    if (RES && (!PHI || phi[(int64_t)m_tile * phi_cols + (c0 + c) / phi_chunks] != 0)) {
+                    if (RES && res_chunk<PHI>(phi, m_tile, phi_cols, phi_chunks, c0 + c)) {
                         const uint4 vr = *reinterpret_cast<const uint4 *>(st.sfr + c * ATOM + lane * 16);
-                        tmem_st_32x32b_x4(tb + 4 * KC + 4 * c, vr.x, vr.y, vr.z, vr.w);
+                        tmem_st_32x32b_x4(tb + 8 + 4 * c, vr.x, vr.y, vr.z, vr.w);
                     }
-                    tmem_st_32x32b_x4(tb + 8 * KC + 8 * c, vb0.x, vb0.y, vb0.z, vb0.w);
-                    tmem_st_32x32b_x4(tb + 8 * KC + 8 * c + 4, vb1.x, vb1.y, vb1.z, vb1.w);
+                    tmem_st_32x32b_x4(tb + 16 + 8 * c, vb0.x, vb0.y, vb0.z, vb0.w);
+                    tmem_st_32x32b_x4(tb + 20 + 8 * c, vb1.x, vb1.y, vb1.z, vb1.w);
                 }
                 tmem_st_wait();
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0)
-                    mbar_arrive(&S.sf_ready[p % SF_SLOTS]);
+                    mbar_arrive(&S.sf_ready[sfs]);
             }
         }
     }
@@ -407,38 +414,36 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
 }
 
-template <int KC, bool RES, bool PHI, bool OUT>
+template <bool RES, bool PHI, bool OUT>
 cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const CUtensorMap &tb,
                            const CUtensorMap &ty, const GemmMxf4Args &a, cudaStream_t st)
 {
-    auto kern = gemm_mxf4_kernel<KC, RES, PHI, OUT>;
-    constexpr size_t smem = smem_bytes<KC>();
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    auto kern = gemm_mxf4_kernel<RES, PHI, OUT>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (e != cudaSuccess)
         return e;
     const int64_t tiles = ((a.N + BN - 1) / BN) * ((a.M + BM - 1) / BM);
     const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
     const int phi_chunks = a.phi_r_s / 128;
     const int phi_cols = a.phi ? (int)((a.K + a.phi_r_s - 1) / a.phi_r_s) : 0;
-    kern<<<grid, THREADS, smem, st>>>(ta, tr, tb, ty, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf,
-                                      (const uint8_t *)a.b_sf, a.phi, phi_chunks, phi_cols, a.y, (int)a.M, (int)a.N,
-                                      (int)a.K, a.status);
+    kern<<<grid, THREADS, kSmemBytes, st>>>(ta, tr, tb, ty, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf,
+                                            (const uint8_t *)a.b_sf, a.phi, phi_chunks, phi_cols, (int)a.M,
+                                            (int)a.N, (int)a.K, a.status);
     return cudaGetLastError();
 }
 
-template <int KC>
-cudaError_t launch_kc(const GemmMxf4Args &a, cudaStream_t st)
+} // namespace
+
+cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st)
 {
     CUtensorMap ta, tr, tb;
     const uint64_t kb = (uint64_t)a.K / 2;
-    constexpr uint32_t row = Cfg<KC>::ROW;
-    constexpr int swz = KC == 1 ? 64 : 128;
-    if (!encode_tmap_2d_u8(&ta, a.a_codes, kb, (uint64_t)a.M, kb, row, BM, swz))
+    if (!encode_tmap_2d_u8(&ta, a.a_codes, kb, (uint64_t)a.M, kb, ROW, BM, 128))
         return cudaErrorInvalidValue;
-    if (!encode_tmap_2d_u8(&tb, a.b_codes, kb, (uint64_t)a.N, kb, row, BN, swz))
+    if (!encode_tmap_2d_u8(&tb, a.b_codes, kb, (uint64_t)a.N, kb, ROW, BN, 128))
         return cudaErrorInvalidValue;
     if (a.r_codes) {
-        if (!encode_tmap_2d_u8(&tr, a.r_codes, kb, (uint64_t)a.M, kb, row, BM, swz))
+        if (!encode_tmap_2d_u8(&tr, a.r_codes, kb, (uint64_t)a.M, kb, ROW, BM, 128))
             return cudaErrorInvalidValue;
     } else {
         tr = ta;
@@ -449,7 +454,7 @@ cudaError_t launch_kc(const GemmMxf4Args &a, cudaStream_t st)
     if (!encode_tmap_2d_u8(&ty, a.y, yrow, (uint64_t)a.M, yrow, 64, 32, 64))
         return cudaErrorInvalidValue;
     const bool res = a.r_codes != nullptr, phi = res && a.phi != nullptr;
-#define RFQ_GV(R, P, O) return launch_variant<KC, R, P, O>(ta, tr, tb, ty, a, st)
+#define RFQ_GV(R, P, O) return launch_variant<R, P, O>(ta, tr, tb, ty, a, st)
     if (!res) {
         if (a.out_bf16) RFQ_GV(false, false, true);
         RFQ_GV(false, false, false);
@@ -461,17 +466,6 @@ cudaError_t launch_kc(const GemmMxf4Args &a, cudaStream_t st)
     if (a.out_bf16) RFQ_GV(true, false, true);
     RFQ_GV(true, false, false);
 #undef RFQ_GV
-}
-
-} // namespace
-
-cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st)
-{
-#ifdef RFQ_GEMM_KC
-    return launch_kc<RFQ_GEMM_KC>(a, st);
-#else
-    return launch_kc<2>(a, st);
-#endif
 }
 
 } // namespace rfq
