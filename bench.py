@@ -136,6 +136,24 @@ def _dist():
     return ws, rank, local
 
 
+def _max_over_ranks(value: float, ws: int, dist, device) -> float:
+    """The largest `value` over all ranks (the job's time is its slowest
+    rank's); `dist` is torch.distributed with an initialised group."""
+    if ws == 1:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def _job_rate(units_per_rank: float, ws: int, ms: float) -> float:
+    """Whole-job throughput in units per second: every rank processes its own
+    copy of the workload (weak scaling), the job takes the slowest rank's
+    time."""
+    return ws * units_per_rank / (ms * 1e-3)
+
+
 def _workload(rows: int = 0, name: str = WORKLOAD):
     """The benchmark workload; rows > 0 keeps only the first `rows` token
     rows (a smaller case of the same kernels, for profiler captures)."""
@@ -171,52 +189,73 @@ def _config(spec, extra=None):
     return c
 
 
-def cpu_oracle_sample(rows_per_call: int = 8, calls: int = 2):
-    """Times the CPU oracle (single thread, fp64) on a bounded sample of the
-    workload: `calls` x (quantize + RFQ GEMM of `rows_per_call` token rows
-    against the full quantized weight).  Returns (TFLOP/s, seconds, sample)."""
+_ORACLE_W = {}
+
+
+def _oracle_weight(spec):
+    """The oracle's quantized weight of a workload (computed once per process:
+    weight quantization is an offline step, not part of the timed sample)."""
     import oracle
-    from paper_2608_26581_gb300.synth import ActSpec, make_activation, make_weight
-    spec = _workload()
-    K, N = spec.act.K, spec.N
-    a = spec.act
-    xb = make_activation(ActSpec(rows_per_call * calls, K, a.body, a.body_scale, a.chan_frac, a.chan_count,
+    from paper_2608_26581_gb300.synth import make_weight
+    if spec.name not in _ORACLE_W:
+        fmt = oracle.FMT_HIF4 if spec.fmt == "hif4" else oracle.FMT_MXFP4
+        _ORACLE_W[spec.name] = oracle.quantize_weight(make_weight(spec.act.K, spec.N, seed=spec.act.seed), fmt)
+    return _ORACLE_W[spec.name]
+
+
+def cpu_oracle_sample(spec, rows_per_call: int = 8, calls: int = 4):
+    """Times the CPU oracle (single thread, fp64) on a bounded sample of the
+    workload `spec`: `calls` x (quantize + RFQ GEMM of `rows_per_call` token
+    rows against the full quantized weight), or quantization alone for the
+    quantizer-only workload.  Returns (value, unit, seconds, sample) in the
+    bench's own metric: TFLOP/s of the main + residual product, or GB/s of
+    the quantizer's algorithmic bytes."""
+    import oracle
+    from paper_2608_26581_gb300.synth import ActSpec, make_activation
+    K, N, a = spec.act.K, spec.N, spec.act
+    fmt = oracle.FMT_HIF4 if spec.fmt == "hif4" else oracle.FMT_MXFP4
+    rows = rows_per_call * calls
+    xb = make_activation(ActSpec(rows, K, a.body, a.body_scale, a.chan_frac, a.chan_count,
                                  a.chan_scale, 0.0, None, 1.0, a.seed))
-    wb = make_weight(K, N, seed=a.seed)
-    wc, ws = oracle.quantize_weight(wb)
+    wq = _oracle_weight(spec) if N else None
     t0 = time.perf_counter()
     for i in range(calls):
         x = xb[i * rows_per_call:(i + 1) * rows_per_call]
-        q = oracle.quantize_act(x)
-        oracle.linear(0, q["main_codes"], q["main_scales"], q["res_codes"], q["res_scales"], wc, ws,
-                      rows_per_call, K, N)
+        q = oracle.quantize_act(x, fmt)
+        if N:
+            oracle.linear(fmt, q["main_codes"], q["main_scales"], q["res_codes"], q["res_scales"], wq[0], wq[1],
+                          rows_per_call, K, N)
     dt = time.perf_counter() - t0
-    flop = 2.0 * 2.0 * rows_per_call * calls * N * K
-    sample = (f"{calls} x (quantize_act + RFQ linear) of {rows_per_call} rows of X [.., {K}] "
-              f"against the full W~ [{N} x {K}] (weight quantization untimed)")
-    return flop / dt / 1e12, dt, sample
+    if N:
+        sample = (f"{calls} x (quantize_act + RFQ linear) of {rows_per_call} rows of X [.., {K}] "
+                  f"against the full W~ [{N} x {K}] (weight quantization untimed)")
+        return 2.0 * 2.0 * rows * N * K / dt / 1e12, UNIT, dt, sample
+    per_elem = 3.125 if fmt == oracle.FMT_HIF4 else 3.0625
+    sample = f"{calls} x quantize_act (main + residual) of {rows_per_call} rows of X [.., {K}]"
+    return rows * K * per_elem / dt / 1e9, "GB/s", dt, sample
 
 
 def run_reference(args):
     ws, rank, _ = _dist()
     if rank != 0:
         return
-    spec = _workload()
+    spec = _workload(0, args.workload)
+    rows = 2 if spec.N else 64
     for _ in range(args.warmup):
-        cpu_oracle_sample(rows_per_call=2, calls=1)
+        cpu_oracle_sample(spec, rows_per_call=rows, calls=1)
     vals, times = [], []
-    sample = ""
+    sample, unit = "", UNIT
     for _ in range(args.steps):
-        v, dt, sample = cpu_oracle_sample(rows_per_call=2, calls=1)
+        v, unit, dt, sample = cpu_oracle_sample(spec, rows_per_call=rows, calls=1)
         vals.append(v)
         times.append(dt)
     value = statistics.median(vals)
-    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": unit, "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * statistics.median(times),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "config": _config(spec, {"sample": sample}),
-            "cpu_baseline": {"kind": "oracle", "cores": 1, "sample": sample, "value": value, "unit": UNIT},
-            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "cpu_baseline": {"kind": "oracle", "cores": 1, "sample": sample, "value": value, "unit": unit},
+            "e2e": {"value": value, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
             "gpu_launches": 0}
     print(json.dumps(line), flush=True)
 
@@ -315,10 +354,7 @@ def run_rfq(args):
     q_ms = statistics.mean(a.elapsed_time(b) for a, b, _, _ in per_step)
     x_ms = statistics.mean(b.elapsed_time(c) for _, b, c, _ in per_step)   # HiF4 expansions (0 otherwise)
     g_ms = statistics.mean(c.elapsed_time(d) for _, _, c, d in per_step)
-    if ws > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = _max_over_ranks(ms, ws, dist, dev)
 
     # end to end through the public API with host buffers
     e2e_ms = None
@@ -340,10 +376,8 @@ def run_rfq(args):
         torch.cuda.synchronize()
         barrier()
         e2e_ms = e0.elapsed_time(e1) / args.steps
-    if ws > 1 and e2e_ms is not None:
-        t = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    if e2e_ms is not None:
+        e2e_ms = _max_over_ranks(e2e_ms, ws, dist, dev)
     if rfq.rfq_workspace_status(wsp) != rfq.RFQ_OK:
         raise RuntimeError("rfq_linear reported a device timeout")
 
@@ -372,11 +406,11 @@ def run_rfq(args):
                  "frac": aq_gbs / pk["hbm"], "bytes_per_launch": aq_bytes, "ms_per_launch": q_ms,
                  "traffic": _kernel_traffic(aq_kernel, spec.name)}
     if quant_only:
-        value = ws * aq_bytes / (ms * 1e-3) / 1e9
+        value = _job_rate(aq_bytes, ws, ms) / 1e9
         unit = "GB/s"
         roofline = dict(act_quant)
     else:
-        value = ws * flop / (ms * 1e-3) / 1e12
+        value = _job_rate(flop, ws, ms) / 1e12
         unit = UNIT
         gemm_tflops = flop / (g_ms * 1e-3) / 1e12
         roofline = {"bound": "tensor", "kernel": t_kernel, "achieved": gemm_tflops, "peak": t_peak,
@@ -385,7 +419,7 @@ def run_rfq(args):
                     "peak_source": t_src, "frac_of_sustained_peak": gemm_tflops / t_peak_sust}
     clocks = clk.summary()
     if e2e_ms is not None:
-        e2e = {"value": ws * (aq_bytes / 1e9 if quant_only else flop / 1e12) / (e2e_ms * 1e-3), "unit": unit,
+        e2e = {"value": _job_rate(aq_bytes / 1e9 if quant_only else flop / 1e12, ws, e2e_ms), "unit": unit,
                "ms_per_step": e2e_ms, "h2d_bytes_per_step": M * K * 2,
                "d2h_bytes_per_step": q_bytes if quant_only else M * N * 2}
     else:
@@ -393,9 +427,9 @@ def run_rfq(args):
 
     if rank == 0:
         cpu = None
-        if ws == 1 and not args.no_cpu_baseline and args.workload == WORKLOAD:
-            v, dt, sample = cpu_oracle_sample()
-            cpu = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample,
+        if ws == 1 and not args.no_cpu_baseline and not args.rows:
+            v, u, dt, sample = cpu_oracle_sample(spec)
+            cpu = {"value": v, "unit": u, "cores": 1, "kind": "oracle", "sample": sample,
                    "seconds": round(dt, 2)}
         line = {
             "metric": METRIC, "value": value, "unit": unit, "n_gpus": ws, "steps": args.steps,
@@ -413,7 +447,7 @@ def run_rfq(args):
             "cpu_baseline": cpu,
         }
         if not quant_only:
-            line["effective_tflops_2mnk"] = ws * flop / 2 / (ms * 1e-3) / 1e12
+            line["effective_tflops_2mnk"] = _job_rate(flop / 2, ws, ms) / 1e12
         print(json.dumps(line), flush=True)
     if ws > 1:
         dist.destroy_process_group()
