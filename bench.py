@@ -50,7 +50,8 @@ def _peaks():
 
 # source file of each timed kernel: its DRAM counters hold only for the
 # sources they were taken on (the kernel's file plus the shared headers)
-_KERNEL_SRC = {"gemm_mxf4_kernel": "gemm_mxf4.cu", "act_quant_mxfp4_kernel": "quant_mxfp4.cu",
+_KERNEL_SRC = {"gemm_mxf4_kernel": "gemm_mxf4.cu", "gemm_mxf4_pair_kernel": "gemm_mxf4_pair.cu",
+               "act_quant_mxfp4_kernel": "quant_mxfp4.cu",
                "gemm_hif4_kernel": "gemm_hif4.cu", "act_quant_hif4_kernel": "quant_hif4.cu"}
 
 
@@ -394,7 +395,8 @@ def run_rfq(args):
         t_peak, t_peak_sust = pk["bf16_burst"] * FP4_OVER_BF16, pk["bf16_sust"] * FP4_OVER_BF16
         t_src = (f"{pk['src']} bf16 burst {pk['bf16_burst']} TFLOP/s x {FP4_OVER_BF16:g} "
                  f"(nominal dense FP4/BF16 ratio), of {pk['src']}")
-        t_kernel = "gemm_mxf4_kernel"
+        # more than one 128-row tile runs on CTA pairs (see launch_gemm_mxf4)
+        t_kernel = "gemm_mxf4_pair_kernel" if M > 128 else "gemm_mxf4_kernel"
     if hif4:
         aq_bytes = M * K * 2 + 2 * (M * K // 2) + 2 * (((M + 127) // 128) * 128 * (K // 64) * 4)
         aq_kernel = "act_quant_hif4_kernel"

@@ -1,0 +1,525 @@
+// gemm_mxf4_pair.cu -- RFQ GEMM on CTA pairs (Algorithm 1, Eq. rfq):
+//   Y = X~ W~ + phi X^ W~
+// with tcgen05 cta_group::2 MMAs: the two CTAs of a cluster compute one
+// 256 x 256 output tile.  Each CTA stages its own 128 rows of X~ and X^ and
+// HALF of the tile's 256 W~ rows; one thread of the even CTA issues M = 256
+// MMAs that read the A rows and W~ halves of both CTAs.  Per 256-element
+// k-stage an SM streams 52 KB (codes and scale atoms) for 1,024 cycles of MMA
+// work, 24% less than the 68 KB of a single-CTA 128 x 256 tile.
+//
+// Per CTA (448 threads, one CTA per SM):
+//   warp 0      TMA producer.  The codes (own A and R rows, own W~ half) are
+//               CTA-pair copies that complete on the EVEN CTA's stage
+//               barrier, which the even CTA's producer arms with the bytes of
+//               both CTAs; the scale atoms (own A / R rows, both 128-row W~
+//               atoms of the tile) are bulk copies into this CTA's shared
+//               memory, on its own barrier.
+//   warp 1      even CTA: MMA issuer (main + residual MMA per K=64 step,
+//               same W~ descriptor, same accumulator: Sec. 4.3)
+//   warps 2-9   epilogue: TMEM -> registers -> bf16 / fp32 -> shared-memory
+//               staging -> TMA stores of this CTA's 128 rows
+//   warps 10-13 scale writers: this CTA's scale words from shared memory into
+//               its TMEM with tcgen05.st, one warp per TMEM lane quarter
+// TMEM (512 columns per CTA): a 256-column accumulator (this CTA's 128 rows
+// of the tile) and four 32-column scale slots; each CTA holds the scales of
+// its own A / R rows and of ALL 256 W~ rows of the tile (the layout the pair
+// MMA reads).  A slot is rewritten four stages after its last use, after the
+// stage's copies, which the producer issued once the MMAs of that earlier
+// stage had completed.
+//
+// Cross-CTA signals (the odd CTA's scale writers and epilogue warps telling
+// the even CTA's MMA thread that a scale slot is filled or the accumulator
+// drained) are relaxed arrives on the even CTA's barriers, issued after the
+// signalling warp's own tcgen05 stores / loads have completed (wait::st /
+// wait::ld); the MMA thread observes them with cluster-scope acquire waits
+// and orders its MMAs after them with tcgen05.fence.  A release arrive at
+// cluster scope would stall the arriving warp for hundreds of cycles.
+//
+// Residual MMAs of 128-element k-chunks whose phi is 0 for both row tiles of
+// the pair are skipped (the stored residual of a phi = 0 tile is zero, so a
+// pair whose other tile has phi = 1 adds exact zeros).
+//
+// Every mbarrier wait is bounded (kWaitLimitNs) and also gives up when any
+// CTA has recorded a timeout in the caller's status word.  Neither CTA of a
+// pair leaves before the final cluster barrier, so the peer never signals a
+// CTA that has exited; the even CTA drains its MMAs before that barrier.
+#include <cuda_bf16.h>
+#include <cstdint>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace rfq {
+namespace {
+
+constexpr int BM = 128;                  // rows per CTA (256 per pair)
+constexpr int BN = 256;                  // output columns per pair tile
+constexpr int BN_HALF = BN / 2;          // W~ rows staged per CTA
+constexpr int ROW = 128;                 // bytes of codes per row per stage (256 elements)
+constexpr int STAGES = 4;
+constexpr int A_BYTES = BM * ROW;
+constexpr int B_BYTES = BN_HALF * ROW;
+constexpr int ATOM = 512;                // scale bytes of 128 rows x one 128-element chunk
+constexpr int TMEM_COLS = 512;
+constexpr int SF_COL0 = BN;              // scale slots after the accumulator
+constexpr int SF_SLOT_COLS = 32;         // A chunk c at 4c, R at 8 + 4c, W~ at 16 + 8c (+4: rows 128-255)
+constexpr int SF_SLOTS = 4;
+constexpr int EPI_WARPS = 8;
+constexpr int SF_WARPS = 4;
+constexpr int THREADS = 64 + 32 * (EPI_WARPS + SF_WARPS);
+constexpr int YSTAGE = 2048;             // per epilogue warp: 32 rows x 64 bytes of Y
+static_assert(SF_COL0 + SF_SLOTS * SF_SLOT_COLS <= TMEM_COLS, "TMEM budget");
+static_assert(SF_SLOTS >= STAGES, "a scale slot is rewritten only after its stage's MMAs completed");
+
+struct alignas(1024) Stage {
+    uint8_t a[A_BYTES];
+    uint8_t r[A_BYTES];
+    uint8_t b[B_BYTES];
+    uint8_t sfa[2 * ATOM];               // chunk c at c * ATOM
+    uint8_t sfr[2 * ATOM];
+    uint8_t sfb[4 * ATOM];               // W~ rows 128 h..128 h + 127 of the tile: chunk c at (2 h + c) * ATOM
+};
+static_assert(sizeof(Stage) % 1024 == 0, "stages keep the 1024-byte swizzle alignment");
+
+struct Smem {
+    Stage st[STAGES];
+    alignas(1024) uint8_t ystage[EPI_WARPS * YSTAGE];
+    uint64_t full[STAGES];        // (even CTA) both CTAs' code copies landed
+    uint64_t sf_full[STAGES];     // this CTA's scale atoms landed
+    uint64_t empty[STAGES];       // the stage's MMAs completed (both CTAs)
+    uint64_t sf_ready[SF_SLOTS];  // (even CTA) both CTAs' scale writers filled the slot
+    uint64_t acc_full;            // accumulator complete (both CTAs)
+    uint64_t acc_empty;           // (even CTA) both CTAs' epilogue warps drained it
+    uint64_t drain;
+    uint32_t tmem_base;
+    int32_t abort_flag;
+};
+constexpr size_t kSmemBytes = sizeof(Smem) + 1024;
+static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+
+__device__ __forceinline__ void flag_timeout(Smem &S, int32_t *status)
+{
+    S.abort_flag = 1;
+    atomicExch(status, kDevTimeout);
+}
+
+// Does the residual term of 128-element chunk `chunk` apply to either row
+// tile of the pair?
+template <bool PHI>
+__device__ __forceinline__ bool res_chunk(const uint8_t *phi, int m_pair, int m_tiles, int phi_cols, int phi_chunks,
+                                          int chunk)
+{
+    if (!PHI)
+        return true;
+    bool on = false;
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+        const int mt = 2 * m_pair + r;
+        if (mt < m_tiles)
+            on |= __ldg(phi + (int64_t)mt * phi_cols + chunk / phi_chunks) != 0;
+    }
+    return on;
+}
+
+template <bool RES, bool PHI, bool OUT_BF16>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
+    gemm_mxf4_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmR,
+                          const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmY,
+                          const uint8_t *__restrict__ sfa, const uint8_t *__restrict__ sfr,
+                          const uint8_t *__restrict__ sfb, const uint8_t *__restrict__ phi, int phi_chunks,
+                          int phi_cols, int M, int N, int K, int32_t *status)
+{
+    extern __shared__ uint8_t smem_raw[];
+    Smem &S = *reinterpret_cast<Smem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();
+    const bool lead = rank == 0;
+    const volatile int32_t *gstat = status;
+
+    const int kc = K >> 7;                  // 128-element chunks
+    const int nks = (kc + 1) >> 1;          // 256-element stages (the last may hold one chunk)
+    const int n_tiles = (N + BN - 1) / BN;
+    const int m_tiles = (M + BM - 1) / BM;  // 128-row tiles: scale atoms and phi rows
+    const int m_pairs = (M + 2 * BM - 1) / (2 * BM);
+    const int tiles = n_tiles * m_pairs;
+    const int n_atoms = (N + 127) >> 7;     // 128-row scale atoms of W~
+    const int pair = blockIdx.x >> 1, pairs = gridDim.x >> 1;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(&S.full[s], 1);
+            mbar_init(&S.sf_full[s], 1);
+            mbar_init(&S.empty[s], 1);
+        }
+        for (int i = 0; i < SF_SLOTS; ++i)
+            mbar_init(&S.sf_ready[i], 2 * SF_WARPS);
+        mbar_init(&S.acc_full, 1);
+        mbar_init(&S.acc_empty, 2 * EPI_WARPS);
+        mbar_init(&S.drain, 1);
+        // A bounded wait of an earlier CTA or call gave up: skip the work
+        // (both CTAs still meet at the cluster barriers).
+        S.abort_flag = *gstat;
+        fence_mbar_init();
+    }
+    if (warp == 0 && lane == 0) {
+        prefetch_tmap(&tmA);
+        if (RES)
+            prefetch_tmap(&tmR);
+        prefetch_tmap(&tmB);
+        prefetch_tmap(&tmY);
+    }
+    if (warp == 1) {
+        tmem_alloc_pair(&S.tmem_base, TMEM_COLS);
+        tmem_relinquish_pair();
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync(); // both CTAs' barriers initialised and TMEM allocated
+    tc_fence_after();
+    const uint32_t tmem = S.tmem_base;
+    const bool skip = S.abort_flag != 0;
+
+    if (warp == 0) {
+        // ------------------------------------------------ TMA producer (both CTAs)
+        if (lane == 0 && !skip) {
+            const uint32_t full0 = mapa_shared(smem_u32(&S.full[0]), 0);   // the even CTA's barriers
+            int p = 0;
+            bool stop = false;
+            for (int tile = pair; tile < tiles && !stop; tile += pairs) {
+                const int m_pair = tile / n_tiles, n_tile = tile - m_pair * n_tiles;
+                const int m_tile = 2 * m_pair + (int)rank;
+                const bool rows_in = m_tile < m_tiles;
+                const int atom0 = 2 * n_tile;
+                const int nb = atom0 + 1 < n_atoms ? 2 : 1;
+                for (int ks = 0; ks < nks; ++ks, ++p) {
+                    const int slot = p % STAGES;
+                    if (!mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, kWaitLimitNs, gstat)) {
+                        flag_timeout(S, status);
+                        stop = true;
+                        break;
+                    }
+                    const int c0 = 2 * ks, nch = min(2, kc - c0);
+                    bool res_on = false;
+                    if (RES)
+                        for (int c = 0; c < nch; ++c)
+                            res_on |= res_chunk<PHI>(phi, m_pair, m_tiles, phi_cols, phi_chunks, c0 + c);
+                    Stage &st = S.st[slot];
+                    // codes: both CTAs' copies complete on the even CTA's barrier
+                    if (lead)
+                        mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES + B_BYTES + (res_on ? A_BYTES : 0)));
+                    const uint32_t bar = full0 + 8 * slot;
+                    tma_load_2d_pair(st.a, &tmA, bar, c0 * 64, m_tile * BM);
+                    if (res_on)
+                        tma_load_2d_pair(st.r, &tmR, bar, c0 * 64, m_tile * BM);
+                    tma_load_2d_pair(st.b, &tmB, bar, c0 * 64, n_tile * BN + (int)rank * BN_HALF);
+                    // scale atoms: this CTA's own barrier
+                    const uint32_t sfbytes = (uint32_t)nch * ATOM;
+                    uint64_t *sbar = &S.sf_full[slot];
+                    mbar_arrive_expect_tx(sbar, nb * sfbytes + (rows_in ? (res_on ? 2 : 1) * sfbytes : 0));
+                    if (rows_in) {
+                        bulk_load(st.sfa, sfa + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, sbar);
+                        if (res_on)
+                            bulk_load(st.sfr, sfr + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, sbar);
+                    }
+                    for (int h = 0; h < nb; ++h)
+                        bulk_load(st.sfb + h * 2 * ATOM, sfb + ((int64_t)(atom0 + h) * kc + c0) * ATOM, sfbytes,
+                                  sbar);
+                }
+            }
+            if (stop || S.abort_flag)
+                // wait (bounded) until the copies of the last stages landed: this
+                // CTA's scale atoms, and (even CTA) both CTAs' codes
+                for (int q = max(0, p - STAGES); q < p; ++q) {
+                    (void)mbar_wait(&S.sf_full[q % STAGES], (q / STAGES) & 1, kWaitLimitNs);
+                    if (lead)
+                        (void)mbar_wait(&S.full[q % STAGES], (q / STAGES) & 1, kWaitLimitNs);
+                }
+        }
+    } else if (warp == 1) {
+        if (lane == 0 && !skip && lead) {
+            // -------------------------------------------- MMA issuer (even CTA)
+            int p = 0, it = 0;
+            bool stop = false;
+            for (int tile = pair; tile < tiles && !stop; tile += pairs, ++it) {
+                const int m_pair = tile / n_tiles;
+                if (!mbar_wait<true>(&S.acc_empty, (it & 1) ^ 1, kWaitLimitNs, gstat)) {
+                    flag_timeout(S, status);
+                    break;
+                }
+                tc_fence_after();
+                for (int ks = 0; ks < nks; ++ks, ++p) {
+                    const int slot = p % STAGES, sfs = p % SF_SLOTS;
+                    if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat) ||
+                        !mbar_wait<true>(&S.sf_ready[sfs], (p / SF_SLOTS) & 1, kWaitLimitNs, gstat)) {
+                        flag_timeout(S, status);
+                        stop = true;
+                        break;
+                    }
+                    tc_fence_after();
+                    const int c0 = 2 * ks, nch = min(2, kc - c0);
+                    const uint32_t sf = tmem + SF_COL0 + SF_SLOT_COLS * sfs;
+                    const Stage &st = S.st[slot];
+                    const uint32_t a0 = smem_u32(st.a), r0 = smem_u32(st.r), b0 = smem_u32(st.b);
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const int c = j >> 1;
+                        if (c >= nch)
+                            break;
+                        const uint32_t id = idesc_mxf4(2 * BM, BN, 2 * (j & 1), 2 * (j & 1));
+                        const uint64_t bd = sdesc_k_sw128(b0 + 32 * j);
+                        const uint32_t sfb_t = sf + 16 + 8 * c;
+                        tc_mma_mxf4_pair(tmem, sdesc_k_sw128(a0 + 32 * j), bd, id, sf + 4 * c, sfb_t, (ks | j) != 0);
+                        if (RES && res_chunk<PHI>(phi, m_pair, m_tiles, phi_cols, phi_chunks, c0 + c))
+                            tc_mma_mxf4_pair(tmem, sdesc_k_sw128(r0 + 32 * j), bd, id, sf + 8 + 4 * c, sfb_t, 1);
+                    }
+                    tc_commit_pair_mc(&S.empty[slot], 0x3);
+                }
+                if (!stop)
+                    tc_commit_pair_mc(&S.acc_full, 0x3);
+            }
+            // every MMA (and its commits to both CTAs) completes before the
+            // final cluster barrier
+            tc_commit_pair_mc(&S.drain, 0x1);
+            (void)mbar_wait(&S.drain, 0, kWaitLimitNs);
+        }
+    } else if (warp < 2 + EPI_WARPS) {
+        // ------------------------------------------------ epilogue (warps 2..9)
+        const int q = warp & 3;          // TMEM lane quarter this warp may access
+        const int h = (warp - 2) >> 2;   // column half of the tile
+        const uint32_t acc_empty_lead = mapa_shared(smem_u32(&S.acc_empty), 0);
+        uint8_t *stg = S.ystage + (warp - 2) * YSTAGE;
+        const uint32_t sw = (uint32_t)((lane >> 1) & 3);   // 64B swizzle: chunk j of row r at (j ^ ((r >> 1) & 3))
+        int it = 0;
+        for (int tile = pair; tile < tiles && !skip; tile += pairs, ++it) {
+            const int m_pair = tile / n_tiles, n_tile = tile - m_pair * n_tiles;
+            // warp-uniform outcome: the tcgen05 loads below need the whole warp
+            if (!__all_sync(0xffffffffu, mbar_wait(&S.acc_full, it & 1, kWaitLimitNs, gstat))) {
+                if (lane == 0)
+                    flag_timeout(S, status);
+                break;
+            }
+            tc_fence_after();
+            const int row0 = (2 * m_pair + (int)rank) * BM + q * 32;
+            const uint32_t tcol = tmem + ((uint32_t)(q * 32) << 16) + h * (BN / 2);
+            auto release = [&]() {
+                // the accumulator goes back to the MMA thread
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) {
+                    if (lead)
+                        mbar_arrive(&S.acc_empty);
+                    else
+                        mbar_arrive_remote_relaxed(acc_empty_lead);
+                }
+            };
+            if (OUT_BF16) {
+                // all 128 columns of this warp into registers as packed bf16
+                uint32_t pk[64];
+#pragma unroll
+                for (int g = 0; g < 2; ++g) {
+                    uint32_t v[2][32];
+                    tmem_ld_32x32b_x32(tcol + 64 * g, v[0]);
+                    tmem_ld_32x32b_x32(tcol + 64 * g + 32, v[1]);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int c = 0; c < 2; ++c)
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            __nv_bfloat162 b2 = __floats2bfloat162_rn(__uint_as_float(v[c][2 * i]),
+                                                                      __uint_as_float(v[c][2 * i + 1]));
+                            pk[32 * g + 16 * c + i] = *reinterpret_cast<uint32_t *>(&b2);
+                        }
+                }
+                release();
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {   // 32-column chunks: one 64-byte TMA box row per lane
+                    const int col = n_tile * BN + h * (BN / 2) + 32 * c;
+                    if (col >= N || row0 >= M)
+                        break;
+                    if (lane == 0)
+                        bulk_wait_group_read<0>();
+                    __syncwarp();
+#pragma unroll
+                    for (int j = 0; j < 4; ++j)
+                        *reinterpret_cast<uint4 *>(stg + lane * 64 + ((j ^ sw) << 4)) =
+                            make_uint4(pk[16 * c + 4 * j], pk[16 * c + 4 * j + 1], pk[16 * c + 4 * j + 2],
+                                       pk[16 * c + 4 * j + 3]);
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tma_store_2d(&tmY, stg, col * 2, row0);
+                        bulk_commit_group();
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int half = 0; half < 2; ++half) {
+                    uint32_t v[2][32];
+#pragma unroll
+                    for (int c = 0; c < 2; ++c)
+                        tmem_ld_32x32b_x32(tcol + (2 * half + c) * 32, v[c]);
+                    tmem_ld_wait();
+                    if (half == 1)
+                        release();
+#pragma unroll
+                    for (int c = 0; c < 2; ++c) {
+                        const int col = n_tile * BN + h * (BN / 2) + (2 * half + c) * 32;
+                        if (col >= N || row0 >= M)
+                            continue;
+#pragma unroll
+                        for (int hb = 0; hb < 2; ++hb) { // 16 fp32 columns (64 bytes) per store
+                            if (col + 16 * hb >= N)
+                                break;
+                            if (lane == 0)
+                                bulk_wait_group_read<0>();
+                            __syncwarp();
+#pragma unroll
+                            for (int j = 0; j < 4; ++j)
+                                *reinterpret_cast<uint4 *>(stg + lane * 64 + ((j ^ sw) << 4)) =
+                                    make_uint4(v[c][16 * hb + 4 * j], v[c][16 * hb + 4 * j + 1],
+                                               v[c][16 * hb + 4 * j + 2], v[c][16 * hb + 4 * j + 3]);
+                            fence_proxy_async_smem();
+                            __syncwarp();
+                            if (lane == 0) {
+                                tma_store_2d(&tmY, stg, (col + 16 * hb) * 4, row0);
+                                bulk_commit_group();
+                            }
+                        }
+                    }
+                }
+            }
+            if (S.abort_flag)
+                break;
+        }
+        if (lane == 0)
+            bulk_wait_group<0>(); // every TMA store of this warp has completed
+    } else {
+        // ------------------------------------------------ scale writers (warps 10..13)
+        // Warp quarter q writes TMEM lanes 32q..32q+31; every quarter holds
+        // the same words: column j of lane i carries the four scales of row
+        // 32 j + i (of this CTA's 128 A rows; of the tile's W~ rows).
+        const int q = warp & 3;
+        const uint32_t sf_ready_lead = mapa_shared(smem_u32(&S.sf_ready[0]), 0);
+        int p = 0;
+        bool stop = false;
+        for (int tile = pair; tile < tiles && !stop && !skip; tile += pairs) {
+            const int m_pair = tile / n_tiles, n_tile = tile - m_pair * n_tiles;
+            const bool rows_in = 2 * m_pair + (int)rank < m_tiles;
+            const bool b1_in = 2 * n_tile + 1 < n_atoms;
+            for (int ks = 0; ks < nks; ++ks, ++p) {
+                const int slot = p % STAGES, sfs = p % SF_SLOTS;
+                // warp-uniform outcome: the tcgen05 stores below need the whole warp
+                if (!__all_sync(0xffffffffu, mbar_wait(&S.sf_full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat))) {
+                    if (lane == 0)
+                        flag_timeout(S, status);
+                    stop = true;
+                    break;
+                }
+                tc_fence_after();
+                const int c0 = 2 * ks, nch = min(2, kc - c0);
+                const Stage &st = S.st[slot];
+                const uint32_t tb = tmem + ((uint32_t)(q * 32) << 16) + SF_COL0 + SF_SLOT_COLS * sfs;
+                const uint4 z = make_uint4(0, 0, 0, 0);
+#pragma unroll
+                for (int c = 0; c < 2; ++c) {
+                    if (c >= nch)
+                        break;
+                    const uint4 va = rows_in ? *reinterpret_cast<const uint4 *>(st.sfa + c * ATOM + lane * 16) : z;
+                    const uint4 vb0 = *reinterpret_cast<const uint4 *>(st.sfb + c * ATOM + lane * 16);
+                    const uint4 vb1 = b1_in ? *reinterpret_cast<const uint4 *>(st.sfb + (2 + c) * ATOM + lane * 16) : z;
+                    tmem_st_32x32b_x4(tb + 4 * c, va.x, va.y, va.z, va.w);
+                    if (RES && res_chunk<PHI>(phi, m_pair, m_tiles, phi_cols, phi_chunks, c0 + c)) {
+                        const uint4 vr = rows_in ? *reinterpret_cast<const uint4 *>(st.sfr + c * ATOM + lane * 16) : z;
+                        tmem_st_32x32b_x4(tb + 8 + 4 * c, vr.x, vr.y, vr.z, vr.w);
+                    }
+                    tmem_st_32x32b_x4(tb + 16 + 8 * c, vb0.x, vb0.y, vb0.z, vb0.w);
+                    tmem_st_32x32b_x4(tb + 20 + 8 * c, vb1.x, vb1.y, vb1.z, vb1.w);
+                }
+                tmem_st_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) {
+                    if (lead)
+                        mbar_arrive(&S.sf_ready[sfs]);
+                    else
+                        mbar_arrive_remote_relaxed(sf_ready_lead + 8 * sfs);
+                }
+            }
+        }
+    }
+
+    // ---------------------------------------------------- teardown
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync(); // the peer no longer signals this CTA, the pair's MMAs are complete
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc_pair(tmem, TMEM_COLS);
+    }
+}
+
+template <bool RES, bool PHI, bool OUT>
+cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const CUtensorMap &tb,
+                           const CUtensorMap &ty, const GemmMxf4Args &a, cudaStream_t st)
+{
+    auto kern = gemm_mxf4_pair_kernel<RES, PHI, OUT>;
+    static int max_pairs = 0; // per variant: clusters of two that fit on the device at once
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+    if (e != cudaSuccess)
+        return e;
+    if (max_pairs == 0) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(2 * (num_sms() / 2));
+        cfg.blockDim = dim3(THREADS);
+        cfg.dynamicSmemBytes = kSmemBytes;
+        int n = 0;
+        e = cudaOccupancyMaxActiveClusters(&n, kern, &cfg);
+        if (e != cudaSuccess)
+            return e;
+        max_pairs = n > 0 ? n : 1;
+    }
+    const int64_t tiles = ((a.N + BN - 1) / BN) * ((a.M + 2 * BM - 1) / (2 * BM));
+    const int grid = 2 * (int)(tiles < max_pairs ? tiles : max_pairs);
+    const int phi_chunks = a.phi_r_s / 128;
+    const int phi_cols = a.phi ? (int)((a.K + a.phi_r_s - 1) / a.phi_r_s) : 0;
+    kern<<<grid, THREADS, kSmemBytes, st>>>(ta, tr, tb, ty, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf,
+                                            (const uint8_t *)a.b_sf, a.phi, phi_chunks, phi_cols, (int)a.M,
+                                            (int)a.N, (int)a.K, a.status);
+    return cudaGetLastError();
+}
+
+} // namespace
+
+cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
+{
+    CUtensorMap ta, tr, tb, ty;
+    const uint64_t kb = (uint64_t)a.K / 2;
+    if (!encode_tmap_2d_u8(&ta, a.a_codes, kb, (uint64_t)a.M, kb, ROW, BM, 128) ||
+        !encode_tmap_2d_u8(&tb, a.b_codes, kb, (uint64_t)a.N, kb, ROW, BN_HALF, 128))
+        return cudaErrorInvalidValue;
+    if (a.r_codes) {
+        if (!encode_tmap_2d_u8(&tr, a.r_codes, kb, (uint64_t)a.M, kb, ROW, BM, 128))
+            return cudaErrorInvalidValue;
+    } else {
+        tr = ta;
+    }
+    // Y [M][N] (bf16 or fp32) as bytes; boxes of 64 bytes x 32 rows, 64B swizzle
+    const uint64_t yrow = (uint64_t)a.N * (a.out_bf16 ? 2 : 4);
+    if (!encode_tmap_2d_u8(&ty, a.y, yrow, (uint64_t)a.M, yrow, 64, 32, 64))
+        return cudaErrorInvalidValue;
+    const bool res = a.r_codes != nullptr, phi = res && a.phi != nullptr;
+#define RFQ_GV(R, P, O) return launch_variant<R, P, O>(ta, tr, tb, ty, a, st)
+    if (!res) {
+        if (a.out_bf16) RFQ_GV(false, false, true);
+        RFQ_GV(false, false, false);
+    }
+    if (phi) {
+        if (a.out_bf16) RFQ_GV(true, true, true);
+        RFQ_GV(true, true, false);
+    }
+    if (a.out_bf16) RFQ_GV(true, false, true);
+    RFQ_GV(true, false, false);
+#undef RFQ_GV
+}
+
+} // namespace rfq

@@ -49,6 +49,8 @@ struct GemmMxf4Args {
     int32_t *status;
 };
 cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st);
+// CTA-pair kernel (gemm_mxf4_pair.cu), used by launch_gemm_mxf4 when M > 128.
+cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st);
 
 // ---- HiF4 quantization (quant_hif4.cu); metadata layout RFQ_SCALE_MMA is
 // block-major [K/64][rows rounded up to 128]
