@@ -51,6 +51,7 @@ def _peaks():
 # source file of each timed kernel: its DRAM counters hold only for the
 # sources they were taken on (the kernel's file plus the shared headers)
 _KERNEL_SRC = {"gemm_mxf4_kernel": "gemm_mxf4.cu", "gemm_mxf4_pair_kernel": "gemm_mxf4_pair.cu",
+               "gemm_mxf4_fused_kernel": "gemm_mxf4_fused.cu",
                "act_quant_mxfp4_kernel": "quant_mxfp4.cu",
                "gemm_hif4_kernel": "gemm_hif4.cu", "act_quant_hif4_kernel": "quant_hif4.cu"}
 
@@ -277,6 +278,9 @@ def run_rfq(args):
     M, K, N = spec.act.M, spec.act.K, spec.N
     hif4 = spec.fmt == "hif4"
     quant_only = N == 0
+    fused = args.variant == "fused"
+    if fused and (hif4 or quant_only):
+        raise SystemExit("--variant fused applies to the MXFP4 linear workloads")
     F = rfq.RFQ_FMT_HIF4 if hif4 else rfq.RFQ_FMT_MXFP4
     L = rfq.RFQ_SCALE_MMA
 
@@ -314,6 +318,16 @@ def run_rfq(args):
     per_step = [(ev(), ev(), ev(), ev()) for _ in range(args.steps)]
 
     def step(i=None):
+        if fused:
+            # the quantizer runs inside the GEMM: one kernel per step
+            if i is not None:
+                per_step[i][0].record(stream)
+                per_step[i][1].record(stream)
+                per_step[i][2].record(stream)
+            rfq.rfq_linear_fused(x, wop, y, rfq.RFQ_OUT_BF16, wsp, stream=stream)
+            if i is not None:
+                per_step[i][3].record(stream)
+            return
         if i is not None:
             per_step[i][0].record(stream)
         rfq.rfq_quantize_act(x, xq, xr, None, stream=stream)
@@ -396,17 +410,21 @@ def run_rfq(args):
         t_src = (f"{pk['src']} bf16 burst {pk['bf16_burst']} TFLOP/s x {FP4_OVER_BF16:g} "
                  f"(nominal dense FP4/BF16 ratio), of {pk['src']}")
         # more than one 128-row tile runs on CTA pairs (see launch_gemm_mxf4)
-        t_kernel = "gemm_mxf4_pair_kernel" if M > 128 else "gemm_mxf4_kernel"
+        t_kernel = "gemm_mxf4_fused_kernel" if fused else (
+            "gemm_mxf4_pair_kernel" if M > 128 else "gemm_mxf4_kernel")
     if hif4:
         aq_bytes = M * K * 2 + 2 * (M * K // 2) + 2 * (((M + 127) // 128) * 128 * (K // 64) * 4)
         aq_kernel = "act_quant_hif4_kernel"
     else:
         aq_bytes = M * K * 2 + 2 * (M * K // 2) + 2 * (((M + 127) // 128) * 128 * K // 32)
         aq_kernel = "act_quant_mxfp4_kernel"
-    aq_gbs = aq_bytes / (q_ms * 1e-3) / 1e9
-    act_quant = {"bound": "hbm", "kernel": aq_kernel, "achieved": aq_gbs, "peak": pk["hbm"], "unit": "GB/s",
-                 "frac": aq_gbs / pk["hbm"], "bytes_per_launch": aq_bytes, "ms_per_launch": q_ms,
-                 "traffic": _kernel_traffic(aq_kernel, spec.name)}
+    if fused:
+        act_quant = None   # quantization happens inside the GEMM
+    else:
+        aq_gbs = aq_bytes / (q_ms * 1e-3) / 1e9
+        act_quant = {"bound": "hbm", "kernel": aq_kernel, "achieved": aq_gbs, "peak": pk["hbm"], "unit": "GB/s",
+                     "frac": aq_gbs / pk["hbm"], "bytes_per_launch": aq_bytes, "ms_per_launch": q_ms,
+                     "traffic": _kernel_traffic(aq_kernel, spec.name)}
     if quant_only:
         value = _job_rate(aq_bytes, ws, ms) / 1e9
         unit = "GB/s"
@@ -439,12 +457,14 @@ def run_rfq(args):
             "vs_baseline": None,
             "dtype": "hif4 (exact bf16 x bf16, fp32 accumulate)" if hif4 else "mxfp4 (e2m1 x e2m1, fp32 accumulate)",
             "data": "synthetic",
-            "config": _config(spec, {"parallelism": f"dp{ws} over token rows" if ws > 1 else "single GPU"}),
+            "config": _config(spec, {"parallelism": f"dp{ws} over token rows" if ws > 1 else "single GPU",
+                                     "variant": ("fused prologue: X quantized inside the GEMM" if fused
+                                                 else "quantizer kernel + GEMM kernel")}),
             "roofline": roofline,
             "act_quant": act_quant,
             "expand_ms_per_step": x_ms if hif4 else None,
             "e2e": e2e,
-            "gpu_launches": (1 if quant_only else (4 if hif4 else 2)) * args.steps,
+            "gpu_launches": (1 if quant_only or fused else (4 if hif4 else 2)) * args.steps,
             "clocks": clocks,
             "cpu_baseline": cpu,
         }
@@ -464,6 +484,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffer) timing")
     ap.add_argument("--rows", type=int, default=0, help="profile a smaller case: the first ROWS token rows")
+    ap.add_argument("--variant", default="two-kernel", choices=["two-kernel", "fused"],
+                    help="fused: rfq_linear_fused, the activation quantizer inside the GEMM")
     ap.add_argument("--workload", default=WORKLOAD,
                     choices=["wan_ffn_up", "qwen_gate_up", "qwen_down_hif4", "act_quant", "tiny"])
     args = ap.parse_args()

@@ -175,6 +175,25 @@ RFQ_API rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, cons
                       int32_t phi_r_s, const rfq_qtensor *wq, void *y, int32_t out_dtype,
                       void *workspace, void *stream);
 
+/* RFQ linear layer with the activation quantizer fused into the GEMM (the
+ * on-the-fly residual of Sec. 4.3): Y = Q(X) W~ + phi Q(X - Q(X)) W~ with X
+ * read as bf16 and quantized inside the GEMM, block by block, exactly as
+ * rfq_quantize_act would (MXFP4: E8M0 scale floor(log2 amax) - 2, RNE
+ * saturating E2M1 codes, exact residual) -- no quantized copy of X is
+ * written to memory.  x_bf16: device bf16 [M][K] row-major (16-byte
+ * aligned).  wq: MXFP4 weight [N x K] with RFQ_SCALE_MMA scales.
+ * fb: NULL or mode RFQ_FALLBACK_ALL (residual on every block) or
+ * RFQ_FALLBACK_NONE (plain W4A4); RFQ_FALLBACK_AMAX returns
+ * RFQ_ERR_UNSUPPORTED.  K % 128 == 0, N % 16 == 0, M >= 0.  y, out_dtype,
+ * workspace: as for rfq_linear.  Each output tile quantizes its 128 rows of
+ * X again, so this variant pays off for narrow layers (N of a few tiles of
+ * 256); for wide ones rfq_quantize_act + rfq_linear is faster.
+ * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
+ * RFQ_ERR_UNSUPPORTED, RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */
+RFQ_API rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, const rfq_qtensor *wq,
+                                    const rfq_fallback *fb, void *y, int32_t out_dtype, void *workspace,
+                                    void *stream);
+
 /* Synchronizes `stream` and returns the device status left in a workspace by
  * earlier calls (RFQ_OK or RFQ_ERR_TIMEOUT); clears it when `clear` != 0. */
 RFQ_API rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *stream);

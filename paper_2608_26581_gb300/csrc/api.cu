@@ -326,6 +326,50 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
     return from_cuda(launch_gemm_mxf4(a, st));
 }
 
+rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, const rfq_qtensor *wq,
+                            const rfq_fallback *fb, void *y, int32_t out_dtype, void *workspace, void *stream)
+{
+    if (!x_bf16 || !wq || !y || !workspace)
+        return RFQ_ERR_INVALID_ARG;
+    if (out_dtype != RFQ_OUT_F32 && out_dtype != RFQ_OUT_BF16)
+        return RFQ_ERR_INVALID_ARG;
+    const int32_t mode = fb ? fb->mode : RFQ_FALLBACK_ALL;
+    if (mode != RFQ_FALLBACK_ALL && mode != RFQ_FALLBACK_NONE && mode != RFQ_FALLBACK_AMAX)
+        return RFQ_ERR_INVALID_ARG;
+    const int64_t N = wq->rows;
+    if (M < 0 || N < 0 || K <= 0 || wq->k != K)
+        return RFQ_ERR_SHAPE;
+    rfq_status s = check_qtensor(wq, N, K);
+    if (s != RFQ_OK)
+        return s;
+    if (wq->fmt != RFQ_FMT_MXFP4)
+        return RFQ_ERR_INVALID_ARG;
+    if (K % 128 != 0 || N % 16 != 0)
+        return RFQ_ERR_SHAPE;
+    if (M > (int64_t)INT32_MAX || N > (int64_t)INT32_MAX || K > (int64_t)INT32_MAX)
+        return RFQ_ERR_SHAPE;
+    if (!aligned16(x_bf16) || !aligned16(y) || !aligned16(workspace))
+        return RFQ_ERR_ALIGNMENT;
+    if (mode == RFQ_FALLBACK_AMAX || wq->scale_layout != RFQ_SCALE_MMA)
+        return RFQ_ERR_UNSUPPORTED;
+    if ((s = check_device()) != RFQ_OK)
+        return s;
+    if (M == 0 || N == 0)
+        return RFQ_OK;
+    GemmFusedArgs a;
+    a.x = x_bf16;
+    a.b_codes = wq->codes;
+    a.b_sf = wq->scales;
+    a.y = y;
+    a.out_bf16 = out_dtype == RFQ_OUT_BF16;
+    a.residual = mode == RFQ_FALLBACK_ALL;
+    a.M = M;
+    a.N = N;
+    a.K = K;
+    a.status = static_cast<int32_t *>(workspace);
+    return from_cuda(launch_gemm_mxf4_fused(a, static_cast<cudaStream_t>(stream)));
+}
+
 rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *stream)
 {
     if (!workspace)

@@ -52,6 +52,18 @@ cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st);
 // CTA-pair kernel (gemm_mxf4_pair.cu), used by launch_gemm_mxf4 when M > 128.
 cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st);
 
+// ---- RFQ linear with the quantizer fused into the GEMM (gemm_mxf4_fused.cu)
+struct GemmFusedArgs {
+    const void *x;                 // bf16 [M][K]
+    const void *b_codes, *b_sf;    // MXFP4 weight, MMA-layout scales
+    void *y;
+    int out_bf16;
+    int residual;                  // 1: phi = 1 everywhere, 0: plain W4A4
+    int64_t M, N, K;
+    int32_t *status;
+};
+cudaError_t launch_gemm_mxf4_fused(const GemmFusedArgs &a, cudaStream_t st);
+
 // ---- HiF4 quantization (quant_hif4.cu); metadata layout RFQ_SCALE_MMA is
 // block-major [K/64][rows rounded up to 128]
 cudaError_t launch_act_quant_hif4(const void *x, int64_t M, int64_t K, int mode, int p_s, int r_s, void *mcodes,

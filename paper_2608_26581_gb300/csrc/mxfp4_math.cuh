@@ -1,0 +1,172 @@
+// mxfp4_math.cuh -- per-lane MXFP4 quantization arithmetic (Sec. 3.2 Eq. 3-4,
+// Sec. 4.3), shared by the activation quantizer and the fused-prologue GEMM.
+//
+// Four consecutive lanes hold one 32-element block, eight elements each.
+// The E8M0 byte is the fp32 exponent field of the block's amax minus 2 (OCP
+// rule floor(log2 amax) - 2, clamped at 0), every scaling is by a power of
+// two, the E2M1 conversion rounds to nearest even and saturates, and the
+// residual x - q 2^e is exact in fp32 (at most 11 significant bits), so the
+// result is the fp64 definition bit for bit.
+#pragma once
+
+#include <cuda_fp16.h>
+#include <cstdint>
+
+namespace rfq {
+
+// Four E2M1 conversions (round-to-nearest-even, saturating): eight fp32
+// values -> eight codes, element 2i in the low nibble of byte i.
+__device__ __forceinline__ uint32_t e2m1x8(const float (&y)[8])
+{
+    uint32_t out;
+    asm("{\n\t.reg .b8 b0, b1, b2, b3;\n\t"
+        "cvt.rn.satfinite.e2m1x2.f32 b0, %2, %1;\n\t"
+        "cvt.rn.satfinite.e2m1x2.f32 b1, %4, %3;\n\t"
+        "cvt.rn.satfinite.e2m1x2.f32 b2, %6, %5;\n\t"
+        "cvt.rn.satfinite.e2m1x2.f32 b3, %8, %7;\n\t"
+        "mov.b32 %0, {b0, b1, b2, b3};\n\t}"
+        : "=r"(out)
+        : "f"(y[0]), "f"(y[1]), "f"(y[2]), "f"(y[3]), "f"(y[4]), "f"(y[5]), "f"(y[6]), "f"(y[7]));
+    return out;
+}
+
+// Eight E2M1 codes -> their values (exact), via the e2m1x2 -> f16x2 decode.
+__device__ __forceinline__ void e2m1x8_decode(uint32_t codes, float (&q)[8])
+{
+    uint32_t h[4];
+    asm("{\n\t.reg .b8 b0, b1, b2, b3;\n\t"
+        "mov.b32 {b0, b1, b2, b3}, %4;\n\t"
+        "cvt.rn.f16x2.e2m1x2 %0, b0;\n\t"
+        "cvt.rn.f16x2.e2m1x2 %1, b1;\n\t"
+        "cvt.rn.f16x2.e2m1x2 %2, b2;\n\t"
+        "cvt.rn.f16x2.e2m1x2 %3, b3;\n\t}"
+        : "=r"(h[0]), "=r"(h[1]), "=r"(h[2]), "=r"(h[3])
+        : "r"(codes));
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        __half2 v = *reinterpret_cast<__half2 *>(&h[i]);
+        q[2 * i] = __low2float(v);
+        q[2 * i + 1] = __high2float(v);
+    }
+}
+
+// E8M0 byte of a block from the fp32 exponent field of its amax:
+// floor(log2 amax) - 2 + 127 = field - 2, clamped at 0 (2^-127; also amax = 0).
+__device__ __forceinline__ int scale_byte_from_f32_bits(uint32_t amax_bits)
+{
+    return max((int)((amax_bits >> 23) & 0xFF) - 2, 0);
+}
+
+__device__ __forceinline__ float pow2_neg_e(int byte) // 2^-(byte-127), normal for byte <= 252
+{
+    return __uint_as_float((uint32_t)(254 - byte) << 23);
+}
+
+__device__ __forceinline__ float pow2_e(int byte) // 2^(byte-127); byte 0 -> subnormal 2^-127
+{
+    return byte ? __uint_as_float((uint32_t)byte << 23) : __uint_as_float(0x00400000u);
+}
+
+__device__ __forceinline__ void bf16x8_to_f32(const uint4 &v, float (&x)[8])
+{
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        x[2 * i] = __uint_as_float(w[i] << 16);
+        x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+    }
+}
+
+// Packed fp32 pairs (Blackwell f32x2 arithmetic): one instruction for two
+// multiplies or fused multiply-adds, both rounded to nearest even.
+__device__ __forceinline__ uint64_t f2pack(float a, float b)
+{
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+    return r;
+}
+
+__device__ __forceinline__ void f2unpack(uint64_t v, float &a, float &b)
+{
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
+}
+
+__device__ __forceinline__ uint64_t fmul2(uint64_t a, uint64_t b)
+{
+    uint64_t r;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c)
+{
+    uint64_t r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+
+__device__ __forceinline__ float fmax3(float a, float b, float c)
+{
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
+// max |v_i| over eight values
+__device__ __forceinline__ float absmax8(const float (&v)[8])
+{
+    const float m0 = fmax3(fabsf(v[0]), fabsf(v[1]), fabsf(v[2]));
+    const float m1 = fmax3(fabsf(v[3]), fabsf(v[4]), fabsf(v[5]));
+    return fmax3(m0, m1, fmaxf(fabsf(v[6]), fabsf(v[7])));
+}
+
+// Quantizes this lane's eight elements (its 32-element block is spread over
+// four consecutive lanes, all 32 lanes take part): the E2M1 codes (element
+// 2i in the low nibble of byte i) and E8M0 byte of X~, and with RES those of
+// the residual X - X~.
+struct Mx8 {
+    uint32_t code, rcode;
+    int sb, rb;
+};
+
+template <bool RES>
+__device__ __forceinline__ Mx8 mxfp4_quant8(const float (&xf)[8])
+{
+    Mx8 o;
+    float am = absmax8(xf);
+    am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 1));
+    am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 2));
+    o.sb = scale_byte_from_f32_bits(__float_as_uint(am));
+    const float inv = pow2_neg_e(o.sb);
+    const uint64_t inv2 = f2pack(inv, inv);
+    float y[8];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+        f2unpack(fmul2(f2pack(xf[2 * i], xf[2 * i + 1]), inv2), y[2 * i], y[2 * i + 1]);
+    o.code = e2m1x8(y);
+    o.rcode = 0;
+    o.rb = 0;
+    if (RES) {
+        float q[8], r[8];
+        e2m1x8_decode(o.code, q);
+        const float nsc = -pow2_e(o.sb);
+        const uint64_t nsc2 = f2pack(nsc, nsc);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) // x - x~ (exact)
+            f2unpack(ffma2(f2pack(q[2 * i], q[2 * i + 1]), nsc2, f2pack(xf[2 * i], xf[2 * i + 1])), r[2 * i],
+                     r[2 * i + 1]);
+        float ra = absmax8(r);
+        ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, 1));
+        ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, 2));
+        o.rb = scale_byte_from_f32_bits(__float_as_uint(ra));
+        const float rinv = pow2_neg_e(o.rb);
+        const uint64_t rinv2 = f2pack(rinv, rinv);
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            f2unpack(fmul2(f2pack(r[2 * i], r[2 * i + 1]), rinv2), r[2 * i], r[2 * i + 1]);
+        o.rcode = e2m1x8(r);
+    }
+    return o;
+}
+
+} // namespace rfq

@@ -18,72 +18,10 @@
 #include <cstdint>
 
 #include "internal.h"
+#include "mxfp4_math.cuh"
 
 namespace rfq {
 namespace {
-
-// Four E2M1 conversions (round-to-nearest-even, saturating): eight fp32
-// values -> eight codes, element 2i in the low nibble of byte i.
-__device__ __forceinline__ uint32_t e2m1x8(const float (&y)[8])
-{
-    uint32_t out;
-    asm("{\n\t.reg .b8 b0, b1, b2, b3;\n\t"
-        "cvt.rn.satfinite.e2m1x2.f32 b0, %2, %1;\n\t"
-        "cvt.rn.satfinite.e2m1x2.f32 b1, %4, %3;\n\t"
-        "cvt.rn.satfinite.e2m1x2.f32 b2, %6, %5;\n\t"
-        "cvt.rn.satfinite.e2m1x2.f32 b3, %8, %7;\n\t"
-        "mov.b32 %0, {b0, b1, b2, b3};\n\t}"
-        : "=r"(out)
-        : "f"(y[0]), "f"(y[1]), "f"(y[2]), "f"(y[3]), "f"(y[4]), "f"(y[5]), "f"(y[6]), "f"(y[7]));
-    return out;
-}
-
-// Eight E2M1 codes -> their values (exact), via the e2m1x2 -> f16x2 decode.
-__device__ __forceinline__ void e2m1x8_decode(uint32_t codes, float (&q)[8])
-{
-    uint32_t h[4];
-    asm("{\n\t.reg .b8 b0, b1, b2, b3;\n\t"
-        "mov.b32 {b0, b1, b2, b3}, %4;\n\t"
-        "cvt.rn.f16x2.e2m1x2 %0, b0;\n\t"
-        "cvt.rn.f16x2.e2m1x2 %1, b1;\n\t"
-        "cvt.rn.f16x2.e2m1x2 %2, b2;\n\t"
-        "cvt.rn.f16x2.e2m1x2 %3, b3;\n\t}"
-        : "=r"(h[0]), "=r"(h[1]), "=r"(h[2]), "=r"(h[3])
-        : "r"(codes));
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        __half2 v = *reinterpret_cast<__half2 *>(&h[i]);
-        q[2 * i] = __low2float(v);
-        q[2 * i + 1] = __high2float(v);
-    }
-}
-
-// E8M0 byte of a block from the fp32 exponent field of its amax:
-// floor(log2 amax) - 2 + 127 = field - 2, clamped at 0 (2^-127; also amax = 0).
-__device__ __forceinline__ int scale_byte_from_f32_bits(uint32_t amax_bits)
-{
-    return max((int)((amax_bits >> 23) & 0xFF) - 2, 0);
-}
-
-__device__ __forceinline__ float pow2_neg_e(int byte) // 2^-(byte-127), normal for byte <= 252
-{
-    return __uint_as_float((uint32_t)(254 - byte) << 23);
-}
-
-__device__ __forceinline__ float pow2_e(int byte) // 2^(byte-127); byte 0 -> subnormal 2^-127
-{
-    return byte ? __uint_as_float((uint32_t)byte << 23) : __uint_as_float(0x00400000u);
-}
-
-__device__ __forceinline__ void bf16x8_to_f32(const uint4 &v, float (&x)[8])
-{
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        x[2 * i] = __uint_as_float(w[i] << 16);
-        x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
-    }
-}
 
 template <int LAYOUT>
 __device__ __forceinline__ int64_t scale_index(int64_t m, int64_t b, int64_t kblocks)
@@ -91,49 +29,6 @@ __device__ __forceinline__ int64_t scale_index(int64_t m, int64_t b, int64_t kbl
     if (LAYOUT == RFQ_SCALE_MMA)
         return sf_mma_offset(m, b, kblocks >> 2);
     return m * kblocks + b;
-}
-
-// Packed fp32 pairs (Blackwell f32x2 arithmetic): one instruction for two
-// multiplies or fused multiply-adds, both rounded to nearest even.
-__device__ __forceinline__ uint64_t f2pack(float a, float b)
-{
-    uint64_t r;
-    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
-    return r;
-}
-
-__device__ __forceinline__ void f2unpack(uint64_t v, float &a, float &b)
-{
-    asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
-}
-
-__device__ __forceinline__ uint64_t fmul2(uint64_t a, uint64_t b)
-{
-    uint64_t r;
-    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
-    return r;
-}
-
-__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c)
-{
-    uint64_t r;
-    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
-    return r;
-}
-
-__device__ __forceinline__ float fmax3(float a, float b, float c)
-{
-    float d;
-    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
-    return d;
-}
-
-// max |v_i| over eight values
-__device__ __forceinline__ float absmax8(const float (&v)[8])
-{
-    const float m0 = fmax3(fabsf(v[0]), fabsf(v[1]), fabsf(v[2]));
-    const float m1 = fmax3(fabsf(v[3]), fabsf(v[4]), fabsf(v[5]));
-    return fmax3(m0, m1, fmaxf(fabsf(v[6]), fabsf(v[7])));
 }
 
 // Items are (row, 1024-element segment); a warp handles one item with four
@@ -197,47 +92,18 @@ __global__ void __launch_bounds__(256) act_quant_mxfp4_kernel(const uint4 *__res
             const int64_t soff = LAYOUT == RFQ_SCALE_MMA ? srow + ((b >> 2) << 9) + (b & 3) : srow + b;
             float xf[8];
             bf16x8_to_f32(v[j], xf);
-            // block amax -> E8M0 byte from the exponent field (Sec. 3.2 Eq. 3, OCP rule)
-            float am = absmax8(xf);
-            am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 1));
-            am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 2));
-            const int sb = scale_byte_from_f32_bits(__float_as_uint(am));
-            const float inv = pow2_neg_e(sb);
-            const uint64_t inv2 = f2pack(inv, inv);
-            float y[8];
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-                f2unpack(fmul2(f2pack(xf[2 * i], xf[2 * i + 1]), inv2), y[2 * i], y[2 * i + 1]);
-            const uint32_t qc = e2m1x8(y);
+            const Mx8 qz = mxfp4_quant8<RES>(xf);
             if (ok) {
-                mrow[c] = qc;
+                mrow[c] = qz.code;
                 if ((lane & 3) == 0)
-                    mscales[soff] = (uint8_t)sb;
+                    mscales[soff] = (uint8_t)qz.sb;
             }
             if (RES) {
                 const bool on = !PHI || (ok && prow[(c * 8) / r_s] != 0);
-                float q[8], r[8];
-                e2m1x8_decode(qc, q);
-                const float nsc = -pow2_e(sb);
-                const uint64_t nsc2 = f2pack(nsc, nsc);
-#pragma unroll
-                for (int i = 0; i < 4; ++i) // x - x~ (exact)
-                    f2unpack(ffma2(f2pack(q[2 * i], q[2 * i + 1]), nsc2, f2pack(xf[2 * i], xf[2 * i + 1])),
-                             r[2 * i], r[2 * i + 1]);
-                float ra = absmax8(r);
-                ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, 1));
-                ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, 2));
-                const int rb = scale_byte_from_f32_bits(__float_as_uint(ra));
-                const float rinv = pow2_neg_e(rb);
-                const uint64_t rinv2 = f2pack(rinv, rinv);
-#pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    f2unpack(fmul2(f2pack(r[2 * i], r[2 * i + 1]), rinv2), r[2 * i], r[2 * i + 1]);
-                const uint32_t rc = e2m1x8(r);
                 if (ok) {
-                    rrow[c] = on ? rc : 0u;
+                    rrow[c] = on ? qz.rcode : 0u;
                     if ((lane & 3) == 0)
-                        rscales[soff] = on ? (uint8_t)rb : 0;
+                        rscales[soff] = on ? (uint8_t)qz.rb : 0;
                 }
             }
         }

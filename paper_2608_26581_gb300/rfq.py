@@ -20,12 +20,14 @@ RFQ_FMT_MXFP4, RFQ_FMT_HIF4, RFQ_FMT_BF16 = 0, 1, 2
 RFQ_SCALE_ROWMAJOR, RFQ_SCALE_MMA = 0, 1
 RFQ_FALLBACK_NONE, RFQ_FALLBACK_ALL, RFQ_FALLBACK_AMAX = 0, 1, 2
 RFQ_OUT_F32, RFQ_OUT_BF16 = 0, 1
+(RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT, RFQ_ERR_UNSUPPORTED, RFQ_ERR_CUDA, RFQ_ERR_TIMEOUT,
+ RFQ_ERR_DEVICE) = range(1, 8)
 STATUS_NAMES = {0: "RFQ_OK", 1: "RFQ_ERR_INVALID_ARG", 2: "RFQ_ERR_SHAPE", 3: "RFQ_ERR_ALIGNMENT",
                 4: "RFQ_ERR_UNSUPPORTED", 5: "RFQ_ERR_CUDA", 6: "RFQ_ERR_TIMEOUT", 7: "RFQ_ERR_DEVICE"}
 
 EXPORTED = ("rfq_status_string", "rfq_qtensor_bytes", "rfq_quantize_weight", "rfq_quantize_act",
             "rfq_linear_workspace_bytes", "rfq_linear", "rfq_workspace_status", "rfq_dequant",
-            "rfq_linear_noalloc")
+            "rfq_linear_noalloc", "rfq_linear_fused")
 
 
 class RFQError(RuntimeError):
@@ -74,6 +76,8 @@ def load_library(path: str = LIB_PATH):
         lib.rfq_dequant.argtypes = [QTP, P, I32, P]
         lib.rfq_linear_noalloc.restype = I32
         lib.rfq_linear_noalloc.argtypes = [QTP, QTP, P, I32, QTP, P, I32, P]
+        lib.rfq_linear_fused.restype = I32
+        lib.rfq_linear_fused.argtypes = [P, I64, I64, QTP, ctypes.POINTER(_FB), P, I32, P, P]
         _lib = lib
     return _lib
 
@@ -190,3 +194,14 @@ def rfq_linear_noalloc(xq: QTensor, xr: QTensor | None, phi: torch.Tensor | None
     _check(load_library().rfq_linear_noalloc(ctypes.byref(q), ctypes.byref(r) if r is not None else None,
                                              _ptr(phi), phi_r_s, ctypes.byref(w), _ptr(y), out_dtype,
                                              _stream(stream)), "rfq_linear_noalloc")
+
+
+def rfq_linear_fused(x: torch.Tensor, wq: QTensor, y: torch.Tensor, out_dtype: int, workspace: torch.Tensor,
+                     mode: int = RFQ_FALLBACK_ALL, stream=None):
+    """Y = Q(X) W~ + phi Q(X - Q(X)) W~ with X (bf16 [M, K]) quantized inside
+    the GEMM; mode RFQ_FALLBACK_ALL or RFQ_FALLBACK_NONE."""
+    M, K = x.shape
+    fb = _FB(mode, 0.0, 128, 256)
+    w = wq.c()
+    _check(load_library().rfq_linear_fused(_ptr(x), M, K, ctypes.byref(w), ctypes.byref(fb), _ptr(y), out_dtype,
+                                           _ptr(workspace), _stream(stream)), "rfq_linear_fused")

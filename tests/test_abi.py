@@ -75,3 +75,27 @@ def test_null_arguments_rejected_before_any_device_work(lib):
                                 None, None) == 2
     qt = rfq._QT(0, 0, 4, 64, 8, 16)              # misaligned codes pointer
     assert lib.rfq_dequant(ctypes.byref(qt), ctypes.c_void_p(16), 0, None) == 3
+
+
+def test_fused_linear_host_checks(lib):
+    """rfq_linear_fused validates its arguments on the host: null pointers,
+    K not a multiple of 128, N not a multiple of 16, the phi = AMAX mode it
+    does not implement and misaligned pointers are all rejected before any
+    device work."""
+    from paper_2608_26581_gb300 import rfq
+    P = ctypes.c_void_p
+    assert lib.rfq_linear_fused(None, 1, 128, None, None, None, 0, None, None) == rfq.RFQ_ERR_INVALID_ARG
+    # every call below is rejected on the host: none may reach a launch, since
+    # the pointers are not device memory
+    wq = rfq._QT(rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA, 256, 128, 16, 16)
+    bad_k = rfq._QT(rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA, 256, 96, 16, 16)
+    assert lib.rfq_linear_fused(P(16), 4, 96, ctypes.byref(bad_k), None, P(16), 1, P(16), None) == \
+        rfq.RFQ_ERR_SHAPE
+    bad_n = rfq._QT(rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA, 40, 128, 16, 16)
+    assert lib.rfq_linear_fused(P(16), 4, 128, ctypes.byref(bad_n), None, P(16), 1, P(16), None) == \
+        rfq.RFQ_ERR_SHAPE
+    amax = rfq._FB(rfq.RFQ_FALLBACK_AMAX, 1.0, 128, 256)
+    assert lib.rfq_linear_fused(P(16), 4, 128, ctypes.byref(wq), ctypes.byref(amax), P(16), 1, P(16), None) == \
+        rfq.RFQ_ERR_UNSUPPORTED
+    assert lib.rfq_linear_fused(P(8), 4, 128, ctypes.byref(wq), None, P(16), 1, P(16), None) == \
+        rfq.RFQ_ERR_ALIGNMENT
