@@ -281,6 +281,11 @@ def run_rfq(args):
     fused = args.variant == "fused"
     if fused and (hif4 or quant_only):
         raise SystemExit("--variant fused applies to the MXFP4 linear workloads")
+    # selective fallback: phi(p, r) = [max |x| over the 128 x 256 tile > tau]
+    # (Sec. 4.3); the GEMMs skip the residual loads and MMAs of phi = 0 tiles
+    amax_phi = args.phi_tau is not None
+    if amax_phi and (fused or quant_only):
+        raise SystemExit("--phi-tau applies to the two-kernel linear workloads")
     F = rfq.RFQ_FMT_HIF4 if hif4 else rfq.RFQ_FMT_MXFP4
     L = rfq.RFQ_SCALE_MMA
 
@@ -301,6 +306,8 @@ def run_rfq(args):
         del w
     xq = rfq.empty_qtensor(F, L, M, K, device=dev)
     xr = rfq.empty_qtensor(F, L, M, K, device=dev)
+    phi_buf = (torch.empty(((M + 127) // 128) * ((K + 255) // 256), dtype=torch.uint8, device=dev)
+               if args.phi_tau is not None else None)
     # HiF4: the GEMM takes the exact bf16 expansions of X~ and X^ (expanding
     # once per activation, not once per output tile inside the GEMM)
     xq16 = rfq.empty_bf16_operand(M, K, device=dev) if hif4 and not quant_only else None
@@ -330,7 +337,11 @@ def run_rfq(args):
             return
         if i is not None:
             per_step[i][0].record(stream)
-        rfq.rfq_quantize_act(x, xq, xr, None, stream=stream)
+        if amax_phi:
+            rfq.rfq_quantize_act(x, xq, xr, phi_buf, mode=rfq.RFQ_FALLBACK_AMAX, tau=args.phi_tau, p_s=128,
+                                 r_s=256, stream=stream)
+        else:
+            rfq.rfq_quantize_act(x, xq, xr, None, stream=stream)
         if i is not None:
             per_step[i][1].record(stream)
         if hif4 and not quant_only:
@@ -339,9 +350,11 @@ def run_rfq(args):
         if i is not None:
             per_step[i][2].record(stream)
         if hif4 and not quant_only:
-            rfq.rfq_linear(xq16, xr16, None, 256, wop, y, rfq.RFQ_OUT_BF16, wsp, stream=stream)
+            rfq.rfq_linear(xq16, xr16, phi_buf if amax_phi else None, 256, wop, y, rfq.RFQ_OUT_BF16, wsp,
+                           stream=stream)
         elif not quant_only:
-            rfq.rfq_linear(xq, xr, None, 256, wop, y, rfq.RFQ_OUT_BF16, wsp, stream=stream)
+            rfq.rfq_linear(xq, xr, phi_buf if amax_phi else None, 256, wop, y, rfq.RFQ_OUT_BF16, wsp,
+                           stream=stream)
         if i is not None:
             per_step[i][3].record(stream)
 
@@ -396,7 +409,9 @@ def run_rfq(args):
     if rfq.rfq_workspace_status(wsp) != rfq.RFQ_OK:
         raise RuntimeError("rfq_linear reported a device timeout")
 
-    flop = 2.0 * 2.0 * M * N * K                 # main + residual product, phi = 1 everywhere
+    # executed MMA work: the main product, and the residual product on the phi = 1 tiles
+    phi_frac = float(phi_buf.float().mean().item()) if amax_phi else 1.0
+    flop = 2.0 * M * N * K * (1.0 + phi_frac)
     pk = _peaks()
     # The timed loop is short (tens of ms at full clocks), so the kernels are
     # held against the burst figure; the sustained one is reported beside it.
@@ -459,7 +474,10 @@ def run_rfq(args):
             "data": "synthetic",
             "config": _config(spec, {"parallelism": f"dp{ws} over token rows" if ws > 1 else "single GPU",
                                      "variant": ("fused prologue: X quantized inside the GEMM" if fused
-                                                 else "quantizer kernel + GEMM kernel")}),
+                                                 else "quantizer kernel + GEMM kernel"),
+                                     **({"phi": f"AMAX: phi = [max |x| over the 128 x 256 tile > {args.phi_tau}], "
+                                                f"fraction of phi = 1 tiles f = {phi_frac:.4f}",
+                                         "phi_fraction": phi_frac} if amax_phi else {})}),
             "roofline": roofline,
             "act_quant": act_quant,
             "expand_ms_per_step": x_ms if hif4 else None,
@@ -484,6 +502,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffer) timing")
     ap.add_argument("--rows", type=int, default=0, help="profile a smaller case: the first ROWS token rows")
+    ap.add_argument("--phi-tau", type=float, default=None,
+                    help="selective fallback: residual only on 128 x 256 tiles whose max |x| exceeds TAU")
     ap.add_argument("--variant", default="two-kernel", choices=["two-kernel", "fused"],
                     help="fused: rfq_linear_fused, the activation quantizer inside the GEMM")
     ap.add_argument("--workload", default=WORKLOAD,

@@ -68,6 +68,7 @@ struct Smem {
     uint64_t acc_full[2];
     uint64_t acc_empty[2];
     uint64_t drain;
+    uint32_t res_on[STAGES];   // the residual of the stage applies (from phi, published by the producer)
     uint32_t tmem_base;
     int32_t abort_flag;
     int32_t issued;
@@ -167,15 +168,17 @@ __global__ void __launch_bounds__(THREADS, 1)
     tc_fence_after();
     const uint32_t tmem = S.tmem_base;
 
-    auto res_on = [&](int m_tile, int ks) -> bool {
-        return RES && (!PHI || phi[(int64_t)m_tile * phi_cols + ks / phi_blocks] != 0);
-    };
-
     if (warp == 0) {
         // ------------------------------------------------ TMA producer
         if (lane == 0) {
             int p = 0;
             bool stop = false;
+            // phi byte of the next k-stage: loaded one stage ahead and tested
+            // only after the next wait, so its global-memory latency overlaps
+            // that wait
+            uint32_t ph = 0;
+            if (PHI && (int)blockIdx.x < tiles)
+                ph = __ldg(phi + (int64_t)(blockIdx.x / n_tiles) * phi_cols);
             for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x) {
                 const int m_tile = tile / n_tiles, n_tile = tile - m_tile * n_tiles;
                 for (int ks = 0; ks < nks; ++ks, ++p) {
@@ -185,7 +188,10 @@ __global__ void __launch_bounds__(THREADS, 1)
                         stop = true;
                         break;
                     }
-                    const bool ron = res_on(m_tile, ks);
+                    // published to the MMA thread and the converters through the
+                    // stage's barrier
+                    const bool ron = RES && (!PHI || ph != 0);
+                    S.res_on[slot] = ron;
                     auto &st = S.st[slot];
                     uint64_t *bar = &S.full[slot];
                     if (CONV) {
@@ -209,6 +215,11 @@ __global__ void __launch_bounds__(THREADS, 1)
                         if (ron)
                             tma_load_2d(st.r16, &tmR, bar, ks * BK * 2, m_tile * BM);
                     }
+                    if (PHI) {
+                        const int nt = ks + 1 < nks ? tile : tile + (int)gridDim.x, nk = ks + 1 < nks ? ks + 1 : 0;
+                        if (nt < tiles)
+                            ph = __ldg(phi + (int64_t)(nt / n_tiles) * phi_cols + nk / phi_blocks);
+                    }
                 }
             }
             S.issued = p;
@@ -220,7 +231,6 @@ __global__ void __launch_bounds__(THREADS, 1)
             bool stop = false;
             const uint32_t idesc = idesc_bf16(BM, BN);
             for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x, ++it) {
-                const int m_tile = tile / n_tiles;
                 const int buf = it & 1;
                 if (!mbar_wait(&S.acc_empty[buf], ((it >> 1) & 1) ^ 1, kWaitLimitNs, gstat)) {
                     flag_timeout(S, status);
@@ -239,7 +249,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     tc_fence_after();
                     const auto &st = S.st[slot];
                     const uint32_t a0 = smem_u32(st.a16), r0 = smem_u32(st.r16), b0 = smem_u32(st.b);
-                    const bool ron = res_on(m_tile, ks);
+                    const bool ron = RES && (!PHI || S.res_on[slot] != 0);
 #pragma unroll
                     for (int j = 0; j < BK / 16; ++j) {
                         const uint64_t bd = sdesc_k_sw128(b0 + 32 * j);
@@ -361,7 +371,6 @@ __global__ void __launch_bounds__(THREADS, 1)
         int p = 0;
         bool stop = false;
         for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x) {
-            const int m_tile = tile / n_tiles;
             for (int ks = 0; ks < nks; ++ks, ++p) {
                 const int slot = p % STAGES;
                 if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat)) {
@@ -371,7 +380,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     break;
                 }
                 auto &st = S.st[slot];
-                const bool ron = res_on(m_tile, ks);
+                const bool ron = RES && (!PHI || S.res_on[slot] != 0);
 #pragma unroll 2
                 for (int ch = u; ch < 2 * BM * 8; ch += 32 * CONV_WARPS) {
                     const bool isr = ch >= BM * 8;

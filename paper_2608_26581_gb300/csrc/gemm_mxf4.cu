@@ -16,7 +16,10 @@
 // SAME shared-memory W~ tile into the SAME TMEM accumulator: W~ is read once
 // for both products and the correction costs only MMA issue (the on-the-fly
 // residual accumulation of Sec. 4.3).  Residual MMAs of k-chunks with
-// phi = 0 are not issued and their A tiles are not loaded.  Eight epilogue
+// phi = 0 are not issued and their A tiles are not loaded; with selective phi
+// an extra warp turns the phi bytes into per-stage residual masks in shared
+// memory a block of 256 stages ahead (a global load issued by the producer
+// would wait behind the stage copies in flight).  Eight epilogue
 // warps drain the fp32 accumulator; with bf16 Y each warp first loads and
 // packs all 128 of its columns, hands the accumulator back to the MMA thread,
 // then stages and stores them (shared memory + TMA stores), so the next
@@ -55,6 +58,8 @@ constexpr int SF_SLOTS = 4;
 constexpr int EPI_WARPS = 8;
 constexpr int SF_WARPS = 4;
 constexpr int THREADS = 64 + 32 * EPI_WARPS + 32 * SF_WARPS;
+constexpr int PHI_WARP = THREADS / 32;  // the phi reader: one warp beyond THREADS
+constexpr int PHI_BLK = 256;            // stage masks per phi block
 static_assert(SF_COL0 + SF_SLOTS * SF_SLOT_COLS <= TMEM_COLS, "TMEM budget");
 static_assert(SF_SLOTS >= STAGES, "a scale slot is rewritten only after its stage's MMAs completed");
 
@@ -78,6 +83,10 @@ struct Smem {
     uint64_t acc_empty;
     uint64_t drain;
     uint64_t sf_ready[SF_SLOTS];      // the scale writers filled the slot
+    uint64_t phi_full[2];             // the phi reader filled the mask block
+    uint64_t phi_empty[2];            // the producer consumed the mask block
+    uint8_t phi_mask[2][PHI_BLK];     // per stage of a block: bit c, phi of chunk c is 1
+    uint32_t res_mask[STAGES];        // bit c: the residual of 128-element chunk c of the stage applies
     uint32_t tmem_base;
     int32_t abort_flag;
     int32_t issued;
@@ -92,14 +101,8 @@ __device__ __forceinline__ void flag_timeout(Smem &S, int32_t *status)
     atomicExch(status, kDevTimeout);
 }
 
-template <bool PHI>
-__device__ __forceinline__ bool res_chunk(const uint8_t *phi, int m_tile, int phi_cols, int phi_chunks, int chunk)
-{
-    return !PHI || phi[(int64_t)m_tile * phi_cols + chunk / phi_chunks] != 0;
-}
-
 template <bool RES, bool PHI, bool OUT_BF16>
-__global__ void __launch_bounds__(THREADS, 1)
+__global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     gemm_mxf4_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmR,
                      const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmY,
                      const uint8_t *__restrict__ sfa, const uint8_t *__restrict__ sfr,
@@ -136,6 +139,10 @@ __global__ void __launch_bounds__(THREADS, 1)
         mbar_init(&S.drain, 1);
         for (int i = 0; i < SF_SLOTS; ++i)
             mbar_init(&S.sf_ready[i], SF_WARPS);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&S.phi_full[i], 32);
+            mbar_init(&S.phi_empty[i], 1);
+        }
         S.issued = 0;
         fence_mbar_init();
     }
@@ -170,10 +177,22 @@ __global__ void __launch_bounds__(THREADS, 1)
                         break;
                     }
                     const int c0 = 2 * ks, nch = min(2, kc - c0);
-                    bool res_on = false;
-                    if (RES)
-                        for (int c = 0; c < nch; ++c)
-                            res_on |= res_chunk<PHI>(phi, m_tile, phi_cols, phi_chunks, c0 + c);
+                    // residual chunks of the stage, published to the MMA thread and
+                    // the writers through the stage's barrier
+                    uint32_t mask = RES ? (nch == 2 ? 3u : 1u) : 0u;
+                    if (PHI) {
+                        const int blk = p / PHI_BLK, e = p - blk * PHI_BLK;
+                        if (e == 0 && !mbar_wait(&S.phi_full[blk & 1], (blk >> 1) & 1, kWaitLimitNs, gstat)) {
+                            flag_timeout(S, status);
+                            stop = true;
+                            break;
+                        }
+                        mask = S.phi_mask[blk & 1][e];
+                        if (e == PHI_BLK - 1)
+                            mbar_arrive(&S.phi_empty[blk & 1]);
+                    }
+                    const bool res_on = mask != 0;
+                    S.res_mask[slot] = mask;
                     const int atom0 = n_tile * 2;
                     const int nb = atom0 + 1 < n_atoms ? 2 : 1;
                     const uint32_t sfbytes = (uint32_t)nch * ATOM;
@@ -200,7 +219,6 @@ __global__ void __launch_bounds__(THREADS, 1)
             int p = 0, it = 0;
             bool stop = false;
             for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x, ++it) {
-                const int m_tile = tile / n_tiles;
                 if (!mbar_wait(&S.acc_empty, (it & 1) ^ 1, kWaitLimitNs, gstat)) {
                     flag_timeout(S, status);
                     break;
@@ -218,6 +236,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                     const int c0 = 2 * ks, nch = min(2, kc - c0);
                     const uint32_t sf = tmem + SF_COL0 + SF_SLOT_COLS * sfs;
                     const Stage &st = S.st[slot];
+                    // without selective phi the mask is fixed: no shared-memory read on the issue path
+                    const uint32_t res_mask = PHI ? S.res_mask[slot] : (RES ? (nch == 2 ? 3u : 1u) : 0u);
                     const uint32_t a0 = smem_u32(st.a), r0 = smem_u32(st.r), b0 = smem_u32(st.b);
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
@@ -228,7 +248,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                         const uint64_t bd = sdesc_k_sw128(b0 + 32 * j);
                         const uint32_t sfb_t = sf + 16 + 8 * c;
                         tc_mma_mxf4(tmem, sdesc_k_sw128(a0 + 32 * j), bd, id, sf + 4 * c, sfb_t, (ks | j) != 0);
-                        if (RES && res_chunk<PHI>(phi, m_tile, phi_cols, phi_chunks, c0 + c))
+                        if (RES && ((res_mask >> c) & 1))
                             tc_mma_mxf4(tmem, sdesc_k_sw128(r0 + 32 * j), bd, id, sf + 8 + 4 * c, sfb_t, 1);
                     }
                     tc_commit(&S.empty[slot]);
@@ -351,7 +371,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         if (lane == 0)
             bulk_wait_group<0>(); // every TMA store of this warp has completed
-    } else {
+    } else if (warp < PHI_WARP) {
         // ------------------------------------------------ scale writers (warps 10..13)
         // Warp quarter q writes TMEM lanes 32q..32q+31; every quarter holds
         // the same scale words (the MMA reads row 32 j + i from column j of
@@ -360,7 +380,6 @@ __global__ void __launch_bounds__(THREADS, 1)
         int p = 0;
         bool stop = false;
         for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x) {
-            const int m_tile = tile / n_tiles;
             for (int ks = 0; ks < nks; ++ks, ++p) {
                 const int slot = p % STAGES, sfs = p % SF_SLOTS;
                 // warp-uniform outcome: the tcgen05 stores below need the whole warp
@@ -382,7 +401,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     const uint4 vb0 = *reinterpret_cast<const uint4 *>(st.sfb + c * ATOM + lane * 16);
                     const uint4 vb1 = *reinterpret_cast<const uint4 *>(st.sfb + (2 + c) * ATOM + lane * 16);
                     tmem_st_32x32b_x4(tb + 4 * c, va.x, va.y, va.z, va.w);
-                    if (RES && res_chunk<PHI>(phi, m_tile, phi_cols, phi_chunks, c0 + c)) {
+                    if (RES && (!PHI || ((S.res_mask[slot] >> c) & 1))) {
                         const uint4 vr = *reinterpret_cast<const uint4 *>(st.sfr + c * ATOM + lane * 16);
                         tmem_st_32x32b_x4(tb + 8 + 4 * c, vr.x, vr.y, vr.z, vr.w);
                     }
@@ -395,6 +414,36 @@ __global__ void __launch_bounds__(THREADS, 1)
                 if (lane == 0)
                     mbar_arrive(&S.sf_ready[sfs]);
             }
+        }
+    } else if (PHI) {
+        // ------------------------------------------------ phi reader (warp 14)
+        // Stage g of this CTA (the producer's running stage index) is k-stage
+        // g mod nks of the CTA's tile number g / nks; its mask has bit c set
+        // when chunk c exists and its phi is 1.
+        const int my_tiles = (int)blockIdx.x < tiles ? (tiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x : 0;
+        const int total = my_tiles * nks;
+        for (int blk = 0; blk * PHI_BLK < total; ++blk) {
+            const int b = blk & 1;
+            if (blk >= 2 && !__all_sync(0xffffffffu, mbar_wait(&S.phi_empty[b], ((blk >> 1) - 1) & 1,
+                                                               kWaitLimitNs, gstat))) {
+                if (lane == 0)
+                    flag_timeout(S, status);
+                break;
+            }
+            for (int e = lane; e < PHI_BLK; e += 32) {
+                const int g = blk * PHI_BLK + e;
+                if (g >= total)
+                    break;
+                const int j = g / nks, ks = g - j * nks;
+                const int m_tile = ((int)blockIdx.x + j * (int)gridDim.x) / n_tiles;
+                uint32_t mask = 0;
+#pragma unroll
+                for (int c = 0; c < 2; ++c)
+                    if (2 * ks + c < kc && __ldg(phi + (int64_t)m_tile * phi_cols + (2 * ks + c) / phi_chunks) != 0)
+                        mask |= 1u << c;
+                S.phi_mask[b][e] = (uint8_t)mask;
+            }
+            mbar_arrive(&S.phi_full[b]);
         }
     }
 
@@ -426,7 +475,7 @@ cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const C
     const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
     const int phi_chunks = a.phi_r_s / 128;
     const int phi_cols = a.phi ? (int)((a.K + a.phi_r_s - 1) / a.phi_r_s) : 0;
-    kern<<<grid, THREADS, kSmemBytes, st>>>(ta, tr, tb, ty, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf,
+    kern<<<grid, PHI ? THREADS + 32 : THREADS, kSmemBytes, st>>>(ta, tr, tb, ty, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf,
                                             (const uint8_t *)a.b_sf, a.phi, phi_chunks, phi_cols, (int)a.M,
                                             (int)a.N, (int)a.K, a.status);
     return cudaGetLastError();

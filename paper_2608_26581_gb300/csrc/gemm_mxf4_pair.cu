@@ -7,7 +7,7 @@
 // k-stage an SM streams 52 KB (codes and scale atoms) for 1,024 cycles of MMA
 // work, 24% less than the 68 KB of a single-CTA 128 x 256 tile.
 //
-// Per CTA (448 threads, one CTA per SM):
+// Per CTA (448 threads, 480 with selective phi; one CTA per SM):
 //   warp 0      TMA producer.  The codes (own A and R rows, own W~ half) are
 //               CTA-pair copies that complete on the EVEN CTA's stage
 //               barrier, which the even CTA's producer arms with the bytes of
@@ -20,6 +20,9 @@
 //               staging -> TMA stores of this CTA's 128 rows
 //   warps 10-13 scale writers: this CTA's scale words from shared memory into
 //               its TMEM with tcgen05.st, one warp per TMEM lane quarter
+//   warp 14     (selective phi only) phi reader: turns the phi bytes of this
+//               CTA's k-stages into per-stage residual masks in shared
+//               memory, in double-buffered blocks of 256 stages
 // TMEM (512 columns per CTA): a 256-column accumulator (this CTA's 128 rows
 // of the tile) and four 32-column scale slots; each CTA holds the scales of
 // its own A / R rows and of ALL 256 W~ rows of the tile (the layout the pair
@@ -37,7 +40,10 @@
 //
 // Residual MMAs of 128-element k-chunks whose phi is 0 for both row tiles of
 // the pair are skipped (the stored residual of a phi = 0 tile is zero, so a
-// pair whose other tile has phi = 1 adds exact zeros).
+// pair whose other tile has phi = 1 adds exact zeros).  The phi bytes come
+// from a warp of their own, a block of stages ahead: a global load issued by
+// the producer waits behind the stage copies already in flight on its SM
+// (thousands of cycles), far more than one stage of MMA work.
 //
 // Every mbarrier wait is bounded (kWaitLimitNs) and also gives up when any
 // CTA has recorded a timeout in the caller's status word.  Neither CTA of a
@@ -67,6 +73,8 @@ constexpr int SF_SLOTS = 4;
 constexpr int EPI_WARPS = 8;
 constexpr int SF_WARPS = 4;
 constexpr int THREADS = 64 + 32 * (EPI_WARPS + SF_WARPS);
+constexpr int PHI_WARP = THREADS / 32;   // the phi reader: one warp beyond THREADS
+constexpr int PHI_BLK = 256;             // stage masks per phi block
 constexpr int YSTAGE = 2048;             // per epilogue warp: 32 rows x 64 bytes of Y
 static_assert(SF_COL0 + SF_SLOTS * SF_SLOT_COLS <= TMEM_COLS, "TMEM budget");
 static_assert(SF_SLOTS >= STAGES, "a scale slot is rewritten only after its stage's MMAs completed");
@@ -91,6 +99,10 @@ struct Smem {
     uint64_t acc_full;            // accumulator complete (both CTAs)
     uint64_t acc_empty;           // (even CTA) both CTAs' epilogue warps drained it
     uint64_t drain;
+    uint64_t phi_full[2];         // the phi reader filled the mask block
+    uint64_t phi_empty[2];        // the producer consumed the mask block
+    uint8_t phi_mask[2][PHI_BLK]; // per stage of a block: bit c, phi of chunk c is 1 in either row tile
+    uint32_t res_mask[STAGES];    // bit c: the residual of 128-element chunk c of the stage applies
     uint32_t tmem_base;
     int32_t abort_flag;
 };
@@ -103,26 +115,8 @@ __device__ __forceinline__ void flag_timeout(Smem &S, int32_t *status)
     atomicExch(status, kDevTimeout);
 }
 
-// Does the residual term of 128-element chunk `chunk` apply to either row
-// tile of the pair?
-template <bool PHI>
-__device__ __forceinline__ bool res_chunk(const uint8_t *phi, int m_pair, int m_tiles, int phi_cols, int phi_chunks,
-                                          int chunk)
-{
-    if (!PHI)
-        return true;
-    bool on = false;
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-        const int mt = 2 * m_pair + r;
-        if (mt < m_tiles)
-            on |= __ldg(phi + (int64_t)mt * phi_cols + chunk / phi_chunks) != 0;
-    }
-    return on;
-}
-
 template <bool RES, bool PHI, bool OUT_BF16>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     gemm_mxf4_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmR,
                           const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmY,
                           const uint8_t *__restrict__ sfa, const uint8_t *__restrict__ sfr,
@@ -156,6 +150,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
         mbar_init(&S.acc_full, 1);
         mbar_init(&S.acc_empty, 2 * EPI_WARPS);
         mbar_init(&S.drain, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&S.phi_full[i], 32);
+            mbar_init(&S.phi_empty[i], 1);
+        }
         // A bounded wait of an earlier CTA or call gave up: skip the work
         // (both CTAs still meet at the cluster barriers).
         S.abort_flag = *gstat;
@@ -199,10 +197,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                         break;
                     }
                     const int c0 = 2 * ks, nch = min(2, kc - c0);
-                    bool res_on = false;
-                    if (RES)
-                        for (int c = 0; c < nch; ++c)
-                            res_on |= res_chunk<PHI>(phi, m_pair, m_tiles, phi_cols, phi_chunks, c0 + c);
+                    // residual chunks of the stage, published to the MMA thread and
+                    // the writers through the stage's barriers
+                    uint32_t mask = RES ? (nch == 2 ? 3u : 1u) : 0u;
+                    if (PHI) {
+                        const int blk = p / PHI_BLK, e = p - blk * PHI_BLK;
+                        if (e == 0 && !mbar_wait(&S.phi_full[blk & 1], (blk >> 1) & 1, kWaitLimitNs, gstat)) {
+                            flag_timeout(S, status);
+                            stop = true;
+                            break;
+                        }
+                        mask = S.phi_mask[blk & 1][e];
+                        if (e == PHI_BLK - 1)
+                            mbar_arrive(&S.phi_empty[blk & 1]);
+                    }
+                    const bool res_on = mask != 0;
+                    S.res_mask[slot] = mask;
                     Stage &st = S.st[slot];
                     // codes: both CTAs' copies complete on the even CTA's barrier
                     if (lead)
@@ -241,7 +251,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             int p = 0, it = 0;
             bool stop = false;
             for (int tile = pair; tile < tiles && !stop; tile += pairs, ++it) {
-                const int m_pair = tile / n_tiles;
                 if (!mbar_wait<true>(&S.acc_empty, (it & 1) ^ 1, kWaitLimitNs, gstat)) {
                     flag_timeout(S, status);
                     break;
@@ -259,6 +268,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                     const int c0 = 2 * ks, nch = min(2, kc - c0);
                     const uint32_t sf = tmem + SF_COL0 + SF_SLOT_COLS * sfs;
                     const Stage &st = S.st[slot];
+                    // without selective phi the mask is fixed: no shared-memory read on the issue path
+                    const uint32_t res_mask = PHI ? S.res_mask[slot] : (RES ? (nch == 2 ? 3u : 1u) : 0u);
                     const uint32_t a0 = smem_u32(st.a), r0 = smem_u32(st.r), b0 = smem_u32(st.b);
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
@@ -269,7 +280,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                         const uint64_t bd = sdesc_k_sw128(b0 + 32 * j);
                         const uint32_t sfb_t = sf + 16 + 8 * c;
                         tc_mma_mxf4_pair(tmem, sdesc_k_sw128(a0 + 32 * j), bd, id, sf + 4 * c, sfb_t, (ks | j) != 0);
-                        if (RES && res_chunk<PHI>(phi, m_pair, m_tiles, phi_cols, phi_chunks, c0 + c))
+                        if (RES && ((res_mask >> c) & 1))
                             tc_mma_mxf4_pair(tmem, sdesc_k_sw128(r0 + 32 * j), bd, id, sf + 8 + 4 * c, sfb_t, 1);
                     }
                     tc_commit_pair_mc(&S.empty[slot], 0x3);
@@ -393,7 +404,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
         }
         if (lane == 0)
             bulk_wait_group<0>(); // every TMA store of this warp has completed
-    } else {
+    } else if (warp < PHI_WARP) {
         // ------------------------------------------------ scale writers (warps 10..13)
         // Warp quarter q writes TMEM lanes 32q..32q+31; every quarter holds
         // the same words: column j of lane i carries the four scales of row
@@ -428,7 +439,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                     const uint4 vb0 = *reinterpret_cast<const uint4 *>(st.sfb + c * ATOM + lane * 16);
                     const uint4 vb1 = b1_in ? *reinterpret_cast<const uint4 *>(st.sfb + (2 + c) * ATOM + lane * 16) : z;
                     tmem_st_32x32b_x4(tb + 4 * c, va.x, va.y, va.z, va.w);
-                    if (RES && res_chunk<PHI>(phi, m_pair, m_tiles, phi_cols, phi_chunks, c0 + c)) {
+                    if (RES && (!PHI || ((S.res_mask[slot] >> c) & 1))) {
                         const uint4 vr = rows_in ? *reinterpret_cast<const uint4 *>(st.sfr + c * ATOM + lane * 16) : z;
                         tmem_st_32x32b_x4(tb + 8 + 4 * c, vr.x, vr.y, vr.z, vr.w);
                     }
@@ -445,6 +456,44 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                         mbar_arrive_remote_relaxed(sf_ready_lead + 8 * sfs);
                 }
             }
+        }
+    } else if (PHI) {
+        // ------------------------------------------------ phi reader (warp 14)
+        // Stage g of this CTA (the producer's running stage index) is k-stage
+        // g mod nks of the pair's tile number g / nks; its mask has bit c set
+        // when chunk c exists and either row tile of the pair has phi = 1 there.
+        const int my_tiles = pair < tiles ? (tiles - pair + pairs - 1) / pairs : 0;
+        const int total = skip ? 0 : my_tiles * nks;
+        for (int blk = 0; blk * PHI_BLK < total; ++blk) {
+            const int b = blk & 1;
+            if (blk >= 2 && !__all_sync(0xffffffffu, mbar_wait(&S.phi_empty[b], ((blk >> 1) - 1) & 1,
+                                                               kWaitLimitNs, gstat))) {
+                if (lane == 0)
+                    flag_timeout(S, status);
+                break;
+            }
+            for (int e = lane; e < PHI_BLK; e += 32) {
+                const int g = blk * PHI_BLK + e;
+                if (g >= total)
+                    break;
+                const int j = g / nks, ks = g - j * nks;
+                const int m_pair = (pair + j * pairs) / n_tiles;
+                uint32_t mask = 0;
+#pragma unroll
+                for (int c = 0; c < 2; ++c) {
+                    if (2 * ks + c >= kc)
+                        break;
+                    const int col = (2 * ks + c) / phi_chunks;
+#pragma unroll
+                    for (int r = 0; r < 2; ++r) {
+                        const int mt = 2 * m_pair + r;
+                        if (mt < m_tiles && __ldg(phi + (int64_t)mt * phi_cols + col) != 0)
+                            mask |= 1u << c;
+                    }
+                }
+                S.phi_mask[b][e] = (uint8_t)mask;
+            }
+            mbar_arrive(&S.phi_full[b]);
         }
     }
 
@@ -470,7 +519,7 @@ cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const C
     if (max_pairs == 0) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2 * (num_sms() / 2));
-        cfg.blockDim = dim3(THREADS);
+        cfg.blockDim = dim3(PHI ? THREADS + 32 : THREADS);
         cfg.dynamicSmemBytes = kSmemBytes;
         int n = 0;
         e = cudaOccupancyMaxActiveClusters(&n, kern, &cfg);
@@ -482,9 +531,9 @@ cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const C
     const int grid = 2 * (int)(tiles < max_pairs ? tiles : max_pairs);
     const int phi_chunks = a.phi_r_s / 128;
     const int phi_cols = a.phi ? (int)((a.K + a.phi_r_s - 1) / a.phi_r_s) : 0;
-    kern<<<grid, THREADS, kSmemBytes, st>>>(ta, tr, tb, ty, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf,
-                                            (const uint8_t *)a.b_sf, a.phi, phi_chunks, phi_cols, (int)a.M,
-                                            (int)a.N, (int)a.K, a.status);
+    kern<<<grid, PHI ? THREADS + 32 : THREADS, kSmemBytes, st>>>(
+        ta, tr, tb, ty, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf, (const uint8_t *)a.b_sf, a.phi, phi_chunks,
+        phi_cols, (int)a.M, (int)a.N, (int)a.K, a.status);
     return cudaGetLastError();
 }
 

@@ -78,15 +78,37 @@ def test_plain_w4a4_without_residual(orc):
     check_y(y, _ref(orc, xq, None, wq, M, K, N))
 
 
-@pytest.mark.parametrize("r_s,tau", [(256, 30.0), (128, 20.0), (512, 1e30), (256, 0.0)])
-def test_phi_amax_skips_residual_tiles(orc, r_s, tau):
-    M, K, N = 384, 1024, 256
+@pytest.mark.parametrize("M,K,r_s,tau", [(384, 1024, 256, 30.0), (384, 1024, 128, 20.0), (384, 1024, 512, 1e30),
+                                         (384, 1024, 256, 0.0), (100, 1152, 128, 20.0), (300, 1152, 256, 20.0)])
+def test_phi_amax_skips_residual_tiles(orc, M, K, r_s, tau):
+    N = 256
     xb = make_activation(ActSpec(M, K, "normal", chan_count=3, chan_scale=64.0, seed=9))
     wb = make_weight(K, N, seed=9)
     xq, xr, wq, y, phi = _run(xb, wb, mode=rfq.RFQ_FALLBACK_AMAX, tau=tau, r_s=r_s, use_phi=True)
     check_y(y, _ref(orc, xq, xr, wq, M, K, N))
     q = orc.quantize_act(xb, orc.FMT_MXFP4, orc.PHI_AMAX, tau, 128, r_s)
     assert np.array_equal(phi.cpu().numpy().reshape(q["phi"].shape), q["phi"])
+
+
+@pytest.mark.parametrize("M", [100, 256])
+def test_phi_amax_many_stage_blocks(orc, M):
+    """K = 135168: one output tile of 528 k-stages, so its CTA(s) walk more
+    than two blocks of 256 per-stage residual masks; about half the 128 x 256
+    tiles have phi = 1.  Y is checked on sampled rows."""
+    K, N, r_s, tau = 135168, 256, 256, 30.0
+    xb = make_activation(ActSpec(M, K, "normal", chan_count=360, chan_scale=64.0, seed=11))
+    wb = make_weight(K, N, seed=11)
+    xq, xr, wq, y, phi = _run(xb, wb, mode=rfq.RFQ_FALLBACK_AMAX, tau=tau, r_s=r_s, use_phi=True)
+    q = orc.quantize_act(xb, orc.FMT_MXFP4, orc.PHI_AMAX, tau, 128, r_s)
+    assert np.array_equal(phi.cpu().numpy().reshape(q["phi"].shape), q["phi"])
+    assert 0.2 < q["phi"].mean() < 0.8
+    rwc, rws = orc.quantize_weight(wb)
+    wc, ws = qtensor_host(wq)
+    assert np.array_equal(wc, rwc) and np.array_equal(ws, rws)
+    rows = np.unique(np.concatenate([np.random.default_rng(1).choice(M, 10, replace=False), [0, M - 1]]))
+    ref = orc.linear(0, q["main_codes"][rows], q["main_scales"][rows], q["res_codes"][rows], q["res_scales"][rows],
+                     rwc, rws, len(rows), K, N)
+    check_y(y[rows], ref)
 
 
 def test_bf16_output(orc):
