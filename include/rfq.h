@@ -156,6 +156,10 @@ RFQ_API size_t rfq_linear_workspace_bytes(void);
  * (plain W4A4); phi: device bytes [ceil(M/128)][K/r_s] selecting the
  * residual k-tiles per 128-row tile, or NULL (= all ones); phi_r_s: the
  * column tile r_s of phi (a multiple of 128; ignored when phi is NULL).
+ * The residual of every phi = 0 tile must be stored as zero, as
+ * rfq_quantize_act writes it: phi only lets the GEMM skip residual loads and
+ * products, at its own granularity (it may still include a phi = 0 tile that
+ * shares a 256-row or 256-column block with a phi = 1 one).
  * wq: [N x K] weight.  MXFP4: every operand MXFP4 with RFQ_SCALE_MMA,
  * K % 128 == 0.  HiF4 (Sec. 3.3): wq is the exact bf16 expansion of the HiF4
  * weight (RFQ_FMT_BF16, from rfq_dequant), K % 64 == 0, phi_r_s a multiple

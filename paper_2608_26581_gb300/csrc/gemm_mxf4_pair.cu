@@ -20,9 +20,9 @@
 //               staging -> TMA stores of this CTA's 128 rows
 //   warps 10-13 scale writers: this CTA's scale words from shared memory into
 //               its TMEM with tcgen05.st, one warp per TMEM lane quarter
-//   warp 14     (selective phi only) phi reader: turns the phi bytes of this
-//               CTA's k-stages into per-stage residual masks in shared
-//               memory, in double-buffered blocks of 256 stages
+//   warp 14     (selective phi only) phi reader: one record per output tile
+//               of this CTA (double-buffered) with a bit per k-stage, set
+//               when the stage needs its residual, and their count
 // TMEM (512 columns per CTA): a 256-column accumulator (this CTA's 128 rows
 // of the tile) and four 32-column scale slots; each CTA holds the scales of
 // its own A / R rows and of ALL 256 W~ rows of the tile (the layout the pair
@@ -38,12 +38,21 @@
 // and orders its MMAs after them with tcgen05.fence.  A release arrive at
 // cluster scope would stall the arriving warp for hundreds of cycles.
 //
-// Residual MMAs of 128-element k-chunks whose phi is 0 for both row tiles of
-// the pair are skipped (the stored residual of a phi = 0 tile is zero, so a
-// pair whose other tile has phi = 1 adds exact zeros).  The phi bytes come
-// from a warp of their own, a block of stages ahead: a global load issued by
-// the producer waits behind the stage copies already in flight on its SM
-// (thousands of cycles), far more than one stage of MMA work.
+// Selective phi: the residual loads and MMAs of a 256-element k-stage are
+// skipped when phi is 0 for both of its 128-element chunks in both row tiles
+// of the pair (the stored residual of a phi = 0 tile is zero, so including a
+// phi = 0 chunk or row tile beside a phi = 1 one adds exact zeros).  Each
+// tile's stages run in a data-dependent ORDER -- the stages with a residual
+// first, then those without, each in k order, an odd last chunk last -- so
+// the MMA thread and the scale writers run two loops with compile-time
+// residual masks and data-dependent trip counts (the sum over k does not
+// depend on its order).  A branch on a per-stage mask value in the MMA
+// thread slowed its MMA issue by ~150 cycles per stage; the loop bounds cost
+// nothing measurable.  Only the producer follows the order, from the bits of
+// the tile's record; it publishes the tile's residual-stage count with every
+// stage.  The records come from a warp of their own, a tile ahead: a global
+// load issued by the producer waits behind the stage copies in flight on its
+// SM (thousands of cycles).
 //
 // Every mbarrier wait is bounded (kWaitLimitNs) and also gives up when any
 // CTA has recorded a timeout in the caller's status word.  Neither CTA of a
@@ -74,7 +83,7 @@ constexpr int EPI_WARPS = 8;
 constexpr int SF_WARPS = 4;
 constexpr int THREADS = 64 + 32 * (EPI_WARPS + SF_WARPS);
 constexpr int PHI_WARP = THREADS / 32;   // the phi reader: one warp beyond THREADS
-constexpr int PHI_BLK = 256;             // stage masks per phi block
+constexpr int REC_WORDS = 64;            // phi record: up to 2048 full k-stages (K <= 524288)
 constexpr int YSTAGE = 2048;             // per epilogue warp: 32 rows x 64 bytes of Y
 static_assert(SF_COL0 + SF_SLOTS * SF_SLOT_COLS <= TMEM_COLS, "TMEM budget");
 static_assert(SF_SLOTS >= STAGES, "a scale slot is rewritten only after its stage's MMAs completed");
@@ -89,6 +98,15 @@ struct alignas(1024) Stage {
 };
 static_assert(sizeof(Stage) % 1024 == 0, "stages keep the 1024-byte swizzle alignment");
 
+// Selective phi, one output tile: bit ks of bits (ks < K / 256, the full
+// k-stages) set when phi is 1 for either 128-element chunk of stage ks in
+// either row tile; info = the number of set bits | (phi of the odd last
+// chunk, when K / 128 is odd) << 31.
+struct PhiRec {
+    uint32_t bits[REC_WORDS];
+    uint32_t info;
+};
+
 struct Smem {
     Stage st[STAGES];
     alignas(1024) uint8_t ystage[EPI_WARPS * YSTAGE];
@@ -99,10 +117,10 @@ struct Smem {
     uint64_t acc_full;            // accumulator complete (both CTAs)
     uint64_t acc_empty;           // (even CTA) both CTAs' epilogue warps drained it
     uint64_t drain;
-    uint64_t phi_full[2];         // the phi reader filled the mask block
-    uint64_t phi_empty[2];        // the producer consumed the mask block
-    uint8_t phi_mask[2][PHI_BLK]; // per stage of a block: bit c, phi of chunk c is 1 in either row tile
-    uint32_t res_mask[STAGES];    // bit c: the residual of 128-element chunk c of the stage applies
+    uint64_t phi_full[2];         // the phi reader filled the record
+    uint64_t phi_empty[2];        // the producer consumed the record
+    PhiRec rec[2];
+    uint32_t stage_info[STAGES];  // the tile's residual-stage count | odd last chunk's residual << 31
     uint32_t tmem_base;
     int32_t abort_flag;
 };
@@ -114,6 +132,15 @@ __device__ __forceinline__ void flag_timeout(Smem &S, int32_t *status)
     S.abort_flag = 1;
     atomicExch(status, kDevTimeout);
 }
+
+template <bool B>
+struct Bool {
+    static constexpr bool value = B;
+};
+template <uint32_t V>
+struct Mask {
+    static constexpr uint32_t value = V;
+};
 
 template <bool RES, bool PHI, bool OUT_BF16>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
@@ -132,6 +159,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
 
     const int kc = K >> 7;                  // 128-element chunks
     const int nks = (kc + 1) >> 1;          // 256-element stages (the last may hold one chunk)
+    const int nf = kc >> 1;                 // stages with two chunks
     const int n_tiles = (N + BN - 1) / BN;
     const int m_tiles = (M + BM - 1) / BM;  // 128-row tiles: scale atoms and phi rows
     const int m_pairs = (M + 2 * BM - 1) / (2 * BM);
@@ -181,50 +209,37 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
         // ------------------------------------------------ TMA producer (both CTAs)
         if (lane == 0 && !skip) {
             const uint32_t full0 = mapa_shared(smem_u32(&S.full[0]), 0);   // the even CTA's barriers
-            int p = 0;
+            int p = 0, it = 0;
             bool stop = false;
-            for (int tile = pair; tile < tiles && !stop; tile += pairs) {
+            for (int tile = pair; tile < tiles && !stop; tile += pairs, ++it) {
                 const int m_pair = tile / n_tiles, n_tile = tile - m_pair * n_tiles;
                 const int m_tile = 2 * m_pair + (int)rank;
                 const bool rows_in = m_tile < m_tiles;
                 const int atom0 = 2 * n_tile;
                 const int nb = atom0 + 1 < n_atoms ? 2 : 1;
-                for (int ks = 0; ks < nks; ++ks, ++p) {
+                // one k-stage: wait for its ring slot, publish the tile's info,
+                // issue the copies (codes: both CTAs' copies complete on the even
+                // CTA's barrier; scale atoms: this CTA's own barrier)
+                auto produce = [&](int ks, uint32_t info, auto res_t) {
+                    constexpr bool res_on = decltype(res_t)::value;
                     const int slot = p % STAGES;
                     if (!mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, kWaitLimitNs, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
-                        break;
+                        return;
                     }
                     const int c0 = 2 * ks, nch = min(2, kc - c0);
-                    // residual chunks of the stage, published to the MMA thread and
-                    // the writers through the stage's barriers
-                    uint32_t mask = RES ? (nch == 2 ? 3u : 1u) : 0u;
-                    if (PHI) {
-                        const int blk = p / PHI_BLK, e = p - blk * PHI_BLK;
-                        if (e == 0 && !mbar_wait(&S.phi_full[blk & 1], (blk >> 1) & 1, kWaitLimitNs, gstat)) {
-                            flag_timeout(S, status);
-                            stop = true;
-                            break;
-                        }
-                        mask = S.phi_mask[blk & 1][e];
-                        if (e == PHI_BLK - 1)
-                            mbar_arrive(&S.phi_empty[blk & 1]);
-                    }
-                    const bool res_on = mask != 0;
-                    S.res_mask[slot] = mask;
+                    S.stage_info[slot] = info;
                     Stage &st = S.st[slot];
-                    // codes: both CTAs' copies complete on the even CTA's barrier
+                    const uint32_t bar = full0 + 8 * slot;
+                    const uint32_t sfbytes = (uint32_t)nch * ATOM;
+                    uint64_t *sbar = &S.sf_full[slot];
                     if (lead)
                         mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES + B_BYTES + (res_on ? A_BYTES : 0)));
-                    const uint32_t bar = full0 + 8 * slot;
                     tma_load_2d_pair(st.a, &tmA, bar, c0 * 64, m_tile * BM);
                     if (res_on)
                         tma_load_2d_pair(st.r, &tmR, bar, c0 * 64, m_tile * BM);
                     tma_load_2d_pair(st.b, &tmB, bar, c0 * 64, n_tile * BN + (int)rank * BN_HALF);
-                    // scale atoms: this CTA's own barrier
-                    const uint32_t sfbytes = (uint32_t)nch * ATOM;
-                    uint64_t *sbar = &S.sf_full[slot];
                     mbar_arrive_expect_tx(sbar, nb * sfbytes + (rows_in ? (res_on ? 2 : 1) * sfbytes : 0));
                     if (rows_in) {
                         bulk_load(st.sfa, sfa + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, sbar);
@@ -234,6 +249,45 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     for (int h = 0; h < nb; ++h)
                         bulk_load(st.sfb + h * 2 * ATOM, sfb + ((int64_t)(atom0 + h) * kc + c0) * ATOM, sfbytes,
                                   sbar);
+                    ++p;
+                };
+                if constexpr (!PHI) {
+                    for (int ks = 0; ks < nks && !stop; ++ks)
+                        produce(ks, 0u, Bool<RES>{});
+                } else {
+                    const int r = it & 1;
+                    if (!mbar_wait(&S.phi_full[r], (it >> 1) & 1, kWaitLimitNs, gstat)) {
+                        flag_timeout(S, status);
+                        stop = true;
+                        break;
+                    }
+                    const PhiRec &rec = S.rec[r];
+                    const uint32_t info = rec.info;
+                    // stages with a residual, then the others, each in k order
+                    for (int w = 0; 32 * w < nf && !stop; ++w) {
+                        uint32_t x = rec.bits[w];
+                        while (x != 0 && !stop) {
+                            const int b = __ffs(x) - 1;
+                            x &= x - 1;
+                            produce(32 * w + b, info, Bool<true>{});
+                        }
+                    }
+                    for (int w = 0; 32 * w < nf && !stop; ++w) {
+                        const int left = nf - 32 * w;
+                        uint32_t x = ~rec.bits[w] & (left >= 32 ? 0xffffffffu : (1u << left) - 1u);
+                        while (x != 0 && !stop) {
+                            const int b = __ffs(x) - 1;
+                            x &= x - 1;
+                            produce(32 * w + b, info, Bool<false>{});
+                        }
+                    }
+                    if (nf < nks && !stop) {   // the odd last chunk
+                        if (info >> 31)
+                            produce(nf, info, Bool<true>{});
+                        else
+                            produce(nf, info, Bool<false>{});
+                    }
+                    mbar_arrive(&S.phi_empty[r]);
                 }
             }
             if (stop || S.abort_flag)
@@ -256,20 +310,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     break;
                 }
                 tc_fence_after();
-                for (int ks = 0; ks < nks; ++ks, ++p) {
+                // the MMAs of the stage at position pos of the tile, with residual
+                // mask rm (bit c: chunk c's residual product) known at compile time
+                auto mma_stage = [&](int pos, int nch, auto rm_t) {
+                    constexpr uint32_t rm = decltype(rm_t)::value;
                     const int slot = p % STAGES, sfs = p % SF_SLOTS;
                     if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat) ||
                         !mbar_wait<true>(&S.sf_ready[sfs], (p / SF_SLOTS) & 1, kWaitLimitNs, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
-                        break;
+                        return;
                     }
                     tc_fence_after();
-                    const int c0 = 2 * ks, nch = min(2, kc - c0);
                     const uint32_t sf = tmem + SF_COL0 + SF_SLOT_COLS * sfs;
                     const Stage &st = S.st[slot];
-                    // without selective phi the mask is fixed: no shared-memory read on the issue path
-                    const uint32_t res_mask = PHI ? S.res_mask[slot] : (RES ? (nch == 2 ? 3u : 1u) : 0u);
                     const uint32_t a0 = smem_u32(st.a), r0 = smem_u32(st.r), b0 = smem_u32(st.b);
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
@@ -279,11 +333,35 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                         const uint32_t id = idesc_mxf4(2 * BM, BN, 2 * (j & 1), 2 * (j & 1));
                         const uint64_t bd = sdesc_k_sw128(b0 + 32 * j);
                         const uint32_t sfb_t = sf + 16 + 8 * c;
-                        tc_mma_mxf4_pair(tmem, sdesc_k_sw128(a0 + 32 * j), bd, id, sf + 4 * c, sfb_t, (ks | j) != 0);
-                        if (RES && ((res_mask >> c) & 1))
+                        tc_mma_mxf4_pair(tmem, sdesc_k_sw128(a0 + 32 * j), bd, id, sf + 4 * c, sfb_t, (pos | j) != 0);
+                        if ((rm >> c) & 1)
                             tc_mma_mxf4_pair(tmem, sdesc_k_sw128(r0 + 32 * j), bd, id, sf + 8 + 4 * c, sfb_t, 1);
                     }
                     tc_commit_pair_mc(&S.empty[slot], 0x3);
+                    ++p;
+                };
+                if constexpr (!PHI) {
+                    for (int ks = 0; ks < nks && !stop; ++ks)
+                        mma_stage(ks, min(2, kc - 2 * ks), Mask<RES ? 3u : 0u>{});
+                } else {
+                    // the tile's residual-stage count arrives with its first stage
+                    if (!mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs, gstat)) {
+                        flag_timeout(S, status);
+                        break;
+                    }
+                    const uint32_t info = S.stage_info[p % STAGES];
+                    const int n_res = (int)(info & 0x7fffffffu);
+                    int pos = 0;
+                    for (; pos < n_res && !stop; ++pos)
+                        mma_stage(pos, 2, Mask<3u>{});
+                    for (; pos < nf && !stop; ++pos)
+                        mma_stage(pos, 2, Mask<0u>{});
+                    if (nf < nks && !stop) {
+                        if (info >> 31)
+                            mma_stage(pos, 1, Mask<1u>{});
+                        else
+                            mma_stage(pos, 1, Mask<0u>{});
+                    }
                 }
                 if (!stop)
                     tc_commit_pair_mc(&S.acc_full, 0x3);
@@ -417,17 +495,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
             const int m_pair = tile / n_tiles, n_tile = tile - m_pair * n_tiles;
             const bool rows_in = 2 * m_pair + (int)rank < m_tiles;
             const bool b1_in = 2 * n_tile + 1 < n_atoms;
-            for (int ks = 0; ks < nks; ++ks, ++p) {
+            // the scale words of the next stage (in the producer's order), with
+            // the residual mask rm known at compile time
+            auto write_stage = [&](int nch, auto rm_t) {
+                constexpr uint32_t rm = decltype(rm_t)::value;
                 const int slot = p % STAGES, sfs = p % SF_SLOTS;
                 // warp-uniform outcome: the tcgen05 stores below need the whole warp
                 if (!__all_sync(0xffffffffu, mbar_wait(&S.sf_full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat))) {
                     if (lane == 0)
                         flag_timeout(S, status);
                     stop = true;
-                    break;
+                    return;
                 }
                 tc_fence_after();
-                const int c0 = 2 * ks, nch = min(2, kc - c0);
                 const Stage &st = S.st[slot];
                 const uint32_t tb = tmem + ((uint32_t)(q * 32) << 16) + SF_COL0 + SF_SLOT_COLS * sfs;
                 const uint4 z = make_uint4(0, 0, 0, 0);
@@ -439,7 +519,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     const uint4 vb0 = *reinterpret_cast<const uint4 *>(st.sfb + c * ATOM + lane * 16);
                     const uint4 vb1 = b1_in ? *reinterpret_cast<const uint4 *>(st.sfb + (2 + c) * ATOM + lane * 16) : z;
                     tmem_st_32x32b_x4(tb + 4 * c, va.x, va.y, va.z, va.w);
-                    if (RES && (!PHI || ((S.res_mask[slot] >> c) & 1))) {
+                    if ((rm >> c) & 1) {
                         const uint4 vr = rows_in ? *reinterpret_cast<const uint4 *>(st.sfr + c * ATOM + lane * 16) : z;
                         tmem_st_32x32b_x4(tb + 8 + 4 * c, vr.x, vr.y, vr.z, vr.w);
                     }
@@ -455,45 +535,73 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     else
                         mbar_arrive_remote_relaxed(sf_ready_lead + 8 * sfs);
                 }
+                ++p;
+            };
+            if constexpr (!PHI) {
+                for (int ks = 0; ks < nks && !stop; ++ks)
+                    write_stage(min(2, kc - 2 * ks), Mask<RES ? 3u : 0u>{});
+            } else {
+                // the tile's residual-stage count arrives with its first stage
+                if (!__all_sync(0xffffffffu, mbar_wait(&S.sf_full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs, gstat))) {
+                    if (lane == 0)
+                        flag_timeout(S, status);
+                    break;
+                }
+                const uint32_t info = S.stage_info[p % STAGES];
+                const int n_res = (int)(info & 0x7fffffffu);
+                int pos = 0;
+                for (; pos < n_res && !stop; ++pos)
+                    write_stage(2, Mask<3u>{});
+                for (; pos < nf && !stop; ++pos)
+                    write_stage(2, Mask<0u>{});
+                if (nf < nks && !stop) {
+                    if (info >> 31)
+                        write_stage(1, Mask<1u>{});
+                    else
+                        write_stage(1, Mask<0u>{});
+                }
             }
         }
     } else if (PHI) {
         // ------------------------------------------------ phi reader (warp 14)
-        // Stage g of this CTA (the producer's running stage index) is k-stage
-        // g mod nks of the pair's tile number g / nks; its mask has bit c set
-        // when chunk c exists and either row tile of the pair has phi = 1 there.
+        // Record of the CTA's j-th tile: chunk c of the pair's row tile
+        // 2 m_pair + r needs its residual when phi[2 m_pair + r][c / phi_chunks]
+        // is non-zero.
         const int my_tiles = pair < tiles ? (tiles - pair + pairs - 1) / pairs : 0;
-        const int total = skip ? 0 : my_tiles * nks;
-        for (int blk = 0; blk * PHI_BLK < total; ++blk) {
-            const int b = blk & 1;
-            if (blk >= 2 && !__all_sync(0xffffffffu, mbar_wait(&S.phi_empty[b], ((blk >> 1) - 1) & 1,
-                                                               kWaitLimitNs, gstat))) {
+        auto chunk_on = [&](int m_pair, int c) {
+            const int col = c / phi_chunks;
+            bool on = false;
+#pragma unroll
+            for (int r = 0; r < 2; ++r) {
+                const int mt = 2 * m_pair + r;
+                if (mt < m_tiles && __ldg(phi + (int64_t)mt * phi_cols + col) != 0)
+                    on = true;
+            }
+            return on;
+        };
+        for (int j = 0; j < (skip ? 0 : my_tiles); ++j) {
+            const int r = j & 1;
+            if (j >= 2 && !__all_sync(0xffffffffu, mbar_wait(&S.phi_empty[r], ((j >> 1) - 1) & 1,
+                                                             kWaitLimitNs, gstat))) {
                 if (lane == 0)
                     flag_timeout(S, status);
                 break;
             }
-            for (int e = lane; e < PHI_BLK; e += 32) {
-                const int g = blk * PHI_BLK + e;
-                if (g >= total)
-                    break;
-                const int j = g / nks, ks = g - j * nks;
-                const int m_pair = (pair + j * pairs) / n_tiles;
-                uint32_t mask = 0;
-#pragma unroll
-                for (int c = 0; c < 2; ++c) {
-                    if (2 * ks + c >= kc)
-                        break;
-                    const int col = (2 * ks + c) / phi_chunks;
-#pragma unroll
-                    for (int r = 0; r < 2; ++r) {
-                        const int mt = 2 * m_pair + r;
-                        if (mt < m_tiles && __ldg(phi + (int64_t)mt * phi_cols + col) != 0)
-                            mask |= 1u << c;
-                    }
-                }
-                S.phi_mask[b][e] = (uint8_t)mask;
+            const int m_pair = (pair + j * pairs) / n_tiles;
+            PhiRec &rec = S.rec[r];
+            uint32_t n_res = 0;
+            for (int w = 0; 32 * w < nf; ++w) {
+                const int ks = 32 * w + lane;
+                const bool on = ks < nf && (chunk_on(m_pair, 2 * ks) || chunk_on(m_pair, 2 * ks + 1));
+                const uint32_t word = __ballot_sync(0xffffffffu, on);
+                if (lane == 0)
+                    rec.bits[w] = word;
+                n_res += __popc(word);
             }
-            mbar_arrive(&S.phi_full[b]);
+            const uint32_t tail = nf < nks && chunk_on(m_pair, 2 * nf) ? 1u : 0u;
+            if (lane == 0)
+                rec.info = n_res | tail << 31;
+            mbar_arrive(&S.phi_full[r]);
         }
     }
 
@@ -556,7 +664,10 @@ cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
     const uint64_t yrow = (uint64_t)a.N * (a.out_bf16 ? 2 : 4);
     if (!encode_tmap_2d_u8(&ty, a.y, yrow, (uint64_t)a.M, yrow, 64, 32, 64))
         return cudaErrorInvalidValue;
-    const bool res = a.r_codes != nullptr, phi = res && a.phi != nullptr;
+    // Beyond REC_WORDS * 32 full k-stages the record does not fit: every
+    // residual product is then issued (exact: phi = 0 residuals are zero).
+    const bool res = a.r_codes != nullptr;
+    const bool phi = res && a.phi != nullptr && a.K / 256 <= REC_WORDS * 32;
 #define RFQ_GV(R, P, O) return launch_variant<R, P, O>(ta, tr, tb, ty, a, st)
     if (!res) {
         if (a.out_bf16) RFQ_GV(false, false, true);
