@@ -16,6 +16,13 @@
 // TMEM accumulator.  The accumulator is double-buffered (2 x 256 columns; no
 // scale columns are needed), so four epilogue warps drain tile t while the
 // MMAs of tile t+1 run.  Waits are bounded as in the MXFP4 GEMM.
+//
+// Selective phi: stages of phi = 0 skip the residual load and MMAs.  As in
+// the CTA-pair MXFP4 GEMM, an extra warp writes one record per output tile (a
+// bit per k-stage, set when phi = 1, and their count), the producer issues
+// the residual stages first and publishes the count with every stage, and
+// the MMA thread runs two loops with compile-time residual flags: a branch
+// on a per-stage flag in the MMA thread slows its MMA issue.
 #include <cuda_bf16.h>
 #include <cstdint>
 #include <type_traits>
@@ -37,6 +44,15 @@ constexpr int B16_BYTES = BN * BK * 2;        // 32 KB bf16 tile
 constexpr int CONV_WARPS = 8;
 constexpr int EPI_WARPS = 4;
 constexpr int THREADS = 64 + 32 * EPI_WARPS + 32 * CONV_WARPS;
+constexpr int PHI_WARP = THREADS / 32;        // the phi reader: one warp beyond THREADS
+constexpr int REC_WORDS = 64;                 // phi record: up to 2048 k-stages (K <= 131072)
+
+// Selective phi, one output tile: bit ks of bits set when the residual of
+// k-stage ks applies; count = the number of set bits.
+struct PhiRec {
+    uint32_t bits[REC_WORDS];
+    uint32_t count;
+};
 constexpr int TMEM_COLS = 512;
 
 struct alignas(1024) Stage {
@@ -68,7 +84,10 @@ struct Smem {
     uint64_t acc_full[2];
     uint64_t acc_empty[2];
     uint64_t drain;
-    uint32_t res_on[STAGES];   // the residual of the stage applies (from phi, published by the producer)
+    uint64_t phi_full[2];      // the phi reader filled the record
+    uint64_t phi_empty[2];     // the producer consumed the record
+    PhiRec rec[2];
+    uint32_t stage_info[STAGES]; // the tile's residual-stage count | (this stage's residual applies) << 31
     uint32_t tmem_base;
     int32_t abort_flag;
     int32_t issued;
@@ -110,8 +129,13 @@ __device__ __forceinline__ uint4 hif4_group_to_bf16(uint32_t cw, uint32_t meta, 
 
 // CONV: the activation operands are HiF4 codes + metadata expanded in the
 // kernel; otherwise they are bf16 expansions loaded by TMA like W~.
+template <bool B>
+struct Bool {
+    static constexpr bool value = B;
+};
+
 template <bool CONV, bool RES, bool PHI, bool OUT_BF16>
-__global__ void __launch_bounds__(THREADS, 1)
+__global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     gemm_hif4_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmR,
                      const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmY,
                      const uint32_t *__restrict__ ameta,
@@ -148,6 +172,10 @@ __global__ void __launch_bounds__(THREADS, 1)
             mbar_init(&S.acc_empty[b], EPI_WARPS);
         }
         mbar_init(&S.drain, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&S.phi_full[i], 32);
+            mbar_init(&S.phi_empty[i], 1);
+        }
         S.issued = 0;
         fence_mbar_init();
     }
@@ -171,42 +199,34 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (warp == 0) {
         // ------------------------------------------------ TMA producer
         if (lane == 0) {
-            int p = 0;
+            int p = 0, it = 0;
             bool stop = false;
-            // phi byte of the next k-stage: loaded one stage ahead and tested
-            // only after the next wait, so its global-memory latency overlaps
-            // that wait
-            uint32_t ph = 0;
-            if (PHI && (int)blockIdx.x < tiles)
-                ph = __ldg(phi + (int64_t)(blockIdx.x / n_tiles) * phi_cols);
-            for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x) {
+            for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x, ++it) {
                 const int m_tile = tile / n_tiles, n_tile = tile - m_tile * n_tiles;
-                for (int ks = 0; ks < nks; ++ks, ++p) {
+                // one k-stage: wait for its ring slot, publish the tile's info and
+                // the stage's residual flag, issue the copies
+                auto produce = [&](int ks, uint32_t count, auto res_t) {
+                    constexpr bool ron = decltype(res_t)::value;
                     const int slot = p % STAGES;
                     if (!mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, kWaitLimitNs, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
-                        break;
+                        return;
                     }
-                    // published to the MMA thread and the converters through the
-                    // stage's barrier
-                    const bool ron = RES && (!PHI || ph != 0);
-                    S.res_on[slot] = ron;
+                    S.stage_info[slot] = count | (ron ? 1u << 31 : 0u);
                     auto &st = S.st[slot];
                     uint64_t *bar = &S.full[slot];
-                    if (CONV) {
+                    if constexpr (CONV) {
                         uint32_t bytes = B16_BYTES + CODE_BYTES + META_BYTES;
                         if (ron)
                             bytes += CODE_BYTES + META_BYTES;
                         mbar_arrive_expect_tx(bar, bytes);
                         tma_load_2d(st.b, &tmB, bar, ks * BK * 2, n_tile * BN);
-                        if constexpr (CONV) {
-                            tma_load_2d(st.acode, &tmA, bar, ks * BK / 2, m_tile * BM);
-                            bulk_load(st.ameta, ameta + ks * mpad + (int64_t)m_tile * BM, META_BYTES, bar);
-                            if (ron) {
-                                tma_load_2d(st.rcode, &tmR, bar, ks * BK / 2, m_tile * BM);
-                                bulk_load(st.rmeta, rmeta + ks * mpad + (int64_t)m_tile * BM, META_BYTES, bar);
-                            }
+                        tma_load_2d(st.acode, &tmA, bar, ks * BK / 2, m_tile * BM);
+                        bulk_load(st.ameta, ameta + ks * mpad + (int64_t)m_tile * BM, META_BYTES, bar);
+                        if (ron) {
+                            tma_load_2d(st.rcode, &tmR, bar, ks * BK / 2, m_tile * BM);
+                            bulk_load(st.rmeta, rmeta + ks * mpad + (int64_t)m_tile * BM, META_BYTES, bar);
                         }
                     } else {
                         mbar_arrive_expect_tx(bar, B16_BYTES + A16_BYTES + (ron ? A16_BYTES : 0));
@@ -215,11 +235,39 @@ __global__ void __launch_bounds__(THREADS, 1)
                         if (ron)
                             tma_load_2d(st.r16, &tmR, bar, ks * BK * 2, m_tile * BM);
                     }
-                    if (PHI) {
-                        const int nt = ks + 1 < nks ? tile : tile + (int)gridDim.x, nk = ks + 1 < nks ? ks + 1 : 0;
-                        if (nt < tiles)
-                            ph = __ldg(phi + (int64_t)(nt / n_tiles) * phi_cols + nk / phi_blocks);
+                    ++p;
+                };
+                if constexpr (!PHI) {
+                    for (int ks = 0; ks < nks && !stop; ++ks)
+                        produce(ks, 0u, Bool<RES>{});
+                } else {
+                    const int r = it & 1;
+                    if (!mbar_wait(&S.phi_full[r], (it >> 1) & 1, kWaitLimitNs, gstat)) {
+                        flag_timeout(S, status);
+                        stop = true;
+                        break;
                     }
+                    const PhiRec &rec = S.rec[r];
+                    const uint32_t count = rec.count;
+                    // stages with a residual, then the others, each in k order
+                    for (int w = 0; 32 * w < nks && !stop; ++w) {
+                        uint32_t x = rec.bits[w];
+                        while (x != 0 && !stop) {
+                            const int b = __ffs(x) - 1;
+                            x &= x - 1;
+                            produce(32 * w + b, count, Bool<true>{});
+                        }
+                    }
+                    for (int w = 0; 32 * w < nks && !stop; ++w) {
+                        const int left = nks - 32 * w;
+                        uint32_t x = ~rec.bits[w] & (left >= 32 ? 0xffffffffu : (1u << left) - 1u);
+                        while (x != 0 && !stop) {
+                            const int b = __ffs(x) - 1;
+                            x &= x - 1;
+                            produce(32 * w + b, count, Bool<false>{});
+                        }
+                    }
+                    mbar_arrive(&S.phi_empty[r]);
                 }
             }
             S.issued = p;
@@ -238,26 +286,44 @@ __global__ void __launch_bounds__(THREADS, 1)
                 }
                 tc_fence_after();
                 const uint32_t acc = tmem + 256 * buf;
-                for (int ks = 0; ks < nks; ++ks, ++p) {
+                // the MMAs of the stage at position pos of the tile
+                auto mma_stage = [&](int pos, auto res_t) {
+                    constexpr bool ron = decltype(res_t)::value;
                     const int slot = p % STAGES;
                     if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat) ||
                         (CONV && !mbar_wait(&S.conv[slot], (p / STAGES) & 1, kWaitLimitNs, gstat))) {
                         flag_timeout(S, status);
                         stop = true;
-                        break;
+                        return;
                     }
                     tc_fence_after();
                     const auto &st = S.st[slot];
                     const uint32_t a0 = smem_u32(st.a16), r0 = smem_u32(st.r16), b0 = smem_u32(st.b);
-                    const bool ron = RES && (!PHI || S.res_on[slot] != 0);
 #pragma unroll
                     for (int j = 0; j < BK / 16; ++j) {
                         const uint64_t bd = sdesc_k_sw128(b0 + 32 * j);
-                        tc_mma_f16(acc, sdesc_k_sw128(a0 + 32 * j), bd, idesc, (ks | j) != 0);
+                        tc_mma_f16(acc, sdesc_k_sw128(a0 + 32 * j), bd, idesc, (pos | j) != 0);
                         if (ron)
                             tc_mma_f16(acc, sdesc_k_sw128(r0 + 32 * j), bd, idesc, 1);
                     }
                     tc_commit(&S.empty[slot]);
+                    ++p;
+                };
+                if constexpr (!PHI) {
+                    for (int ks = 0; ks < nks && !stop; ++ks)
+                        mma_stage(ks, Bool<RES>{});
+                } else {
+                    // the tile's residual-stage count arrives with its first stage
+                    if (!mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs, gstat)) {
+                        flag_timeout(S, status);
+                        break;
+                    }
+                    const int n_res = (int)(S.stage_info[p % STAGES] & 0x7fffffffu);
+                    int pos = 0;
+                    for (; pos < n_res && !stop; ++pos)
+                        mma_stage(pos, Bool<true>{});
+                    for (; pos < nks && !stop; ++pos)
+                        mma_stage(pos, Bool<false>{});
                 }
                 if (!stop)
                     tc_commit(&S.acc_full[buf]);
@@ -362,7 +428,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         if (!CONV && lane == 0)
             bulk_wait_group<0>(); // every TMA store of this warp has completed
-    } else {
+    } else if (warp < PHI_WARP) {
         if constexpr (CONV) {
         // ------------------------------------------------ converters (warps 6..13)
         // 2 x 128 rows x 8 groups of 8 elements per stage; thread u handles
@@ -380,7 +446,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     break;
                 }
                 auto &st = S.st[slot];
-                const bool ron = RES && (!PHI || S.res_on[slot] != 0);
+                const bool ron = RES && (!PHI || (S.stage_info[slot] >> 31) != 0);
 #pragma unroll 2
                 for (int ch = u; ch < 2 * BM * 8; ch += 32 * CONV_WARPS) {
                     const bool isr = ch >= BM * 8;
@@ -401,6 +467,38 @@ __global__ void __launch_bounds__(THREADS, 1)
                     mbar_arrive(&S.conv[slot]);
             }
         }
+        }
+    }
+    if constexpr (PHI) {
+        if (warp == PHI_WARP) {
+            // -------------------------------------------- phi reader
+            // Record of the CTA's j-th tile: stage ks of row tile m needs its
+            // residual when phi[m][ks / phi_blocks] is non-zero.
+            const int my_tiles =
+                (int)blockIdx.x < tiles ? (tiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x : 0;
+            for (int j = 0; j < my_tiles; ++j) {
+                const int r = j & 1;
+                if (j >= 2 && !__all_sync(0xffffffffu, mbar_wait(&S.phi_empty[r], ((j >> 1) - 1) & 1,
+                                                                 kWaitLimitNs, gstat))) {
+                    if (lane == 0)
+                        flag_timeout(S, status);
+                    break;
+                }
+                const int m_tile = ((int)blockIdx.x + j * (int)gridDim.x) / n_tiles;
+                PhiRec &rec = S.rec[r];
+                uint32_t count = 0;
+                for (int w = 0; 32 * w < nks; ++w) {
+                    const int ks = 32 * w + lane;
+                    const bool on = ks < nks && __ldg(phi + (int64_t)m_tile * phi_cols + ks / phi_blocks) != 0;
+                    const uint32_t word = __ballot_sync(0xffffffffu, on);
+                    if (lane == 0)
+                        rec.bits[w] = word;
+                    count += __popc(word);
+                }
+                if (lane == 0)
+                    rec.count = count;
+                mbar_arrive(&S.phi_full[r]);
+            }
         }
     }
 
@@ -432,7 +530,7 @@ cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const C
     const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
     const int phi_blocks = a.phi_r_s / BK;
     const int phi_cols = a.phi ? (int)((a.K + a.phi_r_s - 1) / a.phi_r_s) : 0;
-    kern<<<grid, THREADS, smem, st>>>(ta, tr, tb, ty, (const uint32_t *)a.a_meta, (const uint32_t *)a.r_meta, a.phi,
+    kern<<<grid, PHI ? THREADS + 32 : THREADS, smem, st>>>(ta, tr, tb, ty, (const uint32_t *)a.a_meta, (const uint32_t *)a.r_meta, a.phi,
                                       phi_blocks, phi_cols, a.y, (int)a.M, (int)a.N, (int)a.K, a.status);
     return cudaGetLastError();
 }
@@ -457,7 +555,10 @@ cudaError_t launch_conv(const GemmHif4Args &a, cudaStream_t st)
     const uint64_t yrow = (uint64_t)a.N * (a.out_bf16 ? 2 : 4);
     if (!encode_tmap_2d_u8(&ty, a.y, yrow, (uint64_t)a.M, yrow, 64, 32, 64))
         return cudaErrorInvalidValue;
-    const bool res = a.r_codes != nullptr, phi = res && a.phi != nullptr;
+    // Beyond REC_WORDS * 32 k-stages the record does not fit: every residual
+    // product is then issued (exact: phi = 0 residuals are zero).
+    const bool res = a.r_codes != nullptr;
+    const bool phi = res && a.phi != nullptr && a.K / BK <= REC_WORDS * 32;
 #define RFQ_GV(R, P, O) return launch_variant<CONV, R, P, O>(ta, tr, tb, ty, a, st)
     if (!res) {
         if (a.out_bf16) RFQ_GV(false, false, true);

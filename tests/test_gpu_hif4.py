@@ -179,6 +179,19 @@ def test_linear_no_residual_and_phi(orc, expand):
     check_y(y, _ref(orc, xq, xr, wq, M, K, N))
 
 
+@pytest.mark.parametrize("expand", [False, True])
+def test_phi_records_wrap(orc, expand):
+    """320 output tiles (several per CTA, so the per-tile phi records wrap
+    their two buffers) with a mixed phi pattern at r_s = 64."""
+    M, K, N = 640, 1024, 16384
+    xb = make_activation(ActSpec(M, K, "laplace", body_scale=0.3, chan_count=24, chan_scale=50.0, seed=21))
+    wb = make_weight(K, N, seed=21)
+    xq, xr, wq, y = _linear(xb, wb, mode=rfq.RFQ_FALLBACK_AMAX, tau=10.0, r_s=64, use_phi=True, expand=expand)
+    q = orc.quantize_act(xb, orc.FMT_HIF4, orc.PHI_AMAX, 10.0, 128, 64)
+    assert 0.1 < q["phi"].mean() < 0.9
+    check_y(y, _ref(orc, xq, xr, wq, M, K, N))
+
+
 @pytest.mark.parametrize("out,expand", [(rfq.RFQ_OUT_BF16, True), (rfq.RFQ_OUT_F32, True), (rfq.RFQ_OUT_BF16, False)])
 def test_full_size_qwen_down_hif4(orc, out, expand):
     spec = WORKLOADS["qwen_down_hif4"]

@@ -111,6 +111,20 @@ def test_phi_amax_many_stage_blocks(orc, M):
     check_y(y[rows], ref)
 
 
+def test_phi_amax_records_wrap(orc):
+    """180 output tiles of 256 x 256 (up to three per CTA pair, so the
+    per-tile phi records wrap their two buffers), a ragged last row pair, an
+    odd number of 128-element chunks and a mixed phi pattern at r_s = 128."""
+    M, K, N, r_s, tau = 600, 640, 15360, 128, 30.0
+    xb = make_activation(ActSpec(M, K, "normal", chan_count=3, chan_scale=64.0, seed=31))
+    wb = make_weight(K, N, seed=31)
+    xq, xr, wq, y, phi = _run(xb, wb, mode=rfq.RFQ_FALLBACK_AMAX, tau=tau, r_s=r_s, use_phi=True)
+    q = orc.quantize_act(xb, orc.FMT_MXFP4, orc.PHI_AMAX, tau, 128, r_s)
+    assert np.array_equal(phi.cpu().numpy().reshape(q["phi"].shape), q["phi"])
+    assert 0.1 < q["phi"].mean() < 0.9
+    check_y(y, _ref(orc, xq, xr, wq, M, K, N))
+
+
 def test_bf16_output(orc):
     M, K, N = 256, 1024, 512
     xb = make_activation(ActSpec(M, K, "normal", chan_count=4, chan_scale=64.0, seed=4))
