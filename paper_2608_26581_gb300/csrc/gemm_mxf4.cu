@@ -16,10 +16,15 @@
 // SAME shared-memory W~ tile into the SAME TMEM accumulator: W~ is read once
 // for both products and the correction costs only MMA issue (the on-the-fly
 // residual accumulation of Sec. 4.3).  Residual MMAs of k-chunks with
-// phi = 0 are not issued and their A tiles are not loaded; with selective phi
-// an extra warp turns the phi bytes into per-stage residual masks in shared
-// memory a block of 256 stages ahead (a global load issued by the producer
-// would wait behind the stage copies in flight).  Eight epilogue
+// phi = 0 are not issued and their A tiles are not loaded.  With selective
+// phi an extra warp writes one record per output tile (a bit per 256-element
+// k-stage, set when either chunk's phi is 1, and their count; a global load
+// issued by the producer would wait behind the stage copies in flight); the
+// producer issues the residual stages first and publishes the count with
+// every stage, so the MMA thread and the scale writers run loops with
+// compile-time residual masks (a branch on a per-stage mask in the MMA
+// thread slows its MMA issue; the sum over k does not depend on its order;
+// a phi = 0 chunk beside a phi = 1 one adds exact zeros).  Eight epilogue
 // warps drain the fp32 accumulator; with bf16 Y each warp first loads and
 // packs all 128 of its columns, hands the accumulator back to the MMA thread,
 // then stages and stores them (shared memory + TMA stores), so the next
@@ -59,7 +64,7 @@ constexpr int EPI_WARPS = 8;
 constexpr int SF_WARPS = 4;
 constexpr int THREADS = 64 + 32 * EPI_WARPS + 32 * SF_WARPS;
 constexpr int PHI_WARP = THREADS / 32;  // the phi reader: one warp beyond THREADS
-constexpr int PHI_BLK = 256;            // stage masks per phi block
+constexpr int REC_WORDS = 64;           // phi record: up to 2048 full k-stages (K <= 524288)
 static_assert(SF_COL0 + SF_SLOTS * SF_SLOT_COLS <= TMEM_COLS, "TMEM budget");
 static_assert(SF_SLOTS >= STAGES, "a scale slot is rewritten only after its stage's MMAs completed");
 
@@ -74,6 +79,15 @@ struct alignas(1024) Stage {
 
 constexpr int YSTAGE = 2048;          // per epilogue warp: 32 rows x 64 bytes of Y
 
+// Selective phi, one output tile: bit ks of bits (ks < K / 256, the full
+// k-stages) set when phi is 1 for either 128-element chunk of stage ks;
+// info = the number of set bits | (phi of the odd last chunk, when K / 128
+// is odd) << 31.
+struct PhiRec {
+    uint32_t bits[REC_WORDS];
+    uint32_t info;
+};
+
 struct Smem {
     Stage st[STAGES];
     alignas(1024) uint8_t ystage[EPI_WARPS * YSTAGE]; // 64B-swizzled staging for the TMA stores of Y
@@ -83,10 +97,10 @@ struct Smem {
     uint64_t acc_empty;
     uint64_t drain;
     uint64_t sf_ready[SF_SLOTS];      // the scale writers filled the slot
-    uint64_t phi_full[2];             // the phi reader filled the mask block
-    uint64_t phi_empty[2];            // the producer consumed the mask block
-    uint8_t phi_mask[2][PHI_BLK];     // per stage of a block: bit c, phi of chunk c is 1
-    uint32_t res_mask[STAGES];        // bit c: the residual of 128-element chunk c of the stage applies
+    uint64_t phi_full[2];             // the phi reader filled the record
+    uint64_t phi_empty[2];            // the producer consumed the record
+    PhiRec rec[2];
+    uint32_t stage_info[STAGES];      // the tile's info (PhiRec::info), published with each stage
     uint32_t tmem_base;
     int32_t abort_flag;
     int32_t issued;
@@ -100,6 +114,15 @@ __device__ __forceinline__ void flag_timeout(Smem &S, int32_t *status)
     S.abort_flag = 1;
     atomicExch(status, kDevTimeout);
 }
+
+template <bool B>
+struct Bool {
+    static constexpr bool value = B;
+};
+template <uint32_t V>
+struct Mask {
+    static constexpr uint32_t value = V;
+};
 
 template <bool RES, bool PHI, bool OUT_BF16>
 __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
@@ -124,6 +147,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
 
     const int kc = K >> 7;                 // 128-element chunks
     const int nks = (kc + 1) >> 1;         // k-stages (the last may hold one chunk)
+    const int nf = kc >> 1;                // stages with two chunks
     const int n_tiles = (N + BN - 1) / BN;
     const int m_tiles = (M + BM - 1) / BM;
     const int tiles = n_tiles * m_tiles;
@@ -165,36 +189,24 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     if (warp == 0) {
         // ------------------------------------------------ TMA producer
         if (lane == 0) {
-            int p = 0; // stages issued so far (ring position)
+            int p = 0, it = 0; // p: stages issued so far (ring position)
             bool stop = false;
-            for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x) {
+            for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x, ++it) {
                 const int m_tile = tile / n_tiles, n_tile = tile - m_tile * n_tiles;
-                for (int ks = 0; ks < nks; ++ks, ++p) {
+                const int atom0 = n_tile * 2;
+                const int nb = atom0 + 1 < n_atoms ? 2 : 1;
+                // one k-stage: wait for its ring slot, publish the tile's info,
+                // issue the copies
+                auto produce = [&](int ks, uint32_t info, auto res_t) {
+                    constexpr bool res_on = decltype(res_t)::value;
                     const int slot = p % STAGES;
                     if (!mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, kWaitLimitNs, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
-                        break;
+                        return;
                     }
                     const int c0 = 2 * ks, nch = min(2, kc - c0);
-                    // residual chunks of the stage, published to the MMA thread and
-                    // the writers through the stage's barrier
-                    uint32_t mask = RES ? (nch == 2 ? 3u : 1u) : 0u;
-                    if (PHI) {
-                        const int blk = p / PHI_BLK, e = p - blk * PHI_BLK;
-                        if (e == 0 && !mbar_wait(&S.phi_full[blk & 1], (blk >> 1) & 1, kWaitLimitNs, gstat)) {
-                            flag_timeout(S, status);
-                            stop = true;
-                            break;
-                        }
-                        mask = S.phi_mask[blk & 1][e];
-                        if (e == PHI_BLK - 1)
-                            mbar_arrive(&S.phi_empty[blk & 1]);
-                    }
-                    const bool res_on = mask != 0;
-                    S.res_mask[slot] = mask;
-                    const int atom0 = n_tile * 2;
-                    const int nb = atom0 + 1 < n_atoms ? 2 : 1;
+                    S.stage_info[slot] = info;
                     const uint32_t sfbytes = (uint32_t)nch * ATOM;
                     Stage &st = S.st[slot];
                     uint64_t *bar = &S.full[slot];
@@ -209,6 +221,45 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                         bulk_load(st.sfr, sfr + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, bar);
                     for (int h = 0; h < nb; ++h)
                         bulk_load(st.sfb + h * 2 * ATOM, sfb + ((int64_t)(atom0 + h) * kc + c0) * ATOM, sfbytes, bar);
+                    ++p;
+                };
+                if constexpr (!PHI) {
+                    for (int ks = 0; ks < nks && !stop; ++ks)
+                        produce(ks, 0u, Bool<RES>{});
+                } else {
+                    const int r = it & 1;
+                    if (!mbar_wait(&S.phi_full[r], (it >> 1) & 1, kWaitLimitNs, gstat)) {
+                        flag_timeout(S, status);
+                        stop = true;
+                        break;
+                    }
+                    const PhiRec &rec = S.rec[r];
+                    const uint32_t info = rec.info;
+                    // stages with a residual, then the others, each in k order
+                    for (int w = 0; 32 * w < nf && !stop; ++w) {
+                        uint32_t x = rec.bits[w];
+                        while (x != 0 && !stop) {
+                            const int b = __ffs(x) - 1;
+                            x &= x - 1;
+                            produce(32 * w + b, info, Bool<true>{});
+                        }
+                    }
+                    for (int w = 0; 32 * w < nf && !stop; ++w) {
+                        const int left = nf - 32 * w;
+                        uint32_t x = ~rec.bits[w] & (left >= 32 ? 0xffffffffu : (1u << left) - 1u);
+                        while (x != 0 && !stop) {
+                            const int b = __ffs(x) - 1;
+                            x &= x - 1;
+                            produce(32 * w + b, info, Bool<false>{});
+                        }
+                    }
+                    if (nf < nks && !stop) {   // the odd last chunk
+                        if (info >> 31)
+                            produce(nf, info, Bool<true>{});
+                        else
+                            produce(nf, info, Bool<false>{});
+                    }
+                    mbar_arrive(&S.phi_empty[r]);
                 }
             }
             S.issued = p;
@@ -224,20 +275,20 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                     break;
                 }
                 tc_fence_after();
-                for (int ks = 0; ks < nks; ++ks, ++p) {
+                // the MMAs of the stage at position pos of the tile, with residual
+                // mask rm (bit c: chunk c's residual product) known at compile time
+                auto mma_stage = [&](int pos, int nch, auto rm_t) {
+                    constexpr uint32_t rm = decltype(rm_t)::value;
                     const int slot = p % STAGES, sfs = p % SF_SLOTS;
                     if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat) ||
                         !mbar_wait(&S.sf_ready[sfs], (p / SF_SLOTS) & 1, kWaitLimitNs, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
-                        break;
+                        return;
                     }
                     tc_fence_after();
-                    const int c0 = 2 * ks, nch = min(2, kc - c0);
                     const uint32_t sf = tmem + SF_COL0 + SF_SLOT_COLS * sfs;
                     const Stage &st = S.st[slot];
-                    // without selective phi the mask is fixed: no shared-memory read on the issue path
-                    const uint32_t res_mask = PHI ? S.res_mask[slot] : (RES ? (nch == 2 ? 3u : 1u) : 0u);
                     const uint32_t a0 = smem_u32(st.a), r0 = smem_u32(st.r), b0 = smem_u32(st.b);
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
@@ -247,11 +298,35 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                         const uint32_t id = idesc_mxf4(BM, BN, 2 * (j & 1), 2 * (j & 1));
                         const uint64_t bd = sdesc_k_sw128(b0 + 32 * j);
                         const uint32_t sfb_t = sf + 16 + 8 * c;
-                        tc_mma_mxf4(tmem, sdesc_k_sw128(a0 + 32 * j), bd, id, sf + 4 * c, sfb_t, (ks | j) != 0);
-                        if (RES && ((res_mask >> c) & 1))
+                        tc_mma_mxf4(tmem, sdesc_k_sw128(a0 + 32 * j), bd, id, sf + 4 * c, sfb_t, (pos | j) != 0);
+                        if ((rm >> c) & 1)
                             tc_mma_mxf4(tmem, sdesc_k_sw128(r0 + 32 * j), bd, id, sf + 8 + 4 * c, sfb_t, 1);
                     }
                     tc_commit(&S.empty[slot]);
+                    ++p;
+                };
+                if constexpr (!PHI) {
+                    for (int ks = 0; ks < nks && !stop; ++ks)
+                        mma_stage(ks, min(2, kc - 2 * ks), Mask<RES ? 3u : 0u>{});
+                } else {
+                    // the tile's residual-stage count arrives with its first stage
+                    if (!mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs, gstat)) {
+                        flag_timeout(S, status);
+                        break;
+                    }
+                    const uint32_t info = S.stage_info[p % STAGES];
+                    const int n_res = (int)(info & 0x7fffffffu);
+                    int pos = 0;
+                    for (; pos < n_res && !stop; ++pos)
+                        mma_stage(pos, 2, Mask<3u>{});
+                    for (; pos < nf && !stop; ++pos)
+                        mma_stage(pos, 2, Mask<0u>{});
+                    if (nf < nks && !stop) {
+                        if (info >> 31)
+                            mma_stage(pos, 1, Mask<1u>{});
+                        else
+                            mma_stage(pos, 1, Mask<0u>{});
+                    }
                 }
                 if (!stop)
                     tc_commit(&S.acc_full);
@@ -380,17 +455,19 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
         int p = 0;
         bool stop = false;
         for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x) {
-            for (int ks = 0; ks < nks; ++ks, ++p) {
+            // the scale words of the next stage (in the producer's order), with
+            // the residual mask rm known at compile time
+            auto write_stage = [&](int nch, auto rm_t) {
+                constexpr uint32_t rm = decltype(rm_t)::value;
                 const int slot = p % STAGES, sfs = p % SF_SLOTS;
                 // warp-uniform outcome: the tcgen05 stores below need the whole warp
                 if (!__all_sync(0xffffffffu, mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat))) {
                     if (lane == 0)
                         flag_timeout(S, status);
                     stop = true;
-                    break;
+                    return;
                 }
                 tc_fence_after();
-                const int c0 = 2 * ks, nch = min(2, kc - c0);
                 const Stage &st = S.st[slot];
                 const uint32_t tb = tmem + ((uint32_t)(q * 32) << 16) + SF_COL0 + SF_SLOT_COLS * sfs;
 #pragma unroll
@@ -401,7 +478,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                     const uint4 vb0 = *reinterpret_cast<const uint4 *>(st.sfb + c * ATOM + lane * 16);
                     const uint4 vb1 = *reinterpret_cast<const uint4 *>(st.sfb + (2 + c) * ATOM + lane * 16);
                     tmem_st_32x32b_x4(tb + 4 * c, va.x, va.y, va.z, va.w);
-                    if (RES && (!PHI || ((S.res_mask[slot] >> c) & 1))) {
+                    if ((rm >> c) & 1) {
                         const uint4 vr = *reinterpret_cast<const uint4 *>(st.sfr + c * ATOM + lane * 16);
                         tmem_st_32x32b_x4(tb + 8 + 4 * c, vr.x, vr.y, vr.z, vr.w);
                     }
@@ -413,37 +490,63 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                 __syncwarp();
                 if (lane == 0)
                     mbar_arrive(&S.sf_ready[sfs]);
+                ++p;
+            };
+            if constexpr (!PHI) {
+                for (int ks = 0; ks < nks && !stop; ++ks)
+                    write_stage(min(2, kc - 2 * ks), Mask<RES ? 3u : 0u>{});
+            } else {
+                // the tile's residual-stage count arrives with its first stage
+                if (!__all_sync(0xffffffffu, mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs, gstat))) {
+                    if (lane == 0)
+                        flag_timeout(S, status);
+                    break;
+                }
+                const uint32_t info = S.stage_info[p % STAGES];
+                const int n_res = (int)(info & 0x7fffffffu);
+                int pos = 0;
+                for (; pos < n_res && !stop; ++pos)
+                    write_stage(2, Mask<3u>{});
+                for (; pos < nf && !stop; ++pos)
+                    write_stage(2, Mask<0u>{});
+                if (nf < nks && !stop) {
+                    if (info >> 31)
+                        write_stage(1, Mask<1u>{});
+                    else
+                        write_stage(1, Mask<0u>{});
+                }
             }
         }
     } else if (PHI) {
         // ------------------------------------------------ phi reader (warp 14)
-        // Stage g of this CTA (the producer's running stage index) is k-stage
-        // g mod nks of the CTA's tile number g / nks; its mask has bit c set
-        // when chunk c exists and its phi is 1.
-        const int my_tiles = (int)blockIdx.x < tiles ? (tiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x : 0;
-        const int total = my_tiles * nks;
-        for (int blk = 0; blk * PHI_BLK < total; ++blk) {
-            const int b = blk & 1;
-            if (blk >= 2 && !__all_sync(0xffffffffu, mbar_wait(&S.phi_empty[b], ((blk >> 1) - 1) & 1,
-                                                               kWaitLimitNs, gstat))) {
+        // Record of the CTA's j-th tile: chunk c of row tile m needs its
+        // residual when phi[m][c / phi_chunks] is non-zero.
+        const int my_tiles =
+            (int)blockIdx.x < tiles ? (tiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x : 0;
+        for (int j = 0; j < my_tiles; ++j) {
+            const int r = j & 1;
+            if (j >= 2 && !__all_sync(0xffffffffu, mbar_wait(&S.phi_empty[r], ((j >> 1) - 1) & 1,
+                                                             kWaitLimitNs, gstat))) {
                 if (lane == 0)
                     flag_timeout(S, status);
                 break;
             }
-            for (int e = lane; e < PHI_BLK; e += 32) {
-                const int g = blk * PHI_BLK + e;
-                if (g >= total)
-                    break;
-                const int j = g / nks, ks = g - j * nks;
-                const int m_tile = ((int)blockIdx.x + j * (int)gridDim.x) / n_tiles;
-                uint32_t mask = 0;
-#pragma unroll
-                for (int c = 0; c < 2; ++c)
-                    if (2 * ks + c < kc && __ldg(phi + (int64_t)m_tile * phi_cols + (2 * ks + c) / phi_chunks) != 0)
-                        mask |= 1u << c;
-                S.phi_mask[b][e] = (uint8_t)mask;
+            const uint8_t *row = phi + (int64_t)(((int)blockIdx.x + j * (int)gridDim.x) / n_tiles) * phi_cols;
+            PhiRec &rec = S.rec[r];
+            uint32_t n_res = 0;
+            for (int w = 0; 32 * w < nf; ++w) {
+                const int ks = 32 * w + lane;
+                const bool on = ks < nf && (__ldg(row + (2 * ks) / phi_chunks) != 0 ||
+                                            __ldg(row + (2 * ks + 1) / phi_chunks) != 0);
+                const uint32_t word = __ballot_sync(0xffffffffu, on);
+                if (lane == 0)
+                    rec.bits[w] = word;
+                n_res += __popc(word);
             }
-            mbar_arrive(&S.phi_full[b]);
+            const uint32_t tail = nf < nks && __ldg(row + (2 * nf) / phi_chunks) != 0 ? 1u : 0u;
+            if (lane == 0)
+                rec.info = n_res | tail << 31;
+            mbar_arrive(&S.phi_full[r]);
         }
     }
 
@@ -505,7 +608,10 @@ cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st)
     const uint64_t yrow = (uint64_t)a.N * (a.out_bf16 ? 2 : 4);
     if (!encode_tmap_2d_u8(&ty, a.y, yrow, (uint64_t)a.M, yrow, 64, 32, 64))
         return cudaErrorInvalidValue;
-    const bool res = a.r_codes != nullptr, phi = res && a.phi != nullptr;
+    // Beyond REC_WORDS * 32 full k-stages the record does not fit: every
+    // residual product is then issued (exact: phi = 0 residuals are zero).
+    const bool res = a.r_codes != nullptr;
+    const bool phi = res && a.phi != nullptr && a.K / 256 <= REC_WORDS * 32;
 #define RFQ_GV(R, P, O) return launch_variant<R, P, O>(ta, tr, tb, ty, a, st)
     if (!res) {
         if (a.out_bf16) RFQ_GV(false, false, true);
