@@ -197,7 +197,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                 const int nb = atom0 + 1 < n_atoms ? 2 : 1;
                 // one k-stage: wait for its ring slot, publish the tile's info,
                 // issue the copies
-                auto produce = [&](int ks, uint32_t info, auto res_t) {
+                auto produce = [&](int ks, int nch, uint32_t info, auto res_t) {
                     constexpr bool res_on = decltype(res_t)::value;
                     const int slot = p % STAGES;
                     if (!mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, kWaitLimitNs, gstat)) {
@@ -205,8 +205,9 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                         stop = true;
                         return;
                     }
-                    const int c0 = 2 * ks, nch = min(2, kc - c0);
-                    S.stage_info[slot] = info;
+                    const int c0 = 2 * ks;
+                    if (PHI)
+                        S.stage_info[slot] = info;
                     const uint32_t sfbytes = (uint32_t)nch * ATOM;
                     Stage &st = S.st[slot];
                     uint64_t *bar = &S.full[slot];
@@ -224,8 +225,11 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                     ++p;
                 };
                 if constexpr (!PHI) {
-                    for (int ks = 0; ks < nks && !stop; ++ks)
-                        produce(ks, 0u, Bool<RES>{});
+                    // full stages, then an odd last chunk (chunk counts known at compile time)
+                    for (int ks = 0; ks < nf && !stop; ++ks)
+                        produce(ks, 2, 0u, Bool<RES>{});
+                    if (nf < nks && !stop)
+                        produce(nf, 1, 0u, Bool<RES>{});
                 } else {
                     const int r = it & 1;
                     if (!mbar_wait(&S.phi_full[r], (it >> 1) & 1, kWaitLimitNs, gstat)) {
@@ -241,7 +245,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                         while (x != 0 && !stop) {
                             const int b = __ffs(x) - 1;
                             x &= x - 1;
-                            produce(32 * w + b, info, Bool<true>{});
+                            produce(32 * w + b, 2, info, Bool<true>{});
                         }
                     }
                     for (int w = 0; 32 * w < nf && !stop; ++w) {
@@ -250,14 +254,14 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                         while (x != 0 && !stop) {
                             const int b = __ffs(x) - 1;
                             x &= x - 1;
-                            produce(32 * w + b, info, Bool<false>{});
+                            produce(32 * w + b, 2, info, Bool<false>{});
                         }
                     }
                     if (nf < nks && !stop) {   // the odd last chunk
                         if (info >> 31)
-                            produce(nf, info, Bool<true>{});
+                            produce(nf, 1, info, Bool<true>{});
                         else
-                            produce(nf, info, Bool<false>{});
+                            produce(nf, 1, info, Bool<false>{});
                     }
                     mbar_arrive(&S.phi_empty[r]);
                 }
@@ -306,8 +310,10 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                     ++p;
                 };
                 if constexpr (!PHI) {
-                    for (int ks = 0; ks < nks && !stop; ++ks)
-                        mma_stage(ks, min(2, kc - 2 * ks), Mask<RES ? 3u : 0u>{});
+                    for (int ks = 0; ks < nf && !stop; ++ks)
+                        mma_stage(ks, 2, Mask<RES ? 3u : 0u>{});
+                    if (nf < nks && !stop)
+                        mma_stage(nf, 1, Mask<RES ? 1u : 0u>{});
                 } else {
                     // the tile's residual-stage count arrives with its first stage
                     if (!mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs, gstat)) {
@@ -493,8 +499,10 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                 ++p;
             };
             if constexpr (!PHI) {
-                for (int ks = 0; ks < nks && !stop; ++ks)
-                    write_stage(min(2, kc - 2 * ks), Mask<RES ? 3u : 0u>{});
+                for (int ks = 0; ks < nf && !stop; ++ks)
+                    write_stage(2, Mask<RES ? 3u : 0u>{});
+                if (nf < nks && !stop)
+                    write_stage(1, Mask<RES ? 1u : 0u>{});
             } else {
                 // the tile's residual-stage count arrives with its first stage
                 if (!__all_sync(0xffffffffu, mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs, gstat))) {

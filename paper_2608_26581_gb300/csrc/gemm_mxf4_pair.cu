@@ -220,7 +220,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 // one k-stage: wait for its ring slot, publish the tile's info,
                 // issue the copies (codes: both CTAs' copies complete on the even
                 // CTA's barrier; scale atoms: this CTA's own barrier)
-                auto produce = [&](int ks, uint32_t info, auto res_t) {
+                auto produce = [&](int ks, int nch, uint32_t info, auto res_t) {
                     constexpr bool res_on = decltype(res_t)::value;
                     const int slot = p % STAGES;
                     if (!mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, kWaitLimitNs, gstat)) {
@@ -228,8 +228,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                         stop = true;
                         return;
                     }
-                    const int c0 = 2 * ks, nch = min(2, kc - c0);
-                    S.stage_info[slot] = info;
+                    const int c0 = 2 * ks;
+                    if (PHI)
+                        S.stage_info[slot] = info;
                     Stage &st = S.st[slot];
                     const uint32_t bar = full0 + 8 * slot;
                     const uint32_t sfbytes = (uint32_t)nch * ATOM;
@@ -252,8 +253,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     ++p;
                 };
                 if constexpr (!PHI) {
-                    for (int ks = 0; ks < nks && !stop; ++ks)
-                        produce(ks, 0u, Bool<RES>{});
+                    // full stages, then an odd last chunk (chunk counts known at compile time)
+                    for (int ks = 0; ks < nf && !stop; ++ks)
+                        produce(ks, 2, 0u, Bool<RES>{});
+                    if (nf < nks && !stop)
+                        produce(nf, 1, 0u, Bool<RES>{});
                 } else {
                     const int r = it & 1;
                     if (!mbar_wait(&S.phi_full[r], (it >> 1) & 1, kWaitLimitNs, gstat)) {
@@ -269,7 +273,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                         while (x != 0 && !stop) {
                             const int b = __ffs(x) - 1;
                             x &= x - 1;
-                            produce(32 * w + b, info, Bool<true>{});
+                            produce(32 * w + b, 2, info, Bool<true>{});
                         }
                     }
                     for (int w = 0; 32 * w < nf && !stop; ++w) {
@@ -278,14 +282,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                         while (x != 0 && !stop) {
                             const int b = __ffs(x) - 1;
                             x &= x - 1;
-                            produce(32 * w + b, info, Bool<false>{});
+                            produce(32 * w + b, 2, info, Bool<false>{});
                         }
                     }
                     if (nf < nks && !stop) {   // the odd last chunk
                         if (info >> 31)
-                            produce(nf, info, Bool<true>{});
+                            produce(nf, 1, info, Bool<true>{});
                         else
-                            produce(nf, info, Bool<false>{});
+                            produce(nf, 1, info, Bool<false>{});
                     }
                     mbar_arrive(&S.phi_empty[r]);
                 }
@@ -341,8 +345,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     ++p;
                 };
                 if constexpr (!PHI) {
-                    for (int ks = 0; ks < nks && !stop; ++ks)
-                        mma_stage(ks, min(2, kc - 2 * ks), Mask<RES ? 3u : 0u>{});
+                    for (int ks = 0; ks < nf && !stop; ++ks)
+                        mma_stage(ks, 2, Mask<RES ? 3u : 0u>{});
+                    if (nf < nks && !stop)
+                        mma_stage(nf, 1, Mask<RES ? 1u : 0u>{});
                 } else {
                     // the tile's residual-stage count arrives with its first stage
                     if (!mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs, gstat)) {
@@ -538,8 +544,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 ++p;
             };
             if constexpr (!PHI) {
-                for (int ks = 0; ks < nks && !stop; ++ks)
-                    write_stage(min(2, kc - 2 * ks), Mask<RES ? 3u : 0u>{});
+                for (int ks = 0; ks < nf && !stop; ++ks)
+                    write_stage(2, Mask<RES ? 3u : 0u>{});
+                if (nf < nks && !stop)
+                    write_stage(1, Mask<RES ? 1u : 0u>{});
             } else {
                 // the tile's residual-stage count arrives with its first stage
                 if (!__all_sync(0xffffffffu, mbar_wait(&S.sf_full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs, gstat))) {

@@ -111,17 +111,42 @@ __global__ void __launch_bounds__(256) act_quant_mxfp4_kernel(const uint4 *__res
 }
 
 // phi(p, r) = [max |x| over the p_s x r_s tile > tau]; one block per tile.
+// |x| of a bf16 is its low 15 bits, and for non-NaN values the order of
+// those bits as integers is the order of the magnitudes, so the block takes
+// a packed unsigned max over 16-byte loads (two bf16 per 32-bit lane, NaN
+// halves dropped as fmaxf would) and converts the winner to fp32 once.
+// Rows are 16-byte aligned (K % 32 == 0); tiles whose column range is not a
+// whole number of 8-element chunks take the scalar loop.
 __global__ void __launch_bounds__(256) phi_amax_kernel(const __nv_bfloat16 *__restrict__ x, int64_t M, int64_t K,
                                                       int p_s, int r_s, float tau, uint8_t *__restrict__ phi)
 {
     const int64_t nr = (K + r_s - 1) / r_s;
     const int64_t p = blockIdx.x / nr, r = blockIdx.x % nr;
     const int64_t m0 = p * p_s, k0 = r * r_s;
-    const int64_t m1 = min(M, m0 + p_s), k1 = min(K, k0 + r_s);
-    const int64_t w = k1 - k0;
-    float a = 0.f;
-    for (int64_t i = threadIdx.x; i < (m1 - m0) * w; i += blockDim.x)
-        a = fmaxf(a, fabsf(__bfloat162float(x[(m0 + i / w) * K + k0 + i % w])));
+    const int rows = (int)(min(M, m0 + p_s) - m0), w = (int)(min(K, k0 + r_s) - k0);
+    uint32_t acc = 0; // two packed 15-bit magnitudes
+    if ((k0 & 7) == 0 && (w & 7) == 0) {
+        const int cw = w >> 3, n = rows * cw;
+        const __nv_bfloat16 *base = x + m0 * K + k0;
+#pragma unroll 4
+        for (int i = threadIdx.x; i < n; i += blockDim.x) {
+            const int row = i / cw, c = i - row * cw;
+            const uint4 v = __ldg(reinterpret_cast<const uint4 *>(base + (int64_t)row * K + 8 * c));
+            const uint32_t q[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const uint32_t mag = q[j] & 0x7fff7fffu;
+                acc = __vmaxu2(acc, mag & ~__vcmpgtu2(mag, 0x7f807f80u));
+            }
+        }
+    } else {
+        for (int row = 0; row < rows; ++row)
+            for (int c = threadIdx.x; c < w; c += blockDim.x) {
+                const uint32_t mag = __bfloat16_as_ushort(x[(m0 + row) * K + k0 + c]) & 0x7fffu;
+                acc = __vmaxu2(acc, mag > 0x7f80u ? 0u : mag);
+            }
+    }
+    float a = __uint_as_float(max(acc & 0xffffu, acc >> 16) << 16);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1)
         a = fmaxf(a, __shfl_xor_sync(0xFFFFFFFFu, a, o));
