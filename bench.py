@@ -74,7 +74,8 @@ def _kernel_traffic(kernel: str, workload: str):
 def _src_hash(kernel: str):
     d = os.path.join(HERE, "paper_2608_26581_gb300", "csrc")
     m = hashlib.sha256()
-    for n in (_KERNEL_SRC[kernel], "ptx.cuh", "internal.h"):
+    extra = ("mxfp4_math.cuh",) if kernel in ("act_quant_mxfp4_kernel", "gemm_mxf4_fused_kernel") else ()
+    for n in (_KERNEL_SRC[kernel], "ptx.cuh", "internal.h") + extra:
         m.update(open(os.path.join(d, n), "rb").read())
     return m.hexdigest()[:16]
 
@@ -286,6 +287,10 @@ def run_rfq(args):
     amax_phi = args.phi_tau is not None
     if amax_phi and (fused or quant_only):
         raise SystemExit("--phi-tau applies to the two-kernel linear workloads")
+    # plain W4A4 (no residual pathway): the baseline RFQ's correction adds to
+    no_res = args.no_residual
+    if no_res and (fused or quant_only or amax_phi):
+        raise SystemExit("--no-residual applies to the two-kernel linear workloads without --phi-tau")
     F = rfq.RFQ_FMT_HIF4 if hif4 else rfq.RFQ_FMT_MXFP4
     L = rfq.RFQ_SCALE_MMA
 
@@ -305,7 +310,7 @@ def run_rfq(args):
             wop = wq
         del w
     xq = rfq.empty_qtensor(F, L, M, K, device=dev)
-    xr = rfq.empty_qtensor(F, L, M, K, device=dev)
+    xr = rfq.empty_qtensor(F, L, M, K, device=dev) if not no_res else None
     phi_buf = (torch.empty(((M + 127) // 128) * ((K + 255) // 256), dtype=torch.uint8, device=dev)
                if args.phi_tau is not None else None)
     # HiF4: the GEMM takes the exact bf16 expansions of X~ and X^ (expanding
@@ -341,16 +346,18 @@ def run_rfq(args):
             rfq.rfq_quantize_act(x, xq, xr, phi_buf, mode=rfq.RFQ_FALLBACK_AMAX, tau=args.phi_tau, p_s=128,
                                  r_s=256, stream=stream)
         else:
-            rfq.rfq_quantize_act(x, xq, xr, None, stream=stream)
+            rfq.rfq_quantize_act(x, xq, xr, None, mode=rfq.RFQ_FALLBACK_NONE if no_res else rfq.RFQ_FALLBACK_ALL,
+                                 stream=stream)
         if i is not None:
             per_step[i][1].record(stream)
         if hif4 and not quant_only:
             rfq.rfq_dequant(xq, xq16.codes, stream=stream)
-            rfq.rfq_dequant(xr, xr16.codes, stream=stream)
+            if xr is not None:
+                rfq.rfq_dequant(xr, xr16.codes, stream=stream)
         if i is not None:
             per_step[i][2].record(stream)
         if hif4 and not quant_only:
-            rfq.rfq_linear(xq16, xr16, phi_buf if amax_phi else None, 256, wop, y, rfq.RFQ_OUT_BF16, wsp,
+            rfq.rfq_linear(xq16, xr16 if xr is not None else None, phi_buf if amax_phi else None, 256, wop, y, rfq.RFQ_OUT_BF16, wsp,
                            stream=stream)
         elif not quant_only:
             rfq.rfq_linear(xq, xr, phi_buf if amax_phi else None, 256, wop, y, rfq.RFQ_OUT_BF16, wsp,
@@ -410,7 +417,7 @@ def run_rfq(args):
         raise RuntimeError("rfq_linear reported a device timeout")
 
     # executed MMA work: the main product, and the residual product on the phi = 1 tiles
-    phi_frac = float(phi_buf.float().mean().item()) if amax_phi else 1.0
+    phi_frac = float(phi_buf.float().mean().item()) if amax_phi else (0.0 if no_res else 1.0)
     flop = 2.0 * M * N * K * (1.0 + phi_frac)
     pk = _peaks()
     # The timed loop is short (tens of ms at full clocks), so the kernels are
@@ -428,10 +435,12 @@ def run_rfq(args):
         t_kernel = "gemm_mxf4_fused_kernel" if fused else (
             "gemm_mxf4_pair_kernel" if M > 128 else "gemm_mxf4_kernel")
     if hif4:
-        aq_bytes = M * K * 2 + 2 * (M * K // 2) + 2 * (((M + 127) // 128) * 128 * (K // 64) * 4)
+        npath = 1 if no_res else 2   # main (and residual) codes + metadata written
+        aq_bytes = M * K * 2 + npath * (M * K // 2) + npath * (((M + 127) // 128) * 128 * (K // 64) * 4)
         aq_kernel = "act_quant_hif4_kernel"
     else:
-        aq_bytes = M * K * 2 + 2 * (M * K // 2) + 2 * (((M + 127) // 128) * 128 * K // 32)
+        npath = 1 if no_res else 2
+        aq_bytes = M * K * 2 + npath * (M * K // 2) + npath * (((M + 127) // 128) * 128 * K // 32)
         aq_kernel = "act_quant_mxfp4_kernel"
     if fused:
         act_quant = None   # quantization happens inside the GEMM
@@ -450,7 +459,7 @@ def run_rfq(args):
         gemm_tflops = flop / (g_ms * 1e-3) / 1e12
         roofline = {"bound": "tensor", "kernel": t_kernel, "achieved": gemm_tflops, "peak": t_peak,
                     "unit": "TFLOP/s", "frac": gemm_tflops / t_peak,
-                    "traffic": _kernel_traffic(t_kernel, spec.name), "flop_per_launch": flop, "ms_per_launch": g_ms,
+                    "traffic": _kernel_traffic(t_kernel, spec.name + ("+phi" if amax_phi else "")), "flop_per_launch": flop, "ms_per_launch": g_ms,
                     "peak_source": t_src, "frac_of_sustained_peak": gemm_tflops / t_peak_sust}
     clocks = clk.summary()
     if e2e_ms is not None:
@@ -475,6 +484,7 @@ def run_rfq(args):
             "config": _config(spec, {"parallelism": f"dp{ws} over token rows" if ws > 1 else "single GPU",
                                      "variant": ("fused prologue: X quantized inside the GEMM" if fused
                                                  else "quantizer kernel + GEMM kernel"),
+                                     **({"residual": "none: plain W4A4 (Q(X) W~ only)"} if no_res else {}),
                                      **({"phi": f"AMAX: phi = [max |x| over the 128 x 256 tile > {args.phi_tau}], "
                                                 f"fraction of phi = 1 tiles f = {phi_frac:.4f}",
                                          "phi_fraction": phi_frac} if amax_phi else {})}),
@@ -504,6 +514,8 @@ def main():
     ap.add_argument("--rows", type=int, default=0, help="profile a smaller case: the first ROWS token rows")
     ap.add_argument("--phi-tau", type=float, default=None,
                     help="selective fallback: residual only on 128 x 256 tiles whose max |x| exceeds TAU")
+    ap.add_argument("--no-residual", action="store_true",
+                    help="plain W4A4: no residual pathway (the baseline the correction is added to)")
     ap.add_argument("--variant", default="two-kernel", choices=["two-kernel", "fused"],
                     help="fused: rfq_linear_fused, the activation quantizer inside the GEMM")
     ap.add_argument("--workload", default=WORKLOAD,
