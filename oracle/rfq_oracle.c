@@ -37,7 +37,18 @@
  *       bits [15:8] E1_8 (bit g = group g), bits [31:16] E1_16 (bit j =
  *       sub-group j).
  *   R8  The residual pathway uses the same 4-bit format as the main one
- *       (Sec. 4.3, Eq. for the re-quantized residual).
+ *       (Sec. 4.3, Eq. for the re-quantized residual); the FP4-to-FP8
+ *       variant named in Sec. 4.2 re-quantizes the residual of an MXFP4 main
+ *       pathway in MXFP8 E4M3 (reading R12).
+ *   R11 MXFP8 E4M3 (Sec. 3.2.1): the OCP E4M3 element, Eq. 1 with 4
+ *       exponent bits, 3 mantissa bits and bias 7, exponent field 0
+ *       subnormal, no infinities, S.1111.111 = NaN, largest finite 448; block
+ *       scale 2^(floor(log2 amax) - 8) (emax_elem = 8, as R1); elements round
+ *       to nearest, ties to even mantissa, saturating at +-448; a code keeps
+ *       the sign of its input (as R3); one byte per element.
+ *   R12 FP8 residual pathway (Sec. 4.2 names an FP4-to-FP8 pathway without
+ *       defining it): X~ = Q_MXFP4(X) and X^ = Q_MXFP8(X - X~), both with
+ *       32-element blocks along K; the GEMM multiplies X^ by the same W~.
  *
  * Parity status: the MXFP4 encoder (R1-R4), the residual, phi = "all" and the
  * GEMM are pinned by the tests in tests/test_oracle_*.py against the format
@@ -53,6 +64,7 @@
 
 #define RFQ_O_FMT_MXFP4 0
 #define RFQ_O_FMT_HIF4 1
+#define RFQ_O_FMT_MXFP8 2
 
 #define RFQ_O_PHI_NONE 0
 #define RFQ_O_PHI_ALL 1
@@ -196,6 +208,100 @@ void rfq_o_mxfp4_dequant(const uint8_t *codes, const uint8_t *scales,
 }
 
 /* ------------------------------------------------------------------ */
+/* E4M3 element and MXFP8, Sec. 3.1 Eq. 1 and Sec. 3.2.1 (reading R11) */
+/* ------------------------------------------------------------------ */
+
+/* Eq. 1 with E = 4 exponent bits, M = 3 mantissa bits and bias 7.  Exponent
+ * field 0 is subnormal: 2^(1 - bias) (0 + m/8).  The two codes S.1111.111
+ * are NaN; there is no infinity. */
+double rfq_o_e4m3_decode(int code)
+{
+    int s = (code >> 7) & 1;
+    int e = (code >> 3) & 15;
+    int m = code & 7;
+    const int bias = 7;
+    double mag;
+    if (e == 15 && m == 7)
+        return NAN;
+    if (e == 0)
+        mag = ldexp((double)m / 8.0, 1 - bias);
+    else
+        mag = ldexp(1.0 + (double)m / 8.0, e - bias);
+    return s ? -mag : mag;
+}
+
+/* Round y to the E4M3 grid (reading R11): a 3-bit mantissa with
+ * round-half-even, subnormal spacing 2^-9, saturating at 448.  Returns the
+ * 8-bit code. */
+int rfq_o_e4m3_encode(double y)
+{
+    int s = signbit(y) ? 1 : 0;
+    double a = fabs(y);
+    int code;
+    if (a < ldexp(1.0, -6)) {
+        /* subnormal binade: spacing 2^-9; 8 steps reach the first normal */
+        double q = nearbyint(ldexp(a, 9)); /* 0..8 */
+        code = (int)q;                     /* q = 8 is the code of 2^-6 */
+    } else {
+        int ex;
+        frexp(a, &ex);
+        int e = ex - 1;                    /* floor(log2 a) >= -6 */
+        if (e > 8) {
+            code = 0x7E;                   /* |y| >= 512: saturate to 448 */
+        } else {
+            double m = ldexp(a, -e) - 1.0; /* fraction in [0, 1) */
+            double q = nearbyint(m * 8.0); /* 0..8 */
+            int ef = e + 7;
+            if (q >= 8.0) { ef += 1; q = 0.0; }
+            if (ef > 15 || (ef == 15 && q > 6.0)) { ef = 15; q = 6.0; } /* past 448 */
+            code = (ef << 3) | (int)q;
+        }
+    }
+    return (s << 7) | code;
+}
+
+/* Shared exponent of one MXFP8 block: floor(log2 amax) - 8 (emax of E4M3),
+ * clamped to [-127, 127]; amax = 0 gives -127 (scale byte 0). */
+int rfq_o_mx8_scale_exp(double amax)
+{
+    if (!(amax > 0.0))
+        return -127;
+    int ex;
+    frexp(amax, &ex);
+    int e = (ex - 1) - 8;
+    if (e < -127) e = -127;
+    if (e > 127) e = 127;
+    return e;
+}
+
+/* MXFP8 quantization of [rows x k] along k in blocks of 32 (Sec. 3.2 Eqs.
+ * 3-4 with the E4M3 element).  codes: [rows][k] bytes; scales: [rows][k/32]. */
+void rfq_o_mxfp8_quantize(const double *x, int64_t rows, int64_t k,
+                          uint8_t *codes, uint8_t *scales)
+{
+    const int B = 32;
+    for (int64_t r = 0; r < rows; r++)
+        for (int64_t j = 0; j < k / B; j++) {
+            const double *xb = x + r * k + j * B;
+            double amax = 0.0;
+            for (int i = 0; i < B; i++)
+                if (fabs(xb[i]) > amax) amax = fabs(xb[i]);
+            int e = rfq_o_mx8_scale_exp(amax);
+            for (int i = 0; i < B; i++)
+                codes[r * k + j * B + i] = (uint8_t)rfq_o_e4m3_encode(ldexp(xb[i], -e));
+            scales[r * (k / B) + j] = (uint8_t)(e + 127);
+        }
+}
+
+void rfq_o_mxfp8_dequant(const uint8_t *codes, const uint8_t *scales,
+                         int64_t rows, int64_t k, double *out)
+{
+    for (int64_t r = 0; r < rows; r++)
+        for (int64_t i = 0; i < k; i++)
+            out[r * k + i] = ldexp(rfq_o_e4m3_decode(codes[r * k + i]), scales[r * (k / 32) + i / 32] - 127);
+}
+
+/* ------------------------------------------------------------------ */
 /* HiF4, Sec. 3.3                                                      */
 /* ------------------------------------------------------------------ */
 
@@ -307,6 +413,8 @@ static void quantize_fmt(int fmt, const double *x, int64_t rows, int64_t k,
 {
     if (fmt == RFQ_O_FMT_HIF4)
         rfq_o_hif4_quantize(x, rows, k, codes, (uint32_t *)scales);
+    else if (fmt == RFQ_O_FMT_MXFP8)
+        rfq_o_mxfp8_quantize(x, rows, k, codes, (uint8_t *)scales);
     else
         rfq_o_mxfp4_quantize(x, rows, k, codes, (uint8_t *)scales);
 }
@@ -316,9 +424,12 @@ void rfq_o_dequant(int fmt, const uint8_t *codes, const void *scales,
 {
     if (fmt == RFQ_O_FMT_HIF4)
         rfq_o_hif4_dequant(codes, (const uint32_t *)scales, rows, k, out);
+    else if (fmt == RFQ_O_FMT_MXFP8)
+        rfq_o_mxfp8_dequant(codes, (const uint8_t *)scales, rows, k, out);
     else
         rfq_o_mxfp4_dequant(codes, (const uint8_t *)scales, rows, k, out);
 }
+
 
 /* ------------------------------------------------------------------ */
 /* RFQ activation decomposition, Sec. 4.3 and Algorithm 1              */
@@ -356,10 +467,10 @@ void rfq_o_phi(const double *x, int64_t M, int64_t K, int mode, double tau,
  * main/res codes: [M][K/2]; scales: [M][K/32] bytes (MXFP4) or [M][K/64]
  * words (HiF4); phi: [ceil(M/p_s)][ceil(K/r_s)], may be NULL.
  * rc/rs may be NULL when mode is RFQ_O_PHI_NONE. */
-void rfq_o_quantize_act(const uint16_t *x_bf16, int64_t M, int64_t K, int fmt,
-                        int mode, double tau, int64_t p_s, int64_t r_s,
-                        uint8_t *mc, void *ms, uint8_t *rc, void *rs,
-                        uint8_t *phi_out)
+void rfq_o_quantize_act2(const uint16_t *x_bf16, int64_t M, int64_t K, int fmt,
+                         int res_fmt, int mode, double tau, int64_t p_s, int64_t r_s,
+                         uint8_t *mc, void *ms, uint8_t *rc, void *rs,
+                         uint8_t *phi_out)
 {
     double *x = (double *)malloc(sizeof(double) * M * K);
     double *xt = (double *)malloc(sizeof(double) * M * K);
@@ -376,14 +487,17 @@ void rfq_o_quantize_act(const uint16_t *x_bf16, int64_t M, int64_t K, int fmt,
                 /* exact in fp64: both operands have few significant bits */
                 xt[m * K + c] = on ? x[m * K + c] - xt[m * K + c] : 0.0;
             }
-        quantize_fmt(fmt, xt, M, K, rc, rs);
+        quantize_fmt(res_fmt, xt, M, K, rc, rs);
         /* phi = 0 blocks: codes and scale words are written as zero */
-        int64_t bs = fmt == RFQ_O_FMT_HIF4 ? 64 : 32;
+        int64_t bs = res_fmt == RFQ_O_FMT_HIF4 ? 64 : 32;
         for (int64_t m = 0; m < M; m++)
-            for (int64_t j = 0; j < scale_count(fmt, K); j++) {
+            for (int64_t j = 0; j < scale_count(res_fmt, K); j++) {
                 if (phi[(m / p_s) * nr + (j * bs) / r_s]) continue;
-                for (int64_t c = j * bs; c < (j + 1) * bs; c++) put_nibble(rc + m * (K / 2), c, 0);
-                if (fmt == RFQ_O_FMT_HIF4) ((uint32_t *)rs)[m * (K / 64) + j] = 0;
+                for (int64_t c = j * bs; c < (j + 1) * bs; c++) {
+                    if (res_fmt == RFQ_O_FMT_MXFP8) rc[m * K + c] = 0;
+                    else put_nibble(rc + m * (K / 2), c, 0);
+                }
+                if (res_fmt == RFQ_O_FMT_HIF4) ((uint32_t *)rs)[m * (K / 64) + j] = 0;
                 else ((uint8_t *)rs)[m * (K / 32) + j] = 0;
             }
     }
@@ -391,6 +505,15 @@ void rfq_o_quantize_act(const uint16_t *x_bf16, int64_t M, int64_t K, int fmt,
     free(phi);
     free(xt);
     free(x);
+}
+
+/* The decomposition with one format for both pathways (R8). */
+void rfq_o_quantize_act(const uint16_t *x_bf16, int64_t M, int64_t K, int fmt,
+                        int mode, double tau, int64_t p_s, int64_t r_s,
+                        uint8_t *mc, void *ms, uint8_t *rc, void *rs,
+                        uint8_t *phi_out)
+{
+    rfq_o_quantize_act2(x_bf16, M, K, fmt, fmt, mode, tau, p_s, r_s, mc, ms, rc, rs, phi_out);
 }
 
 /* Weight quantization Y~ = Q(Y) (Sec. 4.3; Algorithm 1): W is bf16 [K x N]
@@ -416,20 +539,21 @@ void rfq_o_quantize_weight(const uint16_t *w_bf16, int64_t K, int64_t N, int fmt
  * then the correction term).  The residual codes are zero where phi = 0,
  * so phi enters through them.  xr_codes may be NULL (plain W4A4).
  * W~ is K-major: codes [N][K/2].  Output Y: [M][N] doubles. */
-void rfq_o_linear(int fmt, const uint8_t *xm_codes, const void *xm_scales,
-                  const uint8_t *xr_codes, const void *xr_scales,
-                  int64_t M, int64_t K, const uint8_t *w_codes,
-                  const void *w_scales, int64_t N, double *Y)
+void rfq_o_linear2(int fmt, int res_fmt, int w_fmt,
+                   const uint8_t *xm_codes, const void *xm_scales,
+                   const uint8_t *xr_codes, const void *xr_scales,
+                   int64_t M, int64_t K, const uint8_t *w_codes,
+                   const void *w_scales, int64_t N, double *Y)
 {
     double *xm = (double *)malloc(sizeof(double) * M * K);
     double *xr = (double *)malloc(sizeof(double) * M * K);
     double *w = (double *)malloc(sizeof(double) * N * K);
     rfq_o_dequant(fmt, xm_codes, xm_scales, M, K, xm);
     if (xr_codes)
-        rfq_o_dequant(fmt, xr_codes, xr_scales, M, K, xr);
+        rfq_o_dequant(res_fmt, xr_codes, xr_scales, M, K, xr);
     else
         memset(xr, 0, sizeof(double) * M * K);
-    rfq_o_dequant(fmt, w_codes, w_scales, N, K, w);
+    rfq_o_dequant(w_fmt, w_codes, w_scales, N, K, w);
     for (int64_t m = 0; m < M; m++)
         for (int64_t n = 0; n < N; n++) {
             double z = 0.0;
@@ -442,4 +566,13 @@ void rfq_o_linear(int fmt, const uint8_t *xm_codes, const void *xm_scales,
     free(w);
     free(xr);
     free(xm);
+}
+
+/* The GEMM with one format for every operand. */
+void rfq_o_linear(int fmt, const uint8_t *xm_codes, const void *xm_scales,
+                  const uint8_t *xr_codes, const void *xr_scales,
+                  int64_t M, int64_t K, const uint8_t *w_codes,
+                  const void *w_scales, int64_t N, double *Y)
+{
+    rfq_o_linear2(fmt, fmt, fmt, xm_codes, xm_scales, xr_codes, xr_scales, M, K, w_codes, w_scales, N, Y);
 }
