@@ -50,6 +50,14 @@
  *   BF16    an exact bf16 expansion of a quantized matrix, [rows][k]
  *           (codes = the bf16 data, scales unused): rfq_dequant writes it,
  *           and rfq_linear takes the HiF4 weight in this form.
+ *   MXFP8   E4M3 codes (Sec. 3.2.1: sign, 4 exponent bits with bias 7, 3
+ *           mantissa bits; exponent field 0 subnormal; no infinity;
+ *           S.1111.111 is NaN; largest finite 448), one byte per element:
+ *           codes [rows][k]; one E8M0 scale byte per 32 elements with the
+ *           MXFP4 scale layouts.  The block exponent is floor(log2 amax) - 8
+ *           (clamped to [-127, 127]); elements round to nearest even and
+ *           saturate at +-448.  An MXFP4 tensor re-encoded by rfq_convert is
+ *           an MXFP8 tensor holding the same values.
  */
 #ifndef RFQ_H
 #define RFQ_H
@@ -78,7 +86,7 @@ typedef enum {
     RFQ_ERR_DEVICE = 7       /* the current device is not an sm_103 GPU */
 } rfq_status;
 
-typedef enum { RFQ_FMT_MXFP4 = 0, RFQ_FMT_HIF4 = 1, RFQ_FMT_BF16 = 2 } rfq_format;
+typedef enum { RFQ_FMT_MXFP4 = 0, RFQ_FMT_HIF4 = 1, RFQ_FMT_BF16 = 2, RFQ_FMT_MXFP8 = 3 } rfq_format;
 
 typedef enum { RFQ_SCALE_ROWMAJOR = 0, RFQ_SCALE_MMA = 1 } rfq_scale_layout;
 
@@ -126,7 +134,8 @@ RFQ_API rfq_status rfq_qtensor_bytes(int32_t fmt, int32_t scale_layout, int64_t 
  * weight block).  W: device bf16 [K][N] row-major.  out->fmt,
  * out->scale_layout, out->codes and out->scales are set by the caller and
  * out->rows must equal N, out->k must equal K; codes are written K-major
- * ([N][K/2]).  Meant to run once per weight, off the hot path.
+ * ([N][K/2]; MXFP8: [N][K]).  Formats: MXFP4, HiF4, MXFP8 (the W8A8
+ * baseline of Table 1).  Meant to run once per weight, off the hot path.
  * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
  * RFQ_ERR_UNSUPPORTED, RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */
 RFQ_API rfq_status rfq_quantize_weight(const void *w_bf16, int64_t K, int64_t N, rfq_qtensor *out,
@@ -139,6 +148,13 @@ RFQ_API rfq_status rfq_quantize_weight(const void *w_bf16, int64_t K, int64_t N,
  * encoder.  X: device bf16 [M][K] row-major.  xq: main pathway output,
  * xr: residual pathway output (both with rows = M, k = K and the same fmt
  * and layout); xr may be NULL only when fb->mode == RFQ_FALLBACK_NONE.
+ * Two more format combinations:
+ *   xq MXFP4, xr MXFP8   the FP4-to-FP8 residual pathway named in Sec. 4.2:
+ *                        X~ = Q_MXFP4(X), X^ = Q_MXFP8(X - X~) (E4M3 scale
+ *                        floor(log2 amax) - 8), one pass over X;
+ *   xq MXFP8, no residual (fb->mode == RFQ_FALLBACK_NONE; a residual
+ *                        returns RFQ_ERR_UNSUPPORTED): X -> MXFP8, the
+ *                        activation of the W4A8 / W8A8 baselines (Table 1).
  * Residual codes and scales of tiles with phi = 0 are written as zero.
  * phi: device bytes [ceil(M/p_s)][ceil(K/r_s)], may be NULL; fb may be
  * NULL (= RFQ_FALLBACK_ALL).  M may be 0 (nothing is launched).
@@ -161,7 +177,10 @@ RFQ_API size_t rfq_linear_workspace_bytes(void);
  * products, at its own granularity (it may still include a phi = 0 tile that
  * shares a 256-row or 256-column block with a phi = 1 one).
  * wq: [N x K] weight.  MXFP4: every operand MXFP4 with RFQ_SCALE_MMA,
- * K % 128 == 0.  HiF4 (Sec. 3.3): wq is the exact bf16 expansion of the HiF4
+ * K % 128 == 0.  MXFP8: every operand MXFP8 (E4M3, kind::mxf8f6f4 MMAs)
+ * with RFQ_SCALE_MMA, K % 128 == 0 -- the W8A8 and W4A8 baselines (an MXFP4
+ * weight re-encoded by rfq_convert) and the FP4-to-FP8 RFQ (X~ re-encoded
+ * by rfq_convert, X^ from the MXFP8 residual pathway).  HiF4 (Sec. 3.3): wq is the exact bf16 expansion of the HiF4
  * weight (RFQ_FMT_BF16, from rfq_dequant), K % 64 == 0, phi_r_s a multiple
  * of 64, and xq/xr are either HiF4 with RFQ_SCALE_MMA metadata (expanded
  * exactly to bf16 in shared memory inside the GEMM) or their exact bf16
@@ -197,6 +216,15 @@ RFQ_API rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, cons
 RFQ_API rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, const rfq_qtensor *wq,
                                     const rfq_fallback *fb, void *y, int32_t out_dtype, void *workspace,
                                     void *stream);
+
+/* Exact re-encoding of an MXFP4 tensor as MXFP8 (every E2M1 value is an
+ * E4M3 value): dst codes [rows][k] E4M3 bytes, dst scales = src scales.
+ * src: fmt MXFP4; dst: fmt MXFP8, the same rows, k and scale layout; both
+ * device, caller-owned.  Used for the weight of the W4A8 baseline and the
+ * main activation of the FP4-to-FP8 RFQ.
+ * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
+ * RFQ_ERR_UNSUPPORTED (other formats), RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */
+RFQ_API rfq_status rfq_convert(const rfq_qtensor *src, rfq_qtensor *dst, void *stream);
 
 /* Synchronizes `stream` and returns the device status left in a workspace by
  * earlier calls (RFQ_OK or RFQ_ERR_TIMEOUT); clears it when `clear` != 0. */

@@ -54,7 +54,10 @@ rfq_status check_device()
 
 rfq_status from_cuda(cudaError_t e) { return e == cudaSuccess ? RFQ_OK : RFQ_ERR_CUDA; }
 
-bool fmt_ok(int32_t f) { return f == RFQ_FMT_MXFP4 || f == RFQ_FMT_HIF4 || f == RFQ_FMT_BF16; }
+bool fmt_ok(int32_t f)
+{
+    return f == RFQ_FMT_MXFP4 || f == RFQ_FMT_HIF4 || f == RFQ_FMT_BF16 || f == RFQ_FMT_MXFP8;
+}
 bool layout_ok(int32_t l) { return l == RFQ_SCALE_ROWMAJOR || l == RFQ_SCALE_MMA; }
 
 // Granule of the k axis for a format / scale layout.
@@ -145,7 +148,7 @@ rfq_status rfq_qtensor_bytes(int32_t fmt, int32_t scale_layout, int64_t rows, in
         return RFQ_ERR_INVALID_ARG;
     if (rows < 0 || k <= 0 || k % k_granule(fmt, scale_layout) != 0)
         return RFQ_ERR_SHAPE;
-    *codes_bytes = (size_t)rows * (size_t)(k / 2);
+    *codes_bytes = (size_t)rows * (size_t)(fmt == RFQ_FMT_MXFP8 ? k : k / 2);
     if (fmt == RFQ_FMT_BF16) {
         *codes_bytes = (size_t)rows * (size_t)k * 2;
         *scale_bytes = 0;
@@ -180,6 +183,8 @@ rfq_status rfq_quantize_weight(const void *w_bf16, int64_t K, int64_t N, rfq_qte
         return from_cuda(launch_weight_quant_mxfp4(w_bf16, K, N, out->codes, out->scales, out->scale_layout, st));
     if (out->fmt == RFQ_FMT_HIF4)
         return from_cuda(launch_weight_quant_hif4(w_bf16, K, N, out->codes, out->scales, out->scale_layout, st));
+    if (out->fmt == RFQ_FMT_MXFP8)
+        return from_cuda(launch_weight_quant_mxfp8(w_bf16, K, N, out->codes, out->scales, out->scale_layout, st));
     return RFQ_ERR_INVALID_ARG;
 }
 
@@ -203,8 +208,13 @@ rfq_status rfq_quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_
             return RFQ_ERR_INVALID_ARG;
         if ((s = check_qtensor(xr, M, K)) != RFQ_OK)
             return s;
-        if (xr->fmt != xq->fmt || xr->scale_layout != xq->scale_layout)
+        // the residual takes the main pathway's format, or MXFP8 under an
+        // MXFP4 main pathway (the FP4-to-FP8 residual of Sec. 4.2)
+        const bool fp8_res = xq->fmt == RFQ_FMT_MXFP4 && xr->fmt == RFQ_FMT_MXFP8;
+        if ((xr->fmt != xq->fmt && !fp8_res) || xr->scale_layout != xq->scale_layout)
             return RFQ_ERR_INVALID_ARG;
+        if (xq->fmt == RFQ_FMT_MXFP8)
+            return RFQ_ERR_UNSUPPORTED;   // an MXFP8 main pathway has no residual here
     }
     if (f.p_s < 1 || f.r_s < 32 || f.r_s % 32 != 0 || (xq->fmt == RFQ_FMT_HIF4 && f.r_s % 64 != 0))
         return RFQ_ERR_SHAPE;
@@ -219,6 +229,15 @@ rfq_status rfq_quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_
     if (M == 0)
         return RFQ_OK;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (xq->fmt == RFQ_FMT_MXFP8) {
+        if (phi)
+            if (cudaError_t e = launch_phi_fill(phi, (M + f.p_s - 1) / f.p_s * ((K + f.r_s - 1) / f.r_s), 0, st))
+                return from_cuda(e);
+        return from_cuda(launch_act_quant_mxfp8(x_bf16, M, K, xq->codes, xq->scales, xq->scale_layout, st));
+    }
+    if (res && xr->fmt == RFQ_FMT_MXFP8)
+        return from_cuda(launch_act_quant_rfq8(x_bf16, M, K, f.mode, f.tau, f.p_s, f.r_s, xq->codes, xq->scales,
+                                               xr->codes, xr->scales, phi, xq->scale_layout, st));
     if (xq->fmt == RFQ_FMT_MXFP4)
         return from_cuda(launch_act_quant_mxfp4(x_bf16, M, K, f.mode, f.tau, f.p_s, f.r_s, xq->codes, xq->scales,
                                                 res ? xr->codes : nullptr, res ? xr->scales : nullptr, phi,
@@ -265,11 +284,13 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
         if (xr->fmt != xq->fmt || xr->scale_layout != xq->scale_layout)
             return RFQ_ERR_INVALID_ARG;
     }
-    // operand formats: MXFP4 x MXFP4, or HiF4 (codes, or their exact bf16
+    // operand formats: MXFP4 x MXFP4; MXFP8 x MXFP8 (E4M3, also holding exact
+    // re-encodings of MXFP4 tensors); or HiF4 (codes, or their exact bf16
     // expansion) x the bf16 expansion of W~
     const bool bf16_act = xq->fmt == RFQ_FMT_BF16;
     const bool hif4 = xq->fmt == RFQ_FMT_HIF4 || bf16_act;
-    if (hif4 ? wq->fmt != RFQ_FMT_BF16 : wq->fmt != RFQ_FMT_MXFP4)
+    const bool f8 = xq->fmt == RFQ_FMT_MXFP8;
+    if (hif4 ? wq->fmt != RFQ_FMT_BF16 : wq->fmt != (f8 ? RFQ_FMT_MXFP8 : RFQ_FMT_MXFP4))
         return RFQ_ERR_INVALID_ARG;
     if (bf16_act && K % 64 != 0)
         return RFQ_ERR_SHAPE;
@@ -323,6 +344,7 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
     a.N = N;
     a.K = K;
     a.status = static_cast<int32_t *>(workspace);
+    a.f8 = f8;
     return from_cuda(launch_gemm_mxf4(a, st));
 }
 
@@ -406,10 +428,34 @@ rfq_status rfq_dequant(const rfq_qtensor *q, void *out, int32_t out_dtype, void 
     const bool bf16 = out_dtype == RFQ_OUT_BF16;
     if (q->fmt == RFQ_FMT_HIF4)
         return from_cuda(launch_dequant_hif4(q->codes, q->scales, q->rows, q->k, q->scale_layout, out, bf16, st));
+    if (q->fmt == RFQ_FMT_MXFP8)
+        return from_cuda(launch_dequant_mxfp8(q->codes, q->scales, q->rows, q->k, q->scale_layout, out, bf16, st));
     if (bf16)
         return from_cuda(launch_dequant_mxfp4_bf16(q->codes, q->scales, q->rows, q->k, q->scale_layout, out, st));
     return from_cuda(
         launch_dequant_mxfp4(q->codes, q->scales, q->rows, q->k, q->scale_layout, static_cast<float *>(out), st));
+}
+
+rfq_status rfq_convert(const rfq_qtensor *src, rfq_qtensor *dst, void *stream)
+{
+    if (!src || !dst)
+        return RFQ_ERR_INVALID_ARG;
+    rfq_status s = check_qtensor(src, src->rows, src->k);
+    if (s != RFQ_OK)
+        return s;
+    if ((s = check_qtensor(dst, src->rows, src->k)) != RFQ_OK)
+        return s;
+    if (src->fmt != RFQ_FMT_MXFP4 || dst->fmt != RFQ_FMT_MXFP8 || src->scale_layout != dst->scale_layout)
+        return RFQ_ERR_UNSUPPORTED;
+    if ((s = check_device()) != RFQ_OK)
+        return s;
+    if (src->rows == 0)
+        return RFQ_OK;
+    size_t cb = 0, sb = 0;
+    if ((s = rfq_qtensor_bytes(src->fmt, src->scale_layout, src->rows, src->k, &cb, &sb)) != RFQ_OK)
+        return s;
+    return from_cuda(launch_convert_mxfp4_mxfp8(src->codes, src->scales, src->rows, src->k, sb, dst->codes,
+                                                dst->scales, static_cast<cudaStream_t>(stream)));
 }
 
 } // extern "C"

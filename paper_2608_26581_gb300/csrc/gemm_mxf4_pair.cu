@@ -142,7 +142,10 @@ struct Mask {
     static constexpr uint32_t value = V;
 };
 
-template <bool RES, bool PHI, bool OUT_BF16>
+// F8: every operand holds E4M3 codes (one byte per element, kind::mxf8f6f4
+// MMAs of K = 32 with one scale per row each); a stage is then one
+// 128-element chunk (the same 128-byte rows).
+template <bool RES, bool PHI, bool OUT_BF16, bool F8>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     gemm_mxf4_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmR,
                           const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmY,
@@ -158,8 +161,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
     const volatile int32_t *gstat = status;
 
     const int kc = K >> 7;                  // 128-element chunks
-    const int nks = (kc + 1) >> 1;          // 256-element stages (the last may hold one chunk)
-    const int nf = kc >> 1;                 // stages with two chunks
+    constexpr int CPS = F8 ? 1 : 2;        // 128-element chunks per stage (128-byte rows either way)
+    const int nks = (kc + CPS - 1) / CPS;   // stages (with MXFP4 the last may hold one chunk)
+    const int nf = kc / CPS;                // stages with CPS chunks
     const int n_tiles = (N + BN - 1) / BN;
     const int m_tiles = (M + BM - 1) / BM;  // 128-row tiles: scale atoms and phi rows
     const int m_pairs = (M + 2 * BM - 1) / (2 * BM);
@@ -228,7 +232,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                         stop = true;
                         return;
                     }
-                    const int c0 = 2 * ks;
+                    const int c0 = CPS * ks, cx = c0 * (F8 ? 128 : 64); // first chunk, its byte column
                     if (PHI)
                         S.stage_info[slot] = info;
                     Stage &st = S.st[slot];
@@ -237,10 +241,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     uint64_t *sbar = &S.sf_full[slot];
                     if (lead)
                         mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES + B_BYTES + (res_on ? A_BYTES : 0)));
-                    tma_load_2d_pair(st.a, &tmA, bar, c0 * 64, m_tile * BM);
+                    tma_load_2d_pair(st.a, &tmA, bar, cx, m_tile * BM);
                     if (res_on)
-                        tma_load_2d_pair(st.r, &tmR, bar, c0 * 64, m_tile * BM);
-                    tma_load_2d_pair(st.b, &tmB, bar, c0 * 64, n_tile * BN + (int)rank * BN_HALF);
+                        tma_load_2d_pair(st.r, &tmR, bar, cx, m_tile * BM);
+                    tma_load_2d_pair(st.b, &tmB, bar, cx, n_tile * BN + (int)rank * BN_HALF);
                     mbar_arrive_expect_tx(sbar, nb * sfbytes + (rows_in ? (res_on ? 2 : 1) * sfbytes : 0));
                     if (rows_in) {
                         bulk_load(st.sfa, sfa + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, sbar);
@@ -255,7 +259,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 if constexpr (!PHI) {
                     // full stages, then an odd last chunk (chunk counts known at compile time)
                     for (int ks = 0; ks < nf && !stop; ++ks)
-                        produce(ks, 2, 0u, Bool<RES>{});
+                        produce(ks, CPS, 0u, Bool<RES>{});
                     if (nf < nks && !stop)
                         produce(nf, 1, 0u, Bool<RES>{});
                 } else {
@@ -273,7 +277,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                         while (x != 0 && !stop) {
                             const int b = __ffs(x) - 1;
                             x &= x - 1;
-                            produce(32 * w + b, 2, info, Bool<true>{});
+                            produce(32 * w + b, CPS, info, Bool<true>{});
                         }
                     }
                     for (int w = 0; 32 * w < nf && !stop; ++w) {
@@ -282,7 +286,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                         while (x != 0 && !stop) {
                             const int b = __ffs(x) - 1;
                             x &= x - 1;
-                            produce(32 * w + b, 2, info, Bool<false>{});
+                            produce(32 * w + b, CPS, info, Bool<false>{});
                         }
                     }
                     if (nf < nks && !stop) {   // the odd last chunk
@@ -331,22 +335,34 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     const uint32_t a0 = smem_u32(st.a), r0 = smem_u32(st.r), b0 = smem_u32(st.b);
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
-                        const int c = j >> 1;
+                        const int c = F8 ? 0 : j >> 1;
                         if (c >= nch)
                             break;
-                        const uint32_t id = idesc_mxf4(2 * BM, BN, 2 * (j & 1), 2 * (j & 1));
+                        // MXFP4: K = 64 per MMA, scale bytes 2 (j & 1) and up; E4M3: K = 32, byte j
+                        const uint32_t id = F8 ? idesc_mxf8(2 * BM, BN, j, j)
+                                               : idesc_mxf4(2 * BM, BN, 2 * (j & 1), 2 * (j & 1));
                         const uint64_t bd = sdesc_k_sw128(b0 + 32 * j);
                         const uint32_t sfb_t = sf + 16 + 8 * c;
-                        tc_mma_mxf4_pair(tmem, sdesc_k_sw128(a0 + 32 * j), bd, id, sf + 4 * c, sfb_t, (pos | j) != 0);
+                        if (F8)
+                            tc_mma_mxf8_pair(tmem, sdesc_k_sw128(a0 + 32 * j), bd, id, sf + 4 * c, sfb_t,
+                                             (pos | j) != 0);
+                        else
+                            tc_mma_mxf4_pair(tmem, sdesc_k_sw128(a0 + 32 * j), bd, id, sf + 4 * c, sfb_t,
+                                             (pos | j) != 0);
                         if ((rm >> c) & 1)
-                            tc_mma_mxf4_pair(tmem, sdesc_k_sw128(r0 + 32 * j), bd, id, sf + 8 + 4 * c, sfb_t, 1);
+                        {
+                            if (F8)
+                                tc_mma_mxf8_pair(tmem, sdesc_k_sw128(r0 + 32 * j), bd, id, sf + 8 + 4 * c, sfb_t, 1);
+                            else
+                                tc_mma_mxf4_pair(tmem, sdesc_k_sw128(r0 + 32 * j), bd, id, sf + 8 + 4 * c, sfb_t, 1);
+                        }
                     }
                     tc_commit_pair_mc(&S.empty[slot], 0x3);
                     ++p;
                 };
                 if constexpr (!PHI) {
                     for (int ks = 0; ks < nf && !stop; ++ks)
-                        mma_stage(ks, 2, Mask<RES ? 3u : 0u>{});
+                        mma_stage(ks, CPS, Mask<RES ? 3u : 0u>{});
                     if (nf < nks && !stop)
                         mma_stage(nf, 1, Mask<RES ? 1u : 0u>{});
                 } else {
@@ -359,9 +375,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     const int n_res = (int)(info & 0x7fffffffu);
                     int pos = 0;
                     for (; pos < n_res && !stop; ++pos)
-                        mma_stage(pos, 2, Mask<3u>{});
+                        mma_stage(pos, CPS, Mask<3u>{});
                     for (; pos < nf && !stop; ++pos)
-                        mma_stage(pos, 2, Mask<0u>{});
+                        mma_stage(pos, CPS, Mask<0u>{});
                     if (nf < nks && !stop) {
                         if (info >> 31)
                             mma_stage(pos, 1, Mask<1u>{});
@@ -545,7 +561,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
             };
             if constexpr (!PHI) {
                 for (int ks = 0; ks < nf && !stop; ++ks)
-                    write_stage(2, Mask<RES ? 3u : 0u>{});
+                    write_stage(CPS, Mask<RES ? 3u : 0u>{});
                 if (nf < nks && !stop)
                     write_stage(1, Mask<RES ? 1u : 0u>{});
             } else {
@@ -559,9 +575,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 const int n_res = (int)(info & 0x7fffffffu);
                 int pos = 0;
                 for (; pos < n_res && !stop; ++pos)
-                    write_stage(2, Mask<3u>{});
+                    write_stage(CPS, Mask<3u>{});
                 for (; pos < nf && !stop; ++pos)
-                    write_stage(2, Mask<0u>{});
+                    write_stage(CPS, Mask<0u>{});
                 if (nf < nks && !stop) {
                     if (info >> 31)
                         write_stage(1, Mask<1u>{});
@@ -600,13 +616,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
             uint32_t n_res = 0;
             for (int w = 0; 32 * w < nf; ++w) {
                 const int ks = 32 * w + lane;
-                const bool on = ks < nf && (chunk_on(m_pair, 2 * ks) || chunk_on(m_pair, 2 * ks + 1));
+                const bool on = ks < nf && (chunk_on(m_pair, CPS * ks) || (!F8 && chunk_on(m_pair, CPS * ks + 1)));
                 const uint32_t word = __ballot_sync(0xffffffffu, on);
                 if (lane == 0)
                     rec.bits[w] = word;
                 n_res += __popc(word);
             }
-            const uint32_t tail = nf < nks && chunk_on(m_pair, 2 * nf) ? 1u : 0u;
+            const uint32_t tail = nf < nks && chunk_on(m_pair, CPS * nf) ? 1u : 0u;
             if (lane == 0)
                 rec.info = n_res | tail << 31;
             mbar_arrive(&S.phi_full[r]);
@@ -623,11 +639,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
     }
 }
 
-template <bool RES, bool PHI, bool OUT>
+template <bool RES, bool PHI, bool OUT, bool F8>
 cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const CUtensorMap &tb,
                            const CUtensorMap &ty, const GemmMxf4Args &a, cudaStream_t st)
 {
-    auto kern = gemm_mxf4_pair_kernel<RES, PHI, OUT>;
+    auto kern = gemm_mxf4_pair_kernel<RES, PHI, OUT, F8>;
     static int max_pairs = 0; // per variant: clusters of two that fit on the device at once
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (e != cudaSuccess)
@@ -658,7 +674,7 @@ cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const C
 cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
 {
     CUtensorMap ta, tr, tb, ty;
-    const uint64_t kb = (uint64_t)a.K / 2;
+    const uint64_t kb = a.f8 ? (uint64_t)a.K : (uint64_t)a.K / 2; // code bytes per row
     if (!encode_tmap_2d_u8(&ta, a.a_codes, kb, (uint64_t)a.M, kb, ROW, BM, 128) ||
         !encode_tmap_2d_u8(&tb, a.b_codes, kb, (uint64_t)a.N, kb, ROW, BN_HALF, 128))
         return cudaErrorInvalidValue;
@@ -675,8 +691,10 @@ cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
     // Beyond REC_WORDS * 32 full k-stages the record does not fit: every
     // residual product is then issued (exact: phi = 0 residuals are zero).
     const bool res = a.r_codes != nullptr;
-    const bool phi = res && a.phi != nullptr && a.K / 256 <= REC_WORDS * 32;
-#define RFQ_GV(R, P, O) return launch_variant<R, P, O>(ta, tr, tb, ty, a, st)
+    const bool phi = res && a.phi != nullptr && a.K / (a.f8 ? 128 : 256) <= REC_WORDS * 32;
+#define RFQ_GV(R, P, O)                                                                                           \
+    return a.f8 ? launch_variant<R, P, O, true>(ta, tr, tb, ty, a, st)                                            \
+                : launch_variant<R, P, O, false>(ta, tr, tb, ty, a, st)
     if (!res) {
         if (a.out_bf16) RFQ_GV(false, false, true);
         RFQ_GV(false, false, false);

@@ -23,6 +23,19 @@ __host__ __device__ inline int64_t sf_mma_offset(int64_t m, int64_t b, int64_t k
     return (((m >> 7) * kc + (b >> 2)) << 9) + ((m & 31) << 4) + (((m >> 5) & 3) << 2) + (b & 3);
 }
 
+// ---- MXFP8 (E4M3) quantization and the FP4-to-FP8 residual (quant_mxfp8.cu)
+cudaError_t launch_act_quant_mxfp8(const void *x, int64_t M, int64_t K, void *codes, void *scales, int layout,
+                                   cudaStream_t st);
+cudaError_t launch_act_quant_rfq8(const void *x, int64_t M, int64_t K, int mode, float tau, int p_s, int r_s,
+                                  void *mcodes, void *mscales, void *rcodes, void *rscales, uint8_t *phi, int layout,
+                                  cudaStream_t st);
+cudaError_t launch_weight_quant_mxfp8(const void *w, int64_t K, int64_t N, void *codes, void *scales, int layout,
+                                      cudaStream_t st);
+cudaError_t launch_convert_mxfp4_mxfp8(const void *src_codes, const void *src_scales, int64_t rows, int64_t k,
+                                       size_t scale_bytes, void *dst_codes, void *dst_scales, cudaStream_t st);
+cudaError_t launch_dequant_mxfp8(const void *codes, const void *scales, int64_t rows, int64_t k, int layout, void *out,
+                                 bool bf16, cudaStream_t st);
+
 // ---- MXFP4 quantization (quant_mxfp4.cu)
 // Activation: main (+ residual) codes and scales in one pass over X.
 cudaError_t launch_act_quant_mxfp4(const void *x, int64_t M, int64_t K, int mode, float tau, int p_s, int r_s,
@@ -39,7 +52,7 @@ cudaError_t launch_dequant_mxfp4(const void *codes, const void *scales, int64_t 
 
 // ---- MXFP4 RFQ GEMM (gemm_mxf4.cu)
 struct GemmMxf4Args {
-    const void *a_codes, *r_codes, *b_codes;   // [M][K/2], [M][K/2] or null, [N][K/2]
+    const void *a_codes, *r_codes, *b_codes;   // [M][K/2], [M][K/2] or null, [N][K/2] (f8: [..][K] E4M3)
     const void *a_sf, *r_sf, *b_sf;            // MMA-layout scales
     const uint8_t *phi;                        // [ceil(M/128)][K/phi_r_s] or null
     int phi_r_s;
@@ -47,6 +60,7 @@ struct GemmMxf4Args {
     int out_bf16;
     int64_t M, N, K;
     int32_t *status;
+    int f8 = 0;                                // every operand MXFP8 (E4M3): kind::mxf8f6f4, CTA pairs
 };
 cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st);
 // CTA-pair kernel (gemm_mxf4_pair.cu), used by launch_gemm_mxf4 when M > 128.

@@ -292,6 +292,20 @@ __device__ __forceinline__ void tc_mma_mxf4_pair(uint32_t d_tmem, uint64_t a_des
         : "memory");
 }
 
+// CTA-pair MMA with E4M3 operands (kind::mxf8f6f4, scale_vec::1X: one E8M0
+// scale per row per K=32 instruction).
+__device__ __forceinline__ void tc_mma_mxf8_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                                 uint32_t sfa_tmem, uint32_t sfb_tmem, uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %6, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], %1, %2, %3, [%4], [%5], p;\n\t}" ::"r"(
+            d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(sfa_tmem), "r"(sfb_tmem), "r"(accumulate)
+        : "memory");
+}
+
 // Arrive on the mbarrier at this shared offset in every CTA of `cta_mask`
 // once every tcgen05 operation issued so far by this thread (for the pair)
 // has completed.
@@ -409,6 +423,15 @@ __device__ __forceinline__ uint64_t sdesc_rows16(uint32_t saddr)
 __host__ __device__ constexpr uint32_t idesc_mxf4(int M, int N, int sfa_id, int sfb_id)
 {
     return ((uint32_t)sfb_id << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | (1u << 23) |
+           ((uint32_t)(M >> 4) << 24) | ((uint32_t)sfa_id << 29);
+}
+
+// Instruction descriptor, kind::mxf8f6f4: E4M3 x E4M3 (format code 0 for
+// both), UE8M0 scales, both operands K-major; sfa_id / sfb_id pick the byte
+// of the 32-bit scale word used by this K=32 instruction (0..3).
+__host__ __device__ constexpr uint32_t idesc_mxf8(int M, int N, int sfa_id, int sfb_id)
+{
+    return ((uint32_t)sfb_id << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(N >> 3) << 17) | (1u << 23) |
            ((uint32_t)(M >> 4) << 24) | ((uint32_t)sfa_id << 29);
 }
 

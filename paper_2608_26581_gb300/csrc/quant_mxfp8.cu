@@ -1,0 +1,376 @@
+// quant_mxfp8.cu -- MXFP8 (E4M3) quantizers (Sec. 3.2.1 with the block rule
+// of Sec. 3.2 Eqs. 3-4) and the FP4-to-FP8 residual pathway (Sec. 4.2,
+// Sec. 4.3):
+//   act_quant_mxfp8      X -> E4M3 codes + E8M0 scales (W4A8 / W8A8 activations)
+//   act_quant_rfq8       X~ = Q_MXFP4(X) and X^ = Q_MXFP8(X - X~) in one pass
+//   weight_quant_mxfp8   W [K x N] -> K-major E4M3 codes + scales
+//   convert_mxfp4_mxfp8  MXFP4 codes -> E4M3 codes of the same values (exact:
+//                        every E2M1 value is an E4M3 value), scales unchanged
+//   dequant_mxfp8        codes x scales -> fp32 or bf16
+// The E8M0 byte of an E4M3 block is the fp32 exponent field of its amax
+// minus 8 (floor(log2 amax) - 8, clamped at 0); x 2^-e is exact, and
+// cvt.rn.satfinite.e4m3x2 rounds to nearest even and saturates at +-448.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cstdint>
+
+#include "internal.h"
+#include "mxfp4_math.cuh"
+
+namespace rfq {
+namespace {
+
+template <int LAYOUT>
+__device__ __forceinline__ int64_t scale_index8(int64_t m, int64_t b, int64_t kblocks)
+{
+    if (LAYOUT == RFQ_SCALE_MMA)
+        return sf_mma_offset(m, b, kblocks >> 2);
+    return m * kblocks + b;
+}
+
+// E8M0 byte of an E4M3 block from the fp32 bits of its amax.
+__device__ __forceinline__ int scale8_byte_from_f32_bits(uint32_t amax_bits)
+{
+    return max((int)((amax_bits >> 23) & 0xFF) - 8, 0);
+}
+
+// Eight fp32 values -> eight E4M3 codes (element i in byte i).
+__device__ __forceinline__ uint2 e4m3x8(const float (&y)[8])
+{
+    uint32_t lo, hi;
+    asm("{\n\t.reg .b16 h0, h1, h2, h3;\n\t"
+        "cvt.rn.satfinite.e4m3x2.f32 h0, %3, %2;\n\t"
+        "cvt.rn.satfinite.e4m3x2.f32 h1, %5, %4;\n\t"
+        "cvt.rn.satfinite.e4m3x2.f32 h2, %7, %6;\n\t"
+        "cvt.rn.satfinite.e4m3x2.f32 h3, %9, %8;\n\t"
+        "mov.b32 %0, {h0, h1};\n\t"
+        "mov.b32 %1, {h2, h3};\n\t}"
+        : "=r"(lo), "=r"(hi)
+        : "f"(y[0]), "f"(y[1]), "f"(y[2]), "f"(y[3]), "f"(y[4]), "f"(y[5]), "f"(y[6]), "f"(y[7]));
+    return make_uint2(lo, hi);
+}
+
+// Two E4M3 codes (a 16-bit pair) -> two floats (exact through f16).
+__device__ __forceinline__ void e4m3x2_decode(uint32_t pair, float &a, float &b)
+{
+    uint32_t h;
+    asm("{\n\t.reg .b16 p;\n\tcvt.u16.u32 p, %1;\n\tcvt.rn.f16x2.e4m3x2 %0, p;\n\t}" : "=r"(h) : "r"(pair));
+    const __half2 v = *reinterpret_cast<const __half2 *>(&h);
+    a = __low2float(v);
+    b = __high2float(v);
+}
+
+// Block-max of this lane's eight values over the four lanes of its block.
+__device__ __forceinline__ float block_amax(const float (&v)[8])
+{
+    float am = absmax8(v);
+    am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 1));
+    return fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 2));
+}
+
+// E4M3 codes and E8M0 byte of this lane's eight values (its block spans
+// four lanes; all 32 lanes take part).
+__device__ __forceinline__ uint2 mxfp8_quant8(const float (&xf)[8], int &sb)
+{
+    sb = scale8_byte_from_f32_bits(__float_as_uint(block_amax(xf)));
+    const float inv = pow2_neg_e(sb);
+    float y[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+        y[i] = xf[i] * inv;
+    return e4m3x8(y);
+}
+
+constexpr int kSeg = 1024;   // elements per (row, segment) item of a warp
+constexpr int kU = kSeg / 256;
+
+// One warp per (row, 1024-element segment); four lanes per 32-element block.
+// RFQ8 = false: X -> MXFP8.  RFQ8 = true: X -> MXFP4 main codes and the
+// MXFP8 residual X - X~ (zero on phi = 0 tiles when PHI).
+template <bool RFQ8, bool PHI, int LAYOUT>
+__global__ void __launch_bounds__(256) act_quant8_kernel(const uint4 *__restrict__ x, int64_t M, int64_t K,
+                                                        uint8_t *__restrict__ mcodes, uint8_t *__restrict__ mscales,
+                                                        uint8_t *__restrict__ rcodes, uint8_t *__restrict__ rscales,
+                                                        const uint8_t *__restrict__ phi, int p_s, int r_s,
+                                                        int64_t pad_rows)
+{
+    const int lane = threadIdx.x & 31;
+    const int kchunks = (int)(K >> 3);
+    const int kblocks = (int)(K >> 5);
+    const int segs = (kchunks + kSeg / 8 - 1) / (kSeg / 8);
+    const int64_t items = M * segs;
+    const int64_t gwarp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+
+    if (LAYOUT == RFQ_SCALE_MMA && pad_rows > 0) {
+        const int64_t n = pad_rows * kblocks;
+        for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+            const int64_t off = scale_index8<LAYOUT>(M + i / kblocks, i % kblocks, kblocks);
+            mscales[off] = 0;
+            if (RFQ8)
+                rscales[off] = 0;
+        }
+    }
+
+    for (int64_t it = gwarp; it < items; it += nwarps) {
+        const int64_t m = it / segs;
+        const int c0 = (int)(it - m * segs) * (kSeg / 8);
+        const uint4 *xr = x + m * kchunks;
+        uint4 v[kU];
+#pragma unroll
+        for (int j = 0; j < kU; ++j) {
+            const int c = c0 + j * 32 + lane;
+            v[j] = c < kchunks ? __ldcs(xr + c) : make_uint4(0, 0, 0, 0);
+        }
+        const uint8_t *prow = PHI ? phi + (m / p_s) * ((K + r_s - 1) / r_s) : nullptr;
+#pragma unroll
+        for (int j = 0; j < kU; ++j) {
+            const int c = c0 + j * 32 + lane;
+            const bool ok = c < kchunks; // uniform over each group of 4 lanes
+            const int64_t soff = scale_index8<LAYOUT>(m, c >> 2, kblocks);
+            float xf[8];
+            bf16x8_to_f32(v[j], xf);
+            if (!RFQ8) {
+                int sb;
+                const uint2 q = mxfp8_quant8(xf, sb);
+                if (ok) {
+                    *reinterpret_cast<uint2 *>(mcodes + m * K + (int64_t)c * 8) = q;
+                    if ((lane & 3) == 0)
+                        mscales[soff] = (uint8_t)sb;
+                }
+            } else {
+                const Mx8 q4 = mxfp4_quant8<false>(xf);
+                // the residual x - x~, exact in fp32
+                float q[8], r[8];
+                e2m1x8_decode(q4.code, q);
+                const float sc = pow2_e(q4.sb);
+#pragma unroll
+                for (int i = 0; i < 8; ++i)
+                    r[i] = fmaf(-q[i], sc, xf[i]);
+                int rb;
+                const uint2 rq = mxfp8_quant8(r, rb);
+                const bool on = !PHI || (ok && prow[(c * 8) / r_s] != 0);
+                if (ok) {
+                    reinterpret_cast<uint32_t *>(mcodes + m * (K >> 1))[c] = q4.code;
+                    *reinterpret_cast<uint2 *>(rcodes + m * K + (int64_t)c * 8) = on ? rq : make_uint2(0, 0);
+                    if ((lane & 3) == 0) {
+                        mscales[soff] = (uint8_t)q4.sb;
+                        rscales[soff] = on ? (uint8_t)rb : 0;
+                    }
+                }
+            }
+        }
+    }
+}
+
+// One thread per (column n, 32-block b) of W [K x N].
+template <int LAYOUT>
+__global__ void __launch_bounds__(256) weight_quant_mxfp8_kernel(const __nv_bfloat16 *__restrict__ w, int64_t K,
+                                                                int64_t N, int64_t Npad, uint8_t *__restrict__ codes,
+                                                                uint8_t *__restrict__ scales)
+{
+    const int64_t kblocks = K >> 5;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t n = t % Npad, b = t / Npad;
+    if (b >= kblocks)
+        return;
+    if (n >= N) {
+        if (LAYOUT == RFQ_SCALE_MMA)
+            scales[scale_index8<LAYOUT>(n, b, kblocks)] = 0;
+        return;
+    }
+    float xf[32];
+    uint32_t am = 0;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+        const uint16_t bits = __bfloat16_as_ushort(w[(b * 32 + i) * N + n]);
+        am = max(am, (uint32_t)(bits & 0x7FFF));
+        xf[i] = __uint_as_float((uint32_t)bits << 16);
+    }
+    const int sb = scale8_byte_from_f32_bits(am << 16);
+    const float inv = pow2_neg_e(sb);
+    uint4 *dst = reinterpret_cast<uint4 *>(codes + n * K + b * 32);
+#pragma unroll
+    for (int g = 0; g < 2; ++g) {
+        float y0[8], y1[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            y0[i] = xf[g * 16 + i] * inv;
+            y1[i] = xf[g * 16 + 8 + i] * inv;
+        }
+        const uint2 a = e4m3x8(y0), c = e4m3x8(y1);
+        dst[g] = make_uint4(a.x, a.y, c.x, c.y);
+    }
+    scales[scale_index8<LAYOUT>(n, b, kblocks)] = (uint8_t)sb;
+}
+
+// E2M1 code -> E4M3 code of the same value: sign moves to bit 7; the
+// magnitudes 0, 0.5, 1, 1.5, 2, 3, 4, 6 are 0x00, 0x30, 0x38, 0x3C, 0x40,
+// 0x44, 0x48, 0x4C (exponent field e + 7, mantissa m / 8).
+__device__ __forceinline__ uint32_t e2m1_to_e4m3(uint32_t c)
+{
+    const uint32_t mag = c & 7u;
+    uint32_t code = 0;
+    if (mag == 1)
+        code = 6u << 3;                                            // 0.5 = 2^-1
+    else if (mag >= 2)
+        code = (((mag >> 1) + 6u) << 3) | ((mag & 1u) << 2);      // 2^(k-1) (1 + m/2), k = mag / 2
+    return ((c & 8u) << 4) | code;
+}
+
+// One thread per 8 elements: 4 bytes of MXFP4 codes -> 8 bytes of E4M3.
+__global__ void convert_mxfp4_mxfp8_kernel(const uint32_t *__restrict__ src, uint2 *__restrict__ dst, int64_t n8)
+{
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n8; i += (int64_t)gridDim.x * blockDim.x) {
+        const uint32_t w = src[i];
+        uint32_t lo = 0, hi = 0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            lo |= e2m1_to_e4m3((w >> (4 * j)) & 0xFu) << (8 * j);
+            hi |= e2m1_to_e4m3((w >> (16 + 4 * j)) & 0xFu) << (8 * j);
+        }
+        dst[i] = make_uint2(lo, hi);
+    }
+}
+
+template <int LAYOUT, bool BF16>
+__global__ void dequant_mxfp8_kernel(const uint2 *__restrict__ codes, const uint8_t *__restrict__ scales, int64_t rows,
+                                     int64_t k, void *__restrict__ out)
+{
+    const int64_t kchunks = k >> 3;
+    for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < rows * kchunks;
+         c += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t m = c / kchunks, cc = c % kchunks;
+        const float s = pow2_e(scales[scale_index8<LAYOUT>(m, cc >> 2, k >> 5)]);
+        const uint2 w = codes[c];
+        float q[8];
+        e4m3x2_decode(w.x & 0xFFFFu, q[0], q[1]);
+        e4m3x2_decode(w.x >> 16, q[2], q[3]);
+        e4m3x2_decode(w.y & 0xFFFFu, q[4], q[5]);
+        e4m3x2_decode(w.y >> 16, q[6], q[7]);
+        if (BF16) {
+            uint32_t p[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                // exact unless below bf16's normal range (round-to-nearest-even there)
+                __nv_bfloat162 b = __floats2bfloat162_rn(q[2 * i] * s, q[2 * i + 1] * s);
+                p[i] = *reinterpret_cast<uint32_t *>(&b);
+            }
+            static_cast<uint4 *>(out)[c] = make_uint4(p[0], p[1], p[2], p[3]);
+        } else {
+            float4 *o = reinterpret_cast<float4 *>(static_cast<float *>(out) + c * 8);
+            o[0] = make_float4(q[0] * s, q[1] * s, q[2] * s, q[3] * s);
+            o[1] = make_float4(q[4] * s, q[5] * s, q[6] * s, q[7] * s);
+        }
+    }
+}
+
+int grid8(int64_t work, int threads, int max_blocks)
+{
+    int64_t b = (work + threads - 1) / threads;
+    if (b > max_blocks)
+        b = max_blocks;
+    return (int)(b < 1 ? 1 : b);
+}
+
+} // namespace
+
+cudaError_t launch_act_quant_mxfp8(const void *x, int64_t M, int64_t K, void *codes, void *scales, int layout,
+                                   cudaStream_t st)
+{
+    const int64_t pad = layout == RFQ_SCALE_MMA ? ((M + 127) / 128) * 128 - M : 0;
+    const int64_t warps = M * ((K + kSeg - 1) / kSeg);
+    const int blocks = grid8(warps * 32 > pad * (K / 32) ? warps * 32 : pad * (K / 32), 256, 152 * 24);
+    auto *xi = static_cast<const uint4 *>(x);
+    auto *c = static_cast<uint8_t *>(codes);
+    auto *s = static_cast<uint8_t *>(scales);
+    if (layout == RFQ_SCALE_MMA)
+        act_quant8_kernel<false, false, RFQ_SCALE_MMA><<<blocks, 256, 0, st>>>(xi, M, K, c, s, nullptr, nullptr,
+                                                                             nullptr, 1, 32, pad);
+    else
+        act_quant8_kernel<false, false, RFQ_SCALE_ROWMAJOR><<<blocks, 256, 0, st>>>(xi, M, K, c, s, nullptr, nullptr,
+                                                                                  nullptr, 1, 32, pad);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_act_quant_rfq8(const void *x, int64_t M, int64_t K, int mode, float tau, int p_s, int r_s,
+                                  void *mcodes, void *mscales, void *rcodes, void *rscales, uint8_t *phi, int layout,
+                                  cudaStream_t st)
+{
+    if (mode == RFQ_FALLBACK_AMAX) {
+        cudaError_t e = launch_phi_amax(x, M, K, p_s, r_s, tau, phi, st);
+        if (e != cudaSuccess)
+            return e;
+    } else if (phi) {
+        cudaError_t e = launch_phi_fill(phi, (M + p_s - 1) / p_s * ((K + r_s - 1) / r_s), 1, st);
+        if (e != cudaSuccess)
+            return e;
+    }
+    const int64_t pad = layout == RFQ_SCALE_MMA ? ((M + 127) / 128) * 128 - M : 0;
+    const int64_t warps = M * ((K + kSeg - 1) / kSeg);
+    const int blocks = grid8(warps * 32 > pad * (K / 32) ? warps * 32 : pad * (K / 32), 256, 152 * 24);
+    auto *xi = static_cast<const uint4 *>(x);
+    auto *mc = static_cast<uint8_t *>(mcodes);
+    auto *ms = static_cast<uint8_t *>(mscales);
+    auto *rc = static_cast<uint8_t *>(rcodes);
+    auto *rs = static_cast<uint8_t *>(rscales);
+    const bool sel = mode == RFQ_FALLBACK_AMAX;
+#define RFQ_AQ8(PHI, LAY) \
+    act_quant8_kernel<true, PHI, LAY><<<blocks, 256, 0, st>>>(xi, M, K, mc, ms, rc, rs, phi, p_s, r_s, pad)
+    if (layout == RFQ_SCALE_MMA) {
+        if (sel) RFQ_AQ8(true, RFQ_SCALE_MMA);
+        else RFQ_AQ8(false, RFQ_SCALE_MMA);
+    } else {
+        if (sel) RFQ_AQ8(true, RFQ_SCALE_ROWMAJOR);
+        else RFQ_AQ8(false, RFQ_SCALE_ROWMAJOR);
+    }
+#undef RFQ_AQ8
+    return cudaGetLastError();
+}
+
+cudaError_t launch_weight_quant_mxfp8(const void *w, int64_t K, int64_t N, void *codes, void *scales, int layout,
+                                      cudaStream_t st)
+{
+    const int64_t Npad = layout == RFQ_SCALE_MMA ? ((N + 127) / 128) * 128 : N;
+    const int64_t work = Npad * (K / 32);
+    const int blocks = (int)((work + 255) / 256);
+    auto *wi = static_cast<const __nv_bfloat16 *>(w);
+    if (layout == RFQ_SCALE_MMA)
+        weight_quant_mxfp8_kernel<RFQ_SCALE_MMA><<<blocks, 256, 0, st>>>(wi, K, N, Npad, static_cast<uint8_t *>(codes),
+                                                                        static_cast<uint8_t *>(scales));
+    else
+        weight_quant_mxfp8_kernel<RFQ_SCALE_ROWMAJOR><<<blocks, 256, 0, st>>>(
+            wi, K, N, Npad, static_cast<uint8_t *>(codes), static_cast<uint8_t *>(scales));
+    return cudaGetLastError();
+}
+
+cudaError_t launch_convert_mxfp4_mxfp8(const void *src_codes, const void *src_scales, int64_t rows, int64_t k,
+                                       size_t scale_bytes, void *dst_codes, void *dst_scales, cudaStream_t st)
+{
+    const int64_t n8 = rows * (k / 8);
+    convert_mxfp4_mxfp8_kernel<<<grid8(n8, 256, 152 * 16), 256, 0, st>>>(static_cast<const uint32_t *>(src_codes),
+                                                                         static_cast<uint2 *>(dst_codes), n8);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess)
+        return e;
+    return cudaMemcpyAsync(dst_scales, src_scales, scale_bytes, cudaMemcpyDeviceToDevice, st);
+}
+
+cudaError_t launch_dequant_mxfp8(const void *codes, const void *scales, int64_t rows, int64_t k, int layout, void *out,
+                                 bool bf16, cudaStream_t st)
+{
+    const int64_t n = rows * (k / 8);
+    const int blocks = grid8(n, 256, 152 * 16);
+    auto *c = static_cast<const uint2 *>(codes);
+    auto *s = static_cast<const uint8_t *>(scales);
+    if (layout == RFQ_SCALE_MMA) {
+        if (bf16) dequant_mxfp8_kernel<RFQ_SCALE_MMA, true><<<blocks, 256, 0, st>>>(c, s, rows, k, out);
+        else dequant_mxfp8_kernel<RFQ_SCALE_MMA, false><<<blocks, 256, 0, st>>>(c, s, rows, k, out);
+    } else {
+        if (bf16) dequant_mxfp8_kernel<RFQ_SCALE_ROWMAJOR, true><<<blocks, 256, 0, st>>>(c, s, rows, k, out);
+        else dequant_mxfp8_kernel<RFQ_SCALE_ROWMAJOR, false><<<blocks, 256, 0, st>>>(c, s, rows, k, out);
+    }
+    return cudaGetLastError();
+}
+
+} // namespace rfq

@@ -16,7 +16,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "librfq.so")
 
 RFQ_OK = 0
-RFQ_FMT_MXFP4, RFQ_FMT_HIF4, RFQ_FMT_BF16 = 0, 1, 2
+RFQ_FMT_MXFP4, RFQ_FMT_HIF4, RFQ_FMT_BF16, RFQ_FMT_MXFP8 = 0, 1, 2, 3
 RFQ_SCALE_ROWMAJOR, RFQ_SCALE_MMA = 0, 1
 RFQ_FALLBACK_NONE, RFQ_FALLBACK_ALL, RFQ_FALLBACK_AMAX = 0, 1, 2
 RFQ_OUT_F32, RFQ_OUT_BF16 = 0, 1
@@ -27,7 +27,7 @@ STATUS_NAMES = {0: "RFQ_OK", 1: "RFQ_ERR_INVALID_ARG", 2: "RFQ_ERR_SHAPE", 3: "R
 
 EXPORTED = ("rfq_status_string", "rfq_qtensor_bytes", "rfq_quantize_weight", "rfq_quantize_act",
             "rfq_linear_workspace_bytes", "rfq_linear", "rfq_workspace_status", "rfq_dequant",
-            "rfq_linear_noalloc", "rfq_linear_fused")
+            "rfq_linear_noalloc", "rfq_linear_fused", "rfq_convert")
 
 
 class RFQError(RuntimeError):
@@ -78,6 +78,8 @@ def load_library(path: str = LIB_PATH):
         lib.rfq_linear_noalloc.argtypes = [QTP, QTP, P, I32, QTP, P, I32, P]
         lib.rfq_linear_fused.restype = I32
         lib.rfq_linear_fused.argtypes = [P, I64, I64, QTP, ctypes.POINTER(_FB), P, I32, P, P]
+        lib.rfq_convert.restype = I32
+        lib.rfq_convert.argtypes = [QTP, QTP, P]
         _lib = lib
     return _lib
 
@@ -176,6 +178,13 @@ def rfq_dequant(q: QTensor, out: torch.Tensor, out_dtype: int | None = None, str
         out_dtype = RFQ_OUT_BF16 if out.dtype == torch.bfloat16 else RFQ_OUT_F32
     qt = q.c()
     _check(load_library().rfq_dequant(ctypes.byref(qt), _ptr(out), out_dtype, _stream(stream)), "rfq_dequant")
+
+
+def rfq_convert(src: QTensor, dst: QTensor, stream=None):
+    """Exact re-encoding of an MXFP4 tensor as MXFP8 (E4M3 codes of the same
+    values, the same scales)."""
+    a, b = src.c(), dst.c()
+    _check(load_library().rfq_convert(ctypes.byref(a), ctypes.byref(b), _stream(stream)), "rfq_convert")
 
 
 def bf16_operand(t: torch.Tensor) -> QTensor:

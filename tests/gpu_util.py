@@ -23,9 +23,11 @@ def mma_scale_to_rowmajor(sf_bytes: np.ndarray, rows: int, k: int) -> np.ndarray
 
 
 def qtensor_host(q: rfq.QTensor):
-    """(codes [rows, k/2] uint8, scales in the oracle's row-major form)."""
+    """(codes [rows, k/2] uint8 ([rows, k] for MXFP8), scales in the oracle's
+    row-major form)."""
     rows, k = q.rows, q.k
-    codes = q.codes[: rows * k // 2].cpu().numpy().reshape(rows, k // 2)
+    kc = k if q.fmt == rfq.RFQ_FMT_MXFP8 else k // 2
+    codes = q.codes[: rows * kc].cpu().numpy().reshape(rows, kc)
     sf = q.scales.cpu().numpy()
     if q.fmt == rfq.RFQ_FMT_HIF4 and q.scale_layout == rfq.RFQ_SCALE_MMA:
         # block-major [k/64][rows rounded up to 128]

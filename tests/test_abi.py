@@ -48,6 +48,8 @@ def test_qtensor_bytes(lib):
     assert rfq.rfq_qtensor_bytes(1, 0, 10, 640) == (10 * 320, 10 * 10 * 4)
     assert rfq.rfq_qtensor_bytes(1, 1, 10, 640) == (10 * 320, 128 * 10 * 4)   # block-major, rows padded
     assert rfq.rfq_qtensor_bytes(2, 0, 10, 640) == (10 * 640 * 2, 0)         # bf16 expansion
+    assert rfq.rfq_qtensor_bytes(3, 0, 10, 640) == (10 * 640, 10 * 20)         # MXFP8: a byte per element
+    assert rfq.rfq_qtensor_bytes(3, 1, 130, 512) == (130 * 512, 256 * 16)      # MMA scales as MXFP4
     # HiF4: 36 bytes per 64 elements (4.5 bits each)
     cb, sb = rfq.rfq_qtensor_bytes(1, 0, 1, 64)
     assert cb + sb == 36
