@@ -51,6 +51,7 @@ def _peaks():
 # source file of each timed kernel: its DRAM counters hold only for the
 # sources they were taken on (the kernel's file plus the shared headers)
 _KERNEL_SRC = {"gemm_mxf4_kernel": "gemm_mxf4.cu", "gemm_mxf4_pair_kernel": "gemm_mxf4_pair.cu",
+               "act_quant8_kernel": "quant_mxfp8.cu",
                "gemm_mxf4_fused_kernel": "gemm_mxf4_fused.cu",
                "act_quant_mxfp4_kernel": "quant_mxfp4.cu",
                "gemm_hif4_kernel": "gemm_hif4.cu", "act_quant_hif4_kernel": "quant_hif4.cu"}
@@ -71,10 +72,23 @@ def _kernel_traffic(kernel: str, workload: str):
     return None
 
 
+def _launches_per_step(quant_only, fused, hif4, no_res, scheme, amax_phi):
+    """This library's kernel launches in one timed step."""
+    if quant_only or fused:
+        return 1
+    n = 1 + (1 if amax_phi else 0)          # quantizer (+ the phi amax kernel)
+    if hif4:
+        n += 1 if no_res else 2             # exact bf16 expansions of X~ (and X^)
+    if scheme == "rfq8":
+        n += 1                              # E4M3 re-encoding of X~
+    return n + 1                            # GEMM
+
+
 def _src_hash(kernel: str):
     d = os.path.join(HERE, "paper_2608_26581_gb300", "csrc")
     m = hashlib.sha256()
-    extra = ("mxfp4_math.cuh",) if kernel in ("act_quant_mxfp4_kernel", "gemm_mxf4_fused_kernel") else ()
+    extra = ("mxfp4_math.cuh",) if kernel in ("act_quant_mxfp4_kernel", "gemm_mxf4_fused_kernel",
+                                              "act_quant8_kernel") else ()
     for n in (_KERNEL_SRC[kernel], "ptx.cuh", "internal.h") + extra:
         m.update(open(os.path.join(d, n), "rb").read())
     return m.hexdigest()[:16]
@@ -291,6 +305,16 @@ def run_rfq(args):
     no_res = args.no_residual
     if no_res and (fused or quant_only or amax_phi):
         raise SystemExit("--no-residual applies to the two-kernel linear workloads without --phi-tau")
+    # MXFP8 schemes (Table 1 baselines and the FP4-to-FP8 residual of Sec. 4.2):
+    #   rfq8: MXFP4 main + MXFP8 residual, both multiplied as E4M3 (X~ and W~
+    #         re-encoded exactly by rfq_convert); w4a8: MXFP8 X x MXFP4 W
+    #         (re-encoded); w8a8: MXFP8 X x MXFP8 W.  All on kind::mxf8f6f4.
+    scheme = args.scheme
+    f8 = scheme != "rfq4"
+    if f8 and (hif4 or quant_only or fused or no_res):
+        raise SystemExit("--scheme applies to the MXFP4 linear workloads (two-kernel, with residual flags unset)")
+    if amax_phi and scheme in ("w4a8", "w8a8"):
+        raise SystemExit("--phi-tau needs a residual pathway")
     F = rfq.RFQ_FMT_HIF4 if hif4 else rfq.RFQ_FMT_MXFP4
     L = rfq.RFQ_SCALE_MMA
 
@@ -301,16 +325,23 @@ def run_rfq(args):
     if not quant_only:
         wb = make_weight(K, N, seed=spec.act.seed)
         w = torch.from_numpy(wb.view(np.int16)).to(dev).view(torch.bfloat16)
-        wq = rfq.empty_qtensor(F, L, N, K, device=dev)
+        wq = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme == "w8a8" else F, L, N, K, device=dev)
         rfq.rfq_quantize_weight(w, wq)                     # offline weight step, untimed
-        if hif4:
+        if scheme in ("rfq8", "w4a8"):
+            wop = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8, L, N, K, device=dev)
+            rfq.rfq_convert(wq, wop)                       # exact E4M3 re-encoding of W~ (offline)
+        elif hif4:
             wop = rfq.empty_bf16_operand(N, K, device=dev)  # exact bf16 expansion of W~ (offline)
             rfq.rfq_dequant(wq, wop.codes)
-        else:
+        elif wop is None:
             wop = wq
         del w
-    xq = rfq.empty_qtensor(F, L, M, K, device=dev)
-    xr = rfq.empty_qtensor(F, L, M, K, device=dev) if not no_res else None
+    xq = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme in ("w4a8", "w8a8") else F, L, M, K, device=dev)
+    xr = (None if no_res or scheme in ("w4a8", "w8a8") else
+          rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme == "rfq8" else F, L, M, K, device=dev))
+    no_res = xr is None
+    # rfq8: the E4M3 re-encoding of X~ that the GEMM multiplies
+    xq8 = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8, L, M, K, device=dev) if scheme == "rfq8" else None
     phi_buf = (torch.empty(((M + 127) // 128) * ((K + 255) // 256), dtype=torch.uint8, device=dev)
                if args.phi_tau is not None else None)
     # HiF4: the GEMM takes the exact bf16 expansions of X~ and X^ (expanding
@@ -354,14 +385,16 @@ def run_rfq(args):
             rfq.rfq_dequant(xq, xq16.codes, stream=stream)
             if xr is not None:
                 rfq.rfq_dequant(xr, xr16.codes, stream=stream)
+        if xq8 is not None:
+            rfq.rfq_convert(xq, xq8, stream=stream)
         if i is not None:
             per_step[i][2].record(stream)
         if hif4 and not quant_only:
             rfq.rfq_linear(xq16, xr16 if xr is not None else None, phi_buf if amax_phi else None, 256, wop, y, rfq.RFQ_OUT_BF16, wsp,
                            stream=stream)
         elif not quant_only:
-            rfq.rfq_linear(xq, xr, phi_buf if amax_phi else None, 256, wop, y, rfq.RFQ_OUT_BF16, wsp,
-                           stream=stream)
+            rfq.rfq_linear(xq8 if xq8 is not None else xq, xr, phi_buf if amax_phi else None, 256, wop, y,
+                           rfq.RFQ_OUT_BF16, wsp, stream=stream)
         if i is not None:
             per_step[i][3].record(stream)
 
@@ -387,7 +420,7 @@ def run_rfq(args):
         barrier()
     ms = t_start.elapsed_time(t_end) / args.steps
     q_ms = statistics.mean(a.elapsed_time(b) for a, b, _, _ in per_step)
-    x_ms = statistics.mean(b.elapsed_time(c) for _, b, c, _ in per_step)   # HiF4 expansions (0 otherwise)
+    x_ms = statistics.mean(b.elapsed_time(c) for _, b, c, _ in per_step)   # HiF4 / rfq8 expansions (0 otherwise)
     g_ms = statistics.mean(c.elapsed_time(d) for _, _, c, d in per_step)
     ms = _max_over_ranks(ms, ws, dist, dev)
 
@@ -427,6 +460,12 @@ def run_rfq(args):
         t_peak, t_peak_sust = pk["bf16_burst"], pk["bf16_sust"]
         t_src = f"{pk['src']} bf16 burst {pk['bf16_burst']} TFLOP/s, of {pk['src']}"
         t_kernel = "gemm_hif4_kernel"
+    elif f8:
+        # kind::mxf8f6f4: the FP8 tensor rate, nominally twice the bf16 one
+        t_peak, t_peak_sust = pk["bf16_burst"] * 2.0, pk["bf16_sust"] * 2.0
+        t_src = (f"{pk['src']} bf16 burst {pk['bf16_burst']} TFLOP/s x 2 (nominal dense FP8/BF16 ratio), "
+                 f"of {pk['src']}")
+        t_kernel = "gemm_mxf4_pair_kernel"   # its E4M3 instantiation, at every M
     else:
         t_peak, t_peak_sust = pk["bf16_burst"] * FP4_OVER_BF16, pk["bf16_sust"] * FP4_OVER_BF16
         t_src = (f"{pk['src']} bf16 burst {pk['bf16_burst']} TFLOP/s x {FP4_OVER_BF16:g} "
@@ -438,6 +477,10 @@ def run_rfq(args):
         npath = 1 if no_res else 2   # main (and residual) codes + metadata written
         aq_bytes = M * K * 2 + npath * (M * K // 2) + npath * (((M + 127) // 128) * 128 * (K // 64) * 4)
         aq_kernel = "act_quant_hif4_kernel"
+    elif f8:
+        sfb = ((M + 127) // 128) * 128 * K // 32
+        aq_bytes = (M * K * 2 + M * K // 2 + M * K + 2 * sfb if scheme == "rfq8" else M * K * 2 + M * K + sfb)
+        aq_kernel = "act_quant8_kernel"
     else:
         npath = 1 if no_res else 2
         aq_bytes = M * K * 2 + npath * (M * K // 2) + npath * (((M + 127) // 128) * 128 * K // 32)
@@ -459,7 +502,9 @@ def run_rfq(args):
         gemm_tflops = flop / (g_ms * 1e-3) / 1e12
         roofline = {"bound": "tensor", "kernel": t_kernel, "achieved": gemm_tflops, "peak": t_peak,
                     "unit": "TFLOP/s", "frac": gemm_tflops / t_peak,
-                    "traffic": _kernel_traffic(t_kernel, spec.name + ("+phi" if amax_phi else "")), "flop_per_launch": flop, "ms_per_launch": g_ms,
+                    "traffic": _kernel_traffic(t_kernel, spec.name + ("+" + scheme if f8 else "")
+                                               + ("+phi" if amax_phi else "")),
+                    "flop_per_launch": flop, "ms_per_launch": g_ms,
                     "peak_source": t_src, "frac_of_sustained_peak": gemm_tflops / t_peak_sust}
     clocks = clk.summary()
     if e2e_ms is not None:
@@ -479,20 +524,26 @@ def run_rfq(args):
             "metric": METRIC, "value": value, "unit": unit, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None,
-            "dtype": "hif4 (exact bf16 x bf16, fp32 accumulate)" if hif4 else "mxfp4 (e2m1 x e2m1, fp32 accumulate)",
+            "dtype": ("hif4 (exact bf16 x bf16, fp32 accumulate)" if hif4 else
+                      "mxfp8 (e4m3 x e4m3, fp32 accumulate)" if f8 else "mxfp4 (e2m1 x e2m1, fp32 accumulate)"),
             "data": "synthetic",
             "config": _config(spec, {"parallelism": f"dp{ws} over token rows" if ws > 1 else "single GPU",
                                      "variant": ("fused prologue: X quantized inside the GEMM" if fused
                                                  else "quantizer kernel + GEMM kernel"),
-                                     **({"residual": "none: plain W4A4 (Q(X) W~ only)"} if no_res else {}),
+                                     **({"residual": "none: plain W4A4 (Q(X) W~ only)"}
+                                        if no_res and not f8 else {}),
+                                     **({"scheme": {"rfq8": "RFQ with an MXFP8 residual: MXFP4 X~ + MXFP8 X^, "
+                                                            "MXFP4 W~, all multiplied as E4M3",
+                                                    "w4a8": "W4A8: MXFP8 X x MXFP4 W~ (as E4M3)",
+                                                    "w8a8": "W8A8: MXFP8 X x MXFP8 W~"}[scheme]} if f8 else {}),
                                      **({"phi": f"AMAX: phi = [max |x| over the 128 x 256 tile > {args.phi_tau}], "
                                                 f"fraction of phi = 1 tiles f = {phi_frac:.4f}",
                                          "phi_fraction": phi_frac} if amax_phi else {})}),
             "roofline": roofline,
             "act_quant": act_quant,
-            "expand_ms_per_step": x_ms if hif4 else None,
+            "expand_ms_per_step": x_ms if (hif4 or scheme == "rfq8") else None,
             "e2e": e2e,
-            "gpu_launches": (1 if quant_only or fused else (4 if hif4 else 2)) * args.steps,
+            "gpu_launches": _launches_per_step(quant_only, fused, hif4, no_res, scheme, amax_phi) * args.steps,
             "clocks": clocks,
             "cpu_baseline": cpu,
         }
@@ -516,6 +567,9 @@ def main():
                     help="selective fallback: residual only on 128 x 256 tiles whose max |x| exceeds TAU")
     ap.add_argument("--no-residual", action="store_true",
                     help="plain W4A4: no residual pathway (the baseline the correction is added to)")
+    ap.add_argument("--scheme", default="rfq4", choices=["rfq4", "rfq8", "w4a8", "w8a8"],
+                    help="rfq4: MXFP4 main + MXFP4 residual (default); rfq8: MXFP8 residual; "
+                         "w4a8 / w8a8: MXFP8 activation baselines")
     ap.add_argument("--variant", default="two-kernel", choices=["two-kernel", "fused"],
                     help="fused: rfq_linear_fused, the activation quantizer inside the GEMM")
     ap.add_argument("--workload", default=WORKLOAD,
