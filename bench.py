@@ -319,16 +319,34 @@ def run_rfq(args):
     L = rfq.RFQ_SCALE_MMA
 
     xb = make_activation(spec.act)
+    # grouped (mixture-of-experts) workload: the routed rows of each expert,
+    # stacked with every expert starting on a 128-row boundary (zero rows
+    # between); one launch multiplies each expert's rows by its own W~
+    grouped = spec.groups > 0
+    Mb = M   # rows of the stacked buffers
+    if grouped:
+        if hif4 or fused or quant_only:
+            raise SystemExit("grouped workloads run the MXFP4 / MXFP8 two-kernel path")
+        from paper_2608_26581_gb300.synth import group_layout, make_group_counts
+        counts = make_group_counts(M, spec.groups, seed=spec.act.seed)
+        starts, ends, Mb = group_layout(counts)
+        xs = np.zeros((Mb, K), np.uint16)
+        cum = np.concatenate([[0], np.cumsum(counts)])
+        for g in range(spec.groups):
+            xs[starts[g]:ends[g]] = xb[cum[g]:cum[g + 1]]
+        xb = xs
+        group_off = torch.tensor(np.concatenate([starts, ends[-1:]]).astype(np.int32), device=dev)
     x_host = torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16).pin_memory()
     x = x_host.to(dev)
     wop = None
+    NW = N * (spec.groups if grouped else 1)   # weight rows (every expert's W~ stacked)
     if not quant_only:
-        wb = make_weight(K, N, seed=spec.act.seed)
+        wb = make_weight(K, NW, seed=spec.act.seed)
         w = torch.from_numpy(wb.view(np.int16)).to(dev).view(torch.bfloat16)
-        wq = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme == "w8a8" else F, L, N, K, device=dev)
+        wq = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme == "w8a8" else F, L, NW, K, device=dev)
         rfq.rfq_quantize_weight(w, wq)                     # offline weight step, untimed
         if scheme in ("rfq8", "w4a8"):
-            wop = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8, L, N, K, device=dev)
+            wop = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8, L, NW, K, device=dev)
             rfq.rfq_convert(wq, wop)                       # exact E4M3 re-encoding of W~ (offline)
         elif hif4:
             wop = rfq.empty_bf16_operand(N, K, device=dev)  # exact bf16 expansion of W~ (offline)
@@ -336,20 +354,20 @@ def run_rfq(args):
         elif wop is None:
             wop = wq
         del w
-    xq = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme in ("w4a8", "w8a8") else F, L, M, K, device=dev)
+    xq = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme in ("w4a8", "w8a8") else F, L, Mb, K, device=dev)
     xr = (None if no_res or scheme in ("w4a8", "w8a8") else
-          rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme == "rfq8" else F, L, M, K, device=dev))
+          rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme == "rfq8" else F, L, Mb, K, device=dev))
     no_res = xr is None
     # rfq8: the E4M3 re-encoding of X~ that the GEMM multiplies
-    xq8 = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8, L, M, K, device=dev) if scheme == "rfq8" else None
-    phi_buf = (torch.empty(((M + 127) // 128) * ((K + 255) // 256), dtype=torch.uint8, device=dev)
+    xq8 = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8, L, Mb, K, device=dev) if scheme == "rfq8" else None
+    phi_buf = (torch.empty(((Mb + 127) // 128) * ((K + 255) // 256), dtype=torch.uint8, device=dev)
                if args.phi_tau is not None else None)
     # HiF4: the GEMM takes the exact bf16 expansions of X~ and X^ (expanding
     # once per activation, not once per output tile inside the GEMM)
     xq16 = rfq.empty_bf16_operand(M, K, device=dev) if hif4 and not quant_only else None
     xr16 = rfq.empty_bf16_operand(M, K, device=dev) if hif4 and not quant_only else None
-    y = torch.empty(M, max(N, 16), dtype=torch.bfloat16, device=dev)
-    y_host = torch.empty(M, max(N, 16), dtype=torch.bfloat16).pin_memory()
+    y = torch.empty(Mb, max(N, 16), dtype=torch.bfloat16, device=dev)
+    y_host = torch.empty(Mb, max(N, 16), dtype=torch.bfloat16).pin_memory()
     wsp = torch.zeros(rfq.rfq_linear_workspace_bytes() // 4, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream(dev)
     # quantizer-only workload: its result (both pathways' codes and scales) is read back
@@ -392,6 +410,9 @@ def run_rfq(args):
         if hif4 and not quant_only:
             rfq.rfq_linear(xq16, xr16 if xr is not None else None, phi_buf if amax_phi else None, 256, wop, y, rfq.RFQ_OUT_BF16, wsp,
                            stream=stream)
+        elif grouped:
+            rfq.rfq_linear_grouped(xq8 if xq8 is not None else xq, xr, phi_buf if amax_phi else None, 256, group_off,
+                                   wop, N, y, rfq.RFQ_OUT_BF16, wsp, stream=stream)
         elif not quant_only:
             rfq.rfq_linear(xq8 if xq8 is not None else xq, xr, phi_buf if amax_phi else None, 256, wop, y,
                            rfq.RFQ_OUT_BF16, wsp, stream=stream)
@@ -472,18 +493,18 @@ def run_rfq(args):
                  f"(nominal dense FP4/BF16 ratio), of {pk['src']}")
         # more than one 128-row tile runs on CTA pairs (see launch_gemm_mxf4)
         t_kernel = "gemm_mxf4_fused_kernel" if fused else (
-            "gemm_mxf4_pair_kernel" if M > 128 else "gemm_mxf4_kernel")
+            "gemm_mxf4_pair_kernel" if M > 128 or grouped else "gemm_mxf4_kernel")
     if hif4:
         npath = 1 if no_res else 2   # main (and residual) codes + metadata written
-        aq_bytes = M * K * 2 + npath * (M * K // 2) + npath * (((M + 127) // 128) * 128 * (K // 64) * 4)
+        aq_bytes = Mb * K * 2 + npath * (Mb * K // 2) + npath * (((Mb + 127) // 128) * 128 * (K // 64) * 4)
         aq_kernel = "act_quant_hif4_kernel"
     elif f8:
-        sfb = ((M + 127) // 128) * 128 * K // 32
-        aq_bytes = (M * K * 2 + M * K // 2 + M * K + 2 * sfb if scheme == "rfq8" else M * K * 2 + M * K + sfb)
+        sfb = ((Mb + 127) // 128) * 128 * K // 32
+        aq_bytes = (Mb * K * 2 + Mb * K // 2 + Mb * K + 2 * sfb if scheme == "rfq8" else Mb * K * 2 + Mb * K + sfb)
         aq_kernel = "act_quant8_kernel"
     else:
         npath = 1 if no_res else 2
-        aq_bytes = M * K * 2 + npath * (M * K // 2) + npath * (((M + 127) // 128) * 128 * K // 32)
+        aq_bytes = Mb * K * 2 + npath * (Mb * K // 2) + npath * (((Mb + 127) // 128) * 128 * K // 32)
         aq_kernel = "act_quant_mxfp4_kernel"
     if fused:
         act_quant = None   # quantization happens inside the GEMM
@@ -509,8 +530,8 @@ def run_rfq(args):
     clocks = clk.summary()
     if e2e_ms is not None:
         e2e = {"value": _job_rate(aq_bytes / 1e9 if quant_only else flop / 1e12, ws, e2e_ms), "unit": unit,
-               "ms_per_step": e2e_ms, "h2d_bytes_per_step": M * K * 2,
-               "d2h_bytes_per_step": q_bytes if quant_only else M * N * 2}
+               "ms_per_step": e2e_ms, "h2d_bytes_per_step": Mb * K * 2,
+               "d2h_bytes_per_step": q_bytes if quant_only else Mb * N * 2}
     else:
         e2e = None
 
@@ -530,6 +551,10 @@ def run_rfq(args):
             "config": _config(spec, {"parallelism": f"dp{ws} over token rows" if ws > 1 else "single GPU",
                                      "variant": ("fused prologue: X quantized inside the GEMM" if fused
                                                  else "quantizer kernel + GEMM kernel"),
+                                     **({"groups": f"{spec.groups} experts, routed rows {M} (min "
+                                                   f"{int(counts.min())}, max {int(counts.max())} per expert), "
+                                                   f"stacked on 128-row starts: {Mb} rows",
+                                         "weight_rows": NW} if grouped else {}),
                                      **({"residual": "none: plain W4A4 (Q(X) W~ only)"}
                                         if no_res and not f8 else {}),
                                      **({"scheme": {"rfq8": "RFQ with an MXFP8 residual: MXFP4 X~ + MXFP8 X^, "
@@ -573,7 +598,7 @@ def main():
     ap.add_argument("--variant", default="two-kernel", choices=["two-kernel", "fused"],
                     help="fused: rfq_linear_fused, the activation quantizer inside the GEMM")
     ap.add_argument("--workload", default=WORKLOAD,
-                    choices=["wan_ffn_up", "qwen_gate_up", "qwen_down_hif4", "act_quant", "tiny"])
+                    choices=["wan_ffn_up", "qwen_gate_up", "qwen_down_hif4", "act_quant", "tiny", "qwen_moe_gate_up"])
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -217,6 +217,30 @@ RFQ_API rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, co
                                     const rfq_fallback *fb, void *y, int32_t out_dtype, void *workspace,
                                     void *stream);
 
+/* Grouped RFQ GEMM for mixture-of-experts layers (SURVEY: the MoE expert
+ * projections of Qwen3-VL, Table 2): every group g (an expert) computes
+ *     Y[rows of g] = X~ W~_g + phi X^ W~_g             (Algorithm 1, Eq. rfq)
+ * in one launch over all groups.  xq / xr: the activations of all groups
+ * stacked along rows (rfq_qtensor as for rfq_linear, rows = the stacked
+ * total); group_off: device int32 [groups + 1], rows [group_off[g],
+ * group_off[g+1]) belong to group g; every group start must be a multiple
+ * of 128 (pad each group's rows), the offsets non-decreasing and
+ * group_off[groups] <= rows.  The offsets are read on the device (a router
+ * may write them): a violation is recorded in the workspace, nothing is
+ * computed, and rfq_workspace_status returns RFQ_ERR_SHAPE.  wq: the
+ * weights of all groups stacked, rows = groups * N (group g's W~ rows
+ * [g N, (g+1) N)), N % 128 == 0.  y: device [rows][N]; every row of a
+ * group (the rows padding it to the next group's start included) is
+ * written, rows before group_off[0] or from group_off[groups] on are not.  Operands MXFP4 (or all MXFP8) with
+ * RFQ_SCALE_MMA, K % 128 == 0; phi, phi_r_s, out_dtype and workspace as
+ * for rfq_linear.  1 <= groups <= 128.
+ * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
+ * RFQ_ERR_UNSUPPORTED, RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */
+RFQ_API rfq_status rfq_linear_grouped(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_t *phi,
+                                      int32_t phi_r_s, const int32_t *group_off, int32_t groups,
+                                      const rfq_qtensor *wq, int64_t N, void *y, int32_t out_dtype,
+                                      void *workspace, void *stream);
+
 /* Exact re-encoding of an MXFP4 tensor as MXFP8 (every E2M1 value is an
  * E4M3 value): dst codes [rows][k] E4M3 bytes, dst scales = src scales.
  * src: fmt MXFP4; dst: fmt MXFP8, the same rows, k and scale layout; both
@@ -227,7 +251,9 @@ RFQ_API rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, co
 RFQ_API rfq_status rfq_convert(const rfq_qtensor *src, rfq_qtensor *dst, void *stream);
 
 /* Synchronizes `stream` and returns the device status left in a workspace by
- * earlier calls (RFQ_OK or RFQ_ERR_TIMEOUT); clears it when `clear` != 0. */
+ * earlier calls (RFQ_OK, RFQ_ERR_TIMEOUT, or RFQ_ERR_SHAPE for group
+ * offsets that break rfq_linear_grouped's contract); clears it when
+ * `clear` != 0. */
 RFQ_API rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *stream);
 
 /* Allocation-free variant of rfq_linear.  The paper has no counterpart: this

@@ -406,7 +406,7 @@ rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *stream)
         if (cudaMemsetAsync(workspace, 0, sizeof(int32_t), st) != cudaSuccess)
             return RFQ_ERR_CUDA;
     }
-    return v == kDevOk ? RFQ_OK : RFQ_ERR_TIMEOUT;
+    return v == kDevOk ? RFQ_OK : v == kDevBadGroups ? RFQ_ERR_SHAPE : RFQ_ERR_TIMEOUT;
 }
 
 rfq_status rfq_dequant(const rfq_qtensor *q, void *out, int32_t out_dtype, void *stream)
@@ -456,6 +456,69 @@ rfq_status rfq_convert(const rfq_qtensor *src, rfq_qtensor *dst, void *stream)
         return s;
     return from_cuda(launch_convert_mxfp4_mxfp8(src->codes, src->scales, src->rows, src->k, sb, dst->codes,
                                                 dst->scales, static_cast<cudaStream_t>(stream)));
+}
+
+rfq_status rfq_linear_grouped(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_t *phi, int32_t phi_r_s,
+                              const int32_t *group_off, int32_t groups, const rfq_qtensor *wq, int64_t N, void *y,
+                              int32_t out_dtype, void *workspace, void *stream)
+{
+    if (!xq || !wq || !y || !workspace || !group_off)
+        return RFQ_ERR_INVALID_ARG;
+    if (out_dtype != RFQ_OUT_F32 && out_dtype != RFQ_OUT_BF16)
+        return RFQ_ERR_INVALID_ARG;
+    if (groups < 1 || groups > 128)
+        return RFQ_ERR_SHAPE;
+    const int64_t M = xq->rows, K = xq->k;
+    if (M < 0 || N <= 0 || K <= 0 || wq->k != K || wq->rows != N * groups)
+        return RFQ_ERR_SHAPE;
+    rfq_status s = check_qtensor(xq, M, K);
+    if (s != RFQ_OK)
+        return s;
+    if ((s = check_qtensor(wq, wq->rows, K)) != RFQ_OK)
+        return s;
+    if (xr) {
+        if ((s = check_qtensor(xr, M, K)) != RFQ_OK)
+            return s;
+        if (xr->fmt != xq->fmt || xr->scale_layout != xq->scale_layout)
+            return RFQ_ERR_INVALID_ARG;
+    }
+    const bool f8 = xq->fmt == RFQ_FMT_MXFP8;
+    if ((xq->fmt != RFQ_FMT_MXFP4 && !f8) || wq->fmt != xq->fmt)
+        return RFQ_ERR_UNSUPPORTED;
+    // every group's W~ rows start on a 128-row scale atom and a 16-column Y boundary
+    if (N % 128 != 0 || K % 128 != 0)
+        return RFQ_ERR_SHAPE;
+    if (M > (int64_t)INT32_MAX || N * groups > (int64_t)INT32_MAX || K > (int64_t)INT32_MAX)
+        return RFQ_ERR_SHAPE;
+    if (phi && xr && (phi_r_s < 128 || phi_r_s % 128 != 0))
+        return RFQ_ERR_SHAPE;
+    if (!aligned16(y) || !aligned16(workspace) || !aligned16(group_off))
+        return RFQ_ERR_ALIGNMENT;
+    if (xq->scale_layout != RFQ_SCALE_MMA || wq->scale_layout != RFQ_SCALE_MMA)
+        return RFQ_ERR_UNSUPPORTED;
+    if ((s = check_device()) != RFQ_OK)
+        return s;
+    if (M == 0)
+        return RFQ_OK;
+    GemmMxf4Args a;
+    a.a_codes = xq->codes;
+    a.a_sf = xq->scales;
+    a.r_codes = xr ? xr->codes : nullptr;
+    a.r_sf = xr ? xr->scales : nullptr;
+    a.b_codes = wq->codes;
+    a.b_sf = wq->scales;
+    a.phi = xr ? phi : nullptr;
+    a.phi_r_s = phi_r_s;
+    a.y = y;
+    a.out_bf16 = out_dtype == RFQ_OUT_BF16;
+    a.M = M;
+    a.N = N;
+    a.K = K;
+    a.status = static_cast<int32_t *>(workspace);
+    a.f8 = f8;
+    a.group_off = group_off;
+    a.groups = groups;
+    return from_cuda(launch_gemm_mxf4(a, static_cast<cudaStream_t>(stream)));
 }
 
 } // extern "C"

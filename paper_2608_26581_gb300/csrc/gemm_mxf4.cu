@@ -597,7 +597,7 @@ cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const C
 cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st)
 {
     // more than one 128-row tile: CTA pairs (M = 256 MMAs, half the W~ bytes per SM)
-    if (a.M > BM || a.f8)   // (E4M3 operands run on the pair kernel at every M)
+    if (a.M > BM || a.f8 || a.groups > 0)   // (E4M3 operands and groups run on the pair kernel at every M)
         return launch_gemm_mxf4_pair(a, st);
     CUtensorMap ta, tr, tb;
     const uint64_t kb = (uint64_t)a.K / 2;

@@ -84,6 +84,7 @@ constexpr int SF_WARPS = 4;
 constexpr int THREADS = 64 + 32 * (EPI_WARPS + SF_WARPS);
 constexpr int PHI_WARP = THREADS / 32;   // the phi reader: one warp beyond THREADS
 constexpr int REC_WORDS = 64;            // phi record: up to 2048 full k-stages (K <= 524288)
+constexpr int GRP_MAX = 128;             // groups of the grouped GEMM
 constexpr int YSTAGE = 2048;             // per epilogue warp: 32 rows x 64 bytes of Y
 static_assert(SF_COL0 + SF_SLOTS * SF_SLOT_COLS <= TMEM_COLS, "TMEM budget");
 static_assert(SF_SLOTS >= STAGES, "a scale slot is rewritten only after its stage's MMAs completed");
@@ -121,6 +122,9 @@ struct Smem {
     uint64_t phi_empty[2];        // the producer consumed the record
     PhiRec rec[2];
     uint32_t stage_info[STAGES];  // the tile's residual-stage count | odd last chunk's residual << 31
+    int32_t grp_off[GRP_MAX + 1];   // grouped GEMM: first row of each group (and the end)
+    int32_t grp_pairs[GRP_MAX + 1]; // grouped GEMM: 256-row pairs of the groups before each group
+    int32_t grp_bad;                // grouped GEMM: the row offsets break the contract
     uint32_t tmem_base;
     int32_t abort_flag;
 };
@@ -132,6 +136,13 @@ __device__ __forceinline__ void flag_timeout(Smem &S, int32_t *status)
     S.abort_flag = 1;
     atomicExch(status, kDevTimeout);
 }
+
+// Where an output tile lives: the pair's first A row, the end of its rows
+// (the group's end, or M), its first W~ row and Y column, and the end of
+// its group's 128-row W~ scale atoms.
+struct TileCoord {
+    int a_row0, row_end, w_row0, col0, wa_end;
+};
 
 template <bool B>
 struct Bool {
@@ -145,13 +156,17 @@ struct Mask {
 // F8: every operand holds E4M3 codes (one byte per element, kind::mxf8f6f4
 // MMAs of K = 32 with one scale per row each); a stage is then one
 // 128-element chunk (the same 128-byte rows).
-template <bool RES, bool PHI, bool OUT_BF16, bool F8>
+// GRP: the grouped (mixture-of-experts) form, G groups of rows with their
+// own W~ (row offsets read on the device); the plain form is compiled
+// without any of it.
+template <bool RES, bool PHI, bool OUT_BF16, bool F8, bool GRP>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     gemm_mxf4_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmR,
                           const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmY,
                           const uint8_t *__restrict__ sfa, const uint8_t *__restrict__ sfr,
                           const uint8_t *__restrict__ sfb, const uint8_t *__restrict__ phi, int phi_chunks,
-                          int phi_cols, int M, int N, int K, int32_t *status)
+                          int phi_cols, int M, int N, int K, int32_t *status,
+                          const int32_t *__restrict__ group_off, int G, void *__restrict__ y)
 {
     extern __shared__ uint8_t smem_raw[];
     Smem &S = *reinterpret_cast<Smem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -167,8 +182,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
     const int n_tiles = (N + BN - 1) / BN;
     const int m_tiles = (M + BM - 1) / BM;  // 128-row tiles: scale atoms and phi rows
     const int m_pairs = (M + 2 * BM - 1) / (2 * BM);
-    const int tiles = n_tiles * m_pairs;
-    const int n_atoms = (N + 127) >> 7;     // 128-row scale atoms of W~
+    const int n_atoms = (N + 127) >> 7;     // 128-row scale atoms of W~ (one group's with G > 0)
     const int pair = blockIdx.x >> 1, pairs = gridDim.x >> 1;
 
     if (threadIdx.x == 0) {
@@ -202,12 +216,81 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
         tmem_alloc_pair(&S.tmem_base, TMEM_COLS);
         tmem_relinquish_pair();
     }
+    if (GRP && warp == 2) {
+        // Grouped GEMM (G > 0): rows [group_off[g], group_off[g+1]) of X and Y
+        // belong to group g, whose W~ rows are [g N, (g+1) N).  Every group
+        // start must be a multiple of 128 with the offsets non-decreasing and
+        // group_off[G] <= M; otherwise the kernel records kDevBadGroups and
+        // computes nothing.  The prefix of 256-row pairs maps a tile index to
+        // its group.
+        int bad = 0;
+        if (G > 0) {
+            for (int e = lane; e <= G; e += 32)
+                S.grp_off[e] = __ldg(group_off + e);
+            __syncwarp();
+            int carry = 0;
+            if (lane == 0)
+                S.grp_pairs[0] = 0;
+            for (int base = 0; base < G; base += 32) {
+                const int e = base + lane;
+                int cnt = 0;
+                if (e < G) {
+                    const int a = S.grp_off[e], b = S.grp_off[e + 1];
+                    if (a < 0 || (a & (BM - 1)) != 0 || b < a || b > M)
+                        bad = 1;
+                    else
+                        cnt = (b - a + 2 * BM - 1) / (2 * BM);
+                }
+                int v = cnt;
+#pragma unroll
+                for (int d = 1; d < 32; d <<= 1) {
+                    const int t = __shfl_up_sync(0xffffffffu, v, d);
+                    if (lane >= d)
+                        v += t;
+                }
+                if (e < G)
+                    S.grp_pairs[e + 1] = carry + v;
+                carry += __shfl_sync(0xffffffffu, v, 31);
+            }
+            bad = __any_sync(0xffffffffu, bad);
+            if (bad && lane == 0)
+                atomicExch(status, kDevBadGroups);
+        }
+        if (lane == 0)
+            S.grp_bad = bad;
+    }
     tc_fence_before();
     __syncthreads();
     cluster_sync(); // both CTAs' barriers initialised and TMEM allocated
     tc_fence_after();
     const uint32_t tmem = S.tmem_base;
-    const bool skip = S.abort_flag != 0;
+    const bool skip = S.abort_flag != 0 || (GRP && S.grp_bad != 0);
+    const int tiles = n_tiles * (GRP ? S.grp_pairs[G] : m_pairs);
+    auto coord = [&](int tile) {
+        const int pi = tile / n_tiles, nt = tile - pi * n_tiles;
+        TileCoord c;
+        c.col0 = nt * BN;
+        if (!GRP) {
+            c.a_row0 = pi * 2 * BM;
+            c.row_end = M;
+            c.w_row0 = nt * BN;
+            c.wa_end = n_atoms;
+        } else {
+            int lo = 0, hi = G; // grp_pairs[lo] <= pi < grp_pairs[hi]
+            while (hi - lo > 1) {
+                const int mid = (lo + hi) >> 1;
+                if (S.grp_pairs[mid] <= pi)
+                    lo = mid;
+                else
+                    hi = mid;
+            }
+            c.a_row0 = S.grp_off[lo] + (pi - S.grp_pairs[lo]) * 2 * BM;
+            c.row_end = S.grp_off[lo + 1];
+            c.w_row0 = lo * N + nt * BN;
+            c.wa_end = (lo + 1) * n_atoms;
+        }
+        return c;
+    };
 
     if (warp == 0) {
         // ------------------------------------------------ TMA producer (both CTAs)
@@ -216,11 +299,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
             int p = 0, it = 0;
             bool stop = false;
             for (int tile = pair; tile < tiles && !stop; tile += pairs, ++it) {
-                const int m_pair = tile / n_tiles, n_tile = tile - m_pair * n_tiles;
-                const int m_tile = 2 * m_pair + (int)rank;
-                const bool rows_in = m_tile < m_tiles;
-                const int atom0 = 2 * n_tile;
-                const int nb = atom0 + 1 < n_atoms ? 2 : 1;
+                const TileCoord tc = coord(tile);
+                const int a_row = tc.a_row0 + (int)rank * BM;   // this CTA's first A row
+                const int m_tile = a_row / BM;
+                const bool rows_in = a_row < tc.row_end;
+                const int atom0 = tc.w_row0 >> 7;
+                const int nb = atom0 + 1 < tc.wa_end ? 2 : 1;
                 // one k-stage: wait for its ring slot, publish the tile's info,
                 // issue the copies (codes: both CTAs' copies complete on the even
                 // CTA's barrier; scale atoms: this CTA's own barrier)
@@ -241,10 +325,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     uint64_t *sbar = &S.sf_full[slot];
                     if (lead)
                         mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES + B_BYTES + (res_on ? A_BYTES : 0)));
-                    tma_load_2d_pair(st.a, &tmA, bar, cx, m_tile * BM);
+                    tma_load_2d_pair(st.a, &tmA, bar, cx, a_row);
                     if (res_on)
-                        tma_load_2d_pair(st.r, &tmR, bar, cx, m_tile * BM);
-                    tma_load_2d_pair(st.b, &tmB, bar, cx, n_tile * BN + (int)rank * BN_HALF);
+                        tma_load_2d_pair(st.r, &tmR, bar, cx, a_row);
+                    tma_load_2d_pair(st.b, &tmB, bar, cx, tc.w_row0 + (int)rank * BN_HALF);
                     mbar_arrive_expect_tx(sbar, nb * sfbytes + (rows_in ? (res_on ? 2 : 1) * sfbytes : 0));
                     if (rows_in) {
                         bulk_load(st.sfa, sfa + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, sbar);
@@ -402,7 +486,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
         const uint32_t sw = (uint32_t)((lane >> 1) & 3);   // 64B swizzle: chunk j of row r at (j ^ ((r >> 1) & 3))
         int it = 0;
         for (int tile = pair; tile < tiles && !skip; tile += pairs, ++it) {
-            const int m_pair = tile / n_tiles, n_tile = tile - m_pair * n_tiles;
             // warp-uniform outcome: the tcgen05 loads below need the whole warp
             if (!__all_sync(0xffffffffu, mbar_wait(&S.acc_full, it & 1, kWaitLimitNs, gstat))) {
                 if (lane == 0)
@@ -410,7 +493,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 break;
             }
             tc_fence_after();
-            const int row0 = (2 * m_pair + (int)rank) * BM + q * 32;
+            const TileCoord tc = coord(tile);   // (computed here: fewer registers live across the wait)
+            const int row0 = tc.a_row0 + (int)rank * BM + q * 32;
             const uint32_t tcol = tmem + ((uint32_t)(q * 32) << 16) + h * (BN / 2);
             auto release = [&]() {
                 // the accumulator goes back to the MMA thread
@@ -444,9 +528,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 release();
 #pragma unroll
                 for (int c = 0; c < 4; ++c) {   // 32-column chunks: one 64-byte TMA box row per lane
-                    const int col = n_tile * BN + h * (BN / 2) + 32 * c;
-                    if (col >= N || row0 >= M)
+                    const int col = tc.col0 + h * (BN / 2) + 32 * c;
+                    if (col >= N || row0 >= tc.row_end)
                         break;
+                    if (GRP && row0 + 32 > tc.row_end && tc.row_end < M) {
+                        // a group ends inside this 32-row box: rows past it are
+                        // another group's or padding, so each lane stores its own row
+                        if (row0 + lane < tc.row_end) {
+                            uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(y) +
+                                                                   (int64_t)(row0 + lane) * N + col);
+#pragma unroll
+                            for (int j = 0; j < 4; ++j)
+                                dst[j] = make_uint4(pk[16 * c + 4 * j], pk[16 * c + 4 * j + 1],
+                                                    pk[16 * c + 4 * j + 2], pk[16 * c + 4 * j + 3]);
+                        }
+                        continue;
+                    }
                     if (lane == 0)
                         bulk_wait_group_read<0>();
                     __syncwarp();
@@ -474,13 +571,25 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                         release();
 #pragma unroll
                     for (int c = 0; c < 2; ++c) {
-                        const int col = n_tile * BN + h * (BN / 2) + (2 * half + c) * 32;
-                        if (col >= N || row0 >= M)
+                        const int col = tc.col0 + h * (BN / 2) + (2 * half + c) * 32;
+                        if (col >= N || row0 >= tc.row_end)
                             continue;
 #pragma unroll
                         for (int hb = 0; hb < 2; ++hb) { // 16 fp32 columns (64 bytes) per store
                             if (col + 16 * hb >= N)
                                 break;
+                            if (GRP && row0 + 32 > tc.row_end && tc.row_end < M) {
+                                // a group ends inside this 32-row box (see the bf16 path)
+                                if (row0 + lane < tc.row_end) {
+                                    uint4 *dst = reinterpret_cast<uint4 *>(static_cast<float *>(y) +
+                                                                           (int64_t)(row0 + lane) * N + col + 16 * hb);
+#pragma unroll
+                                    for (int j = 0; j < 4; ++j)
+                                        dst[j] = make_uint4(v[c][16 * hb + 4 * j], v[c][16 * hb + 4 * j + 1],
+                                                            v[c][16 * hb + 4 * j + 2], v[c][16 * hb + 4 * j + 3]);
+                                }
+                                continue;
+                            }
                             if (lane == 0)
                                 bulk_wait_group_read<0>();
                             __syncwarp();
@@ -514,9 +623,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
         int p = 0;
         bool stop = false;
         for (int tile = pair; tile < tiles && !stop && !skip; tile += pairs) {
-            const int m_pair = tile / n_tiles, n_tile = tile - m_pair * n_tiles;
-            const bool rows_in = 2 * m_pair + (int)rank < m_tiles;
-            const bool b1_in = 2 * n_tile + 1 < n_atoms;
+            const TileCoord tc = coord(tile);
+            const bool rows_in = tc.a_row0 + (int)rank * BM < tc.row_end;
+            const bool b1_in = (tc.w_row0 >> 7) + 1 < tc.wa_end;
             // the scale words of the next stage (in the producer's order), with
             // the residual mask rm known at compile time
             auto write_stage = [&](int nch, auto rm_t) {
@@ -588,17 +697,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
         }
     } else if (PHI) {
         // ------------------------------------------------ phi reader (warp 14)
-        // Record of the CTA's j-th tile: chunk c of the pair's row tile
-        // 2 m_pair + r needs its residual when phi[2 m_pair + r][c / phi_chunks]
-        // is non-zero.
+        // Record of the CTA's j-th tile: chunk c of the pair's row tile m
+        // (128 rows) needs its residual when phi[m][c / phi_chunks] is non-zero.
         const int my_tiles = pair < tiles ? (tiles - pair + pairs - 1) / pairs : 0;
-        auto chunk_on = [&](int m_pair, int c) {
+        auto chunk_on = [&](const TileCoord &tc, int c) {
             const int col = c / phi_chunks;
             bool on = false;
 #pragma unroll
             for (int r = 0; r < 2; ++r) {
-                const int mt = 2 * m_pair + r;
-                if (mt < m_tiles && __ldg(phi + (int64_t)mt * phi_cols + col) != 0)
+                const int row = tc.a_row0 + r * BM, mt = row / BM;
+                if (row < tc.row_end && mt < m_tiles && __ldg(phi + (int64_t)mt * phi_cols + col) != 0)
                     on = true;
             }
             return on;
@@ -611,18 +719,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     flag_timeout(S, status);
                 break;
             }
-            const int m_pair = (pair + j * pairs) / n_tiles;
+            const TileCoord tcj = coord(pair + j * pairs);
             PhiRec &rec = S.rec[r];
             uint32_t n_res = 0;
             for (int w = 0; 32 * w < nf; ++w) {
                 const int ks = 32 * w + lane;
-                const bool on = ks < nf && (chunk_on(m_pair, CPS * ks) || (!F8 && chunk_on(m_pair, CPS * ks + 1)));
+                const bool on = ks < nf && (chunk_on(tcj, CPS * ks) || (!F8 && chunk_on(tcj, CPS * ks + 1)));
                 const uint32_t word = __ballot_sync(0xffffffffu, on);
                 if (lane == 0)
                     rec.bits[w] = word;
                 n_res += __popc(word);
             }
-            const uint32_t tail = nf < nks && chunk_on(m_pair, CPS * nf) ? 1u : 0u;
+            const uint32_t tail = nf < nks && chunk_on(tcj, CPS * nf) ? 1u : 0u;
             if (lane == 0)
                 rec.info = n_res | tail << 31;
             mbar_arrive(&S.phi_full[r]);
@@ -639,11 +747,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
     }
 }
 
-template <bool RES, bool PHI, bool OUT, bool F8>
+template <bool RES, bool PHI, bool OUT, bool F8, bool GRP>
 cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const CUtensorMap &tb,
                            const CUtensorMap &ty, const GemmMxf4Args &a, cudaStream_t st)
 {
-    auto kern = gemm_mxf4_pair_kernel<RES, PHI, OUT, F8>;
+    auto kern = gemm_mxf4_pair_kernel<RES, PHI, OUT, F8, GRP>;
     static int max_pairs = 0; // per variant: clusters of two that fit on the device at once
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (e != cudaSuccess)
@@ -659,13 +767,15 @@ cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const C
             return e;
         max_pairs = n > 0 ? n : 1;
     }
-    const int64_t tiles = ((a.N + BN - 1) / BN) * ((a.M + 2 * BM - 1) / (2 * BM));
+    // grouped: the tile count depends on the device-side row offsets; every
+    // pair of the grid walks the tiles that exist
+    const int64_t tiles = a.groups > 0 ? INT64_MAX : ((a.N + BN - 1) / BN) * ((a.M + 2 * BM - 1) / (2 * BM));
     const int grid = 2 * (int)(tiles < max_pairs ? tiles : max_pairs);
     const int phi_chunks = a.phi_r_s / 128;
     const int phi_cols = a.phi ? (int)((a.K + a.phi_r_s - 1) / a.phi_r_s) : 0;
     kern<<<grid, PHI ? THREADS + 32 : THREADS, kSmemBytes, st>>>(
         ta, tr, tb, ty, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf, (const uint8_t *)a.b_sf, a.phi, phi_chunks,
-        phi_cols, (int)a.M, (int)a.N, (int)a.K, a.status);
+        phi_cols, (int)a.M, (int)a.N, (int)a.K, a.status, a.group_off, a.groups, a.y);
     return cudaGetLastError();
 }
 
@@ -675,8 +785,9 @@ cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
 {
     CUtensorMap ta, tr, tb, ty;
     const uint64_t kb = a.f8 ? (uint64_t)a.K : (uint64_t)a.K / 2; // code bytes per row
+    const uint64_t w_rows = (uint64_t)a.N * (a.groups > 0 ? (uint64_t)a.groups : 1u);
     if (!encode_tmap_2d_u8(&ta, a.a_codes, kb, (uint64_t)a.M, kb, ROW, BM, 128) ||
-        !encode_tmap_2d_u8(&tb, a.b_codes, kb, (uint64_t)a.N, kb, ROW, BN_HALF, 128))
+        !encode_tmap_2d_u8(&tb, a.b_codes, kb, w_rows, kb, ROW, BN_HALF, 128))
         return cudaErrorInvalidValue;
     if (a.r_codes) {
         if (!encode_tmap_2d_u8(&tr, a.r_codes, kb, (uint64_t)a.M, kb, ROW, BM, 128))
@@ -693,8 +804,10 @@ cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
     const bool res = a.r_codes != nullptr;
     const bool phi = res && a.phi != nullptr && a.K / (a.f8 ? 128 : 256) <= REC_WORDS * 32;
 #define RFQ_GV(R, P, O)                                                                                           \
-    return a.f8 ? launch_variant<R, P, O, true>(ta, tr, tb, ty, a, st)                                            \
-                : launch_variant<R, P, O, false>(ta, tr, tb, ty, a, st)
+    return a.groups > 0 ? (a.f8 ? launch_variant<R, P, O, true, true>(ta, tr, tb, ty, a, st)                       \
+                                : launch_variant<R, P, O, false, true>(ta, tr, tb, ty, a, st))                     \
+                        : (a.f8 ? launch_variant<R, P, O, true, false>(ta, tr, tb, ty, a, st)                      \
+                                : launch_variant<R, P, O, false, false>(ta, tr, tb, ty, a, st))
     if (!res) {
         if (a.out_bf16) RFQ_GV(false, false, true);
         RFQ_GV(false, false, false);

@@ -12,6 +12,7 @@ namespace rfq {
 // Device status word values written into a workspace by kernels.
 constexpr int32_t kDevOk = 0;
 constexpr int32_t kDevTimeout = 1;
+constexpr int32_t kDevBadGroups = 2;   // grouped GEMM: device-side row offsets break the contract
 
 // Bounded waits in the GEMM give up after this many nanoseconds.
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
@@ -61,6 +62,8 @@ struct GemmMxf4Args {
     int64_t M, N, K;
     int32_t *status;
     int f8 = 0;                                // every operand MXFP8 (E4M3): kind::mxf8f6f4, CTA pairs
+    const int32_t *group_off = nullptr;        // grouped GEMM: device row offsets [groups + 1]
+    int groups = 0;                            // grouped GEMM: N is per group, W~ has groups * N rows
 };
 cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st);
 // CTA-pair kernel (gemm_mxf4_pair.cu), used by launch_gemm_mxf4 when M > 128.

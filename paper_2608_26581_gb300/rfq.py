@@ -27,7 +27,7 @@ STATUS_NAMES = {0: "RFQ_OK", 1: "RFQ_ERR_INVALID_ARG", 2: "RFQ_ERR_SHAPE", 3: "R
 
 EXPORTED = ("rfq_status_string", "rfq_qtensor_bytes", "rfq_quantize_weight", "rfq_quantize_act",
             "rfq_linear_workspace_bytes", "rfq_linear", "rfq_workspace_status", "rfq_dequant",
-            "rfq_linear_noalloc", "rfq_linear_fused", "rfq_convert")
+            "rfq_linear_noalloc", "rfq_linear_fused", "rfq_convert", "rfq_linear_grouped")
 
 
 class RFQError(RuntimeError):
@@ -80,6 +80,8 @@ def load_library(path: str = LIB_PATH):
         lib.rfq_linear_fused.argtypes = [P, I64, I64, QTP, ctypes.POINTER(_FB), P, I32, P, P]
         lib.rfq_convert.restype = I32
         lib.rfq_convert.argtypes = [QTP, QTP, P]
+        lib.rfq_linear_grouped.restype = I32
+        lib.rfq_linear_grouped.argtypes = [QTP, QTP, P, I32, P, I32, QTP, I64, P, I32, P, P]
         _lib = lib
     return _lib
 
@@ -178,6 +180,21 @@ def rfq_dequant(q: QTensor, out: torch.Tensor, out_dtype: int | None = None, str
         out_dtype = RFQ_OUT_BF16 if out.dtype == torch.bfloat16 else RFQ_OUT_F32
     qt = q.c()
     _check(load_library().rfq_dequant(ctypes.byref(qt), _ptr(out), out_dtype, _stream(stream)), "rfq_dequant")
+
+
+def rfq_linear_grouped(xq: QTensor, xr: QTensor | None, phi: torch.Tensor | None, phi_r_s: int,
+                       group_off: torch.Tensor, wq: QTensor, N: int, y: torch.Tensor, out_dtype: int,
+                       workspace: torch.Tensor, stream=None):
+    """Grouped RFQ GEMM (one launch over all groups).  group_off: device int32
+    [groups + 1] row offsets (group starts multiples of 128); wq holds the
+    groups' weights stacked, rows = groups * N."""
+    a = xq.c()
+    r = xr.c() if xr is not None else None
+    w = wq.c()
+    groups = group_off.numel() - 1
+    _check(load_library().rfq_linear_grouped(ctypes.byref(a), ctypes.byref(r) if r is not None else None, _ptr(phi),
+                                             phi_r_s, _ptr(group_off), groups, ctypes.byref(w), N, _ptr(y), out_dtype,
+                                             _ptr(workspace), _stream(stream)), "rfq_linear_grouped")
 
 
 def rfq_convert(src: QTensor, dst: QTensor, stream=None):

@@ -61,6 +61,28 @@ class LinearSpec:
     w_std: float = 0.02
     fmt: str = "mxfp4"            # mxfp4 | hif4
     notes: dict = field(default_factory=dict)
+    groups: int = 0               # > 0: act.M token rows routed over this many experts (grouped GEMM)
+
+
+def make_group_counts(rows: int, groups: int, seed: int = 0) -> np.ndarray:
+    """Rows per group for a routed (mixture-of-experts) workload: a
+    multinomial draw of `rows` over `groups` with seeded, unevenly spread
+    probabilities (softmax of standard normal logits)."""
+    rng = np.random.default_rng(seed + 7919)
+    logits = rng.standard_normal(groups)
+    p = np.exp(logits - logits.max())
+    return rng.multinomial(rows, p / p.sum())
+
+
+def group_layout(counts: np.ndarray, align: int = 128):
+    """Row layout of routed groups: every group starts on a multiple of
+    `align` rows.  Returns (starts [G], ends [G], padded total rows)."""
+    starts, pos = [], 0
+    for c in counts:
+        starts.append(pos)
+        pos = -(-(pos + int(c)) // align) * align
+    starts = np.array(starts, np.int64)
+    return starts, starts + np.asarray(counts, np.int64), max(pos, align)
 
 
 def _count(frac, count, dim):
@@ -101,7 +123,7 @@ def make_weight(K: int, N: int, std: float = 0.02, seed: int = 0) -> np.ndarray:
     return f32_to_bf16_bits(w)
 
 
-# The five workloads: shapes of the paper's model families (Qwen3-VL-8B
+# The workloads: shapes of the paper's model families (Qwen3-VL-8B and -30B-A3B
 # projections and a Wan2.2-14B DiT FFN), with seeded synthetic values.
 WORKLOADS = {
     "tiny": LinearSpec(
@@ -120,6 +142,12 @@ WORKLOADS = {
         "qwen3vl8b_down_hif4_4096x12288x4096",
         ActSpec(4096, 12288, "laplace", body_scale=0.3, chan_frac=0.01, chan_scale=50.0, seed=3),
         N=4096, fmt="hif4"),
+    # Qwen3-VL-30B-A3B expert gate/up projection (hidden 2048, 2 x 768 expert
+    # width, 128 experts, 8 per token): 4096 tokens give 32768 routed rows.
+    "qwen_moe_gate_up": LinearSpec(
+        "qwen3vl30b_a3b_moe_gate_up_32768x2048x1536_128experts",
+        ActSpec(32768, 2048, "normal", chan_frac=0.01, chan_scale=50.0, tok_count=8, tok_scale=500.0, seed=5),
+        N=1536, groups=128),
     "wan_ffn_up": LinearSpec(
         "wan22_14b_ffn_up_32760x5120x13824",
         ActSpec(32760, 5120, "normal", chan_frac=0.01, chan_scale=64.0,
