@@ -378,6 +378,9 @@ def run_rfq(args):
     ev = lambda: torch.cuda.Event(enable_timing=True)
     per_step = [(ev(), ev(), ev(), ev()) for _ in range(args.steps)]
 
+    # the step's input and output buffers (the end-to-end loop double-buffers them)
+    io = {"x": x, "y": y}
+
     def step(i=None):
         if fused:
             # the quantizer runs inside the GEMM: one kernel per step
@@ -385,17 +388,17 @@ def run_rfq(args):
                 per_step[i][0].record(stream)
                 per_step[i][1].record(stream)
                 per_step[i][2].record(stream)
-            rfq.rfq_linear_fused(x, wop, y, rfq.RFQ_OUT_BF16, wsp, stream=stream)
+            rfq.rfq_linear_fused(io["x"], wop, io["y"], rfq.RFQ_OUT_BF16, wsp, stream=stream)
             if i is not None:
                 per_step[i][3].record(stream)
             return
         if i is not None:
             per_step[i][0].record(stream)
         if amax_phi:
-            rfq.rfq_quantize_act(x, xq, xr, phi_buf, mode=rfq.RFQ_FALLBACK_AMAX, tau=args.phi_tau, p_s=128,
+            rfq.rfq_quantize_act(io["x"], xq, xr, phi_buf, mode=rfq.RFQ_FALLBACK_AMAX, tau=args.phi_tau, p_s=128,
                                  r_s=256, stream=stream)
         else:
-            rfq.rfq_quantize_act(x, xq, xr, None, mode=rfq.RFQ_FALLBACK_NONE if no_res else rfq.RFQ_FALLBACK_ALL,
+            rfq.rfq_quantize_act(io["x"], xq, xr, None, mode=rfq.RFQ_FALLBACK_NONE if no_res else rfq.RFQ_FALLBACK_ALL,
                                  stream=stream)
         if i is not None:
             per_step[i][1].record(stream)
@@ -408,13 +411,13 @@ def run_rfq(args):
         if i is not None:
             per_step[i][2].record(stream)
         if hif4 and not quant_only:
-            rfq.rfq_linear(xq16, xr16 if xr is not None else None, phi_buf if amax_phi else None, 256, wop, y, rfq.RFQ_OUT_BF16, wsp,
+            rfq.rfq_linear(xq16, xr16 if xr is not None else None, phi_buf if amax_phi else None, 256, wop, io["y"], rfq.RFQ_OUT_BF16, wsp,
                            stream=stream)
         elif grouped:
             rfq.rfq_linear_grouped(xq8 if xq8 is not None else xq, xr, phi_buf if amax_phi else None, 256, group_off,
-                                   wop, N, y, rfq.RFQ_OUT_BF16, wsp, stream=stream)
+                                   wop, N, io["y"], rfq.RFQ_OUT_BF16, wsp, stream=stream)
         elif not quant_only:
-            rfq.rfq_linear(xq8 if xq8 is not None else xq, xr, phi_buf if amax_phi else None, 256, wop, y,
+            rfq.rfq_linear(xq8 if xq8 is not None else xq, xr, phi_buf if amax_phi else None, 256, wop, io["y"],
                            rfq.RFQ_OUT_BF16, wsp, stream=stream)
         if i is not None:
             per_step[i][3].record(stream)
@@ -445,26 +448,61 @@ def run_rfq(args):
     g_ms = statistics.mean(c.elapsed_time(d) for _, _, c, d in per_step)
     ms = _max_over_ranks(ms, ws, dist, dev)
 
-    # end to end through the public API with host buffers
+    # End to end through the public API with host buffers: every step copies
+    # its X from pinned host memory and its result back to pinned host
+    # memory.  The copies run on their own streams against double-buffered
+    # device X / Y, so step i's device work overlaps the copies of steps
+    # i - 1 and i + 1 (the copy engines give ~200 GB/s per direction).
     e2e_ms = None
-    for i in range(0 if args.no_e2e else args.warmup + args.steps):
-        if i == args.warmup:
-            barrier()
-            torch.cuda.synchronize()
-            e0, e1 = ev(), ev()
-            e0.record(stream)
-        x.copy_(x_host, non_blocking=True)
-        step()
-        if quant_only:
-            for dst, src in host_q:
-                dst.copy_(src, non_blocking=True)
-        else:
-            y_host.copy_(y, non_blocking=True)
     if not args.no_e2e:
+        h2d, d2h = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+        xs = [x, torch.empty_like(x)]
+        ysb = [y, torch.empty_like(y)]
+        x_ready = [torch.cuda.Event(), torch.cuda.Event()]
+        x_free = [torch.cuda.Event(), torch.cuda.Event()]
+        y_done = [torch.cuda.Event(), torch.cuda.Event()]
+        y_free = [torch.cuda.Event(), torch.cuda.Event()]
+        total = args.warmup + args.steps
+        for i in range(total):
+            sl = i & 1
+            if i == args.warmup:
+                for st_ in (h2d, d2h):
+                    stream.wait_stream(st_)
+                barrier()
+                torch.cuda.synchronize()
+                e0, e1 = ev(), ev()
+                e0.record(stream)
+                h2d.wait_stream(stream)
+                d2h.wait_stream(stream)
+            with torch.cuda.stream(h2d):
+                if i >= 2:
+                    h2d.wait_event(x_free[sl])          # step i - 2 has read this X buffer
+                xs[sl].copy_(x_host, non_blocking=True)
+                x_ready[sl].record(h2d)
+            stream.wait_event(x_ready[sl])
+            if i >= 2:
+                stream.wait_event(y_free[sl])           # step i - 2's result has left this Y buffer
+            if quant_only and i >= 1:
+                stream.wait_event(y_free[sl ^ 1])       # the quantizer's outputs are single-buffered
+            io["x"], io["y"] = xs[sl], ysb[sl]
+            step()
+            x_free[sl].record(stream)
+            y_done[sl].record(stream)
+            with torch.cuda.stream(d2h):
+                d2h.wait_event(y_done[sl])
+                if quant_only:
+                    for dst, src in host_q:
+                        dst.copy_(src, non_blocking=True)
+                else:
+                    y_host.copy_(ysb[sl], non_blocking=True)
+                y_free[sl].record(d2h)
+        stream.wait_stream(h2d)
+        stream.wait_stream(d2h)
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
         e2e_ms = e0.elapsed_time(e1) / args.steps
+        io["x"], io["y"] = x, y
     if e2e_ms is not None:
         e2e_ms = _max_over_ranks(e2e_ms, ws, dist, dev)
     if rfq.rfq_workspace_status(wsp) != rfq.RFQ_OK:
