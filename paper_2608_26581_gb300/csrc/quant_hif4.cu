@@ -118,7 +118,13 @@ __device__ __forceinline__ int64_t meta_index(int64_t m, int64_t blk, int64_t ro
 }
 
 // Eight consecutive lanes hold one 64-element block (lane l: group l % 8).
-// Quantizes x (main), and with RES its residual x - x~ (Sec. 4.3).
+// Quantizes x (main), and with RES its residual x - x~ (Sec. 4.3).  Items
+// are (row, 1024-element segment): a warp loads its four 16-byte chunks per
+// lane up front, and the row and block indices come from the item without a
+// 64-bit division per chunk.
+constexpr int kHSeg = 1024;
+constexpr int kHU = kHSeg / 256;
+
 template <bool RES, bool PHI, int LAYOUT>
 __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__restrict__ x, int64_t M, int64_t K,
                                                             uint32_t *__restrict__ mcodes,
@@ -129,70 +135,86 @@ __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__rest
 {
     const int lane = threadIdx.x & 31;
     const int g = lane & 7;
-    const int64_t kchunks = K >> 3;
+    const int kchunks = (int)(K >> 3);
     const int64_t kblocks = K >> 6;
-    const int64_t total = M * kchunks;
-    for (int64_t base = ((int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31)) * 1;; base += (int64_t)gridDim.x * blockDim.x) {
-        if (base >= total)
-            break;
-        const int64_t c = base + lane;            // chunk of 8 elements; a block never straddles rows
-        const bool ok = c < total;
-        const uint4 v = ok ? __ldcs(x + c) : make_uint4(0, 0, 0, 0);
-        float xf[8];
-        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    const int segs = (kchunks + kHSeg / 8 - 1) / (kHSeg / 8);
+    const int64_t items = M * segs;
+    const int phi_cols = PHI ? (int)((K + r_s - 1) / r_s) : 0;
+    const int64_t gwarp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t item = gwarp; item < items; item += nwarps) {
+        const int64_t m = item / segs;
+        const int c0 = (int)(item - m * segs) * (kHSeg / 8);
+        const uint4 *xr = x + m * kchunks;
+        uint4 vv[kHU];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            xf[2 * i] = __uint_as_float(w[i] << 16);
-            xf[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+        for (int j = 0; j < kHU; ++j) {
+            const int c = c0 + j * 32 + lane;
+            vv[j] = c < kchunks ? __ldcs(xr + c) : make_uint4(0, 0, 0, 0);
         }
-        const int64_t m = c / kchunks, blk = (c % kchunks) >> 3;
-        float am = 0.f;
+        const uint8_t *prow = PHI ? phi + (m / p_s) * phi_cols : nullptr;
 #pragma unroll
-        for (int i = 0; i < 8; ++i)
-            am = fmaxf(am, fabsf(xf[i]));
+        for (int j = 0; j < kHU; ++j) {
+            const int cr = c0 + j * 32 + lane;             // chunk of 8 elements within the row
+            const bool ok = cr < kchunks;                  // uniform over each block's eight lanes
+            const int64_t c = m * kchunks + cr;
+            const int64_t blk = cr >> 3;
+            float xf[8];
+            const uint32_t w[4] = {vv[j].x, vv[j].y, vv[j].z, vv[j].w};
 #pragma unroll
-        for (int o = 1; o < 8; o <<= 1)
-            am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, o));
-        const int sb = am > 0.f ? hif4_scale_byte(am) : 0;
-        const float S = ue6m2_value(sb >> 2, sb & 3);
-        uint32_t bits;
-        float deq[8];
-        uint32_t code = hif4_group(xf, S, g, bits, deq);
-        if (am == 0.f) {
-            bits = 0;   // all-zero block: metadata 0, codes keep the sign of zero
-        }
+            for (int i = 0; i < 4; ++i) {
+                xf[2 * i] = __uint_as_float(w[i] << 16);
+                xf[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+            }
+            float am = 0.f;
 #pragma unroll
-        for (int o = 1; o < 8; o <<= 1)
-            bits |= __shfl_xor_sync(0xFFFFFFFFu, bits, o);
-        if (ok) {
-            mcodes[c] = code;
-            if (g == 0)
-                mmeta[meta_index<LAYOUT>(m, blk, M, kblocks)] = am == 0.f ? 0u : (bits | (uint32_t)sb);
-        }
-        if (RES) {
-            const bool on = !PHI || (ok && phi[(m / p_s) * ((K + r_s - 1) / r_s) + (blk * 64) / r_s] != 0);
-            float r[8];
-            float ra = 0.f;
+            for (int i = 0; i < 8; ++i)
+                am = fmaxf(am, fabsf(xf[i]));
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                r[i] = xf[i] - deq[i]; // exact
-                ra = fmaxf(ra, fabsf(r[i]));
+            for (int o = 1; o < 8; o <<= 1)
+                am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, o));
+            const int sb = am > 0.f ? hif4_scale_byte(am) : 0;
+            const float S = ue6m2_value(sb >> 2, sb & 3);
+            uint32_t bits;
+            float deq[8];
+            uint32_t code = hif4_group(xf, S, g, bits, deq);
+            if (am == 0.f) {
+                bits = 0;   // all-zero block: metadata 0, codes keep the sign of zero
             }
 #pragma unroll
             for (int o = 1; o < 8; o <<= 1)
-                ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, o));
-            const int rsb = ra > 0.f ? hif4_scale_byte(ra) : 0;
-            const float RS = ue6m2_value(rsb >> 2, rsb & 3);
-            uint32_t rbits;
-            float rdeq[8];
-            const uint32_t rcode = hif4_group(r, RS, g, rbits, rdeq);
-#pragma unroll
-            for (int o = 1; o < 8; o <<= 1)
-                rbits |= __shfl_xor_sync(0xFFFFFFFFu, rbits, o);
+                bits |= __shfl_xor_sync(0xFFFFFFFFu, bits, o);
             if (ok) {
-                rcodes[c] = on ? rcode : 0u;
+                mcodes[c] = code;
                 if (g == 0)
-                    rmeta[meta_index<LAYOUT>(m, blk, M, kblocks)] = (on && ra > 0.f) ? (rbits | (uint32_t)rsb) : 0u;
+                    mmeta[meta_index<LAYOUT>(m, blk, M, kblocks)] = am == 0.f ? 0u : (bits | (uint32_t)sb);
+            }
+            if (RES) {
+                const bool on = !PHI || (ok && prow[(cr * 8) / r_s] != 0);
+                float r[8];
+                float ra = 0.f;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    r[i] = xf[i] - deq[i]; // exact
+                    ra = fmaxf(ra, fabsf(r[i]));
+                }
+#pragma unroll
+                for (int o = 1; o < 8; o <<= 1)
+                    ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, o));
+                const int rsb = ra > 0.f ? hif4_scale_byte(ra) : 0;
+                const float RS = ue6m2_value(rsb >> 2, rsb & 3);
+                uint32_t rbits;
+                float rdeq[8];
+                const uint32_t rcode = hif4_group(r, RS, g, rbits, rdeq);
+#pragma unroll
+                for (int o = 1; o < 8; o <<= 1)
+                    rbits |= __shfl_xor_sync(0xFFFFFFFFu, rbits, o);
+                if (ok) {
+                    rcodes[c] = on ? rcode : 0u;
+                    if (g == 0)
+                        rmeta[meta_index<LAYOUT>(m, blk, M, kblocks)] =
+                            (on && ra > 0.f) ? (rbits | (uint32_t)rsb) : 0u;
+                }
             }
         }
     }
@@ -283,7 +305,8 @@ cudaError_t launch_act_quant_hif4(const void *x, int64_t M, int64_t K, int mode,
                                   void *mmeta, void *rcodes, void *rmeta, const uint8_t *phi, int layout,
                                   cudaStream_t st)
 {
-    const int blocks = grid_for(M * (K / 8), 256, 152 * 8);
+    const int64_t items = M * ((K / 8 + kHSeg / 8 - 1) / (kHSeg / 8));
+    const int blocks = grid_for(items * 32, 256, 152 * 24);
     auto *xi = static_cast<const uint4 *>(x);
     auto *mc = static_cast<uint32_t *>(mcodes);
     auto *mm = static_cast<uint32_t *>(mmeta);
