@@ -83,7 +83,8 @@ typedef enum {
     RFQ_ERR_UNSUPPORTED = 4, /* valid but unimplemented combination */
     RFQ_ERR_CUDA = 5,        /* a CUDA runtime call or a launch failed */
     RFQ_ERR_TIMEOUT = 6,     /* a kernel's bounded wait expired (device status) */
-    RFQ_ERR_DEVICE = 7       /* the current device is not an sm_103 GPU */
+    RFQ_ERR_DEVICE = 7,      /* the current device is not an sm_103 GPU */
+    RFQ_ERR_NONFINITE = 8    /* rfq_check_finite found an Inf or NaN (device status) */
 } rfq_status;
 
 typedef enum { RFQ_FMT_MXFP4 = 0, RFQ_FMT_HIF4 = 1, RFQ_FMT_BF16 = 2, RFQ_FMT_MXFP8 = 3 } rfq_format;
@@ -250,10 +251,21 @@ RFQ_API rfq_status rfq_linear_grouped(const rfq_qtensor *xq, const rfq_qtensor *
  * RFQ_ERR_UNSUPPORTED (other formats), RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */
 RFQ_API rfq_status rfq_convert(const rfq_qtensor *src, rfq_qtensor *dst, void *stream);
 
+/* Checked mode for inputs: the quantizers and GEMMs take finite bf16 inputs
+ * (non-finite ones give unspecified codes but never a fault); a caller that
+ * cannot vouch for X runs this check first.  It scans the bf16 matrix
+ * x [rows][k] (device, 16-byte aligned, k % 8 == 0) and, if any element is
+ * Inf or NaN, records RFQ_ERR_NONFINITE in `workspace` (the GEMM workspace,
+ * rfq_linear_workspace_bytes() bytes), where rfq_workspace_status reports
+ * it.  Asynchronous on `stream`; one read of x.
+ * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT, RFQ_ERR_CUDA,
+ * RFQ_ERR_DEVICE. */
+RFQ_API rfq_status rfq_check_finite(const void *x_bf16, int64_t rows, int64_t k, void *workspace, void *stream);
+
 /* Synchronizes `stream` and returns the device status left in a workspace by
- * earlier calls (RFQ_OK, RFQ_ERR_TIMEOUT, or RFQ_ERR_SHAPE for group
- * offsets that break rfq_linear_grouped's contract); clears it when
- * `clear` != 0. */
+ * earlier calls (RFQ_OK, RFQ_ERR_TIMEOUT, RFQ_ERR_SHAPE for group offsets
+ * that break rfq_linear_grouped's contract, or RFQ_ERR_NONFINITE from
+ * rfq_check_finite); clears it when `clear` != 0. */
 RFQ_API rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *stream);
 
 /* Allocation-free variant of rfq_linear.  The paper has no counterpart: this

@@ -137,6 +137,7 @@ const char *rfq_status_string(rfq_status s)
     case RFQ_ERR_CUDA: return "RFQ_ERR_CUDA: CUDA runtime call or launch failed";
     case RFQ_ERR_TIMEOUT: return "RFQ_ERR_TIMEOUT: a kernel's bounded wait expired";
     case RFQ_ERR_DEVICE: return "RFQ_ERR_DEVICE: current device is not an sm_103 GPU";
+    case RFQ_ERR_NONFINITE: return "RFQ_ERR_NONFINITE: the checked input holds an Inf or NaN";
     }
     return "RFQ_ERR_UNKNOWN";
 }
@@ -406,7 +407,10 @@ rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *stream)
         if (cudaMemsetAsync(workspace, 0, sizeof(int32_t), st) != cudaSuccess)
             return RFQ_ERR_CUDA;
     }
-    return v == kDevOk ? RFQ_OK : v == kDevBadGroups ? RFQ_ERR_SHAPE : RFQ_ERR_TIMEOUT;
+    return v == kDevOk ? RFQ_OK
+           : v == kDevBadGroups ? RFQ_ERR_SHAPE
+           : v == kDevNonFinite ? RFQ_ERR_NONFINITE
+                                : RFQ_ERR_TIMEOUT;
 }
 
 rfq_status rfq_dequant(const rfq_qtensor *q, void *out, int32_t out_dtype, void *stream)
@@ -434,6 +438,23 @@ rfq_status rfq_dequant(const rfq_qtensor *q, void *out, int32_t out_dtype, void 
         return from_cuda(launch_dequant_mxfp4_bf16(q->codes, q->scales, q->rows, q->k, q->scale_layout, out, st));
     return from_cuda(
         launch_dequant_mxfp4(q->codes, q->scales, q->rows, q->k, q->scale_layout, static_cast<float *>(out), st));
+}
+
+rfq_status rfq_check_finite(const void *x_bf16, int64_t rows, int64_t k, void *workspace, void *stream)
+{
+    if (!x_bf16 || !workspace)
+        return RFQ_ERR_INVALID_ARG;
+    if (rows < 0 || k <= 0 || k % 8 != 0)
+        return RFQ_ERR_SHAPE;
+    if (!aligned16(x_bf16) || !aligned16(workspace))
+        return RFQ_ERR_ALIGNMENT;
+    rfq_status s = check_device();
+    if (s != RFQ_OK)
+        return s;
+    if (rows == 0)
+        return RFQ_OK;
+    return from_cuda(launch_check_finite(x_bf16, rows * (k / 8), static_cast<int32_t *>(workspace),
+                                         static_cast<cudaStream_t>(stream)));
 }
 
 rfq_status rfq_convert(const rfq_qtensor *src, rfq_qtensor *dst, void *stream)

@@ -13,6 +13,7 @@ namespace rfq {
 constexpr int32_t kDevOk = 0;
 constexpr int32_t kDevTimeout = 1;
 constexpr int32_t kDevBadGroups = 2;   // grouped GEMM: device-side row offsets break the contract
+constexpr int32_t kDevNonFinite = 3;   // rfq_check_finite found an Inf or NaN
 
 // Bounded waits in the GEMM give up after this many nanoseconds.
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
@@ -36,6 +37,9 @@ cudaError_t launch_convert_mxfp4_mxfp8(const void *src_codes, const void *src_sc
                                        size_t scale_bytes, void *dst_codes, void *dst_scales, cudaStream_t st);
 cudaError_t launch_dequant_mxfp8(const void *codes, const void *scales, int64_t rows, int64_t k, int layout, void *out,
                                  bool bf16, cudaStream_t st);
+
+// ---- input check (quant_mxfp4.cu): records kDevNonFinite if x holds an Inf / NaN
+cudaError_t launch_check_finite(const void *x, int64_t n8, int32_t *status, cudaStream_t st);
 
 // ---- MXFP4 quantization (quant_mxfp4.cu)
 // Activation: main (+ residual) codes and scales in one pass over X.

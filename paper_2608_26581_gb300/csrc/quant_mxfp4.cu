@@ -161,6 +161,22 @@ __global__ void __launch_bounds__(256) phi_amax_kernel(const __nv_bfloat16 *__re
     }
 }
 
+// Any bf16 with an all-ones exponent field (Inf or NaN) sets the status word.
+__global__ void __launch_bounds__(256) check_finite_kernel(const uint4 *__restrict__ x, int64_t n8,
+                                                          int32_t *__restrict__ status)
+{
+    bool bad = false;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n8; i += (int64_t)gridDim.x * blockDim.x) {
+        const uint4 v = __ldcs(x + i);
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j)   // both halves: exponent bits all ones
+            bad |= ((w[j] & 0x7F800000u) == 0x7F800000u) || ((w[j] & 0x00007F80u) == 0x00007F80u);
+    }
+    if (__any_sync(0xFFFFFFFFu, bad) && (threadIdx.x & 31) == 0)
+        atomicCAS(status, kDevOk, kDevNonFinite);
+}
+
 __global__ void fill_u8_kernel(uint8_t *p, int64_t n, uint8_t v)
 {
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
@@ -264,6 +280,12 @@ cudaError_t launch_phi_amax(const void *x, int64_t M, int64_t K, int p_s, int r_
 {
     const int64_t np = (M + p_s - 1) / p_s, nr = (K + r_s - 1) / r_s;
     phi_amax_kernel<<<(unsigned)(np * nr), 256, 0, st>>>((const __nv_bfloat16 *)x, M, K, p_s, r_s, tau, phi);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_check_finite(const void *x, int64_t n8, int32_t *status, cudaStream_t st)
+{
+    check_finite_kernel<<<grid_for(n8, 256, 152 * 16), 256, 0, st>>>(static_cast<const uint4 *>(x), n8, status);
     return cudaGetLastError();
 }
 

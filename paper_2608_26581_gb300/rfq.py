@@ -21,13 +21,14 @@ RFQ_SCALE_ROWMAJOR, RFQ_SCALE_MMA = 0, 1
 RFQ_FALLBACK_NONE, RFQ_FALLBACK_ALL, RFQ_FALLBACK_AMAX = 0, 1, 2
 RFQ_OUT_F32, RFQ_OUT_BF16 = 0, 1
 (RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT, RFQ_ERR_UNSUPPORTED, RFQ_ERR_CUDA, RFQ_ERR_TIMEOUT,
- RFQ_ERR_DEVICE) = range(1, 8)
+ RFQ_ERR_DEVICE, RFQ_ERR_NONFINITE) = range(1, 9)
 STATUS_NAMES = {0: "RFQ_OK", 1: "RFQ_ERR_INVALID_ARG", 2: "RFQ_ERR_SHAPE", 3: "RFQ_ERR_ALIGNMENT",
-                4: "RFQ_ERR_UNSUPPORTED", 5: "RFQ_ERR_CUDA", 6: "RFQ_ERR_TIMEOUT", 7: "RFQ_ERR_DEVICE"}
+                4: "RFQ_ERR_UNSUPPORTED", 5: "RFQ_ERR_CUDA", 6: "RFQ_ERR_TIMEOUT", 7: "RFQ_ERR_DEVICE",
+                8: "RFQ_ERR_NONFINITE"}
 
 EXPORTED = ("rfq_status_string", "rfq_qtensor_bytes", "rfq_quantize_weight", "rfq_quantize_act",
             "rfq_linear_workspace_bytes", "rfq_linear", "rfq_workspace_status", "rfq_dequant",
-            "rfq_linear_noalloc", "rfq_linear_fused", "rfq_convert", "rfq_linear_grouped")
+            "rfq_linear_noalloc", "rfq_linear_fused", "rfq_convert", "rfq_linear_grouped", "rfq_check_finite")
 
 
 class RFQError(RuntimeError):
@@ -80,6 +81,8 @@ def load_library(path: str = LIB_PATH):
         lib.rfq_linear_fused.argtypes = [P, I64, I64, QTP, ctypes.POINTER(_FB), P, I32, P, P]
         lib.rfq_convert.restype = I32
         lib.rfq_convert.argtypes = [QTP, QTP, P]
+        lib.rfq_check_finite.restype = I32
+        lib.rfq_check_finite.argtypes = [P, I64, I64, P, P]
         lib.rfq_linear_grouped.restype = I32
         lib.rfq_linear_grouped.argtypes = [QTP, QTP, P, I32, P, I32, QTP, I64, P, I32, P, P]
         _lib = lib
@@ -180,6 +183,13 @@ def rfq_dequant(q: QTensor, out: torch.Tensor, out_dtype: int | None = None, str
         out_dtype = RFQ_OUT_BF16 if out.dtype == torch.bfloat16 else RFQ_OUT_F32
     qt = q.c()
     _check(load_library().rfq_dequant(ctypes.byref(qt), _ptr(out), out_dtype, _stream(stream)), "rfq_dequant")
+
+
+def rfq_check_finite(x: torch.Tensor, workspace: torch.Tensor, stream=None):
+    """Records RFQ_ERR_NONFINITE in the workspace if the bf16 matrix x holds an
+    Inf or NaN (read it back with rfq_workspace_status)."""
+    rows, k = x.shape
+    _check(load_library().rfq_check_finite(_ptr(x), rows, k, _ptr(workspace), _stream(stream)), "rfq_check_finite")
 
 
 def rfq_linear_grouped(xq: QTensor, xr: QTensor | None, phi: torch.Tensor | None, phi_r_s: int,

@@ -77,6 +77,11 @@ def test_null_arguments_rejected_before_any_device_work(lib):
                                 None, None) == 2
     qt = rfq._QT(0, 0, 4, 64, 8, 16)              # misaligned codes pointer
     assert lib.rfq_dequant(ctypes.byref(qt), ctypes.c_void_p(16), 0, None) == 3
+    # the checked mode: every call below is rejected on the host, before the device check
+    assert lib.rfq_check_finite(None, 4, 64, ctypes.c_void_p(16), None) == 1
+    assert lib.rfq_check_finite(ctypes.c_void_p(16), 4, 60, ctypes.c_void_p(16), None) == 2   # k % 8
+    assert lib.rfq_check_finite(ctypes.c_void_p(8), 4, 64, ctypes.c_void_p(16), None) == 3    # misaligned
+    assert lib.rfq_linear_grouped(None, None, None, 0, None, 1, None, 128, None, 0, None, None) == 1
 
 
 def test_fused_linear_host_checks(lib):

@@ -170,3 +170,33 @@ def test_dequant_matches_oracle(orc):
             rfq.rfq_dequant(q, out16)
             torch.cuda.synchronize()
             assert np.array_equal(out16.double().cpu().numpy(), ref)   # in bf16's normal range: exact
+
+
+def test_check_finite_flags_inf_and_nan():
+    """Checked mode: rfq_check_finite records RFQ_ERR_NONFINITE for any Inf or
+    NaN in X (every position class: first, last, interior element of a
+    16-byte chunk), nothing for finite X (including max bf16 and -0), and a
+    GEMM given that workspace computes nothing until the record is cleared."""
+    M, K = 300, 640
+    xb = make_activation(ActSpec(M, K, "normal", chan_count=2, chan_scale=64.0, seed=12))
+    xb[3, 5] = 0x7F7F      # the largest finite bf16
+    xb[4, 6] = 0x8000      # -0
+    ws = torch.zeros(rfq.rfq_linear_workspace_bytes() // 4, dtype=torch.int32, device=DEV)
+    rfq.rfq_check_finite(to_dev_bf16(xb), ws)
+    assert rfq.rfq_workspace_status(ws) == rfq.RFQ_OK
+    for (r, c, bits) in [(0, 0, 0x7F80), (M - 1, K - 1, 0xFF80), (150, 333, 0x7FC0), (7, 1, 0xFFC1)]:
+        bad = xb.copy()
+        bad[r, c] = bits
+        rfq.rfq_check_finite(to_dev_bf16(bad), ws)
+        assert rfq.rfq_workspace_status(ws) == rfq.RFQ_ERR_NONFINITE, (r, c, hex(bits))
+        # a GEMM with the flagged workspace leaves Y untouched
+        N = 256
+        wq = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA, N, K)
+        rfq.rfq_quantize_weight(to_dev_bf16(make_weight(K, N, seed=1)), wq)
+        xq = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA, M, K)
+        rfq.rfq_quantize_act(to_dev_bf16(xb), xq, None, None, mode=rfq.RFQ_FALLBACK_NONE)
+        y = torch.full((M, N), 7.0, dtype=torch.float32, device=DEV)
+        rfq.rfq_linear(xq, None, None, 256, wq, y, rfq.RFQ_OUT_F32, ws)
+        assert rfq.rfq_workspace_status(ws, clear=True) == rfq.RFQ_ERR_NONFINITE
+        assert (y == 7.0).all()
+    assert rfq.rfq_workspace_status(ws) == rfq.RFQ_OK
