@@ -177,3 +177,20 @@ def test_full_size_wan_ffn_up_fp32(orc):
 
 def test_full_size_qwen_gate_up_bf16(orc):
     _full_size(orc, "qwen_gate_up", rfq.RFQ_OUT_BF16, n_rows=12)
+
+
+@pytest.mark.parametrize("M", [100, 130])
+def test_phi_beyond_record_capacity_falls_back_exactly(orc, M):
+    """K / 256 = 2049 full k-stages: more than a phi record holds, so the GEMM
+    issues every residual product (exact, since phi = 0 residuals are stored
+    as zero) -- on the single-CTA (M <= 128) and the CTA-pair path."""
+    K, N, r_s = 524544, 16, 256
+    xb = make_activation(ActSpec(M, K, "normal", chan_count=400, chan_scale=64.0, seed=17))
+    wb = make_weight(K, N, seed=17)
+    xq, xr, wq, y, phi = _run(xb, wb, mode=rfq.RFQ_FALLBACK_AMAX, tau=30.0, r_s=r_s, use_phi=True)
+    q = orc.quantize_act(xb, orc.FMT_MXFP4, orc.PHI_AMAX, 30.0, 128, r_s)
+    assert np.array_equal(phi.cpu().numpy().reshape(q["phi"].shape), q["phi"])
+    assert 0.0 < q["phi"].mean() < 1.0
+    rwc, rws = orc.quantize_weight(wb)
+    ref = orc.linear(0, q["main_codes"], q["main_scales"], q["res_codes"], q["res_scales"], rwc, rws, M, K, N)
+    check_y(y, ref)
