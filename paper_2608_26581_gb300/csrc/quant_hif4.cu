@@ -29,34 +29,52 @@
 namespace rfq {
 namespace {
 
+__device__ __forceinline__ float fmax3(float a, float b, float c)
+{
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
 __device__ __forceinline__ float ue6m2_value(int E, int M) // 2^(E-48) (1 + M/4), E in [0, 63]
 {
     return __uint_as_float(((uint32_t)(E - 48 + 127) << 23) | ((uint32_t)M << 21));
 }
 
 // Smallest UE6M2 byte with 7 * value >= amax (amax > 0), clamped to [0, 255].
+// With amax = sig 2^ea (sig in [1, 2)), the candidates 7 (1 + M/4) 2^(E-48)
+// in increasing order are, for E - 48 = ea - 3, sig x {0.875, 1.09375,
+// 1.3125, 1.53125} and then, for E - 48 = ea - 2, {1.75, 2.1875, ...}; so
+// the answer follows from the significand bits of amax alone (thresholds
+// 0.09375, 0.3125, 0.53125 and 0.75 of the fraction: 0x0C0000, 0x280000,
+// 0x440000, 0x600000 in the 23-bit field), then the E range [0, 63].
 __device__ __forceinline__ int hif4_scale_byte(float amax)
 {
-    // floor(log2 amax) for a normal amax; a subnormal amax is below every
-    // 7 S, so byte 0 is the answer for it
-    if (__float_as_uint(amax) < 0x00800000u)
+    const uint32_t b = __float_as_uint(amax);
+    if (b < 0x00800000u)   // a subnormal amax is below every 7 S: byte 0
         return 0;
-    const int ea = (int)((__float_as_uint(amax) >> 23) & 0xFF) - 127;
-    // 7 (1 + M/4) 2^(E-48) spans [7, 12.25] 2^(E-48), so the smallest valid
-    // (E, M) has E - 48 in {ea - 3, ea - 2}; scan those eight candidates in
-    // increasing order, skipping exponents below the format's range.
-    const int e_lo = ea - 3 + 48;
-    for (int d = 0; d < 2; ++d) {
-        const int E = e_lo + d;
-        if (E < 0)
-            continue;
-        if (E > 63)
-            return 255; // above the largest macro scale: saturate
-        for (int M = 0; M < 4; ++M)
-            if (7.0f * ue6m2_value(E, M) >= amax)
-                return (E << 2) | M;
+    const uint32_t f = b & 0x7FFFFFu;
+    const int e0 = (int)(b >> 23) - 127 - 3 + 48;   // E of the first candidate row
+    int E, M;
+    if (f <= 0x600000u && e0 >= 0) {
+        // first row, M = 1..3, or (E0 + 1, 0)
+        M = 1 + (f > 0x0C0000u) + (f > 0x280000u) + (f > 0x440000u);
+        E = e0;
+        if (M == 4) {
+            M = 0;
+            E = e0 + 1;
+        }
+    } else if (e0 >= -1) {
+        // second row: (E0 + 1, 0) if sig <= 1.75, else (E0 + 1, 1); with
+        // E0 = -1 the first row is out of range and this is the smallest
+        E = e0 + 1;
+        M = f > 0x600000u ? 1 : 0;
+    } else {
+        return 0;          // below the smallest macro scale: 2^-48 covers it
     }
-    return e_lo + 1 < 0 ? 0 : 255;
+    if (E > 63)
+        return 255;        // above the largest macro scale: saturate
+    return (E << 2) | M;
 }
 
 // Quantizes the eight elements x[0..7] of group g (sub-groups 2g, 2g+1) of a
@@ -69,10 +87,7 @@ __device__ __forceinline__ uint32_t hif4_group(const float (&x)[8], float S, int
     int t[2];
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-        float a = 0.f;
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-            a = fmaxf(a, fabsf(x[4 * h + i]));
+        const float a = fmax3(fmaxf(fabsf(x[4 * h]), fabsf(x[4 * h + 1])), fabsf(x[4 * h + 2]), fabsf(x[4 * h + 3]));
         t[h] = a <= 1.75f * S ? 0 : (a <= 3.5f * S ? 1 : 2);
     }
     const int e18 = (t[0] == 2 || t[1] == 2) ? 1 : 0;
