@@ -104,16 +104,17 @@ __device__ __forceinline__ uint32_t hif4_group(const float (&x)[8], float S, int
         for (int i = 0; i < 4; ++i) {
             const float v = x[4 * h + i];
             const float a = fabsf(v);
-            // nearest k from the (approximate) quotient, kept in fp32, then
-            // fixed up with exact comparisons against the midpoints
-            // (k +- 1/2) step; ties go to even k
+            // nearest k from the fp32 quotient.  a has 8 significant bits and
+            // step = D 2^s with D in {4,5,6,7}/4, so a quotient that is not
+            // exactly a half-integer lies at least 2^-9 / 7 of it away from
+            // every half-integer it could round across, while a * inv is
+            // within 2^-20 of it (relative error 2^-23, quotient below 8):
+            // rint is exact except at true ties, which the exact midpoint
+            // tests below send to the even k
             float k = rintf(fminf(a * inv, 8.0f));
             const float hi = fmaf(k, step, hstep), lo = fmaf(k, step, -hstep);   // exact
             const bool odd = (__float_as_uint(k + 8388608.0f) & 1u) != 0;
-            if (a > hi || (a == hi && odd))
-                k += 1.0f;
-            else if (k > 0.0f && (a < lo || (a == lo && odd)))
-                k -= 1.0f;
+            k += odd ? (a == hi ? 1.0f : (a == lo ? -1.0f : 0.0f)) : 0.0f;
             k = fminf(k, 7.0f);
             const uint32_t ki = __float_as_uint(k + 8388608.0f) & 7u;   // k as an integer, exactly
             const uint32_t sgn = __float_as_uint(v) >> 31;
