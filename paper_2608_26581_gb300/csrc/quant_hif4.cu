@@ -117,10 +117,8 @@ __device__ __forceinline__ uint32_t hif4_group(const float (&x)[8], float S, int
             k += odd ? (a == hi ? 1.0f : (a == lo ? -1.0f : 0.0f)) : 0.0f;
             k = fminf(k, 7.0f);
             const uint32_t ki = __float_as_uint(k + 8388608.0f) & 7u;   // k as an integer, exactly
-            const uint32_t sgn = __float_as_uint(v) >> 31;
-            codes |= ((sgn << 3) | ki) << (4 * (4 * h + i));
-            const float q = k * step;
-            deq[4 * h + i] = sgn ? -q : q;
+            codes |= (((__float_as_uint(v) >> 28) & 8u) | ki) << (4 * (4 * h + i));
+            deq[4 * h + i] = copysignf(k * step, v);
         }
     }
     return codes;
@@ -182,10 +180,8 @@ __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__rest
                 xf[2 * i] = __uint_as_float(w[i] << 16);
                 xf[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
             }
-            float am = 0.f;
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-                am = fmaxf(am, fabsf(xf[i]));
+            float am = fmax3(fmax3(fabsf(xf[0]), fabsf(xf[1]), fabsf(xf[2])),
+                             fmax3(fabsf(xf[3]), fabsf(xf[4]), fabsf(xf[5])), fmaxf(fabsf(xf[6]), fabsf(xf[7])));
 #pragma unroll
             for (int o = 1; o < 8; o <<= 1)
                 am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, o));
@@ -208,12 +204,11 @@ __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__rest
             if (RES) {
                 const bool on = !PHI || (ok && prow[(cr * 8) / r_s] != 0);
                 float r[8];
-                float ra = 0.f;
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
+                for (int i = 0; i < 8; ++i)
                     r[i] = xf[i] - deq[i]; // exact
-                    ra = fmaxf(ra, fabsf(r[i]));
-                }
+                float ra = fmax3(fmax3(fabsf(r[0]), fabsf(r[1]), fabsf(r[2])),
+                                 fmax3(fabsf(r[3]), fabsf(r[4]), fabsf(r[5])), fmaxf(fabsf(r[6]), fabsf(r[7])));
 #pragma unroll
                 for (int o = 1; o < 8; o <<= 1)
                     ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, o));
