@@ -376,51 +376,54 @@ def run_rfq(args):
     q_bytes = sum(t.numel() for _, t in host_q)
 
     ev = lambda: torch.cuda.Event(enable_timing=True)
-    per_step = [(ev(), ev(), ev(), ev()) for _ in range(args.steps)]
 
     # the step's input and output buffers (the end-to-end loop double-buffers them)
     io = {"x": x, "y": y}
 
+    # Events between the step's phases, recorded inside the captured graph
+    # (event-record nodes): q = the quantizer, x = the HiF4 bf16 expansions
+    # or the rfq8 E4M3 re-encoding of X~ (empty otherwise), g = the GEMM.
+    per_step = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(4)]
+                for _ in range(args.steps)]
+
     def step(i=None):
+        # (recorded on the current stream: the capture stream inside the graph)
+        mark = ((lambda j: per_step[i][j].record(torch.cuda.current_stream(dev))) if i is not None
+                else (lambda j: None))
         if fused:
             # the quantizer runs inside the GEMM: one kernel per step
-            if i is not None:
-                per_step[i][0].record(stream)
-                per_step[i][1].record(stream)
-                per_step[i][2].record(stream)
-            rfq.rfq_linear_fused(io["x"], wop, io["y"], rfq.RFQ_OUT_BF16, wsp, stream=stream)
-            if i is not None:
-                per_step[i][3].record(stream)
+            for j in range(3):
+                mark(j)
+            rfq.rfq_linear_fused(io["x"], wop, io["y"], rfq.RFQ_OUT_BF16, wsp, stream=None)
+            mark(3)
             return
-        if i is not None:
-            per_step[i][0].record(stream)
+        mark(0)
         if amax_phi:
-            rfq.rfq_quantize_act(io["x"], xq, xr, phi_buf, mode=rfq.RFQ_FALLBACK_AMAX, tau=args.phi_tau, p_s=128,
-                                 r_s=256, stream=stream)
+            rfq.rfq_quantize_act(io["x"], xq, xr, phi_buf, mode=rfq.RFQ_FALLBACK_AMAX, tau=args.phi_tau,
+                                 p_s=128, r_s=256, stream=None)
         else:
-            rfq.rfq_quantize_act(io["x"], xq, xr, None, mode=rfq.RFQ_FALLBACK_NONE if no_res else rfq.RFQ_FALLBACK_ALL,
-                                 stream=stream)
-        if i is not None:
-            per_step[i][1].record(stream)
+            rfq.rfq_quantize_act(io["x"], xq, xr, None,
+                                 mode=rfq.RFQ_FALLBACK_NONE if no_res else rfq.RFQ_FALLBACK_ALL, stream=None)
+        mark(1)
         if hif4 and not quant_only:
-            rfq.rfq_dequant(xq, xq16.codes, stream=stream)
+            rfq.rfq_dequant(xq, xq16.codes, stream=None)
             if xr is not None:
-                rfq.rfq_dequant(xr, xr16.codes, stream=stream)
+                rfq.rfq_dequant(xr, xr16.codes, stream=None)
         if xq8 is not None:
-            rfq.rfq_convert(xq, xq8, stream=stream)
-        if i is not None:
-            per_step[i][2].record(stream)
-        if hif4 and not quant_only:
-            rfq.rfq_linear(xq16, xr16 if xr is not None else None, phi_buf if amax_phi else None, 256, wop, io["y"], rfq.RFQ_OUT_BF16, wsp,
-                           stream=stream)
+            rfq.rfq_convert(xq, xq8, stream=None)
+        mark(2)
+        if quant_only:
+            pass
+        elif hif4:
+            rfq.rfq_linear(xq16, xr16 if xr is not None else None, phi_buf if amax_phi else None, 256, wop,
+                           io["y"], rfq.RFQ_OUT_BF16, wsp, stream=None)
         elif grouped:
             rfq.rfq_linear_grouped(xq8 if xq8 is not None else xq, xr, phi_buf if amax_phi else None, 256, group_off,
-                                   wop, N, io["y"], rfq.RFQ_OUT_BF16, wsp, stream=stream)
-        elif not quant_only:
+                                   wop, N, io["y"], rfq.RFQ_OUT_BF16, wsp, stream=None)
+        else:
             rfq.rfq_linear(xq8 if xq8 is not None else xq, xr, phi_buf if amax_phi else None, 256, wop, io["y"],
-                           rfq.RFQ_OUT_BF16, wsp, stream=stream)
-        if i is not None:
-            per_step[i][3].record(stream)
+                           rfq.RFQ_OUT_BF16, wsp, stream=None)
+        mark(3)
 
     for _ in range(args.warmup):
         step()
@@ -432,20 +435,46 @@ def run_rfq(args):
         if ws > 1:
             dist.barrier()
 
+    def capture(instrumented):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for i in range(args.steps):
+                step(i if instrumented else None)
+        for _ in range(args.warmup):
+            g.replay()
+        torch.cuda.synchronize()
+        return g
+
+    # The timed loop: the K steps captured once in a CUDA graph and replayed
+    # between CUDA events, so that the steps run back to back at the device's
+    # rate and not at that of the Python code calling the library (tens of
+    # microseconds per call).
+    graph = capture(False)
     t_start, t_end = ev(), ev()
     with ClockSampler(local) as clk:
         barrier()
         torch.cuda.synchronize()
         t_start.record(stream)
-        for i in range(args.steps):
-            step(i)
+        graph.replay()
         t_end.record(stream)
         torch.cuda.synchronize()
         barrier()
     ms = t_start.elapsed_time(t_end) / args.steps
-    q_ms = statistics.mean(a.elapsed_time(b) for a, b, _, _ in per_step)
-    x_ms = statistics.mean(b.elapsed_time(c) for _, b, c, _ in per_step)   # HiF4 / rfq8 expansions (0 otherwise)
-    g_ms = statistics.mean(c.elapsed_time(d) for _, _, c, d in per_step)
+    # Per-kernel times: a second graph of the same steps with event-record
+    # nodes between the phases, replayed once after the timed one.  Each
+    # event node costs a few microseconds, so a step of one kernel (the
+    # quantizer alone, the fused linear) takes the timed loop's own step time.
+    graph_ev = capture(True)
+    graph_ev.replay()
+    torch.cuda.synchronize()
+    q_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in per_step)
+    x_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in per_step)   # HiF4 / rfq8 expansions (0 otherwise)
+    g_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in per_step)
+    if quant_only:
+        q_ms = ms
+    elif fused:
+        g_ms = ms
+    del graph, graph_ev
     ms = _max_over_ranks(ms, ws, dist, dev)
 
     # End to end through the public API with host buffers: every step copies
@@ -587,6 +616,8 @@ def run_rfq(args):
                       "mxfp8 (e4m3 x e4m3, fp32 accumulate)" if f8 else "mxfp4 (e2m1 x e2m1, fp32 accumulate)"),
             "data": "synthetic",
             "config": _config(spec, {"parallelism": f"dp{ws} over token rows" if ws > 1 else "single GPU",
+                                     "timing": "the K timed steps captured in one CUDA graph, replayed once "
+                                               "between CUDA events (per-kernel times: a second graph with events between the kernels)",
                                      "variant": ("fused prologue: X quantized inside the GEMM" if fused
                                                  else "quantizer kernel + GEMM kernel"),
                                      **({"groups": f"{spec.groups} experts, routed rows {M} (min "
