@@ -17,6 +17,7 @@ exchange): weak scaling.
 from __future__ import annotations
 
 import argparse
+import datetime
 import hashlib
 import json
 import os
@@ -95,8 +96,10 @@ def _src_hash(kernel: str):
 
 
 class ClockSampler:
-    """Samples SM clocks and throttle reasons with nvidia-smi while running."""
-    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+    """Samples SM clocks and throttle reasons with nvidia-smi (every 20 ms,
+    each sample time-stamped) while running; `summary` keeps the samples
+    inside a host-time window (the GPU's loaded interval)."""
+    Q = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
          "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
          "clocks_event_reasons.sw_power_cap")
 
@@ -110,7 +113,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
-                 "-lms", "100"], stdout=self.f, stderr=subprocess.DEVNULL)
+                 "-lms", "20"], stdout=self.f, stderr=subprocess.DEVNULL)
         except OSError:
             self.proc = None
         time.sleep(0.3)
@@ -118,32 +121,36 @@ class ClockSampler:
 
     def __exit__(self, *a):
         if self.proc is not None:
-            time.sleep(0.25)
+            time.sleep(0.1)
             self.proc.terminate()
             self.proc.wait()
 
-    def summary(self):
+    def summary(self, t0=None, t1=None):
+        """Median SM clock, max clock and the throttle reasons of the samples
+        taken in [t0, t1] (host seconds, time.time()); all samples when no
+        window is given or none falls inside it."""
         if self.proc is None:
             return None
         self.f.seek(0)
-        sm, mx, reasons = [], [], set()
+        rows = []
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for line in self.f:
             f = [x.strip() for x in line.split(",")]
-            if len(f) < 7:
+            if len(f) < 8:
                 continue
             try:
-                sm.append(float(f[0]))
-                mx.append(float(f[1]))
+                ts = datetime.datetime.strptime(f[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                rows.append((ts, float(f[1]), float(f[2]), f[4:8]))
             except ValueError:
                 continue
-            for n, v in zip(names, f[3:7]):
-                if v.lower().startswith("active"):
-                    reasons.add(n)
-        if not sm:
+        if not rows:
             return None
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
-                "reasons": sorted(reasons)}
+        inside = [r for r in rows if t0 is not None and t0 <= r[0] <= t1]
+        use = inside or rows
+        reasons = sorted({n for r in use for n, v in zip(names, r[3]) if v.lower().startswith("active")})
+        return {"sm_mhz": statistics.median(r[1] for r in use), "sm_max_mhz": max(r[2] for r in use),
+                "samples": len(use), "window": "timed and warm-up replays" if inside else "whole run",
+                "reasons": reasons}
 
 
 def _dist():
@@ -440,33 +447,37 @@ def run_rfq(args):
         with torch.cuda.graph(g):
             for i in range(args.steps):
                 step(i if instrumented else None)
-        for _ in range(args.warmup):
-            g.replay()
+        g.replay()          # the first replay uploads the graph
         torch.cuda.synchronize()
         return g
 
     # The timed loop: the K steps captured once in a CUDA graph and replayed
     # between CUDA events, so that the steps run back to back at the device's
     # rate and not at that of the Python code calling the library (tens of
-    # microseconds per call).
+    # microseconds per call).  Per-kernel times: a second graph of the same
+    # steps with event-record nodes between the phases, replayed right before
+    # the timed replay (the same power and clock history).  Each event node
+    # costs a few microseconds, so a step of one kernel (the quantizer alone,
+    # the fused linear) takes the timed loop's own step time.
+    # The clock samples kept are those of the loaded interval: the warm-up
+    # replays, the instrumented one and the timed one, back to back.
     graph = capture(False)
+    graph_ev = capture(True)
     t_start, t_end = ev(), ev()
     with ClockSampler(local) as clk:
         barrier()
         torch.cuda.synchronize()
+        h0 = time.time()
+        for _ in range(args.warmup):
+            graph.replay()
+        graph_ev.replay()
         t_start.record(stream)
         graph.replay()
         t_end.record(stream)
         torch.cuda.synchronize()
+        h1 = time.time()
         barrier()
     ms = t_start.elapsed_time(t_end) / args.steps
-    # Per-kernel times: a second graph of the same steps with event-record
-    # nodes between the phases, replayed once after the timed one.  Each
-    # event node costs a few microseconds, so a step of one kernel (the
-    # quantizer alone, the fused linear) takes the timed loop's own step time.
-    graph_ev = capture(True)
-    graph_ev.replay()
-    torch.cuda.synchronize()
     q_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in per_step)
     x_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in per_step)   # HiF4 / rfq8 expansions (0 otherwise)
     g_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in per_step)
@@ -594,7 +605,7 @@ def run_rfq(args):
                                                + ("+phi" if amax_phi else "")),
                     "flop_per_launch": flop, "ms_per_launch": g_ms,
                     "peak_source": t_src, "frac_of_sustained_peak": gemm_tflops / t_peak_sust}
-    clocks = clk.summary()
+    clocks = clk.summary(h0, h1)
     if e2e_ms is not None:
         e2e = {"value": _job_rate(aq_bytes / 1e9 if quant_only else flop / 1e12, ws, e2e_ms), "unit": unit,
                "ms_per_step": e2e_ms, "h2d_bytes_per_step": Mb * K * 2,
