@@ -54,7 +54,7 @@ def _peaks():
 _KERNEL_SRC = {"gemm_mxf4_kernel": "gemm_mxf4.cu", "gemm_mxf4_pair_kernel": "gemm_mxf4_pair.cu",
                "act_quant8_kernel": "quant_mxfp8.cu",
                "gemm_mxf4_fused_kernel": "gemm_mxf4_fused.cu",
-               "act_quant_mxfp4_kernel": "quant_mxfp4.cu",
+               "act_quant_mxfp4_kernel": "quant_mxfp4.cu", "act_quant_mxfp4_amax_kernel": "quant_mxfp4.cu",
                "gemm_hif4_kernel": "gemm_hif4.cu", "act_quant_hif4_kernel": "quant_hif4.cu"}
 
 
@@ -73,11 +73,11 @@ def _kernel_traffic(kernel: str, workload: str):
     return None
 
 
-def _launches_per_step(quant_only, fused, hif4, no_res, scheme, amax_phi):
+def _launches_per_step(quant_only, fused, hif4, no_res, scheme, amax_phi, amax_fused=False):
     """This library's kernel launches in one timed step."""
     if quant_only or fused:
         return 1
-    n = 1 + (1 if amax_phi else 0)          # quantizer (+ the phi amax kernel)
+    n = 1 + (1 if amax_phi and not amax_fused else 0)   # quantizer (+ the phi amax kernel)
     if hif4:
         n += 1 if no_res else 2             # exact bf16 expansions of X~ (and X^)
     if scheme == "rfq8":
@@ -88,8 +88,8 @@ def _launches_per_step(quant_only, fused, hif4, no_res, scheme, amax_phi):
 def _src_hash(kernel: str):
     d = os.path.join(HERE, "paper_2608_26581_gb300", "csrc")
     m = hashlib.sha256()
-    extra = ("mxfp4_math.cuh",) if kernel in ("act_quant_mxfp4_kernel", "gemm_mxf4_fused_kernel",
-                                              "act_quant8_kernel") else ()
+    extra = ("mxfp4_math.cuh",) if kernel in ("act_quant_mxfp4_kernel", "act_quant_mxfp4_amax_kernel",
+                                              "gemm_mxf4_fused_kernel", "act_quant8_kernel") else ()
     for n in (_KERNEL_SRC[kernel], "ptx.cuh", "internal.h") + extra:
         m.update(open(os.path.join(d, n), "rb").read())
     return m.hexdigest()[:16]
@@ -323,6 +323,7 @@ def run_rfq(args):
     if amax_phi and scheme in ("w4a8", "w8a8"):
         raise SystemExit("--phi-tau needs a residual pathway")
     F = rfq.RFQ_FMT_HIF4 if hif4 else rfq.RFQ_FMT_MXFP4
+    amax_fused = amax_phi and not hif4 and not f8 and K % 256 == 0
     L = rfq.RFQ_SCALE_MMA
 
     xb = make_activation(spec.act)
@@ -583,7 +584,8 @@ def run_rfq(args):
     else:
         npath = 1 if no_res else 2
         aq_bytes = Mb * K * 2 + npath * (Mb * K // 2) + npath * (((Mb + 127) // 128) * 128 * K // 32)
-        aq_kernel = "act_quant_mxfp4_kernel"
+        # AMAX phi on 128 x 256 tiles: phi and the quantization in one kernel
+        aq_kernel = "act_quant_mxfp4_amax_kernel" if amax_fused else "act_quant_mxfp4_kernel"
     if fused:
         act_quant = None   # quantization happens inside the GEMM
     else:
@@ -648,7 +650,8 @@ def run_rfq(args):
             "act_quant": act_quant,
             "expand_ms_per_step": x_ms if (hif4 or scheme == "rfq8") else None,
             "e2e": e2e,
-            "gpu_launches": _launches_per_step(quant_only, fused, hif4, no_res, scheme, amax_phi) * args.steps,
+            "gpu_launches": _launches_per_step(quant_only, fused, hif4, no_res, scheme, amax_phi,
+                                                amax_fused) * args.steps,
             "clocks": clocks,
             "cpu_baseline": cpu,
         }

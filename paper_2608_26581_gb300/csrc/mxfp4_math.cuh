@@ -120,13 +120,40 @@ __device__ __forceinline__ float absmax8(const float (&v)[8])
     return fmax3(m0, m1, fmaxf(fabsf(v[6]), fabsf(v[7])));
 }
 
+// The residual X - X~ of this lane's eight elements (its 32-element block
+// spread over four consecutive lanes, all 32 lanes take part), given their
+// E2M1 codes and E8M0 byte: the residual's E2M1 codes and E8M0 byte.
+__device__ __forceinline__ void mxfp4_resid8(const float (&xf)[8], uint32_t code, int sb, uint32_t &rcode, int &rb)
+{
+    float q[8], r[8];
+    e2m1x8_decode(code, q);
+    const float nsc = -pow2_e(sb);
+    const uint64_t nsc2 = f2pack(nsc, nsc);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) // x - x~ (exact)
+        f2unpack(ffma2(f2pack(q[2 * i], q[2 * i + 1]), nsc2, f2pack(xf[2 * i], xf[2 * i + 1])), r[2 * i],
+                 r[2 * i + 1]);
+    float ra = absmax8(r);
+    ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, 1));
+    ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, 2));
+    rb = scale_byte_from_f32_bits(__float_as_uint(ra));
+    const float rinv = pow2_neg_e(rb);
+    const uint64_t rinv2 = f2pack(rinv, rinv);
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+        f2unpack(fmul2(f2pack(r[2 * i], r[2 * i + 1]), rinv2), r[2 * i], r[2 * i + 1]);
+    rcode = e2m1x8(r);
+}
+
 // Quantizes this lane's eight elements (its 32-element block is spread over
 // four consecutive lanes, all 32 lanes take part): the E2M1 codes (element
-// 2i in the low nibble of byte i) and E8M0 byte of X~, and with RES those of
-// the residual X - X~.
+// 2i in the low nibble of byte i) and E8M0 byte of X~, the block's max |x|
+// (NaN elements dropped), and with RES the codes and byte of the residual
+// X - X~.
 struct Mx8 {
     uint32_t code, rcode;
     int sb, rb;
+    float am;
 };
 
 template <bool RES>
@@ -136,6 +163,7 @@ __device__ __forceinline__ Mx8 mxfp4_quant8(const float (&xf)[8])
     float am = absmax8(xf);
     am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 1));
     am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 2));
+    o.am = am;
     o.sb = scale_byte_from_f32_bits(__float_as_uint(am));
     const float inv = pow2_neg_e(o.sb);
     const uint64_t inv2 = f2pack(inv, inv);
@@ -146,26 +174,8 @@ __device__ __forceinline__ Mx8 mxfp4_quant8(const float (&xf)[8])
     o.code = e2m1x8(y);
     o.rcode = 0;
     o.rb = 0;
-    if (RES) {
-        float q[8], r[8];
-        e2m1x8_decode(o.code, q);
-        const float nsc = -pow2_e(o.sb);
-        const uint64_t nsc2 = f2pack(nsc, nsc);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) // x - x~ (exact)
-            f2unpack(ffma2(f2pack(q[2 * i], q[2 * i + 1]), nsc2, f2pack(xf[2 * i], xf[2 * i + 1])), r[2 * i],
-                     r[2 * i + 1]);
-        float ra = absmax8(r);
-        ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, 1));
-        ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, 2));
-        o.rb = scale_byte_from_f32_bits(__float_as_uint(ra));
-        const float rinv = pow2_neg_e(o.rb);
-        const uint64_t rinv2 = f2pack(rinv, rinv);
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-            f2unpack(fmul2(f2pack(r[2 * i], r[2 * i + 1]), rinv2), r[2 * i], r[2 * i + 1]);
-        o.rcode = e2m1x8(r);
-    }
+    if (RES)
+        mxfp4_resid8(xf, o.code, o.sb, o.rcode, o.rb);
     return o;
 }
 

@@ -161,6 +161,99 @@ __global__ void __launch_bounds__(256) phi_amax_kernel(const __nv_bfloat16 *__re
     }
 }
 
+// AMAX fallback (Sec. 4.3) for phi tiles of 128 rows x 256 columns, fused
+// into the quantizer: one block per tile keeps the tile's 64 KB in registers
+// (warp w holds rows 16w .. 16w + 15, lane l the l-th 16-byte chunk of each),
+// reduces max |x| over it (NaN dropped, as by phi_amax_kernel), writes phi,
+// then quantizes the tile.  A phi = 0
+// tile's residual is written as zero codes and zero scales without being
+// computed.  X is read from DRAM once, against twice for phi_amax_kernel
+// followed by act_quant_mxfp4_kernel.  (Measured slower: splitting a tile
+// over a cluster of 2 or 4 blocks that exchange their maxima through
+// distributed shared memory; a persistent 512-thread form streaming the
+// tiles through a cp.async ring.)
+constexpr int kAmaxRows = 16; // rows per warp (8 warps = 128 rows)
+
+template <int LAYOUT>
+__global__ void __launch_bounds__(256, 2) act_quant_mxfp4_amax_kernel(const uint4 *__restrict__ x, int64_t M,
+                                                                     int64_t K, uint32_t *__restrict__ mcodes,
+                                                                     uint8_t *__restrict__ mscales,
+                                                                     uint32_t *__restrict__ rcodes,
+                                                                     uint8_t *__restrict__ rscales,
+                                                                     uint8_t *__restrict__ phi, float tau)
+{
+    constexpr int R = kAmaxRows;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t kchunks = K >> 3;
+    const int kblocks = (int)(K >> 5);
+    const int nr = (int)(K >> 8);
+    const int64_t tile = blockIdx.x;
+    const int64_t p = tile / nr;
+    const int r = (int)(tile - p * nr);
+    const int64_t m0 = p * 128 + warp * R;
+    const int c = r * 32 + lane;
+    uint4 v[R];
+#pragma unroll
+    for (int i = 0; i < R; ++i)
+        v[i] = m0 + i < M ? __ldcs(x + (m0 + i) * kchunks + c) : make_uint4(0, 0, 0, 0);
+    // max |x| as two packed bf16 magnitudes: sign bits cleared, then the
+    // bf16x2 max, which returns the other operand where one is NaN (NaN
+    // dropped, as in phi_amax_kernel); starts at +0
+    uint32_t acc = 0;
+#pragma unroll
+    for (int i = 0; i < R; ++i) {
+        const uint32_t q[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            asm("max.bf16x2 %0, %1, %2;" : "=r"(acc) : "r"(acc), "r"(q[j] & 0x7fff7fffu));
+    }
+    const float am = fmaxf(__uint_as_float(acc << 16), __uint_as_float(acc & 0xffff0000u));
+    __shared__ uint32_t red[8];
+    const uint32_t wmax = __reduce_max_sync(0xFFFFFFFFu, __float_as_uint(am)); // am >= 0: integer order
+    if (lane == 0)
+        red[warp] = wmax;
+    __syncthreads();
+    uint32_t tmax = red[0];
+#pragma unroll
+    for (int i = 1; i < 8; ++i)
+        tmax = max(tmax, red[i]);
+    const bool on = __uint_as_float(tmax) > tau;
+    if (threadIdx.x == 0)
+        phi[tile] = on ? 1 : 0;
+
+    const int b = c >> 2;
+#pragma unroll
+    for (int i = 0; i < R; ++i) {
+        const int64_t m = m0 + i; // uniform over the warp
+        const int64_t soff = scale_index<LAYOUT>(m, b, kblocks);
+        if (m < M) {
+            float xf[8];
+            bf16x8_to_f32(v[i], xf);
+            if (on) {
+                const Mx8 qz = mxfp4_quant8<true>(xf);
+                mcodes[m * kchunks + c] = qz.code;
+                rcodes[m * kchunks + c] = qz.rcode;
+                if ((lane & 3) == 0) {
+                    mscales[soff] = (uint8_t)qz.sb;
+                    rscales[soff] = (uint8_t)qz.rb;
+                }
+            } else {
+                const Mx8 qz = mxfp4_quant8<false>(xf);
+                mcodes[m * kchunks + c] = qz.code;
+                rcodes[m * kchunks + c] = 0u;
+                if ((lane & 3) == 0) {
+                    mscales[soff] = (uint8_t)qz.sb;
+                    rscales[soff] = 0;
+                }
+            }
+        } else if (LAYOUT == RFQ_SCALE_MMA && (lane & 3) == 0) {
+            // rows M .. of the last tile are the layout's padding rows
+            mscales[soff] = 0;
+            rscales[soff] = 0;
+        }
+    }
+}
+
 // Any bf16 with an all-ones exponent field (Inf or NaN) sets the status word.
 __global__ void __launch_bounds__(256) check_finite_kernel(const uint4 *__restrict__ x, int64_t n8,
                                                           int32_t *__restrict__ status)
@@ -300,6 +393,20 @@ cudaError_t launch_act_quant_mxfp4(const void *x, int64_t M, int64_t K, int mode
                                    int layout, cudaStream_t st)
 {
     const int64_t np = (M + p_s - 1) / p_s, nr = (K + r_s - 1) / r_s;
+    if (mode == RFQ_FALLBACK_AMAX && p_s == 128 && r_s == 256 && K % 256 == 0) {
+        // the GEMMs' phi granularity: one fused kernel (X read once)
+        const unsigned tiles = (unsigned)(np * nr);
+        auto *xi = static_cast<const uint4 *>(x);
+        auto *mc = static_cast<uint32_t *>(mcodes);
+        auto *ms = static_cast<uint8_t *>(mscales);
+        auto *rc = static_cast<uint32_t *>(rcodes);
+        auto *rs = static_cast<uint8_t *>(rscales);
+        if (layout == RFQ_SCALE_MMA)
+            act_quant_mxfp4_amax_kernel<RFQ_SCALE_MMA><<<tiles, 256, 0, st>>>(xi, M, K, mc, ms, rc, rs, phi, tau);
+        else
+            act_quant_mxfp4_amax_kernel<RFQ_SCALE_ROWMAJOR><<<tiles, 256, 0, st>>>(xi, M, K, mc, ms, rc, rs, phi, tau);
+        return cudaGetLastError();
+    }
     if (mode == RFQ_FALLBACK_AMAX) {
         phi_amax_kernel<<<(unsigned)(np * nr), 256, 0, st>>>((const __nv_bfloat16 *)x, M, K, p_s, r_s, tau, phi);
     } else if (phi) {

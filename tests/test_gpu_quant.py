@@ -131,6 +131,42 @@ def test_phi_amax_mode(orc, p_s, r_s, tau):
     _compare(orc, xb, rfq.RFQ_SCALE_MMA, mode=rfq.RFQ_FALLBACK_AMAX, tau=tau, p_s=p_s, r_s=r_s)
 
 
+@pytest.mark.parametrize("layout", [rfq.RFQ_SCALE_MMA, rfq.RFQ_SCALE_ROWMAJOR])
+@pytest.mark.parametrize("M,K", [(1, 256), (200, 768), (385, 1024)])
+def test_phi_amax_fused_tiles(orc, layout, M, K):
+    """128 x 256 phi tiles (the GEMMs' granularity, K % 256 == 0) take the
+    fused quantizer, which reduces each tile's max |x| and quantizes it in
+    one pass.  tau is set to tile (0, 0)'s own max |x|: phi is a strict
+    comparison (Sec. 4.3), so that tile falls back to no residual."""
+    xb = make_activation(ActSpec(M, K, "student_t3", chan_count=4, chan_scale=80.0, seed=M + K))
+    x = (xb.astype(np.uint32) << 16).view(np.float32)
+    tau = float(np.abs(x[:128, :256]).max())
+    xq, xr = _compare(orc, xb, layout, mode=rfq.RFQ_FALLBACK_AMAX, tau=tau, p_s=128, r_s=256)
+    _, _, phi = _act_quant(xb, layout, rfq.RFQ_FALLBACK_AMAX, tau, 128, 256)
+    assert phi[0].item() == 0
+
+
+@pytest.mark.parametrize("r_s", [256, 128])
+def test_phi_amax_nan_dropped_inf_kept(orc, r_s):
+    """A NaN element does not count towards a tile's max |x| (the maximum
+    skips it, as the oracle's comparison does) and an Inf does, both in the
+    fused 128 x 256 quantizer (r_s = 256) and in the separate phi pass
+    (r_s = 128).  Only phi is compared: the codes of NaN elements are not
+    specified."""
+    M, K, tau = 256, 512, 50.0
+    xb = make_activation(ActSpec(M, K, "normal", seed=21))   # |x| < 6 here
+    xb[5, 7] = 0x7FC0       # NaN in tile (0, 0)
+    xb[200, 10] = 0xFFC1    # negative NaN with a payload in tile (1, 0)
+    xb[130, 300] = 0x7F80   # +Inf in tile (1, 300 // r_s)
+    _, _, phi = _act_quant(xb, rfq.RFQ_SCALE_MMA, rfq.RFQ_FALLBACK_AMAX, tau, 128, r_s)
+    ref = orc.quantize_act(xb, orc.FMT_MXFP4, rfq.RFQ_FALLBACK_AMAX, tau, 128, r_s)["phi"]
+    got = phi.cpu().numpy().reshape(ref.shape)
+    assert np.array_equal(got, ref)
+    want = np.zeros_like(ref)
+    want[1, 300 // r_s] = 1
+    assert np.array_equal(got, want)
+
+
 def test_tiny_workload_both_layouts(orc):
     spec = WORKLOADS["tiny"]
     xb = make_activation(spec.act)
