@@ -111,10 +111,10 @@ __global__ void __launch_bounds__(256) act_quant_mxfp4_kernel(const uint4 *__res
 }
 
 // phi(p, r) = [max |x| over the p_s x r_s tile > tau]; one block per tile.
-// |x| of a bf16 is its low 15 bits, and for non-NaN values the order of
-// those bits as integers is the order of the magnitudes, so the block takes
-// a packed unsigned max over 16-byte loads (two bf16 per 32-bit lane, NaN
-// halves dropped as fmaxf would) and converts the winner to fp32 once.
+// |x| of a bf16 is the bf16 with its sign bit cleared, so the block takes a
+// packed bf16x2 max over 16-byte loads (two bf16 per 32-bit lane; where one
+// operand is NaN the max returns the other, so NaN is dropped as fmaxf
+// would) and converts the winner to fp32 once.
 // Rows are 16-byte aligned (K % 32 == 0); tiles whose column range is not a
 // whole number of 8-element chunks take the scalar loop.
 __global__ void __launch_bounds__(256) phi_amax_kernel(const __nv_bfloat16 *__restrict__ x, int64_t M, int64_t K,
@@ -134,19 +134,17 @@ __global__ void __launch_bounds__(256) phi_amax_kernel(const __nv_bfloat16 *__re
             const uint4 v = __ldg(reinterpret_cast<const uint4 *>(base + (int64_t)row * K + 8 * c));
             const uint32_t q[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const uint32_t mag = q[j] & 0x7fff7fffu;
-                acc = __vmaxu2(acc, mag & ~__vcmpgtu2(mag, 0x7f807f80u));
-            }
+            for (int j = 0; j < 4; ++j)
+                asm("max.bf16x2 %0, %1, %2;" : "=r"(acc) : "r"(acc), "r"(q[j] & 0x7fff7fffu));
         }
     } else {
         for (int row = 0; row < rows; ++row)
             for (int c = threadIdx.x; c < w; c += blockDim.x) {
                 const uint32_t mag = __bfloat16_as_ushort(x[(m0 + row) * K + k0 + c]) & 0x7fffu;
-                acc = __vmaxu2(acc, mag > 0x7f80u ? 0u : mag);
+                asm("max.bf16x2 %0, %1, %2;" : "=r"(acc) : "r"(acc), "r"(mag));
             }
     }
-    float a = __uint_as_float(max(acc & 0xffffu, acc >> 16) << 16);
+    float a = fmaxf(__uint_as_float(acc << 16), __uint_as_float(acc & 0xffff0000u));
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1)
         a = fmaxf(a, __shfl_xor_sync(0xFFFFFFFFu, a, o));
