@@ -206,8 +206,9 @@ def _config(spec, extra=None):
     c = {"workload": spec.name, "M": M, "K": K, "N": N, "main_format": spec.fmt,
          "residual_format": spec.fmt, "phi": "all tiles (phi = 1)", "y_dtype": "bf16",
          "inputs": _inputs_desc(spec.act),
-         "l2": (f"inputs larger than L2 (X {x_mb:.0f} MB, Y {y_mb:.0f} MB per step), no flush"
-                if x_mb + y_mb > 129 else "working set below L2 size")}
+         "l2": (f"inputs larger than L2 (X {x_mb:.0f} MB, Y {y_mb:.0f} MB per step; two buffer sets "
+                f"alternate between steps), no flush" if x_mb + y_mb > 129 else
+                "working set below L2 size (two buffer sets alternate between steps)")}
     if extra:
         c.update(extra)
     return c
@@ -362,31 +363,38 @@ def run_rfq(args):
         elif wop is None:
             wop = wq
         del w
-    xq = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme in ("w4a8", "w8a8") else F, L, Mb, K, device=dev)
-    xr = (None if no_res or scheme in ("w4a8", "w8a8") else
-          rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme == "rfq8" else F, L, Mb, K, device=dev))
-    no_res = xr is None
-    # rfq8: the E4M3 re-encoding of X~ that the GEMM multiplies
-    xq8 = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8, L, Mb, K, device=dev) if scheme == "rfq8" else None
-    phi_buf = (torch.empty(((Mb + 127) // 128) * ((K + 255) // 256), dtype=torch.uint8, device=dev)
-               if args.phi_tau is not None else None)
-    # HiF4: the GEMM takes the exact bf16 expansions of X~ and X^ (expanding
-    # once per activation, not once per output tile inside the GEMM)
-    xq16 = rfq.empty_bf16_operand(M, K, device=dev) if hif4 and not quant_only else None
-    xr16 = rfq.empty_bf16_operand(M, K, device=dev) if hif4 and not quant_only else None
-    y = torch.empty(Mb, max(N, 16), dtype=torch.bfloat16, device=dev)
+    no_res = no_res or scheme in ("w4a8", "w8a8")
+
+    def buffer_set(xd):
+        """The device buffers of one step: X and everything the step writes."""
+        b = {"x": xd,
+             "xq": rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme in ("w4a8", "w8a8") else F, L, Mb, K, device=dev),
+             "xr": None if no_res else
+                   rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme == "rfq8" else F, L, Mb, K, device=dev),
+             # rfq8: the E4M3 re-encoding of X~ that the GEMM multiplies
+             "xq8": rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8, L, Mb, K, device=dev) if scheme == "rfq8" else None,
+             "phi": (torch.empty(((Mb + 127) // 128) * ((K + 255) // 256), dtype=torch.uint8, device=dev)
+                     if amax_phi else None),
+             # HiF4: the GEMM takes the exact bf16 expansions of X~ and X^
+             # (expanding once per activation, not once per output tile)
+             "xq16": rfq.empty_bf16_operand(M, K, device=dev) if hif4 and not quant_only else None,
+             "xr16": rfq.empty_bf16_operand(M, K, device=dev) if hif4 and not quant_only and not no_res else None,
+             "y": torch.empty(Mb, max(N, 16), dtype=torch.bfloat16, device=dev)}
+        return b
+
+    # Two buffer sets, used by alternate steps: no step finds in L2 what the
+    # step before it read or wrote (each set's X plus its outputs exceeds
+    # L2 for every workload but the tiny parity case).
+    bufs = [buffer_set(x), buffer_set(x.clone())]
     y_host = torch.empty(Mb, max(N, 16), dtype=torch.bfloat16).pin_memory()
     wsp = torch.zeros(rfq.rfq_linear_workspace_bytes() // 4, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream(dev)
     # quantizer-only workload: its result (both pathways' codes and scales) is read back
-    host_q = [(torch.empty_like(t, device="cpu").pin_memory(), t)
-              for t in (xq.codes, xq.scales, xr.codes, xr.scales)] if quant_only else []
-    q_bytes = sum(t.numel() for _, t in host_q)
+    q_out = lambda b: [b["xq"].codes, b["xq"].scales, b["xr"].codes, b["xr"].scales]
+    host_q = [torch.empty_like(t, device="cpu").pin_memory() for t in q_out(bufs[0])] if quant_only else []
+    q_bytes = sum(t.numel() for t in host_q)
 
     ev = lambda: torch.cuda.Event(enable_timing=True)
-
-    # the step's input and output buffers (the end-to-end loop double-buffers them)
-    io = {"x": x, "y": y}
 
     # Events between the step's phases, recorded inside the captured graph
     # (event-record nodes): q = the quantizer, x = the HiF4 bf16 expansions
@@ -394,7 +402,10 @@ def run_rfq(args):
     per_step = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(4)]
                 for _ in range(args.steps)]
 
-    def step(i=None):
+    def step(i=None, r=0):
+        """One step on buffer set r; with i, events mark its phases."""
+        bs = bufs[r]
+        x_, xq, xr, xq8, ph, y_ = bs["x"], bs["xq"], bs["xr"], bs["xq8"], bs["phi"], bs["y"]
         # (recorded on the current stream: the capture stream inside the graph)
         mark = ((lambda j: per_step[i][j].record(torch.cuda.current_stream(dev))) if i is not None
                 else (lambda j: None))
@@ -402,39 +413,38 @@ def run_rfq(args):
             # the quantizer runs inside the GEMM: one kernel per step
             for j in range(3):
                 mark(j)
-            rfq.rfq_linear_fused(io["x"], wop, io["y"], rfq.RFQ_OUT_BF16, wsp, stream=None)
+            rfq.rfq_linear_fused(x_, wop, y_, rfq.RFQ_OUT_BF16, wsp, stream=None)
             mark(3)
             return
         mark(0)
         if amax_phi:
-            rfq.rfq_quantize_act(io["x"], xq, xr, phi_buf, mode=rfq.RFQ_FALLBACK_AMAX, tau=args.phi_tau,
+            rfq.rfq_quantize_act(x_, xq, xr, ph, mode=rfq.RFQ_FALLBACK_AMAX, tau=args.phi_tau,
                                  p_s=128, r_s=256, stream=None)
         else:
-            rfq.rfq_quantize_act(io["x"], xq, xr, None,
+            rfq.rfq_quantize_act(x_, xq, xr, None,
                                  mode=rfq.RFQ_FALLBACK_NONE if no_res else rfq.RFQ_FALLBACK_ALL, stream=None)
         mark(1)
         if hif4 and not quant_only:
-            rfq.rfq_dequant(xq, xq16.codes, stream=None)
+            rfq.rfq_dequant(xq, bs["xq16"].codes, stream=None)
             if xr is not None:
-                rfq.rfq_dequant(xr, xr16.codes, stream=None)
+                rfq.rfq_dequant(xr, bs["xr16"].codes, stream=None)
         if xq8 is not None:
             rfq.rfq_convert(xq, xq8, stream=None)
         mark(2)
         if quant_only:
             pass
         elif hif4:
-            rfq.rfq_linear(xq16, xr16 if xr is not None else None, phi_buf if amax_phi else None, 256, wop,
-                           io["y"], rfq.RFQ_OUT_BF16, wsp, stream=None)
+            rfq.rfq_linear(bs["xq16"], bs["xr16"], ph, 256, wop, y_, rfq.RFQ_OUT_BF16, wsp, stream=None)
         elif grouped:
-            rfq.rfq_linear_grouped(xq8 if xq8 is not None else xq, xr, phi_buf if amax_phi else None, 256, group_off,
-                                   wop, N, io["y"], rfq.RFQ_OUT_BF16, wsp, stream=None)
+            rfq.rfq_linear_grouped(xq8 if xq8 is not None else xq, xr, ph, 256, group_off,
+                                   wop, N, y_, rfq.RFQ_OUT_BF16, wsp, stream=None)
         else:
-            rfq.rfq_linear(xq8 if xq8 is not None else xq, xr, phi_buf if amax_phi else None, 256, wop, io["y"],
-                           rfq.RFQ_OUT_BF16, wsp, stream=None)
+            rfq.rfq_linear(xq8 if xq8 is not None else xq, xr, ph, 256, wop, y_, rfq.RFQ_OUT_BF16, wsp,
+                           stream=None)
         mark(3)
 
-    for _ in range(args.warmup):
-        step()
+    for i in range(args.warmup):
+        step(None, i & 1)
     torch.cuda.synchronize()
     if rfq.rfq_workspace_status(wsp) != rfq.RFQ_OK:
         raise RuntimeError("rfq_linear reported a device timeout")
@@ -447,7 +457,7 @@ def run_rfq(args):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g):
             for i in range(args.steps):
-                step(i if instrumented else None)
+                step(i if instrumented else None, i & 1)
         g.replay()          # the first replay uploads the graph
         torch.cuda.synchronize()
         return g
@@ -497,8 +507,6 @@ def run_rfq(args):
     e2e_ms = None
     if not args.no_e2e:
         h2d, d2h = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
-        xs = [x, torch.empty_like(x)]
-        ysb = [y, torch.empty_like(y)]
         x_ready = [torch.cuda.Event(), torch.cuda.Event()]
         x_free = [torch.cuda.Event(), torch.cuda.Event()]
         y_done = [torch.cuda.Event(), torch.cuda.Event()]
@@ -518,24 +526,21 @@ def run_rfq(args):
             with torch.cuda.stream(h2d):
                 if i >= 2:
                     h2d.wait_event(x_free[sl])          # step i - 2 has read this X buffer
-                xs[sl].copy_(x_host, non_blocking=True)
+                bufs[sl]["x"].copy_(x_host, non_blocking=True)
                 x_ready[sl].record(h2d)
             stream.wait_event(x_ready[sl])
             if i >= 2:
-                stream.wait_event(y_free[sl])           # step i - 2's result has left this Y buffer
-            if quant_only and i >= 1:
-                stream.wait_event(y_free[sl ^ 1])       # the quantizer's outputs are single-buffered
-            io["x"], io["y"] = xs[sl], ysb[sl]
-            step()
+                stream.wait_event(y_free[sl])           # step i - 2's result has left this buffer set
+            step(None, sl)
             x_free[sl].record(stream)
             y_done[sl].record(stream)
             with torch.cuda.stream(d2h):
                 d2h.wait_event(y_done[sl])
                 if quant_only:
-                    for dst, src in host_q:
+                    for dst, src in zip(host_q, q_out(bufs[sl])):
                         dst.copy_(src, non_blocking=True)
                 else:
-                    y_host.copy_(ysb[sl], non_blocking=True)
+                    y_host.copy_(bufs[sl]["y"], non_blocking=True)
                 y_free[sl].record(d2h)
         stream.wait_stream(h2d)
         stream.wait_stream(d2h)
@@ -543,14 +548,13 @@ def run_rfq(args):
         torch.cuda.synchronize()
         barrier()
         e2e_ms = e0.elapsed_time(e1) / args.steps
-        io["x"], io["y"] = x, y
     if e2e_ms is not None:
         e2e_ms = _max_over_ranks(e2e_ms, ws, dist, dev)
     if rfq.rfq_workspace_status(wsp) != rfq.RFQ_OK:
         raise RuntimeError("rfq_linear reported a device timeout")
 
     # executed MMA work: the main product, and the residual product on the phi = 1 tiles
-    phi_frac = float(phi_buf.float().mean().item()) if amax_phi else (0.0 if no_res else 1.0)
+    phi_frac = float(bufs[0]["phi"].float().mean().item()) if amax_phi else (0.0 if no_res else 1.0)
     flop = 2.0 * M * N * K * (1.0 + phi_frac)
     pk = _peaks()
     # The timed loop is short (tens of ms at full clocks), so the kernels are
