@@ -77,9 +77,8 @@ def _launches_per_step(quant_only, fused, hif4, no_res, scheme, amax_phi, amax_f
     """This library's kernel launches in one timed step."""
     if quant_only or fused:
         return 1
-    n = 1 + (1 if amax_phi and not amax_fused else 0)   # quantizer (+ the phi amax kernel)
-    if hif4:
-        n += 1 if no_res else 2             # exact bf16 expansions of X~ (and X^)
+    n = 1 + (1 if amax_phi and not amax_fused else 0)   # quantizer (+ the phi amax kernel; the
+                                                        # HiF4 quantizer also writes the bf16 values)
     if scheme == "rfq8":
         n += 1                              # E4M3 re-encoding of X~
     return n + 1                            # GEMM
@@ -397,8 +396,9 @@ def run_rfq(args):
     ev = lambda: torch.cuda.Event(enable_timing=True)
 
     # Events between the step's phases, recorded inside the captured graph
-    # (event-record nodes): q = the quantizer, x = the HiF4 bf16 expansions
-    # or the rfq8 E4M3 re-encoding of X~ (empty otherwise), g = the GEMM.
+    # (event-record nodes): q = the quantizer (for HiF4 it also writes the
+    # bf16 values of X~ and X^), x = the rfq8 E4M3 re-encoding of X~ (empty
+    # otherwise), g = the GEMM.
     per_step = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(4)]
                 for _ in range(args.steps)]
 
@@ -417,17 +417,16 @@ def run_rfq(args):
             mark(3)
             return
         mark(0)
-        if amax_phi:
-            rfq.rfq_quantize_act(x_, xq, xr, ph, mode=rfq.RFQ_FALLBACK_AMAX, tau=args.phi_tau,
-                                 p_s=128, r_s=256, stream=None)
-        else:
-            rfq.rfq_quantize_act(x_, xq, xr, None,
-                                 mode=rfq.RFQ_FALLBACK_NONE if no_res else rfq.RFQ_FALLBACK_ALL, stream=None)
-        mark(1)
+        mode = rfq.RFQ_FALLBACK_AMAX if amax_phi else (rfq.RFQ_FALLBACK_NONE if no_res else rfq.RFQ_FALLBACK_ALL)
+        tau = args.phi_tau if amax_phi else 0.0
         if hif4 and not quant_only:
-            rfq.rfq_dequant(xq, bs["xq16"].codes, stream=None)
-            if xr is not None:
-                rfq.rfq_dequant(xr, bs["xr16"].codes, stream=None)
+            # HiF4: the quantizer also writes the exact bf16 values of X~ and
+            # X^ that the bf16 GEMM multiplies (no separate expansion pass)
+            rfq.rfq_quantize_act_expand(x_, xq, xr, bs["xq16"], bs["xr16"], ph, mode=mode, tau=tau,
+                                        p_s=128, r_s=256, stream=None)
+        else:
+            rfq.rfq_quantize_act(x_, xq, xr, ph, mode=mode, tau=tau, p_s=128, r_s=256, stream=None)
+        mark(1)
         if xq8 is not None:
             rfq.rfq_convert(xq, xq8, stream=None)
         mark(2)
@@ -490,7 +489,7 @@ def run_rfq(args):
         barrier()
     ms = t_start.elapsed_time(t_end) / args.steps
     q_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in per_step)
-    x_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in per_step)   # HiF4 / rfq8 expansions (0 otherwise)
+    x_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in per_step)   # rfq8 re-encoding of X~ (0 otherwise)
     g_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in per_step)
     if quant_only:
         q_ms = ms
@@ -578,8 +577,9 @@ def run_rfq(args):
         t_kernel = "gemm_mxf4_fused_kernel" if fused else (
             "gemm_mxf4_pair_kernel" if M > 128 or grouped else "gemm_mxf4_kernel")
     if hif4:
-        npath = 1 if no_res else 2   # main (and residual) codes + metadata written
-        aq_bytes = Mb * K * 2 + npath * (Mb * K // 2) + npath * (((Mb + 127) // 128) * 128 * (K // 64) * 4)
+        npath = 1 if no_res else 2   # main (and residual) codes + metadata written, and their bf16 values
+        aq_bytes = (Mb * K * 2 + npath * (Mb * K // 2) + npath * (((Mb + 127) // 128) * 128 * (K // 64) * 4)
+                    + (0 if quant_only else npath * Mb * K * 2))
         aq_kernel = "act_quant_hif4_kernel"
     elif f8:
         sfb = ((Mb + 127) // 128) * 128 * K // 32
@@ -652,7 +652,7 @@ def run_rfq(args):
                                          "phi_fraction": phi_frac} if amax_phi else {})}),
             "roofline": roofline,
             "act_quant": act_quant,
-            "expand_ms_per_step": x_ms if (hif4 or scheme == "rfq8") else None,
+            "expand_ms_per_step": x_ms if scheme == "rfq8" else None,
             "e2e": e2e,
             "gpu_launches": _launches_per_step(quant_only, fused, hif4, no_res, scheme, amax_phi,
                                                 amax_fused) * args.steps,

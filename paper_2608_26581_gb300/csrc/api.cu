@@ -189,8 +189,39 @@ rfq_status rfq_quantize_weight(const void *w_bf16, int64_t K, int64_t N, rfq_qte
     return RFQ_ERR_INVALID_ARG;
 }
 
+namespace {
+rfq_status quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_fallback *fb, rfq_qtensor *xq,
+                        rfq_qtensor *xr, uint8_t *phi, void *stream, void *m16, void *r16);
+} // namespace
+
 rfq_status rfq_quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_fallback *fb, rfq_qtensor *xq,
                             rfq_qtensor *xr, uint8_t *phi, void *stream)
+{
+    return quantize_act(x_bf16, M, K, fb, xq, xr, phi, stream, nullptr, nullptr);
+}
+
+rfq_status rfq_quantize_act_expand(const void *x_bf16, int64_t M, int64_t K, const rfq_fallback *fb,
+                                   rfq_qtensor *xq, rfq_qtensor *xr, uint8_t *phi, rfq_qtensor *xq16,
+                                   rfq_qtensor *xr16, void *stream)
+{
+    const rfq_fallback_mode mode = fb ? (rfq_fallback_mode)fb->mode : RFQ_FALLBACK_ALL;
+    if (!xq || !xq16 || (mode != RFQ_FALLBACK_NONE && !xr16) || (mode == RFQ_FALLBACK_NONE && xr16))
+        return RFQ_ERR_INVALID_ARG;
+    if (xq->fmt != RFQ_FMT_HIF4)
+        return RFQ_ERR_UNSUPPORTED;   // the bf16 operands serve the HiF4 GEMM
+    rfq_status s = check_qtensor(xq16, M, K);
+    if (s != RFQ_OK)
+        return s;
+    if (xq16->fmt != RFQ_FMT_BF16 || (xr16 && xr16->fmt != RFQ_FMT_BF16))
+        return RFQ_ERR_INVALID_ARG;
+    if (xr16 && (s = check_qtensor(xr16, M, K)) != RFQ_OK)
+        return s;
+    return quantize_act(x_bf16, M, K, fb, xq, xr, phi, stream, xq16->codes, xr16 ? xr16->codes : nullptr);
+}
+
+namespace {
+rfq_status quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_fallback *fb, rfq_qtensor *xq,
+                        rfq_qtensor *xr, uint8_t *phi, void *stream, void *m16, void *r16)
 {
     rfq_fallback def = {RFQ_FALLBACK_ALL, 0.f, 128, 256};
     const rfq_fallback &f = fb ? *fb : def;
@@ -257,10 +288,11 @@ rfq_status rfq_quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_
         }
         return from_cuda(launch_act_quant_hif4(x_bf16, M, K, f.mode, f.p_s, f.r_s, xq->codes, xq->scales,
                                                res ? xr->codes : nullptr, res ? xr->scales : nullptr, phi,
-                                               xq->scale_layout, st));
+                                               xq->scale_layout, st, m16, r16));
     }
     return RFQ_ERR_INVALID_ARG;
 }
+} // namespace
 
 size_t rfq_linear_workspace_bytes(void) { return 256; }
 

@@ -14,7 +14,8 @@
 // Every comparison is exact in fp32 (all products carry a few significant
 // bits), so the kernels reproduce the fp64 definition bit for bit.
 //
-//   act_quant_hif4     main (+ residual, Sec. 4.3) codes and metadata of X
+//   act_quant_hif4     main (+ residual, Sec. 4.3) codes and metadata of X,
+//                      optionally with their exact bf16 values
 //   weight_quant_hif4  W [K x N] -> K-major HiF4
 //   dequant_hif4       -> fp32 or bf16 values
 //
@@ -135,17 +136,32 @@ __device__ __forceinline__ int64_t meta_index(int64_t m, int64_t blk, int64_t ro
 // Quantizes x (main), and with RES its residual x - x~ (Sec. 4.3).  Items
 // are (row, 1024-element segment): a warp loads its four 16-byte chunks per
 // lane up front, and the row and block indices come from the item without a
-// 64-bit division per chunk.
+// 64-bit division per chunk.  With EXP the kernel also writes the exact bf16
+// values of X~ (and X^; zeros where phi = 0) as [M][K] row-major, the
+// operands of the bf16 tensor-core GEMM: every HiF4 value has at most six
+// significant bits and an exponent inside bf16's range.
 constexpr int kHSeg = 1024;
 constexpr int kHU = kHSeg / 256;
 
-template <bool RES, bool PHI, int LAYOUT>
+__device__ __forceinline__ uint4 bf16x8_pack(const float (&v)[8]) // exact for the values above
+{
+    uint32_t p[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        __nv_bfloat162 b = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+        p[i] = *reinterpret_cast<uint32_t *>(&b);
+    }
+    return make_uint4(p[0], p[1], p[2], p[3]);
+}
+
+template <bool RES, bool PHI, int LAYOUT, bool EXP>
 __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__restrict__ x, int64_t M, int64_t K,
                                                             uint32_t *__restrict__ mcodes,
                                                             uint32_t *__restrict__ mmeta,
                                                             uint32_t *__restrict__ rcodes,
                                                             uint32_t *__restrict__ rmeta,
-                                                            const uint8_t *__restrict__ phi, int p_s, int r_s)
+                                                            const uint8_t *__restrict__ phi, int p_s, int r_s,
+                                                            uint4 *__restrict__ m16, uint4 *__restrict__ r16)
 {
     const int lane = threadIdx.x & 31;
     const int g = lane & 7;
@@ -200,6 +216,8 @@ __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__rest
                 mcodes[c] = code;
                 if (g == 0)
                     mmeta[meta_index<LAYOUT>(m, blk, M, kblocks)] = am == 0.f ? 0u : (bits | (uint32_t)sb);
+                if (EXP)
+                    m16[c] = bf16x8_pack(deq);
             }
             if (RES) {
                 const bool on = !PHI || (ok && prow[(cr * 8) / r_s] != 0);
@@ -225,6 +243,8 @@ __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__rest
                     if (g == 0)
                         rmeta[meta_index<LAYOUT>(m, blk, M, kblocks)] =
                             (on && ra > 0.f) ? (rbits | (uint32_t)rsb) : 0u;
+                    if (EXP)
+                        r16[c] = on ? bf16x8_pack(rdeq) : make_uint4(0, 0, 0, 0);
                 }
             }
         }
@@ -314,7 +334,7 @@ int grid_for(int64_t work, int threads, int max_blocks)
 
 cudaError_t launch_act_quant_hif4(const void *x, int64_t M, int64_t K, int mode, int p_s, int r_s, void *mcodes,
                                   void *mmeta, void *rcodes, void *rmeta, const uint8_t *phi, int layout,
-                                  cudaStream_t st)
+                                  cudaStream_t st, void *m16, void *r16)
 {
     const int64_t items = M * ((K / 8 + kHSeg / 8 - 1) / (kHSeg / 8));
     const int blocks = grid_for(items * 32, 256, 152 * 24);
@@ -323,18 +343,26 @@ cudaError_t launch_act_quant_hif4(const void *x, int64_t M, int64_t K, int mode,
     auto *mm = static_cast<uint32_t *>(mmeta);
     auto *rc = static_cast<uint32_t *>(rcodes);
     auto *rm = static_cast<uint32_t *>(rmeta);
-#define RFQ_HQ(RES, PHI, LAY)                                                                                     \
-    act_quant_hif4_kernel<RES, PHI, LAY><<<blocks, 256, 0, st>>>(xi, M, K, mc, mm, rc, rm, phi, p_s, r_s)
+    auto *e0 = static_cast<uint4 *>(m16);
+    auto *e1 = static_cast<uint4 *>(r16);
+#define RFQ_HQ(RES, PHI, LAY, EXP)                                                                                \
+    act_quant_hif4_kernel<RES, PHI, LAY, EXP><<<blocks, 256, 0, st>>>(xi, M, K, mc, mm, rc, rm, phi, p_s, r_s, e0, e1)
+#define RFQ_HQ_E(RES, PHI, LAY)                                                                                   \
+    do {                                                                                                          \
+        if (e0) RFQ_HQ(RES, PHI, LAY, true);                                                                      \
+        else RFQ_HQ(RES, PHI, LAY, false);                                                                        \
+    } while (0)
     if (mode == RFQ_FALLBACK_NONE) {
-        if (layout == RFQ_SCALE_MMA) RFQ_HQ(false, false, RFQ_SCALE_MMA);
-        else RFQ_HQ(false, false, RFQ_SCALE_ROWMAJOR);
+        if (layout == RFQ_SCALE_MMA) RFQ_HQ_E(false, false, RFQ_SCALE_MMA);
+        else RFQ_HQ_E(false, false, RFQ_SCALE_ROWMAJOR);
     } else if (mode == RFQ_FALLBACK_ALL) {
-        if (layout == RFQ_SCALE_MMA) RFQ_HQ(true, false, RFQ_SCALE_MMA);
-        else RFQ_HQ(true, false, RFQ_SCALE_ROWMAJOR);
+        if (layout == RFQ_SCALE_MMA) RFQ_HQ_E(true, false, RFQ_SCALE_MMA);
+        else RFQ_HQ_E(true, false, RFQ_SCALE_ROWMAJOR);
     } else {
-        if (layout == RFQ_SCALE_MMA) RFQ_HQ(true, true, RFQ_SCALE_MMA);
-        else RFQ_HQ(true, true, RFQ_SCALE_ROWMAJOR);
+        if (layout == RFQ_SCALE_MMA) RFQ_HQ_E(true, true, RFQ_SCALE_MMA);
+        else RFQ_HQ_E(true, true, RFQ_SCALE_ROWMAJOR);
     }
+#undef RFQ_HQ_E
 #undef RFQ_HQ
     return cudaGetLastError();
 }

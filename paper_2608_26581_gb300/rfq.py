@@ -28,7 +28,8 @@ STATUS_NAMES = {0: "RFQ_OK", 1: "RFQ_ERR_INVALID_ARG", 2: "RFQ_ERR_SHAPE", 3: "R
 
 EXPORTED = ("rfq_status_string", "rfq_qtensor_bytes", "rfq_quantize_weight", "rfq_quantize_act",
             "rfq_linear_workspace_bytes", "rfq_linear", "rfq_workspace_status", "rfq_dequant",
-            "rfq_linear_noalloc", "rfq_linear_fused", "rfq_convert", "rfq_linear_grouped", "rfq_check_finite")
+            "rfq_linear_noalloc", "rfq_linear_fused", "rfq_convert", "rfq_linear_grouped", "rfq_check_finite",
+            "rfq_quantize_act_expand")
 
 
 class RFQError(RuntimeError):
@@ -67,6 +68,8 @@ def load_library(path: str = LIB_PATH):
         lib.rfq_quantize_weight.argtypes = [P, I64, I64, QTP, P]
         lib.rfq_quantize_act.restype = I32
         lib.rfq_quantize_act.argtypes = [P, I64, I64, ctypes.POINTER(_FB), QTP, QTP, P, P]
+        lib.rfq_quantize_act_expand.restype = I32
+        lib.rfq_quantize_act_expand.argtypes = [P, I64, I64, ctypes.POINTER(_FB), QTP, QTP, P, QTP, QTP, P]
         lib.rfq_linear_workspace_bytes.restype = SZ
         lib.rfq_linear_workspace_bytes.argtypes = []
         lib.rfq_linear.restype = I32
@@ -159,6 +162,22 @@ def rfq_quantize_act(x: torch.Tensor, xq: QTensor, xr: QTensor | None, phi: torc
     _check(load_library().rfq_quantize_act(_ptr(x), M, K, ctypes.byref(fb), ctypes.byref(q),
                                            ctypes.byref(r) if r is not None else None, _ptr(phi),
                                            _stream(stream)), "rfq_quantize_act")
+
+
+def rfq_quantize_act_expand(x: torch.Tensor, xq: QTensor, xr: QTensor | None, xq16: QTensor,
+                            xr16: QTensor | None, phi: torch.Tensor | None = None, mode: int = RFQ_FALLBACK_ALL,
+                            tau: float = 0.0, p_s: int = 128, r_s: int = 256, stream=None):
+    """HiF4 activation quantization that also writes the exact bf16 values of
+    X~ (into xq16) and X^ (into xr16) in the same pass."""
+    M, K = x.shape
+    fb = _FB(mode, tau, p_s, r_s)
+    q, q16 = xq.c(), xq16.c()
+    r = xr.c() if xr is not None else None
+    r16 = xr16.c() if xr16 is not None else None
+    _check(load_library().rfq_quantize_act_expand(
+        _ptr(x), M, K, ctypes.byref(fb), ctypes.byref(q), ctypes.byref(r) if r is not None else None, _ptr(phi),
+        ctypes.byref(q16), ctypes.byref(r16) if r16 is not None else None, _stream(stream)),
+        "rfq_quantize_act_expand")
 
 
 def rfq_linear_workspace_bytes() -> int:

@@ -106,3 +106,27 @@ def test_fused_linear_host_checks(lib):
         rfq.RFQ_ERR_UNSUPPORTED
     assert lib.rfq_linear_fused(P(8), 4, 128, ctypes.byref(wq), None, P(16), 1, P(16), None) == \
         rfq.RFQ_ERR_ALIGNMENT
+
+
+def test_quantize_act_expand_host_checks(lib):
+    """rfq_quantize_act_expand validates on the host: the bf16 outputs must be
+    present (xr16 exactly when there is a residual), of format RFQ_FMT_BF16,
+    shape [M][K] and 16-byte aligned, and the pathway must be HiF4."""
+    from paper_2608_26581_gb300 import rfq
+    P = ctypes.c_void_p
+    M, K = 4, 128
+    hq = rfq._QT(rfq.RFQ_FMT_HIF4, rfq.RFQ_SCALE_MMA, M, K, 16, 16)
+    mq = rfq._QT(rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA, M, K, 16, 16)
+    b16 = rfq._QT(rfq.RFQ_FMT_BF16, 0, M, K, 16, 0)
+    b16_shape = rfq._QT(rfq.RFQ_FMT_BF16, 0, M, 64, 16, 0)
+    b16_align = rfq._QT(rfq.RFQ_FMT_BF16, 0, M, K, 8, 0)
+    none = rfq._FB(rfq.RFQ_FALLBACK_NONE, 0.0, 128, 256)
+    r = ctypes.byref
+    call = lib.rfq_quantize_act_expand
+    assert call(P(16), M, K, None, r(hq), r(hq), None, None, r(b16), None) == rfq.RFQ_ERR_INVALID_ARG
+    assert call(P(16), M, K, None, r(hq), r(hq), None, r(b16), None, None) == rfq.RFQ_ERR_INVALID_ARG
+    assert call(P(16), M, K, r(none), r(hq), None, None, r(b16), r(b16), None) == rfq.RFQ_ERR_INVALID_ARG
+    assert call(P(16), M, K, None, r(mq), r(mq), None, r(b16), r(b16), None) == rfq.RFQ_ERR_UNSUPPORTED
+    assert call(P(16), M, K, None, r(hq), r(hq), None, r(b16_shape), r(b16), None) == rfq.RFQ_ERR_SHAPE
+    assert call(P(16), M, K, None, r(hq), r(hq), None, r(b16), r(hq), None) == rfq.RFQ_ERR_INVALID_ARG
+    assert call(P(16), M, K, None, r(hq), r(hq), None, r(b16_align), r(b16), None) == rfq.RFQ_ERR_ALIGNMENT

@@ -128,6 +128,44 @@ def test_dequant_fp32_and_bf16_exact(orc):
                 assert np.array_equal(out.double().cpu().numpy(), ref)
 
 
+@pytest.mark.parametrize("mode,tau,r_s,layout", [
+    (rfq.RFQ_FALLBACK_ALL, 0.0, 256, rfq.RFQ_SCALE_MMA), (rfq.RFQ_FALLBACK_ALL, 0.0, 256, rfq.RFQ_SCALE_ROWMAJOR),
+    (rfq.RFQ_FALLBACK_NONE, 0.0, 256, rfq.RFQ_SCALE_MMA), (rfq.RFQ_FALLBACK_AMAX, 10.0, 128, rfq.RFQ_SCALE_MMA)])
+def test_quantize_act_expand(orc, mode, tau, r_s, layout):
+    """The quantizer's own bf16 values of X~ and X^ are bit for bit the
+    oracle's dequantization of its codes (Sec. 3.3 decoder), with X^ zero on
+    phi = 0 tiles; the codes and metadata are those of rfq_quantize_act."""
+    M, K = 300, 1024
+    xb = make_activation(ActSpec(M, K, "laplace", body_scale=0.3, chan_count=5, chan_scale=50.0, seed=13))
+    xb[7, :64] = 0                                   # an all-zero block
+    xb[9, 64] = 0x8000                               # a negative zero
+    x = to_dev_bf16(xb)
+    res = mode != rfq.RFQ_FALLBACK_NONE
+    xq = rfq.empty_qtensor(H, layout, M, K)
+    xr = rfq.empty_qtensor(H, layout, M, K) if res else None
+    xq16 = rfq.empty_bf16_operand(M, K)
+    xr16 = rfq.empty_bf16_operand(M, K) if res else None
+    for t in (xq16, xr16):
+        if t is not None:
+            t.codes.fill_(float("nan"))
+    phi = torch.empty(((M + 127) // 128) * ((K + r_s - 1) // r_s), dtype=torch.uint8, device=DEV)
+    rfq.rfq_quantize_act_expand(x, xq, xr, xq16, xr16, phi, mode=mode, tau=tau, p_s=128, r_s=r_s)
+    torch.cuda.synchronize()
+    ref = orc.quantize_act(xb, orc.FMT_HIF4, mode, tau, 128, r_s)
+    mc, mm = qtensor_host(xq)
+    assert np.array_equal(mc, ref["main_codes"]) and np.array_equal(mm, ref["main_scales"])
+    pairs = [(xq16, ref["main_codes"], ref["main_scales"])]
+    if res:
+        rc, rm = qtensor_host(xr)
+        assert np.array_equal(rc, ref["res_codes"]) and np.array_equal(rm, ref["res_scales"])
+        pairs.append((xr16, ref["res_codes"], ref["res_scales"]))
+    for t, c, m in pairs:
+        want = orc.dequant(orc.FMT_HIF4, c, m, M, K)
+        got = t.codes.view(torch.int16).cpu().numpy().view(np.uint16)
+        assert np.array_equal(got, f32_to_bf16_bits(want.astype(np.float32))), "bf16 values differ"
+        assert np.array_equal(np.signbit(got.view(np.int16)), np.signbit(want)), "signs of zero differ"
+
+
 def _expand(q):
     t = rfq.empty_bf16_operand(q.rows, q.k)
     rfq.rfq_dequant(q, t.codes)
