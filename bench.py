@@ -79,8 +79,6 @@ def _launches_per_step(quant_only, fused, hif4, no_res, scheme, amax_phi, amax_f
         return 1
     n = 1 + (1 if amax_phi and not amax_fused else 0)   # quantizer (+ the phi amax kernel; the
                                                         # HiF4 quantizer also writes the bf16 values)
-    if scheme == "rfq8":
-        n += 1                              # E4M3 re-encoding of X~
     return n + 1                            # GEMM
 
 
@@ -313,9 +311,10 @@ def run_rfq(args):
     if no_res and (fused or quant_only or amax_phi):
         raise SystemExit("--no-residual applies to the two-kernel linear workloads without --phi-tau")
     # MXFP8 schemes (Table 1 baselines and the FP4-to-FP8 residual of Sec. 4.2):
-    #   rfq8: MXFP4 main + MXFP8 residual, both multiplied as E4M3 (X~ and W~
-    #         re-encoded exactly by rfq_convert); w4a8: MXFP8 X x MXFP4 W
-    #         (re-encoded); w8a8: MXFP8 X x MXFP8 W.  All on kind::mxf8f6f4.
+    #   rfq8: MXFP4 main + MXFP8 residual, both multiplied as E4M3 (X~
+    #         re-encoded exactly by the quantizer in the same pass, W~ by
+    #         rfq_convert offline); w4a8: MXFP8 X x MXFP4 W (re-encoded);
+    #         w8a8: MXFP8 X x MXFP8 W.  All on kind::mxf8f6f4.
     scheme = args.scheme
     f8 = scheme != "rfq4"
     if f8 and (hif4 or quant_only or fused or no_res):
@@ -397,8 +396,8 @@ def run_rfq(args):
 
     # Events between the step's phases, recorded inside the captured graph
     # (event-record nodes): q = the quantizer (for HiF4 it also writes the
-    # bf16 values of X~ and X^), x = the rfq8 E4M3 re-encoding of X~ (empty
-    # otherwise), g = the GEMM.
+    # bf16 values of X~ and X^, for rfq8 X~ as E4M3), g = the GEMM (events 2
+    # and 3; event 1 = event 2 marks the end of the quantizer).
     per_step = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(4)]
                 for _ in range(args.steps)]
 
@@ -424,11 +423,13 @@ def run_rfq(args):
             # X^ that the bf16 GEMM multiplies (no separate expansion pass)
             rfq.rfq_quantize_act_expand(x_, xq, xr, bs["xq16"], bs["xr16"], ph, mode=mode, tau=tau,
                                         p_s=128, r_s=256, stream=None)
+        elif xq8 is not None:
+            # rfq8: the quantizer also writes X~ re-encoded as MXFP8 (E4M3)
+            rfq.rfq_quantize_act_expand(x_, xq, xr, xq8, None, ph, mode=mode, tau=tau, p_s=128, r_s=256,
+                                        stream=None)
         else:
             rfq.rfq_quantize_act(x_, xq, xr, ph, mode=mode, tau=tau, p_s=128, r_s=256, stream=None)
         mark(1)
-        if xq8 is not None:
-            rfq.rfq_convert(xq, xq8, stream=None)
         mark(2)
         if quant_only:
             pass
@@ -489,7 +490,6 @@ def run_rfq(args):
         barrier()
     ms = t_start.elapsed_time(t_end) / args.steps
     q_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in per_step)
-    x_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in per_step)   # rfq8 re-encoding of X~ (0 otherwise)
     g_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in per_step)
     if quant_only:
         q_ms = ms
@@ -583,7 +583,9 @@ def run_rfq(args):
         aq_kernel = "act_quant_hif4_kernel"
     elif f8:
         sfb = ((Mb + 127) // 128) * 128 * K // 32
-        aq_bytes = (Mb * K * 2 + Mb * K // 2 + Mb * K + 2 * sfb if scheme == "rfq8" else Mb * K * 2 + Mb * K + sfb)
+        # rfq8: X read, X~ codes (E2M1) and scales, X^ (E4M3) and scales, X~ as E4M3 and scales
+        aq_bytes = (Mb * K * 2 + Mb * K // 2 + Mb * K + 2 * sfb + Mb * K + sfb if scheme == "rfq8"
+                    else Mb * K * 2 + Mb * K + sfb)
         aq_kernel = "act_quant8_kernel"
     else:
         npath = 1 if no_res else 2
@@ -652,7 +654,6 @@ def run_rfq(args):
                                          "phi_fraction": phi_frac} if amax_phi else {})}),
             "roofline": roofline,
             "act_quant": act_quant,
-            "expand_ms_per_step": x_ms if scheme == "rfq8" else None,
             "e2e": e2e,
             "gpu_launches": _launches_per_step(quant_only, fused, hif4, no_res, scheme, amax_phi,
                                                 amax_fused) * args.steps,

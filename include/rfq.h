@@ -164,20 +164,26 @@ RFQ_API rfq_status rfq_quantize_weight(const void *w_bf16, int64_t K, int64_t N,
 RFQ_API rfq_status rfq_quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_fallback *fb,
                             rfq_qtensor *xq, rfq_qtensor *xr, uint8_t *phi, void *stream);
 
-/* rfq_quantize_act for HiF4 (Sec. 3.3, Sec. 4.3) that in the same pass over
- * X also writes the exact bf16 values of X~ and X^ (the products of
- * rfq_dequant(xq) and rfq_dequant(xr)), the operands rfq_linear multiplies on
- * the bf16 tensor path.  Every HiF4 value has at most six significant bits
- * and an exponent inside bf16's range, so the values are exact; the X^
- * values of phi = 0 tiles are zero.  xq (and xr) as for rfq_quantize_act,
- * with fmt RFQ_FMT_HIF4 (else RFQ_ERR_UNSUPPORTED); xq16, xr16: caller-owned
- * RFQ_FMT_BF16 operands of rows = M, k = K (device bf16 [M][K] row-major,
- * 16-byte aligned); xr16 is required with a residual and must be NULL when
- * fb->mode == RFQ_FALLBACK_NONE.  Asynchronous on `stream`.
+/* rfq_quantize_act that in the same pass over X also writes X~ (and X^) in
+ * the form rfq_linear multiplies, replacing a separate conversion pass:
+ *   xq, xr HiF4 (Sec. 3.3):  xq_op (and xr_op) receive the exact bf16 values
+ *       of X~ (and X^), the products of rfq_dequant(xq) and rfq_dequant(xr):
+ *       every HiF4 value has at most six significant bits and an exponent
+ *       inside bf16's range.  RFQ_FMT_BF16 operands of rows = M, k = K
+ *       (device bf16 [M][K] row-major, 16-byte aligned); xr_op is required
+ *       with a residual and must be NULL when fb->mode == RFQ_FALLBACK_NONE.
+ *       X^ values of phi = 0 tiles are zero.
+ *   xq MXFP4, xr MXFP8 (the FP4-to-FP8 residual, Sec. 4.2):  xq_op receives
+ *       X~ re-encoded as MXFP8 (RFQ_FMT_MXFP8, the layout of xq), the
+ *       product of rfq_convert(xq): every E2M1 value is an E4M3 value, so
+ *       the codes change and the scale bytes do not.  xr_op must be NULL
+ *       (X^ is already MXFP8) and the mode must have a residual.
+ * Other format combinations return RFQ_ERR_UNSUPPORTED.  xq, xr, phi and fb
+ * as for rfq_quantize_act.  Asynchronous on `stream`.
  * Errors: as rfq_quantize_act. */
 RFQ_API rfq_status rfq_quantize_act_expand(const void *x_bf16, int64_t M, int64_t K, const rfq_fallback *fb,
-                                           rfq_qtensor *xq, rfq_qtensor *xr, uint8_t *phi, rfq_qtensor *xq16,
-                                           rfq_qtensor *xr16, void *stream);
+                                           rfq_qtensor *xq, rfq_qtensor *xr, uint8_t *phi, rfq_qtensor *xq_op,
+                                           rfq_qtensor *xr_op, void *stream);
 
 /* Bytes of device workspace rfq_linear needs (a status word, padded). */
 RFQ_API size_t rfq_linear_workspace_bytes(void);

@@ -190,6 +190,9 @@ rfq_status rfq_quantize_weight(const void *w_bf16, int64_t K, int64_t N, rfq_qte
 }
 
 namespace {
+// m16, r16: the GEMM operand forms written in the same pass (HiF4: the bf16
+// values of X~ and X^; MXFP4 main with an MXFP8 residual: the MXFP8 codes and
+// scales of X~); null for none
 rfq_status quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_fallback *fb, rfq_qtensor *xq,
                         rfq_qtensor *xr, uint8_t *phi, void *stream, void *m16, void *r16);
 } // namespace
@@ -201,22 +204,35 @@ rfq_status rfq_quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_
 }
 
 rfq_status rfq_quantize_act_expand(const void *x_bf16, int64_t M, int64_t K, const rfq_fallback *fb,
-                                   rfq_qtensor *xq, rfq_qtensor *xr, uint8_t *phi, rfq_qtensor *xq16,
-                                   rfq_qtensor *xr16, void *stream)
+                                   rfq_qtensor *xq, rfq_qtensor *xr, uint8_t *phi, rfq_qtensor *xq_op,
+                                   rfq_qtensor *xr_op, void *stream)
 {
     const rfq_fallback_mode mode = fb ? (rfq_fallback_mode)fb->mode : RFQ_FALLBACK_ALL;
-    if (!xq || !xq16 || (mode != RFQ_FALLBACK_NONE && !xr16) || (mode == RFQ_FALLBACK_NONE && xr16))
+    if (!xq || !xq_op)
+        return RFQ_ERR_INVALID_ARG;
+    rfq_status s;
+    if (xq->fmt == RFQ_FMT_MXFP4 && xr && xr->fmt == RFQ_FMT_MXFP8) {
+        // the FP4-to-FP8 residual: X~ re-encoded as MXFP8 for the E4M3 GEMM;
+        // the residual is already MXFP8, so there is no second operand
+        if (mode == RFQ_FALLBACK_NONE || xr_op)
+            return RFQ_ERR_INVALID_ARG;
+        if ((s = check_qtensor(xq_op, M, K)) != RFQ_OK)
+            return s;
+        if (xq_op->fmt != RFQ_FMT_MXFP8 || xq_op->scale_layout != xq->scale_layout)
+            return RFQ_ERR_INVALID_ARG;
+        return quantize_act(x_bf16, M, K, fb, xq, xr, phi, stream, xq_op->codes, xq_op->scales);
+    }
+    if ((mode != RFQ_FALLBACK_NONE && !xr_op) || (mode == RFQ_FALLBACK_NONE && xr_op))
         return RFQ_ERR_INVALID_ARG;
     if (xq->fmt != RFQ_FMT_HIF4)
         return RFQ_ERR_UNSUPPORTED;   // the bf16 operands serve the HiF4 GEMM
-    rfq_status s = check_qtensor(xq16, M, K);
-    if (s != RFQ_OK)
+    if ((s = check_qtensor(xq_op, M, K)) != RFQ_OK)
         return s;
-    if (xq16->fmt != RFQ_FMT_BF16 || (xr16 && xr16->fmt != RFQ_FMT_BF16))
+    if (xq_op->fmt != RFQ_FMT_BF16 || (xr_op && xr_op->fmt != RFQ_FMT_BF16))
         return RFQ_ERR_INVALID_ARG;
-    if (xr16 && (s = check_qtensor(xr16, M, K)) != RFQ_OK)
+    if (xr_op && (s = check_qtensor(xr_op, M, K)) != RFQ_OK)
         return s;
-    return quantize_act(x_bf16, M, K, fb, xq, xr, phi, stream, xq16->codes, xr16 ? xr16->codes : nullptr);
+    return quantize_act(x_bf16, M, K, fb, xq, xr, phi, stream, xq_op->codes, xr_op ? xr_op->codes : nullptr);
 }
 
 namespace {
@@ -269,7 +285,7 @@ rfq_status quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_fall
     }
     if (res && xr->fmt == RFQ_FMT_MXFP8)
         return from_cuda(launch_act_quant_rfq8(x_bf16, M, K, f.mode, f.tau, f.p_s, f.r_s, xq->codes, xq->scales,
-                                               xr->codes, xr->scales, phi, xq->scale_layout, st));
+                                               xr->codes, xr->scales, phi, xq->scale_layout, st, m16, r16));
     if (xq->fmt == RFQ_FMT_MXFP4)
         return from_cuda(launch_act_quant_mxfp4(x_bf16, M, K, f.mode, f.tau, f.p_s, f.r_s, xq->codes, xq->scales,
                                                 res ? xr->codes : nullptr, res ? xr->scales : nullptr, phi,

@@ -28,9 +28,10 @@ __host__ __device__ inline int64_t sf_mma_offset(int64_t m, int64_t b, int64_t k
 // ---- MXFP8 (E4M3) quantization and the FP4-to-FP8 residual (quant_mxfp8.cu)
 cudaError_t launch_act_quant_mxfp8(const void *x, int64_t M, int64_t K, void *codes, void *scales, int layout,
                                    cudaStream_t st);
+// m8codes / m8scales (may be null): X~ re-encoded as MXFP8 in the same pass
 cudaError_t launch_act_quant_rfq8(const void *x, int64_t M, int64_t K, int mode, float tau, int p_s, int r_s,
                                   void *mcodes, void *mscales, void *rcodes, void *rscales, uint8_t *phi, int layout,
-                                  cudaStream_t st);
+                                  cudaStream_t st, void *m8codes = nullptr, void *m8scales = nullptr);
 cudaError_t launch_weight_quant_mxfp8(const void *w, int64_t K, int64_t N, void *codes, void *scales, int layout,
                                       cudaStream_t st);
 cudaError_t launch_convert_mxfp4_mxfp8(const void *src_codes, const void *src_scales, int64_t rows, int64_t k,

@@ -2,7 +2,8 @@
 // of Sec. 3.2 Eqs. 3-4) and the FP4-to-FP8 residual pathway (Sec. 4.2,
 // Sec. 4.3):
 //   act_quant_mxfp8      X -> E4M3 codes + E8M0 scales (W4A8 / W8A8 activations)
-//   act_quant_rfq8       X~ = Q_MXFP4(X) and X^ = Q_MXFP8(X - X~) in one pass
+//   act_quant_rfq8       X~ = Q_MXFP4(X) and X^ = Q_MXFP8(X - X~) in one pass,
+//                        optionally with X~ re-encoded as MXFP8
 //   weight_quant_mxfp8   W [K x N] -> K-major E4M3 codes + scales
 //   convert_mxfp4_mxfp8  MXFP4 codes -> E4M3 codes of the same values (exact:
 //                        every E2M1 value is an E4M3 value), scales unchanged
@@ -86,13 +87,16 @@ constexpr int kU = kSeg / 256;
 
 // One warp per (row, 1024-element segment); four lanes per 32-element block.
 // RFQ8 = false: X -> MXFP8.  RFQ8 = true: X -> MXFP4 main codes and the
-// MXFP8 residual X - X~ (zero on phi = 0 tiles when PHI).
-template <bool RFQ8, bool PHI, int LAYOUT>
+// MXFP8 residual X - X~ (zero on phi = 0 tiles when PHI); with OP also X~
+// re-encoded as MXFP8 (the E4M3 code of each E2M1 value, which is exact,
+// under the same scale byte), the operand the E4M3 GEMM multiplies.
+template <bool RFQ8, bool PHI, int LAYOUT, bool OP = false>
 __global__ void __launch_bounds__(256) act_quant8_kernel(const uint4 *__restrict__ x, int64_t M, int64_t K,
                                                         uint8_t *__restrict__ mcodes, uint8_t *__restrict__ mscales,
                                                         uint8_t *__restrict__ rcodes, uint8_t *__restrict__ rscales,
                                                         const uint8_t *__restrict__ phi, int p_s, int r_s,
-                                                        int64_t pad_rows)
+                                                        int64_t pad_rows, uint8_t *__restrict__ m8codes = nullptr,
+                                                        uint8_t *__restrict__ m8scales = nullptr)
 {
     const int lane = threadIdx.x & 31;
     const int kchunks = (int)(K >> 3);
@@ -109,6 +113,8 @@ __global__ void __launch_bounds__(256) act_quant8_kernel(const uint4 *__restrict
             mscales[off] = 0;
             if (RFQ8)
                 rscales[off] = 0;
+            if (OP)
+                m8scales[off] = 0;
         }
     }
 
@@ -153,9 +159,13 @@ __global__ void __launch_bounds__(256) act_quant8_kernel(const uint4 *__restrict
                 if (ok) {
                     reinterpret_cast<uint32_t *>(mcodes + m * (K >> 1))[c] = q4.code;
                     *reinterpret_cast<uint2 *>(rcodes + m * K + (int64_t)c * 8) = on ? rq : make_uint2(0, 0);
+                    if (OP)
+                        *reinterpret_cast<uint2 *>(m8codes + m * K + (int64_t)c * 8) = e4m3x8(q);
                     if ((lane & 3) == 0) {
                         mscales[soff] = (uint8_t)q4.sb;
                         rscales[soff] = on ? (uint8_t)rb : 0;
+                        if (OP)
+                            m8scales[soff] = (uint8_t)q4.sb;
                     }
                 }
             }
@@ -295,7 +305,7 @@ cudaError_t launch_act_quant_mxfp8(const void *x, int64_t M, int64_t K, void *co
 
 cudaError_t launch_act_quant_rfq8(const void *x, int64_t M, int64_t K, int mode, float tau, int p_s, int r_s,
                                   void *mcodes, void *mscales, void *rcodes, void *rscales, uint8_t *phi, int layout,
-                                  cudaStream_t st)
+                                  cudaStream_t st, void *m8codes, void *m8scales)
 {
     if (mode == RFQ_FALLBACK_AMAX) {
         cudaError_t e = launch_phi_amax(x, M, K, p_s, r_s, tau, phi, st);
@@ -315,8 +325,15 @@ cudaError_t launch_act_quant_rfq8(const void *x, int64_t M, int64_t K, int mode,
     auto *rc = static_cast<uint8_t *>(rcodes);
     auto *rs = static_cast<uint8_t *>(rscales);
     const bool sel = mode == RFQ_FALLBACK_AMAX;
-#define RFQ_AQ8(PHI, LAY) \
-    act_quant8_kernel<true, PHI, LAY><<<blocks, 256, 0, st>>>(xi, M, K, mc, ms, rc, rs, phi, p_s, r_s, pad)
+    auto *oc = static_cast<uint8_t *>(m8codes);
+    auto *os = static_cast<uint8_t *>(m8scales);
+#define RFQ_AQ8O(PHI, LAY, OP)                                                                                    \
+    act_quant8_kernel<true, PHI, LAY, OP><<<blocks, 256, 0, st>>>(xi, M, K, mc, ms, rc, rs, phi, p_s, r_s, pad, oc, os)
+#define RFQ_AQ8(PHI, LAY)                                                                                         \
+    do {                                                                                                          \
+        if (oc) RFQ_AQ8O(PHI, LAY, true);                                                                         \
+        else RFQ_AQ8O(PHI, LAY, false);                                                                           \
+    } while (0)
     if (layout == RFQ_SCALE_MMA) {
         if (sel) RFQ_AQ8(true, RFQ_SCALE_MMA);
         else RFQ_AQ8(false, RFQ_SCALE_MMA);
@@ -324,6 +341,7 @@ cudaError_t launch_act_quant_rfq8(const void *x, int64_t M, int64_t K, int mode,
         if (sel) RFQ_AQ8(true, RFQ_SCALE_ROWMAJOR);
         else RFQ_AQ8(false, RFQ_SCALE_ROWMAJOR);
     }
+#undef RFQ_AQ8O
 #undef RFQ_AQ8
     return cudaGetLastError();
 }

@@ -164,19 +164,21 @@ def rfq_quantize_act(x: torch.Tensor, xq: QTensor, xr: QTensor | None, phi: torc
                                            _stream(stream)), "rfq_quantize_act")
 
 
-def rfq_quantize_act_expand(x: torch.Tensor, xq: QTensor, xr: QTensor | None, xq16: QTensor,
-                            xr16: QTensor | None, phi: torch.Tensor | None = None, mode: int = RFQ_FALLBACK_ALL,
+def rfq_quantize_act_expand(x: torch.Tensor, xq: QTensor, xr: QTensor | None, xq_op: QTensor,
+                            xr_op: QTensor | None, phi: torch.Tensor | None = None, mode: int = RFQ_FALLBACK_ALL,
                             tau: float = 0.0, p_s: int = 128, r_s: int = 256, stream=None):
-    """HiF4 activation quantization that also writes the exact bf16 values of
-    X~ (into xq16) and X^ (into xr16) in the same pass."""
+    """Activation quantization that also writes X~ (and X^) in the form the
+    GEMM multiplies, in the same pass: the exact bf16 values for HiF4 (xq_op,
+    xr_op), X~ re-encoded as MXFP8 for an MXFP4 main pathway under an MXFP8
+    residual (xq_op; xr_op None)."""
     M, K = x.shape
     fb = _FB(mode, tau, p_s, r_s)
-    q, q16 = xq.c(), xq16.c()
+    q, qo = xq.c(), xq_op.c()
     r = xr.c() if xr is not None else None
-    r16 = xr16.c() if xr16 is not None else None
+    ro = xr_op.c() if xr_op is not None else None
     _check(load_library().rfq_quantize_act_expand(
         _ptr(x), M, K, ctypes.byref(fb), ctypes.byref(q), ctypes.byref(r) if r is not None else None, _ptr(phi),
-        ctypes.byref(q16), ctypes.byref(r16) if r16 is not None else None, _stream(stream)),
+        ctypes.byref(qo), ctypes.byref(ro) if ro is not None else None, _stream(stream)),
         "rfq_quantize_act_expand")
 
 

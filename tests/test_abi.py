@@ -130,3 +130,25 @@ def test_quantize_act_expand_host_checks(lib):
     assert call(P(16), M, K, None, r(hq), r(hq), None, r(b16_shape), r(b16), None) == rfq.RFQ_ERR_SHAPE
     assert call(P(16), M, K, None, r(hq), r(hq), None, r(b16), r(hq), None) == rfq.RFQ_ERR_INVALID_ARG
     assert call(P(16), M, K, None, r(hq), r(hq), None, r(b16_align), r(b16), None) == rfq.RFQ_ERR_ALIGNMENT
+
+
+def test_quantize_act_expand_fp8_residual_host_checks(lib):
+    """The FP4-to-FP8 form of rfq_quantize_act_expand: X~'s operand is MXFP8
+    in the layout of xq, there is no second operand, and the mode must keep
+    the residual."""
+    from paper_2608_26581_gb300 import rfq
+    P = ctypes.c_void_p
+    M, K = 4, 128
+    x4 = rfq._QT(rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA, M, K, 16, 16)
+    x8 = rfq._QT(rfq.RFQ_FMT_MXFP8, rfq.RFQ_SCALE_MMA, M, K, 16, 16)
+    x8_row = rfq._QT(rfq.RFQ_FMT_MXFP8, rfq.RFQ_SCALE_ROWMAJOR, M, K, 16, 16)
+    b16 = rfq._QT(rfq.RFQ_FMT_BF16, 0, M, K, 16, 0)
+    none = rfq._FB(rfq.RFQ_FALLBACK_NONE, 0.0, 128, 256)
+    r = ctypes.byref
+    call = lib.rfq_quantize_act_expand
+    assert call(P(16), M, K, None, r(x4), r(x8), None, r(x8), r(x8), None) == rfq.RFQ_ERR_INVALID_ARG
+    assert call(P(16), M, K, r(none), r(x4), r(x8), None, r(x8), None, None) == rfq.RFQ_ERR_INVALID_ARG
+    assert call(P(16), M, K, None, r(x4), r(x8), None, r(b16), None, None) == rfq.RFQ_ERR_INVALID_ARG
+    assert call(P(16), M, K, None, r(x4), r(x8), None, r(x8_row), None, None) == rfq.RFQ_ERR_INVALID_ARG
+    # an MXFP4 residual has no operand form to write
+    assert call(P(16), M, K, None, r(x4), r(x4), None, r(x8), r(x8), None) == rfq.RFQ_ERR_UNSUPPORTED

@@ -133,6 +133,40 @@ def test_convert_mxfp4_to_mxfp8_is_exact(orc, layout):
     assert np.array_equal(orc.dequant(orc.FMT_MXFP8, c8, s8, M, K), orc.dequant(orc.FMT_MXFP4, c4, s4, M, K))
 
 
+@pytest.mark.parametrize("layout,mode,tau", [(MMA, rfq.RFQ_FALLBACK_ALL, 0.0), (ROW, rfq.RFQ_FALLBACK_ALL, 0.0),
+                                             (MMA, rfq.RFQ_FALLBACK_AMAX, 30.0)])
+def test_quantize_act_expand_fp8_residual(orc, layout, mode, tau):
+    """The FP4-to-FP8 quantizer writing X~ re-encoded as MXFP8 in the same
+    pass: the E4M3 codes are the oracle's E4M3 encoding of each E2M1 value,
+    the scale bytes those of X~, and X~ and X^ are the oracle's bit for bit.
+    Every finite bf16 pattern (255 rows of 256: M % 128 != 0)."""
+    xb = _all_bf16_patterns()
+    M, K = xb.shape
+    x4 = rfq.empty_qtensor(F4, layout, M, K)
+    xr = rfq.empty_qtensor(F8, layout, M, K)
+    x8 = rfq.empty_qtensor(F8, layout, M, K)
+    _poison(x4, xr, x8)
+    phi = torch.empty(((M + 127) // 128) * (K // 256), dtype=torch.uint8, device=DEV)
+    rfq.rfq_quantize_act_expand(to_dev_bf16(xb), x4, xr, x8, None, phi, mode=mode, tau=tau)
+    torch.cuda.synchronize()
+    ref = orc.quantize_act(xb, orc.FMT_MXFP4, mode, tau, 128, 256, res_fmt=orc.FMT_MXFP8)
+    c4, s4 = qtensor_host(x4)
+    cr, sr = qtensor_host(xr)
+    assert np.array_equal(c4, ref["main_codes"]), _diff(c4, ref["main_codes"])
+    assert np.array_equal(s4, ref["main_scales"]), _diff(s4, ref["main_scales"])
+    assert np.array_equal(cr, ref["res_codes"]), _diff(cr, ref["res_codes"])
+    assert np.array_equal(sr, ref["res_scales"]), _diff(sr, ref["res_scales"])
+    c8, s8 = qtensor_host(x8)
+    assert np.array_equal(s8, s4)
+    e4 = np.array([orc.e4m3_encode(orc.e2m1_decode(c)) for c in range(16)], np.uint8)
+    want = np.stack([e4[c4 & 0xF], e4[c4 >> 4]], axis=2).reshape(M, K)
+    assert np.array_equal(c8, want), _diff(c8, want)
+    if layout == MMA:   # padding rows of the tensor-core scale layout hold zeros
+        from gpu_util import mma_scale_to_rowmajor
+        full = mma_scale_to_rowmajor(x8.scales.cpu().numpy(), -(-M // 128) * 128, K)
+        assert not full[M:].any()
+
+
 def _gemm_case(orc, M, K, N, kind, out=rfq.RFQ_OUT_F32, mode=rfq.RFQ_FALLBACK_ALL, tau=0.0, r_s=256, seed=1,
                rows=None, xb=None, wb=None):
     """kind: 'w8a8', 'w4a8' or 'rfq8' (MXFP4 main + MXFP8 residual)."""
