@@ -574,8 +574,11 @@ def run_rfq(args):
         t_src = (f"{pk['src']} bf16 burst {pk['bf16_burst']} TFLOP/s x {FP4_OVER_BF16:g} "
                  f"(nominal dense FP4/BF16 ratio), of {pk['src']}")
         # more than one 128-row tile runs on CTA pairs (see launch_gemm_mxf4)
+        # CTA pairs beyond one 128-row tile; grouped launches whose groups
+        # average under 2048 stacked rows run 128-row tiles on single CTAs
+        grouped_single = grouped and Mb < 2048 * spec.groups
         t_kernel = "gemm_mxf4_fused_kernel" if fused else (
-            "gemm_mxf4_pair_kernel" if M > 128 or grouped else "gemm_mxf4_kernel")
+            "gemm_mxf4_kernel" if M <= 128 or grouped_single else "gemm_mxf4_pair_kernel")
     if hif4:
         npath = 1 if no_res else 2   # main (and residual) codes + metadata written, and their bf16 values
         aq_bytes = (Mb * K * 2 + npath * (Mb * K // 2) + npath * (((Mb + 127) // 128) * 128 * (K // 64) * 4)

@@ -1,7 +1,8 @@
 // gemm_mxf4.cu -- RFQ GEMM on the sm_103a tensor cores (Algorithm 1,
 // Eq. rfq):  Y = X~ W~ + phi X^ W~.
 //
-// Persistent kernel: one CTA per SM walks output tiles of 128 x 256.  Per
+// Persistent kernel: one CTA per SM walks output tiles of 128 x 256 (of
+// one matrix, or of G row groups each with its own W~: the grouped form).  Per
 // 256-element k-stage the TMA producer stages the main A tile (X~ codes), the
 // residual A tile (X^ codes), the W~ tile (128-byte rows, 128-byte swizzle)
 // and their E8M0 scale atoms (bulk copies) in shared memory, three 68 KB
@@ -65,6 +66,7 @@ constexpr int SF_WARPS = 4;
 constexpr int THREADS = 64 + 32 * EPI_WARPS + 32 * SF_WARPS;
 constexpr int PHI_WARP = THREADS / 32;  // the phi reader: one warp beyond THREADS
 constexpr int REC_WORDS = 64;           // phi record: up to 2048 full k-stages (K <= 524288)
+constexpr int GRP_MAX = 128;            // groups of the grouped GEMM
 static_assert(SF_COL0 + SF_SLOTS * SF_SLOT_COLS <= TMEM_COLS, "TMEM budget");
 static_assert(SF_SLOTS >= STAGES, "a scale slot is rewritten only after its stage's MMAs completed");
 
@@ -104,6 +106,9 @@ struct Smem {
     uint32_t tmem_base;
     int32_t abort_flag;
     int32_t issued;
+    int32_t grp_off[GRP_MAX + 1];     // grouped GEMM: first row of each group (and the end)
+    int32_t grp_tiles[GRP_MAX + 1];   // grouped GEMM: 128-row tiles of the groups before each group
+    int32_t grp_bad;
 };
 
 constexpr size_t kSmemBytes = sizeof(Smem) + 1024;
@@ -124,13 +129,24 @@ struct Mask {
     static constexpr uint32_t value = V;
 };
 
-template <bool RES, bool PHI, bool OUT_BF16>
+// An output tile: its first A row, the end of its rows' group (M without
+// groups), its first W~ row, its first Y column and the end of its group's
+// W~ scale atoms.
+struct TileCoord {
+    int a_row0, row_end, w_row0, col0, wa_end;
+};
+
+// GRP: the grouped (mixture-of-experts) form: G groups of rows with their own
+// W~ (row offsets read on the device), tiles of 128 rows inside each group;
+// the plain form is compiled without any of it.
+template <bool RES, bool PHI, bool OUT_BF16, bool GRP>
 __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     gemm_mxf4_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmR,
                      const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmY,
                      const uint8_t *__restrict__ sfa, const uint8_t *__restrict__ sfr,
                      const uint8_t *__restrict__ sfb, const uint8_t *__restrict__ phi, int phi_chunks,
-                     int phi_cols, int M, int N, int K, int32_t *status)
+                     int phi_cols, int M, int N, int K, int32_t *status, const int32_t *__restrict__ group_off,
+                     int G, void *__restrict__ y)
 {
     extern __shared__ uint8_t smem_raw[];
     Smem &S = *reinterpret_cast<Smem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -150,8 +166,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     const int nf = kc >> 1;                // stages with two chunks
     const int n_tiles = (N + BN - 1) / BN;
     const int m_tiles = (M + BM - 1) / BM;
-    const int tiles = n_tiles * m_tiles;
-    const int n_atoms = (N + 127) >> 7;    // 128-row scale atoms of W~
+    const int n_atoms = (N + 127) >> 7;    // 128-row scale atoms of W~ (one group's with G > 0)
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -181,10 +196,78 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
         tmem_alloc(&S.tmem_base, TMEM_COLS);
         tmem_relinquish();
     }
+    if (GRP && warp == 2) {
+        // Grouped GEMM: rows [group_off[g], group_off[g+1]) of X and Y belong
+        // to group g, whose W~ rows are [g N, (g+1) N).  Every group start
+        // must be a multiple of 128 with the offsets non-decreasing and
+        // group_off[G] <= M; otherwise the kernel records kDevBadGroups and
+        // computes nothing.  The prefix of 128-row tiles maps a tile index
+        // to its group.
+        int bad = 0;
+        for (int e = lane; e <= G; e += 32)
+            S.grp_off[e] = __ldg(group_off + e);
+        __syncwarp();
+        int carry = 0;
+        if (lane == 0)
+            S.grp_tiles[0] = 0;
+        for (int base = 0; base < G; base += 32) {
+            const int e = base + lane;
+            int cnt = 0;
+            if (e < G) {
+                const int a = S.grp_off[e], b = S.grp_off[e + 1];
+                if (a < 0 || (a & (BM - 1)) != 0 || b < a || b > M)
+                    bad = 1;
+                else
+                    cnt = (b - a + BM - 1) / BM;
+            }
+            int v = cnt;
+#pragma unroll
+            for (int d = 1; d < 32; d <<= 1) {
+                const int t = __shfl_up_sync(0xffffffffu, v, d);
+                if (lane >= d)
+                    v += t;
+            }
+            if (e < G)
+                S.grp_tiles[e + 1] = carry + v;
+            carry += __shfl_sync(0xffffffffu, v, 31);
+        }
+        bad = __any_sync(0xffffffffu, bad);
+        if (bad && lane == 0)
+            atomicExch(status, kDevBadGroups);
+        if (lane == 0)
+            S.grp_bad = bad;
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = S.tmem_base;
+    // bad group offsets: no tile (every role skips straight to the teardown)
+    const int tiles = n_tiles * (GRP ? (S.grp_bad ? 0 : S.grp_tiles[G]) : m_tiles);
+    auto coord = [&](int tile) {
+        const int mi = tile / n_tiles, nt = tile - mi * n_tiles;
+        TileCoord c;
+        c.col0 = nt * BN;
+        if (!GRP) {
+            c.a_row0 = mi * BM;
+            c.row_end = M;
+            c.w_row0 = nt * BN;
+            c.wa_end = n_atoms;
+        } else {
+            int lo = 0, hi = G; // grp_tiles[lo] <= mi < grp_tiles[hi]
+            while (hi - lo > 1) {
+                const int mid = (lo + hi) >> 1;
+                if (S.grp_tiles[mid] <= mi)
+                    lo = mid;
+                else
+                    hi = mid;
+            }
+            c.a_row0 = S.grp_off[lo] + (mi - S.grp_tiles[lo]) * BM;
+            c.row_end = S.grp_off[lo + 1];
+            c.w_row0 = lo * N + nt * BN;
+            c.wa_end = (lo + 1) * n_atoms;
+        }
+        return c;
+    };
 
     if (warp == 0) {
         // ------------------------------------------------ TMA producer
@@ -192,9 +275,10 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
             int p = 0, it = 0; // p: stages issued so far (ring position)
             bool stop = false;
             for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x, ++it) {
-                const int m_tile = tile / n_tiles, n_tile = tile - m_tile * n_tiles;
-                const int atom0 = n_tile * 2;
-                const int nb = atom0 + 1 < n_atoms ? 2 : 1;
+                const TileCoord tc = coord(tile);
+                const int m_tile = tc.a_row0 / BM;    // scale atoms and A rows
+                const int atom0 = tc.w_row0 >> 7;
+                const int nb = atom0 + 1 < tc.wa_end ? 2 : 1;
                 // one k-stage: wait for its ring slot, publish the tile's info,
                 // issue the copies
                 auto produce = [&](int ks, int nch, uint32_t info, auto res_t) {
@@ -213,10 +297,10 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                     uint64_t *bar = &S.full[slot];
                     mbar_arrive_expect_tx(bar, A_BYTES + B_BYTES + (1 + nb) * sfbytes +
                                                    (res_on ? A_BYTES + sfbytes : 0));
-                    tma_load_2d(st.a, &tmA, bar, c0 * 64, m_tile * BM);
+                    tma_load_2d(st.a, &tmA, bar, c0 * 64, tc.a_row0);
                     if (res_on)
-                        tma_load_2d(st.r, &tmR, bar, c0 * 64, m_tile * BM);
-                    tma_load_2d(st.b, &tmB, bar, c0 * 64, n_tile * BN);
+                        tma_load_2d(st.r, &tmR, bar, c0 * 64, tc.a_row0);
+                    tma_load_2d(st.b, &tmB, bar, c0 * 64, tc.w_row0);
                     bulk_load(st.sfa, sfa + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, bar);
                     if (res_on)
                         bulk_load(st.sfr, sfr + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, bar);
@@ -351,7 +435,6 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
         const uint32_t sw = (uint32_t)((lane >> 1) & 3);   // 64B swizzle: chunk j of row r at (j ^ ((r >> 1) & 3))
         int it = 0;
         for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++it) {
-            const int m_tile = tile / n_tiles, n_tile = tile - m_tile * n_tiles;
             // warp-uniform outcome: the tcgen05 loads below need the whole warp
             if (!__all_sync(0xffffffffu, mbar_wait(&S.acc_full, it & 1, kWaitLimitNs, gstat))) {
                 if (lane == 0)
@@ -359,7 +442,8 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                 break;
             }
             tc_fence_after();
-            const int row0 = m_tile * BM + q * 32;
+            const TileCoord tc = coord(tile);
+            const int row0 = tc.a_row0 + q * 32;
             const uint32_t tcol = tmem + ((uint32_t)(q * 32) << 16) + h * (BN / 2);
             if (OUT_BF16) {
                 // all 128 columns of this warp into registers as packed bf16,
@@ -386,9 +470,22 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                     mbar_arrive(&S.acc_empty);
 #pragma unroll
                 for (int c = 0; c < 4; ++c) {   // 32-column chunks: one 64-byte TMA box row per lane
-                    const int col = n_tile * BN + h * (BN / 2) + 32 * c;
-                    if (col >= N)
+                    const int col = tc.col0 + h * (BN / 2) + 32 * c;
+                    if (col >= N || row0 >= tc.row_end)
                         break;
+                    if (GRP && row0 + 32 > tc.row_end && tc.row_end < M) {
+                        // a group ends inside this 32-row box: rows past it are
+                        // another group's or padding, so each lane stores its own row
+                        if (row0 + lane < tc.row_end) {
+                            uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(y) +
+                                                                   (int64_t)(row0 + lane) * N + col);
+#pragma unroll
+                            for (int j = 0; j < 4; ++j)
+                                dst[j] = make_uint4(pk[16 * c + 4 * j], pk[16 * c + 4 * j + 1],
+                                                    pk[16 * c + 4 * j + 2], pk[16 * c + 4 * j + 3]);
+                        }
+                        continue;
+                    }
                     if (lane == 0)
                         bulk_wait_group_read<0>();
                     __syncwarp();
@@ -422,13 +519,25 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                     }
 #pragma unroll
                     for (int c = 0; c < 2; ++c) {
-                        const int col = n_tile * BN + h * (BN / 2) + (2 * half + c) * 32;
-                        if (col >= N)
+                        const int col = tc.col0 + h * (BN / 2) + (2 * half + c) * 32;
+                        if (col >= N || row0 >= tc.row_end)
                             continue;
 #pragma unroll
                         for (int hb = 0; hb < 2; ++hb) { // 16 fp32 columns (64 bytes) per store
                             if (col + 16 * hb >= N)
                                 break;
+                            if (GRP && row0 + 32 > tc.row_end && tc.row_end < M) {
+                                // a group ends inside this 32-row box (see the bf16 path)
+                                if (row0 + lane < tc.row_end) {
+                                    uint4 *dst = reinterpret_cast<uint4 *>(static_cast<float *>(y) +
+                                                                           (int64_t)(row0 + lane) * N + col + 16 * hb);
+#pragma unroll
+                                    for (int j = 0; j < 4; ++j)
+                                        dst[j] = make_uint4(v[c][16 * hb + 4 * j], v[c][16 * hb + 4 * j + 1],
+                                                            v[c][16 * hb + 4 * j + 2], v[c][16 * hb + 4 * j + 3]);
+                                }
+                                continue;
+                            }
                             if (lane == 0)
                                 bulk_wait_group_read<0>();
                             __syncwarp();
@@ -461,6 +570,10 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
         int p = 0;
         bool stop = false;
         for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x) {
+            // the tile's second W~ scale atom exists (else zeros: its W~ rows
+            // are past N, or another group's)
+            const TileCoord tc = coord(tile);
+            const bool b1_in = (tc.w_row0 >> 7) + 1 < tc.wa_end;
             // the scale words of the next stage (in the producer's order), with
             // the residual mask rm known at compile time
             auto write_stage = [&](int nch, auto rm_t) {
@@ -482,7 +595,8 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                         break;
                     const uint4 va = *reinterpret_cast<const uint4 *>(st.sfa + c * ATOM + lane * 16);
                     const uint4 vb0 = *reinterpret_cast<const uint4 *>(st.sfb + c * ATOM + lane * 16);
-                    const uint4 vb1 = *reinterpret_cast<const uint4 *>(st.sfb + (2 + c) * ATOM + lane * 16);
+                    const uint4 vb1 = b1_in ? *reinterpret_cast<const uint4 *>(st.sfb + (2 + c) * ATOM + lane * 16)
+                                            : make_uint4(0, 0, 0, 0);
                     tmem_st_32x32b_x4(tb + 4 * c, va.x, va.y, va.z, va.w);
                     if ((rm >> c) & 1) {
                         const uint4 vr = *reinterpret_cast<const uint4 *>(st.sfr + c * ATOM + lane * 16);
@@ -539,7 +653,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                     flag_timeout(S, status);
                 break;
             }
-            const uint8_t *row = phi + (int64_t)(((int)blockIdx.x + j * (int)gridDim.x) / n_tiles) * phi_cols;
+            const uint8_t *row = phi + (int64_t)(coord((int)blockIdx.x + j * (int)gridDim.x).a_row0 / BM) * phi_cols;
             PhiRec &rec = S.rec[r];
             uint32_t n_res = 0;
             for (int w = 0; 32 * w < nf; ++w) {
@@ -574,21 +688,23 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     }
 }
 
-template <bool RES, bool PHI, bool OUT>
+template <bool RES, bool PHI, bool OUT, bool GRP>
 cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const CUtensorMap &tb,
                            const CUtensorMap &ty, const GemmMxf4Args &a, cudaStream_t st)
 {
-    auto kern = gemm_mxf4_kernel<RES, PHI, OUT>;
+    auto kern = gemm_mxf4_kernel<RES, PHI, OUT, GRP>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (e != cudaSuccess)
         return e;
-    const int64_t tiles = ((a.N + BN - 1) / BN) * ((a.M + BM - 1) / BM);
+    // grouped: the tile count depends on the device-side row offsets; every
+    // CTA of the grid walks the tiles that exist
+    const int64_t tiles = GRP ? INT64_MAX : ((a.N + BN - 1) / BN) * ((a.M + BM - 1) / BM);
     const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
     const int phi_chunks = a.phi_r_s / 128;
     const int phi_cols = a.phi ? (int)((a.K + a.phi_r_s - 1) / a.phi_r_s) : 0;
-    kern<<<grid, PHI ? THREADS + 32 : THREADS, kSmemBytes, st>>>(ta, tr, tb, ty, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf,
-                                            (const uint8_t *)a.b_sf, a.phi, phi_chunks, phi_cols, (int)a.M,
-                                            (int)a.N, (int)a.K, a.status);
+    kern<<<grid, PHI ? THREADS + 32 : THREADS, kSmemBytes, st>>>(
+        ta, tr, tb, ty, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf, (const uint8_t *)a.b_sf, a.phi, phi_chunks,
+        phi_cols, (int)a.M, (int)a.N, (int)a.K, a.status, a.group_off, a.groups, a.y);
     return cudaGetLastError();
 }
 
@@ -596,14 +712,23 @@ cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const C
 
 cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st)
 {
-    // more than one 128-row tile: CTA pairs (M = 256 MMAs, half the W~ bytes per SM)
-    if (a.M > BM || a.f8 || a.groups > 0)   // (E4M3 operands and groups run on the pair kernel at every M)
+    // More than one 128-row tile: CTA pairs (M = 256 MMAs, half the W~ bytes
+    // per SM); E4M3 operands run on the pair kernel at every M.  Grouped
+    // MXFP4: 128-row tiles inside each group here while the groups average
+    // fewer than 2048 stacked rows.  A group's 256-row pairs compute 64 rows
+    // past its 128-row tiles on average, which for short groups costs more
+    // than the pair saves (Qwen3-VL-30B experts, ~320 rows each: 0.106 ms
+    // here against 0.112 ms on pairs).
+    const bool grp = a.groups > 0;
+    const bool grp_single = grp && !a.f8 && a.M < (int64_t)2048 * a.groups;
+    if ((a.M > BM && !grp_single) || a.f8 || (grp && !grp_single))
         return launch_gemm_mxf4_pair(a, st);
     CUtensorMap ta, tr, tb;
     const uint64_t kb = (uint64_t)a.K / 2;
+    const uint64_t w_rows = (uint64_t)a.N * (grp ? (uint64_t)a.groups : 1u);
     if (!encode_tmap_2d_u8(&ta, a.a_codes, kb, (uint64_t)a.M, kb, ROW, BM, 128))
         return cudaErrorInvalidValue;
-    if (!encode_tmap_2d_u8(&tb, a.b_codes, kb, (uint64_t)a.N, kb, ROW, BN, 128))
+    if (!encode_tmap_2d_u8(&tb, a.b_codes, kb, w_rows, kb, ROW, BN, 128))
         return cudaErrorInvalidValue;
     if (a.r_codes) {
         if (!encode_tmap_2d_u8(&tr, a.r_codes, kb, (uint64_t)a.M, kb, ROW, BM, 128))
@@ -620,7 +745,8 @@ cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st)
     // residual product is then issued (exact: phi = 0 residuals are zero).
     const bool res = a.r_codes != nullptr;
     const bool phi = res && a.phi != nullptr && a.K / 256 <= REC_WORDS * 32;
-#define RFQ_GV(R, P, O) return launch_variant<R, P, O>(ta, tr, tb, ty, a, st)
+#define RFQ_GV(R, P, O)                                                                                           \
+    return grp ? launch_variant<R, P, O, true>(ta, tr, tb, ty, a, st) : launch_variant<R, P, O, false>(ta, tr, tb, ty, a, st)
     if (!res) {
         if (a.out_bf16) RFQ_GV(false, false, true);
         RFQ_GV(false, false, false);

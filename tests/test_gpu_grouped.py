@@ -110,6 +110,14 @@ def test_grouped_many_groups_many_tiles(orc):
     _case(orc, counts, 256, 768, out=rfq.RFQ_OUT_BF16, seed=7)
 
 
+def test_grouped_long_groups_on_cta_pairs(orc):
+    """Groups averaging 2048 stacked rows or more run on 256-row CTA pairs
+    (shorter ones on 128-row tiles of single CTAs): both forms are checked,
+    with a group ending inside a 32-row output box."""
+    _case(orc, [2100, 2500], 256, 256, seed=13)
+    _case(orc, [2100, 2500], 256, 256, out=rfq.RFQ_OUT_BF16, seed=14)
+
+
 def test_grouped_selective_phi(orc):
     _case(orc, [200, 333, 70], 1152, 256, mode=rfq.RFQ_FALLBACK_AMAX, tau=30.0, r_s=128, seed=9)
 
