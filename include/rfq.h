@@ -239,8 +239,9 @@ RFQ_API rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, co
                                     const rfq_fallback *fb, void *y, int32_t out_dtype, void *workspace,
                                     void *stream);
 
-/* Grouped RFQ GEMM for mixture-of-experts layers (SURVEY: the MoE expert
- * projections of Qwen3-VL, Table 2): every group g (an expert) computes
+/* Grouped RFQ GEMM for mixture-of-experts layers (the MoE expert
+ * projections that hold most of Qwen3-VL-30B's weights, Table 2): every
+ * group g (an expert) computes
  *     Y[rows of g] = X~ W~_g + phi X^ W~_g             (Algorithm 1, Eq. rfq)
  * in one launch over all groups.  xq / xr: the activations of all groups
  * stacked along rows (rfq_qtensor as for rfq_linear, rows = the stacked
