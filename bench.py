@@ -55,7 +55,8 @@ _KERNEL_SRC = {"gemm_mxf4_kernel": "gemm_mxf4.cu", "gemm_mxf4_pair_kernel": "gem
                "act_quant8_kernel": "quant_mxfp8.cu",
                "gemm_mxf4_fused_kernel": "gemm_mxf4_fused.cu",
                "act_quant_mxfp4_kernel": "quant_mxfp4.cu", "act_quant_mxfp4_amax_kernel": "quant_mxfp4.cu",
-               "gemm_hif4_kernel": "gemm_hif4.cu", "act_quant_hif4_kernel": "quant_hif4.cu"}
+               "gemm_hif4_kernel": "gemm_hif4.cu", "act_quant_hif4_kernel": "quant_hif4.cu",
+               "act_quant_hif4_amax_kernel": "quant_hif4.cu"}
 
 
 def _kernel_traffic(kernel: str, workload: str):
@@ -322,7 +323,7 @@ def run_rfq(args):
     if amax_phi and scheme in ("w4a8", "w8a8"):
         raise SystemExit("--phi-tau needs a residual pathway")
     F = rfq.RFQ_FMT_HIF4 if hif4 else rfq.RFQ_FMT_MXFP4
-    amax_fused = amax_phi and not hif4 and not f8 and K % 256 == 0
+    amax_fused = amax_phi and not f8 and K % 256 == 0   # phi computed in the quantizer's pass
     L = rfq.RFQ_SCALE_MMA
 
     xb = make_activation(spec.act)
@@ -583,7 +584,7 @@ def run_rfq(args):
         npath = 1 if no_res else 2   # main (and residual) codes + metadata written, and their bf16 values
         aq_bytes = (Mb * K * 2 + npath * (Mb * K // 2) + npath * (((Mb + 127) // 128) * 128 * (K // 64) * 4)
                     + (0 if quant_only else npath * Mb * K * 2))
-        aq_kernel = "act_quant_hif4_kernel"
+        aq_kernel = "act_quant_hif4_amax_kernel" if amax_fused else "act_quant_hif4_kernel"
     elif f8:
         sfb = ((Mb + 127) // 128) * 128 * K // 32
         # rfq8: X read, X~ codes (E2M1) and scales, X^ (E4M3) and scales, X~ as E4M3 and scales

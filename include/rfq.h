@@ -267,8 +267,9 @@ RFQ_API rfq_status rfq_linear_grouped(const rfq_qtensor *xq, const rfq_qtensor *
 /* Exact re-encoding of an MXFP4 tensor as MXFP8 (every E2M1 value is an
  * E4M3 value): dst codes [rows][k] E4M3 bytes, dst scales = src scales.
  * src: fmt MXFP4; dst: fmt MXFP8, the same rows, k and scale layout; both
- * device, caller-owned.  Used for the weight of the W4A8 baseline and the
- * main activation of the FP4-to-FP8 RFQ.
+ * device, caller-owned.  Used for the weight of the W4A8 baseline and of
+ * the FP4-to-FP8 RFQ (rfq_quantize_act_expand writes the activation's in
+ * the quantizer's own pass).
  * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
  * RFQ_ERR_UNSUPPORTED (other formats), RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */
 RFQ_API rfq_status rfq_convert(const rfq_qtensor *src, rfq_qtensor *dst, void *stream);

@@ -290,22 +290,10 @@ rfq_status quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_fall
         return from_cuda(launch_act_quant_mxfp4(x_bf16, M, K, f.mode, f.tau, f.p_s, f.r_s, xq->codes, xq->scales,
                                                 res ? xr->codes : nullptr, res ? xr->scales : nullptr, phi,
                                                 xq->scale_layout, st));
-    if (xq->fmt == RFQ_FMT_HIF4) {
-        if (f.mode == RFQ_FALLBACK_AMAX) {
-            // the indicator tiles are computed by the MXFP4 path's phi kernel
-            cudaError_t e = launch_phi_amax(x_bf16, M, K, f.p_s, f.r_s, f.tau, phi, st);
-            if (e != cudaSuccess)
-                return RFQ_ERR_CUDA;
-        } else if (phi) {
-            cudaError_t e = launch_phi_fill(phi, (M + f.p_s - 1) / f.p_s * ((K + f.r_s - 1) / f.r_s),
-                                            f.mode == RFQ_FALLBACK_ALL ? 1 : 0, st);
-            if (e != cudaSuccess)
-                return RFQ_ERR_CUDA;
-        }
-        return from_cuda(launch_act_quant_hif4(x_bf16, M, K, f.mode, f.p_s, f.r_s, xq->codes, xq->scales,
+    if (xq->fmt == RFQ_FMT_HIF4)
+        return from_cuda(launch_act_quant_hif4(x_bf16, M, K, f.mode, f.tau, f.p_s, f.r_s, xq->codes, xq->scales,
                                                res ? xr->codes : nullptr, res ? xr->scales : nullptr, phi,
                                                xq->scale_layout, st, m16, r16));
-    }
     return RFQ_ERR_INVALID_ARG;
 }
 } // namespace

@@ -88,9 +88,10 @@ cudaError_t launch_gemm_mxf4_fused(const GemmFusedArgs &a, cudaStream_t st);
 
 // ---- HiF4 quantization (quant_hif4.cu); metadata layout RFQ_SCALE_MMA is
 // block-major [K/64][rows rounded up to 128]
-// m16 / r16 (may be null): bf16 [M][K] receiving the exact values of X~ / X^
-cudaError_t launch_act_quant_hif4(const void *x, int64_t M, int64_t K, int mode, int p_s, int r_s, void *mcodes,
-                                  void *mmeta, void *rcodes, void *rmeta, const uint8_t *phi, int layout,
+// phi: computed (AMAX) or filled (other modes) here when given; m16 / r16
+// (may be null): bf16 [M][K] receiving the exact values of X~ / X^
+cudaError_t launch_act_quant_hif4(const void *x, int64_t M, int64_t K, int mode, float tau, int p_s, int r_s,
+                                  void *mcodes, void *mmeta, void *rcodes, void *rmeta, uint8_t *phi, int layout,
                                   cudaStream_t st, void *m16 = nullptr, void *r16 = nullptr);
 cudaError_t launch_weight_quant_hif4(const void *w, int64_t K, int64_t N, void *codes, void *meta, int layout,
                                      cudaStream_t st);

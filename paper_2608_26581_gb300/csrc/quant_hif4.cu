@@ -154,6 +154,68 @@ __device__ __forceinline__ uint4 bf16x8_pack(const float (&v)[8]) // exact for t
     return make_uint4(p[0], p[1], p[2], p[3]);
 }
 
+// One lane's eight elements xf (group g of its 64-element block; the block's
+// eight lanes take part together) at chunk c of the [M][K / 8] chunk grid:
+// the main codes and metadata, with RES the residual's (zeros when !on),
+// with EXP the exact bf16 values of both.  ok: the chunk is inside the row
+// (uniform over the block's lanes); stores happen only then.
+template <bool RES, bool EXP, int LAYOUT>
+__device__ __forceinline__ void hif4_chunk(const float (&xf)[8], int g, bool ok, bool on, int64_t c, int64_t moff,
+                                           uint32_t *__restrict__ mcodes, uint32_t *__restrict__ mmeta,
+                                           uint32_t *__restrict__ rcodes, uint32_t *__restrict__ rmeta,
+                                           uint4 *__restrict__ m16, uint4 *__restrict__ r16)
+{
+    float am = fmax3(fmax3(fabsf(xf[0]), fabsf(xf[1]), fabsf(xf[2])),
+                     fmax3(fabsf(xf[3]), fabsf(xf[4]), fabsf(xf[5])), fmaxf(fabsf(xf[6]), fabsf(xf[7])));
+#pragma unroll
+    for (int o = 1; o < 8; o <<= 1)
+        am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, o));
+    const int sb = am > 0.f ? hif4_scale_byte(am) : 0;
+    const float S = ue6m2_value(sb >> 2, sb & 3);
+    uint32_t bits;
+    float deq[8];
+    uint32_t code = hif4_group(xf, S, g, bits, deq);
+    if (am == 0.f) {
+        bits = 0;   // all-zero block: metadata 0, codes keep the sign of zero
+    }
+#pragma unroll
+    for (int o = 1; o < 8; o <<= 1)
+        bits |= __shfl_xor_sync(0xFFFFFFFFu, bits, o);
+    if (ok) {
+        mcodes[c] = code;
+        if (g == 0)
+            mmeta[moff] = am == 0.f ? 0u : (bits | (uint32_t)sb);
+        if (EXP)
+            m16[c] = bf16x8_pack(deq);
+    }
+    if (RES) {
+        float r[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            r[i] = xf[i] - deq[i]; // exact
+        float ra = fmax3(fmax3(fabsf(r[0]), fabsf(r[1]), fabsf(r[2])),
+                         fmax3(fabsf(r[3]), fabsf(r[4]), fabsf(r[5])), fmaxf(fabsf(r[6]), fabsf(r[7])));
+#pragma unroll
+        for (int o = 1; o < 8; o <<= 1)
+            ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, o));
+        const int rsb = ra > 0.f ? hif4_scale_byte(ra) : 0;
+        const float RS = ue6m2_value(rsb >> 2, rsb & 3);
+        uint32_t rbits;
+        float rdeq[8];
+        const uint32_t rcode = hif4_group(r, RS, g, rbits, rdeq);
+#pragma unroll
+        for (int o = 1; o < 8; o <<= 1)
+            rbits |= __shfl_xor_sync(0xFFFFFFFFu, rbits, o);
+        if (ok) {
+            rcodes[c] = on ? rcode : 0u;
+            if (g == 0)
+                rmeta[moff] = (on && ra > 0.f) ? (rbits | (uint32_t)rsb) : 0u;
+            if (EXP)
+                r16[c] = on ? bf16x8_pack(rdeq) : make_uint4(0, 0, 0, 0);
+        }
+    }
+}
+
 template <bool RES, bool PHI, int LAYOUT, bool EXP>
 __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__restrict__ x, int64_t M, int64_t K,
                                                             uint32_t *__restrict__ mcodes,
@@ -187,8 +249,6 @@ __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__rest
         for (int j = 0; j < kHU; ++j) {
             const int cr = c0 + j * 32 + lane;             // chunk of 8 elements within the row
             const bool ok = cr < kchunks;                  // uniform over each block's eight lanes
-            const int64_t c = m * kchunks + cr;
-            const int64_t blk = cr >> 3;
             float xf[8];
             const uint32_t w[4] = {vv[j].x, vv[j].y, vv[j].z, vv[j].w};
 #pragma unroll
@@ -196,57 +256,90 @@ __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__rest
                 xf[2 * i] = __uint_as_float(w[i] << 16);
                 xf[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
             }
-            float am = fmax3(fmax3(fabsf(xf[0]), fabsf(xf[1]), fabsf(xf[2])),
-                             fmax3(fabsf(xf[3]), fabsf(xf[4]), fabsf(xf[5])), fmaxf(fabsf(xf[6]), fabsf(xf[7])));
+            const bool on = !PHI || (ok && prow[(cr * 8) / r_s] != 0);
+            hif4_chunk<RES, EXP, LAYOUT>(xf, g, ok, on, m * kchunks + cr, meta_index<LAYOUT>(m, cr >> 3, M, kblocks),
+                                         mcodes, mmeta, rcodes, rmeta, m16, r16);
+        }
+    }
+}
+
+// AMAX fallback (Sec. 4.3) for phi tiles of 128 rows x 256 columns, fused
+// into the quantizer (as act_quant_mxfp4_amax_kernel): one 512-thread block
+// per tile keeps its 64 KB in registers (warp w rows 8w .. 8w + 7, lane l
+// the l-th 16-byte chunk of each; lanes 8b .. 8b + 7 hold 64-element block
+// b), reduces max |x| (packed bf16x2 max, NaN dropped, as phi_amax_kernel),
+// writes phi, then quantizes; the residual of a phi = 0 tile is written as
+// zeros without being computed.  X is read once.
+constexpr int kHAmaxRows = 8;
+
+template <int LAYOUT, bool EXP>
+__global__ void __launch_bounds__(512, 1) act_quant_hif4_amax_kernel(const uint4 *__restrict__ x, int64_t M,
+                                                                    int64_t K, uint32_t *__restrict__ mcodes,
+                                                                    uint32_t *__restrict__ mmeta,
+                                                                    uint32_t *__restrict__ rcodes,
+                                                                    uint32_t *__restrict__ rmeta,
+                                                                    uint8_t *__restrict__ phi, float tau,
+                                                                    uint4 *__restrict__ m16, uint4 *__restrict__ r16)
+{
+    constexpr int R = kHAmaxRows, NW = 16;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t kchunks = K >> 3;
+    const int64_t kblocks = K >> 6;
+    const int nr = (int)(K >> 8);
+    const int64_t tile = blockIdx.x;
+    const int64_t p = tile / nr;
+    const int r = (int)(tile - p * nr);
+    const int64_t m0 = p * 128 + warp * R;
+    const int cr = r * 32 + lane;
+    uint4 v[R];
 #pragma unroll
-            for (int o = 1; o < 8; o <<= 1)
-                am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, o));
-            const int sb = am > 0.f ? hif4_scale_byte(am) : 0;
-            const float S = ue6m2_value(sb >> 2, sb & 3);
-            uint32_t bits;
-            float deq[8];
-            uint32_t code = hif4_group(xf, S, g, bits, deq);
-            if (am == 0.f) {
-                bits = 0;   // all-zero block: metadata 0, codes keep the sign of zero
-            }
+    for (int i = 0; i < R; ++i)
+        v[i] = m0 + i < M ? __ldcs(x + (m0 + i) * kchunks + cr) : make_uint4(0, 0, 0, 0);
+    uint32_t acc = 0;
 #pragma unroll
-            for (int o = 1; o < 8; o <<= 1)
-                bits |= __shfl_xor_sync(0xFFFFFFFFu, bits, o);
-            if (ok) {
-                mcodes[c] = code;
-                if (g == 0)
-                    mmeta[meta_index<LAYOUT>(m, blk, M, kblocks)] = am == 0.f ? 0u : (bits | (uint32_t)sb);
-                if (EXP)
-                    m16[c] = bf16x8_pack(deq);
-            }
-            if (RES) {
-                const bool on = !PHI || (ok && prow[(cr * 8) / r_s] != 0);
-                float r[8];
+    for (int i = 0; i < R; ++i) {
+        const uint32_t q[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
 #pragma unroll
-                for (int i = 0; i < 8; ++i)
-                    r[i] = xf[i] - deq[i]; // exact
-                float ra = fmax3(fmax3(fabsf(r[0]), fabsf(r[1]), fabsf(r[2])),
-                                 fmax3(fabsf(r[3]), fabsf(r[4]), fabsf(r[5])), fmaxf(fabsf(r[6]), fabsf(r[7])));
+        for (int j = 0; j < 4; ++j)
+            asm("max.bf16x2 %0, %1, %2;" : "=r"(acc) : "r"(acc), "r"(q[j] & 0x7fff7fffu));
+    }
+    const float am = fmaxf(__uint_as_float(acc << 16), __uint_as_float(acc & 0xffff0000u));
+    __shared__ uint32_t red[NW];
+    const uint32_t wmax = __reduce_max_sync(0xFFFFFFFFu, __float_as_uint(am)); // am >= 0: integer order
+    if (lane == 0)
+        red[warp] = wmax;
+    __syncthreads();
+    uint32_t tmax = red[0];
 #pragma unroll
-                for (int o = 1; o < 8; o <<= 1)
-                    ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, o));
-                const int rsb = ra > 0.f ? hif4_scale_byte(ra) : 0;
-                const float RS = ue6m2_value(rsb >> 2, rsb & 3);
-                uint32_t rbits;
-                float rdeq[8];
-                const uint32_t rcode = hif4_group(r, RS, g, rbits, rdeq);
+    for (int i = 1; i < NW; ++i)
+        tmax = max(tmax, red[i]);
+    const bool on = __uint_as_float(tmax) > tau;
+    if (threadIdx.x == 0)
+        phi[tile] = on ? 1 : 0;
+    const int g = lane & 7;
 #pragma unroll
-                for (int o = 1; o < 8; o <<= 1)
-                    rbits |= __shfl_xor_sync(0xFFFFFFFFu, rbits, o);
-                if (ok) {
-                    rcodes[c] = on ? rcode : 0u;
-                    if (g == 0)
-                        rmeta[meta_index<LAYOUT>(m, blk, M, kblocks)] =
-                            (on && ra > 0.f) ? (rbits | (uint32_t)rsb) : 0u;
-                    if (EXP)
-                        r16[c] = on ? bf16x8_pack(rdeq) : make_uint4(0, 0, 0, 0);
-                }
-            }
+    for (int i = 0; i < R; ++i) {
+        const int64_t m = m0 + i; // uniform over the warp
+        if (m >= M)
+            break;
+        float xf[8];
+        const uint32_t w[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            xf[2 * k] = __uint_as_float(w[k] << 16);
+            xf[2 * k + 1] = __uint_as_float(w[k] & 0xFFFF0000u);
+        }
+        const int64_t c = m * kchunks + cr;
+        const int64_t moff = meta_index<LAYOUT>(m, cr >> 3, M, kblocks);
+        if (on) {
+            hif4_chunk<true, EXP, LAYOUT>(xf, g, true, true, c, moff, mcodes, mmeta, rcodes, rmeta, m16, r16);
+        } else {
+            hif4_chunk<false, EXP, LAYOUT>(xf, g, true, true, c, moff, mcodes, mmeta, rcodes, rmeta, m16, r16);
+            rcodes[c] = 0u;
+            if (g == 0)
+                rmeta[moff] = 0u;
+            if (EXP)
+                r16[c] = make_uint4(0, 0, 0, 0);
         }
     }
 }
@@ -332,10 +425,42 @@ int grid_for(int64_t work, int threads, int max_blocks)
 
 } // namespace
 
-cudaError_t launch_act_quant_hif4(const void *x, int64_t M, int64_t K, int mode, int p_s, int r_s, void *mcodes,
-                                  void *mmeta, void *rcodes, void *rmeta, const uint8_t *phi, int layout,
+cudaError_t launch_act_quant_hif4(const void *x, int64_t M, int64_t K, int mode, float tau, int p_s, int r_s,
+                                  void *mcodes, void *mmeta, void *rcodes, void *rmeta, uint8_t *phi, int layout,
                                   cudaStream_t st, void *m16, void *r16)
 {
+    const int64_t np = (M + p_s - 1) / p_s, nr = (K + r_s - 1) / r_s;
+    if (mode == RFQ_FALLBACK_AMAX && p_s == 128 && r_s == 256 && K % 256 == 0) {
+        // the GEMMs' phi granularity: phi computed in the quantizer's pass
+        auto *xi = static_cast<const uint4 *>(x);
+        auto *mc = static_cast<uint32_t *>(mcodes);
+        auto *mm = static_cast<uint32_t *>(mmeta);
+        auto *rc = static_cast<uint32_t *>(rcodes);
+        auto *rm = static_cast<uint32_t *>(rmeta);
+        auto *e0 = static_cast<uint4 *>(m16);
+        auto *e1 = static_cast<uint4 *>(r16);
+        const unsigned tiles = (unsigned)(np * nr);
+#define RFQ_HA(LAY, EXP) \
+    act_quant_hif4_amax_kernel<LAY, EXP><<<tiles, 512, 0, st>>>(xi, M, K, mc, mm, rc, rm, phi, tau, e0, e1)
+        if (layout == RFQ_SCALE_MMA) {
+            if (e0) RFQ_HA(RFQ_SCALE_MMA, true);
+            else RFQ_HA(RFQ_SCALE_MMA, false);
+        } else {
+            if (e0) RFQ_HA(RFQ_SCALE_ROWMAJOR, true);
+            else RFQ_HA(RFQ_SCALE_ROWMAJOR, false);
+        }
+#undef RFQ_HA
+        return cudaGetLastError();
+    }
+    if (mode == RFQ_FALLBACK_AMAX) {
+        cudaError_t e = launch_phi_amax(x, M, K, p_s, r_s, tau, phi, st);
+        if (e != cudaSuccess)
+            return e;
+    } else if (phi) {
+        cudaError_t e = launch_phi_fill(phi, np * nr, mode == RFQ_FALLBACK_ALL ? 1 : 0, st);
+        if (e != cudaSuccess)
+            return e;
+    }
     const int64_t items = M * ((K / 8 + kHSeg / 8 - 1) / (kHSeg / 8));
     const int blocks = grid_for(items * 32, 256, 152 * 24);
     auto *xi = static_cast<const uint4 *>(x);

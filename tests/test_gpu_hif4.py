@@ -95,10 +95,25 @@ def test_degenerate_blocks(orc):
 
 
 @pytest.mark.parametrize("mode,tau,r_s", [(rfq.RFQ_FALLBACK_NONE, 0.0, 256), (rfq.RFQ_FALLBACK_AMAX, 20.0, 128),
-                                          (rfq.RFQ_FALLBACK_AMAX, 10.0, 64)])
+                                          (rfq.RFQ_FALLBACK_AMAX, 10.0, 64), (rfq.RFQ_FALLBACK_AMAX, 20.0, 256)])
 def test_phi_modes(orc, mode, tau, r_s):
+    """AMAX on 128 x 256 tiles runs the fused kernel (phi computed in the
+    quantizer's pass); other tile widths the separate phi pass."""
     xb = make_activation(ActSpec(300, 1024, "laplace", body_scale=0.3, chan_count=5, chan_scale=50.0, seed=3))
     _compare(orc, xb, rfq.RFQ_SCALE_MMA, mode=mode, tau=tau, r_s=r_s)
+
+
+@pytest.mark.parametrize("layout", [rfq.RFQ_SCALE_MMA, rfq.RFQ_SCALE_ROWMAJOR])
+@pytest.mark.parametrize("M,K", [(1, 256), (200, 768)])
+def test_phi_amax_fused_tiles(orc, layout, M, K):
+    """The fused AMAX quantizer on ragged rows, tau set to tile (0, 0)'s own
+    max |x| (phi is strict: that tile keeps no residual)."""
+    xb = make_activation(ActSpec(M, K, "laplace", body_scale=0.3, chan_count=4, chan_scale=50.0, seed=M + K))
+    x = (xb.astype(np.uint32) << 16).view(np.float32)
+    tau = float(np.abs(x[:128, :256]).max())
+    _compare(orc, xb, layout, mode=rfq.RFQ_FALLBACK_AMAX, tau=tau, r_s=256)
+    _, _, phi = _quant(xb, layout, rfq.RFQ_FALLBACK_AMAX, tau, 128, 256)
+    assert phi[0].item() == 0
 
 
 @pytest.mark.parametrize("K,N", [(64, 16), (640, 272), (12288, 64)])
@@ -130,7 +145,8 @@ def test_dequant_fp32_and_bf16_exact(orc):
 
 @pytest.mark.parametrize("mode,tau,r_s,layout", [
     (rfq.RFQ_FALLBACK_ALL, 0.0, 256, rfq.RFQ_SCALE_MMA), (rfq.RFQ_FALLBACK_ALL, 0.0, 256, rfq.RFQ_SCALE_ROWMAJOR),
-    (rfq.RFQ_FALLBACK_NONE, 0.0, 256, rfq.RFQ_SCALE_MMA), (rfq.RFQ_FALLBACK_AMAX, 10.0, 128, rfq.RFQ_SCALE_MMA)])
+    (rfq.RFQ_FALLBACK_NONE, 0.0, 256, rfq.RFQ_SCALE_MMA), (rfq.RFQ_FALLBACK_AMAX, 10.0, 128, rfq.RFQ_SCALE_MMA),
+    (rfq.RFQ_FALLBACK_AMAX, 10.0, 256, rfq.RFQ_SCALE_MMA), (rfq.RFQ_FALLBACK_AMAX, 10.0, 256, rfq.RFQ_SCALE_ROWMAJOR)])
 def test_quantize_act_expand(orc, mode, tau, r_s, layout):
     """The quantizer's own bf16 values of X~ and X^ are bit for bit the
     oracle's dequantization of its codes (Sec. 3.3 decoder), with X^ zero on
@@ -214,6 +230,8 @@ def test_linear_no_residual_and_phi(orc, expand):
     xq, xr, wq, y = _linear(xb, wb, mode=rfq.RFQ_FALLBACK_NONE, expand=expand)
     check_y(y, _ref(orc, xq, None, wq, M, K, N))
     xq, xr, wq, y = _linear(xb, wb, mode=rfq.RFQ_FALLBACK_AMAX, tau=10.0, r_s=128, use_phi=True, expand=expand)
+    check_y(y, _ref(orc, xq, xr, wq, M, K, N))
+    xq, xr, wq, y = _linear(xb, wb, mode=rfq.RFQ_FALLBACK_AMAX, tau=10.0, r_s=256, use_phi=True, expand=expand)
     check_y(y, _ref(orc, xq, xr, wq, M, K, N))
 
 
