@@ -52,7 +52,7 @@ def _peaks():
 # source file of each timed kernel: its DRAM counters hold only for the
 # sources they were taken on (the kernel's file plus the shared headers)
 _KERNEL_SRC = {"gemm_mxf4_kernel": "gemm_mxf4.cu", "gemm_mxf4_pair_kernel": "gemm_mxf4_pair.cu",
-               "act_quant8_kernel": "quant_mxfp8.cu",
+               "act_quant8_kernel": "quant_mxfp8.cu", "act_quant_rfq8_amax_kernel": "quant_mxfp8.cu",
                "gemm_mxf4_fused_kernel": "gemm_mxf4_fused.cu",
                "act_quant_mxfp4_kernel": "quant_mxfp4.cu", "act_quant_mxfp4_amax_kernel": "quant_mxfp4.cu",
                "gemm_hif4_kernel": "gemm_hif4.cu", "act_quant_hif4_kernel": "quant_hif4.cu",
@@ -87,7 +87,8 @@ def _src_hash(kernel: str):
     d = os.path.join(HERE, "paper_2608_26581_gb300", "csrc")
     m = hashlib.sha256()
     extra = ("mxfp4_math.cuh",) if kernel in ("act_quant_mxfp4_kernel", "act_quant_mxfp4_amax_kernel",
-                                              "gemm_mxf4_fused_kernel", "act_quant8_kernel") else ()
+                                              "gemm_mxf4_fused_kernel", "act_quant8_kernel",
+                                              "act_quant_rfq8_amax_kernel") else ()
     for n in (_KERNEL_SRC[kernel], "ptx.cuh", "internal.h") + extra:
         m.update(open(os.path.join(d, n), "rb").read())
     return m.hexdigest()[:16]
@@ -323,7 +324,7 @@ def run_rfq(args):
     if amax_phi and scheme in ("w4a8", "w8a8"):
         raise SystemExit("--phi-tau needs a residual pathway")
     F = rfq.RFQ_FMT_HIF4 if hif4 else rfq.RFQ_FMT_MXFP4
-    amax_fused = amax_phi and not f8 and K % 256 == 0   # phi computed in the quantizer's pass
+    amax_fused = amax_phi and K % 256 == 0   # phi computed in the quantizer's pass
     L = rfq.RFQ_SCALE_MMA
 
     xb = make_activation(spec.act)
@@ -590,7 +591,7 @@ def run_rfq(args):
         # rfq8: X read, X~ codes (E2M1) and scales, X^ (E4M3) and scales, X~ as E4M3 and scales
         aq_bytes = (Mb * K * 2 + Mb * K // 2 + Mb * K + 2 * sfb + Mb * K + sfb if scheme == "rfq8"
                     else Mb * K * 2 + Mb * K + sfb)
-        aq_kernel = "act_quant8_kernel"
+        aq_kernel = "act_quant_rfq8_amax_kernel" if amax_fused else "act_quant8_kernel"
     else:
         npath = 1 if no_res else 2
         aq_bytes = Mb * K * 2 + npath * (Mb * K // 2) + npath * (((Mb + 127) // 128) * 128 * K // 32)

@@ -173,6 +173,101 @@ __global__ void __launch_bounds__(256) act_quant8_kernel(const uint4 *__restrict
     }
 }
 
+// The FP4-to-FP8 quantizer with AMAX phi on 128 x 256 tiles (Sec. 4.3),
+// fused as act_quant_mxfp4_amax_kernel: one 512-thread block per tile keeps
+// its 64 KB in registers (warp w rows 8w .. 8w + 7, lane l the l-th 16-byte
+// chunk of each), reduces max |x| (packed bf16x2 max, NaN dropped, as
+// phi_amax_kernel), writes phi, then writes X~ (MXFP4; with OP also as
+// MXFP8) and, on a phi = 1 tile, the MXFP8 residual (zeros otherwise,
+// without computing it).  X is read once.
+template <int LAYOUT, bool OP>
+__global__ void __launch_bounds__(512, 1) act_quant_rfq8_amax_kernel(const uint4 *__restrict__ x, int64_t M,
+                                                                    int64_t K, uint8_t *__restrict__ mcodes,
+                                                                    uint8_t *__restrict__ mscales,
+                                                                    uint8_t *__restrict__ rcodes,
+                                                                    uint8_t *__restrict__ rscales,
+                                                                    uint8_t *__restrict__ phi, float tau,
+                                                                    uint8_t *__restrict__ m8codes,
+                                                                    uint8_t *__restrict__ m8scales)
+{
+    constexpr int R = 8, NW = 16;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t kchunks = K >> 3;
+    const int kblocks = (int)(K >> 5);
+    const int nr = (int)(K >> 8);
+    const int64_t tile = blockIdx.x;
+    const int64_t p = tile / nr;
+    const int r = (int)(tile - p * nr);
+    const int64_t m0 = p * 128 + warp * R;
+    const int c = r * 32 + lane;
+    uint4 v[R];
+#pragma unroll
+    for (int i = 0; i < R; ++i)
+        v[i] = m0 + i < M ? __ldcs(x + (m0 + i) * kchunks + c) : make_uint4(0, 0, 0, 0);
+    uint32_t acc = 0;
+#pragma unroll
+    for (int i = 0; i < R; ++i) {
+        const uint32_t q[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            asm("max.bf16x2 %0, %1, %2;" : "=r"(acc) : "r"(acc), "r"(q[j] & 0x7fff7fffu));
+    }
+    const float am = fmaxf(__uint_as_float(acc << 16), __uint_as_float(acc & 0xffff0000u));
+    __shared__ uint32_t red[NW];
+    const uint32_t wmax = __reduce_max_sync(0xFFFFFFFFu, __float_as_uint(am)); // am >= 0: integer order
+    if (lane == 0)
+        red[warp] = wmax;
+    __syncthreads();
+    uint32_t tmax = red[0];
+#pragma unroll
+    for (int i = 1; i < NW; ++i)
+        tmax = max(tmax, red[i]);
+    const bool on = __uint_as_float(tmax) > tau;
+    if (threadIdx.x == 0)
+        phi[tile] = on ? 1 : 0;
+#pragma unroll
+    for (int i = 0; i < R; ++i) {
+        const int64_t m = m0 + i; // uniform over the warp
+        const int64_t soff = scale_index8<LAYOUT>(m, c >> 2, kblocks);
+        if (m >= M) {
+            if (LAYOUT == RFQ_SCALE_MMA && (lane & 3) == 0) {
+                // rows M .. of the last tile are the layout's padding rows
+                mscales[soff] = 0;
+                rscales[soff] = 0;
+                if (OP)
+                    m8scales[soff] = 0;
+            }
+            continue;
+        }
+        float xf[8];
+        bf16x8_to_f32(v[i], xf);
+        const Mx8 q4 = mxfp4_quant8<false>(xf);
+        float q[8];
+        e2m1x8_decode(q4.code, q);
+        reinterpret_cast<uint32_t *>(mcodes + m * (K >> 1))[c] = q4.code;
+        if (OP)
+            *reinterpret_cast<uint2 *>(m8codes + m * K + (int64_t)c * 8) = e4m3x8(q);
+        uint2 rq = make_uint2(0, 0);
+        int rb = 0;
+        if (on) {
+            // the residual x - x~, exact in fp32
+            const float sc = pow2_e(q4.sb);
+            float rr[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+                rr[k] = fmaf(-q[k], sc, xf[k]);
+            rq = mxfp8_quant8(rr, rb);
+        }
+        *reinterpret_cast<uint2 *>(rcodes + m * K + (int64_t)c * 8) = rq;
+        if ((lane & 3) == 0) {
+            mscales[soff] = (uint8_t)q4.sb;
+            rscales[soff] = (uint8_t)rb;
+            if (OP)
+                m8scales[soff] = (uint8_t)q4.sb;
+        }
+    }
+}
+
 // One thread per (column n, 32-block b) of W [K x N].
 template <int LAYOUT>
 __global__ void __launch_bounds__(256) weight_quant_mxfp8_kernel(const __nv_bfloat16 *__restrict__ w, int64_t K,
@@ -307,6 +402,28 @@ cudaError_t launch_act_quant_rfq8(const void *x, int64_t M, int64_t K, int mode,
                                   void *mcodes, void *mscales, void *rcodes, void *rscales, uint8_t *phi, int layout,
                                   cudaStream_t st, void *m8codes, void *m8scales)
 {
+    if (mode == RFQ_FALLBACK_AMAX && p_s == 128 && r_s == 256 && K % 256 == 0) {
+        // the GEMMs' phi granularity: phi computed in the quantizer's pass
+        const unsigned tiles = (unsigned)(((M + 127) / 128) * (K / 256));
+        auto *xi = static_cast<const uint4 *>(x);
+        auto *mc = static_cast<uint8_t *>(mcodes);
+        auto *ms = static_cast<uint8_t *>(mscales);
+        auto *rc = static_cast<uint8_t *>(rcodes);
+        auto *rs = static_cast<uint8_t *>(rscales);
+        auto *oc = static_cast<uint8_t *>(m8codes);
+        auto *os = static_cast<uint8_t *>(m8scales);
+#define RFQ_A8(LAY, OP) \
+    act_quant_rfq8_amax_kernel<LAY, OP><<<tiles, 512, 0, st>>>(xi, M, K, mc, ms, rc, rs, phi, tau, oc, os)
+        if (layout == RFQ_SCALE_MMA) {
+            if (oc) RFQ_A8(RFQ_SCALE_MMA, true);
+            else RFQ_A8(RFQ_SCALE_MMA, false);
+        } else {
+            if (oc) RFQ_A8(RFQ_SCALE_ROWMAJOR, true);
+            else RFQ_A8(RFQ_SCALE_ROWMAJOR, false);
+        }
+#undef RFQ_A8
+        return cudaGetLastError();
+    }
     if (mode == RFQ_FALLBACK_AMAX) {
         cudaError_t e = launch_phi_amax(x, M, K, p_s, r_s, tau, phi, st);
         if (e != cudaSuccess)

@@ -77,9 +77,11 @@ def test_act_quant_mxfp8_bit_exact(orc, layout, src):
 
 
 @pytest.mark.parametrize("layout", [ROW, MMA])
-@pytest.mark.parametrize("mode,tau,r_s", [(rfq.RFQ_FALLBACK_ALL, 0.0, 256), (rfq.RFQ_FALLBACK_AMAX, 30.0, 128)])
+@pytest.mark.parametrize("mode,tau,r_s", [(rfq.RFQ_FALLBACK_ALL, 0.0, 256), (rfq.RFQ_FALLBACK_AMAX, 30.0, 128),
+                                          (rfq.RFQ_FALLBACK_AMAX, 30.0, 256)])
 def test_act_quant_fp8_residual_bit_exact(orc, layout, mode, tau, r_s):
-    """X~ = Q_MXFP4(X) and X^ = Q_MXFP8(X - X~) in one pass (with phi)."""
+    """X~ = Q_MXFP4(X) and X^ = Q_MXFP8(X - X~) in one pass (with phi; on
+    128 x 256 tiles phi is computed in the same pass)."""
     for xb in (_all_bf16_patterns(), make_activation(ActSpec(300, 1024, "normal", chan_count=3, chan_scale=64.0,
                                                              tok_count=2, tok_scale=200.0, seed=7))):
         M, K = xb.shape
