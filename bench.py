@@ -227,36 +227,113 @@ def _oracle_weight(spec):
     return _ORACLE_W[spec.name]
 
 
-def cpu_oracle_sample(spec, rows_per_call: int = 8, calls: int = 4):
-    """Times the CPU oracle (single thread, fp64) on a bounded sample of the
-    workload `spec`: `calls` x (quantize + RFQ GEMM of `rows_per_call` token
-    rows against the full quantized weight), or quantization alone for the
-    quantizer-only workload.  Returns (value, unit, seconds, sample) in the
-    bench's own metric: TFLOP/s of the main + residual product, or GB/s of
-    the quantizer's algorithmic bytes."""
-    import oracle
+def _oracle_rows(spec, rows: int, part: int = 0):
+    """Synthetic token rows for the CPU oracle sample (the workload's
+    distribution; `part` selects a distinct seeded draw per worker)."""
     from paper_2608_26581_gb300.synth import ActSpec, make_activation
-    K, N, a = spec.act.K, spec.N, spec.act
+    a = spec.act
+    return make_activation(ActSpec(rows, a.K, a.body, a.body_scale, a.chan_frac, a.chan_count,
+                                   a.chan_scale, 0.0, None, 1.0, a.seed + 1000 * part))
+
+
+def _oracle_run(spec, xb, rows_per_call: int, calls: int, wq):
+    """The timed oracle work: `calls` x (quantize + RFQ GEMM of
+    `rows_per_call` rows against the full quantized weight), or quantization
+    alone for the quantizer-only workload."""
+    import oracle
     fmt = oracle.FMT_HIF4 if spec.fmt == "hif4" else oracle.FMT_MXFP4
-    rows = rows_per_call * calls
-    xb = make_activation(ActSpec(rows, K, a.body, a.body_scale, a.chan_frac, a.chan_count,
-                                 a.chan_scale, 0.0, None, 1.0, a.seed))
-    wq = _oracle_weight(spec) if N else None
-    t0 = time.perf_counter()
+    K, N = spec.act.K, spec.N
     for i in range(calls):
         x = xb[i * rows_per_call:(i + 1) * rows_per_call]
         q = oracle.quantize_act(x, fmt)
         if N:
             oracle.linear(fmt, q["main_codes"], q["main_scales"], q["res_codes"], q["res_scales"], wq[0], wq[1],
                           rows_per_call, K, N)
-    dt = time.perf_counter() - t0
-    if N:
-        sample = (f"{calls} x (quantize_act + RFQ linear) of {rows_per_call} rows of X [.., {K}] "
-                  f"against the full W~ [{N} x {K}] (weight quantization untimed)")
-        return 2.0 * 2.0 * rows * N * K / dt / 1e12, UNIT, dt, sample
-    per_elem = 3.125 if fmt == oracle.FMT_HIF4 else 3.0625
-    sample = f"{calls} x quantize_act (main + residual) of {rows_per_call} rows of X [.., {K}]"
-    return rows * K * per_elem / dt / 1e9, "GB/s", dt, sample
+
+
+def _oracle_units(spec, rows: int):
+    """(work, unit, divisor) of `rows` oracle rows in the bench's metric:
+    TFLOP of the main + residual product, or GB of the quantizer's bytes."""
+    if spec.N:
+        return 2.0 * 2.0 * rows * spec.N * spec.act.K, UNIT, 1e12
+    per_elem = 3.125 if spec.fmt == "hif4" else 3.0625
+    return rows * spec.act.K * per_elem, "GB/s", 1e9
+
+
+def _oracle_sample_desc(spec, rows_per_call: int, calls: int, workers: int):
+    K, N = spec.act.K, spec.N
+    per = (f"{calls} x (quantize_act + RFQ linear) of {rows_per_call} rows of X [.., {K}] against the full "
+           f"W~ [{N} x {K}] (weight quantization untimed)" if N else
+           f"{calls} x quantize_act (main + residual) of {rows_per_call} rows of X [.., {K}]")
+    return (f"{workers} processes on {workers} host cores, each: {per}; wall time from a common start"
+            if workers > 1 else per)
+
+
+def _oracle_workers(spec) -> int:
+    """Processes for the CPU baseline: one per host core while the free
+    memory holds each one's copy of the quantized weight and the oracle's
+    fp64 expansion of it (plus headroom)."""
+    n = os.cpu_count() or 1
+    need = (spec.N * spec.act.K * 12 + (1 << 30)) if spec.N else (1 << 30)
+    try:
+        with open("/proc/meminfo") as f:
+            avail = next(int(l.split()[1]) * 1024 for l in f if l.startswith("MemAvailable:"))
+        n = min(n, max(1, avail // 2 // need))
+    except (OSError, StopIteration, ValueError):
+        n = 1
+    return int(max(1, n))
+
+
+def _oracle_proc(key, rows_per_call, calls, reps, part, barrier, q):
+    """One worker of the multi-core CPU baseline: its own rows, the same
+    bounded sample as the others, every repetition started together at a
+    barrier (spawned process: no CUDA in it)."""
+    try:
+        spec = _workload(0, key)
+        wq = _oracle_weight(spec) if spec.N else None
+        xb = _oracle_rows(spec, rows_per_call * calls, part)
+        for r in range(reps):
+            barrier.wait(timeout=1800)
+            t0 = time.monotonic()
+            _oracle_run(spec, xb, rows_per_call, calls, wq)
+            q.put((r, t0, time.monotonic()))
+    except Exception as e:  # reported to the parent, which raises
+        q.put(("error", repr(e), 0.0))
+
+
+def cpu_oracle_timed(key: str, rows_per_call: int, calls: int, reps: int):
+    """Times the CPU oracle (fp64, as it stands) on a bounded sample of the
+    workload `key` (of synth.WORKLOADS) on the host cores: one spawned process per core (as memory
+    allows), each running `calls` x `rows_per_call` rows, `reps` times, all
+    starting together.  Returns (workers, unit, sample, [(value, seconds)]
+    per repetition), the value being the whole sample's work over the
+    repetition's wall time in the bench's metric."""
+    import multiprocessing
+    spec = _workload(0, key)
+    n = _oracle_workers(spec)
+    ctx = multiprocessing.get_context("spawn")
+    barrier, q = ctx.Barrier(n), ctx.Queue()
+    procs = [ctx.Process(target=_oracle_proc, args=(key, rows_per_call, calls, reps, i, barrier, q),
+                         daemon=True) for i in range(n)]
+    for p_ in procs:
+        p_.start()
+    got = []
+    try:
+        for _ in range(n * reps):
+            r = q.get(timeout=3600)
+            if r[0] == "error":
+                raise RuntimeError(f"CPU oracle worker failed: {r[1]}")
+            got.append(r)
+    finally:
+        for p_ in procs:
+            p_.join(timeout=60)
+    work, unit, div = _oracle_units(spec, n * rows_per_call * calls)
+    out = []
+    for rep in range(reps):
+        t = [(t0, t1) for r_, t0, t1 in got if r_ == rep]
+        wall = max(b for _, b in t) - min(a for a, _ in t)
+        out.append((work / wall / div, wall))
+    return n, unit, _oracle_sample_desc(spec, rows_per_call, calls, n), out
 
 
 def run_reference(args):
@@ -264,21 +341,15 @@ def run_reference(args):
     if rank != 0:
         return
     spec = _workload(0, args.workload)
-    rows = 2 if spec.N else 64
-    for _ in range(args.warmup):
-        cpu_oracle_sample(spec, rows_per_call=rows, calls=1)
-    vals, times = [], []
-    sample, unit = "", UNIT
-    for _ in range(args.steps):
-        v, unit, dt, sample = cpu_oracle_sample(spec, rows_per_call=rows, calls=1)
-        vals.append(v)
-        times.append(dt)
-    value = statistics.median(vals)
+    rows = 8 if spec.N else 64   # 8 rows share each call's fp64 expansion of W~
+    n, unit, sample, reps = cpu_oracle_timed(args.workload, rows, 1, args.warmup + args.steps)
+    timed = reps[args.warmup:]
+    value = statistics.median(v for v, _ in timed)
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": unit, "n_gpus": ws,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * statistics.median(times),
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * statistics.median(t for _, t in timed),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "config": _config(spec, {"sample": sample}),
-            "cpu_baseline": {"kind": "oracle", "cores": 1, "sample": sample, "value": value, "unit": unit},
+            "cpu_baseline": {"kind": "oracle", "cores": n, "sample": sample, "value": value, "unit": unit},
             "e2e": {"value": value, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
             "gpu_launches": 0}
     print(json.dumps(line), flush=True)
@@ -629,8 +700,9 @@ def run_rfq(args):
     if rank == 0:
         cpu = None
         if ws == 1 and not args.no_cpu_baseline and not args.rows:
-            v, u, dt, sample = cpu_oracle_sample(spec)
-            cpu = {"value": v, "unit": u, "cores": 1, "kind": "oracle", "sample": sample,
+            n, u, sample, reps = cpu_oracle_timed(args.workload, 8, 4, 1)
+            v, dt = reps[0]
+            cpu = {"value": v, "unit": u, "cores": n, "kind": "oracle", "sample": sample,
                    "seconds": round(dt, 2)}
         line = {
             "metric": METRIC, "value": value, "unit": unit, "n_gpus": ws, "steps": args.steps,
