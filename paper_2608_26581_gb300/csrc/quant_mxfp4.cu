@@ -160,25 +160,39 @@ __global__ void __launch_bounds__(256) phi_amax_kernel(const __nv_bfloat16 *__re
 }
 
 // AMAX fallback (Sec. 4.3) for phi tiles of 128 rows x 256 columns, fused
-// into the quantizer: one block per tile keeps the tile's 64 KB in registers
-// (warp w holds rows 16w .. 16w + 15, lane l the l-th 16-byte chunk of each),
-// reduces max |x| over it (NaN dropped, as by phi_amax_kernel), writes phi,
-// then quantizes the tile.  A phi = 0
-// tile's residual is written as zero codes and zero scales without being
-// computed.  X is read from DRAM once, against twice for phi_amax_kernel
-// followed by act_quant_mxfp4_kernel.  (Measured slower: splitting a tile
-// over a cluster of 2 or 4 blocks that exchange their maxima through
-// distributed shared memory; a persistent 512-thread form streaming the
-// tiles through a cp.async ring.)
+// into the quantizer: one block per tile stages the tile's 64 KB in shared
+// memory with cp.async (warp w holds rows 16w .. 16w + 15, lane l the l-th
+// 16-byte chunk of each; three blocks per SM), reduces max |x| over it (NaN
+// dropped, as by phi_amax_kernel), writes phi, then quantizes the tile.  A
+// phi = 0 tile's residual is written as zero codes and zero scales without
+// being computed.  X is read from DRAM once, against twice for
+// phi_amax_kernel followed by act_quant_mxfp4_kernel.  (Measured slower:
+// the tile held in registers, two blocks per SM; splitting a tile over a
+// cluster of 2 or 4 blocks that exchange their maxima through distributed
+// shared memory; a persistent 512-thread form streaming the tiles through a
+// cp.async ring.)
 constexpr int kAmaxRows = 16; // rows per warp (8 warps = 128 rows)
 
+__device__ __forceinline__ void cp_async16_zfill(uint32_t saddr, const void *g, uint32_t src_bytes)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(saddr), "l"(g), "r"(src_bytes) : "memory");
+}
+
+__device__ __forceinline__ uint4 lds128(uint32_t saddr)
+{
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"(saddr)
+                 : "memory");
+    return v;
+}
+
 template <int LAYOUT>
-__global__ void __launch_bounds__(256, 2) act_quant_mxfp4_amax_kernel(const uint4 *__restrict__ x, int64_t M,
-                                                                     int64_t K, uint32_t *__restrict__ mcodes,
-                                                                     uint8_t *__restrict__ mscales,
-                                                                     uint32_t *__restrict__ rcodes,
-                                                                     uint8_t *__restrict__ rscales,
-                                                                     uint8_t *__restrict__ phi, float tau)
+__global__ void __launch_bounds__(256, 3)
+    act_quant_mxfp4_amax_kernel(const uint4 *__restrict__ x, int64_t M, int64_t K, uint32_t *__restrict__ mcodes,
+                                uint8_t *__restrict__ mscales, uint32_t *__restrict__ rcodes,
+                                uint8_t *__restrict__ rscales, uint8_t *__restrict__ phi, float tau)
 {
     constexpr int R = kAmaxRows;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -190,17 +204,24 @@ __global__ void __launch_bounds__(256, 2) act_quant_mxfp4_amax_kernel(const uint
     const int r = (int)(tile - p * nr);
     const int64_t m0 = p * 128 + warp * R;
     const int c = r * 32 + lane;
-    uint4 v[R];
+    extern __shared__ __align__(16) uint8_t tile_smem[];
+    // this thread's row i sits at sbase + 512 i; no other thread reads it
+    const uint32_t sbase = (uint32_t)__cvta_generic_to_shared(tile_smem) + (uint32_t)(((warp * R) * 32 + lane) * 16);
 #pragma unroll
-    for (int i = 0; i < R; ++i)
-        v[i] = m0 + i < M ? __ldcs(x + (m0 + i) * kchunks + c) : make_uint4(0, 0, 0, 0);
+    for (int i = 0; i < R; ++i) {
+        const bool ok = m0 + i < M; // rows past M are zero-filled, not read
+        cp_async16_zfill(sbase + 512 * i, ok ? x + (m0 + i) * kchunks + c : x, ok ? 16u : 0u);
+    }
+    asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+    auto row = [&](int i) { return lds128(sbase + 512 * i); };
     // max |x| as two packed bf16 magnitudes: sign bits cleared, then the
     // bf16x2 max, which returns the other operand where one is NaN (NaN
     // dropped, as in phi_amax_kernel); starts at +0
     uint32_t acc = 0;
 #pragma unroll
     for (int i = 0; i < R; ++i) {
-        const uint32_t q[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+        const uint4 vi = row(i);
+        const uint32_t q[4] = {vi.x, vi.y, vi.z, vi.w};
 #pragma unroll
         for (int j = 0; j < 4; ++j)
             asm("max.bf16x2 %0, %1, %2;" : "=r"(acc) : "r"(acc), "r"(q[j] & 0x7fff7fffu));
@@ -226,7 +247,7 @@ __global__ void __launch_bounds__(256, 2) act_quant_mxfp4_amax_kernel(const uint
         const int64_t soff = scale_index<LAYOUT>(m, b, kblocks);
         if (m < M) {
             float xf[8];
-            bf16x8_to_f32(v[i], xf);
+            bf16x8_to_f32(row(i), xf);
             if (on) {
                 const Mx8 qz = mxfp4_quant8<true>(xf);
                 mcodes[m * kchunks + c] = qz.code;
@@ -399,10 +420,13 @@ cudaError_t launch_act_quant_mxfp4(const void *x, int64_t M, int64_t K, int mode
         auto *ms = static_cast<uint8_t *>(mscales);
         auto *rc = static_cast<uint32_t *>(rcodes);
         auto *rs = static_cast<uint8_t *>(rscales);
-        if (layout == RFQ_SCALE_MMA)
-            act_quant_mxfp4_amax_kernel<RFQ_SCALE_MMA><<<tiles, 256, 0, st>>>(xi, M, K, mc, ms, rc, rs, phi, tau);
-        else
-            act_quant_mxfp4_amax_kernel<RFQ_SCALE_ROWMAJOR><<<tiles, 256, 0, st>>>(xi, M, K, mc, ms, rc, rs, phi, tau);
+        constexpr int smem = 128 * 256 * 2;   // the tile, staged in shared memory
+        auto k = layout == RFQ_SCALE_MMA ? act_quant_mxfp4_amax_kernel<RFQ_SCALE_MMA>
+                                         : act_quant_mxfp4_amax_kernel<RFQ_SCALE_ROWMAJOR>;
+        cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (e != cudaSuccess)
+            return e;
+        k<<<tiles, 256, smem, st>>>(xi, M, K, mc, ms, rc, rs, phi, tau);
         return cudaGetLastError();
     }
     if (mode == RFQ_FALLBACK_AMAX) {

@@ -174,14 +174,29 @@ __global__ void __launch_bounds__(256) act_quant8_kernel(const uint4 *__restrict
 }
 
 // The FP4-to-FP8 quantizer with AMAX phi on 128 x 256 tiles (Sec. 4.3),
-// fused as act_quant_mxfp4_amax_kernel: one 512-thread block per tile keeps
-// its 64 KB in registers (warp w rows 8w .. 8w + 7, lane l the l-th 16-byte
-// chunk of each), reduces max |x| (packed bf16x2 max, NaN dropped, as
-// phi_amax_kernel), writes phi, then writes X~ (MXFP4; with OP also as
-// MXFP8) and, on a phi = 1 tile, the MXFP8 residual (zeros otherwise,
-// without computing it).  X is read once.
+// fused as act_quant_mxfp4_amax_kernel: one 256-thread block per tile
+// stages its 64 KB in shared memory with cp.async (warp w rows 16w .. 16w +
+// 15, lane l the l-th 16-byte chunk of each), reduces max |x| (packed
+// bf16x2 max, NaN dropped, as phi_amax_kernel), writes phi, then writes X~
+// (MXFP4; with OP also as MXFP8) and, on a phi = 1 tile, the MXFP8
+// residual (zeros otherwise, without computing it).  X is read once.
+__device__ __forceinline__ void cp_async16_zfill(uint32_t saddr, const void *g, uint32_t src_bytes)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(saddr), "l"(g), "r"(src_bytes) : "memory");
+}
+
+__device__ __forceinline__ uint4 lds128(uint32_t saddr)
+{
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"(saddr)
+                 : "memory");
+    return v;
+}
+
 template <int LAYOUT, bool OP>
-__global__ void __launch_bounds__(512, 1) act_quant_rfq8_amax_kernel(const uint4 *__restrict__ x, int64_t M,
+__global__ void __launch_bounds__(256, 3) act_quant_rfq8_amax_kernel(const uint4 *__restrict__ x, int64_t M,
                                                                     int64_t K, uint8_t *__restrict__ mcodes,
                                                                     uint8_t *__restrict__ mscales,
                                                                     uint8_t *__restrict__ rcodes,
@@ -190,7 +205,7 @@ __global__ void __launch_bounds__(512, 1) act_quant_rfq8_amax_kernel(const uint4
                                                                     uint8_t *__restrict__ m8codes,
                                                                     uint8_t *__restrict__ m8scales)
 {
-    constexpr int R = 8, NW = 16;
+    constexpr int R = 16, NW = 8;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t kchunks = K >> 3;
     const int kblocks = (int)(K >> 5);
@@ -200,14 +215,20 @@ __global__ void __launch_bounds__(512, 1) act_quant_rfq8_amax_kernel(const uint4
     const int r = (int)(tile - p * nr);
     const int64_t m0 = p * 128 + warp * R;
     const int c = r * 32 + lane;
-    uint4 v[R];
+    extern __shared__ __align__(16) uint8_t tile_smem[];
+    // this thread's row i sits at sbase + 512 i; no other thread reads it
+    const uint32_t sbase = (uint32_t)__cvta_generic_to_shared(tile_smem) + (uint32_t)(((warp * R) * 32 + lane) * 16);
 #pragma unroll
-    for (int i = 0; i < R; ++i)
-        v[i] = m0 + i < M ? __ldcs(x + (m0 + i) * kchunks + c) : make_uint4(0, 0, 0, 0);
+    for (int i = 0; i < R; ++i) {
+        const bool ok = m0 + i < M; // rows past M are zero-filled, not read
+        cp_async16_zfill(sbase + 512 * i, ok ? x + (m0 + i) * kchunks + c : x, ok ? 16u : 0u);
+    }
+    asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
     uint32_t acc = 0;
 #pragma unroll
     for (int i = 0; i < R; ++i) {
-        const uint32_t q[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+        const uint4 vi = lds128(sbase + 512 * i);
+        const uint32_t q[4] = {vi.x, vi.y, vi.z, vi.w};
 #pragma unroll
         for (int j = 0; j < 4; ++j)
             asm("max.bf16x2 %0, %1, %2;" : "=r"(acc) : "r"(acc), "r"(q[j] & 0x7fff7fffu));
@@ -240,7 +261,7 @@ __global__ void __launch_bounds__(512, 1) act_quant_rfq8_amax_kernel(const uint4
             continue;
         }
         float xf[8];
-        bf16x8_to_f32(v[i], xf);
+        bf16x8_to_f32(lds128(sbase + 512 * i), xf);
         const Mx8 q4 = mxfp4_quant8<false>(xf);
         float q[8];
         e2m1x8_decode(q4.code, q);
@@ -412,16 +433,15 @@ cudaError_t launch_act_quant_rfq8(const void *x, int64_t M, int64_t K, int mode,
         auto *rs = static_cast<uint8_t *>(rscales);
         auto *oc = static_cast<uint8_t *>(m8codes);
         auto *os = static_cast<uint8_t *>(m8scales);
-#define RFQ_A8(LAY, OP) \
-    act_quant_rfq8_amax_kernel<LAY, OP><<<tiles, 512, 0, st>>>(xi, M, K, mc, ms, rc, rs, phi, tau, oc, os)
-        if (layout == RFQ_SCALE_MMA) {
-            if (oc) RFQ_A8(RFQ_SCALE_MMA, true);
-            else RFQ_A8(RFQ_SCALE_MMA, false);
-        } else {
-            if (oc) RFQ_A8(RFQ_SCALE_ROWMAJOR, true);
-            else RFQ_A8(RFQ_SCALE_ROWMAJOR, false);
-        }
-#undef RFQ_A8
+        constexpr int smem = 128 * 256 * 2;   // the tile, staged in shared memory
+        auto k = layout == RFQ_SCALE_MMA ? (oc ? act_quant_rfq8_amax_kernel<RFQ_SCALE_MMA, true>
+                                               : act_quant_rfq8_amax_kernel<RFQ_SCALE_MMA, false>)
+                                         : (oc ? act_quant_rfq8_amax_kernel<RFQ_SCALE_ROWMAJOR, true>
+                                               : act_quant_rfq8_amax_kernel<RFQ_SCALE_ROWMAJOR, false>);
+        cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (e != cudaSuccess)
+            return e;
+        k<<<tiles, 256, smem, st>>>(xi, M, K, mc, ms, rc, rs, phi, tau, oc, os);
         return cudaGetLastError();
     }
     if (mode == RFQ_FALLBACK_AMAX) {
