@@ -273,7 +273,7 @@ def _oracle_workers(spec) -> int:
     """Processes for the CPU baseline: one per host core while the free
     memory holds each one's copy of the quantized weight and the oracle's
     fp64 expansion of it (plus headroom)."""
-    n = os.cpu_count() or 1
+    n = min(os.cpu_count() or 1, 64)
     need = (spec.N * spec.act.K * 12 + (1 << 30)) if spec.N else (1 << 30)
     try:
         with open("/proc/meminfo") as f:
@@ -301,16 +301,17 @@ def _oracle_proc(key, rows_per_call, calls, reps, part, barrier, q):
         q.put(("error", repr(e), 0.0))
 
 
-def cpu_oracle_timed(key: str, rows_per_call: int, calls: int, reps: int):
+def cpu_oracle_timed(key: str, rows_per_call: int, calls: int, reps: int, workers: int = 0):
     """Times the CPU oracle (fp64, as it stands) on a bounded sample of the
-    workload `key` (of synth.WORKLOADS) on the host cores: one spawned process per core (as memory
-    allows), each running `calls` x `rows_per_call` rows, `reps` times, all
-    starting together.  Returns (workers, unit, sample, [(value, seconds)]
-    per repetition), the value being the whole sample's work over the
+    workload `key` (of synth.WORKLOADS) on the host cores: one spawned
+    process per core (up to 64, as memory allows; or `workers`), each
+    running `calls` x `rows_per_call` rows, `reps` times, all starting
+    together.  Returns (workers, unit, sample, [(value, seconds)] per
+    repetition), the value being the whole sample's work over the
     repetition's wall time in the bench's metric."""
     import multiprocessing
     spec = _workload(0, key)
-    n = _oracle_workers(spec)
+    n = workers if workers > 0 else _oracle_workers(spec)
     ctx = multiprocessing.get_context("spawn")
     barrier, q = ctx.Barrier(n), ctx.Queue()
     procs = [ctx.Process(target=_oracle_proc, args=(key, rows_per_call, calls, reps, i, barrier, q),

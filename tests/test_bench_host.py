@@ -64,7 +64,9 @@ def test_oracle_units():
 def test_oracle_timed_on_host_cores():
     """Spawned oracle processes on the tiny workload: one timing per
     repetition, a positive rate, the worker count in the sample text."""
-    n, unit, sample, reps = bench.cpu_oracle_timed("tiny", 2, 1, 2)
-    assert n >= 1 and unit == bench.UNIT and len(reps) == 2
+    n, unit, sample, reps = bench.cpu_oracle_timed("tiny", 2, 1, 2, workers=2)
+    assert n == 2 and unit == bench.UNIT and len(reps) == 2
     assert all(v > 0 and dt > 0 for v, dt in reps)
-    assert (f"{n} processes" in sample) == (n > 1)
+    assert "2 processes on 2 host cores" in sample
+    n, _, sample, reps = bench.cpu_oracle_timed("act_quant", 64, 1, 1, workers=1)
+    assert n == 1 and reps[0][0] > 0 and "processes" not in sample
