@@ -74,6 +74,28 @@ def _kernel_traffic(kernel: str, workload: str):
     return None
 
 
+def _act_quant_bytes(rows: int, K: int, kind: str, residual: bool, operand: bool = False) -> int:
+    """Algorithmic DRAM bytes of one activation-quantizer launch: X (bf16)
+    read once and every output written once.  kind: "mxfp4" (E2M1 codes,
+    E8M0 scales per 32, scale rows padded to 128), "hif4" (codes, a 32-bit
+    metadata word per 64, rows padded to 128; operand: the bf16 values of X~
+    and X^ too), "rfq8" (MXFP4 X~ and an MXFP8 residual; operand: X~ as
+    E4M3 with its scales too), "mxfp8" (E4M3 codes and scales)."""
+    rows_pad = (rows + 127) // 128 * 128
+    x = rows * K * 2
+    sf = rows_pad * (K // 32)
+    paths = 2 if residual else 1
+    if kind == "mxfp4":
+        return x + paths * (rows * K // 2 + sf)
+    if kind == "hif4":
+        return x + paths * (rows * K // 2 + rows_pad * (K // 64) * 4) + (paths * rows * K * 2 if operand else 0)
+    if kind == "rfq8":
+        return x + (rows * K // 2 + sf) + (rows * K + sf) + ((rows * K + sf) if operand else 0)
+    if kind == "mxfp8":
+        return x + rows * K + sf
+    raise ValueError(kind)
+
+
 def _launches_per_step(quant_only, fused, hif4, no_res, scheme, amax_phi, amax_fused=False):
     """This library's kernel launches in one timed step."""
     if quant_only or fused:
@@ -647,26 +669,20 @@ def run_rfq(args):
         t_peak, t_peak_sust = pk["bf16_burst"] * FP4_OVER_BF16, pk["bf16_sust"] * FP4_OVER_BF16
         t_src = (f"{pk['src']} bf16 burst {pk['bf16_burst']} TFLOP/s x {FP4_OVER_BF16:g} "
                  f"(nominal dense FP4/BF16 ratio), of {pk['src']}")
-        # more than one 128-row tile runs on CTA pairs (see launch_gemm_mxf4)
         # CTA pairs beyond one 128-row tile; grouped launches whose groups
         # average under 2048 stacked rows run 128-row tiles on single CTAs
         grouped_single = grouped and Mb < 2048 * spec.groups
         t_kernel = "gemm_mxf4_fused_kernel" if fused else (
             "gemm_mxf4_kernel" if M <= 128 or grouped_single else "gemm_mxf4_pair_kernel")
     if hif4:
-        npath = 1 if no_res else 2   # main (and residual) codes + metadata written, and their bf16 values
-        aq_bytes = (Mb * K * 2 + npath * (Mb * K // 2) + npath * (((Mb + 127) // 128) * 128 * (K // 64) * 4)
-                    + (0 if quant_only else npath * Mb * K * 2))
+        aq_bytes = _act_quant_bytes(Mb, K, "hif4", not no_res, operand=not quant_only)
         aq_kernel = "act_quant_hif4_amax_kernel" if amax_fused else "act_quant_hif4_kernel"
     elif f8:
-        sfb = ((Mb + 127) // 128) * 128 * K // 32
-        # rfq8: X read, X~ codes (E2M1) and scales, X^ (E4M3) and scales, X~ as E4M3 and scales
-        aq_bytes = (Mb * K * 2 + Mb * K // 2 + Mb * K + 2 * sfb + Mb * K + sfb if scheme == "rfq8"
-                    else Mb * K * 2 + Mb * K + sfb)
+        aq_bytes = _act_quant_bytes(Mb, K, "rfq8" if scheme == "rfq8" else "mxfp8", scheme == "rfq8",
+                                    operand=scheme == "rfq8")
         aq_kernel = "act_quant_rfq8_amax_kernel" if amax_fused else "act_quant8_kernel"
     else:
-        npath = 1 if no_res else 2
-        aq_bytes = Mb * K * 2 + npath * (Mb * K // 2) + npath * (((Mb + 127) // 128) * 128 * K // 32)
+        aq_bytes = _act_quant_bytes(Mb, K, "mxfp4", not no_res)
         # AMAX phi on 128 x 256 tiles: phi and the quantization in one kernel
         aq_kernel = "act_quant_mxfp4_amax_kernel" if amax_fused else "act_quant_mxfp4_kernel"
     if fused:

@@ -70,3 +70,20 @@ def test_oracle_timed_on_host_cores():
     assert "2 processes on 2 host cores" in sample
     n, _, sample, reps = bench.cpu_oracle_timed("act_quant", 64, 1, 1, workers=1)
     assert n == 1 and reps[0][0] > 0 and "processes" not in sample
+
+
+def test_act_quant_algorithmic_bytes():
+    """The per-launch byte counts the roofline divides by (X read once,
+    every output written once)."""
+    B = bench._act_quant_bytes
+    # Wan FFN, MXFP4 main + residual: 3.0625 B per element + the 128-row scale padding
+    assert B(32760, 5120, "mxfp4", True) == 32760 * 5120 * 2 + 2 * (32760 * 5120 // 2 + 32768 * 160)
+    assert B(32760, 5120, "mxfp4", True) == 513_679_360
+    assert B(16384, 4096, "mxfp4", True) == 205_520_896          # the act-quant workload
+    assert B(16384, 4096, "mxfp4", False) == 16384 * 4096 * 2 + 16384 * 4096 // 2 + 16384 * 128
+    # HiF4 (Qwen down): codes, metadata and the bf16 values of X~ and X^
+    hif4 = B(4096, 12288, "hif4", True, operand=True)
+    assert hif4 == 4096 * 12288 * (2 + 2 * 0.5 + 2 * 2) + 2 * 4096 * 192 * 4
+    # FP4-to-FP8 residual with X~ as E4M3: 2 + 0.5 + 1 + 1 bytes per element + three scale planes
+    assert B(32760, 5120, "rfq8", True, operand=True) == 32760 * 5120 * 9 // 2 + 3 * 32768 * 160
+    assert B(4096, 4096, "mxfp8", False) == 4096 * 4096 * 3 + 4096 * 128
