@@ -691,7 +691,8 @@ def run_rfq(args):
         aq_gbs = aq_bytes / (q_ms * 1e-3) / 1e9
         act_quant = {"bound": "hbm", "kernel": aq_kernel, "achieved": aq_gbs, "peak": pk["hbm"], "unit": "GB/s",
                      "frac": aq_gbs / pk["hbm"], "bytes_per_launch": aq_bytes, "ms_per_launch": q_ms,
-                     "traffic": _kernel_traffic(aq_kernel, spec.name)}
+                     "traffic": _kernel_traffic(aq_kernel, spec.name + ("+" + scheme if f8 else "")
+                                                + ("+w4a4" if no_res and not f8 else ""))}
     if quant_only:
         value = _job_rate(aq_bytes, ws, ms) / 1e9
         unit = "GB/s"
@@ -703,7 +704,8 @@ def run_rfq(args):
         roofline = {"bound": "tensor", "kernel": t_kernel, "achieved": gemm_tflops, "peak": t_peak,
                     "unit": "TFLOP/s", "frac": gemm_tflops / t_peak,
                     "traffic": _kernel_traffic(t_kernel, spec.name + ("+" + scheme if f8 else "")
-                                               + ("+phi" if amax_phi else "")),
+                                               + ("+phi" if amax_phi else "")
+                                               + ("+w4a4" if no_res and not f8 else "")),
                     "flop_per_launch": flop, "ms_per_launch": g_ms,
                     "peak_source": t_src, "frac_of_sustained_peak": gemm_tflops / t_peak_sust}
     clocks = clk.summary(h0, h1)
