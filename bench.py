@@ -146,7 +146,7 @@ class ClockSampler:
             self.proc.terminate()
             self.proc.wait()
 
-    def summary(self, t0=None, t1=None):
+    def summary(self, t0=None, t1=None, label="timed and warm-up replays"):
         """Median SM clock, max clock and the throttle reasons of the samples
         taken in [t0, t1] (host seconds, time.time()); all samples when no
         window is given or none falls inside it."""
@@ -170,7 +170,7 @@ class ClockSampler:
         use = inside or rows
         reasons = sorted({n for r in use for n, v in zip(names, r[3]) if v.lower().startswith("active")})
         return {"sm_mhz": statistics.median(r[1] for r in use), "sm_max_mhz": max(r[2] for r in use),
-                "samples": len(use), "window": "timed and warm-up replays" if inside else "whole run",
+                "samples": len(use), "window": label if inside else "whole run",
                 "reasons": reasons}
 
 
@@ -584,6 +584,16 @@ def run_rfq(args):
         torch.cuda.synchronize()
         h1 = time.time()
         barrier()
+        # the dense FP4 tensor rate with MMAs alone (both MMA forms), timed
+        # right after the step under the same sampler
+        mma_peak = None
+        if not args.no_mma_peak and ws == 1 and not (quant_only or hif4 or f8):
+            h2 = time.time()
+            mma_peak = _fp4_mma_peak(rfq, wsp, stream, ev)
+            mma_peak["clocks"] = clk.summary(h2, time.time(), "the MMA-only launches")
+            if mma_peak["clocks"]:
+                mma_peak["flop_per_sm_clock"] = (mma_peak["tflops"] * 1e12 / mma_peak["sms"]
+                                                 / (mma_peak["clocks"]["sm_mhz"] * 1e6))
     ms = t_start.elapsed_time(t_end) / args.steps
     q_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in per_step)
     g_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in per_step)
@@ -708,6 +718,10 @@ def run_rfq(args):
                                                + ("+w4a4" if no_res and not f8 else "")),
                     "flop_per_launch": flop, "ms_per_launch": g_ms,
                     "peak_source": t_src, "frac_of_sustained_peak": gemm_tflops / t_peak_sust}
+        if mma_peak is not None and not (hif4 or f8):
+            # against this GPU's measured MMA-only FP4 rate (the nominal 6x ratio is not reached)
+            roofline["measured_fp4_mma_tflops"] = mma_peak["tflops"]
+            roofline["frac_of_measured_fp4_mma"] = gemm_tflops / mma_peak["tflops"]
     clocks = clk.summary(h0, h1)
     if e2e_ms is not None:
         e2e = {"value": _job_rate(aq_bytes / 1e9 if quant_only else flop / 1e12, ws, e2e_ms), "unit": unit,
@@ -758,9 +772,76 @@ def run_rfq(args):
         }
         if not quant_only:
             line["effective_tflops_2mnk"] = _job_rate(flop / 2, ws, ms) / 1e12
+        if mma_peak is not None:
+            line["fp4_mma_peak"] = mma_peak
+        if ws == 1 and not args.no_extras and not args.rows:
+            line["other_configs"] = _other_configs(args)
         print(json.dumps(line), flush=True)
     if ws > 1:
         dist.destroy_process_group()
+
+
+def _fp4_mma_peak(rfq, wsp, stream, ev, iters: int = 16384, reps: int = 5):
+    """MMA-only FP4 rate (rfq_fp4_mma_peak): per form, 3 untimed launches,
+    then `reps` launches each timed with CUDA events on the launching stream;
+    TFLOP/s of the mean launch.  `tflops` is the faster form's, and
+    flop_per_sm_clock divides it by the SM count and the median SM clock the
+    sampler saw (filled in by the caller's clock summary when available)."""
+    import torch
+    out = {"iters_per_launch": iters, "launches": reps}
+    best = 0.0
+    for name, pair in (("cta1", False), ("cta_pair", True)):
+        for _ in range(3):
+            rfq.rfq_fp4_mma_peak(pair, iters, wsp)
+        ms = []
+        for _ in range(reps):
+            a, b = ev(), ev()
+            a.record(stream)
+            flop = rfq.rfq_fp4_mma_peak(pair, iters, wsp)
+            b.record(stream)
+            b.synchronize()
+            ms.append(a.elapsed_time(b))
+        t = flop / (statistics.mean(ms) * 1e-3) / 1e12
+        out[f"tflops_{name}"] = t
+        out[f"ms_per_launch_{name}"] = statistics.mean(ms)
+        best = max(best, t)
+    if rfq.rfq_workspace_status(wsp) != rfq.RFQ_OK:
+        raise RuntimeError("rfq_fp4_mma_peak reported a device timeout")
+    out["tflops"] = best
+    out["sms"] = torch.cuda.get_device_properties(0).multi_processor_count
+    return out
+
+
+# The other workloads of the benchmark's configuration list, each timed by a
+# child run of this script (its own process, inputs, CUDA graph and clock
+# samples) after the headline one: the standalone activation quantizer
+# (16384 x 4096, Student-t), the Qwen3-VL-8B gate/up and HiF4 down
+# projections, and the Wan2.2 FFN up projection on the fused-prologue variant.
+_EXTRAS = (("act_quant_16384x4096", ["--workload", "act_quant"]),
+           ("qwen3vl8b_gate_up", ["--workload", "qwen_gate_up"]),
+           ("qwen3vl8b_down_hif4", ["--workload", "qwen_down_hif4"]),
+           ("wan22_ffn_up_fused", ["--workload", "wan_ffn_up", "--variant", "fused"]))
+
+
+def _other_configs(args):
+    out = {}
+    for name, extra in _EXTRAS:
+        cmd = [sys.executable, os.path.abspath(__file__), "--steps", str(args.steps), "--warmup", str(args.warmup),
+               "--no-cpu-baseline", "--no-e2e", "--no-extras", "--no-mma-peak", *extra]
+        try:
+            r = subprocess.run(cmd, capture_output=True, text=True, timeout=600)
+            line = json.loads([ln for ln in r.stdout.splitlines() if ln.startswith("{")][-1])
+        except (subprocess.TimeoutExpired, IndexError, ValueError) as e:
+            out[name] = {"error": f"{type(e).__name__}: {str(e)[:200]}"}
+            continue
+        rl = line.get("roofline") or {}
+        out[name] = {"value": line["value"], "unit": line["unit"], "ms_per_step": line["ms_per_step"],
+                     "kernel": rl.get("kernel"), "kernel_ms_per_launch": rl.get("ms_per_launch"),
+                     "kernel_frac": rl.get("frac"), "peak": rl.get("peak"), "peak_unit": rl.get("unit"),
+                     "act_quant_frac": (line.get("act_quant") or {}).get("frac"),
+                     "variant": line["config"].get("variant"), "workload": line["config"]["workload"],
+                     "clocks": line.get("clocks")}
+    return out
 
 
 def main():
@@ -783,6 +864,10 @@ def main():
                     help="fused: rfq_linear_fused, the activation quantizer inside the GEMM")
     ap.add_argument("--workload", default=WORKLOAD,
                     choices=["wan_ffn_up", "qwen_gate_up", "qwen_down_hif4", "act_quant", "tiny", "qwen_moe_gate_up"])
+    ap.add_argument("--no-extras", action="store_true",
+                    help="skip the child runs that time the other workloads of the configuration list")
+    ap.add_argument("--no-mma-peak", action="store_true",
+                    help="skip the MMA-only FP4 rate measurement")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

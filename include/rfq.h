@@ -185,7 +185,15 @@ RFQ_API rfq_status rfq_quantize_act_expand(const void *x_bf16, int64_t M, int64_
                                            rfq_qtensor *xq, rfq_qtensor *xr, uint8_t *phi, rfq_qtensor *xq_op,
                                            rfq_qtensor *xr_op, void *stream);
 
-/* Bytes of device workspace rfq_linear needs (a status word, padded). */
+/* Bytes of device workspace rfq_linear needs (a status word, padded).  The
+ * caller zeroes it.  Its int32 words: [0] the device status that
+ * rfq_workspace_status reads; [1] the limit of the call's bounded waits in
+ * microseconds (0: two seconds); [2] held start: when non-zero, the GEMM's
+ * copy producers wait (within that limit) for word [3] to become non-zero
+ * before their first copy and record RFQ_ERR_TIMEOUT if it stays zero -- a
+ * way to run a kernel's timeout path with no copy or MMA in flight.  Every
+ * GEMM entry point (rfq_linear, rfq_linear_fused, rfq_linear_grouped)
+ * honours words [1] to [3]; leave them zero in normal use. */
 RFQ_API size_t rfq_linear_workspace_bytes(void);
 
 /* RFQ GEMM (Algorithm 1, Eq. rfq): Y = X~ W~ + phi X^ W~ with both products
@@ -291,6 +299,22 @@ RFQ_API rfq_status rfq_check_finite(const void *x_bf16, int64_t rows, int64_t k,
  * rfq_check_finite); clears it when `clear` != 0. */
 RFQ_API rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *stream);
 
+/* Measurement of the ceiling the RFQ GEMM is held against: the dense
+ * block-scaled FP4 tensor rate of this GPU (the kind::mxf4 MMA that carries
+ * both products of Algorithm 1 / Eq. rfq), with MMAs alone.  Every SM
+ * (cta_pair = 0: 128 x 256 x 64 MMAs, one CTA per SM) or every CTA pair
+ * (cta_pair = 1: 256 x 256 x 64 cta_group::2 MMAs, the RFQ GEMM's form)
+ * issues `iters` back-to-back MMAs from one shared-memory tile of
+ * pseudo-random E2M1 codes (scales 2^0) into one TMEM accumulator; no
+ * copies, scale writes or epilogue.  Time the launch on `stream` with
+ * events; *flop_per_launch (host) receives its MMA work, 2 M N K per MMA
+ * summed over the grid.  workspace: as for rfq_linear (a bounded final wait
+ * that runs out records RFQ_ERR_TIMEOUT there).  iters in [1, 2^24].
+ * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
+ * RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */
+RFQ_API rfq_status rfq_fp4_mma_peak(int32_t cta_pair, int64_t iters, void *workspace, double *flop_per_launch,
+                                    void *stream);
+
 /* Allocation-free variant of rfq_linear.  The paper has no counterpart: this
  * entry point exists for callers that cannot allocate device memory, such as
  * a serving loop that must not stall the device on cudaMalloc, a plug-in
@@ -306,10 +330,15 @@ RFQ_API rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *st
  * accepts fits today.
  *
  * The first call on each device looks up the array's device address with
- * that device current; make that first call before any stream capture.
- * Every call clears the array on `stream` before the GEMM runs, because all
- * calls share it and it keeps what the last call left.  Calls that overlap
- * on the GPU (other streams, other host threads) race on the array.  A
+ * that device current; make that first call before any stream capture.  The
+ * address is kept for the life of the process: a cudaDeviceReset reloads
+ * the library's device code and makes it stale, so a caller of this entry
+ * point does not reset the device.  A call passes rfq_linear's argument
+ * checks first (a rejected call, or one with M == 0 or N == 0, leaves the
+ * array untouched), then clears the array on `stream` before the GEMM runs,
+ * because all calls share it and it keeps what the last call left.  Calls
+ * that overlap on the GPU (other streams, other host threads) race on the
+ * array.  A
  * timeout of a bounded wait is not reported by this variant (use rfq_linear
  * with a workspace to read it); Y is then left unwritten.
  * Errors: those of rfq_linear, and RFQ_ERR_SHAPE as above. */

@@ -300,10 +300,17 @@ rfq_status quantize_act(const void *x_bf16, int64_t M, int64_t K, const rfq_fall
 
 size_t rfq_linear_workspace_bytes(void) { return 256; }
 
-rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_t *phi, int32_t phi_r_s,
-                      const rfq_qtensor *wq, void *y, int32_t out_dtype, void *workspace, void *stream)
+} // extern "C"
+
+namespace rfq {
+// The host-side checks of rfq_linear, in its order; *launch is set when the
+// call would launch a GEMM (false for M == 0 or N == 0).
+rfq_status linear_check(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_t *phi, int32_t phi_r_s,
+                        const rfq_qtensor *wq, void *y, int32_t out_dtype, void *workspace, bool *launch,
+                        bool check_ws)
 {
-    if (!xq || !wq || !y || !workspace)
+    *launch = false;
+    if (!xq || !wq || !y || (check_ws && !workspace))
         return RFQ_ERR_INVALID_ARG;
     if (out_dtype != RFQ_OUT_F32 && out_dtype != RFQ_OUT_BF16)
         return RFQ_ERR_INVALID_ARG;
@@ -337,7 +344,7 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
         return RFQ_ERR_SHAPE;
     if (phi && xr && (hif4 ? (phi_r_s < 64 || phi_r_s % 64 != 0) : (phi_r_s < 128 || phi_r_s % 128 != 0)))
         return RFQ_ERR_SHAPE;
-    if (!aligned16(y) || !aligned16(workspace))
+    if (!aligned16(y) || (check_ws && !aligned16(workspace)))
         return RFQ_ERR_ALIGNMENT;
     if ((s = check_device()) != RFQ_OK)
         return s;
@@ -345,6 +352,26 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
         return RFQ_OK;
     if (!bf16_act && xq->scale_layout != RFQ_SCALE_MMA)
         return RFQ_ERR_UNSUPPORTED;
+    if (!hif4 && wq->scale_layout != RFQ_SCALE_MMA)
+        return RFQ_ERR_UNSUPPORTED;
+    *launch = true;
+    return RFQ_OK;
+}
+} // namespace rfq
+
+extern "C" {
+
+rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_t *phi, int32_t phi_r_s,
+                      const rfq_qtensor *wq, void *y, int32_t out_dtype, void *workspace, void *stream)
+{
+    bool launch = false;
+    const rfq_status s = linear_check(xq, xr, phi, phi_r_s, wq, y, out_dtype, workspace, &launch, true);
+    if (s != RFQ_OK || !launch)
+        return s;
+    const int64_t M = xq->rows, K = xq->k, N = wq->rows;
+    const bool bf16_act = xq->fmt == RFQ_FMT_BF16;
+    const bool hif4 = xq->fmt == RFQ_FMT_HIF4 || bf16_act;
+    const bool f8 = xq->fmt == RFQ_FMT_MXFP8;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (hif4) {
         GemmHif4Args a;
@@ -364,8 +391,6 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
         a.status = static_cast<int32_t *>(workspace);
         return from_cuda(launch_gemm_hif4(a, st));
     }
-    if (wq->scale_layout != RFQ_SCALE_MMA)
-        return RFQ_ERR_UNSUPPORTED;
     GemmMxf4Args a;
     a.a_codes = xq->codes;
     a.a_sf = xq->scales;
@@ -427,6 +452,22 @@ rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, const rfq_
     a.K = K;
     a.status = static_cast<int32_t *>(workspace);
     return from_cuda(launch_gemm_mxf4_fused(a, static_cast<cudaStream_t>(stream)));
+}
+
+rfq_status rfq_fp4_mma_peak(int32_t cta_pair, int64_t iters, void *workspace, double *flop_per_launch,
+                            void *stream)
+{
+    if (!workspace || !flop_per_launch || (cta_pair != 0 && cta_pair != 1))
+        return RFQ_ERR_INVALID_ARG;
+    if (iters < 1 || iters > ((int64_t)1 << 24))
+        return RFQ_ERR_SHAPE;
+    if (!aligned16(workspace))
+        return RFQ_ERR_ALIGNMENT;
+    rfq_status s = check_device();
+    if (s != RFQ_OK)
+        return s;
+    return from_cuda(launch_fp4_mma_peak(cta_pair, iters, static_cast<int32_t *>(workspace), flop_per_launch,
+                                         static_cast<cudaStream_t>(stream)));
 }
 
 rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *stream)

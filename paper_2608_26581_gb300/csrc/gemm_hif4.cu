@@ -89,6 +89,7 @@ struct Smem {
     PhiRec rec[2];
     uint32_t stage_info[STAGES]; // the tile's residual-stage count | (this stage's residual applies) << 31
     uint32_t tmem_base;
+    uint64_t wait_ns;             // limit of the bounded waits (workspace word 1, else wl)
     int32_t abort_flag;
     int32_t issued;
 };
@@ -148,11 +149,14 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const volatile int32_t *gstat = status;
 
-    if (threadIdx.x == 0)
+    if (threadIdx.x == 0) {
         S.abort_flag = *gstat;
+        S.wait_ns = ws_wait_limit_ns(status);
+    }
     __syncthreads();
     if (S.abort_flag != 0)
         return;
+    const uint64_t wl = S.wait_ns;
     __syncthreads();
 
     const int nks = K / BK;
@@ -201,6 +205,10 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
         if (lane == 0) {
             int p = 0, it = 0;
             bool stop = false;
+            if (!held_start_wait(status, wl)) { // a test-held start never opened
+                flag_timeout(S, status);
+                stop = true;
+            }
             for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x, ++it) {
                 const int m_tile = tile / n_tiles, n_tile = tile - m_tile * n_tiles;
                 // one k-stage: wait for its ring slot, publish the tile's info and
@@ -208,7 +216,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                 auto produce = [&](int ks, uint32_t count, auto res_t) {
                     constexpr bool ron = decltype(res_t)::value;
                     const int slot = p % STAGES;
-                    if (!mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, kWaitLimitNs, gstat)) {
+                    if (!mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, wl, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
                         return;
@@ -242,7 +250,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                         produce(ks, 0u, Bool<RES>{});
                 } else {
                     const int r = it & 1;
-                    if (!mbar_wait(&S.phi_full[r], (it >> 1) & 1, kWaitLimitNs, gstat)) {
+                    if (!mbar_wait(&S.phi_full[r], (it >> 1) & 1, wl, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
                         break;
@@ -280,7 +288,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
             const uint32_t idesc = idesc_bf16(BM, BN);
             for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x, ++it) {
                 const int buf = it & 1;
-                if (!mbar_wait(&S.acc_empty[buf], ((it >> 1) & 1) ^ 1, kWaitLimitNs, gstat)) {
+                if (!mbar_wait(&S.acc_empty[buf], ((it >> 1) & 1) ^ 1, wl, gstat)) {
                     flag_timeout(S, status);
                     break;
                 }
@@ -290,8 +298,8 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                 auto mma_stage = [&](int pos, auto res_t) {
                     constexpr bool ron = decltype(res_t)::value;
                     const int slot = p % STAGES;
-                    if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat) ||
-                        (CONV && !mbar_wait(&S.conv[slot], (p / STAGES) & 1, kWaitLimitNs, gstat))) {
+                    if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, wl, gstat) ||
+                        (CONV && !mbar_wait(&S.conv[slot], (p / STAGES) & 1, wl, gstat))) {
                         flag_timeout(S, status);
                         stop = true;
                         return;
@@ -314,7 +322,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                         mma_stage(ks, Bool<RES>{});
                 } else {
                     // the tile's residual-stage count arrives with its first stage
-                    if (!mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs, gstat)) {
+                    if (!mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, wl, gstat)) {
                         flag_timeout(S, status);
                         break;
                     }
@@ -330,7 +338,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
             }
             if (S.abort_flag) {
                 tc_commit(&S.drain);
-                (void)mbar_wait(&S.drain, 0, kWaitLimitNs);
+                (void)mbar_wait(&S.drain, 0, wl);
             }
         }
     } else if (warp < 2 + EPI_WARPS) {
@@ -340,7 +348,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
         for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++it) {
             const int m_tile = tile / n_tiles, n_tile = tile - m_tile * n_tiles;
             const int buf = it & 1;
-            if (!mbar_wait(&S.acc_full[buf], (it >> 1) & 1, kWaitLimitNs, gstat)) {
+            if (!mbar_wait(&S.acc_full[buf], (it >> 1) & 1, wl, gstat)) {
                 if (lane == 0)
                     flag_timeout(S, status);
                 break;
@@ -439,7 +447,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
         for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x) {
             for (int ks = 0; ks < nks; ++ks, ++p) {
                 const int slot = p % STAGES;
-                if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat)) {
+                if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, wl, gstat)) {
                     if (lane == 0)
                         flag_timeout(S, status);
                     stop = true;
@@ -479,7 +487,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
             for (int j = 0; j < my_tiles; ++j) {
                 const int r = j & 1;
                 if (j >= 2 && !__all_sync(0xffffffffu, mbar_wait(&S.phi_empty[r], ((j >> 1) - 1) & 1,
-                                                                 kWaitLimitNs, gstat))) {
+                                                                 wl, gstat))) {
                     if (lane == 0)
                         flag_timeout(S, status);
                     break;
@@ -508,7 +516,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     if (threadIdx.x == 0 && S.abort_flag) {
         const int issued = S.issued;
         for (int p = max(0, issued - STAGES); p < issued; ++p)
-            (void)mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs);
+            (void)mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, wl);
     }
     __syncthreads();
     if (warp == 1) {

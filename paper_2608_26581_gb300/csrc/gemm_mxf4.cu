@@ -37,9 +37,10 @@
 // 512-byte MMA-layout atom.  A slot holds one stage: A chunk c at 4c, R at
 // 8 + 4c, W~ rows 0-127 at 16 + 8c and rows 128-255 at 20 + 8c.
 //
-// Every mbarrier wait is bounded (kWaitLimitNs) and also gives up as soon as
-// any CTA has recorded a timeout in the caller's status word; the CTA then
-// drains its in-flight copies and MMAs (bounded), frees TMEM and returns.
+// Every mbarrier wait is bounded (kWaitLimitNs, or the limit in the caller's
+// workspace) and also gives up as soon as any CTA has recorded a timeout in
+// the caller's status word; the CTA then drains its in-flight copies and MMAs
+// (bounded), frees TMEM and returns.
 #include <cuda_bf16.h>
 #include <cstdint>
 
@@ -104,6 +105,7 @@ struct Smem {
     PhiRec rec[2];
     uint32_t stage_info[STAGES];      // the tile's info (PhiRec::info), published with each stage
     uint32_t tmem_base;
+    uint64_t wait_ns;             // limit of the bounded waits (workspace word 1, else wl)
     int32_t abort_flag;
     int32_t issued;
     int32_t grp_off[GRP_MAX + 1];     // grouped GEMM: first row of each group (and the end)
@@ -154,11 +156,14 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     const volatile int32_t *gstat = status;
 
     // A bounded wait of an earlier CTA or call gave up: do nothing.
-    if (threadIdx.x == 0)
+    if (threadIdx.x == 0) {
         S.abort_flag = *gstat;
+        S.wait_ns = ws_wait_limit_ns(status);
+    }
     __syncthreads();
     if (S.abort_flag != 0)
         return;
+    const uint64_t wl = S.wait_ns;
     __syncthreads();
 
     const int kc = K >> 7;                 // 128-element chunks
@@ -274,6 +279,10 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
         if (lane == 0) {
             int p = 0, it = 0; // p: stages issued so far (ring position)
             bool stop = false;
+            if (!held_start_wait(status, wl)) { // a test-held start never opened
+                flag_timeout(S, status);
+                stop = true;
+            }
             for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x, ++it) {
                 const TileCoord tc = coord(tile);
                 const int m_tile = tc.a_row0 / BM;    // scale atoms and A rows
@@ -284,7 +293,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                 auto produce = [&](int ks, int nch, uint32_t info, auto res_t) {
                     constexpr bool res_on = decltype(res_t)::value;
                     const int slot = p % STAGES;
-                    if (!mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, kWaitLimitNs, gstat)) {
+                    if (!mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, wl, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
                         return;
@@ -316,7 +325,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                         produce(nf, 1, 0u, Bool<RES>{});
                 } else {
                     const int r = it & 1;
-                    if (!mbar_wait(&S.phi_full[r], (it >> 1) & 1, kWaitLimitNs, gstat)) {
+                    if (!mbar_wait(&S.phi_full[r], (it >> 1) & 1, wl, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
                         break;
@@ -358,7 +367,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
             int p = 0, it = 0;
             bool stop = false;
             for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x, ++it) {
-                if (!mbar_wait(&S.acc_empty, (it & 1) ^ 1, kWaitLimitNs, gstat)) {
+                if (!mbar_wait(&S.acc_empty, (it & 1) ^ 1, wl, gstat)) {
                     flag_timeout(S, status);
                     break;
                 }
@@ -368,8 +377,8 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                 auto mma_stage = [&](int pos, int nch, auto rm_t) {
                     constexpr uint32_t rm = decltype(rm_t)::value;
                     const int slot = p % STAGES, sfs = p % SF_SLOTS;
-                    if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat) ||
-                        !mbar_wait(&S.sf_ready[sfs], (p / SF_SLOTS) & 1, kWaitLimitNs, gstat)) {
+                    if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, wl, gstat) ||
+                        !mbar_wait(&S.sf_ready[sfs], (p / SF_SLOTS) & 1, wl, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
                         return;
@@ -400,7 +409,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                         mma_stage(nf, 1, Mask<RES ? 1u : 0u>{});
                 } else {
                     // the tile's residual-stage count arrives with its first stage
-                    if (!mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs, gstat)) {
+                    if (!mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, wl, gstat)) {
                         flag_timeout(S, status);
                         break;
                     }
@@ -424,7 +433,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
             if (S.abort_flag) {
                 // wait (bounded) until every MMA issued above has completed
                 tc_commit(&S.drain);
-                (void)mbar_wait(&S.drain, 0, kWaitLimitNs);
+                (void)mbar_wait(&S.drain, 0, wl);
             }
         }
     } else if (warp < 2 + EPI_WARPS) {
@@ -436,7 +445,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
         int it = 0;
         for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++it) {
             // warp-uniform outcome: the tcgen05 loads below need the whole warp
-            if (!__all_sync(0xffffffffu, mbar_wait(&S.acc_full, it & 1, kWaitLimitNs, gstat))) {
+            if (!__all_sync(0xffffffffu, mbar_wait(&S.acc_full, it & 1, wl, gstat))) {
                 if (lane == 0)
                     flag_timeout(S, status);
                 break;
@@ -580,7 +589,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                 constexpr uint32_t rm = decltype(rm_t)::value;
                 const int slot = p % STAGES, sfs = p % SF_SLOTS;
                 // warp-uniform outcome: the tcgen05 stores below need the whole warp
-                if (!__all_sync(0xffffffffu, mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat))) {
+                if (!__all_sync(0xffffffffu, mbar_wait(&S.full[slot], (p / STAGES) & 1, wl, gstat))) {
                     if (lane == 0)
                         flag_timeout(S, status);
                     stop = true;
@@ -619,7 +628,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                     write_stage(1, Mask<RES ? 1u : 0u>{});
             } else {
                 // the tile's residual-stage count arrives with its first stage
-                if (!__all_sync(0xffffffffu, mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs, gstat))) {
+                if (!__all_sync(0xffffffffu, mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, wl, gstat))) {
                     if (lane == 0)
                         flag_timeout(S, status);
                     break;
@@ -648,7 +657,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
         for (int j = 0; j < my_tiles; ++j) {
             const int r = j & 1;
             if (j >= 2 && !__all_sync(0xffffffffu, mbar_wait(&S.phi_empty[r], ((j >> 1) - 1) & 1,
-                                                             kWaitLimitNs, gstat))) {
+                                                             wl, gstat))) {
                 if (lane == 0)
                     flag_timeout(S, status);
                 break;
@@ -679,7 +688,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
         // wait (bounded) for the copies of the last stages still in flight
         const int issued = S.issued;
         for (int p = max(0, issued - STAGES); p < issued; ++p)
-            (void)mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs);
+            (void)mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, wl);
     }
     __syncthreads();
     if (warp == 1) {

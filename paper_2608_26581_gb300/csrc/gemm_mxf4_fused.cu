@@ -24,9 +24,10 @@
 //
 // fallback: ALL (phi = 1, residual everywhere) or NONE (plain W4A4).
 //
-// Every mbarrier wait is bounded (kWaitLimitNs) and also gives up as soon as
-// any CTA has recorded a timeout in the caller's status word; the CTA then
-// drains its in-flight copies and MMAs (bounded), frees TMEM and returns.
+// Every mbarrier wait is bounded (kWaitLimitNs, or the limit in the caller's
+// workspace) and also gives up as soon as any CTA has recorded a timeout in
+// the caller's status word; the CTA then drains its in-flight copies and MMAs
+// (bounded), frees TMEM and returns.
 #include <cuda_bf16.h>
 #include <cstdint>
 
@@ -79,6 +80,7 @@ struct Smem {
     uint64_t drain;
     uint64_t sf_ready[SF_SLOTS];
     uint32_t tmem_base;
+    uint64_t wait_ns;             // limit of the bounded waits (workspace word 1, else wl)
     int32_t abort_flag;
     int32_t issued;
 };
@@ -103,11 +105,14 @@ __global__ void __launch_bounds__(THREADS, 1)
     const volatile int32_t *gstat = status;
 
     // A bounded wait of an earlier CTA or call gave up: do nothing.
-    if (threadIdx.x == 0)
+    if (threadIdx.x == 0) {
         S.abort_flag = *gstat;
+        S.wait_ns = ws_wait_limit_ns(status);
+    }
     __syncthreads();
     if (S.abort_flag != 0)
         return;
+    const uint64_t wl = S.wait_ns;
     __syncthreads();
 
     const int kc = K >> 7;                 // 128-element chunks
@@ -149,13 +154,17 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (lane == 0) {
             int p = 0;
             bool stop = false;
+            if (!held_start_wait(status, wl)) { // a test-held start never opened
+                flag_timeout(S, status);
+                stop = true;
+            }
             for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x) {
                 const int n_tile = tile % n_tiles;
                 const int atom0 = n_tile * 2;
                 const int nb = atom0 + 1 < n_atoms ? 2 : 1;
                 for (int ks = 0; ks < nks; ++ks, ++p) {
                     const int slot = p % STAGES;
-                    if (!mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, kWaitLimitNs, gstat)) {
+                    if (!mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, wl, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
                         break;
@@ -178,16 +187,16 @@ __global__ void __launch_bounds__(THREADS, 1)
             int p = 0, it = 0;
             bool stop = false;
             for (int tile = blockIdx.x; tile < tiles && !stop; tile += gridDim.x, ++it) {
-                if (!mbar_wait(&S.acc_empty, (it & 1) ^ 1, kWaitLimitNs, gstat)) {
+                if (!mbar_wait(&S.acc_empty, (it & 1) ^ 1, wl, gstat)) {
                     flag_timeout(S, status);
                     break;
                 }
                 tc_fence_after();
                 for (int ks = 0; ks < nks; ++ks, ++p) {
                     const int slot = p % STAGES, sfs = p % SF_SLOTS;
-                    if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat) ||
-                        !mbar_wait(&S.conv[slot], (p / STAGES) & 1, kWaitLimitNs, gstat) ||
-                        !mbar_wait(&S.sf_ready[sfs], (p / SF_SLOTS) & 1, kWaitLimitNs, gstat)) {
+                    if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, wl, gstat) ||
+                        !mbar_wait(&S.conv[slot], (p / STAGES) & 1, wl, gstat) ||
+                        !mbar_wait(&S.sf_ready[sfs], (p / SF_SLOTS) & 1, wl, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
                         break;
@@ -217,7 +226,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             if (S.abort_flag) {
                 // wait (bounded) until every MMA issued above has completed
                 tc_commit(&S.drain);
-                (void)mbar_wait(&S.drain, 0, kWaitLimitNs);
+                (void)mbar_wait(&S.drain, 0, wl);
             }
         }
     } else if (warp < 2 + EPI_WARPS) {
@@ -230,7 +239,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++it) {
             const int m_tile = tile / n_tiles, n_tile = tile - m_tile * n_tiles;
             // warp-uniform outcome: the tcgen05 loads below need the whole warp
-            if (!__all_sync(0xffffffffu, mbar_wait(&S.acc_full, it & 1, kWaitLimitNs, gstat))) {
+            if (!__all_sync(0xffffffffu, mbar_wait(&S.acc_full, it & 1, wl, gstat))) {
                 if (lane == 0)
                     flag_timeout(S, status);
                 break;
@@ -319,8 +328,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             for (int ks = 0; ks < nks; ++ks, ++p) {
                 const int slot = p % STAGES, sfs = p % SF_SLOTS;
                 // warp-uniform outcome: the tcgen05 stores below need the whole warp
-                if (!__all_sync(0xffffffffu, mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat) &&
-                                                 mbar_wait(&S.conv[slot], (p / STAGES) & 1, kWaitLimitNs, gstat))) {
+                if (!__all_sync(0xffffffffu, mbar_wait(&S.full[slot], (p / STAGES) & 1, wl, gstat) &&
+                                                 mbar_wait(&S.conv[slot], (p / STAGES) & 1, wl, gstat))) {
                     if (lane == 0)
                         flag_timeout(S, status);
                     stop = true;
@@ -368,7 +377,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 const int c0 = 2 * ks, nch = min(2, kc - c0);
                 const bool lane_in = (lane >> 4) < nch;   // lanes 16..31 hold the second 128-element chunk
                 // the stage's A / R / scale buffers are free once its previous MMAs completed
-                if (!__all_sync(0xffffffffu, mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, kWaitLimitNs, gstat))) {
+                if (!__all_sync(0xffffffffu, mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, wl, gstat))) {
                     if (lane == 0)
                         flag_timeout(S, status);
                     stop = true;
@@ -422,7 +431,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         // wait (bounded) for the copies of the last stages still in flight
         const int issued = S.issued;
         for (int p = max(0, issued - STAGES); p < issued; ++p)
-            (void)mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs);
+            (void)mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, wl);
     }
     __syncthreads();
     if (warp == 1) {

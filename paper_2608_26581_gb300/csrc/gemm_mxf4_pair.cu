@@ -54,10 +54,11 @@
 // load issued by the producer waits behind the stage copies in flight on its
 // SM (thousands of cycles).
 //
-// Every mbarrier wait is bounded (kWaitLimitNs) and also gives up when any
-// CTA has recorded a timeout in the caller's status word.  Neither CTA of a
-// pair leaves before the final cluster barrier, so the peer never signals a
-// CTA that has exited; the even CTA drains its MMAs before that barrier.
+// Every mbarrier wait is bounded (kWaitLimitNs, or the limit in the caller's
+// workspace) and also gives up when any CTA has recorded a timeout in the
+// caller's status word.  Neither CTA of a pair leaves before the final
+// cluster barrier, so the peer never signals a CTA that has exited; the even
+// CTA drains its MMAs before that barrier.
 #include <cuda_bf16.h>
 #include <cstdint>
 
@@ -126,6 +127,7 @@ struct Smem {
     int32_t grp_pairs[GRP_MAX + 1]; // grouped GEMM: 256-row pairs of the groups before each group
     int32_t grp_bad;                // grouped GEMM: the row offsets break the contract
     uint32_t tmem_base;
+    uint64_t wait_ns;             // limit of the bounded waits (workspace word 1, else wl)
     int32_t abort_flag;
 };
 constexpr size_t kSmemBytes = sizeof(Smem) + 1024;
@@ -203,6 +205,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
         // A bounded wait of an earlier CTA or call gave up: skip the work
         // (both CTAs still meet at the cluster barriers).
         S.abort_flag = *gstat;
+        S.wait_ns = ws_wait_limit_ns(status);
         fence_mbar_init();
     }
     if (warp == 0 && lane == 0) {
@@ -265,6 +268,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
     tc_fence_after();
     const uint32_t tmem = S.tmem_base;
     const bool skip = S.abort_flag != 0 || (GRP && S.grp_bad != 0);
+    const uint64_t wl = S.wait_ns;
     const int tiles = n_tiles * (GRP ? S.grp_pairs[G] : m_pairs);
     auto coord = [&](int tile) {
         const int pi = tile / n_tiles, nt = tile - pi * n_tiles;
@@ -298,6 +302,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
             const uint32_t full0 = mapa_shared(smem_u32(&S.full[0]), 0);   // the even CTA's barriers
             int p = 0, it = 0;
             bool stop = false;
+            if (!held_start_wait(status, wl)) { // a test-held start never opened
+                flag_timeout(S, status);
+                stop = true;
+            }
             for (int tile = pair; tile < tiles && !stop; tile += pairs, ++it) {
                 const TileCoord tc = coord(tile);
                 const int a_row = tc.a_row0 + (int)rank * BM;   // this CTA's first A row
@@ -311,7 +319,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 auto produce = [&](int ks, int nch, uint32_t info, auto res_t) {
                     constexpr bool res_on = decltype(res_t)::value;
                     const int slot = p % STAGES;
-                    if (!mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, kWaitLimitNs, gstat)) {
+                    if (!mbar_wait(&S.empty[slot], ((p / STAGES) & 1) ^ 1, wl, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
                         return;
@@ -348,7 +356,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                         produce(nf, 1, 0u, Bool<RES>{});
                 } else {
                     const int r = it & 1;
-                    if (!mbar_wait(&S.phi_full[r], (it >> 1) & 1, kWaitLimitNs, gstat)) {
+                    if (!mbar_wait(&S.phi_full[r], (it >> 1) & 1, wl, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
                         break;
@@ -386,9 +394,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 // wait (bounded) until the copies of the last stages landed: this
                 // CTA's scale atoms, and (even CTA) both CTAs' codes
                 for (int q = max(0, p - STAGES); q < p; ++q) {
-                    (void)mbar_wait(&S.sf_full[q % STAGES], (q / STAGES) & 1, kWaitLimitNs);
+                    (void)mbar_wait(&S.sf_full[q % STAGES], (q / STAGES) & 1, wl);
                     if (lead)
-                        (void)mbar_wait(&S.full[q % STAGES], (q / STAGES) & 1, kWaitLimitNs);
+                        (void)mbar_wait(&S.full[q % STAGES], (q / STAGES) & 1, wl);
                 }
         }
     } else if (warp == 1) {
@@ -397,7 +405,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
             int p = 0, it = 0;
             bool stop = false;
             for (int tile = pair; tile < tiles && !stop; tile += pairs, ++it) {
-                if (!mbar_wait<true>(&S.acc_empty, (it & 1) ^ 1, kWaitLimitNs, gstat)) {
+                if (!mbar_wait<true>(&S.acc_empty, (it & 1) ^ 1, wl, gstat)) {
                     flag_timeout(S, status);
                     break;
                 }
@@ -407,8 +415,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 auto mma_stage = [&](int pos, int nch, auto rm_t) {
                     constexpr uint32_t rm = decltype(rm_t)::value;
                     const int slot = p % STAGES, sfs = p % SF_SLOTS;
-                    if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat) ||
-                        !mbar_wait<true>(&S.sf_ready[sfs], (p / SF_SLOTS) & 1, kWaitLimitNs, gstat)) {
+                    if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, wl, gstat) ||
+                        !mbar_wait<true>(&S.sf_ready[sfs], (p / SF_SLOTS) & 1, wl, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
                         return;
@@ -451,7 +459,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                         mma_stage(nf, 1, Mask<RES ? 1u : 0u>{});
                 } else {
                     // the tile's residual-stage count arrives with its first stage
-                    if (!mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs, gstat)) {
+                    if (!mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, wl, gstat)) {
                         flag_timeout(S, status);
                         break;
                     }
@@ -475,7 +483,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
             // every MMA (and its commits to both CTAs) completes before the
             // final cluster barrier
             tc_commit_pair_mc(&S.drain, 0x1);
-            (void)mbar_wait(&S.drain, 0, kWaitLimitNs);
+            (void)mbar_wait(&S.drain, 0, wl);
         }
     } else if (warp < 2 + EPI_WARPS) {
         // ------------------------------------------------ epilogue (warps 2..9)
@@ -487,7 +495,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
         int it = 0;
         for (int tile = pair; tile < tiles && !skip; tile += pairs, ++it) {
             // warp-uniform outcome: the tcgen05 loads below need the whole warp
-            if (!__all_sync(0xffffffffu, mbar_wait(&S.acc_full, it & 1, kWaitLimitNs, gstat))) {
+            if (!__all_sync(0xffffffffu, mbar_wait(&S.acc_full, it & 1, wl, gstat))) {
                 if (lane == 0)
                     flag_timeout(S, status);
                 break;
@@ -632,7 +640,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 constexpr uint32_t rm = decltype(rm_t)::value;
                 const int slot = p % STAGES, sfs = p % SF_SLOTS;
                 // warp-uniform outcome: the tcgen05 stores below need the whole warp
-                if (!__all_sync(0xffffffffu, mbar_wait(&S.sf_full[slot], (p / STAGES) & 1, kWaitLimitNs, gstat))) {
+                if (!__all_sync(0xffffffffu, mbar_wait(&S.sf_full[slot], (p / STAGES) & 1, wl, gstat))) {
                     if (lane == 0)
                         flag_timeout(S, status);
                     stop = true;
@@ -675,7 +683,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     write_stage(1, Mask<RES ? 1u : 0u>{});
             } else {
                 // the tile's residual-stage count arrives with its first stage
-                if (!__all_sync(0xffffffffu, mbar_wait(&S.sf_full[p % STAGES], (p / STAGES) & 1, kWaitLimitNs, gstat))) {
+                if (!__all_sync(0xffffffffu, mbar_wait(&S.sf_full[p % STAGES], (p / STAGES) & 1, wl, gstat))) {
                     if (lane == 0)
                         flag_timeout(S, status);
                     break;
@@ -714,7 +722,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
         for (int j = 0; j < (skip ? 0 : my_tiles); ++j) {
             const int r = j & 1;
             if (j >= 2 && !__all_sync(0xffffffffu, mbar_wait(&S.phi_empty[r], ((j >> 1) - 1) & 1,
-                                                             kWaitLimitNs, gstat))) {
+                                                             wl, gstat))) {
                 if (lane == 0)
                     flag_timeout(S, status);
                 break;

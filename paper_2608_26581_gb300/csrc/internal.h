@@ -18,6 +18,23 @@ constexpr int32_t kDevNonFinite = 3;   // rfq_check_finite found an Inf or NaN
 // Bounded waits in the GEMM give up after this many nanoseconds.
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
+// Words (int32) of a GEMM call's workspace, zeroed by the caller:
+//   [kWsStatus] device status (kDevOk, kDevTimeout, ...), sticky;
+//   [kWsWaitUs] limit of this call's bounded waits in microseconds
+//               (0: kWaitLimitNs);
+//   [kWsHold]   held start: when non-zero, each TMA producer waits (bounded)
+//               for word [kWsOpen] to become non-zero before its first copy,
+//               so a caller can make a wait run out with no copy or MMA in
+//               flight and check the kernel's timeout path.
+constexpr int kWsStatus = 0, kWsWaitUs = 1, kWsHold = 2, kWsOpen = 3;
+
+// The wait limit a workspace asks for.
+__device__ __forceinline__ uint64_t ws_wait_limit_ns(const int32_t *ws)
+{
+    const int32_t us = reinterpret_cast<const volatile int32_t *>(ws)[kWsWaitUs];
+    return us > 0 ? (uint64_t)us * 1000ull : kWaitLimitNs;
+}
+
 // Byte offset of E8M0 scale (row m, 32-element block b) in the MMA layout
 // (512-byte atoms of 128 rows x 4 blocks; kc = K / 128 atoms per row band).
 __host__ __device__ inline int64_t sf_mma_offset(int64_t m, int64_t b, int64_t kc)
@@ -119,6 +136,18 @@ cudaError_t launch_gemm_hif4(const GemmHif4Args &a, cudaStream_t st);
 // swizzle: 0 none, 64 or 128 (bytes)
 bool encode_tmap_2d_u8(CUtensorMap *map, const void *base, uint64_t inner_bytes, uint64_t rows,
                        uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows, int swizzle);
+
+// ---- the dense FP4 MMA rate alone (mma_peak.cu): `iters` MMAs per SM (pair
+// = 0, 128 x 256 x 64) or per CTA pair (pair = 1, 256 x 256 x 64); *flop =
+// the launch's MMA work
+cudaError_t launch_fp4_mma_peak(int pair, int64_t iters, int32_t *status, double *flop, cudaStream_t st);
+
+// rfq_linear's host-side checks (api.cu): RFQ_OK with *launch set when the
+// call would launch a GEMM, else the status rfq_linear returns; check_ws =
+// false leaves the workspace pointer out of the checks.
+rfq_status linear_check(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_t *phi, int32_t phi_r_s,
+                        const rfq_qtensor *wq, void *y, int32_t out_dtype, void *workspace, bool *launch,
+                        bool check_ws);
 
 // Number of SMs of the current device (cached).
 int num_sms();

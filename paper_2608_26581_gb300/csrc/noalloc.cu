@@ -31,7 +31,10 @@ std::mutex g_mu;
 void *g_scratch_addr[kMaxDevices] = {};
 
 // Device address of the scratch array on the current device (looked up on
-// the first call on that device, with that device current).
+// the first call on that device, with that device current, and kept for the
+// life of the process: a cudaDeviceReset, which reloads the library's device
+// code, makes the kept address stale, so callers of this entry point do not
+// reset the device).
 rfq_status scratch_address(void **out)
 {
     int dev = 0;
@@ -56,9 +59,14 @@ extern "C" rfq_status rfq_linear_noalloc(const rfq_qtensor *xq, const rfq_qtenso
 {
     if (rfq_linear_workspace_bytes() > kNoallocScratchBytes)
         return RFQ_ERR_SHAPE;   // the GEMM needs more scratch than the fixed array holds
+    // rfq_linear's own checks first: a call it would reject, or one with
+    // nothing to compute, leaves the shared array untouched.
+    bool launch = false;
+    rfq_status s = rfq::linear_check(xq, xr, phi, phi_r_s, wq, y, out_dtype, nullptr, &launch, false);
+    if (s != RFQ_OK || !launch)
+        return s;
     void *scratch = nullptr;
-    rfq_status s = scratch_address(&scratch);
-    if (s != RFQ_OK)
+    if ((s = scratch_address(&scratch)) != RFQ_OK)
         return s;
     // The array keeps whatever the previous call left; its status word must
     // start at zero or the GEMM returns without computing.

@@ -97,6 +97,24 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint64
     }
 }
 
+// The held start of a GEMM call (workspace word [2] non-zero): waits until
+// word [3] becomes non-zero, for at most `limit_ns`, or until the status word
+// [0] records a failure.  Returns false if the start stayed held.
+__device__ __forceinline__ bool held_start_wait(const int32_t *ws, uint64_t limit_ns)
+{
+    const volatile int32_t *w = ws;
+    if (w[2] == 0)
+        return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (;;) {
+        if (w[3] != 0)
+            return true;
+        if (w[0] != 0 || globaltimer_ns() - t0 > limit_ns)
+            return false;
+        __nanosleep(256);
+    }
+}
+
 // ---------------------------------------------------------------- clusters
 
 __device__ __forceinline__ uint32_t cluster_ctarank()

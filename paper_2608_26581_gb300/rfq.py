@@ -29,7 +29,7 @@ STATUS_NAMES = {0: "RFQ_OK", 1: "RFQ_ERR_INVALID_ARG", 2: "RFQ_ERR_SHAPE", 3: "R
 EXPORTED = ("rfq_status_string", "rfq_qtensor_bytes", "rfq_quantize_weight", "rfq_quantize_act",
             "rfq_linear_workspace_bytes", "rfq_linear", "rfq_workspace_status", "rfq_dequant",
             "rfq_linear_noalloc", "rfq_linear_fused", "rfq_convert", "rfq_linear_grouped", "rfq_check_finite",
-            "rfq_quantize_act_expand")
+            "rfq_quantize_act_expand", "rfq_fp4_mma_peak")
 
 
 class RFQError(RuntimeError):
@@ -88,6 +88,8 @@ def load_library(path: str = LIB_PATH):
         lib.rfq_check_finite.argtypes = [P, I64, I64, P, P]
         lib.rfq_linear_grouped.restype = I32
         lib.rfq_linear_grouped.argtypes = [QTP, QTP, P, I32, P, I32, QTP, I64, P, I32, P, P]
+        lib.rfq_fp4_mma_peak.restype = I32
+        lib.rfq_fp4_mma_peak.argtypes = [I32, I64, P, ctypes.POINTER(ctypes.c_double), P]
         _lib = lib
     return _lib
 
@@ -262,3 +264,12 @@ def rfq_linear_fused(x: torch.Tensor, wq: QTensor, y: torch.Tensor, out_dtype: i
     w = wq.c()
     _check(load_library().rfq_linear_fused(_ptr(x), M, K, ctypes.byref(w), ctypes.byref(fb), _ptr(y), out_dtype,
                                            _ptr(workspace), _stream(stream)), "rfq_linear_fused")
+
+
+def rfq_fp4_mma_peak(cta_pair: bool, iters: int, workspace: torch.Tensor, stream=None) -> float:
+    """Launches the MMA-only FP4 rate measurement (see include/rfq.h) on the
+    stream; returns the launch's MMA work in FLOP (time it with events)."""
+    flop = ctypes.c_double(0.0)
+    _check(load_library().rfq_fp4_mma_peak(1 if cta_pair else 0, iters, _ptr(workspace), ctypes.byref(flop),
+                                           _stream(stream)), "rfq_fp4_mma_peak")
+    return flop.value

@@ -30,3 +30,19 @@ def orc():
     import oracle
     oracle.build()
     return oracle
+
+
+@pytest.fixture(autouse=True)
+def _canary_guards(request, monkeypatch):
+    """GPU tests: every quantized matrix the test allocates through
+    rfq.empty_qtensor carries canary bytes past its codes and its scales,
+    checked once the test has run (tests/gpu_util.py)."""
+    if request.node.get_closest_marker("gpu") is None:
+        yield
+        return
+    import gpu_util
+    from paper_2608_26581_gb300 import rfq
+    monkeypatch.setattr(rfq, "empty_qtensor", gpu_util.guarded_qtensor)
+    gpu_util._guarded.clear()
+    yield
+    gpu_util.check_guards()

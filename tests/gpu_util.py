@@ -61,3 +61,44 @@ def check_y(y_gpu: np.ndarray, y_ref: np.ndarray, bf16: bool = False):
         assert rel <= 1e-5, f"rel Frobenius {rel:.3e}"
     assert ok_abs, f"max abs err {err.max():.3e} vs max|Y| {amax:.3e}"
     return rel
+
+
+# Canary guard bytes: buffers the kernels write are allocated with GUARD
+# extra bytes filled with CANARY after their end, and every guard is checked
+# after the test (a write past the end of an output shows up there).
+CANARY = 0xA5
+GUARD = 256
+_guarded = []
+
+
+def guarded_bytes(nbytes: int) -> torch.Tensor:
+    """A uint8 device buffer of nbytes followed by GUARD canary bytes; the
+    returned tensor is the nbytes payload (16-byte aligned)."""
+    base = torch.empty(nbytes + GUARD, dtype=torch.uint8, device=DEV)
+    base[nbytes:].fill_(CANARY)
+    _guarded.append((base, nbytes))
+    return base[:nbytes]
+
+
+def guarded_empty(shape, dtype) -> torch.Tensor:
+    n = int(np.prod(shape)) * torch.empty(0, dtype=dtype).element_size()
+    return guarded_bytes(n).view(dtype).view(*shape)
+
+
+def guarded_full(shape, value, dtype) -> torch.Tensor:
+    t = guarded_empty(shape, dtype)
+    t.fill_(value)
+    return t
+
+
+def guarded_qtensor(fmt: int, scale_layout: int, rows: int, k: int, device=DEV) -> rfq.QTensor:
+    cb, sb = rfq.rfq_qtensor_bytes(fmt, scale_layout, rows, k)
+    return rfq.QTensor(fmt, scale_layout, rows, k, guarded_bytes(max(cb, 16)), guarded_bytes(max(sb, 16)))
+
+
+def check_guards():
+    """Every guard allocated since the last check still holds CANARY."""
+    torch.cuda.synchronize()
+    bad = [(n, int((b[n:] != CANARY).sum())) for b, n in _guarded if not bool((b[n:] == CANARY).all())]
+    _guarded.clear()
+    assert not bad, f"bytes past the end of an output buffer were written: {bad}"

@@ -152,3 +152,33 @@ def test_quantize_act_expand_fp8_residual_host_checks(lib):
     assert call(P(16), M, K, None, r(x4), r(x8), None, r(x8_row), None, None) == rfq.RFQ_ERR_INVALID_ARG
     # an MXFP4 residual has no operand form to write
     assert call(P(16), M, K, None, r(x4), r(x4), None, r(x8), r(x8), None) == rfq.RFQ_ERR_UNSUPPORTED
+
+
+def test_fp4_mma_peak_host_checks(lib):
+    """rfq_fp4_mma_peak rejects a null workspace or result pointer, a form
+    other than 0 / 1, an iteration count outside [1, 2^24] and a misaligned
+    workspace on the host (none of these calls reaches a launch)."""
+    from paper_2608_26581_gb300 import rfq
+    P = ctypes.c_void_p
+    flop = ctypes.c_double(0.0)
+    r = ctypes.byref
+    call = lib.rfq_fp4_mma_peak
+    assert call(0, 16, None, r(flop), None) == rfq.RFQ_ERR_INVALID_ARG
+    assert call(0, 16, P(16), None, None) == rfq.RFQ_ERR_INVALID_ARG
+    assert call(2, 16, P(16), r(flop), None) == rfq.RFQ_ERR_INVALID_ARG
+    assert call(1, 0, P(16), r(flop), None) == rfq.RFQ_ERR_SHAPE
+    assert call(1, (1 << 24) + 1, P(16), r(flop), None) == rfq.RFQ_ERR_SHAPE
+    assert call(0, 16, P(8), r(flop), None) == rfq.RFQ_ERR_ALIGNMENT
+
+
+def test_noalloc_rejects_before_touching_its_array(lib):
+    """rfq_linear_noalloc runs rfq_linear's host checks before it clears its
+    shared array: bad arguments return rfq_linear's status (no device work)."""
+    from paper_2608_26581_gb300 import rfq
+    P = ctypes.c_void_p
+    r = ctypes.byref
+    assert lib.rfq_linear_noalloc(None, None, None, 0, None, None, 0, None) == rfq.RFQ_ERR_INVALID_ARG
+    xq = rfq._QT(rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA, 128, 256, 16, 16)
+    wq_bad = rfq._QT(rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA, 40, 256, 16, 16)   # N % 16 != 0
+    assert lib.rfq_linear_noalloc(r(xq), None, None, 0, r(wq_bad), P(16), 0, None) == rfq.RFQ_ERR_SHAPE
+    assert lib.rfq_linear_noalloc(r(xq), None, None, 0, r(xq), P(8), 0, None) == rfq.RFQ_ERR_ALIGNMENT

@@ -8,7 +8,7 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_util import DEV, check_y, qtensor_host, to_dev_bf16
+from gpu_util import DEV, check_y, qtensor_host, to_dev_bf16, guarded_full
 from paper_2608_26581_gb300 import rfq
 from paper_2608_26581_gb300.synth import ActSpec, make_activation, make_weight
 
@@ -36,8 +36,7 @@ def _case(orc, counts, K, N, fmt="rfq4", mode=rfq.RFQ_FALLBACK_ALL, tau=0.0, r_s
     wb = np.concatenate(wbs, axis=1)                  # W for all groups: [K, G N]
     x, w = to_dev_bf16(xb), to_dev_bf16(wb)
     ws = torch.zeros(rfq.rfq_linear_workspace_bytes() // 4, dtype=torch.int32, device=DEV)
-    y = torch.full((total, N), float("nan"), dtype=torch.float32 if out == rfq.RFQ_OUT_F32 else torch.bfloat16,
-                   device=DEV)
+    y = guarded_full((total, N), float("nan"), torch.float32 if out == rfq.RFQ_OUT_F32 else torch.bfloat16)
     phi = None
     f8 = fmt != "rfq4"
     wq = rfq.empty_qtensor(F4, MMA, G * N, K)
@@ -138,7 +137,7 @@ def test_grouped_bad_offsets_are_reported(orc):
     rfq.rfq_quantize_weight(w, wq)
     ws = torch.zeros(rfq.rfq_linear_workspace_bytes() // 4, dtype=torch.int32, device=DEV)
     for bad in ([0, 100, 256], [0, 256, 128], [0, 128, 300]):   # unaligned start, decreasing, past the rows
-        y = torch.full((total, N), float("nan"), dtype=torch.float32, device=DEV)
+        y = guarded_full((total, N), float("nan"), torch.float32)
         off = torch.tensor(bad, dtype=torch.int32, device=DEV)
         rfq.rfq_linear_grouped(xq, None, None, 256, off, wq, N, y, rfq.RFQ_OUT_F32, ws)
         assert rfq.rfq_workspace_status(ws, clear=True) == rfq.RFQ_ERR_SHAPE

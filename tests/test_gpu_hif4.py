@@ -5,7 +5,7 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_util import DEV, check_y, qtensor_host, to_dev_bf16
+from gpu_util import DEV, check_y, qtensor_host, to_dev_bf16, guarded_full
 from paper_2608_26581_gb300 import rfq
 from paper_2608_26581_gb300.synth import WORKLOADS, ActSpec, f32_to_bf16_bits, make_activation, make_weight
 
@@ -197,8 +197,7 @@ def _linear(xb, wb, out=rfq.RFQ_OUT_F32, mode=rfq.RFQ_FALLBACK_ALL, tau=0.0, r_s
     w16 = rfq.empty_bf16_operand(N, K)
     rfq.rfq_dequant(wq, w16.codes)
     xq, xr, phi = _quant(xb, rfq.RFQ_SCALE_MMA, mode, tau, 128, r_s)
-    y = torch.full((M, N), float("nan"), dtype=torch.float32 if out == rfq.RFQ_OUT_F32 else torch.bfloat16,
-                   device=DEV)
+    y = guarded_full((M, N), float("nan"), torch.float32 if out == rfq.RFQ_OUT_F32 else torch.bfloat16)
     ws = torch.zeros(64, dtype=torch.int32, device=DEV)
     a, r = (_expand(xq), _expand(xr) if xr is not None else None) if expand else (xq, xr)
     rfq.rfq_linear(a, r, phi if use_phi else None, r_s, w16, y, out, ws)

@@ -5,7 +5,7 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_util import DEV, check_y, qtensor_host, to_dev_bf16
+from gpu_util import DEV, check_y, qtensor_host, to_dev_bf16, guarded_full
 from paper_2608_26581_gb300 import rfq
 from paper_2608_26581_gb300.synth import WORKLOADS, ActSpec, make_activation, make_weight
 
@@ -28,8 +28,7 @@ def _run(xb, wb, mode=rfq.RFQ_FALLBACK_ALL, out=rfq.RFQ_OUT_F32, tau=0.0, r_s=25
     xr = rfq.empty_qtensor(FMT, MMA, M, K) if mode != rfq.RFQ_FALLBACK_NONE else None
     phi = torch.empty(((M + 127) // 128) * ((K + r_s - 1) // r_s), dtype=torch.uint8, device=DEV)
     rfq.rfq_quantize_act(x, xq, xr, phi, mode=mode, tau=tau, p_s=128, r_s=r_s)
-    y = torch.full((M, N), float("nan"), dtype=torch.float32 if out == rfq.RFQ_OUT_F32 else torch.bfloat16,
-                   device=DEV)
+    y = guarded_full((M, N), float("nan"), torch.float32 if out == rfq.RFQ_OUT_F32 else torch.bfloat16)
     ws = _workspace()
     rfq.rfq_linear(xq, xr, phi if use_phi else None, r_s, wq, y, out, ws)
     assert rfq.rfq_workspace_status(ws) == rfq.RFQ_OK

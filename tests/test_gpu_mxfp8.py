@@ -7,7 +7,7 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_util import DEV, check_y, qtensor_host, to_dev_bf16
+from gpu_util import DEV, check_y, qtensor_host, to_dev_bf16, guarded_full
 from paper_2608_26581_gb300 import rfq
 from paper_2608_26581_gb300.synth import WORKLOADS, ActSpec, f32_to_bf16_bits, make_activation, make_weight
 
@@ -180,8 +180,7 @@ def _gemm_case(orc, M, K, N, kind, out=rfq.RFQ_OUT_F32, mode=rfq.RFQ_FALLBACK_AL
     x = to_dev_bf16(xb)
     w = to_dev_bf16(wb)
     ws = torch.zeros(rfq.rfq_linear_workspace_bytes() // 4, dtype=torch.int32, device=DEV)
-    y = torch.full((M, N), float("nan"), dtype=torch.float32 if out == rfq.RFQ_OUT_F32 else torch.bfloat16,
-                   device=DEV)
+    y = guarded_full((M, N), float("nan"), torch.float32 if out == rfq.RFQ_OUT_F32 else torch.bfloat16)
     phi = None
     if kind == "w8a8":
         wq = rfq.empty_qtensor(F8, MMA, N, K)

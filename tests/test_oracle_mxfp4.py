@@ -58,23 +58,36 @@ def _bruteforce_e2m1(y):
     return best[1] | (8 if math.copysign(1.0, y) < 0 else 0)
 
 
+def _bruteforce_e2m1_vec(y):
+    """_bruteforce_e2m1 over an array: the argmin over the 8 magnitudes, ties
+    to the even mantissa bit, the sign bit of y."""
+    mags = np.array([E2M1_TABLE[c] for c in range(8)])
+    d = np.abs(np.abs(y)[:, None] - mags[None, :])
+    best = d.min(axis=1, keepdims=True)
+    tied = d == best
+    # among the tied codes prefer an even one (at most two codes tie)
+    even = tied & (np.arange(8)[None, :] % 2 == 0)
+    code = np.where(even.any(axis=1), even.argmax(axis=1), tied.argmax(axis=1))
+    return code | np.where(np.signbit(y), 8, 0)
+
+
 def test_e2m1_encode_bruteforce_all_bf16(orc):
-    # Every finite bf16 pattern, divided by each power of two that moves it
-    # into (or near) the E2M1 range, must round like the brute-force argmin.
+    # Every one of the 65 536 bf16 patterns that is finite, divided by each
+    # power of two that moves it into (or near) the E2M1 range, must round
+    # like the brute-force argmin.
     bits = np.arange(0, 1 << 16, dtype=np.uint32)
     f = (bits << 16).view(np.float32)
-    fin = np.isfinite(f)
-    vals = f[fin].astype(np.float64)
-    rng = np.random.default_rng(0)
-    sample = rng.choice(vals.size, 6000, replace=False)
-    for v in vals[sample]:
-        if v == 0:
-            ys = [v]
-        else:
-            ex = math.frexp(abs(v))[1]
-            ys = [math.ldexp(v, -(ex - 1) + s) for s in range(-3, 5)]
-        for y in ys:
-            assert orc.e2m1_encode(y) == _bruteforce_e2m1(y), y
+    vals = f[np.isfinite(f)].astype(np.float64)
+    assert vals.size == 65536 - 2 * 128          # every pattern but the 128 Inf / NaN ones per sign
+    ex = np.frexp(np.abs(vals))[1]
+    ys = np.concatenate([np.where(vals == 0, vals, np.ldexp(vals, -(ex - 1) + s)) for s in range(-3, 5)])
+    want = _bruteforce_e2m1_vec(ys)
+    got = np.fromiter((orc.e2m1_encode(float(y)) for y in ys), np.int64, ys.size)
+    bad = np.nonzero(got != want)[0]
+    assert bad.size == 0, [(ys[i], got[i], want[i]) for i in bad[:5]]
+    # the vectorised brute force agrees with the scalar one on a sample
+    for y in ys[:: 4099]:
+        assert _bruteforce_e2m1(y) == _bruteforce_e2m1_vec(np.array([y]))[0]
 
 
 def test_scale_rule_bruteforce_all_bytes(orc):
