@@ -481,7 +481,10 @@ def run_rfq(args):
     # L2 for every workload but the tiny parity case).
     bufs = [buffer_set(x), buffer_set(x.clone())]
     y_host = torch.empty(Mb, max(N, 16), dtype=torch.bfloat16).pin_memory()
-    wsp = torch.zeros(rfq.rfq_linear_workspace_bytes() // 4, dtype=torch.int32, device=dev)
+    # the GEMM workspace; the fused variant's also holds the in-GEMM quantizer's
+    # unit counters and scratch codes (one workspace: the steps never overlap)
+    wsp = (rfq.fused_workspace(Mb, K, rfq.RFQ_FALLBACK_ALL, device=dev) if fused else
+           torch.zeros(rfq.rfq_linear_workspace_bytes() // 4, dtype=torch.int32, device=dev))
     stream = torch.cuda.current_stream(dev)
     # quantizer-only workload: its result (both pathways' codes and scales) is read back
     q_out = lambda b: [b["xq"].codes, b["xq"].scales, b["xr"].codes, b["xr"].scales]
@@ -682,7 +685,8 @@ def run_rfq(args):
         # CTA pairs beyond one 128-row tile; grouped launches whose groups
         # average under 2048 stacked rows run 128-row tiles on single CTAs
         grouped_single = grouped and Mb < 2048 * spec.groups
-        t_kernel = "gemm_mxf4_fused_kernel" if fused else (
+        # (fused: CTA pairs with the quantizer in their epilogue warps beyond 128 rows)
+        t_kernel = ("gemm_mxf4_pair_kernel" if M > 128 else "gemm_mxf4_fused_kernel") if fused else (
             "gemm_mxf4_kernel" if M <= 128 or grouped_single else "gemm_mxf4_pair_kernel")
     if hif4:
         aq_bytes = _act_quant_bytes(Mb, K, "hif4", not no_res, operand=not quant_only)
@@ -713,7 +717,8 @@ def run_rfq(args):
         gemm_tflops = flop / (g_ms * 1e-3) / 1e12
         roofline = {"bound": "tensor", "kernel": t_kernel, "achieved": gemm_tflops, "peak": t_peak,
                     "unit": "TFLOP/s", "frac": gemm_tflops / t_peak,
-                    "traffic": _kernel_traffic(t_kernel, spec.name + ("+" + scheme if f8 else "")
+                    "traffic": _kernel_traffic(t_kernel, spec.name + ("+fused" if fused else "")
+                                               + ("+" + scheme if f8 else "")
                                                + ("+phi" if amax_phi else "")
                                                + ("+w4a4" if no_res and not f8 else "")),
                     "flop_per_launch": flop, "ms_per_launch": g_ms,

@@ -228,19 +228,34 @@ RFQ_API rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, cons
                       int32_t phi_r_s, const rfq_qtensor *wq, void *y, int32_t out_dtype,
                       void *workspace, void *stream);
 
+/* Workspace bytes rfq_linear_fused needs for an M x K activation and the
+ * fallback mode fb (NULL = RFQ_FALLBACK_ALL); 0 for sizes it rejects
+ * (K % 128 != 0).  For M <= 128 it is rfq_linear_workspace_bytes(); beyond,
+ * it adds the kernel's unit counters and scratch for the quantized X:
+ * about M K bytes of codes and M K / 16 of scales with the residual (half
+ * of each without). */
+RFQ_API size_t rfq_linear_fused_workspace_bytes(int64_t M, int64_t K, const rfq_fallback *fb);
+
 /* RFQ linear layer with the activation quantizer fused into the GEMM (the
  * on-the-fly residual of Sec. 4.3): Y = Q(X) W~ + phi Q(X - Q(X)) W~ with X
- * read as bf16 and quantized inside the GEMM, block by block, exactly as
- * rfq_quantize_act would (MXFP4: E8M0 scale floor(log2 amax) - 2, RNE
- * saturating E2M1 codes, exact residual) -- no quantized copy of X is
- * written to memory.  x_bf16: device bf16 [M][K] row-major (16-byte
- * aligned).  wq: MXFP4 weight [N x K] with RFQ_SCALE_MMA scales.
- * fb: NULL or mode RFQ_FALLBACK_ALL (residual on every block) or
- * RFQ_FALLBACK_NONE (plain W4A4); RFQ_FALLBACK_AMAX returns
- * RFQ_ERR_UNSUPPORTED.  K % 128 == 0, N % 16 == 0, M >= 0.  y, out_dtype,
- * workspace: as for rfq_linear.  Each output tile quantizes its 128 rows of
- * X again, so this variant pays off for narrow layers (N of a few tiles of
- * 256); for wide ones rfq_quantize_act + rfq_linear is faster.
+ * read as bf16 and quantized inside the GEMM kernel, block by block, exactly
+ * as rfq_quantize_act would (MXFP4: E8M0 scale floor(log2 amax) - 2, RNE
+ * saturating E2M1 codes, exact residual): one launch, no separate
+ * quantizer pass.  x_bf16: device bf16 [M][K] row-major (16-byte aligned).
+ * wq: MXFP4 weight [N x K] with RFQ_SCALE_MMA scales.  fb: NULL or mode
+ * RFQ_FALLBACK_ALL (residual on every block) or RFQ_FALLBACK_NONE (plain
+ * W4A4); RFQ_FALLBACK_AMAX returns RFQ_ERR_UNSUPPORTED.  K % 128 == 0,
+ * N % 16 == 0, M >= 0.  y, out_dtype: as for rfq_linear.
+ * workspace: device, rfq_linear_fused_workspace_bytes(M, K, fb) bytes,
+ * 16-byte aligned, zeroed by the caller once; its first 256 bytes are the
+ * GEMM workspace of rfq_linear (status word, wait limit, held start).  For
+ * M > 128 the GEMM runs on CTA pairs whose epilogue warps, between output
+ * tiles, quantize X in units of 8 rows x 256 columns into the rest of the
+ * workspace, each element once; a stage's copies wait (bounded) until its
+ * rows are quantized, and the kernel leaves its unit counters zero for the
+ * next call.  Calls that overlap on the GPU must not share a workspace.
+ * For M <= 128 each output tile quantizes its rows of X itself in shared
+ * memory (one row tile, so nothing is repeated across row tiles).
  * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
  * RFQ_ERR_UNSUPPORTED, RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */
 RFQ_API rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, const rfq_qtensor *wq,

@@ -410,6 +410,49 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
     return from_cuda(launch_gemm_mxf4(a, st));
 }
 
+} // extern "C"
+
+namespace {
+// Workspace of rfq_linear_fused.  M <= 128 (the single-CTA fused kernel):
+// the 256-byte GEMM workspace.  M > 128 (the CTA-pair kernel with its
+// quantizer): the GEMM workspace, the unit counters (2 + T + T S words for T
+// 128-row tiles and S 256-element k-stages), then, each 1024-byte aligned,
+// the scratch codes of X~ [M][K/2], of X^ [M][K/2] (with a residual), and
+// their MMA-layout scales [ceil(M/128) 128][K/32].
+struct FusedLayout {
+    size_t ctr, mcodes, rcodes, msf, rsf, total;
+};
+
+FusedLayout fused_layout(int64_t M, int64_t K, bool res)
+{
+    auto up = [](size_t v) { return (v + 1023) & ~size_t(1023); };
+    FusedLayout L = {};
+    const size_t base = rfq_linear_workspace_bytes();
+    if (M <= 128) {
+        L.total = base;
+        return L;
+    }
+    const size_t tiles = (size_t)((M + 127) / 128), stages = (size_t)((K / 128 + 1) / 2);
+    const size_t codes = (size_t)M * (size_t)(K / 2), sf = tiles * 128 * (size_t)(K / 32);
+    L.ctr = base;
+    L.mcodes = up(L.ctr + 4 * (2 + tiles + tiles * stages));
+    L.rcodes = up(L.mcodes + codes);
+    L.msf = up(L.rcodes + (res ? codes : 0));
+    L.rsf = up(L.msf + sf);
+    L.total = up(L.rsf + (res ? sf : 0));
+    return L;
+}
+} // namespace
+
+extern "C" {
+
+size_t rfq_linear_fused_workspace_bytes(int64_t M, int64_t K, const rfq_fallback *fb)
+{
+    if (M < 0 || K <= 0 || K % 128 != 0)
+        return 0;
+    return fused_layout(M, K, !fb || fb->mode != RFQ_FALLBACK_NONE).total;
+}
+
 rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, const rfq_qtensor *wq,
                             const rfq_fallback *fb, void *y, int32_t out_dtype, void *workspace, void *stream)
 {
@@ -440,6 +483,30 @@ rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, const rfq_
         return s;
     if (M == 0 || N == 0)
         return RFQ_OK;
+    if (M > 128) {
+        // CTA pairs, X quantized once into the workspace's scratch by the GEMM's own warps
+        const bool res = mode == RFQ_FALLBACK_ALL;
+        const FusedLayout L = fused_layout(M, K, res);
+        uint8_t *w = static_cast<uint8_t *>(workspace);
+        GemmMxf4Args a;
+        a.a_codes = w + L.mcodes;
+        a.a_sf = w + L.msf;
+        a.r_codes = res ? w + L.rcodes : nullptr;
+        a.r_sf = res ? w + L.rsf : nullptr;
+        a.b_codes = wq->codes;
+        a.b_sf = wq->scales;
+        a.phi = nullptr;
+        a.phi_r_s = 0;
+        a.y = y;
+        a.out_bf16 = out_dtype == RFQ_OUT_BF16;
+        a.M = M;
+        a.N = N;
+        a.K = K;
+        a.status = static_cast<int32_t *>(workspace);
+        a.fq_x = x_bf16;
+        a.fq_ctr = reinterpret_cast<int32_t *>(w + L.ctr);
+        return from_cuda(launch_gemm_mxf4_pair(a, static_cast<cudaStream_t>(stream)));
+    }
     GemmFusedArgs a;
     a.x = x_bf16;
     a.b_codes = wq->codes;

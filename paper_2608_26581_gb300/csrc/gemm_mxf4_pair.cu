@@ -63,6 +63,7 @@
 #include <cstdint>
 
 #include "internal.h"
+#include "mxfp4_math.cuh"
 #include "ptx.cuh"
 
 namespace rfq {
@@ -87,6 +88,10 @@ constexpr int PHI_WARP = THREADS / 32;   // the phi reader: one warp beyond THRE
 constexpr int REC_WORDS = 64;            // phi record: up to 2048 full k-stages (K <= 524288)
 constexpr int GRP_MAX = 128;             // groups of the grouped GEMM
 constexpr int YSTAGE = 2048;             // per epilogue warp: 32 rows x 64 bytes of Y
+constexpr int FQ_ROWS = 8;               // fused quantizer: rows of X per conversion unit
+constexpr int FQ_SUB = BM / FQ_ROWS;     // units per (128-row tile, k-stage)
+constexpr int FQ_CALL = 4;               // rows quantized per step of a converting warp (loads in flight)
+static_assert(FQ_ROWS % FQ_CALL == 0, "whole steps per unit");
 static_assert(SF_COL0 + SF_SLOTS * SF_SLOT_COLS <= TMEM_COLS, "TMEM budget");
 static_assert(SF_SLOTS >= STAGES, "a scale slot is rewritten only after its stage's MMAs completed");
 
@@ -127,11 +132,32 @@ struct Smem {
     int32_t grp_pairs[GRP_MAX + 1]; // grouped GEMM: 256-row pairs of the groups before each group
     int32_t grp_bad;                // grouped GEMM: the row offsets break the contract
     uint32_t tmem_base;
+    int32_t fq_last;              // fused quantizer: this CTA is the grid's last to finish
     uint64_t wait_ns;             // limit of the bounded waits (workspace word 1, else wl)
     int32_t abort_flag;
 };
 constexpr size_t kSmemBytes = sizeof(Smem) + 1024;
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+
+// Fused quantizer (FQ): the activation quantizer of Sec. 4.3 (X~ = Q(X), the
+// residual dX = X - X~ and X^ = Q(dX), per 32-element block along K) runs
+// inside the GEMM.  X is cut into units of FQ_ROWS rows x one k-stage (256
+// columns, or the odd last 128); the epilogue warps, between draining
+// accumulators, take units in order from a global counter, quantize them
+// into a scratch copy of the codes and MMA-layout scales (the layout the
+// quantizer kernel writes), and count each finished unit for its (128-row
+// tile, k-stage).  The producer issues a stage's A / R copies once that
+// count is complete.  Every element of X is quantized once, however many
+// output tiles read it; the tile walk is row-block major, so the codes are
+// read back while they are still in L2.  The grid's last CTA to finish
+// zeroes the counters for the next call.
+struct FqArgs {
+    const uint4 *x;               // bf16 X [M][K], 8 elements per uint4
+    uint32_t *mcodes, *rcodes;    // scratch codes [M][K/8] words (X~, X^)
+    uint8_t *msf, *rsf;           // scratch scales, MMA layout (rows padded to 128)
+    int32_t *ctr;                 // [0] next unit, [1] CTAs finished, [2, 2 + m_tiles) units done per
+                                  // 128-row tile, then [m_tiles][k-stages] units done per (tile, stage)
+};
 
 __device__ __forceinline__ void flag_timeout(Smem &S, int32_t *status)
 {
@@ -161,15 +187,17 @@ struct Mask {
 // GRP: the grouped (mixture-of-experts) form, G groups of rows with their
 // own W~ (row offsets read on the device); the plain form is compiled
 // without any of it.
-template <bool RES, bool PHI, bool OUT_BF16, bool F8, bool GRP>
+// FQ: the fused quantizer above (MXFP4 operands, no phi records, no groups).
+template <bool RES, bool PHI, bool OUT_BF16, bool F8, bool GRP, bool FQ = false>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     gemm_mxf4_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmR,
                           const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmY,
                           const uint8_t *__restrict__ sfa, const uint8_t *__restrict__ sfr,
                           const uint8_t *__restrict__ sfb, const uint8_t *__restrict__ phi, int phi_chunks,
                           int phi_cols, int M, int N, int K, int32_t *status,
-                          const int32_t *__restrict__ group_off, int G, void *__restrict__ y)
+                          const int32_t *__restrict__ group_off, int G, void *__restrict__ y, const FqArgs fq)
 {
+    static_assert(!FQ || (!PHI && !F8 && !GRP), "the fused quantizer takes plain MXFP4 operands");
     extern __shared__ uint8_t smem_raw[];
     Smem &S = *reinterpret_cast<Smem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -302,6 +330,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
             const uint32_t full0 = mapa_shared(smem_u32(&S.full[0]), 0);   // the even CTA's barriers
             int p = 0, it = 0;
             bool stop = false;
+            int fq_tile_ok = -1;   // FQ: a 128-row tile whose every unit is quantized
             if (!held_start_wait(status, wl)) { // a test-held start never opened
                 flag_timeout(S, status);
                 stop = true;
@@ -323,6 +352,32 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                         flag_timeout(S, status);
                         stop = true;
                         return;
+                    }
+                    if constexpr (FQ) {
+                        // the stage's rows of X quantized (every unit of this 128-row
+                        // tile and k-stage counted, or the whole tile): acquire the
+                        // counts, then order the TMA reads after them
+                        if (rows_in && fq_tile_ok != m_tile) {
+                            const int32_t *dn = fq.ctr + 2 + m_tile;
+                            const int32_t *fl = fq.ctr + 2 + m_tiles + (int64_t)m_tile * nks + ks;
+                            const uint64_t t0 = globaltimer_ns();
+                            for (uint32_t i = 0;; ++i) {
+                                const int32_t a = ld_acquire_gpu(dn), b = ld_acquire_gpu(fl);
+                                if (a == nks * FQ_SUB) {
+                                    fq_tile_ok = m_tile;
+                                    break;
+                                }
+                                if (b == FQ_SUB)
+                                    break;
+                                if ((i & 15) == 15 && (globaltimer_ns() - t0 > wl || *gstat != 0)) {
+                                    flag_timeout(S, status);
+                                    stop = true;
+                                    return;
+                                }
+                                __nanosleep(128);
+                            }
+                            fence_proxy_async_global();
+                        }
                     }
                     const int c0 = CPS * ks, cx = c0 * (F8 ? 128 : 64); // first chunk, its byte column
                     if (PHI)
@@ -492,10 +547,107 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
         const uint32_t acc_empty_lead = mapa_shared(smem_u32(&S.acc_empty), 0);
         uint8_t *stg = S.ystage + (warp - 2) * YSTAGE;
         const uint32_t sw = (uint32_t)((lane >> 1) & 3);   // 64B swizzle: chunk j of row r at (j ^ ((r >> 1) & 3))
+        // FQ: the conversion unit this warp holds (-1: none) and its next row
+        int fq_u = -1, fq_row = 0;
+        bool fq_done = !FQ;
+        const int fq_units = m_tiles * nks * FQ_SUB;
+        // FQ_CALL rows of the held unit (taking the next unit first if none is
+        // held): lane l quantizes elements 8 l .. 8 l + 7 of the stage's
+        // columns (Sec. 3.2 Eq. 3-4 and the residual of Sec. 4.3, the
+        // quantizer kernel's arithmetic), stores its code words, and the
+        // E8M0 bytes go out as one 32-bit word per row and 128-element chunk
+        // (bytes 4 (row % 128 / 32) .. + 3 of the row's 16 in the scale atom)
+        auto fq_rows = [&]() {
+            if constexpr (FQ) {
+                if (fq_u < 0) {
+                    int u = 0;
+                    if (lane == 0)
+                        u = atomicAdd(fq.ctr, 1);
+                    u = __shfl_sync(0xffffffffu, u, 0);
+                    if (u >= fq_units) {
+                        fq_done = true;
+                        return;
+                    }
+                    fq_u = u;
+                    fq_row = 0;
+                }
+                const int t = fq_u / FQ_SUB, sub = fq_u - t * FQ_SUB;   // t: (128-row tile, k-stage)
+                const int mt = t / nks, ks = t - mt * nks;
+                const int kw = K >> 3;                                  // 8-element words per row
+                const int c8 = ks * 32 + lane;
+                const bool col_ok = c8 < kw;                            // (the odd last chunk: 16 lanes)
+                const int m0 = mt * BM + sub * FQ_ROWS + fq_row;
+                uint4 v[FQ_CALL];
+#pragma unroll
+                for (int r = 0; r < FQ_CALL; ++r)
+                    v[r] = (m0 + r < M && col_ok) ? __ldcs(fq.x + (int64_t)(m0 + r) * kw + c8)
+                                                  : make_uint4(0, 0, 0, 0);
+#pragma unroll
+                for (int r = 0; r < FQ_CALL; ++r) {
+                    const int m = m0 + r;
+                    float xf[8];
+                    bf16x8_to_f32(v[r], xf);
+                    const Mx8 qz = mxfp4_quant8<RES>(xf);
+                    if (m < M && col_ok) {
+                        fq.mcodes[(int64_t)m * kw + c8] = qz.code;
+                        if (RES)
+                            fq.rcodes[(int64_t)m * kw + c8] = qz.rcode;
+                    }
+                    // rows past M keep zero scale bytes (zero input), as the quantizer writes them
+                    const int sh = 8 * ((lane >> 2) & 3);
+                    uint32_t wm = (uint32_t)qz.sb << sh, wr = (uint32_t)qz.rb << sh;
+                    wm |= __shfl_xor_sync(0xffffffffu, wm, 4);
+                    wm |= __shfl_xor_sync(0xffffffffu, wm, 8);
+                    if (RES) {
+                        wr |= __shfl_xor_sync(0xffffffffu, wr, 4);
+                        wr |= __shfl_xor_sync(0xffffffffu, wr, 8);
+                    }
+                    if ((lane & 15) == 0 && col_ok) {
+                        const int64_t off = ((int64_t)(mt * kc + 2 * ks + (lane >> 4)) << 9) + ((m & 31) << 4) +
+                                            (((m >> 5) & 3) << 2);
+                        *reinterpret_cast<uint32_t *>(fq.msf + off) = wm;
+                        if (RES)
+                            *reinterpret_cast<uint32_t *>(fq.rsf + off) = wr;
+                    }
+                }
+                fq_row += FQ_CALL;
+                if (fq_row == FQ_ROWS) {
+                    // the unit's stores before its count, for the TMA reads of other SMs
+                    fence_proxy_async_global();
+                    __syncwarp();
+                    if (lane == 0) {
+                        __threadfence();
+                        atomicAdd(fq.ctr + 2 + m_tiles + t, 1);
+                        atomicAdd(fq.ctr + 2 + mt, 1);
+                    }
+                    fq_u = -1;
+                }
+            }
+        };
+        // the accumulator of the warp's next tile (warp-uniform outcome: the
+        // tcgen05 loads need the whole warp); with FQ the warp quantizes
+        // while it waits
+        auto acc_wait = [&](uint32_t parity) -> bool {
+            if constexpr (!FQ) {
+                return __all_sync(0xffffffffu, mbar_wait(&S.acc_full, parity, wl, gstat));
+            } else {
+                const uint32_t a = smem_u32(&S.acc_full);
+                const uint64_t t0 = globaltimer_ns();
+                for (uint32_t i = 0;; ++i) {
+                    // (test_wait returns at once; try_wait may suspend the warp, which
+                    // would starve the conversion)
+                    if (__all_sync(0xffffffffu, fq_done ? mbar_try_wait(a, parity) : mbar_test_wait(a, parity)))
+                        return true;
+                    if (!fq_done)
+                        fq_rows();
+                    if ((i & 63) == 63 && __any_sync(0xffffffffu, globaltimer_ns() - t0 > wl || *gstat != 0))
+                        return false;
+                }
+            }
+        };
         int it = 0;
         for (int tile = pair; tile < tiles && !skip; tile += pairs, ++it) {
-            // warp-uniform outcome: the tcgen05 loads below need the whole warp
-            if (!__all_sync(0xffffffffu, mbar_wait(&S.acc_full, it & 1, wl, gstat))) {
+            if (!acc_wait(it & 1)) {
                 if (lane == 0)
                     flag_timeout(S, status);
                 break;
@@ -618,6 +770,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
             }
             if (S.abort_flag)
                 break;
+        }
+        if constexpr (FQ) {
+            // units no warp has taken yet (this CTA has no tile left)
+            bool go = !skip && S.abort_flag == 0;
+            for (uint32_t i = 0; go && !fq_done; ++i) {
+                fq_rows();
+                if ((i & 63) == 63)
+                    go = !__any_sync(0xffffffffu, *gstat != 0);
+            }
         }
         if (lane == 0)
             bulk_wait_group<0>(); // every TMA store of this warp has completed
@@ -753,13 +914,32 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
         tc_fence_after();
         tmem_dealloc_pair(tmem, TMEM_COLS);
     }
+    if constexpr (FQ) {
+        // the grid's last CTA to get here zeroes the counters for the next call
+        if (threadIdx.x == 0) {
+            __threadfence();
+            S.fq_last = atomicAdd(fq.ctr + 1, 1) == (int)gridDim.x - 1;
+        }
+        __syncthreads();
+        if (S.fq_last) {
+            const int n = 2 + m_tiles + m_tiles * nks;
+            for (int i = threadIdx.x; i < n; i += blockDim.x)
+                if (i != 1)
+                    fq.ctr[i] = 0;
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                __threadfence();
+                fq.ctr[1] = 0;
+            }
+        }
+    }
 }
 
-template <bool RES, bool PHI, bool OUT, bool F8, bool GRP>
+template <bool RES, bool PHI, bool OUT, bool F8, bool GRP, bool FQ = false>
 cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const CUtensorMap &tb,
                            const CUtensorMap &ty, const GemmMxf4Args &a, cudaStream_t st)
 {
-    auto kern = gemm_mxf4_pair_kernel<RES, PHI, OUT, F8, GRP>;
+    auto kern = gemm_mxf4_pair_kernel<RES, PHI, OUT, F8, GRP, FQ>;
     static int max_pairs = 0; // per variant: clusters of two that fit on the device at once
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (e != cudaSuccess)
@@ -781,9 +961,18 @@ cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const C
     const int grid = 2 * (int)(tiles < max_pairs ? tiles : max_pairs);
     const int phi_chunks = a.phi_r_s / 128;
     const int phi_cols = a.phi ? (int)((a.K + a.phi_r_s - 1) / a.phi_r_s) : 0;
+    FqArgs fq = {};
+    if (FQ) {
+        fq.x = static_cast<const uint4 *>(a.fq_x);
+        fq.mcodes = static_cast<uint32_t *>(const_cast<void *>(a.a_codes));
+        fq.rcodes = static_cast<uint32_t *>(const_cast<void *>(a.r_codes));
+        fq.msf = static_cast<uint8_t *>(const_cast<void *>(a.a_sf));
+        fq.rsf = static_cast<uint8_t *>(const_cast<void *>(a.r_sf));
+        fq.ctr = a.fq_ctr;
+    }
     kern<<<grid, PHI ? THREADS + 32 : THREADS, kSmemBytes, st>>>(
         ta, tr, tb, ty, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf, (const uint8_t *)a.b_sf, a.phi, phi_chunks,
-        phi_cols, (int)a.M, (int)a.N, (int)a.K, a.status, a.group_off, a.groups, a.y);
+        phi_cols, (int)a.M, (int)a.N, (int)a.K, a.status, a.group_off, a.groups, a.y, fq);
     return cudaGetLastError();
 }
 
@@ -810,6 +999,16 @@ cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
     // Beyond REC_WORDS * 32 full k-stages the record does not fit: every
     // residual product is then issued (exact: phi = 0 residuals are zero).
     const bool res = a.r_codes != nullptr;
+    if (a.fq_x) {
+        // the fused quantizer: plain MXFP4 operands written by the kernel itself
+        if (a.f8 || a.groups > 0 || a.phi)
+            return cudaErrorInvalidValue;
+        if (res)
+            return a.out_bf16 ? launch_variant<true, false, true, false, false, true>(ta, tr, tb, ty, a, st)
+                              : launch_variant<true, false, false, false, false, true>(ta, tr, tb, ty, a, st);
+        return a.out_bf16 ? launch_variant<false, false, true, false, false, true>(ta, tr, tb, ty, a, st)
+                          : launch_variant<false, false, false, false, false, true>(ta, tr, tb, ty, a, st);
+    }
     const bool phi = res && a.phi != nullptr && a.K / (a.f8 ? 128 : 256) <= REC_WORDS * 32;
 #define RFQ_GV(R, P, O)                                                                                           \
     return a.groups > 0 ? (a.f8 ? launch_variant<R, P, O, true, true>(ta, tr, tb, ty, a, st)                       \

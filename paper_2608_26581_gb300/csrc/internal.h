@@ -86,6 +86,12 @@ struct GemmMxf4Args {
     int f8 = 0;                                // every operand MXFP8 (E4M3): kind::mxf8f6f4, CTA pairs
     const int32_t *group_off = nullptr;        // grouped GEMM: device row offsets [groups + 1]
     int groups = 0;                            // grouped GEMM: N is per group, W~ has groups * N rows
+    // fused quantizer (CTA-pair kernel): bf16 X [M][K]; the kernel quantizes
+    // it into a_codes / a_sf (and r_codes / r_sf) itself, which are then
+    // scratch it writes, and counts finished units in fq_ctr (zero on entry,
+    // left zero on exit)
+    const void *fq_x = nullptr;
+    int32_t *fq_ctr = nullptr;
 };
 cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st);
 // CTA-pair kernel (gemm_mxf4_pair.cu), used by launch_gemm_mxf4 when M > 128.

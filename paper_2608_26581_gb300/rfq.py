@@ -29,7 +29,7 @@ STATUS_NAMES = {0: "RFQ_OK", 1: "RFQ_ERR_INVALID_ARG", 2: "RFQ_ERR_SHAPE", 3: "R
 EXPORTED = ("rfq_status_string", "rfq_qtensor_bytes", "rfq_quantize_weight", "rfq_quantize_act",
             "rfq_linear_workspace_bytes", "rfq_linear", "rfq_workspace_status", "rfq_dequant",
             "rfq_linear_noalloc", "rfq_linear_fused", "rfq_convert", "rfq_linear_grouped", "rfq_check_finite",
-            "rfq_quantize_act_expand", "rfq_fp4_mma_peak")
+            "rfq_quantize_act_expand", "rfq_fp4_mma_peak", "rfq_linear_fused_workspace_bytes")
 
 
 class RFQError(RuntimeError):
@@ -88,6 +88,8 @@ def load_library(path: str = LIB_PATH):
         lib.rfq_check_finite.argtypes = [P, I64, I64, P, P]
         lib.rfq_linear_grouped.restype = I32
         lib.rfq_linear_grouped.argtypes = [QTP, QTP, P, I32, P, I32, QTP, I64, P, I32, P, P]
+        lib.rfq_linear_fused_workspace_bytes.restype = SZ
+        lib.rfq_linear_fused_workspace_bytes.argtypes = [I64, I64, ctypes.POINTER(_FB)]
         lib.rfq_fp4_mma_peak.restype = I32
         lib.rfq_fp4_mma_peak.argtypes = [I32, I64, P, ctypes.POINTER(ctypes.c_double), P]
         _lib = lib
@@ -255,12 +257,26 @@ def rfq_linear_noalloc(xq: QTensor, xr: QTensor | None, phi: torch.Tensor | None
                                              _stream(stream)), "rfq_linear_noalloc")
 
 
+def rfq_linear_fused_workspace_bytes(M: int, K: int, mode: int = RFQ_FALLBACK_ALL) -> int:
+    fb = _FB(mode, 0.0, 128, 256)
+    return load_library().rfq_linear_fused_workspace_bytes(M, K, ctypes.byref(fb))
+
+
+def fused_workspace(M: int, K: int, mode: int = RFQ_FALLBACK_ALL, device="cuda") -> torch.Tensor:
+    """A zeroed workspace for rfq_linear_fused (int32 words)."""
+    n = rfq_linear_fused_workspace_bytes(M, K, mode)
+    return torch.zeros((n + 3) // 4, dtype=torch.int32, device=device)
+
+
 def rfq_linear_fused(x: torch.Tensor, wq: QTensor, y: torch.Tensor, out_dtype: int, workspace: torch.Tensor,
                      mode: int = RFQ_FALLBACK_ALL, stream=None):
     """Y = Q(X) W~ + phi Q(X - Q(X)) W~ with X (bf16 [M, K]) quantized inside
     the GEMM; mode RFQ_FALLBACK_ALL or RFQ_FALLBACK_NONE."""
     M, K = x.shape
     fb = _FB(mode, 0.0, 128, 256)
+    need = rfq_linear_fused_workspace_bytes(M, K, mode)
+    if workspace.numel() * workspace.element_size() < need:
+        raise ValueError(f"rfq_linear_fused needs a workspace of {need} bytes (rfq_linear_fused_workspace_bytes)")
     w = wq.c()
     _check(load_library().rfq_linear_fused(_ptr(x), M, K, ctypes.byref(w), ctypes.byref(fb), _ptr(y), out_dtype,
                                            _ptr(workspace), _stream(stream)), "rfq_linear_fused")

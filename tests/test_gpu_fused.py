@@ -1,12 +1,15 @@
 """GPU parity of rfq_linear_fused (the quantizer inside the GEMM, Sec. 4.3's
 on-the-fly residual) against the fp64 CPU oracle: Y = Q(X) W~ + Q(X - Q(X)) W~
 with the oracle's own quantization of X, and against the two-kernel path
-(rfq_quantize_act + rfq_linear), whose codes are bit-exact."""
+(rfq_quantize_act + rfq_linear), whose codes are bit-exact.  Beyond 128 rows
+the GEMM's own warps quantize X into the workspace's scratch: those codes and
+scale bytes must be the oracle's bit for bit, and the unit counters must be
+left zero for the next call."""
 import numpy as np
 import pytest
 import torch
 
-from gpu_util import DEV, check_y, to_dev_bf16
+from gpu_util import DEV, check_y, guarded_full, mma_scale_to_rowmajor, to_dev_bf16
 from paper_2608_26581_gb300 import rfq
 from paper_2608_26581_gb300.synth import WORKLOADS, ActSpec, make_activation, make_weight
 
@@ -26,12 +29,32 @@ def _weight(wb):
     return wq
 
 
-def _fused(xb, wq, out=rfq.RFQ_OUT_F32, mode=rfq.RFQ_FALLBACK_ALL):
+def _layout(M, K, res):
+    """Byte offsets inside the fused workspace (M > 128), as include/rfq.h
+    states them: the 256-byte GEMM workspace, the unit counters, then the
+    scratch codes of X~ and X^ and their MMA-layout scales, each 1024-byte
+    aligned."""
+    up = lambda v: (v + 1023) // 1024 * 1024
+    tiles, stages = -(-M // 128), (K // 128 + 1) // 2
+    codes, sf = M * K // 2, tiles * 128 * (K // 32)
+    ctr = 256
+    mc = up(ctr + 4 * (2 + tiles + tiles * stages))
+    rc = up(mc + codes)
+    ms = up(rc + (codes if res else 0))
+    rs = up(ms + sf)
+    total = up(rs + (sf if res else 0))
+    return dict(ctr=ctr, n_ctr=2 + tiles + tiles * stages, mc=mc, rc=rc, ms=ms, rs=rs, total=total, codes=codes,
+                sf=sf)
+
+
+def _fused(xb, wq, out=rfq.RFQ_OUT_F32, mode=rfq.RFQ_FALLBACK_ALL, ws=None, calls=1):
     M, K = xb.shape
-    y = torch.full((M, wq.rows), float("nan"), device=DEV,
-                   dtype=torch.float32 if out == rfq.RFQ_OUT_F32 else torch.bfloat16)
-    ws = _ws()
-    rfq.rfq_linear_fused(to_dev_bf16(xb), wq, y, out, ws, mode=mode)
+    y = guarded_full((M, wq.rows), float("nan"), torch.float32 if out == rfq.RFQ_OUT_F32 else torch.bfloat16)
+    if ws is None:
+        ws = rfq.fused_workspace(M, K, mode)
+    x = to_dev_bf16(xb)
+    for _ in range(calls):
+        rfq.rfq_linear_fused(x, wq, y, out, ws, mode=mode)
     assert rfq.rfq_workspace_status(ws) == rfq.RFQ_OK
     return y.float().cpu().numpy()
 
@@ -107,5 +130,77 @@ def test_full_size_wan_ffn_up_sampled_rows(orc):
     y = _fused(xb, _weight(wb), out=rfq.RFQ_OUT_BF16)
     rng = np.random.default_rng(1)
     rows = np.unique(np.concatenate([rng.choice(M, 10, replace=False), [0, M - 1]]))
+    check_y(y[rows], _oracle(orc, xb[rows], wb), bf16=True)
+    assert np.isfinite(y).all()
+
+
+def test_workspace_size():
+    for M, K, mode in [(1, 128, rfq.RFQ_FALLBACK_ALL), (128, 4096, rfq.RFQ_FALLBACK_NONE),
+                       (129, 384, rfq.RFQ_FALLBACK_ALL), (32760, 5120, rfq.RFQ_FALLBACK_ALL),
+                       (1000, 640, rfq.RFQ_FALLBACK_NONE)]:
+        want = rfq.rfq_linear_workspace_bytes() if M <= 128 else _layout(M, K, mode != rfq.RFQ_FALLBACK_NONE)["total"]
+        assert rfq.rfq_linear_fused_workspace_bytes(M, K, mode) == want
+    assert rfq.rfq_linear_fused_workspace_bytes(300, 96) == 0
+    small = torch.zeros(64, dtype=torch.int32, device=DEV)
+    with pytest.raises(ValueError):
+        rfq.rfq_linear_fused(torch.zeros(300, 256, dtype=torch.bfloat16, device=DEV), rfq.empty_qtensor(FMT, MMA, 16, 256),
+                             torch.zeros(300, 16, device=DEV), rfq.RFQ_OUT_F32, small)
+
+
+@pytest.mark.parametrize("M,K,mode", [(129, 384, rfq.RFQ_FALLBACK_ALL), (300, 640, rfq.RFQ_FALLBACK_ALL),
+                                      (1000, 2048, rfq.RFQ_FALLBACK_ALL), (777, 1024, rfq.RFQ_FALLBACK_NONE)])
+def test_in_gemm_quantizer_codes_are_the_oracles(orc, M, K, mode):
+    """The codes and E8M0 bytes the GEMM's warps write into the workspace are
+    the oracle's quantization of X (main and residual, every byte, padding
+    rows' scale bytes zero); the counters are zero after each of three calls
+    on the same workspace, and Y matches the oracle each time."""
+    N = 256
+    res = mode != rfq.RFQ_FALLBACK_NONE
+    xb = make_activation(ActSpec(M, K, "student_t3", chan_count=3, chan_scale=100.0, tok_count=2, tok_scale=200.0,
+                                 seed=M + K))
+    xb[3, :32] = 0                     # an all-zero block
+    xb[5, 40] = 0x8000                 # a negative zero
+    wb = make_weight(K, N, seed=M)
+    wq = _weight(wb)
+    ws = rfq.fused_workspace(M, K, mode)
+    L = _layout(M, K, res)
+    assert ws.numel() * 4 == L["total"]
+    q = orc.quantize_act(xb, orc.FMT_MXFP4, orc.PHI_ALL if res else orc.PHI_NONE)
+    wc, wsf = orc.quantize_weight(wb)
+    ref = orc.linear(orc.FMT_MXFP4, q["main_codes"], q["main_scales"], q["res_codes"] if res else None,
+                     q["res_scales"] if res else None, wc, wsf, M, K, N)
+    for call in range(3):
+        y = _fused(xb, wq, mode=mode, ws=ws)
+        check_y(y, ref)
+        b = ws.view(torch.uint8).cpu().numpy()
+        assert not b[L["ctr"]:L["ctr"] + 4 * L["n_ctr"]].any(), "unit counters left non-zero"
+        mc = b[L["mc"]:L["mc"] + L["codes"]].reshape(M, K // 2)
+        assert np.array_equal(mc, q["main_codes"]), f"call {call}: main codes differ"
+        tiles = -(-M // 128)
+        ms = b[L["ms"]:L["ms"] + L["sf"]]
+        assert np.array_equal(mma_scale_to_rowmajor(ms, M, K), q["main_scales"])
+        full = mma_scale_to_rowmajor(ms, tiles * 128, K)
+        assert not full[M:].any(), "padding rows' scale bytes must be zero"
+        if res:
+            rc = b[L["rc"]:L["rc"] + L["codes"]].reshape(M, K // 2)
+            assert np.array_equal(rc, q["res_codes"]), f"call {call}: residual codes differ"
+            rs = b[L["rs"]:L["rs"] + L["sf"]]
+            assert np.array_equal(mma_scale_to_rowmajor(rs, M, K), q["res_scales"])
+            assert not mma_scale_to_rowmajor(rs, tiles * 128, K)[M:].any()
+        if call == 0:
+            # stale bytes in the scratch must not matter: every one is rewritten
+            ws.view(torch.uint8)[L["mc"]:].fill_(0x77)
+
+
+def test_many_tiles_per_pair(orc):
+    """More output tiles than CTA pairs (tiles walk in row-block order while
+    the quantizer runs ahead): rows sampled across the whole M."""
+    M, K, N = 4096, 1024, 4096
+    xb = make_activation(ActSpec(M, K, "normal", chan_count=8, chan_scale=64.0, tok_count=4, tok_scale=200.0, seed=7))
+    wb = make_weight(K, N, seed=7)
+    wq = _weight(wb)
+    y = _fused(xb, wq, out=rfq.RFQ_OUT_BF16, calls=2)
+    rng = np.random.default_rng(3)
+    rows = np.unique(np.concatenate([rng.choice(M, 24, replace=False), [0, 127, 128, 255, 256, M - 1]]))
     check_y(y[rows], _oracle(orc, xb[rows], wb), bf16=True)
     assert np.isfinite(y).all()

@@ -28,9 +28,9 @@ def _ws():
     return torch.zeros(rfq.rfq_linear_workspace_bytes() // 4, dtype=torch.int32, device=DEV)
 
 
-def _held_then_recovered(launch, y, ref, bf16=False):
+def _held_then_recovered(launch, y, ref, bf16=False, ws=None):
     # the gate stays shut: the producers' wait runs out
-    ws = _ws()
+    ws = _ws() if ws is None else ws
     ws[1] = LIMIT_US
     ws[2] = 1
     launch(ws)
@@ -125,8 +125,9 @@ def test_hif4_gemm_timeout(orc):
     _held_then_recovered(launch, y, orc.linear(orc.FMT_HIF4, mc, mm, rc, rm, wc, wm, M, K, N))
 
 
-def test_fused_gemm_timeout(orc):
-    M, K, N = 300, 512, 256
+@pytest.mark.parametrize("M", [100, 300])   # single CTA; CTA pairs quantizing into the workspace
+def test_fused_gemm_timeout(orc, M):
+    K, N = 512, 256
     xb = make_activation(ActSpec(M, K, "normal", chan_count=2, chan_scale=64.0, seed=31))
     wb = make_weight(K, N, seed=32)
     wq = rfq.empty_qtensor(F4, MMA, N, K)
@@ -138,7 +139,7 @@ def test_fused_gemm_timeout(orc):
     wc, wsf = qtensor_host(wq)
     ref = orc.linear(orc.FMT_MXFP4, q["main_codes"], q["main_scales"], q["res_codes"], q["res_scales"], wc, wsf,
                      M, K, N)
-    _held_then_recovered(launch, y, ref)
+    _held_then_recovered(launch, y, ref, ws=rfq.fused_workspace(M, K))
 
 
 @pytest.mark.parametrize("counts", [[100, 300, 0, 50], [2100, 2500]])   # single-CTA and CTA-pair forms
