@@ -552,13 +552,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
         bool fq_done = !FQ;
         const int fq_units = m_tiles * nks * FQ_SUB;
         // FQ_CALL rows of the held unit (taking the next unit first if none is
-        // held): lane l quantizes elements 8 l .. 8 l + 7 of the stage's
-        // columns (Sec. 3.2 Eq. 3-4 and the residual of Sec. 4.3, the
-        // quantizer kernel's arithmetic), stores its code words, and the
-        // E8M0 bytes go out as one 32-bit word per row and 128-element chunk
-        // (bytes 4 (row % 128 / 32) .. + 3 of the row's 16 in the scale atom)
+        // held): lane l quantizes the 32-element block l % 8 of the stage's
+        // columns in row l / 8 of the step (Sec. 3.2 Eq. 3-4 and the residual
+        // of Sec. 4.3, the quantizer kernel's arithmetic), stores its 16 bytes
+        // of codes and its E8M0 bytes into the scratch
         auto fq_rows = [&]() {
             if constexpr (FQ) {
+                static_assert(FQ_CALL * 8 == 32, "a step is one block per lane");
                 if (fq_u < 0) {
                     int u = 0;
                     if (lane == 0)
@@ -573,42 +573,40 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 }
                 const int t = fq_u / FQ_SUB, sub = fq_u - t * FQ_SUB;   // t: (128-row tile, k-stage)
                 const int mt = t / nks, ks = t - mt * nks;
-                const int kw = K >> 3;                                  // 8-element words per row
-                const int c8 = ks * 32 + lane;
-                const bool col_ok = c8 < kw;                            // (the odd last chunk: 16 lanes)
-                const int m0 = mt * BM + sub * FQ_ROWS + fq_row;
-                uint4 v[FQ_CALL];
+                const int kb = K >> 5;                                  // 32-element blocks per row
+                const int m = mt * BM + sub * FQ_ROWS + fq_row + (lane >> 3);
+                const int b = ks * 8 + (lane & 7);                      // this lane's block
+                const bool ok = m < M && b < kb;                        // (the odd last chunk: 4 blocks)
+                uint32_t w[16];
+                if (ok) {
+                    const uint4 *px = fq.x + (int64_t)m * (K >> 3) + (int64_t)b * 4;
+                    uint32_t t0[8], t1[8];
+                    ldg256_stream(px, t0);
+                    ldg256_stream(px + 2, t1);
 #pragma unroll
-                for (int r = 0; r < FQ_CALL; ++r)
-                    v[r] = (m0 + r < M && col_ok) ? __ldcs(fq.x + (int64_t)(m0 + r) * kw + c8)
-                                                  : make_uint4(0, 0, 0, 0);
+                    for (int i = 0; i < 8; ++i) {
+                        w[i] = t0[i];
+                        w[8 + i] = t1[i];
+                    }
+                } else {
 #pragma unroll
-                for (int r = 0; r < FQ_CALL; ++r) {
-                    const int m = m0 + r;
-                    float xf[8];
-                    bf16x8_to_f32(v[r], xf);
-                    const Mx8 qz = mxfp4_quant8<RES>(xf);
-                    if (m < M && col_ok) {
-                        fq.mcodes[(int64_t)m * kw + c8] = qz.code;
-                        if (RES)
-                            fq.rcodes[(int64_t)m * kw + c8] = qz.rcode;
-                    }
-                    // rows past M keep zero scale bytes (zero input), as the quantizer writes them
-                    const int sh = 8 * ((lane >> 2) & 3);
-                    uint32_t wm = (uint32_t)qz.sb << sh, wr = (uint32_t)qz.rb << sh;
-                    wm |= __shfl_xor_sync(0xffffffffu, wm, 4);
-                    wm |= __shfl_xor_sync(0xffffffffu, wm, 8);
-                    if (RES) {
-                        wr |= __shfl_xor_sync(0xffffffffu, wr, 4);
-                        wr |= __shfl_xor_sync(0xffffffffu, wr, 8);
-                    }
-                    if ((lane & 15) == 0 && col_ok) {
-                        const int64_t off = ((int64_t)(mt * kc + 2 * ks + (lane >> 4)) << 9) + ((m & 31) << 4) +
-                                            (((m >> 5) & 3) << 2);
-                        *reinterpret_cast<uint32_t *>(fq.msf + off) = wm;
-                        if (RES)
-                            *reinterpret_cast<uint32_t *>(fq.rsf + off) = wr;
-                    }
+                    for (int i = 0; i < 16; ++i)
+                        w[i] = 0;
+                }
+                float xf[32];
+                bf16x32_to_f32(w, xf);
+                const Mx32 qz = mxfp4_quant32<RES>(xf);
+                if (ok) {
+                    reinterpret_cast<uint4 *>(fq.mcodes)[(int64_t)m * kb + b] = qz.code;
+                    if (RES)
+                        reinterpret_cast<uint4 *>(fq.rcodes)[(int64_t)m * kb + b] = qz.rcode;
+                }
+                // rows past M keep zero scale bytes (zero input), as the quantizer writes them
+                if (b < kb) {
+                    const int64_t off = sf_mma_offset(m, b, kc);
+                    fq.msf[off] = (uint8_t)qz.sb;
+                    if (RES)
+                        fq.rsf[off] = (uint8_t)qz.rb;
                 }
                 fq_row += FQ_CALL;
                 if (fq_row == FQ_ROWS) {

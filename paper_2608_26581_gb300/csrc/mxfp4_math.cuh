@@ -1,7 +1,10 @@
 // mxfp4_math.cuh -- per-lane MXFP4 quantization arithmetic (Sec. 3.2 Eq. 3-4,
-// Sec. 4.3), shared by the activation quantizer and the fused-prologue GEMM.
+// Sec. 4.3), shared by the activation quantizers and the GEMMs that quantize
+// X themselves.
 //
-// Four consecutive lanes hold one 32-element block, eight elements each.
+// Two arrangements: four consecutive lanes hold one 32-element block, eight
+// elements each (mxfp4_quant8), or one lane holds a whole block
+// (mxfp4_quant32: no shuffles, the block's scale computed once).
 // The E8M0 byte is the fp32 exponent field of the block's amax minus 2 (OCP
 // rule floor(log2 amax) - 2, clamped at 0), every scaling is by a power of
 // two, the E2M1 conversion rounds to nearest even and saturates, and the
@@ -177,6 +180,93 @@ __device__ __forceinline__ Mx8 mxfp4_quant8(const float (&xf)[8])
     if (RES)
         mxfp4_resid8(xf, o.code, o.sb, o.rcode, o.rb);
     return o;
+}
+
+// ---- one lane per 32-element block
+
+// 256-bit load of global memory that is read once (not kept in L1).
+__device__ __forceinline__ void ldg256_stream(const void *p, uint32_t (&r)[8])
+{
+    asm volatile("ld.global.nc.L1::no_allocate.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                 : "l"(p));
+}
+
+// max |v_i| over 32 values (NaN elements dropped)
+__device__ __forceinline__ float absmax32(const float (&v)[32])
+{
+    float m[11];
+#pragma unroll
+    for (int i = 0; i < 10; ++i)
+        m[i] = fmax3(fabsf(v[3 * i]), fabsf(v[3 * i + 1]), fabsf(v[3 * i + 2]));
+    m[10] = fmaxf(fabsf(v[30]), fabsf(v[31]));
+    const float a = fmax3(m[0], m[1], m[2]), b = fmax3(m[3], m[4], m[5]), c = fmax3(m[6], m[7], m[8]);
+    return fmax3(fmax3(a, b, c), m[9], m[10]);
+}
+
+// 32 fp32 values (exact bf16 inputs) -> 32 E2M1 codes (element 2i in the
+// low nibble of byte i) scaled by 2^-(byte - 127)
+__device__ __forceinline__ uint4 e2m1x32_scaled(const float (&v)[32], int byte)
+{
+    const float inv = pow2_neg_e(byte);
+    const uint64_t inv2 = f2pack(inv, inv);
+    uint32_t c[4];
+#pragma unroll
+    for (int g = 0; g < 4; ++g) {
+        float y[8];
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            f2unpack(fmul2(f2pack(v[8 * g + 2 * i], v[8 * g + 2 * i + 1]), inv2), y[2 * i], y[2 * i + 1]);
+        c[g] = e2m1x8(y);
+    }
+    return make_uint4(c[0], c[1], c[2], c[3]);
+}
+
+// One 32-element MXFP4 block held by one lane (Sec. 3.2 Eq. 3-4; with RES
+// the residual block of Sec. 4.3): the codes and E8M0 byte of X~, and of
+// X^ = Q(X - X~).  The same arithmetic as mxfp4_quant8 on four lanes, with
+// the block maximum, the scale and the residual computed once per block.
+struct Mx32 {
+    uint4 code, rcode;
+    int sb, rb;
+};
+
+template <bool RES>
+__device__ __forceinline__ Mx32 mxfp4_quant32(const float (&xf)[32])
+{
+    Mx32 o;
+    o.sb = scale_byte_from_f32_bits(__float_as_uint(absmax32(xf)));
+    o.code = e2m1x32_scaled(xf, o.sb);
+    o.rcode = make_uint4(0, 0, 0, 0);
+    o.rb = 0;
+    if (RES) {
+        const float nsc = -pow2_e(o.sb);
+        const uint64_t nsc2 = f2pack(nsc, nsc);
+        const uint32_t cw[4] = {o.code.x, o.code.y, o.code.z, o.code.w};
+        float r[32];
+#pragma unroll
+        for (int g = 0; g < 4; ++g) {
+            float q[8];
+            e2m1x8_decode(cw[g], q);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) // x - x~ (exact)
+                f2unpack(ffma2(f2pack(q[2 * i], q[2 * i + 1]), nsc2, f2pack(xf[8 * g + 2 * i], xf[8 * g + 2 * i + 1])),
+                         r[8 * g + 2 * i], r[8 * g + 2 * i + 1]);
+        }
+        o.rb = scale_byte_from_f32_bits(__float_as_uint(absmax32(r)));
+        o.rcode = e2m1x32_scaled(r, o.rb);
+    }
+    return o;
+}
+
+// 16 words of bf16 pairs -> 32 fp32 values (exact)
+__device__ __forceinline__ void bf16x32_to_f32(const uint32_t (&w)[16], float (&x)[32])
+{
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        x[2 * i] = __uint_as_float(w[i] << 16);
+        x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+    }
 }
 
 } // namespace rfq
