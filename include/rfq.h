@@ -231,9 +231,10 @@ RFQ_API rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, cons
 /* Workspace bytes rfq_linear_fused needs for an M x K activation and the
  * fallback mode fb (NULL = RFQ_FALLBACK_ALL); 0 for sizes it rejects
  * (K % 128 != 0).  For M <= 128 it is rfq_linear_workspace_bytes(); beyond,
- * it adds the kernel's unit counters and scratch for the quantized X:
- * about M K bytes of codes and M K / 16 of scales with the residual (half
- * of each without). */
+ * it adds the kernel's counters and a scratch ring for the quantized X of
+ * at most 12 blocks of 256 rows: 256 R K (1 + 1/16) bytes with the residual
+ * for R = min(12, ceil(M / 256)) (half without) -- about 17 MB for K = 5120,
+ * whatever M. */
 RFQ_API size_t rfq_linear_fused_workspace_bytes(int64_t M, int64_t K, const rfq_fallback *fb);
 
 /* RFQ linear layer with the activation quantizer fused into the GEMM (the
@@ -251,10 +252,11 @@ RFQ_API size_t rfq_linear_fused_workspace_bytes(int64_t M, int64_t K, const rfq_
  * GEMM workspace of rfq_linear (status word, wait limit, held start).  For
  * M > 128 the GEMM runs on CTA pairs whose epilogue warps, between output
  * tiles, quantize X in units of 8 rows x 256 columns into the rest of the
- * workspace, each element once; a stage's copies wait (bounded) until its
- * rows are quantized, and the kernel leaves its unit counters zero for the
- * next call.  Calls that overlap on the GPU must not share a workspace.
- * For M <= 128 each output tile quantizes its rows of X itself in shared
+ * workspace's ring, each element once; a stage's copies wait (bounded) until
+ * its rows are quantized, a block of rows is written only once every output
+ * tile has loaded the block its slot held before, and the kernel leaves its
+ * counters zero for the next call.  Calls that overlap on the GPU must not
+ * share a workspace.  For M <= 128 each output tile quantizes its rows of X itself in shared
  * memory (one row tile, so nothing is repeated across row tiles).
  * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
  * RFQ_ERR_UNSUPPORTED, RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */

@@ -415,12 +415,14 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
 namespace {
 // Workspace of rfq_linear_fused.  M <= 128 (the single-CTA fused kernel):
 // the 256-byte GEMM workspace.  M > 128 (the CTA-pair kernel with its
-// quantizer): the GEMM workspace, the unit counters (2 + T + T S words for T
-// 128-row tiles and S 256-element k-stages), then, each 1024-byte aligned,
-// the scratch codes of X~ [M][K/2], of X^ [M][K/2] (with a residual), and
-// their MMA-layout scales [ceil(M/128) 128][K/32].
+// quantizer): the GEMM workspace, the counters (2 + T + T S + P words for T
+// 128-row tiles, S 256-element k-stages and P 256-row blocks), then, each
+// 1024-byte aligned, the scratch ring of R = min(kFusedRingPairs, P) slots
+// of 256 rows: codes of X~ [256 R][K/2], of X^ [256 R][K/2] (with a
+// residual), and their MMA-layout scales [256 R][K/32].
 struct FusedLayout {
     size_t ctr, mcodes, rcodes, msf, rsf, total;
+    int ring;
 };
 
 FusedLayout fused_layout(int64_t M, int64_t K, bool res)
@@ -433,9 +435,12 @@ FusedLayout fused_layout(int64_t M, int64_t K, bool res)
         return L;
     }
     const size_t tiles = (size_t)((M + 127) / 128), stages = (size_t)((K / 128 + 1) / 2);
-    const size_t codes = (size_t)M * (size_t)(K / 2), sf = tiles * 128 * (size_t)(K / 32);
+    const size_t pairs = (size_t)((M + 255) / 256);
+    L.ring = (int)(pairs < (size_t)kFusedRingPairs ? pairs : (size_t)kFusedRingPairs);
+    const size_t rows = (size_t)L.ring * 256;
+    const size_t codes = rows * (size_t)(K / 2), sf = rows * (size_t)(K / 32);
     L.ctr = base;
-    L.mcodes = up(L.ctr + 4 * (2 + tiles + tiles * stages));
+    L.mcodes = up(L.ctr + 4 * (2 + tiles + tiles * stages + pairs));
     L.rcodes = up(L.mcodes + codes);
     L.msf = up(L.rcodes + (res ? codes : 0));
     L.rsf = up(L.msf + sf);
@@ -505,6 +510,7 @@ rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, const rfq_
         a.status = static_cast<int32_t *>(workspace);
         a.fq_x = x_bf16;
         a.fq_ctr = reinterpret_cast<int32_t *>(w + L.ctr);
+        a.fq_ring = L.ring;
         return from_cuda(launch_gemm_mxf4_pair(a, static_cast<cudaStream_t>(stream)));
     }
     GemmFusedArgs a;

@@ -148,15 +148,21 @@ static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 // quantizer kernel writes), and count each finished unit for its (128-row
 // tile, k-stage).  The producer issues a stage's A / R copies once that
 // count is complete.  Every element of X is quantized once, however many
-// output tiles read it; the tile walk is row-block major, so the codes are
-// read back while they are still in L2.  The grid's last CTA to finish
-// zeroes the counters for the next call.
+// output tiles read it.  The scratch is a ring of `ring` slots of 256 rows:
+// the rows of 256-row block p live in slot p % ring, and a converter fills
+// block p only once every output tile of block p - ring has loaded its
+// operands (counted by the MMA thread after the tile's last stage), so the
+// scratch stays in L2 (the tile walk is row-block major).  A converter never
+// blocks on a slot: it keeps its unit and goes back to its accumulator
+// wait.  The grid's last CTA to finish zeroes the counters for the next call.
 struct FqArgs {
     const uint4 *x;               // bf16 X [M][K], 8 elements per uint4
-    uint32_t *mcodes, *rcodes;    // scratch codes [M][K/8] words (X~, X^)
-    uint8_t *msf, *rsf;           // scratch scales, MMA layout (rows padded to 128)
+    uint32_t *mcodes, *rcodes;    // scratch codes [ring * 256][K/8] words (X~, X^)
+    uint8_t *msf, *rsf;           // scratch scales, MMA layout, [ring * 256] rows
     int32_t *ctr;                 // [0] next unit, [1] CTAs finished, [2, 2 + m_tiles) units done per
-                                  // 128-row tile, then [m_tiles][k-stages] units done per (tile, stage)
+                                  // 128-row tile, then [m_tiles][k-stages] units done per (tile, stage),
+                                  // then [m_pairs] output tiles that finished loading each 256-row block
+    int ring;                     // slots of 256 rows in the scratch
 };
 
 __device__ __forceinline__ void flag_timeout(Smem &S, int32_t *status)
@@ -340,6 +346,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 const int a_row = tc.a_row0 + (int)rank * BM;   // this CTA's first A row
                 const int m_tile = a_row / BM;
                 const bool rows_in = a_row < tc.row_end;
+                // FQ: the ring slot holding these rows (rows past M: a box past the ring, zero fill)
+                const int fq_slot = FQ ? (tc.a_row0 >> 8) % fq.ring : 0;
+                const int a_y = !FQ ? a_row : rows_in ? fq_slot * 2 * BM + (int)rank * BM : fq.ring * 2 * BM;
+                const int sf_tile = FQ ? fq_slot * 2 + (int)rank : m_tile;
                 const int atom0 = tc.w_row0 >> 7;
                 const int nb = atom0 + 1 < tc.wa_end ? 2 : 1;
                 // one k-stage: wait for its ring slot, publish the tile's info,
@@ -388,15 +398,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     uint64_t *sbar = &S.sf_full[slot];
                     if (lead)
                         mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES + B_BYTES + (res_on ? A_BYTES : 0)));
-                    tma_load_2d_pair(st.a, &tmA, bar, cx, a_row);
+                    tma_load_2d_pair(st.a, &tmA, bar, cx, a_y);
                     if (res_on)
-                        tma_load_2d_pair(st.r, &tmR, bar, cx, a_row);
+                        tma_load_2d_pair(st.r, &tmR, bar, cx, a_y);
                     tma_load_2d_pair(st.b, &tmB, bar, cx, tc.w_row0 + (int)rank * BN_HALF);
                     mbar_arrive_expect_tx(sbar, nb * sfbytes + (rows_in ? (res_on ? 2 : 1) * sfbytes : 0));
                     if (rows_in) {
-                        bulk_load(st.sfa, sfa + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, sbar);
+                        bulk_load(st.sfa, sfa + ((int64_t)sf_tile * kc + c0) * ATOM, sfbytes, sbar);
                         if (res_on)
-                            bulk_load(st.sfr, sfr + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, sbar);
+                            bulk_load(st.sfr, sfr + ((int64_t)sf_tile * kc + c0) * ATOM, sfbytes, sbar);
                     }
                     for (int h = 0; h < nb; ++h)
                         bulk_load(st.sfb + h * 2 * ATOM, sfb + ((int64_t)(atom0 + h) * kc + c0) * ATOM, sfbytes,
@@ -512,6 +522,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                         mma_stage(ks, CPS, Mask<RES ? 3u : 0u>{});
                     if (nf < nks && !stop)
                         mma_stage(nf, 1, Mask<RES ? 1u : 0u>{});
+                    if constexpr (FQ) {
+                        // every stage of the tile landed (both CTAs' codes and scale
+                        // atoms): its 256-row block's ring slot has one reader fewer
+                        if (!stop)
+                            red_release_add_gpu(fq.ctr + 2 + m_tiles + m_tiles * nks + tile / n_tiles, 1);
+                    }
                 } else {
                     // the tile's residual-stage count arrives with its first stage
                     if (!mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, wl, gstat)) {
@@ -548,15 +564,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
         uint8_t *stg = S.ystage + (warp - 2) * YSTAGE;
         const uint32_t sw = (uint32_t)((lane >> 1) & 3);   // 64B swizzle: chunk j of row r at (j ^ ((r >> 1) & 3))
         // FQ: the conversion unit this warp holds (-1: none) and its next row
-        int fq_u = -1, fq_row = 0;
+        int fq_u = -1, fq_row = 0, fq_free = -1;   // fq_free: a 256-row block whose ring slot is free
         bool fq_done = !FQ;
         const int fq_units = m_tiles * nks * FQ_SUB;
         // FQ_CALL rows of the held unit (taking the next unit first if none is
         // held): lane l quantizes the 32-element block l % 8 of the stage's
         // columns in row l / 8 of the step (Sec. 3.2 Eq. 3-4 and the residual
         // of Sec. 4.3, the quantizer kernel's arithmetic), stores its 16 bytes
-        // of codes and its E8M0 bytes into the scratch
-        auto fq_rows = [&]() {
+        // of codes and its E8M0 bytes into the scratch.  Returns false when
+        // the unit's ring slot is still being read (nothing done).
+        auto fq_rows = [&]() -> bool {
             if constexpr (FQ) {
                 static_assert(FQ_CALL * 8 == 32, "a step is one block per lane");
                 if (fq_u < 0) {
@@ -566,15 +583,27 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     u = __shfl_sync(0xffffffffu, u, 0);
                     if (u >= fq_units) {
                         fq_done = true;
-                        return;
+                        return true;
                     }
                     fq_u = u;
                     fq_row = 0;
                 }
                 const int t = fq_u / FQ_SUB, sub = fq_u - t * FQ_SUB;   // t: (128-row tile, k-stage)
                 const int mt = t / nks, ks = t - mt * nks;
+                const int mp = mt >> 1;                                 // 256-row block
+                if (mp >= fq.ring && fq_free != mp) {
+                    // the slot's previous block: every output tile has loaded it?
+                    int ok = 0;
+                    if (lane == 0)
+                        ok = ld_acquire_gpu(fq.ctr + 2 + m_tiles + m_tiles * nks + (mp - fq.ring)) == n_tiles;
+                    if (!__shfl_sync(0xffffffffu, ok, 0))
+                        return false;   // keep the unit, try again later
+                    fence_proxy_async_global();
+                    fq_free = mp;
+                }
                 const int kb = K >> 5;                                  // 32-element blocks per row
                 const int m = mt * BM + sub * FQ_ROWS + fq_row + (lane >> 3);
+                const int mr = (mp % fq.ring) * 2 * BM + (m & (2 * BM - 1));   // its row in the ring
                 const int b = ks * 8 + (lane & 7);                      // this lane's block
                 const bool ok = m < M && b < kb;                        // (the odd last chunk: 4 blocks)
                 uint32_t w[16];
@@ -596,14 +625,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 float xf[32];
                 bf16x32_to_f32(w, xf);
                 const Mx32 qz = mxfp4_quant32<RES>(xf);
-                if (ok) {
-                    reinterpret_cast<uint4 *>(fq.mcodes)[(int64_t)m * kb + b] = qz.code;
-                    if (RES)
-                        reinterpret_cast<uint4 *>(fq.rcodes)[(int64_t)m * kb + b] = qz.rcode;
-                }
-                // rows past M keep zero scale bytes (zero input), as the quantizer writes them
+                // rows past M get zero codes and scale bytes (zero input)
                 if (b < kb) {
-                    const int64_t off = sf_mma_offset(m, b, kc);
+                    reinterpret_cast<uint4 *>(fq.mcodes)[(int64_t)mr * kb + b] = qz.code;
+                    if (RES)
+                        reinterpret_cast<uint4 *>(fq.rcodes)[(int64_t)mr * kb + b] = qz.rcode;
+                    const int64_t off = sf_mma_offset(mr, b, kc);
                     fq.msf[off] = (uint8_t)qz.sb;
                     if (RES)
                         fq.rsf[off] = (uint8_t)qz.rb;
@@ -621,6 +648,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     fq_u = -1;
                 }
             }
+            return true;
         };
         // the accumulator of the warp's next tile (warp-uniform outcome: the
         // tcgen05 loads need the whole warp); with FQ the warp quantizes
@@ -631,13 +659,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
             } else {
                 const uint32_t a = smem_u32(&S.acc_full);
                 const uint64_t t0 = globaltimer_ns();
+                bool busy = true;   // the last conversion step did work
                 for (uint32_t i = 0;; ++i) {
-                    // (test_wait returns at once; try_wait may suspend the warp, which
-                    // would starve the conversion)
-                    if (__all_sync(0xffffffffu, fq_done ? mbar_try_wait(a, parity) : mbar_test_wait(a, parity)))
+                    // test_wait returns at once; try_wait may suspend the warp, which
+                    // would starve the conversion -- and backs off while the next
+                    // unit's ring slot is still being read
+                    const bool poll = !fq_done && busy;
+                    if (__all_sync(0xffffffffu, poll ? mbar_test_wait(a, parity) : mbar_try_wait(a, parity)))
                         return true;
                     if (!fq_done)
-                        fq_rows();
+                        busy = fq_rows();
                     if ((i & 63) == 63 && __any_sync(0xffffffffu, globaltimer_ns() - t0 > wl || *gstat != 0))
                         return false;
                 }
@@ -770,12 +801,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 break;
         }
         if constexpr (FQ) {
-            // units no warp has taken yet (this CTA has no tile left)
+            // units no warp has taken yet (this CTA has no tile left); a unit
+            // whose ring slot is still being read waits here, bounded
             bool go = !skip && S.abort_flag == 0;
+            const uint64_t t0 = globaltimer_ns();
             for (uint32_t i = 0; go && !fq_done; ++i) {
-                fq_rows();
-                if ((i & 63) == 63)
+                if (!fq_rows())
+                    __nanosleep(2000);
+                if ((i & 63) == 63) {
+                    if (__any_sync(0xffffffffu, globaltimer_ns() - t0 > wl)) {
+                        if (lane == 0)
+                            flag_timeout(S, status);
+                        break;
+                    }
                     go = !__any_sync(0xffffffffu, *gstat != 0);
+                }
             }
         }
         if (lane == 0)
@@ -920,7 +960,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
         }
         __syncthreads();
         if (S.fq_last) {
-            const int n = 2 + m_tiles + m_tiles * nks;
+            const int n = 2 + m_tiles + m_tiles * nks + m_pairs;
             for (int i = threadIdx.x; i < n; i += blockDim.x)
                 if (i != 1)
                     fq.ctr[i] = 0;
@@ -967,6 +1007,7 @@ cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const C
         fq.msf = static_cast<uint8_t *>(const_cast<void *>(a.a_sf));
         fq.rsf = static_cast<uint8_t *>(const_cast<void *>(a.r_sf));
         fq.ctr = a.fq_ctr;
+        fq.ring = a.fq_ring;
     }
     kern<<<grid, PHI ? THREADS + 32 : THREADS, kSmemBytes, st>>>(
         ta, tr, tb, ty, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf, (const uint8_t *)a.b_sf, a.phi, phi_chunks,
@@ -981,11 +1022,12 @@ cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
     CUtensorMap ta, tr, tb, ty;
     const uint64_t kb = a.f8 ? (uint64_t)a.K : (uint64_t)a.K / 2; // code bytes per row
     const uint64_t w_rows = (uint64_t)a.N * (a.groups > 0 ? (uint64_t)a.groups : 1u);
-    if (!encode_tmap_2d_u8(&ta, a.a_codes, kb, (uint64_t)a.M, kb, ROW, BM, 128) ||
+    const uint64_t a_rows = a.fq_x ? (uint64_t)a.fq_ring * 2 * BM : (uint64_t)a.M;   // FQ: the ring
+    if (!encode_tmap_2d_u8(&ta, a.a_codes, kb, a_rows, kb, ROW, BM, 128) ||
         !encode_tmap_2d_u8(&tb, a.b_codes, kb, w_rows, kb, ROW, BN_HALF, 128))
         return cudaErrorInvalidValue;
     if (a.r_codes) {
-        if (!encode_tmap_2d_u8(&tr, a.r_codes, kb, (uint64_t)a.M, kb, ROW, BM, 128))
+        if (!encode_tmap_2d_u8(&tr, a.r_codes, kb, a_rows, kb, ROW, BM, 128))
             return cudaErrorInvalidValue;
     } else {
         tr = ta;

@@ -87,12 +87,16 @@ struct GemmMxf4Args {
     const int32_t *group_off = nullptr;        // grouped GEMM: device row offsets [groups + 1]
     int groups = 0;                            // grouped GEMM: N is per group, W~ has groups * N rows
     // fused quantizer (CTA-pair kernel): bf16 X [M][K]; the kernel quantizes
-    // it into a_codes / a_sf (and r_codes / r_sf) itself, which are then
-    // scratch it writes, and counts finished units in fq_ctr (zero on entry,
+    // it into a_codes / a_sf (and r_codes / r_sf) itself, a ring of fq_ring
+    // slots of 256 rows, and counts finished units in fq_ctr (zero on entry,
     // left zero on exit)
     const void *fq_x = nullptr;
     int32_t *fq_ctr = nullptr;
+    int fq_ring = 0;                           // fused quantizer: 256-row slots of the scratch ring
 };
+
+// Slots of 256 rows in the fused quantizer's scratch ring (rfq_linear_fused).
+constexpr int kFusedRingPairs = 12;
 cudaError_t launch_gemm_mxf4(const GemmMxf4Args &a, cudaStream_t st);
 // CTA-pair kernel (gemm_mxf4_pair.cu), used by launch_gemm_mxf4 when M > 128.
 cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st);

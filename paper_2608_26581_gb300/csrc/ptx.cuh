@@ -291,6 +291,13 @@ __device__ __forceinline__ int32_t ld_acquire_gpu(const int32_t *p)
     return v;
 }
 
+// Adds v to a global counter with release semantics at GPU scope, without
+// waiting for the result.
+__device__ __forceinline__ void red_release_add_gpu(int32_t *p, int32_t v)
+{
+    asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
 // ---------------------------------------------------------------- tcgen05
 
 __device__ __forceinline__ void tmem_alloc(uint32_t *dst_smem, uint32_t ncols)

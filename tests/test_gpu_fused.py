@@ -31,20 +31,23 @@ def _weight(wb):
 
 def _layout(M, K, res):
     """Byte offsets inside the fused workspace (M > 128), as include/rfq.h
-    states them: the 256-byte GEMM workspace, the unit counters, then the
-    scratch codes of X~ and X^ and their MMA-layout scales, each 1024-byte
-    aligned."""
+    states them: the 256-byte GEMM workspace, the counters, then the scratch
+    ring of R = min(12, ceil(M / 256)) slots of 256 rows -- codes of X~ and
+    X^ and their MMA-layout scales -- each 1024-byte aligned."""
     up = lambda v: (v + 1023) // 1024 * 1024
-    tiles, stages = -(-M // 128), (K // 128 + 1) // 2
-    codes, sf = M * K // 2, tiles * 128 * (K // 32)
+    tiles, stages, pairs = -(-M // 128), (K // 128 + 1) // 2, -(-M // 256)
+    ring = min(12, pairs)
+    rows = ring * 256
+    codes, sf = rows * K // 2, rows * (K // 32)
     ctr = 256
-    mc = up(ctr + 4 * (2 + tiles + tiles * stages))
+    n_ctr = 2 + tiles + tiles * stages + pairs
+    mc = up(ctr + 4 * n_ctr)
     rc = up(mc + codes)
     ms = up(rc + (codes if res else 0))
     rs = up(ms + sf)
     total = up(rs + (sf if res else 0))
-    return dict(ctr=ctr, n_ctr=2 + tiles + tiles * stages, mc=mc, rc=rc, ms=ms, rs=rs, total=total, codes=codes,
-                sf=sf)
+    return dict(ctr=ctr, n_ctr=n_ctr, mc=mc, rc=rc, ms=ms, rs=rs, total=total, codes=codes, sf=sf, ring=ring,
+                pairs=pairs, rows=rows)
 
 
 def _fused(xb, wq, out=rfq.RFQ_OUT_F32, mode=rfq.RFQ_FALLBACK_ALL, ws=None, calls=1):
@@ -148,12 +151,14 @@ def test_workspace_size():
 
 
 @pytest.mark.parametrize("M,K,mode", [(129, 384, rfq.RFQ_FALLBACK_ALL), (300, 640, rfq.RFQ_FALLBACK_ALL),
-                                      (1000, 2048, rfq.RFQ_FALLBACK_ALL), (777, 1024, rfq.RFQ_FALLBACK_NONE)])
+                                      (1000, 2048, rfq.RFQ_FALLBACK_ALL), (777, 1024, rfq.RFQ_FALLBACK_NONE),
+                                      (4000, 512, rfq.RFQ_FALLBACK_ALL)])   # 16 row blocks: the ring wraps
 def test_in_gemm_quantizer_codes_are_the_oracles(orc, M, K, mode):
-    """The codes and E8M0 bytes the GEMM's warps write into the workspace are
-    the oracle's quantization of X (main and residual, every byte, padding
-    rows' scale bytes zero); the counters are zero after each of three calls
-    on the same workspace, and Y matches the oracle each time."""
+    """The codes and E8M0 bytes the GEMM's warps leave in the workspace's
+    ring (slot s holds the last 256-row block b with b % R == s) are the
+    oracle's quantization of X (main and residual, every byte; rows past M
+    zero); the counters are zero after each of three calls on the same
+    workspace, and Y matches the oracle each time."""
     N = 256
     res = mode != rfq.RFQ_FALLBACK_NONE
     xb = make_activation(ActSpec(M, K, "student_t3", chan_count=3, chan_scale=100.0, tok_count=2, tok_scale=200.0,
@@ -169,24 +174,40 @@ def test_in_gemm_quantizer_codes_are_the_oracles(orc, M, K, mode):
     wc, wsf = orc.quantize_weight(wb)
     ref = orc.linear(orc.FMT_MXFP4, q["main_codes"], q["main_scales"], q["res_codes"] if res else None,
                      q["res_scales"] if res else None, wc, wsf, M, K, N)
+    # what the ring must hold: per slot, the last block written to it, zero
+    # past M; a 128-row half of a slot wholly past M is never written (the
+    # GEMM loads a zero-filled box for it), so only written rows are compared
+    rows_pad = L["pairs"] * 256
+    tiles = -(-M // 128)
+    written = np.zeros(L["rows"], bool)
+    for s_ in range(L["ring"]):
+        b_ = max(p for p in range(L["pairs"]) if p % L["ring"] == s_)
+        for h in range(2):
+            written[s_ * 256 + h * 128:s_ * 256 + (h + 1) * 128] = 2 * b_ + h < tiles
+    want = {}
+    for key in ("main", "res") if res else ("main",):
+        c = np.zeros((rows_pad, K // 2), np.uint8)
+        c[:M] = q[key + "_codes"]
+        sc = np.zeros((rows_pad, K // 32), np.uint8)
+        sc[:M] = q[key + "_scales"]
+        wc_, ws_ = np.zeros((L["rows"], K // 2), np.uint8), np.zeros((L["rows"], K // 32), np.uint8)
+        for s in range(L["ring"]):
+            b = max(p for p in range(L["pairs"]) if p % L["ring"] == s)
+            wc_[s * 256:(s + 1) * 256] = c[b * 256:(b + 1) * 256]
+            ws_[s * 256:(s + 1) * 256] = sc[b * 256:(b + 1) * 256]
+        want[key] = (wc_, ws_)
     for call in range(3):
         y = _fused(xb, wq, mode=mode, ws=ws)
         check_y(y, ref)
         b = ws.view(torch.uint8).cpu().numpy()
-        assert not b[L["ctr"]:L["ctr"] + 4 * L["n_ctr"]].any(), "unit counters left non-zero"
-        mc = b[L["mc"]:L["mc"] + L["codes"]].reshape(M, K // 2)
-        assert np.array_equal(mc, q["main_codes"]), f"call {call}: main codes differ"
-        tiles = -(-M // 128)
-        ms = b[L["ms"]:L["ms"] + L["sf"]]
-        assert np.array_equal(mma_scale_to_rowmajor(ms, M, K), q["main_scales"])
-        full = mma_scale_to_rowmajor(ms, tiles * 128, K)
-        assert not full[M:].any(), "padding rows' scale bytes must be zero"
-        if res:
-            rc = b[L["rc"]:L["rc"] + L["codes"]].reshape(M, K // 2)
-            assert np.array_equal(rc, q["res_codes"]), f"call {call}: residual codes differ"
-            rs = b[L["rs"]:L["rs"] + L["sf"]]
-            assert np.array_equal(mma_scale_to_rowmajor(rs, M, K), q["res_scales"])
-            assert not mma_scale_to_rowmajor(rs, tiles * 128, K)[M:].any()
+        assert not b[L["ctr"]:L["ctr"] + 4 * L["n_ctr"]].any(), "counters left non-zero"
+        for key, (co, so) in (("main", (L["mc"], L["ms"])), ("res", (L["rc"], L["rs"]))):
+            if key not in want:
+                continue
+            got_c = b[co:co + L["codes"]].reshape(L["rows"], K // 2)
+            assert np.array_equal(got_c[written], want[key][0][written]), f"call {call}: {key} codes differ"
+            got_s = mma_scale_to_rowmajor(b[so:so + L["sf"]], L["rows"], K)
+            assert np.array_equal(got_s[written], want[key][1][written]), f"call {call}: {key} scale bytes differ"
         if call == 0:
             # stale bytes in the scratch must not matter: every one is rewritten
             ws.view(torch.uint8)[L["mc"]:].fill_(0x77)
