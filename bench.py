@@ -597,6 +597,11 @@ def run_rfq(args):
             if mma_peak["clocks"]:
                 mma_peak["flop_per_sm_clock"] = (mma_peak["tflops"] * 1e12 / mma_peak["sms"]
                                                  / (mma_peak["clocks"]["sm_mhz"] * 1e6))
+        # where the CTA-pair GEMM's tensor pipe idles: one untimed launch of
+        # its measuring build (rfq_linear_profile) on the same operands
+        mma_prof = None
+        if (ws == 1 and not (quant_only or hif4 or f8 or fused or grouped or amax_phi or no_res) and M > 128):
+            mma_prof = _mma_profile(rfq, bufs[0], wop, K)
     ms = t_start.elapsed_time(t_end) / args.steps
     q_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in per_step)
     g_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in per_step)
@@ -727,6 +732,8 @@ def run_rfq(args):
             # against this GPU's measured MMA-only FP4 rate (the nominal 6x ratio is not reached)
             roofline["measured_fp4_mma_tflops"] = mma_peak["tflops"]
             roofline["frac_of_measured_fp4_mma"] = gemm_tflops / mma_peak["tflops"]
+        if mma_prof is not None:
+            roofline["mma_thread_profile"] = mma_prof
     clocks = clk.summary(h0, h1)
     if e2e_ms is not None:
         e2e = {"value": _job_rate(aq_bytes / 1e9 if quant_only else flop / 1e12, ws, e2e_ms), "unit": unit,
@@ -784,6 +791,26 @@ def run_rfq(args):
         print(json.dumps(line), flush=True)
     if ws > 1:
         dist.destroy_process_group()
+
+
+def _mma_profile(rfq, bs, wop, K):
+    """One launch of the CTA-pair GEMM's measuring build; per CTA pair, its
+    MMA thread's effective SM clock and the shares of its time spent waiting
+    for a drained accumulator, for operand copies and for scale words, and
+    the tensor pipe's busy share (stages x MMA cycles per stage, at the
+    32 768 FLOP per SM clock the MMA-only loop measures)."""
+    import torch
+    wsp = torch.zeros(rfq.rfq_linear_workspace_bytes() // 4, dtype=torch.int32, device=bs["x"].device)
+    c = rfq.rfq_linear_profile(bs["xq"], bs["xr"], wop, bs["y"], rfq.RFQ_OUT_BF16, wsp)
+    if rfq.rfq_workspace_status(wsp) != rfq.RFQ_OK or c["cycles"] <= 0:
+        return None
+    mma_cycles = 4.0 * K * c["tiles"]          # main + residual 256x256xK per pair, 2 SMs at 32 768 FLOP/clock
+    return {"sm_mhz_effective": c["cycles"] / c["ns"] * 1e3, "tensor_busy": mma_cycles / c["cycles"],
+            "wait_accumulator": c["wait_acc_cycles"] / c["cycles"],
+            "wait_copies": c["wait_copies_cycles"] / c["cycles"],
+            "wait_scales": c["wait_scales_cycles"] / c["cycles"],
+            "pairs": c["pairs"], "tiles": c["tiles"], "stages": c["stages"],
+            "how": "rfq_linear_profile: clock64 / globaltimer in each pair's MMA thread, one untimed launch"}
 
 
 def _fp4_mma_peak(rfq, wsp, stream, ev, iters: int = 16384, reps: int = 5):

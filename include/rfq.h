@@ -193,7 +193,8 @@ RFQ_API rfq_status rfq_quantize_act_expand(const void *x_bf16, int64_t M, int64_
  * before their first copy and record RFQ_ERR_TIMEOUT if it stays zero -- a
  * way to run a kernel's timeout path with no copy or MMA in flight.  Every
  * GEMM entry point (rfq_linear, rfq_linear_fused, rfq_linear_grouped)
- * honours words [1] to [3]; leave them zero in normal use. */
+ * honours words [1] to [3]; leave them zero in normal use.  Bytes 32..95
+ * receive rfq_linear_profile's counters. */
 RFQ_API size_t rfq_linear_workspace_bytes(void);
 
 /* RFQ GEMM (Algorithm 1, Eq. rfq): Y = X~ W~ + phi X^ W~ with both products
@@ -331,6 +332,21 @@ RFQ_API rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *st
  * RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */
 RFQ_API rfq_status rfq_fp4_mma_peak(int32_t cta_pair, int64_t iters, void *workspace, double *flop_per_launch,
                                     void *stream);
+
+/* Measurement of where the RFQ GEMM's tensor pipe idles: rfq_linear
+ * (Algorithm 1, Eq. rfq) for MXFP4 operands with a residual and no phi,
+ * M > 128 (the CTA-pair kernel), in a build of that kernel whose MMA-issuing
+ * thread (one per CTA pair) counts, from its first wait to its final drain:
+ * SM clock cycles, wall-clock nanoseconds, cycles waiting for a drained
+ * accumulator, for a stage's operand copies and for a stage's scale words,
+ * stages and tiles.  The sums over all pairs are added to the workspace's
+ * 64-bit words 4..11 (bytes 32..95) in that order, with the number of pairs
+ * in word 10: zero them before the call and read them after the stream has
+ * synchronized.  Y is computed as by rfq_linear; the counters cost a few
+ * instructions per stage, so time rfq_linear, not this call.
+ * Errors: those of rfq_linear; RFQ_ERR_UNSUPPORTED for other operand forms. */
+RFQ_API rfq_status rfq_linear_profile(const rfq_qtensor *xq, const rfq_qtensor *xr, const rfq_qtensor *wq, void *y,
+                                      int32_t out_dtype, void *workspace, void *stream);
 
 /* Allocation-free variant of rfq_linear.  The paper has no counterpart: this
  * entry point exists for callers that cannot allocate device memory, such as

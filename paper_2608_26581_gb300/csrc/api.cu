@@ -527,6 +527,34 @@ rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, const rfq_
     return from_cuda(launch_gemm_mxf4_fused(a, static_cast<cudaStream_t>(stream)));
 }
 
+rfq_status rfq_linear_profile(const rfq_qtensor *xq, const rfq_qtensor *xr, const rfq_qtensor *wq, void *y,
+                              int32_t out_dtype, void *workspace, void *stream)
+{
+    bool launch = false;
+    rfq_status s = linear_check(xq, xr, nullptr, 0, wq, y, out_dtype, workspace, &launch, true);
+    if (s != RFQ_OK || !launch)
+        return s;
+    if (!xr || xq->fmt != RFQ_FMT_MXFP4 || xq->rows <= 128)
+        return RFQ_ERR_UNSUPPORTED;
+    GemmMxf4Args a;
+    a.a_codes = xq->codes;
+    a.a_sf = xq->scales;
+    a.r_codes = xr->codes;
+    a.r_sf = xr->scales;
+    a.b_codes = wq->codes;
+    a.b_sf = wq->scales;
+    a.phi = nullptr;
+    a.phi_r_s = 0;
+    a.y = y;
+    a.out_bf16 = out_dtype == RFQ_OUT_BF16;
+    a.M = xq->rows;
+    a.N = wq->rows;
+    a.K = xq->k;
+    a.status = static_cast<int32_t *>(workspace);
+    a.prof = 1;
+    return from_cuda(launch_gemm_mxf4_pair(a, static_cast<cudaStream_t>(stream)));
+}
+
 rfq_status rfq_fp4_mma_peak(int32_t cta_pair, int64_t iters, void *workspace, double *flop_per_launch,
                             void *stream)
 {

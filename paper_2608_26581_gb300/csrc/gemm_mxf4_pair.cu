@@ -194,7 +194,12 @@ struct Mask {
 // own W~ (row offsets read on the device); the plain form is compiled
 // without any of it.
 // FQ: the fused quantizer above (MXFP4 operands, no phi records, no groups).
-template <bool RES, bool PHI, bool OUT_BF16, bool F8, bool GRP, bool FQ = false>
+// PROF: the MMA thread of each even CTA counts its SM clock cycles and
+// wall-clock nanoseconds from its first wait to its drain, the cycles it
+// waits for a drained accumulator, for a stage's copies and for a stage's
+// scale words, and its stages and tiles, and adds them to the 64-bit
+// workspace words 4..11 (a measurement of where the tensor pipe idles).
+template <bool RES, bool PHI, bool OUT_BF16, bool F8, bool GRP, bool FQ = false, bool PROF = false>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     gemm_mxf4_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmR,
                           const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmY,
@@ -469,22 +474,34 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
             // -------------------------------------------- MMA issuer (even CTA)
             int p = 0, it = 0;
             bool stop = false;
+            const int64_t c_start = PROF ? clock64() : 0;
+            const uint64_t g_start = PROF ? globaltimer_ns() : 0;
+            int64_t w_acc = 0, w_full = 0, w_sf = 0;
             for (int tile = pair; tile < tiles && !stop; tile += pairs, ++it) {
+                const int64_t ta = PROF ? clock64() : 0;
                 if (!mbar_wait<true>(&S.acc_empty, (it & 1) ^ 1, wl, gstat)) {
                     flag_timeout(S, status);
                     break;
                 }
+                if (PROF)
+                    w_acc += clock64() - ta;
                 tc_fence_after();
                 // the MMAs of the stage at position pos of the tile, with residual
                 // mask rm (bit c: chunk c's residual product) known at compile time
                 auto mma_stage = [&](int pos, int nch, auto rm_t) {
                     constexpr uint32_t rm = decltype(rm_t)::value;
                     const int slot = p % STAGES, sfs = p % SF_SLOTS;
-                    if (!mbar_wait(&S.full[slot], (p / STAGES) & 1, wl, gstat) ||
-                        !mbar_wait<true>(&S.sf_ready[sfs], (p / SF_SLOTS) & 1, wl, gstat)) {
+                    const int64_t t1 = PROF ? clock64() : 0;
+                    const bool full_ok = mbar_wait(&S.full[slot], (p / STAGES) & 1, wl, gstat);
+                    const int64_t t2 = PROF ? clock64() : 0;
+                    if (!full_ok || !mbar_wait<true>(&S.sf_ready[sfs], (p / SF_SLOTS) & 1, wl, gstat)) {
                         flag_timeout(S, status);
                         stop = true;
                         return;
+                    }
+                    if (PROF) {
+                        w_full += t2 - t1;
+                        w_sf += clock64() - t2;
                     }
                     tc_fence_after();
                     const uint32_t sf = tmem + SF_COL0 + SF_SLOT_COLS * sfs;
@@ -555,6 +572,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
             // final cluster barrier
             tc_commit_pair_mc(&S.drain, 0x1);
             (void)mbar_wait(&S.drain, 0, wl);
+            if (PROF) {
+                unsigned long long *w = reinterpret_cast<unsigned long long *>(status) + 4;
+                atomicAdd(w + 0, (unsigned long long)(clock64() - c_start));
+                atomicAdd(w + 1, (unsigned long long)(globaltimer_ns() - g_start));
+                atomicAdd(w + 2, (unsigned long long)w_acc);
+                atomicAdd(w + 3, (unsigned long long)w_full);
+                atomicAdd(w + 4, (unsigned long long)w_sf);
+                atomicAdd(w + 5, (unsigned long long)p);
+                atomicAdd(w + 6, 1ull);
+                atomicAdd(w + 7, (unsigned long long)it);
+            }
         }
     } else if (warp < 2 + EPI_WARPS) {
         // ------------------------------------------------ epilogue (warps 2..9)
@@ -973,11 +1001,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
     }
 }
 
-template <bool RES, bool PHI, bool OUT, bool F8, bool GRP, bool FQ = false>
+template <bool RES, bool PHI, bool OUT, bool F8, bool GRP, bool FQ = false, bool PROF = false>
 cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const CUtensorMap &tb,
                            const CUtensorMap &ty, const GemmMxf4Args &a, cudaStream_t st)
 {
-    auto kern = gemm_mxf4_pair_kernel<RES, PHI, OUT, F8, GRP, FQ>;
+    auto kern = gemm_mxf4_pair_kernel<RES, PHI, OUT, F8, GRP, FQ, PROF>;
     static int max_pairs = 0; // per variant: clusters of two that fit on the device at once
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (e != cudaSuccess)
@@ -1039,6 +1067,13 @@ cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
     // Beyond REC_WORDS * 32 full k-stages the record does not fit: every
     // residual product is then issued (exact: phi = 0 residuals are zero).
     const bool res = a.r_codes != nullptr;
+    if (a.prof) {
+        // the measuring instantiation: RFQ with a residual, no phi, MXFP4 operands
+        if (!res || a.f8 || a.groups > 0 || a.phi || a.fq_x)
+            return cudaErrorInvalidValue;
+        return a.out_bf16 ? launch_variant<true, false, true, false, false, false, true>(ta, tr, tb, ty, a, st)
+                          : launch_variant<true, false, false, false, false, false, true>(ta, tr, tb, ty, a, st);
+    }
     if (a.fq_x) {
         // the fused quantizer: plain MXFP4 operands written by the kernel itself
         if (a.f8 || a.groups > 0 || a.phi)

@@ -93,6 +93,7 @@ struct GemmMxf4Args {
     const void *fq_x = nullptr;
     int32_t *fq_ctr = nullptr;
     int fq_ring = 0;                           // fused quantizer: 256-row slots of the scratch ring
+    int prof = 0;                              // CTA-pair kernel: the MMA thread's counters (rfq_linear_profile)
 };
 
 // Slots of 256 rows in the fused quantizer's scratch ring (rfq_linear_fused).

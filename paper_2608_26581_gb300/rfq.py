@@ -29,7 +29,8 @@ STATUS_NAMES = {0: "RFQ_OK", 1: "RFQ_ERR_INVALID_ARG", 2: "RFQ_ERR_SHAPE", 3: "R
 EXPORTED = ("rfq_status_string", "rfq_qtensor_bytes", "rfq_quantize_weight", "rfq_quantize_act",
             "rfq_linear_workspace_bytes", "rfq_linear", "rfq_workspace_status", "rfq_dequant",
             "rfq_linear_noalloc", "rfq_linear_fused", "rfq_convert", "rfq_linear_grouped", "rfq_check_finite",
-            "rfq_quantize_act_expand", "rfq_fp4_mma_peak", "rfq_linear_fused_workspace_bytes")
+            "rfq_quantize_act_expand", "rfq_fp4_mma_peak", "rfq_linear_fused_workspace_bytes",
+            "rfq_linear_profile")
 
 
 class RFQError(RuntimeError):
@@ -90,6 +91,8 @@ def load_library(path: str = LIB_PATH):
         lib.rfq_linear_grouped.argtypes = [QTP, QTP, P, I32, P, I32, QTP, I64, P, I32, P, P]
         lib.rfq_linear_fused_workspace_bytes.restype = SZ
         lib.rfq_linear_fused_workspace_bytes.argtypes = [I64, I64, ctypes.POINTER(_FB)]
+        lib.rfq_linear_profile.restype = I32
+        lib.rfq_linear_profile.argtypes = [QTP, QTP, QTP, P, I32, P, P]
         lib.rfq_fp4_mma_peak.restype = I32
         lib.rfq_fp4_mma_peak.argtypes = [I32, I64, P, ctypes.POINTER(ctypes.c_double), P]
         _lib = lib
@@ -289,3 +292,20 @@ def rfq_fp4_mma_peak(cta_pair: bool, iters: int, workspace: torch.Tensor, stream
     _check(load_library().rfq_fp4_mma_peak(1 if cta_pair else 0, iters, _ptr(workspace), ctypes.byref(flop),
                                            _stream(stream)), "rfq_fp4_mma_peak")
     return flop.value
+
+
+PROFILE_KEYS = ("cycles", "ns", "wait_acc_cycles", "wait_copies_cycles", "wait_scales_cycles", "stages", "pairs",
+                "tiles")
+
+
+def rfq_linear_profile(xq: QTensor, xr: QTensor, wq: QTensor, y: torch.Tensor, out_dtype: int,
+                       workspace: torch.Tensor, stream=None) -> dict:
+    """rfq_linear on the CTA-pair kernel's measuring build: returns the MMA
+    threads' summed counters (see include/rfq.h); synchronizes."""
+    workspace.view(torch.uint8)[32:96].zero_()
+    q, r, w = xq.c(), xr.c(), wq.c()
+    _check(load_library().rfq_linear_profile(ctypes.byref(q), ctypes.byref(r), ctypes.byref(w), _ptr(y), out_dtype,
+                                             _ptr(workspace), _stream(stream)), "rfq_linear_profile")
+    torch.cuda.synchronize(workspace.device)
+    v = workspace.view(torch.uint8)[32:96].cpu().view(torch.int64).tolist()
+    return dict(zip(PROFILE_KEYS, v))

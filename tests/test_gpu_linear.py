@@ -193,3 +193,38 @@ def test_phi_beyond_record_capacity_falls_back_exactly(orc, M):
     rwc, rws = orc.quantize_weight(wb)
     ref = orc.linear(0, q["main_codes"], q["main_scales"], q["res_codes"], q["res_scales"], rwc, rws, M, K, N)
     check_y(y, ref)
+
+
+def test_profile_build_computes_y_and_counts_its_stages(orc):
+    """rfq_linear_profile: the CTA-pair kernel's measuring build gives the
+    same Y (oracle parity) and counters that add up: every tile and stage of
+    the grid counted once, waits within the measured cycles, a plausible SM
+    clock."""
+    M, K, N = 1000, 1280, 784
+    xb = make_activation(ActSpec(M, K, "normal", chan_count=4, chan_scale=64.0, tok_count=2, tok_scale=200.0,
+                                 seed=77))
+    wb = make_weight(K, N, seed=77)
+    x, w = to_dev_bf16(xb), to_dev_bf16(wb)
+    wq = rfq.empty_qtensor(FMT, MMA, N, K)
+    rfq.rfq_quantize_weight(w, wq)
+    xq, xr = rfq.empty_qtensor(FMT, MMA, M, K), rfq.empty_qtensor(FMT, MMA, M, K)
+    rfq.rfq_quantize_act(x, xq, xr)
+    y = guarded_full((M, N), float("nan"), torch.float32)
+    ws = _workspace()
+    c = rfq.rfq_linear_profile(xq, xr, wq, y, rfq.RFQ_OUT_F32, ws)
+    assert rfq.rfq_workspace_status(ws) == rfq.RFQ_OK
+    check_y(y.double().cpu().numpy(), _ref(orc, xq, xr, wq, M, K, N))
+    tiles = -(-N // 256) * -(-M // 256)
+    assert c["tiles"] == tiles
+    assert c["stages"] == tiles * (K // 256) + (tiles if (K // 128) % 2 else 0)
+    assert 0 < c["pairs"] <= 80
+    assert c["cycles"] > 0 and c["ns"] > 0
+    for k in ("wait_acc_cycles", "wait_copies_cycles", "wait_scales_cycles"):
+        assert 0 <= c[k] <= c["cycles"], k
+    mhz = c["cycles"] / c["ns"] * 1e3
+    assert 500 < mhz < 3000, mhz
+    # the measuring build is the CTA-pair kernel's: 128 rows or fewer are refused
+    small = rfq.empty_qtensor(FMT, MMA, 64, K)
+    with pytest.raises(rfq.RFQError) as e:
+        rfq.rfq_linear_profile(small, small, wq, torch.empty(64, N, device=DEV), rfq.RFQ_OUT_F32, ws)
+    assert e.value.status == rfq.RFQ_ERR_UNSUPPORTED
