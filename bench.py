@@ -110,7 +110,7 @@ def _src_hash(kernel: str):
     m = hashlib.sha256()
     extra = ("mxfp4_math.cuh",) if kernel in ("act_quant_mxfp4_kernel", "act_quant_mxfp4_amax_kernel",
                                               "gemm_mxf4_fused_kernel", "act_quant8_kernel",
-                                              "act_quant_rfq8_amax_kernel") else ()
+                                              "act_quant_rfq8_amax_kernel", "gemm_mxf4_pair_kernel") else ()
     for n in (_KERNEL_SRC[kernel], "ptx.cuh", "internal.h") + extra:
         m.update(open(os.path.join(d, n), "rb").read())
     return m.hexdigest()[:16]
