@@ -101,6 +101,28 @@ int num_sms()
     return cache[dev];
 }
 
+int resident_blocks_per_sm(const void *kern, int threads, size_t smem)
+{
+    // (one entry per kernel: a handful of quantizers, looked up once each)
+    struct Entry {
+        const void *kern;
+        int threads, blocks;
+    };
+    static Entry table[64];
+    static int used = 0;
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
+    for (int i = 0; i < used; ++i)
+        if (table[i].kern == kern && table[i].threads == threads)
+            return table[i].blocks;
+    int n = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, threads, smem) != cudaSuccess || n < 1)
+        n = 1;
+    if (used < 64)
+        table[used++] = {kern, threads, n};
+    return n;
+}
+
 bool encode_tmap_2d_u8(CUtensorMap *map, const void *base, uint64_t inner_bytes, uint64_t rows,
                        uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows, int swizzle)
 {

@@ -160,6 +160,11 @@ rfq_status linear_check(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint
                         const rfq_qtensor *wq, void *y, int32_t out_dtype, void *workspace, bool *launch,
                         bool check_ws);
 
+// Blocks of `threads` threads (and `smem` dynamic shared bytes) of `kern`
+// resident on one SM at once (cached per kernel): grid-stride kernels launch
+// at most that many per SM, so no partial second wave trails the first.
+int resident_blocks_per_sm(const void *kern, int threads, size_t smem);
+
 // Number of SMs of the current device (cached).
 int num_sms();
 

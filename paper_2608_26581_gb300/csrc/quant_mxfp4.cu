@@ -430,16 +430,21 @@ cudaError_t launch_act_quant_mxfp4(const void *x, int64_t M, int64_t K, int mode
     }
     const int64_t pad = layout == RFQ_SCALE_MMA ? ((M + 127) / 128) * 128 - M : 0;
     const int64_t warps = M * ((K + kSeg - 1) / kSeg);
-    // (six 256-thread blocks per SM, each warp looping over items: measured
-    // within 1% of four to thirty-two per SM)
-    const int blocks = grid_for(warps * 32 > pad * (K / 32) ? warps * 32 : pad * (K / 32), 256, num_sms() * 6);
+    const int64_t work = warps * 32 > pad * (K / 32) ? warps * 32 : pad * (K / 32);
     auto *xi = static_cast<const uint4 *>(x);
     auto *mc = static_cast<uint32_t *>(mcodes);
     auto *ms = static_cast<uint8_t *>(mscales);
     auto *rc = static_cast<uint32_t *>(rcodes);
     auto *rs = static_cast<uint8_t *>(rscales);
+    // As many 256-thread blocks as are resident at once (registers limit
+    // it), each warp looping over items: a grid beyond that runs a second,
+    // partial wave (10% slower at six blocks per SM against four).
+    auto grid = [&](auto kern) {
+        return grid_for(work, 256, num_sms() * resident_blocks_per_sm((const void *)kern, 256, 0));
+    };
 #define RFQ_AQ(RES, PHI, LAY)                                                                                     \
-    act_quant_mxfp4_kernel<RES, PHI, LAY><<<blocks, 256, 0, st>>>(xi, M, K, mc, ms, rc, rs, phi, p_s, r_s, pad)
+    act_quant_mxfp4_kernel<RES, PHI, LAY><<<grid(act_quant_mxfp4_kernel<RES, PHI, LAY>), 256, 0, st>>>(            \
+        xi, M, K, mc, ms, rc, rs, phi, p_s, r_s, pad)
     if (mode == RFQ_FALLBACK_NONE) {
         if (layout == RFQ_SCALE_MMA) RFQ_AQ(false, false, RFQ_SCALE_MMA);
         else RFQ_AQ(false, false, RFQ_SCALE_ROWMAJOR);
