@@ -174,6 +174,22 @@ class ClockSampler:
                 "reasons": reasons}
 
 
+class _Nvtx:
+    """An NVTX range around a phase of the run (visible in a profiler's
+    timeline; no cost otherwise)."""
+
+    def __init__(self, name: str):
+        self.name = name
+
+    def __enter__(self):
+        import torch
+        torch.cuda.nvtx.range_push(self.name)
+
+    def __exit__(self, *a):
+        import torch
+        torch.cuda.nvtx.range_pop()
+
+
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -199,12 +215,15 @@ def _job_rate(units_per_rank: float, ws: int, ms: float) -> float:
     return ws * units_per_rank / (ms * 1e-3)
 
 
-def _workload(rows: int = 0, name: str = WORKLOAD):
+def _workload(rows: int = 0, name: str = WORKLOAD, seed=None):
     """The benchmark workload; rows > 0 keeps only the first `rows` token
-    rows (a smaller case of the same kernels, for profiler captures)."""
+    rows (a smaller case of the same kernels, for profiler captures); seed
+    replaces its input seed."""
     import dataclasses
     from paper_2608_26581_gb300.synth import WORKLOADS
     spec = WORKLOADS[name]
+    if seed is not None:
+        spec = dataclasses.replace(spec, act=dataclasses.replace(spec.act, seed=seed))
     if rows and rows < spec.act.M:
         spec = dataclasses.replace(spec, name=f"{spec.name}_first{rows}rows",
                                    act=dataclasses.replace(spec.act, M=rows))
@@ -224,7 +243,7 @@ def _inputs_desc(a):
 def _config(spec, extra=None):
     M, K, N = spec.act.M, spec.act.K, spec.N
     x_mb, y_mb = M * K * 2 / 1e6, M * N * 2 / 1e6
-    c = {"workload": spec.name, "M": M, "K": K, "N": N, "main_format": spec.fmt,
+    c = {"workload": spec.name, "M": M, "K": K, "N": N, "seed": spec.act.seed, "main_format": spec.fmt,
          "residual_format": spec.fmt, "phi": "all tiles (phi = 1)", "y_dtype": "bf16",
          "inputs": _inputs_desc(spec.act),
          "l2": (f"inputs larger than L2 (X {x_mb:.0f} MB, Y {y_mb:.0f} MB per step; two buffer sets "
@@ -363,7 +382,7 @@ def run_reference(args):
     ws, rank, _ = _dist()
     if rank != 0:
         return
-    spec = _workload(0, args.workload)
+    spec = _workload(0, args.workload, args.seed)
     rows = 8 if spec.N else 64   # 8 rows share each call's fp64 expansion of W~
     n, unit, sample, reps = cpu_oracle_timed(args.workload, rows, 1, args.warmup + args.steps)
     timed = reps[args.warmup:]
@@ -390,7 +409,7 @@ def run_rfq(args):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    spec = _workload(args.rows, args.workload)
+    spec = _workload(args.rows, args.workload, args.seed)
     M, K, N = spec.act.M, spec.act.K, spec.N
     hif4 = spec.fmt == "hif4"
     quant_only = N == 0
@@ -542,9 +561,10 @@ def run_rfq(args):
                            stream=None)
         mark(3)
 
-    for i in range(args.warmup):
-        step(None, i & 1)
-    torch.cuda.synchronize()
+    with _Nvtx("rfq warm-up steps (eager)"):
+        for i in range(args.warmup):
+            step(None, i & 1)
+        torch.cuda.synchronize()
     if rfq.rfq_workspace_status(wsp) != rfq.RFQ_OK:
         raise RuntimeError("rfq_linear reported a device timeout")
 
@@ -571,20 +591,23 @@ def run_rfq(args):
     # the fused linear) takes the timed loop's own step time.
     # The clock samples kept are those of the loaded interval: the warm-up
     # replays, the instrumented one and the timed one, back to back.
-    graph = capture(False)
-    graph_ev = capture(True)
+    with _Nvtx("rfq graph capture"):
+        graph = capture(False)
+        graph_ev = capture(True)
     t_start, t_end = ev(), ev()
     with ClockSampler(local) as clk:
         barrier()
         torch.cuda.synchronize()
         h0 = time.time()
-        for _ in range(args.warmup):
+        with _Nvtx("rfq warm-up replays + instrumented replay"):
+            for _ in range(args.warmup):
+                graph.replay()
+            graph_ev.replay()
+        with _Nvtx("rfq timed replay"):
+            t_start.record(stream)
             graph.replay()
-        graph_ev.replay()
-        t_start.record(stream)
-        graph.replay()
-        t_end.record(stream)
-        torch.cuda.synchronize()
+            t_end.record(stream)
+            torch.cuda.synchronize()
         h1 = time.time()
         barrier()
         # the dense FP4 tensor rate with MMAs alone (both MMA forms), timed
@@ -592,7 +615,8 @@ def run_rfq(args):
         mma_peak = None
         if not args.no_mma_peak and ws == 1 and not (quant_only or hif4 or f8):
             h2 = time.time()
-            mma_peak = _fp4_mma_peak(rfq, wsp, stream, ev)
+            with _Nvtx("rfq MMA-only FP4 rate"):
+                mma_peak = _fp4_mma_peak(rfq, wsp, stream, ev)
             mma_peak["clocks"] = clk.summary(h2, time.time(), "the MMA-only launches")
             if mma_peak["clocks"]:
                 mma_peak["flop_per_sm_clock"] = (mma_peak["tflops"] * 1e12 / mma_peak["sms"]
@@ -601,7 +625,8 @@ def run_rfq(args):
         # its measuring build (rfq_linear_profile) on the same operands
         mma_prof = None
         if (ws == 1 and not (quant_only or hif4 or f8 or fused or grouped or amax_phi or no_res) and M > 128):
-            mma_prof = _mma_profile(rfq, bufs[0], wop, K)
+            with _Nvtx("rfq GEMM measuring build"):
+                mma_prof = _mma_profile(rfq, bufs[0], wop, K)
     ms = t_start.elapsed_time(t_end) / args.steps
     q_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in per_step)
     g_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in per_step)
@@ -619,6 +644,8 @@ def run_rfq(args):
     # i - 1 and i + 1 (the copy engines give ~200 GB/s per direction).
     e2e_ms = None
     if not args.no_e2e:
+        _nv = _Nvtx("rfq end-to-end loop (host buffers)")
+        _nv.__enter__()
         h2d, d2h = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
         x_ready = [torch.cuda.Event(), torch.cuda.Event()]
         x_free = [torch.cuda.Event(), torch.cuda.Event()]
@@ -661,6 +688,7 @@ def run_rfq(args):
         torch.cuda.synchronize()
         barrier()
         e2e_ms = e0.elapsed_time(e1) / args.steps
+        _nv.__exit__()
     if e2e_ms is not None:
         e2e_ms = _max_over_ranks(e2e_ms, ws, dist, dev)
     if rfq.rfq_workspace_status(wsp) != rfq.RFQ_OK:
@@ -876,6 +904,10 @@ def _other_configs(args):
     return out
 
 
+# the configuration list's entries, in order
+_CONFIGS = {1: "tiny", 2: "act_quant", 3: "qwen_gate_up", 4: "qwen_down_hif4", 5: "wan_ffn_up"}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -896,11 +928,17 @@ def main():
                     help="fused: rfq_linear_fused, the activation quantizer inside the GEMM")
     ap.add_argument("--workload", default=WORKLOAD,
                     choices=["wan_ffn_up", "qwen_gate_up", "qwen_down_hif4", "act_quant", "tiny", "qwen_moe_gate_up"])
+    ap.add_argument("--config", type=int, default=0, choices=[0, 1, 2, 3, 4, 5],
+                    help="the configuration list's entry (1 tiny, 2 act-quant, 3 Qwen3-VL gate/up, 4 Qwen3-VL "
+                         "HiF4 down, 5 Wan2.2 FFN up); overrides --workload")
+    ap.add_argument("--seed", type=int, default=None, help="replace the workload's input seed")
     ap.add_argument("--no-extras", action="store_true",
                     help="skip the child runs that time the other workloads of the configuration list")
     ap.add_argument("--no-mma-peak", action="store_true",
                     help="skip the MMA-only FP4 rate measurement")
     args = ap.parse_args()
+    if args.config:
+        args.workload = _CONFIGS[args.config]
     if args.warmup < 3:
         args.warmup = 3
     if args.impl == "reference":

@@ -194,7 +194,11 @@ RFQ_API rfq_status rfq_quantize_act_expand(const void *x_bf16, int64_t M, int64_
  * way to run a kernel's timeout path with no copy or MMA in flight.  Every
  * GEMM entry point (rfq_linear, rfq_linear_fused, rfq_linear_grouped)
  * honours words [1] to [3]; leave them zero in normal use.  Bytes 32..95
- * receive rfq_linear_profile's counters. */
+ * receive rfq_linear_profile's counters.  With the environment variable
+ * RFQ_DEBUG_SYNC set (to anything but "0") when the library first checks it,
+ * every GEMM entry point synchronizes its stream after the launch and
+ * returns the status the workspace then holds (as rfq_workspace_status
+ * would), so a timeout surfaces at the call that caused it. */
 RFQ_API size_t rfq_linear_workspace_bytes(void);
 
 /* RFQ GEMM (Algorithm 1, Eq. rfq): Y = X~ W~ + phi X^ W~ with both products
@@ -347,6 +351,18 @@ RFQ_API rfq_status rfq_fp4_mma_peak(int32_t cta_pair, int64_t iters, void *works
  * Errors: those of rfq_linear; RFQ_ERR_UNSUPPORTED for other operand forms. */
 RFQ_API rfq_status rfq_linear_profile(const rfq_qtensor *xq, const rfq_qtensor *xr, const rfq_qtensor *wq, void *y,
                                       int32_t out_dtype, void *workspace, void *stream);
+
+/* The debug build (librfq_debug.so, compiled with -DRFQ_DEBUG_BOUNDS): the
+ * activation and weight quantizers and the CTA-pair GEMM check the index of
+ * every direct global store against its buffer's extent (codes, scales, the
+ * fused quantizer's ring, the grouped GEMM's row stores); an out-of-range
+ * store is skipped and the source line of the first one is recorded.  This
+ * call synchronizes the device and reports it: RFQ_OK (none, *line = 0) or
+ * RFQ_ERR_SHAPE with *line set; clear != 0 resets the records.  The normal
+ * build has no checks and returns RFQ_ERR_UNSUPPORTED.  The paper has no
+ * counterpart: a debugging aid of this library.
+ * Errors: RFQ_ERR_INVALID_ARG (line NULL), RFQ_ERR_CUDA. */
+RFQ_API rfq_status rfq_debug_bounds(int32_t *line, int32_t clear);
 
 /* Allocation-free variant of rfq_linear.  The paper has no counterpart: this
  * entry point exists for callers that cannot allocate device memory, such as

@@ -5,6 +5,7 @@
 #include <cuda_runtime.h>
 
 #include <cstdint>
+#include <cstdlib>
 #include <mutex>
 
 #include "internal.h"
@@ -53,6 +54,18 @@ rfq_status check_device()
 }
 
 rfq_status from_cuda(cudaError_t e) { return e == cudaSuccess ? RFQ_OK : RFQ_ERR_CUDA; }
+
+// The environment variable RFQ_DEBUG_SYNC (any value but "0") makes every
+// GEMM entry point synchronize its stream after the launch and return the
+// device status its workspace holds (RFQ_ERR_TIMEOUT, ...) instead of RFQ_OK.
+bool debug_sync()
+{
+    static const int on = [] {
+        const char *v = getenv("RFQ_DEBUG_SYNC");
+        return v && v[0] && !(v[0] == '0' && v[1] == 0) ? 1 : 0;
+    }();
+    return on != 0;
+}
 
 bool fmt_ok(int32_t f)
 {
@@ -145,6 +158,20 @@ bool encode_tmap_2d_u8(CUtensorMap *map, const void *base, uint64_t inner_bytes,
 } // namespace rfq
 
 using namespace rfq;
+
+namespace rfq {
+namespace {
+// The status of a GEMM launch (see debug_sync).
+rfq_status gemm_done(cudaError_t e, void *workspace, cudaStream_t st)
+{
+    if (e != cudaSuccess)
+        return RFQ_ERR_CUDA;
+    if (!debug_sync())
+        return RFQ_OK;
+    return rfq_workspace_status(workspace, 0, st);
+}
+} // namespace
+} // namespace rfq
 
 extern "C" {
 
@@ -411,7 +438,7 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
         a.N = N;
         a.K = K;
         a.status = static_cast<int32_t *>(workspace);
-        return from_cuda(launch_gemm_hif4(a, st));
+        return gemm_done(launch_gemm_hif4(a, st), workspace, st);
     }
     GemmMxf4Args a;
     a.a_codes = xq->codes;
@@ -429,7 +456,7 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
     a.K = K;
     a.status = static_cast<int32_t *>(workspace);
     a.f8 = f8;
-    return from_cuda(launch_gemm_mxf4(a, st));
+    return gemm_done(launch_gemm_mxf4(a, st), workspace, st);
 }
 
 } // extern "C"
@@ -533,7 +560,8 @@ rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, const rfq_
         a.fq_x = x_bf16;
         a.fq_ctr = reinterpret_cast<int32_t *>(w + L.ctr);
         a.fq_ring = L.ring;
-        return from_cuda(launch_gemm_mxf4_pair(a, static_cast<cudaStream_t>(stream)));
+        return gemm_done(launch_gemm_mxf4_pair(a, static_cast<cudaStream_t>(stream)), workspace,
+                         static_cast<cudaStream_t>(stream));
     }
     GemmFusedArgs a;
     a.x = x_bf16;
@@ -546,7 +574,8 @@ rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, const rfq_
     a.N = N;
     a.K = K;
     a.status = static_cast<int32_t *>(workspace);
-    return from_cuda(launch_gemm_mxf4_fused(a, static_cast<cudaStream_t>(stream)));
+    return gemm_done(launch_gemm_mxf4_fused(a, static_cast<cudaStream_t>(stream)), workspace,
+                         static_cast<cudaStream_t>(stream));
 }
 
 rfq_status rfq_linear_profile(const rfq_qtensor *xq, const rfq_qtensor *xr, const rfq_qtensor *wq, void *y,
@@ -574,7 +603,8 @@ rfq_status rfq_linear_profile(const rfq_qtensor *xq, const rfq_qtensor *xr, cons
     a.K = xq->k;
     a.status = static_cast<int32_t *>(workspace);
     a.prof = 1;
-    return from_cuda(launch_gemm_mxf4_pair(a, static_cast<cudaStream_t>(stream)));
+    return gemm_done(launch_gemm_mxf4_pair(a, static_cast<cudaStream_t>(stream)), workspace,
+                         static_cast<cudaStream_t>(stream));
 }
 
 rfq_status rfq_fp4_mma_peak(int32_t cta_pair, int64_t iters, void *workspace, double *flop_per_launch,
@@ -591,6 +621,30 @@ rfq_status rfq_fp4_mma_peak(int32_t cta_pair, int64_t iters, void *workspace, do
         return s;
     return from_cuda(launch_fp4_mma_peak(cta_pair, iters, static_cast<int32_t *>(workspace), flop_per_launch,
                                          static_cast<cudaStream_t>(stream)));
+}
+
+rfq_status rfq_debug_bounds(int32_t *line, int32_t clear)
+{
+#ifdef RFQ_DEBUG_BOUNDS
+    if (!line)
+        return RFQ_ERR_INVALID_ARG;
+    if (cudaDeviceSynchronize() != cudaSuccess)
+        return RFQ_ERR_CUDA;
+    const int words[2] = {debug_word_quant_mxfp4(clear), debug_word_gemm_mxf4_pair(clear)};
+    *line = 0;
+    for (int w : words) {
+        if (w < 0)
+            return RFQ_ERR_CUDA;
+        if (w > 0 && *line == 0)
+            *line = w;
+    }
+    return *line ? RFQ_ERR_SHAPE : RFQ_OK;
+#else
+    (void)clear;
+    if (line)
+        *line = 0;
+    return RFQ_ERR_UNSUPPORTED;
+#endif
 }
 
 rfq_status rfq_workspace_status(void *workspace, int32_t clear, void *stream)
@@ -739,7 +793,8 @@ rfq_status rfq_linear_grouped(const rfq_qtensor *xq, const rfq_qtensor *xr, cons
     a.f8 = f8;
     a.group_off = group_off;
     a.groups = groups;
-    return from_cuda(launch_gemm_mxf4(a, static_cast<cudaStream_t>(stream)));
+    return gemm_done(launch_gemm_mxf4(a, static_cast<cudaStream_t>(stream)), workspace,
+                     static_cast<cudaStream_t>(stream));
 }
 
 } // extern "C"

@@ -69,6 +69,8 @@
 namespace rfq {
 namespace {
 
+RFQ_DEBUG_WORD_DECL
+
 constexpr int BM = 128;                  // rows per CTA (256 per pair)
 constexpr int BN = 256;                  // output columns per pair tile
 constexpr int BN_HALF = BN / 2;          // W~ rows staged per CTA
@@ -654,7 +656,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 bf16x32_to_f32(w, xf);
                 const Mx32 qz = mxfp4_quant32<RES>(xf);
                 // rows past M get zero codes and scale bytes (zero input)
-                if (b < kb) {
+                if (b < kb && RFQ_IN_BOUNDS((int64_t)mr * kb + b, (int64_t)fq.ring * 2 * BM * kb)) {
                     reinterpret_cast<uint4 *>(fq.mcodes)[(int64_t)mr * kb + b] = qz.code;
                     if (RES)
                         reinterpret_cast<uint4 *>(fq.rcodes)[(int64_t)mr * kb + b] = qz.rcode;
@@ -751,7 +753,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     if (GRP && row0 + 32 > tc.row_end && tc.row_end < M) {
                         // a group ends inside this 32-row box: rows past it are
                         // another group's or padding, so each lane stores its own row
-                        if (row0 + lane < tc.row_end) {
+                        if (row0 + lane < tc.row_end &&
+                            RFQ_IN_BOUNDS((int64_t)(row0 + lane) * N + col + 31, (int64_t)M * N)) {
                             uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(y) +
                                                                    (int64_t)(row0 + lane) * N + col);
 #pragma unroll
@@ -797,7 +800,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                                 break;
                             if (GRP && row0 + 32 > tc.row_end && tc.row_end < M) {
                                 // a group ends inside this 32-row box (see the bf16 path)
-                                if (row0 + lane < tc.row_end) {
+                                if (row0 + lane < tc.row_end &&
+                                    RFQ_IN_BOUNDS((int64_t)(row0 + lane) * N + col + 16 * hb + 15, (int64_t)M * N)) {
                                     uint4 *dst = reinterpret_cast<uint4 *>(static_cast<float *>(y) +
                                                                            (int64_t)(row0 + lane) * N + col + 16 * hb);
 #pragma unroll
@@ -1102,5 +1106,7 @@ cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
     RFQ_GV(true, false, false);
 #undef RFQ_GV
 }
+
+RFQ_DEBUG_WORD_ACCESSOR(debug_word_gemm_mxf4_pair)
 
 } // namespace rfq

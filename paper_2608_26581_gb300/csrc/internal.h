@@ -9,6 +9,46 @@
 
 namespace rfq {
 
+// ---- the debug build (compiled with -DRFQ_DEBUG_BOUNDS, librfq_debug.so):
+// every direct global store of the kernels that carry these checks tests
+// its index against its buffer's extent; an out-of-range store is skipped
+// and the source line of the first one is kept in the translation unit's
+// debug word (RFQ_DEBUG_WORD_DECL), which rfq_debug_bounds reads.  In the
+// normal build the checks compile to nothing.
+__device__ __forceinline__ bool debug_in_bounds(int64_t i, int64_t n, int line, int *word)
+{
+    if (i >= 0 && i < n)
+        return true;
+    atomicCAS(word, 0, line);
+    return false;
+}
+#ifdef RFQ_DEBUG_BOUNDS
+#define RFQ_DEBUG_WORD_DECL static __device__ int g_rfq_debug_word = 0;
+#define RFQ_IN_BOUNDS(i, n) ::rfq::debug_in_bounds((int64_t)(i), (int64_t)(n), __LINE__, &g_rfq_debug_word)
+#define RFQ_DEBUG_WORD_ACCESSOR(fn)                                                                               \
+    int fn(int clear)                                                                                             \
+    {                                                                                                             \
+        int v = 0;                                                                                                \
+        if (cudaMemcpyFromSymbol(&v, g_rfq_debug_word, sizeof v) != cudaSuccess)                                  \
+            return -1;                                                                                            \
+        if (clear) {                                                                                              \
+            const int z = 0;                                                                                      \
+            if (cudaMemcpyToSymbol(g_rfq_debug_word, &z, sizeof z) != cudaSuccess)                                \
+                return -1;                                                                                        \
+        }                                                                                                         \
+        return v;                                                                                                 \
+    }
+#else
+#define RFQ_DEBUG_WORD_DECL
+#define RFQ_IN_BOUNDS(i, n) true
+#define RFQ_DEBUG_WORD_ACCESSOR(fn)                                                                               \
+    int fn(int) { return 0; }
+#endif
+// Each translation unit with bounds checks: its debug word (the source line
+// of the first out-of-range store, 0 if none; -1 if it cannot be read).
+int debug_word_quant_mxfp4(int clear);
+int debug_word_gemm_mxf4_pair(int clear);
+
 // Device status word values written into a workspace by kernels.
 constexpr int32_t kDevOk = 0;
 constexpr int32_t kDevTimeout = 1;

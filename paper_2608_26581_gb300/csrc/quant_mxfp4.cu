@@ -23,6 +23,16 @@
 namespace rfq {
 namespace {
 
+RFQ_DEBUG_WORD_DECL
+
+// Bytes of an MXFP4 scale array for `rows` rows of K (the MMA layout pads
+// rows to 128): the extent of the debug build's bounds checks.
+template <int LAYOUT>
+__device__ __forceinline__ int64_t scale_bytes(int64_t rows, int64_t K)
+{
+    return (LAYOUT == RFQ_SCALE_MMA ? (rows + 127) / 128 * 128 : rows) * (K >> 5);
+}
+
 template <int LAYOUT>
 __device__ __forceinline__ int64_t scale_index(int64_t m, int64_t b, int64_t kblocks)
 {
@@ -59,6 +69,8 @@ __global__ void __launch_bounds__(256) act_quant_mxfp4_kernel(const uint4 *__res
         const int64_t n = pad_rows * kblocks;
         for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
             const int64_t off = scale_index<LAYOUT>(M + i / kblocks, i % kblocks, kblocks);
+            if (!RFQ_IN_BOUNDS(off, scale_bytes<LAYOUT>(M, K)))
+                continue;
             mscales[off] = 0;
             if (RES)
                 rscales[off] = 0;
@@ -94,6 +106,8 @@ __global__ void __launch_bounds__(256) act_quant_mxfp4_kernel(const uint4 *__res
             continue;
         const int64_t soff = scale_index<LAYOUT>(m, b, kblocks);
         const int64_t coff = m * kblocks + b;               // 16-byte words of codes
+        if (!RFQ_IN_BOUNDS(coff, M * kblocks) || !RFQ_IN_BOUNDS(soff, scale_bytes<LAYOUT>(M, K)))
+            continue;
         mc4[coff] = qz.code;
         mscales[soff] = (uint8_t)qz.sb;
         if (RES) {
@@ -239,27 +253,35 @@ __global__ void __launch_bounds__(256, 3)
     for (int i = 0; i < R; ++i) {
         const int64_t m = m0 + i; // uniform over the warp
         const int64_t soff = scale_index<LAYOUT>(m, b, kblocks);
+        // (the debug build's checks gate the stores only: the quantization
+        // below takes all 32 lanes)
+        const bool inb = RFQ_IN_BOUNDS(soff, scale_bytes<LAYOUT>(M, K)) &&
+                         (m >= M || RFQ_IN_BOUNDS(m * kchunks + c, M * kchunks));
         if (m < M) {
             float xf[8];
             bf16x8_to_f32(row(i), xf);
             if (on) {
                 const Mx8 qz = mxfp4_quant8<true>(xf);
-                mcodes[m * kchunks + c] = qz.code;
-                rcodes[m * kchunks + c] = qz.rcode;
-                if ((lane & 3) == 0) {
-                    mscales[soff] = (uint8_t)qz.sb;
-                    rscales[soff] = (uint8_t)qz.rb;
+                if (inb) {
+                    mcodes[m * kchunks + c] = qz.code;
+                    rcodes[m * kchunks + c] = qz.rcode;
+                    if ((lane & 3) == 0) {
+                        mscales[soff] = (uint8_t)qz.sb;
+                        rscales[soff] = (uint8_t)qz.rb;
+                    }
                 }
             } else {
                 const Mx8 qz = mxfp4_quant8<false>(xf);
-                mcodes[m * kchunks + c] = qz.code;
-                rcodes[m * kchunks + c] = 0u;
-                if ((lane & 3) == 0) {
-                    mscales[soff] = (uint8_t)qz.sb;
-                    rscales[soff] = 0;
+                if (inb) {
+                    mcodes[m * kchunks + c] = qz.code;
+                    rcodes[m * kchunks + c] = 0u;
+                    if ((lane & 3) == 0) {
+                        mscales[soff] = (uint8_t)qz.sb;
+                        rscales[soff] = 0;
+                    }
                 }
             }
-        } else if (LAYOUT == RFQ_SCALE_MMA && (lane & 3) == 0) {
+        } else if (LAYOUT == RFQ_SCALE_MMA && (lane & 3) == 0 && inb) {
             // rows M .. of the last tile are the layout's padding rows
             mscales[soff] = 0;
             rscales[soff] = 0;
@@ -302,7 +324,7 @@ __global__ void __launch_bounds__(256) weight_quant_mxfp4_kernel(const __nv_bflo
     if (b >= kblocks)
         return;
     if (n >= N) {
-        if (LAYOUT == RFQ_SCALE_MMA)
+        if (LAYOUT == RFQ_SCALE_MMA && RFQ_IN_BOUNDS(scale_index<LAYOUT>(n, b, kblocks), scale_bytes<LAYOUT>(N, K)))
             scales[scale_index<LAYOUT>(n, b, kblocks)] = 0;
         return;
     }
@@ -325,6 +347,9 @@ __global__ void __launch_bounds__(256) weight_quant_mxfp4_kernel(const __nv_bflo
             y[i] = xf[g * 8 + i] * inv;
         out[g] = e2m1x8(y);
     }
+    if (!RFQ_IN_BOUNDS(n * (K >> 1) + b * 16 + 15, N * (K >> 1)) ||
+        !RFQ_IN_BOUNDS(scale_index<LAYOUT>(n, b, kblocks), scale_bytes<LAYOUT>(N, K)))
+        return;
     *reinterpret_cast<uint4 *>(codes + n * (K >> 1) + b * 16) = make_uint4(out[0], out[1], out[2], out[3]);
     scales[scale_index<LAYOUT>(n, b, kblocks)] = (uint8_t)sb;
 }
@@ -499,5 +524,7 @@ cudaError_t launch_dequant_mxfp4_bf16(const void *codes, const void *scales, int
             (const uint32_t *)codes, (const uint8_t *)scales, rows, k, (uint4 *)out);
     return cudaGetLastError();
 }
+
+RFQ_DEBUG_WORD_ACCESSOR(debug_word_quant_mxfp4)
 
 } // namespace rfq

@@ -13,7 +13,8 @@ from dataclasses import dataclass
 import torch
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_HERE, "librfq.so")
+# the library (RFQ_LIBRARY names another build of it, e.g. librfq_debug.so)
+LIB_PATH = os.environ.get("RFQ_LIBRARY") or os.path.join(_HERE, "librfq.so")
 
 RFQ_OK = 0
 RFQ_FMT_MXFP4, RFQ_FMT_HIF4, RFQ_FMT_BF16, RFQ_FMT_MXFP8 = 0, 1, 2, 3
@@ -30,7 +31,7 @@ EXPORTED = ("rfq_status_string", "rfq_qtensor_bytes", "rfq_quantize_weight", "rf
             "rfq_linear_workspace_bytes", "rfq_linear", "rfq_workspace_status", "rfq_dequant",
             "rfq_linear_noalloc", "rfq_linear_fused", "rfq_convert", "rfq_linear_grouped", "rfq_check_finite",
             "rfq_quantize_act_expand", "rfq_fp4_mma_peak", "rfq_linear_fused_workspace_bytes",
-            "rfq_linear_profile")
+            "rfq_linear_profile", "rfq_debug_bounds")
 
 
 class RFQError(RuntimeError):
@@ -91,6 +92,8 @@ def load_library(path: str = LIB_PATH):
         lib.rfq_linear_grouped.argtypes = [QTP, QTP, P, I32, P, I32, QTP, I64, P, I32, P, P]
         lib.rfq_linear_fused_workspace_bytes.restype = SZ
         lib.rfq_linear_fused_workspace_bytes.argtypes = [I64, I64, ctypes.POINTER(_FB)]
+        lib.rfq_debug_bounds.restype = I32
+        lib.rfq_debug_bounds.argtypes = [ctypes.POINTER(I32), I32]
         lib.rfq_linear_profile.restype = I32
         lib.rfq_linear_profile.argtypes = [QTP, QTP, QTP, P, I32, P, P]
         lib.rfq_fp4_mma_peak.restype = I32
@@ -309,3 +312,11 @@ def rfq_linear_profile(xq: QTensor, xr: QTensor, wq: QTensor, y: torch.Tensor, o
     torch.cuda.synchronize(workspace.device)
     v = workspace.view(torch.uint8)[32:96].cpu().view(torch.int64).tolist()
     return dict(zip(PROFILE_KEYS, v))
+
+
+def rfq_debug_bounds(clear: bool = False) -> tuple[int, int]:
+    """(status, source line) of the debug build's first out-of-range store
+    (see include/rfq.h); the normal build returns RFQ_ERR_UNSUPPORTED."""
+    line = ctypes.c_int32(0)
+    st = load_library().rfq_debug_bounds(ctypes.byref(line), 1 if clear else 0)
+    return st, line.value

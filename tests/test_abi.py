@@ -182,3 +182,10 @@ def test_noalloc_rejects_before_touching_its_array(lib):
     wq_bad = rfq._QT(rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA, 40, 256, 16, 16)   # N % 16 != 0
     assert lib.rfq_linear_noalloc(r(xq), None, None, 0, r(wq_bad), P(16), 0, None) == rfq.RFQ_ERR_SHAPE
     assert lib.rfq_linear_noalloc(r(xq), None, None, 0, r(xq), P(8), 0, None) == rfq.RFQ_ERR_ALIGNMENT
+
+
+def test_debug_bounds_is_the_debug_builds(lib):
+    """The normal build carries no bounds checks: rfq_debug_bounds says so."""
+    from paper_2608_26581_gb300 import rfq
+    st, line = rfq.rfq_debug_bounds()
+    assert st == rfq.RFQ_ERR_UNSUPPORTED and line == 0

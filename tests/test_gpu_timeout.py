@@ -15,6 +15,7 @@ import numpy as np
 import pytest
 import torch
 
+from conftest import ROOT
 from gpu_util import DEV, check_y, qtensor_host, to_dev_bf16
 from paper_2608_26581_gb300 import rfq
 from paper_2608_26581_gb300.synth import ActSpec, make_activation, make_weight
@@ -190,3 +191,37 @@ def test_grouped_gemm_timeout(orc, counts):
     launch(ws)
     assert rfq.rfq_workspace_status(ws) == rfq.RFQ_OK
     check(y.double().cpu().numpy(), ref)
+
+
+def test_debug_sync_reports_the_timeout_at_the_call():
+    """With RFQ_DEBUG_SYNC set, rfq_linear synchronizes and returns the
+    workspace's status: a held start that runs out raises RFQ_ERR_TIMEOUT
+    from the call itself (a child process: the variable is read once)."""
+    import os
+    import subprocess
+    import sys
+    code = """
+import sys, torch
+sys.path.insert(0, %r)
+sys.path.insert(0, %r)
+from paper_2608_26581_gb300 import rfq
+from paper_2608_26581_gb300.synth import ActSpec, make_activation, make_weight
+from gpu_util import to_dev_bf16
+M, K, N = 600, 512, 256
+F, L = rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA
+wq = rfq.empty_qtensor(F, L, N, K); rfq.rfq_quantize_weight(to_dev_bf16(make_weight(K, N, seed=1)), wq)
+xq, xr = rfq.empty_qtensor(F, L, M, K), rfq.empty_qtensor(F, L, M, K)
+rfq.rfq_quantize_act(to_dev_bf16(make_activation(ActSpec(M, K, "normal", seed=2))), xq, xr)
+y = torch.empty(M, N, device="cuda")
+ws = torch.zeros(64, dtype=torch.int32, device="cuda")
+rfq.rfq_linear(xq, xr, None, 256, wq, y, rfq.RFQ_OUT_F32, ws)   # computes: RFQ_OK
+ws[1], ws[2] = 20000, 1
+try:
+    rfq.rfq_linear(xq, xr, None, 256, wq, y, rfq.RFQ_OUT_F32, ws)
+except rfq.RFQError as e:
+    print("STATUS", e.status)
+""" % (ROOT, os.path.join(ROOT, "tests"))
+    env = dict(os.environ, RFQ_DEBUG_SYNC="1")
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
+    assert f"STATUS {rfq.RFQ_ERR_TIMEOUT}" in r.stdout, r.stdout + r.stderr[-2000:]
