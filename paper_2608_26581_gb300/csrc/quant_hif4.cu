@@ -79,12 +79,23 @@ __device__ __forceinline__ int hif4_scale_byte(float amax)
 }
 
 // Quantizes the eight elements x[0..7] of group g (sub-groups 2g, 2g+1) of a
-// 64-element block whose macro scale S is given.  Returns the codes (element
-// i in nibble i) and this group's E1_8 / E1_16 bits (placed at their final
-// metadata positions); `deq` receives the dequantized values.
-__device__ __forceinline__ uint32_t hif4_group(const float (&x)[8], float S, int g, uint32_t &meta_bits,
+// 64-element block whose macro scale byte sb = (E << 2) | M is given.
+// Returns the codes (element i in nibble i) and this group's E1_8 / E1_16
+// bits (placed at their final metadata positions); `deq` receives the
+// dequantized values.
+//
+// A sub-group with exponent ex has the step 0.25 S 2^ex = 2^(E - 50 + ex)
+// (1 + M/4), formed from its bits, and its reciprocal is 2^(50 - E - ex)
+// 4 / (4 + M): rounded to fp32 that is the power of two times RN(4 / (4 + M))
+// (scaling by a power of two commutes with rounding in the normal range,
+// which every E in [0, 63] and ex in [0, 2] stays in), i.e. exactly the
+// correctly rounded reciprocal of the step, from one of four constants.
+__device__ __forceinline__ uint32_t hif4_group(const float (&x)[8], int sb, int g, uint32_t &meta_bits,
                                                float (&deq)[8])
 {
+    const int E = sb >> 2, M = sb & 3;
+    const float S = ue6m2_value(E, M);
+    const float recip_m = M == 0 ? 1.0f : M == 1 ? 0.8f : M == 2 ? 0.6666666865348816f : 0.5714285969734192f;
     int t[2];
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
@@ -98,8 +109,8 @@ __device__ __forceinline__ uint32_t hif4_group(const float (&x)[8], float S, int
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
         const int ex = e18 + (h ? e116_1 : e116_0);
-        const float step = 0.25f * S * (float)(1 << ex); // exact: S has 3 significant bits
-        const float inv = __frcp_rn(step);
+        const float step = __uint_as_float(((uint32_t)(E + ex + 77) << 23) | ((uint32_t)M << 21));
+        const float inv = __uint_as_float((uint32_t)(177 - E - ex) << 23) * recip_m;   // RN(1 / step)
         const float hstep = 0.5f * step;
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
@@ -171,10 +182,9 @@ __device__ __forceinline__ void hif4_chunk(const float (&xf)[8], int g, bool ok,
     for (int o = 1; o < 8; o <<= 1)
         am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, o));
     const int sb = am > 0.f ? hif4_scale_byte(am) : 0;
-    const float S = ue6m2_value(sb >> 2, sb & 3);
     uint32_t bits;
     float deq[8];
-    uint32_t code = hif4_group(xf, S, g, bits, deq);
+    uint32_t code = hif4_group(xf, sb, g, bits, deq);
     if (am == 0.f) {
         bits = 0;   // all-zero block: metadata 0, codes keep the sign of zero
     }
@@ -199,10 +209,9 @@ __device__ __forceinline__ void hif4_chunk(const float (&xf)[8], int g, bool ok,
         for (int o = 1; o < 8; o <<= 1)
             ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, o));
         const int rsb = ra > 0.f ? hif4_scale_byte(ra) : 0;
-        const float RS = ue6m2_value(rsb >> 2, rsb & 3);
         uint32_t rbits;
         float rdeq[8];
-        const uint32_t rcode = hif4_group(r, RS, g, rbits, rdeq);
+        const uint32_t rcode = hif4_group(r, rsb, g, rbits, rdeq);
 #pragma unroll
         for (int o = 1; o < 8; o <<= 1)
             rbits |= __shfl_xor_sync(0xFFFFFFFFu, rbits, o);
@@ -360,14 +369,13 @@ __global__ void __launch_bounds__(256) weight_quant_hif4_kernel(const __nv_bfloa
     for (int i = 0; i < 64; ++i)
         am = fmaxf(am, fabsf(__bfloat162float(w[(blk * 64 + i) * N + n])));
     const int sb = am > 0.f ? hif4_scale_byte(am) : 0;
-    const float S = ue6m2_value(sb >> 2, sb & 3);
     uint32_t bits = 0, out[8];
     for (int g = 0; g < 8; ++g) {
         float xf[8], deq[8];
         for (int i = 0; i < 8; ++i)
             xf[i] = __bfloat162float(w[(blk * 64 + 8 * g + i) * N + n]);
         uint32_t gb;
-        out[g] = hif4_group(xf, S, g, gb, deq);
+        out[g] = hif4_group(xf, sb, g, gb, deq);
         bits |= gb;
     }
     uint4 *dst = reinterpret_cast<uint4 *>(codes + n * (K >> 1) + blk * 32);
