@@ -430,12 +430,18 @@ def run_rfq(args):
     #         re-encoded exactly by the quantizer in the same pass, W~ by
     #         rfq_convert offline); w4a8: MXFP8 X x MXFP4 W (re-encoded);
     #         w8a8: MXFP8 X x MXFP8 W.  All on kind::mxf8f6f4.
+    #   rfq8mix: the rfq8 RFQ through rfq_linear_mixed -- the main product
+    #         on kind::mxf4 (X~ and W~ packed), the residual on
+    #         kind::mxf8f6f4 (X^ and W~ as E4M3); no E4M3 copy of X~.
     scheme = args.scheme
+    mixed = scheme == "rfq8mix"
     f8 = scheme != "rfq4"
     if f8 and (hif4 or quant_only or fused or no_res):
         raise SystemExit("--scheme applies to the MXFP4 linear workloads (two-kernel, with residual flags unset)")
     if amax_phi and scheme in ("w4a8", "w8a8"):
         raise SystemExit("--phi-tau needs a residual pathway")
+    if mixed and spec.groups > 0:
+        raise SystemExit("--scheme rfq8mix runs the plain (ungrouped) GEMM")
     F = rfq.RFQ_FMT_HIF4 if hif4 else rfq.RFQ_FMT_MXFP4
     amax_fused = amax_phi and K % 256 == 0   # phi computed in the quantizer's pass
     L = rfq.RFQ_SCALE_MMA
@@ -467,7 +473,7 @@ def run_rfq(args):
         w = torch.from_numpy(wb.view(np.int16)).to(dev).view(torch.bfloat16)
         wq = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme == "w8a8" else F, L, NW, K, device=dev)
         rfq.rfq_quantize_weight(w, wq)                     # offline weight step, untimed
-        if scheme in ("rfq8", "w4a8"):
+        if scheme in ("rfq8", "w4a8", "rfq8mix"):
             wop = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8, L, NW, K, device=dev)
             rfq.rfq_convert(wq, wop)                       # exact E4M3 re-encoding of W~ (offline)
         elif hif4:
@@ -483,7 +489,8 @@ def run_rfq(args):
         b = {"x": xd,
              "xq": rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme in ("w4a8", "w8a8") else F, L, Mb, K, device=dev),
              "xr": None if no_res else
-                   rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme == "rfq8" else F, L, Mb, K, device=dev),
+                   rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme in ("rfq8", "rfq8mix") else F, L, Mb, K,
+                                     device=dev),
              # rfq8: the E4M3 re-encoding of X~ that the GEMM multiplies
              "xq8": rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8, L, Mb, K, device=dev) if scheme == "rfq8" else None,
              "phi": (torch.empty(((Mb + 127) // 128) * ((K + 255) // 256), dtype=torch.uint8, device=dev)
@@ -556,6 +563,8 @@ def run_rfq(args):
         elif grouped:
             rfq.rfq_linear_grouped(xq8 if xq8 is not None else xq, xr, ph, 256, group_off,
                                    wop, N, y_, rfq.RFQ_OUT_BF16, wsp, stream=None)
+        elif mixed:
+            rfq.rfq_linear_mixed(xq, xr, ph, 256, wq, wop, y_, rfq.RFQ_OUT_BF16, wsp, stream=None)
         else:
             rfq.rfq_linear(xq8 if xq8 is not None else xq, xr, ph, 256, wop, y_, rfq.RFQ_OUT_BF16, wsp,
                            stream=None)
@@ -705,6 +714,15 @@ def run_rfq(args):
         t_peak, t_peak_sust = pk["bf16_burst"], pk["bf16_sust"]
         t_src = f"{pk['src']} bf16 burst {pk['bf16_burst']} TFLOP/s, of {pk['src']}"
         t_kernel = "gemm_hif4_kernel"
+    elif mixed:
+        # main product at the FP4 rate (6x bf16, nominal), residual at the FP8
+        # one (2x): the rate the executed FLOP mix allows
+        rate = (1.0 + phi_frac) / (1.0 / FP4_OVER_BF16 + phi_frac / 2.0)
+        t_peak, t_peak_sust = pk["bf16_burst"] * rate, pk["bf16_sust"] * rate
+        t_src = (f"{pk['src']} bf16 burst {pk['bf16_burst']} TFLOP/s x {rate:.3g} (the main product at the nominal "
+                 f"FP4/BF16 ratio {FP4_OVER_BF16:g}, the residual at the FP8 one 2, weighted by their FLOP), "
+                 f"of {pk['src']}")
+        t_kernel = "gemm_mxf4_pair_kernel"   # its mixed-rate instantiation, at every M
     elif f8:
         # kind::mxf8f6f4: the FP8 tensor rate, nominally twice the bf16 one
         t_peak, t_peak_sust = pk["bf16_burst"] * 2.0, pk["bf16_sust"] * 2.0
@@ -725,8 +743,8 @@ def run_rfq(args):
         aq_bytes = _act_quant_bytes(Mb, K, "hif4", not no_res, operand=not quant_only)
         aq_kernel = "act_quant_hif4_amax_kernel" if amax_fused else "act_quant_hif4_kernel"
     elif f8:
-        aq_bytes = _act_quant_bytes(Mb, K, "rfq8" if scheme == "rfq8" else "mxfp8", scheme == "rfq8",
-                                    operand=scheme == "rfq8")
+        aq_bytes = _act_quant_bytes(Mb, K, "rfq8" if scheme in ("rfq8", "rfq8mix") else "mxfp8",
+                                    scheme in ("rfq8", "rfq8mix"), operand=scheme == "rfq8")
         aq_kernel = "act_quant_rfq8_amax_kernel" if amax_fused else "act_quant8_kernel"
     else:
         aq_bytes = _act_quant_bytes(Mb, K, "mxfp4", not no_res)
@@ -795,7 +813,10 @@ def run_rfq(args):
                                          "weight_rows": NW} if grouped else {}),
                                      **({"residual": "none: plain W4A4 (Q(X) W~ only)"}
                                         if no_res and not f8 else {}),
-                                     **({"scheme": {"rfq8": "RFQ with an MXFP8 residual: MXFP4 X~ + MXFP8 X^, "
+                                     **({"scheme": {"rfq8mix": "RFQ with an MXFP8 residual: MXFP4 X~ x MXFP4 W~ "
+                                                               "on the FP4 path + MXFP8 X^ x W~ as E4M3 on "
+                                                               "the FP8 path, one accumulator",
+                                                    "rfq8": "RFQ with an MXFP8 residual: MXFP4 X~ + MXFP8 X^, "
                                                             "MXFP4 W~, all multiplied as E4M3",
                                                     "w4a8": "W4A8: MXFP8 X x MXFP4 W~ (as E4M3)",
                                                     "w8a8": "W8A8: MXFP8 X x MXFP8 W~"}[scheme]} if f8 else {}),
@@ -921,7 +942,7 @@ def main():
                     help="selective fallback: residual only on 128 x 256 tiles whose max |x| exceeds TAU")
     ap.add_argument("--no-residual", action="store_true",
                     help="plain W4A4: no residual pathway (the baseline the correction is added to)")
-    ap.add_argument("--scheme", default="rfq4", choices=["rfq4", "rfq8", "w4a8", "w8a8"],
+    ap.add_argument("--scheme", default="rfq4", choices=["rfq4", "rfq8", "rfq8mix", "w4a8", "w8a8"],
                     help="rfq4: MXFP4 main + MXFP4 residual (default); rfq8: MXFP8 residual; "
                          "w4a8 / w8a8: MXFP8 activation baselines")
     ap.add_argument("--variant", default="two-kernel", choices=["two-kernel", "fused"],

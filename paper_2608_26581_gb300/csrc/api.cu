@@ -578,6 +578,60 @@ rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, const rfq_
                          static_cast<cudaStream_t>(stream));
 }
 
+rfq_status rfq_linear_mixed(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_t *phi, int32_t phi_r_s,
+                            const rfq_qtensor *wq, const rfq_qtensor *wq8, void *y, int32_t out_dtype,
+                            void *workspace, void *stream)
+{
+    if (!xq || !xr || !wq || !wq8 || !y || !workspace)
+        return RFQ_ERR_INVALID_ARG;
+    if (out_dtype != RFQ_OUT_F32 && out_dtype != RFQ_OUT_BF16)
+        return RFQ_ERR_INVALID_ARG;
+    if (xq->fmt != RFQ_FMT_MXFP4 || wq->fmt != RFQ_FMT_MXFP4 || xr->fmt != RFQ_FMT_MXFP8 ||
+        wq8->fmt != RFQ_FMT_MXFP8)
+        return RFQ_ERR_INVALID_ARG;
+    const int64_t M = xq->rows, K = xq->k, N = wq->rows;
+    if (M < 0 || N < 0 || K <= 0 || wq->k != K || wq8->k != K || wq8->rows != N)
+        return RFQ_ERR_SHAPE;
+    rfq_status s;
+    if ((s = check_qtensor(xq, M, K)) != RFQ_OK || (s = check_qtensor(xr, M, K)) != RFQ_OK ||
+        (s = check_qtensor(wq, N, K)) != RFQ_OK || (s = check_qtensor(wq8, N, K)) != RFQ_OK)
+        return s;
+    if (xq->scale_layout != RFQ_SCALE_MMA || xr->scale_layout != RFQ_SCALE_MMA ||
+        wq->scale_layout != RFQ_SCALE_MMA || wq8->scale_layout != RFQ_SCALE_MMA)
+        return RFQ_ERR_UNSUPPORTED;
+    if (K % 128 != 0 || N % 16 != 0)
+        return RFQ_ERR_SHAPE;
+    if (M > (int64_t)INT32_MAX || N > (int64_t)INT32_MAX || K > (int64_t)INT32_MAX)
+        return RFQ_ERR_SHAPE;
+    if (phi && (phi_r_s < 128 || phi_r_s % 128 != 0))
+        return RFQ_ERR_SHAPE;
+    if (!aligned16(y) || !aligned16(workspace))
+        return RFQ_ERR_ALIGNMENT;
+    if ((s = check_device()) != RFQ_OK)
+        return s;
+    if (M == 0 || N == 0)
+        return RFQ_OK;
+    GemmMxf4Args a;
+    a.a_codes = xq->codes;
+    a.a_sf = xq->scales;
+    a.r_codes = xr->codes;
+    a.r_sf = xr->scales;
+    a.b_codes = wq8->codes;
+    a.b_sf = wq->scales;
+    a.b4_codes = wq->codes;
+    a.phi = phi;
+    a.phi_r_s = phi_r_s;
+    a.y = y;
+    a.out_bf16 = out_dtype == RFQ_OUT_BF16;
+    a.M = M;
+    a.N = N;
+    a.K = K;
+    a.status = static_cast<int32_t *>(workspace);
+    a.f8 = 1;
+    return gemm_done(launch_gemm_mxf4_pair(a, static_cast<cudaStream_t>(stream)), workspace,
+                     static_cast<cudaStream_t>(stream));
+}
+
 rfq_status rfq_linear_profile(const rfq_qtensor *xq, const rfq_qtensor *xr, const rfq_qtensor *wq, void *y,
                               int32_t out_dtype, void *workspace, void *stream)
 {

@@ -189,9 +189,17 @@ struct Mask {
     static constexpr uint32_t value = V;
 };
 
-// F8: every operand holds E4M3 codes (one byte per element, kind::mxf8f6f4
-// MMAs of K = 32 with one scale per row each); a stage is then one
-// 128-element chunk (the same 128-byte rows).
+// F8 (operand form): 0 -- every operand E2M1 (kind::mxf4); 1 -- every
+// operand holds E4M3 codes (one byte per element, kind::mxf8f6f4 MMAs of
+// K = 32 with one scale per row each), a stage is then one 128-element chunk
+// (the same 128-byte rows); 2 -- the FP4-to-FP8 residual at two rates
+// (Sec. 4.2, 4.3): a stage is one 128-element chunk holding X~ and W~ packed
+// (E2M1, 64-byte rows, 64-byte swizzle: the main product on kind::mxf4, two
+// K = 64 MMAs) and X^ and W~ as E4M3 (128-byte rows: the residual product
+// on kind::mxf8f6f4, four K = 32 MMAs), into the same accumulator with the
+// same scale words (W~'s E4M3 form keeps its E8M0 bytes); 48 KB per stage
+// for 768 MMA cycles against 1,024 when the main product also runs as E4M3.
+constexpr int F8_MIXED = 2;
 // GRP: the grouped (mixture-of-experts) form, G groups of rows with their
 // own W~ (row offsets read on the device); the plain form is compiled
 // without any of it.
@@ -201,16 +209,18 @@ struct Mask {
 // waits for a drained accumulator, for a stage's copies and for a stage's
 // scale words, and its stages and tiles, and adds them to the 64-bit
 // workspace words 4..11 (a measurement of where the tensor pipe idles).
-template <bool RES, bool PHI, bool OUT_BF16, bool F8, bool GRP, bool FQ = false, bool PROF = false>
+template <bool RES, bool PHI, bool OUT_BF16, int F8, bool GRP, bool FQ = false, bool PROF = false>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     gemm_mxf4_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmR,
                           const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmY,
+                          const __grid_constant__ CUtensorMap tmB4,
                           const uint8_t *__restrict__ sfa, const uint8_t *__restrict__ sfr,
                           const uint8_t *__restrict__ sfb, const uint8_t *__restrict__ phi, int phi_chunks,
                           int phi_cols, int M, int N, int K, int32_t *status,
                           const int32_t *__restrict__ group_off, int G, void *__restrict__ y, const FqArgs fq)
 {
     static_assert(!FQ || (!PHI && !F8 && !GRP), "the fused quantizer takes plain MXFP4 operands");
+    static_assert(F8 != F8_MIXED || (RES && !GRP && !FQ), "the mixed-rate form is the RFQ with a residual");
     extern __shared__ uint8_t smem_raw[];
     Smem &S = *reinterpret_cast<Smem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -255,6 +265,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
             prefetch_tmap(&tmR);
         prefetch_tmap(&tmB);
         prefetch_tmap(&tmY);
+        if (F8 == F8_MIXED)
+            prefetch_tmap(&tmB4);
     }
     if (warp == 1) {
         tmem_alloc_pair(&S.tmem_base, TMEM_COLS);
@@ -403,12 +415,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     const uint32_t bar = full0 + 8 * slot;
                     const uint32_t sfbytes = (uint32_t)nch * ATOM;
                     uint64_t *sbar = &S.sf_full[slot];
-                    if (lead)
-                        mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES + B_BYTES + (res_on ? A_BYTES : 0)));
-                    tma_load_2d_pair(st.a, &tmA, bar, cx, a_y);
-                    if (res_on)
-                        tma_load_2d_pair(st.r, &tmR, bar, cx, a_y);
-                    tma_load_2d_pair(st.b, &tmB, bar, cx, tc.w_row0 + (int)rank * BN_HALF);
+                    if (F8 == F8_MIXED) {
+                        // X~ and W~ packed (64-byte rows) side by side in the A tile,
+                        // X^ and W~ as E4M3 (128-byte rows) in the R and B tiles
+                        if (lead)
+                            mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES + B_BYTES + (res_on ? A_BYTES : 0)));
+                        tma_load_2d_pair(st.a, &tmA, bar, c0 * 64, a_y);
+                        tma_load_2d_pair(st.a + A_BYTES / 2, &tmB4, bar, c0 * 64, tc.w_row0 + (int)rank * BN_HALF);
+                        if (res_on)
+                            tma_load_2d_pair(st.r, &tmR, bar, cx, a_y);
+                        tma_load_2d_pair(st.b, &tmB, bar, cx, tc.w_row0 + (int)rank * BN_HALF);
+                    } else {
+                        if (lead)
+                            mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES + B_BYTES + (res_on ? A_BYTES : 0)));
+                        tma_load_2d_pair(st.a, &tmA, bar, cx, a_y);
+                        if (res_on)
+                            tma_load_2d_pair(st.r, &tmR, bar, cx, a_y);
+                        tma_load_2d_pair(st.b, &tmB, bar, cx, tc.w_row0 + (int)rank * BN_HALF);
+                    }
                     mbar_arrive_expect_tx(sbar, nb * sfbytes + (rows_in ? (res_on ? 2 : 1) * sfbytes : 0));
                     if (rows_in) {
                         bulk_load(st.sfa, sfa + ((int64_t)sf_tile * kc + c0) * ATOM, sfbytes, sbar);
@@ -509,6 +533,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     const uint32_t sf = tmem + SF_COL0 + SF_SLOT_COLS * sfs;
                     const Stage &st = S.st[slot];
                     const uint32_t a0 = smem_u32(st.a), r0 = smem_u32(st.r), b0 = smem_u32(st.b);
+                    if constexpr (F8 == F8_MIXED) {
+                        // main: X~ W~ packed, two K = 64 kind::mxf4 MMAs (scale bytes 0-1, 2-3)
+#pragma unroll
+                        for (int j = 0; j < 2; ++j)
+                            tc_mma_mxf4_pair(tmem, sdesc_k_sw64(a0 + 32 * j), sdesc_k_sw64(a0 + A_BYTES / 2 + 32 * j),
+                                             idesc_mxf4(2 * BM, BN, 2 * j, 2 * j), sf, sf + 16, (pos | j) != 0);
+                        // residual: X^ W~ as E4M3, four K = 32 kind::mxf8f6f4 MMAs (scale byte j)
+                        if (rm & 1) {
+#pragma unroll
+                            for (int j = 0; j < 4; ++j)
+                                tc_mma_mxf8_pair(tmem, sdesc_k_sw128(r0 + 32 * j), sdesc_k_sw128(b0 + 32 * j),
+                                                 idesc_mxf8(2 * BM, BN, j, j), sf + 8, sf + 16, 1);
+                        }
+                    } else {
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
                         const int c = F8 ? 0 : j >> 1;
@@ -532,6 +570,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                             else
                                 tc_mma_mxf4_pair(tmem, sdesc_k_sw128(r0 + 32 * j), bd, id, sf + 8 + 4 * c, sfb_t, 1);
                         }
+                    }
                     }
                     tc_commit_pair_mc(&S.empty[slot], 0x3);
                     ++p;
@@ -1005,9 +1044,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
     }
 }
 
-template <bool RES, bool PHI, bool OUT, bool F8, bool GRP, bool FQ = false, bool PROF = false>
+template <bool RES, bool PHI, bool OUT, int F8, bool GRP, bool FQ = false, bool PROF = false>
 cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const CUtensorMap &tb,
-                           const CUtensorMap &ty, const GemmMxf4Args &a, cudaStream_t st)
+                           const CUtensorMap &ty, const GemmMxf4Args &a, cudaStream_t st,
+                           const CUtensorMap *tb4 = nullptr)
 {
     auto kern = gemm_mxf4_pair_kernel<RES, PHI, OUT, F8, GRP, FQ, PROF>;
     static int max_pairs = 0; // per variant: clusters of two that fit on the device at once
@@ -1042,7 +1082,7 @@ cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const C
         fq.ring = a.fq_ring;
     }
     kern<<<grid, PHI ? THREADS + 32 : THREADS, kSmemBytes, st>>>(
-        ta, tr, tb, ty, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf, (const uint8_t *)a.b_sf, a.phi, phi_chunks,
+        ta, tr, tb, ty, tb4 ? *tb4 : tb, (const uint8_t *)a.a_sf, (const uint8_t *)a.r_sf, (const uint8_t *)a.b_sf, a.phi, phi_chunks,
         phi_cols, (int)a.M, (int)a.N, (int)a.K, a.status, a.group_off, a.groups, a.y, fq);
     return cudaGetLastError();
 }
@@ -1052,6 +1092,26 @@ cudaError_t launch_variant(const CUtensorMap &ta, const CUtensorMap &tr, const C
 cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
 {
     CUtensorMap ta, tr, tb, ty;
+    if (a.b4_codes) {
+        // the mixed-rate FP4-to-FP8 residual: X~ and W~ packed (64-byte boxes,
+        // 64-byte swizzle), X^ and W~ as E4M3 (128-byte boxes)
+        if (!a.r_codes || a.groups > 0 || a.fq_x || a.prof)
+            return cudaErrorInvalidValue;
+        CUtensorMap tb4;
+        const uint64_t kp = (uint64_t)a.K / 2, k8 = (uint64_t)a.K, yrow = (uint64_t)a.N * (a.out_bf16 ? 2 : 4);
+        if (!encode_tmap_2d_u8(&ta, a.a_codes, kp, (uint64_t)a.M, kp, 64, BM, 64) ||
+            !encode_tmap_2d_u8(&tb4, a.b4_codes, kp, (uint64_t)a.N, kp, 64, BN_HALF, 64) ||
+            !encode_tmap_2d_u8(&tr, a.r_codes, k8, (uint64_t)a.M, k8, ROW, BM, 128) ||
+            !encode_tmap_2d_u8(&tb, a.b_codes, k8, (uint64_t)a.N, k8, ROW, BN_HALF, 128) ||
+            !encode_tmap_2d_u8(&ty, a.y, yrow, (uint64_t)a.M, yrow, 64, 32, 64))
+            return cudaErrorInvalidValue;
+        const bool phi = a.phi != nullptr && a.K / 128 <= REC_WORDS * 32;
+        if (phi)
+            return a.out_bf16 ? launch_variant<true, true, true, F8_MIXED, false>(ta, tr, tb, ty, a, st, &tb4)
+                              : launch_variant<true, true, false, F8_MIXED, false>(ta, tr, tb, ty, a, st, &tb4);
+        return a.out_bf16 ? launch_variant<true, false, true, F8_MIXED, false>(ta, tr, tb, ty, a, st, &tb4)
+                          : launch_variant<true, false, false, F8_MIXED, false>(ta, tr, tb, ty, a, st, &tb4);
+    }
     const uint64_t kb = a.f8 ? (uint64_t)a.K : (uint64_t)a.K / 2; // code bytes per row
     const uint64_t w_rows = (uint64_t)a.N * (a.groups > 0 ? (uint64_t)a.groups : 1u);
     const uint64_t a_rows = a.fq_x ? (uint64_t)a.fq_ring * 2 * BM : (uint64_t)a.M;   // FQ: the ring

@@ -134,6 +134,10 @@ struct GemmMxf4Args {
     int32_t *fq_ctr = nullptr;
     int fq_ring = 0;                           // fused quantizer: 256-row slots of the scratch ring
     int prof = 0;                              // CTA-pair kernel: the MMA thread's counters (rfq_linear_profile)
+    // mixed-rate FP4-to-FP8 residual (CTA-pair kernel): W~ packed [N][K/2];
+    // a_codes / a_sf are then X~ packed, r_codes / r_sf X^ as E4M3, b_codes
+    // W~ as E4M3 (its exact re-encoding), b_sf W~'s scales
+    const void *b4_codes = nullptr;
 };
 
 // Slots of 256 rows in the fused quantizer's scratch ring (rfq_linear_fused).

@@ -31,7 +31,7 @@ EXPORTED = ("rfq_status_string", "rfq_qtensor_bytes", "rfq_quantize_weight", "rf
             "rfq_linear_workspace_bytes", "rfq_linear", "rfq_workspace_status", "rfq_dequant",
             "rfq_linear_noalloc", "rfq_linear_fused", "rfq_convert", "rfq_linear_grouped", "rfq_check_finite",
             "rfq_quantize_act_expand", "rfq_fp4_mma_peak", "rfq_linear_fused_workspace_bytes",
-            "rfq_linear_profile", "rfq_debug_bounds")
+            "rfq_linear_profile", "rfq_debug_bounds", "rfq_linear_mixed")
 
 
 class RFQError(RuntimeError):
@@ -92,6 +92,8 @@ def load_library(path: str = LIB_PATH):
         lib.rfq_linear_grouped.argtypes = [QTP, QTP, P, I32, P, I32, QTP, I64, P, I32, P, P]
         lib.rfq_linear_fused_workspace_bytes.restype = SZ
         lib.rfq_linear_fused_workspace_bytes.argtypes = [I64, I64, ctypes.POINTER(_FB)]
+        lib.rfq_linear_mixed.restype = I32
+        lib.rfq_linear_mixed.argtypes = [QTP, QTP, P, I32, QTP, QTP, P, I32, P, P]
         lib.rfq_debug_bounds.restype = I32
         lib.rfq_debug_bounds.argtypes = [ctypes.POINTER(I32), I32]
         lib.rfq_linear_profile.restype = I32
@@ -203,6 +205,16 @@ def rfq_linear(xq: QTensor, xr: QTensor | None, phi: torch.Tensor | None, phi_r_
     _check(load_library().rfq_linear(ctypes.byref(q), ctypes.byref(r) if r is not None else None, _ptr(phi),
                                      phi_r_s, ctypes.byref(w), _ptr(y), out_dtype, _ptr(workspace),
                                      _stream(stream)), "rfq_linear")
+
+
+def rfq_linear_mixed(xq: QTensor, xr: QTensor, phi: torch.Tensor | None, phi_r_s: int, wq: QTensor, wq8: QTensor,
+                     y: torch.Tensor, out_dtype: int, workspace: torch.Tensor, stream=None):
+    """The FP4-to-FP8 RFQ with the main product at the FP4 rate: X~ (MXFP4),
+    X^ (MXFP8), W~ (MXFP4) and its E4M3 re-encoding wq8 (see include/rfq.h)."""
+    q, r, w, w8 = xq.c(), xr.c(), wq.c(), wq8.c()
+    _check(load_library().rfq_linear_mixed(ctypes.byref(q), ctypes.byref(r), _ptr(phi), phi_r_s, ctypes.byref(w),
+                                           ctypes.byref(w8), _ptr(y), out_dtype, _ptr(workspace),
+                                           _stream(stream)), "rfq_linear_mixed")
 
 
 def rfq_workspace_status(workspace: torch.Tensor, clear: bool = False, stream=None) -> int:

@@ -171,7 +171,9 @@ def test_quantize_act_expand_fp8_residual(orc, layout, mode, tau):
 
 def _gemm_case(orc, M, K, N, kind, out=rfq.RFQ_OUT_F32, mode=rfq.RFQ_FALLBACK_ALL, tau=0.0, r_s=256, seed=1,
                rows=None, xb=None, wb=None):
-    """kind: 'w8a8', 'w4a8' or 'rfq8' (MXFP4 main + MXFP8 residual)."""
+    """kind: 'w8a8', 'w4a8', 'rfq8' (MXFP4 main + MXFP8 residual, both
+    products as E4M3) or 'rfq8mix' (the same RFQ through rfq_linear_mixed:
+    the main product on the FP4 path, the residual on the FP8 one)."""
     if xb is None:
         xb = make_activation(ActSpec(M, K, "normal", chan_count=3, chan_scale=64.0, tok_count=1, tok_scale=200.0,
                                      seed=seed))
@@ -207,9 +209,12 @@ def _gemm_case(orc, M, K, N, kind, out=rfq.RFQ_OUT_F32, mode=rfq.RFQ_FALLBACK_AL
         xr = rfq.empty_qtensor(F8, MMA, M, K)
         phi = torch.empty(((M + 127) // 128) * ((K + r_s - 1) // r_s), dtype=torch.uint8, device=DEV)
         rfq.rfq_quantize_act(x, x4, xr, phi, mode=mode, tau=tau, p_s=128, r_s=r_s)
-        xq = rfq.empty_qtensor(F8, MMA, M, K)
-        rfq.rfq_convert(x4, xq)
-        rfq.rfq_linear(xq, xr, phi if mode == rfq.RFQ_FALLBACK_AMAX else None, r_s, wq, y, out, ws)
+        if kind == "rfq8mix":
+            rfq.rfq_linear_mixed(x4, xr, phi if mode == rfq.RFQ_FALLBACK_AMAX else None, r_s, w4, wq, y, out, ws)
+        else:
+            xq = rfq.empty_qtensor(F8, MMA, M, K)
+            rfq.rfq_convert(x4, xq)
+            rfq.rfq_linear(xq, xr, phi if mode == rfq.RFQ_FALLBACK_AMAX else None, r_s, wq, y, out, ws)
         q = orc.quantize_act(xb, orc.FMT_MXFP4, mode, tau, 128, r_s, res_fmt=orc.FMT_MXFP8)
         sel = slice(None) if rows is None else rows
         ref = orc.linear(orc.FMT_MXFP4, q["main_codes"][sel], q["main_scales"][sel], q["res_codes"][sel],
@@ -221,20 +226,49 @@ def _gemm_case(orc, M, K, N, kind, out=rfq.RFQ_OUT_F32, mode=rfq.RFQ_FALLBACK_AL
     return yh
 
 
-@pytest.mark.parametrize("kind", ["w8a8", "w4a8", "rfq8"])
+@pytest.mark.parametrize("kind", ["w8a8", "w4a8", "rfq8", "rfq8mix"])
 @pytest.mark.parametrize("M,K,N", [(1, 128, 16), (128, 512, 256), (129, 384, 272), (300, 640, 528),
                                    (513, 1024, 784)])
 def test_linear_mxfp8_shapes(orc, kind, M, K, N):
     _gemm_case(orc, M, K, N, kind, seed=M + N)
 
 
+@pytest.mark.parametrize("kind", ["rfq8", "rfq8mix"])
 @pytest.mark.parametrize("r_s,tau", [(128, 30.0), (256, 30.0), (256, 1e30)])
-def test_linear_fp8_residual_selective_phi(orc, r_s, tau):
-    _gemm_case(orc, 384, 1152, 512, "rfq8", mode=rfq.RFQ_FALLBACK_AMAX, tau=tau, r_s=r_s, seed=11)
+def test_linear_fp8_residual_selective_phi(orc, kind, r_s, tau):
+    _gemm_case(orc, 384, 1152, 512, kind, mode=rfq.RFQ_FALLBACK_AMAX, tau=tau, r_s=r_s, seed=11)
 
 
-def test_linear_mxfp8_bf16_output(orc):
-    _gemm_case(orc, 256, 1024, 512, "rfq8", out=rfq.RFQ_OUT_BF16, seed=5)
+@pytest.mark.parametrize("kind", ["rfq8", "rfq8mix"])
+def test_linear_mxfp8_bf16_output(orc, kind):
+    _gemm_case(orc, 256, 1024, 512, kind, out=rfq.RFQ_OUT_BF16, seed=5)
+
+
+def test_mixed_rate_matches_all_e4m3_path(orc):
+    """The two ways of multiplying the FP4-to-FP8 RFQ give the same Y up to
+    fp32 accumulation order: every product is exact in both (E2M1 values are
+    E4M3 values), so both match the oracle and each other within the
+    tolerance, on ragged shapes with more tiles than CTA pairs."""
+    M, K, N = 1000, 1280, 1040
+    y8 = _gemm_case(orc, M, K, N, "rfq8", seed=21)
+    ym = _gemm_case(orc, M, K, N, "rfq8mix", seed=21)
+    check_y(ym, y8)
+
+
+def test_mixed_rate_host_checks():
+    """rfq_linear_mixed wants MXFP4 X~ and W~, MXFP8 X^ and W~ (E4M3), one K."""
+    M, K, N = 256, 256, 256
+    x4, w4 = rfq.empty_qtensor(F4, MMA, M, K), rfq.empty_qtensor(F4, MMA, N, K)
+    x8, w8 = rfq.empty_qtensor(F8, MMA, M, K), rfq.empty_qtensor(F8, MMA, N, K)
+    y = torch.empty(M, N, device=DEV)
+    ws = torch.zeros(64, dtype=torch.int32, device=DEV)
+    for args in ((x8, x8, w4, w8), (x4, x4, w4, w8), (x4, x8, w8, w8), (x4, x8, w4, w4)):
+        with pytest.raises(rfq.RFQError) as e:
+            rfq.rfq_linear_mixed(args[0], args[1], None, 256, args[2], args[3], y, rfq.RFQ_OUT_F32, ws)
+        assert e.value.status == rfq.RFQ_ERR_INVALID_ARG
+    with pytest.raises(rfq.RFQError) as e:
+        rfq.rfq_linear_mixed(x4, x8, None, 256, w4, rfq.empty_qtensor(F8, MMA, N, 512), y, rfq.RFQ_OUT_F32, ws)
+    assert e.value.status == rfq.RFQ_ERR_SHAPE
 
 
 def test_fp8_residual_is_closer_than_fp4_residual(orc):
@@ -258,7 +292,7 @@ def test_fp8_residual_is_closer_than_fp4_residual(orc):
     assert e8 < e4 < e0, (e8, e4, e0)
 
 
-@pytest.mark.parametrize("kind", ["w4a8", "rfq8"])
+@pytest.mark.parametrize("kind", ["w4a8", "rfq8", "rfq8mix"])
 def test_full_size_wan_ffn_up_mxfp8(orc, kind):
     spec = WORKLOADS["wan_ffn_up"]
     M, K, N = spec.act.M, spec.act.K, spec.N
@@ -285,9 +319,12 @@ def test_full_size_wan_ffn_up_mxfp8(orc, kind):
         x4 = rfq.empty_qtensor(F4, MMA, M, K)
         xr = rfq.empty_qtensor(F8, MMA, M, K)
         rfq.rfq_quantize_act(x, x4, xr, None)
-        xq = rfq.empty_qtensor(F8, MMA, M, K)
-        rfq.rfq_convert(x4, xq)
-        rfq.rfq_linear(xq, xr, None, 256, w8, y, rfq.RFQ_OUT_BF16, ws)
+        if kind == "rfq8mix":
+            rfq.rfq_linear_mixed(x4, xr, None, 256, w4, w8, y, rfq.RFQ_OUT_BF16, ws)
+        else:
+            xq = rfq.empty_qtensor(F8, MMA, M, K)
+            rfq.rfq_convert(x4, xq)
+            rfq.rfq_linear(xq, xr, None, 256, w8, y, rfq.RFQ_OUT_BF16, ws)
         q = orc.quantize_act(xb[rows], orc.FMT_MXFP4, orc.PHI_ALL, res_fmt=orc.FMT_MXFP8)
         ref = orc.linear(orc.FMT_MXFP4, q["main_codes"], q["main_scales"], q["res_codes"], q["res_scales"], *wref,
                          len(rows), K, N, res_fmt=orc.FMT_MXFP8, w_fmt=orc.FMT_MXFP4)
