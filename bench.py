@@ -432,7 +432,8 @@ def run_rfq(args):
     #         w8a8: MXFP8 X x MXFP8 W.  All on kind::mxf8f6f4.
     #   rfq8mix: the rfq8 RFQ through rfq_linear_mixed -- the main product
     #         on kind::mxf4 (X~ and W~ packed), the residual on
-    #         kind::mxf8f6f4 (X^ and W~ as E4M3); no E4M3 copy of X~.
+    #         kind::mxf8f6f4 (X^ as E4M3, W~ expanded from its packed codes
+    #         by the copy engine); no E4M3 copy of X~ or W~.
     scheme = args.scheme
     mixed = scheme == "rfq8mix"
     f8 = scheme != "rfq4"
@@ -473,7 +474,7 @@ def run_rfq(args):
         w = torch.from_numpy(wb.view(np.int16)).to(dev).view(torch.bfloat16)
         wq = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme == "w8a8" else F, L, NW, K, device=dev)
         rfq.rfq_quantize_weight(w, wq)                     # offline weight step, untimed
-        if scheme in ("rfq8", "w4a8", "rfq8mix"):
+        if scheme in ("rfq8", "w4a8"):
             wop = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8, L, NW, K, device=dev)
             rfq.rfq_convert(wq, wop)                       # exact E4M3 re-encoding of W~ (offline)
         elif hif4:
@@ -564,7 +565,7 @@ def run_rfq(args):
             rfq.rfq_linear_grouped(xq8 if xq8 is not None else xq, xr, ph, 256, group_off,
                                    wop, N, y_, rfq.RFQ_OUT_BF16, wsp, stream=None)
         elif mixed:
-            rfq.rfq_linear_mixed(xq, xr, ph, 256, wq, wop, y_, rfq.RFQ_OUT_BF16, wsp, stream=None)
+            rfq.rfq_linear_mixed(xq, xr, ph, 256, wq, y_, rfq.RFQ_OUT_BF16, wsp, stream=None)
         else:
             rfq.rfq_linear(xq8 if xq8 is not None else xq, xr, ph, 256, wop, y_, rfq.RFQ_OUT_BF16, wsp,
                            stream=None)

@@ -341,20 +341,21 @@ RFQ_API rfq_status rfq_fp4_mma_peak(int32_t cta_pair, int64_t iters, void *works
  * pathway with the Sec. 3.2.1 format; Algorithm 1, Eq. rfq):
  *     Y = X~ W~ + phi X^ W~
  * with the main product X~ W~ on the FP4 tensor path (E2M1 x E2M1) and the
- * residual product X^ W~ on the FP8 one (E4M3 x E4M3), into one fp32
+ * residual product X^ W~ on the FP8 one (E4M3 x E2M1), into one fp32
  * accumulator per output tile.  xq: X~, MXFP4 [M x K]; xr: X^, MXFP8 [M x K]
  * (rfq_quantize_act with an MXFP8 residual writes both); wq: W~, MXFP4
- * [N x K]; wq8: the exact E4M3 re-encoding of wq (rfq_convert), which keeps
- * wq's scale bytes -- the call reads W~'s scales from wq.  Every operand
- * with RFQ_SCALE_MMA scales; K % 128 == 0, N % 16 == 0, M >= 0 (CTA pairs
- * at every M).  phi, phi_r_s, y, out_dtype, workspace: as for rfq_linear.
- * rfq_linear multiplies the same operands with X~ re-encoded as E4M3 too,
- * the main product then at the FP8 rate.
+ * [N x K], its codes 32-byte aligned: the kernel reads them twice per
+ * k-stage, packed for the main product and expanded by the copy engine to
+ * one byte per code for the residual one (no second copy of W~ in memory).
+ * Every operand with RFQ_SCALE_MMA scales; K % 128 == 0, N % 16 == 0,
+ * M >= 0 (CTA pairs at every M).  phi, phi_r_s, y, out_dtype, workspace: as
+ * for rfq_linear.  rfq_linear multiplies the same RFQ with X~ and W~
+ * re-encoded as E4M3 (rfq_convert), both products then at the FP8 rate.
  * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
  * RFQ_ERR_UNSUPPORTED, RFQ_ERR_CUDA, RFQ_ERR_DEVICE. */
 RFQ_API rfq_status rfq_linear_mixed(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_t *phi,
-                                    int32_t phi_r_s, const rfq_qtensor *wq, const rfq_qtensor *wq8, void *y,
-                                    int32_t out_dtype, void *workspace, void *stream);
+                                    int32_t phi_r_s, const rfq_qtensor *wq, void *y, int32_t out_dtype,
+                                    void *workspace, void *stream);
 
 /* Measurement of where the RFQ GEMM's tensor pipe idles: rfq_linear
  * (Algorithm 1, Eq. rfq) for MXFP4 operands with a residual and no phi,

@@ -155,6 +155,22 @@ bool encode_tmap_2d_u8(CUtensorMap *map, const void *base, uint64_t inner_bytes,
     return r == CUDA_SUCCESS;
 }
 
+bool encode_tmap_2d_e2m1_padded(CUtensorMap *map, const void *base, uint64_t k, uint64_t rows,
+                                uint32_t box_rows)
+{
+    PFN_encodeTiled enc = get_encode();
+    if (!enc || (reinterpret_cast<uintptr_t>(base) & 31u) != 0 || k % 128 != 0)
+        return false;
+    cuuint64_t dims[2] = {k, rows};         // in 4-bit codes
+    cuuint64_t strides[1] = {k / 2};        // bytes
+    cuuint32_t box[2] = {128, box_rows};    // 128 codes: 64 bytes read, 128 written
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_16U4_ALIGN16B, 2, const_cast<void *>(base), dims, strides, box,
+                     estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 } // namespace rfq
 
 using namespace rfq;
@@ -579,25 +595,22 @@ rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, const rfq_
 }
 
 rfq_status rfq_linear_mixed(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_t *phi, int32_t phi_r_s,
-                            const rfq_qtensor *wq, const rfq_qtensor *wq8, void *y, int32_t out_dtype,
-                            void *workspace, void *stream)
+                            const rfq_qtensor *wq, void *y, int32_t out_dtype, void *workspace, void *stream)
 {
-    if (!xq || !xr || !wq || !wq8 || !y || !workspace)
+    if (!xq || !xr || !wq || !y || !workspace)
         return RFQ_ERR_INVALID_ARG;
     if (out_dtype != RFQ_OUT_F32 && out_dtype != RFQ_OUT_BF16)
         return RFQ_ERR_INVALID_ARG;
-    if (xq->fmt != RFQ_FMT_MXFP4 || wq->fmt != RFQ_FMT_MXFP4 || xr->fmt != RFQ_FMT_MXFP8 ||
-        wq8->fmt != RFQ_FMT_MXFP8)
+    if (xq->fmt != RFQ_FMT_MXFP4 || wq->fmt != RFQ_FMT_MXFP4 || xr->fmt != RFQ_FMT_MXFP8)
         return RFQ_ERR_INVALID_ARG;
     const int64_t M = xq->rows, K = xq->k, N = wq->rows;
-    if (M < 0 || N < 0 || K <= 0 || wq->k != K || wq8->k != K || wq8->rows != N)
+    if (M < 0 || N < 0 || K <= 0 || wq->k != K)
         return RFQ_ERR_SHAPE;
     rfq_status s;
     if ((s = check_qtensor(xq, M, K)) != RFQ_OK || (s = check_qtensor(xr, M, K)) != RFQ_OK ||
-        (s = check_qtensor(wq, N, K)) != RFQ_OK || (s = check_qtensor(wq8, N, K)) != RFQ_OK)
+        (s = check_qtensor(wq, N, K)) != RFQ_OK)
         return s;
-    if (xq->scale_layout != RFQ_SCALE_MMA || xr->scale_layout != RFQ_SCALE_MMA ||
-        wq->scale_layout != RFQ_SCALE_MMA || wq8->scale_layout != RFQ_SCALE_MMA)
+    if (xq->scale_layout != RFQ_SCALE_MMA || xr->scale_layout != RFQ_SCALE_MMA || wq->scale_layout != RFQ_SCALE_MMA)
         return RFQ_ERR_UNSUPPORTED;
     if (K % 128 != 0 || N % 16 != 0)
         return RFQ_ERR_SHAPE;
@@ -605,7 +618,9 @@ rfq_status rfq_linear_mixed(const rfq_qtensor *xq, const rfq_qtensor *xr, const 
         return RFQ_ERR_SHAPE;
     if (phi && (phi_r_s < 128 || phi_r_s % 128 != 0))
         return RFQ_ERR_SHAPE;
-    if (!aligned16(y) || !aligned16(workspace))
+    // W~'s codes feed a TMA copy of the padded 4-bit type, which wants a
+    // 32-byte aligned base
+    if (!aligned16(y) || !aligned16(workspace) || (reinterpret_cast<uintptr_t>(wq->codes) & 31u) != 0)
         return RFQ_ERR_ALIGNMENT;
     if ((s = check_device()) != RFQ_OK)
         return s;
@@ -616,7 +631,7 @@ rfq_status rfq_linear_mixed(const rfq_qtensor *xq, const rfq_qtensor *xr, const 
     a.a_sf = xq->scales;
     a.r_codes = xr->codes;
     a.r_sf = xr->scales;
-    a.b_codes = wq8->codes;
+    a.b_codes = wq->codes;
     a.b_sf = wq->scales;
     a.b4_codes = wq->codes;
     a.phi = phi;

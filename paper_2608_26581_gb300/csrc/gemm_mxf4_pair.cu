@@ -416,15 +416,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     const uint32_t sfbytes = (uint32_t)nch * ATOM;
                     uint64_t *sbar = &S.sf_full[slot];
                     if (F8 == F8_MIXED) {
-                        // X~ and W~ packed (64-byte rows) side by side in the A tile,
-                        // X^ and W~ as E4M3 (128-byte rows) in the R and B tiles
+                        // X~ and W~ packed (64-byte rows) side by side in the A tile;
+                        // with a residual, X^ as E4M3 in the R tile and W~ again, from
+                        // the same packed codes, in the padded 4-bit form in the B tile
+                        // (128-byte rows, 64 bytes read per row; its x counts codes)
                         if (lead)
-                            mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES + B_BYTES + (res_on ? A_BYTES : 0)));
+                            mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES + (res_on ? A_BYTES + B_BYTES / 2 : 0)));
                         tma_load_2d_pair(st.a, &tmA, bar, c0 * 64, a_y);
                         tma_load_2d_pair(st.a + A_BYTES / 2, &tmB4, bar, c0 * 64, tc.w_row0 + (int)rank * BN_HALF);
-                        if (res_on)
+                        if (res_on) {
                             tma_load_2d_pair(st.r, &tmR, bar, cx, a_y);
-                        tma_load_2d_pair(st.b, &tmB, bar, cx, tc.w_row0 + (int)rank * BN_HALF);
+                            tma_load_2d_pair(st.b, &tmB, bar, cx, tc.w_row0 + (int)rank * BN_HALF);
+                        }
                     } else {
                         if (lead)
                             mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES + B_BYTES + (res_on ? A_BYTES : 0)));
@@ -539,12 +542,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                         for (int j = 0; j < 2; ++j)
                             tc_mma_mxf4_pair(tmem, sdesc_k_sw64(a0 + 32 * j), sdesc_k_sw64(a0 + A_BYTES / 2 + 32 * j),
                                              idesc_mxf4(2 * BM, BN, 2 * j, 2 * j), sf, sf + 16, (pos | j) != 0);
-                        // residual: X^ W~ as E4M3, four K = 32 kind::mxf8f6f4 MMAs (scale byte j)
+                        // residual: X^ (E4M3) times W~ (padded E2M1), four K = 32
+                        // kind::mxf8f6f4 MMAs (scale byte j)
                         if (rm & 1) {
 #pragma unroll
                             for (int j = 0; j < 4; ++j)
                                 tc_mma_mxf8_pair(tmem, sdesc_k_sw128(r0 + 32 * j), sdesc_k_sw128(b0 + 32 * j),
-                                                 idesc_mxf8(2 * BM, BN, j, j), sf + 8, sf + 16, 1);
+                                                 idesc_mxf8_e4m3_e2m1(2 * BM, BN, j, j), sf + 8, sf + 16, 1);
                         }
                     } else {
 #pragma unroll
@@ -1094,7 +1098,8 @@ cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
     CUtensorMap ta, tr, tb, ty;
     if (a.b4_codes) {
         // the mixed-rate FP4-to-FP8 residual: X~ and W~ packed (64-byte boxes,
-        // 64-byte swizzle), X^ and W~ as E4M3 (128-byte boxes)
+        // 64-byte swizzle), X^ as E4M3 (128-byte boxes), W~ once more from
+        // the same codes in the padded 4-bit form (128-code boxes)
         if (!a.r_codes || a.groups > 0 || a.fq_x || a.prof)
             return cudaErrorInvalidValue;
         CUtensorMap tb4;
@@ -1102,7 +1107,7 @@ cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
         if (!encode_tmap_2d_u8(&ta, a.a_codes, kp, (uint64_t)a.M, kp, 64, BM, 64) ||
             !encode_tmap_2d_u8(&tb4, a.b4_codes, kp, (uint64_t)a.N, kp, 64, BN_HALF, 64) ||
             !encode_tmap_2d_u8(&tr, a.r_codes, k8, (uint64_t)a.M, k8, ROW, BM, 128) ||
-            !encode_tmap_2d_u8(&tb, a.b_codes, k8, (uint64_t)a.N, k8, ROW, BN_HALF, 128) ||
+            !encode_tmap_2d_e2m1_padded(&tb, a.b4_codes, k8, (uint64_t)a.N, BN_HALF) ||
             !encode_tmap_2d_u8(&ty, a.y, yrow, (uint64_t)a.M, yrow, 64, 32, 64))
             return cudaErrorInvalidValue;
         const bool phi = a.phi != nullptr && a.K / 128 <= REC_WORDS * 32;

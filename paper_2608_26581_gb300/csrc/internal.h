@@ -191,6 +191,12 @@ cudaError_t launch_gemm_hif4(const GemmHif4Args &a, cudaStream_t st);
 // swizzle: 0 none, 64 or 128 (bytes)
 bool encode_tmap_2d_u8(CUtensorMap *map, const void *base, uint64_t inner_bytes, uint64_t rows,
                        uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows, int swizzle);
+// Packed E2M1 codes [rows x k] (k % 128 == 0, base 32-byte aligned) loaded
+// in 128-code boxes as the padded 4-bit form that kind::mxf8f6f4 reads (16
+// codes in 8 bytes, then 8 bytes of gap: 128-byte rows), 128-byte swizzle.
+// A box's copy counts the 64 bytes per row it reads toward complete_tx.
+bool encode_tmap_2d_e2m1_padded(CUtensorMap *map, const void *base, uint64_t k, uint64_t rows,
+                                uint32_t box_rows);
 
 // ---- the dense FP4 MMA rate alone (mma_peak.cu): `iters` MMAs per SM (pair
 // = 0, 128 x 256 x 64) or per CTA pair (pair = 1, 256 x 256 x 64); *flop =

@@ -527,6 +527,17 @@ __host__ __device__ constexpr uint32_t idesc_mxf8(int M, int N, int sfa_id, int 
            ((uint32_t)(M >> 4) << 24) | ((uint32_t)sfa_id << 29);
 }
 
+// Instruction descriptor, kind::mxf8f6f4 with A E4M3 (format code 0) and B
+// E2M1 (format code 5), UE8M0 scales, both K-major.  B sits in shared memory
+// in the padded 4-bit form (16 codes in 8 bytes, then 8 bytes of gap: one
+// byte of shared memory per element, as E4M3), which a TMA load of type
+// 16U4_ALIGN16B writes from the packed codes; sfa_id / sfb_id as above.
+__host__ __device__ constexpr uint32_t idesc_mxf8_e4m3_e2m1(int M, int N, int sfa_id, int sfb_id)
+{
+    return ((uint32_t)sfb_id << 4) | (0u << 7) | (5u << 10) | ((uint32_t)(N >> 3) << 17) | (1u << 23) |
+           ((uint32_t)(M >> 4) << 24) | ((uint32_t)sfa_id << 29);
+}
+
 // Instruction descriptor, kind::f16: bf16 x bf16 -> fp32, K-major operands.
 __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N)
 {

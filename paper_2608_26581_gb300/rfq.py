@@ -93,7 +93,7 @@ def load_library(path: str = LIB_PATH):
         lib.rfq_linear_fused_workspace_bytes.restype = SZ
         lib.rfq_linear_fused_workspace_bytes.argtypes = [I64, I64, ctypes.POINTER(_FB)]
         lib.rfq_linear_mixed.restype = I32
-        lib.rfq_linear_mixed.argtypes = [QTP, QTP, P, I32, QTP, QTP, P, I32, P, P]
+        lib.rfq_linear_mixed.argtypes = [QTP, QTP, P, I32, QTP, P, I32, P, P]
         lib.rfq_debug_bounds.restype = I32
         lib.rfq_debug_bounds.argtypes = [ctypes.POINTER(I32), I32]
         lib.rfq_linear_profile.restype = I32
@@ -207,14 +207,14 @@ def rfq_linear(xq: QTensor, xr: QTensor | None, phi: torch.Tensor | None, phi_r_
                                      _stream(stream)), "rfq_linear")
 
 
-def rfq_linear_mixed(xq: QTensor, xr: QTensor, phi: torch.Tensor | None, phi_r_s: int, wq: QTensor, wq8: QTensor,
+def rfq_linear_mixed(xq: QTensor, xr: QTensor, phi: torch.Tensor | None, phi_r_s: int, wq: QTensor,
                      y: torch.Tensor, out_dtype: int, workspace: torch.Tensor, stream=None):
     """The FP4-to-FP8 RFQ with the main product at the FP4 rate: X~ (MXFP4),
-    X^ (MXFP8), W~ (MXFP4) and its E4M3 re-encoding wq8 (see include/rfq.h)."""
-    q, r, w, w8 = xq.c(), xr.c(), wq.c(), wq8.c()
+    X^ (MXFP8), W~ (MXFP4, codes 32-byte aligned; see include/rfq.h)."""
+    q, r, w = xq.c(), xr.c(), wq.c()
     _check(load_library().rfq_linear_mixed(ctypes.byref(q), ctypes.byref(r), _ptr(phi), phi_r_s, ctypes.byref(w),
-                                           ctypes.byref(w8), _ptr(y), out_dtype, _ptr(workspace),
-                                           _stream(stream)), "rfq_linear_mixed")
+                                           _ptr(y), out_dtype, _ptr(workspace), _stream(stream)),
+           "rfq_linear_mixed")
 
 
 def rfq_workspace_status(workspace: torch.Tensor, clear: bool = False, stream=None) -> int:

@@ -210,7 +210,7 @@ def _gemm_case(orc, M, K, N, kind, out=rfq.RFQ_OUT_F32, mode=rfq.RFQ_FALLBACK_AL
         phi = torch.empty(((M + 127) // 128) * ((K + r_s - 1) // r_s), dtype=torch.uint8, device=DEV)
         rfq.rfq_quantize_act(x, x4, xr, phi, mode=mode, tau=tau, p_s=128, r_s=r_s)
         if kind == "rfq8mix":
-            rfq.rfq_linear_mixed(x4, xr, phi if mode == rfq.RFQ_FALLBACK_AMAX else None, r_s, w4, wq, y, out, ws)
+            rfq.rfq_linear_mixed(x4, xr, phi if mode == rfq.RFQ_FALLBACK_AMAX else None, r_s, w4, y, out, ws)
         else:
             xq = rfq.empty_qtensor(F8, MMA, M, K)
             rfq.rfq_convert(x4, xq)
@@ -256,19 +256,27 @@ def test_mixed_rate_matches_all_e4m3_path(orc):
 
 
 def test_mixed_rate_host_checks():
-    """rfq_linear_mixed wants MXFP4 X~ and W~, MXFP8 X^ and W~ (E4M3), one K."""
+    """rfq_linear_mixed wants MXFP4 X~ and W~, an MXFP8 X^, one K, and W~'s
+    codes on a 32-byte boundary (the padded 4-bit copy's rule)."""
     M, K, N = 256, 256, 256
     x4, w4 = rfq.empty_qtensor(F4, MMA, M, K), rfq.empty_qtensor(F4, MMA, N, K)
     x8, w8 = rfq.empty_qtensor(F8, MMA, M, K), rfq.empty_qtensor(F8, MMA, N, K)
     y = torch.empty(M, N, device=DEV)
     ws = torch.zeros(64, dtype=torch.int32, device=DEV)
-    for args in ((x8, x8, w4, w8), (x4, x4, w4, w8), (x4, x8, w8, w8), (x4, x8, w4, w4)):
+    for args in ((x8, x8, w4), (x4, x4, w4), (x4, x8, w8)):
         with pytest.raises(rfq.RFQError) as e:
-            rfq.rfq_linear_mixed(args[0], args[1], None, 256, args[2], args[3], y, rfq.RFQ_OUT_F32, ws)
+            rfq.rfq_linear_mixed(args[0], args[1], None, 256, args[2], y, rfq.RFQ_OUT_F32, ws)
         assert e.value.status == rfq.RFQ_ERR_INVALID_ARG
     with pytest.raises(rfq.RFQError) as e:
-        rfq.rfq_linear_mixed(x4, x8, None, 256, w4, rfq.empty_qtensor(F8, MMA, N, 512), y, rfq.RFQ_OUT_F32, ws)
+        rfq.rfq_linear_mixed(x4, x8, None, 256, rfq.empty_qtensor(F4, MMA, N, 512), y, rfq.RFQ_OUT_F32, ws)
     assert e.value.status == rfq.RFQ_ERR_SHAPE
+    # the same W~ codes 16 bytes off a 32-byte boundary
+    buf = torch.zeros(w4.codes.numel() + 16, dtype=torch.uint8, device=DEV)
+    assert buf.data_ptr() % 32 == 0
+    w_off = rfq.QTensor(w4.fmt, w4.scale_layout, N, K, buf[16:16 + w4.codes.numel()], w4.scales)
+    with pytest.raises(rfq.RFQError) as e:
+        rfq.rfq_linear_mixed(x4, x8, None, 256, w_off, y, rfq.RFQ_OUT_F32, ws)
+    assert e.value.status == rfq.RFQ_ERR_ALIGNMENT
 
 
 def test_fp8_residual_is_closer_than_fp4_residual(orc):
@@ -320,7 +328,7 @@ def test_full_size_wan_ffn_up_mxfp8(orc, kind):
         xr = rfq.empty_qtensor(F8, MMA, M, K)
         rfq.rfq_quantize_act(x, x4, xr, None)
         if kind == "rfq8mix":
-            rfq.rfq_linear_mixed(x4, xr, None, 256, w4, w8, y, rfq.RFQ_OUT_BF16, ws)
+            rfq.rfq_linear_mixed(x4, xr, None, 256, w4, y, rfq.RFQ_OUT_BF16, ws)
         else:
             xq = rfq.empty_qtensor(F8, MMA, M, K)
             rfq.rfq_convert(x4, xq)
