@@ -11,8 +11,10 @@
 // slots with tcgen05.st (a scale copy issued by the MMA thread would wait for
 // its earlier MMAs).  With four slots and three stages, a slot is rewritten
 // only after its previous stage's MMAs completed: the writers wait for the
-// stage's copies, which the producer issued after those MMAs released the
-// shared-memory stage.  The MMA
+// stage's scale copies (issued ahead of its operand tiles, on a barrier of
+// their own, so that the scale words reach TMEM while the tiles still land),
+// which the producer issued after those MMAs released the shared-memory
+// stage.  The MMA
 // thread issues, per K=64 step, the main MMA and the residual MMA against the
 // SAME shared-memory W~ tile into the SAME TMEM accumulator: W~ is read once
 // for both products and the correction costs only MMA issue (the on-the-fly
@@ -94,7 +96,8 @@ struct PhiRec {
 struct Smem {
     Stage st[STAGES];
     alignas(1024) uint8_t ystage[EPI_WARPS * YSTAGE]; // 64B-swizzled staging for the TMA stores of Y
-    uint64_t full[STAGES];
+    uint64_t full[STAGES];            // a stage's operand tiles landed
+    uint64_t sf_full[STAGES];         // a stage's scale atoms landed (issued first, awaited apart)
     uint64_t empty[STAGES];
     uint64_t acc_full;
     uint64_t acc_empty;
@@ -176,6 +179,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&S.full[s], 1);
+            mbar_init(&S.sf_full[s], 1);
             mbar_init(&S.empty[s], 1);
         }
         mbar_init(&S.acc_full, 1);
@@ -303,18 +307,21 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                         S.stage_info[slot] = info;
                     const uint32_t sfbytes = (uint32_t)nch * ATOM;
                     Stage &st = S.st[slot];
+                    // the scale atoms first, on their own barrier: the scale
+                    // writers move them into TMEM while the operand tiles land
+                    uint64_t *sbar = &S.sf_full[slot];
+                    mbar_arrive_expect_tx(sbar, (1 + nb) * sfbytes + (res_on ? sfbytes : 0));
+                    bulk_load(st.sfa, sfa + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, sbar);
+                    if (res_on)
+                        bulk_load(st.sfr, sfr + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, sbar);
+                    for (int h = 0; h < nb; ++h)
+                        bulk_load(st.sfb + h * 2 * ATOM, sfb + ((int64_t)(atom0 + h) * kc + c0) * ATOM, sfbytes, sbar);
                     uint64_t *bar = &S.full[slot];
-                    mbar_arrive_expect_tx(bar, A_BYTES + B_BYTES + (1 + nb) * sfbytes +
-                                                   (res_on ? A_BYTES + sfbytes : 0));
+                    mbar_arrive_expect_tx(bar, A_BYTES + B_BYTES + (res_on ? A_BYTES : 0));
                     tma_load_2d(st.a, &tmA, bar, c0 * 64, tc.a_row0);
                     if (res_on)
                         tma_load_2d(st.r, &tmR, bar, c0 * 64, tc.a_row0);
                     tma_load_2d(st.b, &tmB, bar, c0 * 64, tc.w_row0);
-                    bulk_load(st.sfa, sfa + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, bar);
-                    if (res_on)
-                        bulk_load(st.sfr, sfr + ((int64_t)m_tile * kc + c0) * ATOM, sfbytes, bar);
-                    for (int h = 0; h < nb; ++h)
-                        bulk_load(st.sfb + h * 2 * ATOM, sfb + ((int64_t)(atom0 + h) * kc + c0) * ATOM, sfbytes, bar);
                     ++p;
                 };
                 if constexpr (!PHI) {
@@ -589,7 +596,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                 constexpr uint32_t rm = decltype(rm_t)::value;
                 const int slot = p % STAGES, sfs = p % SF_SLOTS;
                 // warp-uniform outcome: the tcgen05 stores below need the whole warp
-                if (!__all_sync(0xffffffffu, mbar_wait(&S.full[slot], (p / STAGES) & 1, wl, gstat))) {
+                if (!__all_sync(0xffffffffu, mbar_wait(&S.sf_full[slot], (p / STAGES) & 1, wl, gstat))) {
                     if (lane == 0)
                         flag_timeout(S, status);
                     stop = true;
@@ -628,7 +635,7 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
                     write_stage(1, Mask<RES ? 1u : 0u>{});
             } else {
                 // the tile's residual-stage count arrives with its first stage
-                if (!__all_sync(0xffffffffu, mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, wl, gstat))) {
+                if (!__all_sync(0xffffffffu, mbar_wait(&S.sf_full[p % STAGES], (p / STAGES) & 1, wl, gstat))) {
                     if (lane == 0)
                         flag_timeout(S, status);
                     break;
@@ -687,8 +694,10 @@ __global__ void __launch_bounds__(PHI ? THREADS + 32 : THREADS, 1)
     if (threadIdx.x == 0 && S.abort_flag) {
         // wait (bounded) for the copies of the last stages still in flight
         const int issued = S.issued;
-        for (int p = max(0, issued - STAGES); p < issued; ++p)
+        for (int p = max(0, issued - STAGES); p < issued; ++p) {
             (void)mbar_wait(&S.full[p % STAGES], (p / STAGES) & 1, wl);
+            (void)mbar_wait(&S.sf_full[p % STAGES], (p / STAGES) & 1, wl);
+        }
     }
     __syncthreads();
     if (warp == 1) {
