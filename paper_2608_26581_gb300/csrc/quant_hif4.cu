@@ -111,23 +111,23 @@ __device__ __forceinline__ uint32_t hif4_group(const float (&x)[8], int sb, int 
         const int ex = e18 + (h ? e116_1 : e116_0);
         const float step = __uint_as_float(((uint32_t)(E + ex + 77) << 23) | ((uint32_t)M << 21));
         const float inv = __uint_as_float((uint32_t)(177 - E - ex) << 23) * recip_m;   // RN(1 / step)
-        const float hstep = 0.5f * step;
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             const float v = x[4 * h + i];
             const float a = fabsf(v);
-            // nearest k from the fp32 quotient.  a has 8 significant bits and
-            // step = D 2^s with D in {4,5,6,7}/4, so a quotient that is not
-            // exactly a half-integer lies at least 2^-9 / 7 of it away from
-            // every half-integer it could round across, while a * inv is
-            // within 2^-20 of it (relative error 2^-23, quotient below 8):
-            // rint is exact except at true ties, which the exact midpoint
-            // tests below send to the even k
-            float k = rintf(fminf(a * inv, 8.0f));
-            const float hi = fmaf(k, step, hstep), lo = fmaf(k, step, -hstep);   // exact
-            const bool odd = (__float_as_uint(k + 8388608.0f) & 1u) != 0;
-            k += odd ? (a == hi ? 1.0f : (a == lo ? -1.0f : 0.0f)) : 0.0f;
-            k = fminf(k, 7.0f);
+            // nearest k, ties to even, from the correctly rounded quotient
+            // a / step: a * inv is within one ulp of it (inv is the correctly
+            // rounded reciprocal), the remainder a - q step is exact (fma),
+            // and one correction q + r inv rounds to the correctly rounded
+            // quotient (Markstein's division refinement, P. Markstein, IA-64
+            // and Elementary Functions, 2000).  A true tie (a half-integer
+            // quotient) is then exact and rintf sends it to the even k; any
+            // other quotient lies at least 2^-9 / 7 from every half-integer
+            // (a has 8 significant bits, step = D 2^s with D in {4,5,6,7}/4),
+            // far beyond the rounding error.  fminf saturates (NaN -> 7).
+            float q = a * inv;
+            q = fmaf(fmaf(-q, step, a), inv, q);
+            const float k = fminf(rintf(q), 7.0f);
             const uint32_t ki = __float_as_uint(k + 8388608.0f) & 7u;   // k as an integer, exactly
             codes |= (((__float_as_uint(v) >> 28) & 8u) | ki) << (4 * (4 * h + i));
             deq[4 * h + i] = copysignf(k * step, v);

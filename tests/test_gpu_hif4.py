@@ -94,6 +94,65 @@ def test_degenerate_blocks(orc):
     _compare(orc, f32_to_bf16_bits(x), rfq.RFQ_SCALE_ROWMAJOR)
 
 
+def _tie_blocks(seed=0):
+    """64-element blocks whose elements sit on and next to the midpoints of
+    the S1P2 grid: per block a macro scale S (one element 7 S, so S is that
+    block's scale), the other elements +-(j + 1/2) or +-j steps of 0.25 S 2^ex
+    for random j and ex in {0, 1, 2} (bf16-exact: at most 7 significant
+    bits), some moved by one bf16 ulp; sub-groups then take exponents that
+    make many of them exact ties of their own grid."""
+    rng = np.random.default_rng(seed)
+    rows = []
+    for E in (0, 5, 20, 47, 48, 49, 60, 63):
+        for Mm in range(4):
+            S = 2.0 ** (E - 48) * (1 + Mm / 4)
+            for _ in range(24):
+                j = rng.integers(0, 7, 64)
+                ex = rng.integers(0, 3, 64)
+                half = rng.random(64) < 0.75
+                blk = (j + np.where(half, 0.5, 0.0)) * 0.25 * S * 2.0 ** ex
+                blk *= np.where(rng.random(64) < 0.5, -1.0, 1.0)
+                blk[rng.integers(0, 64)] = 7 * S
+                bits = f32_to_bf16_bits(blk.astype(np.float32)).astype(np.int32)
+                nudge = rng.choice([-1, 0, 0, 0, 1], 64)
+                nz = (bits & 0x7FFF) > 1
+                bits = np.where(nz, bits + nudge, bits)
+                rows.append(bits.astype(np.uint16))
+    return np.array(rows).reshape(-1, 256)
+
+
+def test_rounding_ties_to_even(orc):
+    """Elements exactly halfway between two grid points round to the even k
+    (the oracle's exact rounding), in both metadata layouts, for the
+    activation quantizer (main and residual) and the weight quantizer."""
+    xb = _tie_blocks()
+    # the blocks do hold exact ties: |x| / step a half-integer for the
+    # element's own step (decoded from the oracle's metadata words)
+    ref = orc.quantize_act(xb, orc.FMT_HIF4, orc.PHI_ALL, 0.0, 128, 256)
+    x = np.abs((xb.astype(np.uint32) << 16).view(np.float32).astype(np.float64))
+    meta = ref["main_scales"].reshape(xb.shape[0], -1).astype(np.int64)
+    sb = meta & 0xFF
+    S = np.exp2((sb >> 2) - 48.0) * (1 + (sb & 3) / 4)
+    i = np.arange(256) % 64
+    e18 = (np.repeat(meta, 64, axis=1) >> (8 + i // 8)) & 1
+    e116 = (np.repeat(meta, 64, axis=1) >> (16 + i // 4)) & 1
+    step = 0.25 * np.repeat(S, 64, axis=1) * np.exp2(e18 + e116)
+    q = x / step
+    ties = np.sum((q - np.floor(q) == 0.5) & (q < 7))
+    assert ties > 1000, ties
+    for layout in (rfq.RFQ_SCALE_ROWMAJOR, rfq.RFQ_SCALE_MMA):
+        _compare(orc, xb, layout)
+    # the same values as a weight [K x N] (quantized along K)
+    wb = np.ascontiguousarray(xb[:64].T)
+    wq = rfq.empty_qtensor(H, rfq.RFQ_SCALE_ROWMAJOR, 64, 256)
+    rfq.rfq_quantize_weight(to_dev_bf16(wb), wq)
+    torch.cuda.synchronize()
+    c, m = qtensor_host(wq)
+    rc, rm = orc.quantize_weight(wb, orc.FMT_HIF4)
+    assert np.array_equal(m, rm), _diff(m, rm)
+    assert np.array_equal(c, rc), _diff(c, rc)
+
+
 @pytest.mark.parametrize("mode,tau,r_s", [(rfq.RFQ_FALLBACK_NONE, 0.0, 256), (rfq.RFQ_FALLBACK_AMAX, 20.0, 128),
                                           (rfq.RFQ_FALLBACK_AMAX, 10.0, 64), (rfq.RFQ_FALLBACK_AMAX, 20.0, 256)])
 def test_phi_modes(orc, mode, tau, r_s):
