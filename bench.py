@@ -426,10 +426,10 @@ def run_rfq(args):
     if no_res and (fused or quant_only or amax_phi):
         raise SystemExit("--no-residual applies to the two-kernel linear workloads without --phi-tau")
     # MXFP8 schemes (Table 1 baselines and the FP4-to-FP8 residual of Sec. 4.2):
-    #   rfq8: MXFP4 main + MXFP8 residual, both multiplied as E4M3 (X~
-    #         re-encoded exactly by the quantizer in the same pass, W~ by
-    #         rfq_convert offline); w4a8: MXFP8 X x MXFP4 W (re-encoded);
-    #         w8a8: MXFP8 X x MXFP8 W.  All on kind::mxf8f6f4.
+    #   rfq8: MXFP4 main + MXFP8 residual, both on the FP8 path (X~
+    #         re-encoded exactly as E4M3 by the quantizer in the same pass,
+    #         W~ multiplied as E2M1 from its packed codes); w4a8: MXFP8 X x
+    #         MXFP4 W (E2M1); w8a8: MXFP8 X x MXFP8 W.  All on kind::mxf8f6f4.
     #   rfq8mix: the rfq8 RFQ through rfq_linear_mixed -- the main product
     #         on kind::mxf4 (X~ and W~ packed), the residual on
     #         kind::mxf8f6f4 (X^ as E4M3, W~ expanded from its packed codes
@@ -474,13 +474,10 @@ def run_rfq(args):
         w = torch.from_numpy(wb.view(np.int16)).to(dev).view(torch.bfloat16)
         wq = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8 if scheme == "w8a8" else F, L, NW, K, device=dev)
         rfq.rfq_quantize_weight(w, wq)                     # offline weight step, untimed
-        if scheme in ("rfq8", "w4a8"):
-            wop = rfq.empty_qtensor(rfq.RFQ_FMT_MXFP8, L, NW, K, device=dev)
-            rfq.rfq_convert(wq, wop)                       # exact E4M3 re-encoding of W~ (offline)
-        elif hif4:
+        if hif4:
             wop = rfq.empty_bf16_operand(N, K, device=dev)  # exact bf16 expansion of W~ (offline)
             rfq.rfq_dequant(wq, wop.codes)
-        elif wop is None:
+        else:
             wop = wq
         del w
     no_res = no_res or scheme in ("w4a8", "w8a8")

@@ -212,10 +212,12 @@ RFQ_API size_t rfq_linear_workspace_bytes(void);
  * products, at its own granularity (it may still include a phi = 0 tile that
  * shares a 256-row or 256-column block with a phi = 1 one).
  * wq: [N x K] weight.  MXFP4: every operand MXFP4 with RFQ_SCALE_MMA,
- * K % 128 == 0.  MXFP8: every operand MXFP8 (E4M3, kind::mxf8f6f4 MMAs)
- * with RFQ_SCALE_MMA, K % 128 == 0 -- the W8A8 and W4A8 baselines (an MXFP4
- * weight re-encoded by rfq_convert) and the FP4-to-FP8 RFQ (X~ re-encoded
- * by rfq_convert, X^ from the MXFP8 residual pathway).  HiF4 (Sec. 3.3): wq is the exact bf16 expansion of the HiF4
+ * K % 128 == 0.  MXFP8: xq (and xr) MXFP8 (E4M3, kind::mxf8f6f4 MMAs)
+ * with RFQ_SCALE_MMA, K % 128 == 0, and wq MXFP8 or MXFP4 -- the W8A8 and
+ * W4A8 baselines and the FP4-to-FP8 RFQ (X~ re-encoded by rfq_convert, X^
+ * from the MXFP8 residual pathway).  An MXFP4 wq (codes 32-byte aligned) is
+ * multiplied as E2M1 (E4M3 x E2M1 MMAs) straight from its packed codes, half
+ * the weight bytes of its E4M3 re-encoding, which gives the same Y.  HiF4 (Sec. 3.3): wq is the exact bf16 expansion of the HiF4
  * weight (RFQ_FMT_BF16, from rfq_dequant), K % 64 == 0, phi_r_s a multiple
  * of 64, and xq/xr are either HiF4 with RFQ_SCALE_MMA metadata (expanded
  * exactly to bf16 in shared memory inside the GEMM) or their exact bf16
@@ -284,7 +286,8 @@ RFQ_API rfq_status rfq_linear_fused(const void *x_bf16, int64_t M, int64_t K, co
  * weights of all groups stacked, rows = groups * N (group g's W~ rows
  * [g N, (g+1) N)), N % 128 == 0.  y: device [rows][N]; every row of a
  * group (the rows padding it to the next group's start included) is
- * written, rows before group_off[0] or from group_off[groups] on are not.  Operands MXFP4 (or all MXFP8) with
+ * written, rows before group_off[0] or from group_off[groups] on are not.  Operands MXFP4, or MXFP8
+ * activations with an MXFP8 or MXFP4 (32-byte aligned) W~, as for rfq_linear; all with
  * RFQ_SCALE_MMA, K % 128 == 0; phi, phi_r_s, out_dtype and workspace as
  * for rfq_linear.  1 <= groups <= 128.
  * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,

@@ -394,13 +394,17 @@ rfq_status linear_check(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint
             return RFQ_ERR_INVALID_ARG;
     }
     // operand formats: MXFP4 x MXFP4; MXFP8 x MXFP8 (E4M3, also holding exact
-    // re-encodings of MXFP4 tensors); or HiF4 (codes, or their exact bf16
-    // expansion) x the bf16 expansion of W~
+    // re-encodings of MXFP4 tensors); MXFP8 x MXFP4 (W~ multiplied as E2M1,
+    // K % 128 == 0, its codes 32-byte aligned); or HiF4 (codes, or their
+    // exact bf16 expansion) x the bf16 expansion of W~
     const bool bf16_act = xq->fmt == RFQ_FMT_BF16;
     const bool hif4 = xq->fmt == RFQ_FMT_HIF4 || bf16_act;
     const bool f8 = xq->fmt == RFQ_FMT_MXFP8;
-    if (hif4 ? wq->fmt != RFQ_FMT_BF16 : wq->fmt != (f8 ? RFQ_FMT_MXFP8 : RFQ_FMT_MXFP4))
+    const bool w4 = f8 && wq->fmt == RFQ_FMT_MXFP4;
+    if (hif4 ? wq->fmt != RFQ_FMT_BF16 : (wq->fmt != (f8 ? RFQ_FMT_MXFP8 : RFQ_FMT_MXFP4) && !w4))
         return RFQ_ERR_INVALID_ARG;
+    if (w4 && K % 128 != 0)
+        return RFQ_ERR_SHAPE;
     if (bf16_act && K % 64 != 0)
         return RFQ_ERR_SHAPE;
     if (N % 16 != 0)
@@ -409,7 +413,8 @@ rfq_status linear_check(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint
         return RFQ_ERR_SHAPE;
     if (phi && xr && (hif4 ? (phi_r_s < 64 || phi_r_s % 64 != 0) : (phi_r_s < 128 || phi_r_s % 128 != 0)))
         return RFQ_ERR_SHAPE;
-    if (!aligned16(y) || (check_ws && !aligned16(workspace)))
+    if (!aligned16(y) || (check_ws && !aligned16(workspace)) ||
+        (w4 && (reinterpret_cast<uintptr_t>(wq->codes) & 31u) != 0))
         return RFQ_ERR_ALIGNMENT;
     if ((s = check_device()) != RFQ_OK)
         return s;
@@ -472,6 +477,7 @@ rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, const uint8_
     a.K = K;
     a.status = static_cast<int32_t *>(workspace);
     a.f8 = f8;
+    a.w4 = f8 && wq->fmt == RFQ_FMT_MXFP4;
     return gemm_done(launch_gemm_mxf4(a, st), workspace, st);
 }
 
@@ -827,7 +833,8 @@ rfq_status rfq_linear_grouped(const rfq_qtensor *xq, const rfq_qtensor *xr, cons
             return RFQ_ERR_INVALID_ARG;
     }
     const bool f8 = xq->fmt == RFQ_FMT_MXFP8;
-    if ((xq->fmt != RFQ_FMT_MXFP4 && !f8) || wq->fmt != xq->fmt)
+    const bool w4 = f8 && wq->fmt == RFQ_FMT_MXFP4;   // W~ multiplied as E2M1
+    if ((xq->fmt != RFQ_FMT_MXFP4 && !f8) || (wq->fmt != xq->fmt && !w4))
         return RFQ_ERR_UNSUPPORTED;
     // every group's W~ rows start on a 128-row scale atom and a 16-column Y boundary
     if (N % 128 != 0 || K % 128 != 0)
@@ -836,7 +843,8 @@ rfq_status rfq_linear_grouped(const rfq_qtensor *xq, const rfq_qtensor *xr, cons
         return RFQ_ERR_SHAPE;
     if (phi && xr && (phi_r_s < 128 || phi_r_s % 128 != 0))
         return RFQ_ERR_SHAPE;
-    if (!aligned16(y) || !aligned16(workspace) || !aligned16(group_off))
+    if (!aligned16(y) || !aligned16(workspace) || !aligned16(group_off) ||
+        (w4 && (reinterpret_cast<uintptr_t>(wq->codes) & 31u) != 0))
         return RFQ_ERR_ALIGNMENT;
     if (xq->scale_layout != RFQ_SCALE_MMA || wq->scale_layout != RFQ_SCALE_MMA)
         return RFQ_ERR_UNSUPPORTED;
@@ -860,6 +868,7 @@ rfq_status rfq_linear_grouped(const rfq_qtensor *xq, const rfq_qtensor *xr, cons
     a.K = K;
     a.status = static_cast<int32_t *>(workspace);
     a.f8 = f8;
+    a.w4 = w4;
     a.group_off = group_off;
     a.groups = groups;
     return gemm_done(launch_gemm_mxf4(a, static_cast<cudaStream_t>(stream)), workspace,

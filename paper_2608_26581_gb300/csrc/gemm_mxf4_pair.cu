@@ -195,11 +195,16 @@ struct Mask {
 // (the same 128-byte rows); 2 -- the FP4-to-FP8 residual at two rates
 // (Sec. 4.2, 4.3): a stage is one 128-element chunk holding X~ and W~ packed
 // (E2M1, 64-byte rows, 64-byte swizzle: the main product on kind::mxf4, two
-// K = 64 MMAs) and X^ and W~ as E4M3 (128-byte rows: the residual product
-// on kind::mxf8f6f4, four K = 32 MMAs), into the same accumulator with the
-// same scale words (W~'s E4M3 form keeps its E8M0 bytes); 48 KB per stage
-// for 768 MMA cycles against 1,024 when the main product also runs as E4M3.
+// K = 64 MMAs), X^ as E4M3 and W~ again in the padded 4-bit form (128-byte
+// rows: the residual product on kind::mxf8f6f4, E4M3 x E2M1, four K = 32
+// MMAs), into the same accumulator with the same scale words; 40 KB read
+// per stage for 768 MMA cycles against 1,024 when the main product also
+// runs on kind::mxf8f6f4.
 constexpr int F8_MIXED = 2;
+// F8 == F8_W4: the E4M3 form with W~ kept as MXFP4 -- every product on
+// kind::mxf8f6f4 as E4M3 x E2M1, W~'s tile copied from its packed codes in
+// the padded 4-bit form (64 bytes read per 128-byte row).
+constexpr int F8_W4 = 3;
 // GRP: the grouped (mixture-of-experts) form, G groups of rows with their
 // own W~ (row offsets read on the device); the plain form is compiled
 // without any of it.
@@ -221,6 +226,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
 {
     static_assert(!FQ || (!PHI && !F8 && !GRP), "the fused quantizer takes plain MXFP4 operands");
     static_assert(F8 != F8_MIXED || (RES && !GRP && !FQ), "the mixed-rate form is the RFQ with a residual");
+    constexpr int B_TX = F8 == F8_W4 ? B_BYTES / 2 : B_BYTES;   // bytes a W~ tile copy reads
     extern __shared__ uint8_t smem_raw[];
     Smem &S = *reinterpret_cast<Smem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -430,7 +436,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                         }
                     } else {
                         if (lead)
-                            mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES + B_BYTES + (res_on ? A_BYTES : 0)));
+                            mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES + B_TX + (res_on ? A_BYTES : 0)));
                         tma_load_2d_pair(st.a, &tmA, bar, cx, a_y);
                         if (res_on)
                             tma_load_2d_pair(st.r, &tmR, bar, cx, a_y);
@@ -557,8 +563,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                         if (c >= nch)
                             break;
                         // MXFP4: K = 64 per MMA, scale bytes 2 (j & 1) and up; E4M3: K = 32, byte j
-                        const uint32_t id = F8 ? idesc_mxf8(2 * BM, BN, j, j)
-                                               : idesc_mxf4(2 * BM, BN, 2 * (j & 1), 2 * (j & 1));
+                        const uint32_t id = F8 == F8_W4 ? idesc_mxf8_e4m3_e2m1(2 * BM, BN, j, j)
+                                            : F8        ? idesc_mxf8(2 * BM, BN, j, j)
+                                                        : idesc_mxf4(2 * BM, BN, 2 * (j & 1), 2 * (j & 1));
                         const uint64_t bd = sdesc_k_sw128(b0 + 32 * j);
                         const uint32_t sfb_t = sf + 16 + 8 * c;
                         if (F8)
@@ -1120,8 +1127,11 @@ cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
     const uint64_t kb = a.f8 ? (uint64_t)a.K : (uint64_t)a.K / 2; // code bytes per row
     const uint64_t w_rows = (uint64_t)a.N * (a.groups > 0 ? (uint64_t)a.groups : 1u);
     const uint64_t a_rows = a.fq_x ? (uint64_t)a.fq_ring * 2 * BM : (uint64_t)a.M;   // FQ: the ring
+    if (a.w4 && !a.f8)
+        return cudaErrorInvalidValue;
     if (!encode_tmap_2d_u8(&ta, a.a_codes, kb, a_rows, kb, ROW, BM, 128) ||
-        !encode_tmap_2d_u8(&tb, a.b_codes, kb, w_rows, kb, ROW, BN_HALF, 128))
+        !(a.w4 ? encode_tmap_2d_e2m1_padded(&tb, a.b_codes, (uint64_t)a.K, w_rows, BN_HALF)
+               : encode_tmap_2d_u8(&tb, a.b_codes, kb, w_rows, kb, ROW, BN_HALF, 128)))
         return cudaErrorInvalidValue;
     if (a.r_codes) {
         if (!encode_tmap_2d_u8(&tr, a.r_codes, kb, a_rows, kb, ROW, BM, 128))
@@ -1154,11 +1164,11 @@ cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
                           : launch_variant<false, false, false, false, false, true>(ta, tr, tb, ty, a, st);
     }
     const bool phi = res && a.phi != nullptr && a.K / (a.f8 ? 128 : 256) <= REC_WORDS * 32;
-#define RFQ_GV(R, P, O)                                                                                           \
-    return a.groups > 0 ? (a.f8 ? launch_variant<R, P, O, true, true>(ta, tr, tb, ty, a, st)                       \
-                                : launch_variant<R, P, O, false, true>(ta, tr, tb, ty, a, st))                     \
-                        : (a.f8 ? launch_variant<R, P, O, true, false>(ta, tr, tb, ty, a, st)                      \
-                                : launch_variant<R, P, O, false, false>(ta, tr, tb, ty, a, st))
+#define RFQ_GV_F(R, P, O, G)                                                                                      \
+    (!a.f8 ? launch_variant<R, P, O, 0, G>(ta, tr, tb, ty, a, st)                                                 \
+           : a.w4 ? launch_variant<R, P, O, F8_W4, G>(ta, tr, tb, ty, a, st)                                      \
+                  : launch_variant<R, P, O, 1, G>(ta, tr, tb, ty, a, st))
+#define RFQ_GV(R, P, O) return a.groups > 0 ? RFQ_GV_F(R, P, O, true) : RFQ_GV_F(R, P, O, false)
     if (!res) {
         if (a.out_bf16) RFQ_GV(false, false, true);
         RFQ_GV(false, false, false);
@@ -1170,6 +1180,7 @@ cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
     if (a.out_bf16) RFQ_GV(true, false, true);
     RFQ_GV(true, false, false);
 #undef RFQ_GV
+#undef RFQ_GV_F
 }
 
 RFQ_DEBUG_WORD_ACCESSOR(debug_word_gemm_mxf4_pair)

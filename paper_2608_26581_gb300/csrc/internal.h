@@ -124,6 +124,8 @@ struct GemmMxf4Args {
     int64_t M, N, K;
     int32_t *status;
     int f8 = 0;                                // every operand MXFP8 (E4M3): kind::mxf8f6f4, CTA pairs
+    int w4 = 0;                                // with f8: W~ MXFP4 [N][K/2] (32-byte aligned), multiplied
+                                               // as E2M1 (E4M3 x E2M1 MMAs) from the padded 4-bit form
     const int32_t *group_off = nullptr;        // grouped GEMM: device row offsets [groups + 1]
     int groups = 0;                            // grouped GEMM: N is per group, W~ has groups * N rows
     // fused quantizer (CTA-pair kernel): bf16 X [M][K]; the kernel quantizes
@@ -134,9 +136,9 @@ struct GemmMxf4Args {
     int32_t *fq_ctr = nullptr;
     int fq_ring = 0;                           // fused quantizer: 256-row slots of the scratch ring
     int prof = 0;                              // CTA-pair kernel: the MMA thread's counters (rfq_linear_profile)
-    // mixed-rate FP4-to-FP8 residual (CTA-pair kernel): W~ packed [N][K/2];
-    // a_codes / a_sf are then X~ packed, r_codes / r_sf X^ as E4M3, b_codes
-    // W~ as E4M3 (its exact re-encoding), b_sf W~'s scales
+    // mixed-rate FP4-to-FP8 residual (CTA-pair kernel): W~ packed [N][K/2]
+    // (32-byte aligned); a_codes / a_sf are then X~ packed, r_codes / r_sf
+    // X^ as E4M3, b_sf W~'s scales (b_codes unused)
     const void *b4_codes = nullptr;
 };
 

@@ -16,7 +16,8 @@ pytestmark = pytest.mark.gpu
 F4, F8, MMA = rfq.RFQ_FMT_MXFP4, rfq.RFQ_FMT_MXFP8, rfq.RFQ_SCALE_MMA
 
 
-def _case(orc, counts, K, N, fmt="rfq4", mode=rfq.RFQ_FALLBACK_ALL, tau=0.0, r_s=256, out=rfq.RFQ_OUT_F32, seed=0):
+def _case(orc, counts, K, N, fmt="rfq4", mode=rfq.RFQ_FALLBACK_ALL, tau=0.0, r_s=256, out=rfq.RFQ_OUT_F32, seed=0,
+          packed_w=False):
     G = len(counts)
     starts = []
     pos = 0
@@ -41,7 +42,9 @@ def _case(orc, counts, K, N, fmt="rfq4", mode=rfq.RFQ_FALLBACK_ALL, tau=0.0, r_s
     f8 = fmt != "rfq4"
     wq = rfq.empty_qtensor(F4, MMA, G * N, K)
     rfq.rfq_quantize_weight(w, wq)
-    if f8:
+    if f8 and packed_w:
+        w8 = wq          # MXFP8 activations x the MXFP4 W~, multiplied as E2M1
+    elif f8:
         w8 = rfq.empty_qtensor(F8, MMA, G * N, K)
         rfq.rfq_convert(wq, w8)
     if fmt == "rfq4":
@@ -121,9 +124,10 @@ def test_grouped_selective_phi(orc):
     _case(orc, [200, 333, 70], 1152, 256, mode=rfq.RFQ_FALLBACK_AMAX, tau=30.0, r_s=128, seed=9)
 
 
+@pytest.mark.parametrize("packed_w", [False, True])
 @pytest.mark.parametrize("fmt", ["w4a8", "rfq8"])
-def test_grouped_mxfp8(orc, fmt):
-    _case(orc, [150, 0, 260, 9], 512, 256, fmt=fmt, seed=11)
+def test_grouped_mxfp8(orc, fmt, packed_w):
+    _case(orc, [150, 0, 260, 9], 512, 256, fmt=fmt, seed=11, packed_w=packed_w)
 
 
 def test_grouped_bad_offsets_are_reported(orc):

@@ -170,10 +170,12 @@ def test_quantize_act_expand_fp8_residual(orc, layout, mode, tau):
 
 
 def _gemm_case(orc, M, K, N, kind, out=rfq.RFQ_OUT_F32, mode=rfq.RFQ_FALLBACK_ALL, tau=0.0, r_s=256, seed=1,
-               rows=None, xb=None, wb=None):
+               rows=None, xb=None, wb=None, packed_w=False):
     """kind: 'w8a8', 'w4a8', 'rfq8' (MXFP4 main + MXFP8 residual, both
-    products as E4M3) or 'rfq8mix' (the same RFQ through rfq_linear_mixed:
-    the main product on the FP4 path, the residual on the FP8 one)."""
+    products on the FP8 path) or 'rfq8mix' (the same RFQ through
+    rfq_linear_mixed: the main product on the FP4 path, the residual on the
+    FP8 one).  packed_w (w4a8, rfq8): W~ passed as MXFP4 (multiplied as
+    E2M1 from its packed codes) instead of its E4M3 re-encoding."""
     if xb is None:
         xb = make_activation(ActSpec(M, K, "normal", chan_count=3, chan_scale=64.0, tok_count=1, tok_scale=200.0,
                                      seed=seed))
@@ -192,8 +194,11 @@ def _gemm_case(orc, M, K, N, kind, out=rfq.RFQ_OUT_F32, mode=rfq.RFQ_FALLBACK_AL
     else:
         w4 = rfq.empty_qtensor(F4, MMA, N, K)
         rfq.rfq_quantize_weight(w, w4)
-        wq = rfq.empty_qtensor(F8, MMA, N, K)
-        rfq.rfq_convert(w4, wq)
+        if packed_w:
+            wq = w4
+        else:
+            wq = rfq.empty_qtensor(F8, MMA, N, K)
+            rfq.rfq_convert(w4, wq)
         wref = orc.quantize_weight(wb, orc.FMT_MXFP4)
         w_fmt = orc.FMT_MXFP4
     if kind in ("w8a8", "w4a8"):
@@ -233,10 +238,19 @@ def test_linear_mxfp8_shapes(orc, kind, M, K, N):
     _gemm_case(orc, M, K, N, kind, seed=M + N)
 
 
-@pytest.mark.parametrize("kind", ["rfq8", "rfq8mix"])
+@pytest.mark.parametrize("kind", ["w4a8", "rfq8"])
+@pytest.mark.parametrize("M,K,N", [(1, 128, 16), (129, 384, 272), (300, 640, 528), (513, 1024, 784)])
+def test_linear_packed_mxfp4_weight(orc, kind, M, K, N):
+    """MXFP8 activations times an MXFP4 W~ multiplied as E2M1 from its
+    packed codes (the padded 4-bit copy), against the oracle."""
+    _gemm_case(orc, M, K, N, kind, seed=M + N + 7, packed_w=True)
+
+
+@pytest.mark.parametrize("kind", ["rfq8", "rfq8mix", "rfq8w4"])
 @pytest.mark.parametrize("r_s,tau", [(128, 30.0), (256, 30.0), (256, 1e30)])
 def test_linear_fp8_residual_selective_phi(orc, kind, r_s, tau):
-    _gemm_case(orc, 384, 1152, 512, kind, mode=rfq.RFQ_FALLBACK_AMAX, tau=tau, r_s=r_s, seed=11)
+    _gemm_case(orc, 384, 1152, 512, kind.replace("w4", ""), mode=rfq.RFQ_FALLBACK_AMAX, tau=tau, r_s=r_s, seed=11,
+               packed_w=kind.endswith("w4"))
 
 
 @pytest.mark.parametrize("kind", ["rfq8", "rfq8mix"])
@@ -245,14 +259,19 @@ def test_linear_mxfp8_bf16_output(orc, kind):
 
 
 def test_mixed_rate_matches_all_e4m3_path(orc):
-    """The two ways of multiplying the FP4-to-FP8 RFQ give the same Y up to
-    fp32 accumulation order: every product is exact in both (E2M1 values are
-    E4M3 values), so both match the oracle and each other within the
-    tolerance, on ragged shapes with more tiles than CTA pairs."""
+    """The ways of multiplying the FP4-to-FP8 RFQ give the same Y up to fp32
+    accumulation order: every product is exact in each (E2M1 values are E4M3
+    values), so all match the oracle and each other within the tolerance,
+    on ragged shapes with more tiles than CTA pairs.  (W~ as E2M1 or as
+    E4M3 gives the same exact products, but the tensor core's summation
+    inside one MMA differs between the operand types, so Y is not
+    bit-identical.)"""
     M, K, N = 1000, 1280, 1040
     y8 = _gemm_case(orc, M, K, N, "rfq8", seed=21)
+    y8w4 = _gemm_case(orc, M, K, N, "rfq8", seed=21, packed_w=True)
     ym = _gemm_case(orc, M, K, N, "rfq8mix", seed=21)
     check_y(ym, y8)
+    check_y(y8w4, y8)
 
 
 def test_mixed_rate_host_checks():
