@@ -105,7 +105,7 @@ __device__ __forceinline__ uint32_t hif4_group(const float (&x)[8], int sb, int 
     const int e18 = (t[0] == 2 || t[1] == 2) ? 1 : 0;
     const int e116_0 = max(t[0] - e18, 0), e116_1 = max(t[1] - e18, 0);
     meta_bits = ((uint32_t)e18 << (8 + g)) | ((uint32_t)e116_0 << (16 + 2 * g)) | ((uint32_t)e116_1 << (17 + 2 * g));
-    uint32_t codes = 0;
+    float kf[8];   // the magnitudes k as floats (exact small integers)
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
         const int ex = e18 + (h ? e116_1 : e116_0);
@@ -121,18 +121,27 @@ __device__ __forceinline__ uint32_t hif4_group(const float (&x)[8], int sb, int 
             // and one correction q + r inv rounds to the correctly rounded
             // quotient (Markstein's division refinement, P. Markstein, IA-64
             // and Elementary Functions, 2000).  A true tie (a half-integer
-            // quotient) is then exact and rintf sends it to the even k; any
-            // other quotient lies at least 2^-9 / 7 from every half-integer
-            // (a has 8 significant bits, step = D 2^s with D in {4,5,6,7}/4),
-            // far beyond the rounding error.  fminf saturates (NaN -> 7).
+            // quotient) is then exact, and adding 2^23 rounds it to the even
+            // integer; any other quotient lies at least 2^-9 / 7 from every
+            // half-integer (a has 8 significant bits, step = D 2^s with D in
+            // {4,5,6,7}/4), far beyond the rounding error.  fminf saturates
+            // (NaN -> 7) before the rounding.
             float q = a * inv;
             q = fmaf(fmaf(-q, step, a), inv, q);
-            const float k = fminf(rintf(q), 7.0f);
-            const uint32_t ki = __float_as_uint(k + 8388608.0f) & 7u;   // k as an integer, exactly
-            codes |= (((__float_as_uint(v) >> 28) & 8u) | ki) << (4 * (4 * h + i));
+            const float k = (fminf(q, 7.0f) + 8388608.0f) - 8388608.0f;
+            kf[4 * h + i] = k;
             deq[4 * h + i] = copysignf(k * step, v);
         }
     }
+    // the eight 3-bit magnitudes into nibbles: two sums of k 16^i (exact
+    // below 2^16), their integer bits by adding 2^23, the low halves joined;
+    // then the sign bits (bit 3 of each nibble) from the inputs' sign bits
+    const float lo = fmaf(kf[3], 4096.0f, fmaf(kf[2], 256.0f, fmaf(kf[1], 16.0f, kf[0])));
+    const float hi = fmaf(kf[7], 4096.0f, fmaf(kf[6], 256.0f, fmaf(kf[5], 16.0f, kf[4])));
+    uint32_t codes = __byte_perm(__float_as_uint(lo + 8388608.0f), __float_as_uint(hi + 8388608.0f), 0x5410);
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+        codes |= (__float_as_uint(x[i]) >> (28 - 4 * i)) & (8u << (4 * i));
     return codes;
 }
 
