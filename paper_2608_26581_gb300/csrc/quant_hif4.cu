@@ -152,11 +152,13 @@ __device__ __forceinline__ int64_t meta_index(int64_t m, int64_t blk, int64_t ro
     return LAYOUT == RFQ_SCALE_MMA ? blk * (((rows + 127) >> 7) << 7) + m : m * kblocks + blk;
 }
 
-// Eight consecutive lanes hold one 64-element block (lane l: group l % 8).
-// Quantizes x (main), and with RES its residual x - x~ (Sec. 4.3).  Items
-// are (row, 1024-element segment): a warp loads its four 16-byte chunks per
-// lane up front, and the row and block indices come from the item without a
-// 64-bit division per chunk.  With EXP the kernel also writes the exact bf16
+// act_quant_hif4_kernel: four consecutive lanes hold one 64-element block
+// (lane l: groups 2 (l % 4) and 2 (l % 4) + 1, hif4_chunk16); the fused
+// AMAX kernel below keeps eight lanes per block (lane l: group l % 8,
+// hif4_chunk).  Quantizes x (main), and with RES its residual x - x~
+// (Sec. 4.3).  Items are (row, 1024-element segment): a warp loads its four
+// 16-byte chunks per lane up front, and the row and block indices come from
+// the item without a 64-bit division per chunk.  With EXP the kernel also writes the exact bf16
 // values of X~ (and X^; zeros where phi = 0) as [M][K] row-major, the
 // operands of the bf16 tensor-core GEMM: every HiF4 value has at most six
 // significant bits and an exponent inside bf16's range.
@@ -234,6 +236,79 @@ __device__ __forceinline__ void hif4_chunk(const float (&xf)[8], int g, bool ok,
     }
 }
 
+// The same for one lane's sixteen elements xf (groups 2 g2 and 2 g2 + 1 of
+// its 64-element block, four lanes per block) at chunks c, c + 1: the
+// block's amax, macro scale and metadata reduce over four lanes instead of
+// eight, so each lane does that per-block work for twice the elements.
+template <bool RES, bool EXP>
+__device__ __forceinline__ void hif4_chunk16(const float (&xf)[16], int g2, bool ok, bool on, int64_t c, int64_t moff,
+                                             uint32_t *__restrict__ mcodes, uint32_t *__restrict__ mmeta,
+                                             uint32_t *__restrict__ rcodes, uint32_t *__restrict__ rmeta,
+                                             uint4 *__restrict__ m16, uint4 *__restrict__ r16)
+{
+    float am = 0.f;
+#pragma unroll
+    for (int i = 0; i < 16; i += 4)
+        am = fmax3(am, fmaxf(fabsf(xf[i]), fabsf(xf[i + 1])), fmaxf(fabsf(xf[i + 2]), fabsf(xf[i + 3])));
+    am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 1));
+    am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 2));
+    const int sb = am > 0.f ? hif4_scale_byte(am) : 0;
+    float x0[8], x1[8], d0[8], d1[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        x0[i] = xf[i];
+        x1[i] = xf[8 + i];
+    }
+    uint32_t b0, b1;
+    const uint32_t code0 = hif4_group(x0, sb, 2 * g2, b0, d0);
+    const uint32_t code1 = hif4_group(x1, sb, 2 * g2 + 1, b1, d1);
+    uint32_t bits = am == 0.f ? 0u : (b0 | b1);   // all-zero block: metadata 0, codes keep the sign of zero
+    bits |= __shfl_xor_sync(0xFFFFFFFFu, bits, 1);
+    bits |= __shfl_xor_sync(0xFFFFFFFFu, bits, 2);
+    if (ok) {
+        *reinterpret_cast<uint2 *>(mcodes + c) = make_uint2(code0, code1);
+        if (g2 == 0)
+            mmeta[moff] = am == 0.f ? 0u : (bits | (uint32_t)sb);
+        if (EXP) {
+            m16[c] = bf16x8_pack(d0);
+            m16[c + 1] = bf16x8_pack(d1);
+        }
+    }
+    if (RES) {
+        float r0[8], r1[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            r0[i] = x0[i] - d0[i]; // exact
+            r1[i] = x1[i] - d1[i];
+        }
+        float ra = 0.f;
+#pragma unroll
+        for (int i = 0; i < 8; i += 4) {
+            ra = fmax3(ra, fmaxf(fabsf(r0[i]), fabsf(r0[i + 1])), fmaxf(fabsf(r0[i + 2]), fabsf(r0[i + 3])));
+            ra = fmax3(ra, fmaxf(fabsf(r1[i]), fabsf(r1[i + 1])), fmaxf(fabsf(r1[i + 2]), fabsf(r1[i + 3])));
+        }
+        ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, 1));
+        ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, 2));
+        const int rsb = ra > 0.f ? hif4_scale_byte(ra) : 0;
+        uint32_t rb0, rb1;
+        float e0[8], e1[8];
+        const uint32_t rcode0 = hif4_group(r0, rsb, 2 * g2, rb0, e0);
+        const uint32_t rcode1 = hif4_group(r1, rsb, 2 * g2 + 1, rb1, e1);
+        uint32_t rbits = rb0 | rb1;
+        rbits |= __shfl_xor_sync(0xFFFFFFFFu, rbits, 1);
+        rbits |= __shfl_xor_sync(0xFFFFFFFFu, rbits, 2);
+        if (ok) {
+            *reinterpret_cast<uint2 *>(rcodes + c) = on ? make_uint2(rcode0, rcode1) : make_uint2(0u, 0u);
+            if (g2 == 0)
+                rmeta[moff] = (on && ra > 0.f) ? (rbits | (uint32_t)rsb) : 0u;
+            if (EXP) {
+                r16[c] = on ? bf16x8_pack(e0) : make_uint4(0, 0, 0, 0);
+                r16[c + 1] = on ? bf16x8_pack(e1) : make_uint4(0, 0, 0, 0);
+            }
+        }
+    }
+}
+
 template <bool RES, bool PHI, int LAYOUT, bool EXP>
 __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__restrict__ x, int64_t M, int64_t K,
                                                             uint32_t *__restrict__ mcodes,
@@ -244,7 +319,7 @@ __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__rest
                                                             uint4 *__restrict__ m16, uint4 *__restrict__ r16)
 {
     const int lane = threadIdx.x & 31;
-    const int g = lane & 7;
+    const int g2 = lane & 3;                       // the lane's quarter of its block
     const int kchunks = (int)(K >> 3);
     const int64_t kblocks = K >> 6;
     const int segs = (kchunks + kHSeg / 8 - 1) / (kHSeg / 8);
@@ -256,27 +331,33 @@ __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__rest
         const int64_t m = item / segs;
         const int c0 = (int)(item - m * segs) * (kHSeg / 8);
         const uint4 *xr = x + m * kchunks;
+        // two 512-element steps; lane l takes chunks 2l, 2l + 1 of each (K is a
+        // multiple of 64, so a block is wholly inside the row or past it)
         uint4 vv[kHU];
 #pragma unroll
         for (int j = 0; j < kHU; ++j) {
-            const int c = c0 + j * 32 + lane;
+            const int c = c0 + (j >> 1) * 64 + 2 * lane + (j & 1);
             vv[j] = c < kchunks ? __ldcs(xr + c) : make_uint4(0, 0, 0, 0);
         }
         const uint8_t *prow = PHI ? phi + (m / p_s) * phi_cols : nullptr;
 #pragma unroll
-        for (int j = 0; j < kHU; ++j) {
-            const int cr = c0 + j * 32 + lane;             // chunk of 8 elements within the row
-            const bool ok = cr < kchunks;                  // uniform over each block's eight lanes
-            float xf[8];
-            const uint32_t w[4] = {vv[j].x, vv[j].y, vv[j].z, vv[j].w};
+        for (int s = 0; s < kHU / 2; ++s) {
+            const int cr = c0 + s * 64 + 2 * lane;         // first of the lane's two chunks
+            const bool ok = cr < kchunks;                  // uniform over each block's four lanes
+            float xf[16];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                xf[2 * i] = __uint_as_float(w[i] << 16);
-                xf[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+            for (int u = 0; u < 2; ++u) {
+                const uint32_t w[4] = {vv[2 * s + u].x, vv[2 * s + u].y, vv[2 * s + u].z, vv[2 * s + u].w};
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    xf[8 * u + 2 * i] = __uint_as_float(w[i] << 16);
+                    xf[8 * u + 2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+                }
             }
+            // r_s is a multiple of 64: the block lies in one phi column
             const bool on = !PHI || (ok && prow[(cr * 8) / r_s] != 0);
-            hif4_chunk<RES, EXP, LAYOUT>(xf, g, ok, on, m * kchunks + cr, meta_index<LAYOUT>(m, cr >> 3, M, kblocks),
-                                         mcodes, mmeta, rcodes, rmeta, m16, r16);
+            hif4_chunk16<RES, EXP>(xf, g2, ok, on, m * kchunks + cr, meta_index<LAYOUT>(m, cr >> 3, M, kblocks),
+                                   mcodes, mmeta, rcodes, rmeta, m16, r16);
         }
     }
 }
