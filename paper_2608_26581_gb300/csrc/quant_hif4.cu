@@ -152,8 +152,8 @@ __device__ __forceinline__ int64_t meta_index(int64_t m, int64_t blk, int64_t ro
     return LAYOUT == RFQ_SCALE_MMA ? blk * (((rows + 127) >> 7) << 7) + m : m * kblocks + blk;
 }
 
-// act_quant_hif4_kernel: four consecutive lanes hold one 64-element block
-// (lane l: groups 2 (l % 4) and 2 (l % 4) + 1, hif4_chunk16); the fused
+// act_quant_hif4_kernel: 8 / kHNG consecutive lanes hold one 64-element
+// block (lane l: kHNG consecutive groups, hif4_chunk_n); the fused
 // AMAX kernel below keeps eight lanes per block (lane l: group l % 8,
 // hif4_chunk).  Quantizes x (main), and with RES its residual x - x~
 // (Sec. 4.3).  Items are (row, 1024-element segment): a warp loads its four
@@ -236,78 +236,115 @@ __device__ __forceinline__ void hif4_chunk(const float (&xf)[8], int g, bool ok,
     }
 }
 
-// The same for one lane's sixteen elements xf (groups 2 g2 and 2 g2 + 1 of
-// its 64-element block, four lanes per block) at chunks c, c + 1: the
-// block's amax, macro scale and metadata reduce over four lanes instead of
-// eight, so each lane does that per-block work for twice the elements.
-template <bool RES, bool EXP>
-__device__ __forceinline__ void hif4_chunk16(const float (&xf)[16], int g2, bool ok, bool on, int64_t c, int64_t moff,
-                                             uint32_t *__restrict__ mcodes, uint32_t *__restrict__ mmeta,
-                                             uint32_t *__restrict__ rcodes, uint32_t *__restrict__ rmeta,
-                                             uint4 *__restrict__ m16, uint4 *__restrict__ r16)
+// The same for one lane's 8 NG elements xf (groups NG gq .. NG gq + NG - 1
+// of its 64-element block, 8 / NG lanes per block) at chunks c .. c + NG - 1:
+// the block's amax, macro scale and metadata reduce over 8 / NG lanes, so
+// each lane does that per-block work for NG times the elements of
+// hif4_chunk.
+template <int NG>
+struct CodeVec;
+template <>
+struct CodeVec<2> {
+    using T = uint2;
+    static __device__ __forceinline__ T make(const uint32_t (&c)[2]) { return make_uint2(c[0], c[1]); }
+};
+template <>
+struct CodeVec<4> {
+    using T = uint4;
+    static __device__ __forceinline__ T make(const uint32_t (&c)[4]) { return make_uint4(c[0], c[1], c[2], c[3]); }
+};
+
+template <bool RES, bool EXP, int NG>
+__device__ __forceinline__ void hif4_chunk_n(const float (&xf)[8 * NG], int gq, bool ok, bool on, int64_t c,
+                                             int64_t moff, uint32_t *__restrict__ mcodes,
+                                             uint32_t *__restrict__ mmeta, uint32_t *__restrict__ rcodes,
+                                             uint32_t *__restrict__ rmeta, uint4 *__restrict__ m16,
+                                             uint4 *__restrict__ r16)
 {
+    using CV = CodeVec<NG>;
     float am = 0.f;
 #pragma unroll
-    for (int i = 0; i < 16; i += 4)
+    for (int i = 0; i < 8 * NG; i += 4)
         am = fmax3(am, fmaxf(fabsf(xf[i]), fabsf(xf[i + 1])), fmaxf(fabsf(xf[i + 2]), fabsf(xf[i + 3])));
-    am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 1));
-    am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 2));
-    const int sb = am > 0.f ? hif4_scale_byte(am) : 0;
-    float x0[8], x1[8], d0[8], d1[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        x0[i] = xf[i];
-        x1[i] = xf[8 + i];
+    for (int o = 1; o < 8 / NG; o <<= 1)
+        am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, o));
+    const int sb = am > 0.f ? hif4_scale_byte(am) : 0;
+    float xg[NG][8], d[NG][8];
+    uint32_t code[NG], bits = 0;
+#pragma unroll
+    for (int j = 0; j < NG; ++j) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            xg[j][i] = xf[8 * j + i];
+        uint32_t b;
+        code[j] = hif4_group(xg[j], sb, NG * gq + j, b, d[j]);
+        bits |= b;
     }
-    uint32_t b0, b1;
-    const uint32_t code0 = hif4_group(x0, sb, 2 * g2, b0, d0);
-    const uint32_t code1 = hif4_group(x1, sb, 2 * g2 + 1, b1, d1);
-    uint32_t bits = am == 0.f ? 0u : (b0 | b1);   // all-zero block: metadata 0, codes keep the sign of zero
-    bits |= __shfl_xor_sync(0xFFFFFFFFu, bits, 1);
-    bits |= __shfl_xor_sync(0xFFFFFFFFu, bits, 2);
+    if (am == 0.f)
+        bits = 0;   // all-zero block: metadata 0, codes keep the sign of zero
+#pragma unroll
+    for (int o = 1; o < 8 / NG; o <<= 1)
+        bits |= __shfl_xor_sync(0xFFFFFFFFu, bits, o);
     if (ok) {
-        *reinterpret_cast<uint2 *>(mcodes + c) = make_uint2(code0, code1);
-        if (g2 == 0)
+        *reinterpret_cast<typename CV::T *>(mcodes + c) = CV::make(code);
+        if (gq == 0)
             mmeta[moff] = am == 0.f ? 0u : (bits | (uint32_t)sb);
         if (EXP) {
-            m16[c] = bf16x8_pack(d0);
-            m16[c + 1] = bf16x8_pack(d1);
+#pragma unroll
+            for (int j = 0; j < NG; ++j)
+                m16[c + j] = bf16x8_pack(d[j]);
         }
     }
     if (RES) {
-        float r0[8], r1[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            r0[i] = x0[i] - d0[i]; // exact
-            r1[i] = x1[i] - d1[i];
-        }
+        float r[NG][8];
         float ra = 0.f;
 #pragma unroll
-        for (int i = 0; i < 8; i += 4) {
-            ra = fmax3(ra, fmaxf(fabsf(r0[i]), fabsf(r0[i + 1])), fmaxf(fabsf(r0[i + 2]), fabsf(r0[i + 3])));
-            ra = fmax3(ra, fmaxf(fabsf(r1[i]), fabsf(r1[i + 1])), fmaxf(fabsf(r1[i + 2]), fabsf(r1[i + 3])));
+        for (int j = 0; j < NG; ++j) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+                r[j][i] = xg[j][i] - d[j][i]; // exact
+#pragma unroll
+            for (int i = 0; i < 8; i += 4)
+                ra = fmax3(ra, fmaxf(fabsf(r[j][i]), fabsf(r[j][i + 1])), fmaxf(fabsf(r[j][i + 2]), fabsf(r[j][i + 3])));
         }
-        ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, 1));
-        ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, 2));
+#pragma unroll
+        for (int o = 1; o < 8 / NG; o <<= 1)
+            ra = fmaxf(ra, __shfl_xor_sync(0xFFFFFFFFu, ra, o));
         const int rsb = ra > 0.f ? hif4_scale_byte(ra) : 0;
-        uint32_t rb0, rb1;
-        float e0[8], e1[8];
-        const uint32_t rcode0 = hif4_group(r0, rsb, 2 * g2, rb0, e0);
-        const uint32_t rcode1 = hif4_group(r1, rsb, 2 * g2 + 1, rb1, e1);
-        uint32_t rbits = rb0 | rb1;
-        rbits |= __shfl_xor_sync(0xFFFFFFFFu, rbits, 1);
-        rbits |= __shfl_xor_sync(0xFFFFFFFFu, rbits, 2);
+        uint32_t rcode[NG], rbits = 0;
+        float e[NG][8];
+#pragma unroll
+        for (int j = 0; j < NG; ++j) {
+            uint32_t b;
+            rcode[j] = hif4_group(r[j], rsb, NG * gq + j, b, e[j]);
+            rbits |= b;
+        }
+#pragma unroll
+        for (int o = 1; o < 8 / NG; o <<= 1)
+            rbits |= __shfl_xor_sync(0xFFFFFFFFu, rbits, o);
         if (ok) {
-            *reinterpret_cast<uint2 *>(rcodes + c) = on ? make_uint2(rcode0, rcode1) : make_uint2(0u, 0u);
-            if (g2 == 0)
+            if (!on) {
+#pragma unroll
+                for (int j = 0; j < NG; ++j)
+                    rcode[j] = 0u;
+            }
+            *reinterpret_cast<typename CV::T *>(rcodes + c) = CV::make(rcode);
+            if (gq == 0)
                 rmeta[moff] = (on && ra > 0.f) ? (rbits | (uint32_t)rsb) : 0u;
             if (EXP) {
-                r16[c] = on ? bf16x8_pack(e0) : make_uint4(0, 0, 0, 0);
-                r16[c + 1] = on ? bf16x8_pack(e1) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+                for (int j = 0; j < NG; ++j)
+                    r16[c + j] = on ? bf16x8_pack(e[j]) : make_uint4(0, 0, 0, 0);
             }
         }
     }
 }
+
+// Groups per lane in act_quant_hif4_kernel: 2 (0.092 ms on the Qwen3-VL
+// down projection) against 1 (0.100 ms, eight lanes per block) and 4
+// (0.102 ms: 115 registers, two blocks per SM).
+constexpr int kHNG = 2;
 
 template <bool RES, bool PHI, int LAYOUT, bool EXP>
 __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__restrict__ x, int64_t M, int64_t K,
@@ -319,7 +356,8 @@ __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__rest
                                                             uint4 *__restrict__ m16, uint4 *__restrict__ r16)
 {
     const int lane = threadIdx.x & 31;
-    const int g2 = lane & 3;                       // the lane's quarter of its block
+    constexpr int NG = kHNG, LPB = 8 / NG;         // groups per lane, lanes per block
+    const int gq = lane & (LPB - 1);               // the lane's place in its block
     const int kchunks = (int)(K >> 3);
     const int64_t kblocks = K >> 6;
     const int segs = (kchunks + kHSeg / 8 - 1) / (kHSeg / 8);
@@ -331,23 +369,24 @@ __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__rest
         const int64_t m = item / segs;
         const int c0 = (int)(item - m * segs) * (kHSeg / 8);
         const uint4 *xr = x + m * kchunks;
-        // two 512-element steps; lane l takes chunks 2l, 2l + 1 of each (K is a
-        // multiple of 64, so a block is wholly inside the row or past it)
+        // steps of 256 NG elements; lane l takes chunks NG l .. NG l + NG - 1
+        // of each (K is a multiple of 64, so a block is wholly inside the row
+        // or past it)
         uint4 vv[kHU];
 #pragma unroll
         for (int j = 0; j < kHU; ++j) {
-            const int c = c0 + (j >> 1) * 64 + 2 * lane + (j & 1);
+            const int c = c0 + (j / NG) * 32 * NG + NG * lane + (j % NG);
             vv[j] = c < kchunks ? __ldcs(xr + c) : make_uint4(0, 0, 0, 0);
         }
         const uint8_t *prow = PHI ? phi + (m / p_s) * phi_cols : nullptr;
 #pragma unroll
-        for (int s = 0; s < kHU / 2; ++s) {
-            const int cr = c0 + s * 64 + 2 * lane;         // first of the lane's two chunks
-            const bool ok = cr < kchunks;                  // uniform over each block's four lanes
-            float xf[16];
+        for (int s = 0; s < kHU / NG; ++s) {
+            const int cr = c0 + s * 32 * NG + NG * lane;   // first of the lane's NG chunks
+            const bool ok = cr < kchunks;                  // uniform over each block's lanes
+            float xf[8 * NG];
 #pragma unroll
-            for (int u = 0; u < 2; ++u) {
-                const uint32_t w[4] = {vv[2 * s + u].x, vv[2 * s + u].y, vv[2 * s + u].z, vv[2 * s + u].w};
+            for (int u = 0; u < NG; ++u) {
+                const uint32_t w[4] = {vv[NG * s + u].x, vv[NG * s + u].y, vv[NG * s + u].z, vv[NG * s + u].w};
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     xf[8 * u + 2 * i] = __uint_as_float(w[i] << 16);
@@ -356,8 +395,9 @@ __global__ void __launch_bounds__(256) act_quant_hif4_kernel(const uint4 *__rest
             }
             // r_s is a multiple of 64: the block lies in one phi column
             const bool on = !PHI || (ok && prow[(cr * 8) / r_s] != 0);
-            hif4_chunk16<RES, EXP>(xf, g2, ok, on, m * kchunks + cr, meta_index<LAYOUT>(m, cr >> 3, M, kblocks),
-                                   mcodes, mmeta, rcodes, rmeta, m16, r16);
+            hif4_chunk_n<RES, EXP, NG>(xf, gq, ok, on, m * kchunks + cr,
+                                       meta_index<LAYOUT>(m, cr >> 3, M, kblocks), mcodes, mmeta, rcodes, rmeta,
+                                       m16, r16);
         }
     }
 }
