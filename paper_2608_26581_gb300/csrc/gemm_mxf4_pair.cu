@@ -121,6 +121,7 @@ struct Smem {
     alignas(1024) uint8_t ystage[EPI_WARPS * YSTAGE];
     uint64_t full[STAGES];        // (even CTA) both CTAs' code copies landed
     uint64_t sf_full[STAGES];     // this CTA's scale atoms landed
+    uint64_t w4_full[STAGES];     // mixed rate: this CTA's packed W~ half landed
     uint64_t empty[STAGES];       // the stage's MMAs completed (both CTAs)
     uint64_t sf_ready[SF_SLOTS];  // (even CTA) both CTAs' scale writers filled the slot
     uint64_t acc_full;            // accumulator complete (both CTAs)
@@ -197,9 +198,10 @@ struct Mask {
 // (E2M1, 64-byte rows, 64-byte swizzle: the main product on kind::mxf4, two
 // K = 64 MMAs), X^ as E4M3 and W~ again in the padded 4-bit form (128-byte
 // rows: the residual product on kind::mxf8f6f4, E4M3 x E2M1, four K = 32
-// MMAs), into the same accumulator with the same scale words; 40 KB read
-// per stage for 768 MMA cycles against 1,024 when the main product also
-// runs on kind::mxf8f6f4.
+// MMAs), into the same accumulator with the same scale words.  The scale
+// writers expand the packed W~ tile into the padded one in shared memory,
+// so a stage reads 32 KB from L2 for 768 MMA cycles (1,024 when the main
+// product also runs on kind::mxf8f6f4).
 constexpr int F8_MIXED = 2;
 // F8 == F8_W4: the E4M3 form with W~ kept as MXFP4 -- every product on
 // kind::mxf8f6f4 as E4M3 x E2M1, W~'s tile copied from its packed codes in
@@ -248,6 +250,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&S.full[s], 1);
             mbar_init(&S.sf_full[s], 1);
+            mbar_init(&S.w4_full[s], 1);
             mbar_init(&S.empty[s], 1);
         }
         for (int i = 0; i < SF_SLOTS; ++i)
@@ -423,17 +426,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     uint64_t *sbar = &S.sf_full[slot];
                     if (F8 == F8_MIXED) {
                         // X~ and W~ packed (64-byte rows) side by side in the A tile;
-                        // with a residual, X^ as E4M3 in the R tile and W~ again, from
-                        // the same packed codes, in the padded 4-bit form in the B tile
-                        // (128-byte rows, 64 bytes read per row; its x counts codes)
+                        // with a residual, X^ as E4M3 in the R tile.  The W~ half lands
+                        // on this CTA's own barrier: its scale writers expand it into
+                        // the B tile in the padded 4-bit form the residual MMAs read
                         if (lead)
-                            mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES + (res_on ? A_BYTES + B_BYTES / 2 : 0)));
+                            mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES / 2 + (res_on ? A_BYTES : 0)));
                         tma_load_2d_pair(st.a, &tmA, bar, c0 * 64, a_y);
-                        tma_load_2d_pair(st.a + A_BYTES / 2, &tmB4, bar, c0 * 64, tc.w_row0 + (int)rank * BN_HALF);
-                        if (res_on) {
+                        mbar_arrive_expect_tx(&S.w4_full[slot], A_BYTES / 2);
+                        tma_load_2d(st.a + A_BYTES / 2, &tmB4, &S.w4_full[slot], c0 * 64,
+                                    tc.w_row0 + (int)rank * BN_HALF);
+                        if (res_on)
                             tma_load_2d_pair(st.r, &tmR, bar, cx, a_y);
-                            tma_load_2d_pair(st.b, &tmB, bar, cx, tc.w_row0 + (int)rank * BN_HALF);
-                        }
                     } else {
                         if (lead)
                             mbar_arrive_expect_tx(&S.full[slot], 2 * (A_BYTES + B_TX + (res_on ? A_BYTES : 0)));
@@ -500,6 +503,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                 // CTA's scale atoms, and (even CTA) both CTAs' codes
                 for (int q = max(0, p - STAGES); q < p; ++q) {
                     (void)mbar_wait(&S.sf_full[q % STAGES], (q / STAGES) & 1, wl);
+                    if (F8 == F8_MIXED)
+                        (void)mbar_wait(&S.w4_full[q % STAGES], (q / STAGES) & 1, wl);
                     if (lead)
                         (void)mbar_wait(&S.full[q % STAGES], (q / STAGES) & 1, wl);
                 }
@@ -945,6 +950,40 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
                     }
                     tmem_st_32x32b_x4(tb + 16 + 8 * c, vb0.x, vb0.y, vb0.z, vb0.w);
                     tmem_st_32x32b_x4(tb + 20 + 8 * c, vb1.x, vb1.y, vb1.z, vb1.w);
+                }
+                if constexpr (F8 == F8_MIXED) {
+                    // this CTA's packed W~ half (the main MMAs read it from both
+                    // CTAs, so the stage is ready only once it landed) and, for a
+                    // residual stage, its padded 4-bit copy: lane l of quarter q
+                    // takes row 32 q + l, 16-code chunk c (8 packed bytes, then an
+                    // 8-byte gap the MMA skips) to 16-byte position c ^ (row & 7)
+                    // of the 128-byte swizzled row, from the 64-byte swizzled
+                    // packed row (16-byte chunk j at j ^ ((row >> 1) & 3))
+                    if (!__all_sync(0xffffffffu, mbar_wait(&S.w4_full[slot], (p / STAGES) & 1, wl, gstat))) {
+                        if (lane == 0)
+                            flag_timeout(S, status);
+                        stop = true;
+                        return;
+                    }
+                    if (rm & 1) {
+                        const int row = q * 32 + lane;
+                        const uint32_t src = smem_u32(st.a + A_BYTES / 2) + row * 64;
+                        const uint32_t dst = smem_u32(st.b) + row * 128;
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            uint32_t w0, w1, w2, w3;
+                            asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                                         : "=r"(w0), "=r"(w1), "=r"(w2), "=r"(w3)
+                                         : "r"(src + ((j ^ ((row >> 1) & 3)) << 4)));
+                            asm volatile("st.shared.v2.u32 [%0], {%1, %2};" ::"r"(dst + (((2 * j) ^ (row & 7)) << 4)),
+                                         "r"(w0), "r"(w1)
+                                         : "memory");
+                            asm volatile("st.shared.v2.u32 [%0], {%1, %2};" ::"r"(dst + (((2 * j + 1) ^ (row & 7)) << 4)),
+                                         "r"(w2), "r"(w3)
+                                         : "memory");
+                        }
+                        fence_proxy_async_smem();   // generic-proxy writes, read by the MMAs
+                    }
                 }
                 tmem_st_wait();
                 tc_fence_before();
