@@ -347,9 +347,9 @@ RFQ_API rfq_status rfq_fp4_mma_peak(int32_t cta_pair, int64_t iters, void *works
  * residual product X^ W~ on the FP8 one (E4M3 x E2M1), into one fp32
  * accumulator per output tile.  xq: X~, MXFP4 [M x K]; xr: X^, MXFP8 [M x K]
  * (rfq_quantize_act with an MXFP8 residual writes both); wq: W~, MXFP4
- * [N x K], its codes 32-byte aligned: the kernel reads them twice per
- * k-stage, packed for the main product and expanded by the copy engine to
- * one byte per code for the residual one (no second copy of W~ in memory).
+ * [N x K]: the kernel reads its packed codes once per k-stage and expands
+ * them in shared memory to the one-byte-per-code form the residual MMAs
+ * read (no second copy of W~ in memory).
  * Every operand with RFQ_SCALE_MMA scales; K % 128 == 0, N % 16 == 0,
  * M >= 0 (CTA pairs at every M).  phi, phi_r_s, y, out_dtype, workspace: as
  * for rfq_linear.  rfq_linear multiplies the same RFQ with X~ and W~

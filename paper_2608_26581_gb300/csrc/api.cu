@@ -624,9 +624,7 @@ rfq_status rfq_linear_mixed(const rfq_qtensor *xq, const rfq_qtensor *xr, const 
         return RFQ_ERR_SHAPE;
     if (phi && (phi_r_s < 128 || phi_r_s % 128 != 0))
         return RFQ_ERR_SHAPE;
-    // W~'s codes feed a TMA copy of the padded 4-bit type, which wants a
-    // 32-byte aligned base
-    if (!aligned16(y) || !aligned16(workspace) || (reinterpret_cast<uintptr_t>(wq->codes) & 31u) != 0)
+    if (!aligned16(y) || !aligned16(workspace))
         return RFQ_ERR_ALIGNMENT;
     if ((s = check_device()) != RFQ_OK)
         return s;

@@ -1144,8 +1144,8 @@ cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
     CUtensorMap ta, tr, tb, ty;
     if (a.b4_codes) {
         // the mixed-rate FP4-to-FP8 residual: X~ and W~ packed (64-byte boxes,
-        // 64-byte swizzle), X^ as E4M3 (128-byte boxes), W~ once more from
-        // the same codes in the padded 4-bit form (128-code boxes)
+        // 64-byte swizzle), X^ as E4M3 (128-byte boxes); the kernel makes
+        // the padded 4-bit W~ tile itself, so no map reads W~ in that form
         if (!a.r_codes || a.groups > 0 || a.fq_x || a.prof)
             return cudaErrorInvalidValue;
         CUtensorMap tb4;
@@ -1153,9 +1153,9 @@ cudaError_t launch_gemm_mxf4_pair(const GemmMxf4Args &a, cudaStream_t st)
         if (!encode_tmap_2d_u8(&ta, a.a_codes, kp, (uint64_t)a.M, kp, 64, BM, 64) ||
             !encode_tmap_2d_u8(&tb4, a.b4_codes, kp, (uint64_t)a.N, kp, 64, BN_HALF, 64) ||
             !encode_tmap_2d_u8(&tr, a.r_codes, k8, (uint64_t)a.M, k8, ROW, BM, 128) ||
-            !encode_tmap_2d_e2m1_padded(&tb, a.b4_codes, k8, (uint64_t)a.N, BN_HALF) ||
             !encode_tmap_2d_u8(&ty, a.y, yrow, (uint64_t)a.M, yrow, 64, 32, 64))
             return cudaErrorInvalidValue;
+        tb = tb4;   // (unused by this form)
         const bool phi = a.phi != nullptr && a.K / 128 <= REC_WORDS * 32;
         if (phi)
             return a.out_bf16 ? launch_variant<true, true, true, F8_MIXED, false>(ta, tr, tb, ty, a, st, &tb4)

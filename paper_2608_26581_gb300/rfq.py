@@ -210,7 +210,7 @@ def rfq_linear(xq: QTensor, xr: QTensor | None, phi: torch.Tensor | None, phi_r_
 def rfq_linear_mixed(xq: QTensor, xr: QTensor, phi: torch.Tensor | None, phi_r_s: int, wq: QTensor,
                      y: torch.Tensor, out_dtype: int, workspace: torch.Tensor, stream=None):
     """The FP4-to-FP8 RFQ with the main product at the FP4 rate: X~ (MXFP4),
-    X^ (MXFP8), W~ (MXFP4, codes 32-byte aligned; see include/rfq.h)."""
+    X^ (MXFP8), W~ (MXFP4; see include/rfq.h)."""
     q, r, w = xq.c(), xr.c(), wq.c()
     _check(load_library().rfq_linear_mixed(ctypes.byref(q), ctypes.byref(r), _ptr(phi), phi_r_s, ctypes.byref(w),
                                            _ptr(y), out_dtype, _ptr(workspace), _stream(stream)),

@@ -193,9 +193,10 @@ def test_debug_bounds_is_the_debug_builds(lib):
 
 def test_fp8_activations_with_fp4_weight_host_checks(lib):
     """MXFP8 activations may meet an MXFP4 W~ (multiplied as E2M1 from its
-    packed codes): rfq_linear, rfq_linear_grouped and rfq_linear_mixed reject
-    on the host a W~ whose codes are not 32-byte aligned (the padded 4-bit
-    copy's rule) and, for rfq_linear, K not a multiple of 128; nothing here
+    packed codes): rfq_linear and rfq_linear_grouped reject on the host a W~
+    whose codes are not 32-byte aligned (the padded 4-bit copy's rule) and,
+    for rfq_linear, K not a multiple of 128; rfq_linear_mixed (which makes
+    its padded copy in shared memory) wants the usual 16 bytes; nothing here
     reaches the device check, since the pointers are not device memory."""
     from paper_2608_26581_gb300 import rfq
     P, r = ctypes.c_void_p, ctypes.byref
@@ -210,7 +211,8 @@ def test_fp8_activations_with_fp4_weight_host_checks(lib):
     wg_off = rfq._QT(rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA, 2 * N, K, 48, 32)
     assert lib.rfq_linear_grouped(r(x8), None, None, 256, P(16), 2, r(wg_off), N, P(16), 1, P(16), None) == \
         rfq.RFQ_ERR_ALIGNMENT
-    assert lib.rfq_linear_mixed(r(x4), r(x8), None, 256, r(w4_off), P(16), 1, P(16), None) == \
+    w4_8 = rfq._QT(rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA, N, K, 40, 32)       # 8 mod 16
+    assert lib.rfq_linear_mixed(r(x4), r(x8), None, 256, r(w4_8), P(16), 1, P(16), None) == \
         rfq.RFQ_ERR_ALIGNMENT
     # an MXFP8 W~ under MXFP4 activations stays an invalid pairing
     w8 = rfq._QT(rfq.RFQ_FMT_MXFP8, rfq.RFQ_SCALE_MMA, N, K, 32, 32)

@@ -275,8 +275,10 @@ def test_mixed_rate_matches_all_e4m3_path(orc):
 
 
 def test_mixed_rate_host_checks():
-    """rfq_linear_mixed wants MXFP4 X~ and W~, an MXFP8 X^, one K, and W~'s
-    codes on a 32-byte boundary (the padded 4-bit copy's rule)."""
+    """rfq_linear_mixed wants MXFP4 X~ and W~, an MXFP8 X^ and one K; W~'s
+    codes need only the 16-byte alignment of every operand (its padded copy
+    is made in shared memory), so a 16-byte offset computes as the aligned
+    tensor does."""
     M, K, N = 256, 256, 256
     x4, w4 = rfq.empty_qtensor(F4, MMA, M, K), rfq.empty_qtensor(F4, MMA, N, K)
     x8, w8 = rfq.empty_qtensor(F8, MMA, M, K), rfq.empty_qtensor(F8, MMA, N, K)
@@ -289,13 +291,19 @@ def test_mixed_rate_host_checks():
     with pytest.raises(rfq.RFQError) as e:
         rfq.rfq_linear_mixed(x4, x8, None, 256, rfq.empty_qtensor(F4, MMA, N, 512), y, rfq.RFQ_OUT_F32, ws)
     assert e.value.status == rfq.RFQ_ERR_SHAPE
-    # the same W~ codes 16 bytes off a 32-byte boundary
+    # the same W~ codes 16 bytes off a 32-byte boundary give the same Y
+    x = to_dev_bf16(make_activation(ActSpec(M, K, "normal", seed=3)))
+    rfq.rfq_quantize_weight(to_dev_bf16(make_weight(K, N, seed=4)), w4)
+    rfq.rfq_quantize_act(x, x4, x8, None)
     buf = torch.zeros(w4.codes.numel() + 16, dtype=torch.uint8, device=DEV)
     assert buf.data_ptr() % 32 == 0
-    w_off = rfq.QTensor(w4.fmt, w4.scale_layout, N, K, buf[16:16 + w4.codes.numel()], w4.scales)
-    with pytest.raises(rfq.RFQError) as e:
-        rfq.rfq_linear_mixed(x4, x8, None, 256, w_off, y, rfq.RFQ_OUT_F32, ws)
-    assert e.value.status == rfq.RFQ_ERR_ALIGNMENT
+    buf[16:].copy_(w4.codes)
+    w_off = rfq.QTensor(w4.fmt, w4.scale_layout, N, K, buf[16:], w4.scales)
+    y0, y1 = torch.empty(M, N, device=DEV), torch.empty(M, N, device=DEV)
+    rfq.rfq_linear_mixed(x4, x8, None, 256, w4, y0, rfq.RFQ_OUT_F32, ws)
+    rfq.rfq_linear_mixed(x4, x8, None, 256, w_off, y1, rfq.RFQ_OUT_F32, ws)
+    assert rfq.rfq_workspace_status(ws) == rfq.RFQ_OK
+    assert torch.equal(y0, y1)
 
 
 def test_fp8_residual_is_closer_than_fp4_residual(orc):
