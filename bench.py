@@ -650,7 +650,34 @@ def run_rfq(args):
     # device X / Y, so step i's device work overlaps the copies of steps
     # i - 1 and i + 1 (the copy engines give ~200 GB/s per direction).
     e2e_ms = None
-    if not args.no_e2e:
+    # the two-kernel MXFP4 linear has a C entry point that takes the host
+    # buffers itself (rfq_linear_host: row chunks, copies on its own
+    # streams); the other variants run the loop below
+    host_api = not (quant_only or hif4 or fused or grouped or f8)
+    e2e_api = None
+    if not args.no_e2e and host_api:
+        _nv = _Nvtx("rfq end-to-end loop (rfq_linear_host)")
+        _nv.__enter__()
+        bs = bufs[0]
+        mode = rfq.RFQ_FALLBACK_AMAX if amax_phi else (rfq.RFQ_FALLBACK_NONE if no_res else rfq.RFQ_FALLBACK_ALL)
+        tau = args.phi_tau if amax_phi else 0.0
+        yh = y_host[:, :N] if y_host.shape[1] != N else y_host
+        total = args.warmup + args.steps
+        for i in range(total):
+            if i == args.warmup:
+                barrier()
+                torch.cuda.synchronize()
+                e0, e1 = ev(), ev()
+                e0.record(stream)
+            rfq.rfq_linear_host(x_host, wop, yh, rfq.RFQ_OUT_BF16, bs["x"], bs["xq"], bs["xr"], bs["phi"],
+                                bs["y"], wsp, mode=mode, tau=tau, chunk_rows=args.e2e_chunk_rows, stream=stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        e2e_ms = e0.elapsed_time(e1) / args.steps
+        e2e_api = f"rfq_linear_host (C ABI, pinned host X and Y, {args.e2e_chunk_rows}-row chunks)"
+        _nv.__exit__()
+    if not args.no_e2e and not host_api:
         _nv = _Nvtx("rfq end-to-end loop (host buffers)")
         _nv.__enter__()
         h2d, d2h = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
@@ -781,7 +808,9 @@ def run_rfq(args):
     clocks = clk.summary(h0, h1)
     if e2e_ms is not None:
         e2e = {"value": _job_rate(aq_bytes / 1e9 if quant_only else flop / 1e12, ws, e2e_ms), "unit": unit,
-               "ms_per_step": e2e_ms, "h2d_bytes_per_step": Mb * K * 2,
+               "ms_per_step": e2e_ms, "api": e2e_api or ("rfq entry points on device buffers, host copies on "
+                                                         "copy streams (double-buffered across steps)"),
+               "h2d_bytes_per_step": Mb * K * 2,
                "d2h_bytes_per_step": q_bytes if quant_only else Mb * N * 2}
     else:
         e2e = None
@@ -935,6 +964,8 @@ def main():
     ap.add_argument("--impl", default="rfq", choices=["rfq", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffer) timing")
+    ap.add_argument("--e2e-chunk-rows", type=int, default=2048,
+                    help="row chunk of rfq_linear_host in the end-to-end timing (a multiple of 128)")
     ap.add_argument("--rows", type=int, default=0, help="profile a smaller case: the first ROWS token rows")
     ap.add_argument("--phi-tau", type=float, default=None,
                     help="selective fallback: residual only on 128 x 256 tiles whose max |x| exceeds TAU")

@@ -235,6 +235,43 @@ RFQ_API rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, cons
                       int32_t phi_r_s, const rfq_qtensor *wq, void *y, int32_t out_dtype,
                       void *workspace, void *stream);
 
+/* The RFQ linear layer end to end from host memory (Algorithm 1, Eq. rfq,
+ * with X and Y in host memory): Y = X~ W~ + phi X^ W~ for a bf16 X on the
+ * host.  The call copies X to the device, quantizes it (rfq_quantize_act,
+ * MXFP4 main and residual pathways per fb), multiplies it by wq (rfq_linear)
+ * and copies Y back, in chunks of chunk_rows rows: each chunk's
+ * host-to-device copy runs on a copy stream of the library's, its two
+ * kernels on `stream`, its device-to-host copy on a second copy stream, so
+ * the copies of one chunk overlap the kernels and copies of the others.
+ * `stream` then waits for the copy streams: y_host is complete once the
+ * stream has passed the call (the call itself returns after enqueueing).
+ * Y equals rfq_linear's on the same operands bit for bit (row chunking
+ * does not change any output element's accumulation).
+ *   x_host: host bf16 [M][K] row-major; page-locked memory lets the copies
+ *           run asynchronously (pageable memory works, with copies that
+ *           then block the host).
+ *   y_host: host [M][N] row-major, bf16 or fp32 per out_dtype.
+ *   fb: NULL (= RFQ_FALLBACK_ALL), RFQ_FALLBACK_NONE (plain W4A4; xr NULL)
+ *       or RFQ_FALLBACK_AMAX with p_s = 128 and r_s a multiple of 128.
+ *   wq: MXFP4 W~ [N x K] with RFQ_SCALE_MMA (device).
+ *   chunk_rows: a multiple of 128; 0 selects 8192.  M = 0 does nothing
+ *   (the host and device buffers may then be NULL).
+ *   Device scratch, all the caller's (the library allocates no device
+ *   memory; it creates two copy streams per device, kept for the process,
+ *   and a few events per call): x_dev bf16 [M][K] (16-byte aligned); xq, xr
+ *   MXFP4 qtensors of M x K with RFQ_SCALE_MMA (xr NULL exactly when fb is
+ *   RFQ_FALLBACK_NONE); phi [ceil(M/128)][ceil(K/r_s)] bytes with
+ *   RFQ_FALLBACK_AMAX, else ignored; y_dev [M][N]; workspace as for
+ *   rfq_linear.  Nothing else may use these buffers until `stream` has
+ *   passed the call.
+ * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
+ * RFQ_ERR_UNSUPPORTED (other formats or layouts), RFQ_ERR_CUDA,
+ * RFQ_ERR_DEVICE; every check happens before the first copy is enqueued. */
+RFQ_API rfq_status rfq_linear_host(const void *x_host, int64_t M, int64_t K, const rfq_fallback *fb,
+                                   const rfq_qtensor *wq, void *y_host, int32_t out_dtype, int64_t chunk_rows,
+                                   void *x_dev, rfq_qtensor *xq, rfq_qtensor *xr, uint8_t *phi, void *y_dev,
+                                   void *workspace, void *stream);
+
 /* Workspace bytes rfq_linear_fused needs for an M x K activation and the
  * fallback mode fb (NULL = RFQ_FALLBACK_ALL); 0 for sizes it rejects
  * (K % 128 != 0).  For M <= 128 it is rfq_linear_workspace_bytes(); beyond,

@@ -31,7 +31,7 @@ EXPORTED = ("rfq_status_string", "rfq_qtensor_bytes", "rfq_quantize_weight", "rf
             "rfq_linear_workspace_bytes", "rfq_linear", "rfq_workspace_status", "rfq_dequant",
             "rfq_linear_noalloc", "rfq_linear_fused", "rfq_convert", "rfq_linear_grouped", "rfq_check_finite",
             "rfq_quantize_act_expand", "rfq_fp4_mma_peak", "rfq_linear_fused_workspace_bytes",
-            "rfq_linear_profile", "rfq_debug_bounds", "rfq_linear_mixed")
+            "rfq_linear_profile", "rfq_debug_bounds", "rfq_linear_mixed", "rfq_linear_host")
 
 
 class RFQError(RuntimeError):
@@ -94,6 +94,8 @@ def load_library(path: str = LIB_PATH):
         lib.rfq_linear_fused_workspace_bytes.argtypes = [I64, I64, ctypes.POINTER(_FB)]
         lib.rfq_linear_mixed.restype = I32
         lib.rfq_linear_mixed.argtypes = [QTP, QTP, P, I32, QTP, P, I32, P, P]
+        lib.rfq_linear_host.restype = I32
+        lib.rfq_linear_host.argtypes = [P, I64, I64, ctypes.POINTER(_FB), QTP, P, I32, I64, P, QTP, QTP, P, P, P, P]
         lib.rfq_debug_bounds.restype = I32
         lib.rfq_debug_bounds.argtypes = [ctypes.POINTER(I32), I32]
         lib.rfq_linear_profile.restype = I32
@@ -215,6 +217,24 @@ def rfq_linear_mixed(xq: QTensor, xr: QTensor, phi: torch.Tensor | None, phi_r_s
     _check(load_library().rfq_linear_mixed(ctypes.byref(q), ctypes.byref(r), _ptr(phi), phi_r_s, ctypes.byref(w),
                                            _ptr(y), out_dtype, _ptr(workspace), _stream(stream)),
            "rfq_linear_mixed")
+
+
+def rfq_linear_host(x_host: torch.Tensor, wq: QTensor, y_host: torch.Tensor, out_dtype: int, x_dev: torch.Tensor,
+                    xq: QTensor, xr: QTensor | None, phi: torch.Tensor | None, y_dev: torch.Tensor,
+                    workspace: torch.Tensor, mode: int = RFQ_FALLBACK_ALL, tau: float = 0.0, r_s: int = 256,
+                    chunk_rows: int = 0, stream=None):
+    """The RFQ linear layer from host memory: x_host (CPU bf16 [M][K],
+    pinned for overlapped copies) in, y_host (CPU [M][N]) out; x_dev, xq,
+    xr, phi, y_dev and workspace are the caller's device scratch (see
+    include/rfq.h)."""
+    M, K = x_host.shape
+    fb = _FB(mode, tau, 128, r_s)
+    w, q = wq.c(), xq.c()
+    r = xr.c() if xr is not None else None
+    _check(load_library().rfq_linear_host(_ptr(x_host), M, K, ctypes.byref(fb), ctypes.byref(w), _ptr(y_host),
+                                          out_dtype, chunk_rows, _ptr(x_dev), ctypes.byref(q),
+                                          ctypes.byref(r) if r is not None else None, _ptr(phi), _ptr(y_dev),
+                                          _ptr(workspace), _stream(stream)), "rfq_linear_host")
 
 
 def rfq_workspace_status(workspace: torch.Tensor, clear: bool = False, stream=None) -> int:

@@ -217,3 +217,33 @@ def test_fp8_activations_with_fp4_weight_host_checks(lib):
     # an MXFP8 W~ under MXFP4 activations stays an invalid pairing
     w8 = rfq._QT(rfq.RFQ_FMT_MXFP8, rfq.RFQ_SCALE_MMA, N, K, 32, 32)
     assert lib.rfq_linear(r(x4), None, None, 256, r(w8), P(16), 1, P(16), None) == rfq.RFQ_ERR_INVALID_ARG
+
+
+def test_linear_host_host_checks(lib):
+    """rfq_linear_host validates on the host before any copy is enqueued:
+    null buffers, a chunk size that is not a multiple of 128, a residual
+    qtensor that does not match the fallback mode, formats other than MXFP4
+    and a misaligned x_dev; none of these calls reaches the device."""
+    from paper_2608_26581_gb300 import rfq
+    P, r = ctypes.c_void_p, ctypes.byref
+    M, K, N = 256, 256, 256
+    xq = rfq._QT(rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA, M, K, 32, 32)
+    wq = rfq._QT(rfq.RFQ_FMT_MXFP4, rfq.RFQ_SCALE_MMA, N, K, 32, 32)
+    hq = rfq._QT(rfq.RFQ_FMT_HIF4, rfq.RFQ_SCALE_MMA, M, K, 32, 32)
+    none = rfq._FB(rfq.RFQ_FALLBACK_NONE, 0.0, 128, 256)
+    call = lib.rfq_linear_host
+    H = P(4096)   # stands for a host buffer
+    assert call(None, M, K, None, r(wq), H, 0, 0, P(16), r(xq), r(xq), None, P(16), P(16), None) == \
+        rfq.RFQ_ERR_INVALID_ARG
+    assert call(H, M, K, None, r(wq), None, 0, 0, P(16), r(xq), r(xq), None, P(16), P(16), None) == \
+        rfq.RFQ_ERR_INVALID_ARG
+    assert call(H, M, K, None, r(wq), H, 0, 100, P(16), r(xq), r(xq), None, P(16), P(16), None) == \
+        rfq.RFQ_ERR_SHAPE
+    assert call(H, M, K, r(none), r(wq), H, 0, 0, P(16), r(xq), r(xq), None, P(16), P(16), None) == \
+        rfq.RFQ_ERR_INVALID_ARG
+    assert call(H, M, K, None, r(wq), H, 0, 0, P(16), r(xq), None, None, P(16), P(16), None) == \
+        rfq.RFQ_ERR_INVALID_ARG
+    assert call(H, M, K, None, r(wq), H, 0, 0, P(16), r(hq), r(hq), None, P(16), P(16), None) == \
+        rfq.RFQ_ERR_UNSUPPORTED
+    assert call(H, M, K, None, r(wq), H, 0, 0, P(8), r(xq), r(xq), None, P(16), P(16), None) == \
+        rfq.RFQ_ERR_ALIGNMENT
