@@ -263,7 +263,8 @@ RFQ_API rfq_status rfq_linear(const rfq_qtensor *xq, const rfq_qtensor *xr, cons
  *   RFQ_FALLBACK_NONE); phi [ceil(M/128)][ceil(K/r_s)] bytes with
  *   RFQ_FALLBACK_AMAX, else ignored; y_dev [M][N]; workspace as for
  *   rfq_linear.  Nothing else may use these buffers until `stream` has
- *   passed the call.
+ *   passed the call.  Calls on one device share the two copy streams, so
+ *   the copies of concurrent calls run one after another.
  * Errors: RFQ_ERR_INVALID_ARG, RFQ_ERR_SHAPE, RFQ_ERR_ALIGNMENT,
  * RFQ_ERR_UNSUPPORTED (other formats or layouts), RFQ_ERR_CUDA,
  * RFQ_ERR_DEVICE; every check happens before the first copy is enqueued. */
