@@ -213,43 +213,6 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap *m, const void *s
                  : "memory");
 }
 
-// L2 cache policies for the copies below: evict_first for data read or
-// written once (it leaves L2 first), evict_last for data many CTAs re-read.
-__device__ __forceinline__ uint64_t l2_policy_evict_first()
-{
-    uint64_t p;
-    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
-    return p;
-}
-
-__device__ __forceinline__ uint64_t l2_policy_evict_last()
-{
-    uint64_t p;
-    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-    return p;
-}
-
-// tma_store_2d with an L2 cache policy.
-__device__ __forceinline__ void tma_store_2d_hint(const CUtensorMap *m, const void *src, int32_t x, int32_t y,
-                                                  uint64_t policy)
-{
-    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group.L2::cache_hint [%0, {%2, %3}], [%1], %4;" ::"l"(
-                     reinterpret_cast<uint64_t>(m)),
-                 "r"(smem_u32(src)), "r"(x), "r"(y), "l"(policy)
-                 : "memory");
-}
-
-// tma_load_2d_pair with an L2 cache policy.
-__device__ __forceinline__ void tma_load_2d_pair_hint(void *dst, const CUtensorMap *m, uint32_t cbar, int32_t x,
-                                                      int32_t y, uint64_t policy)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
-        " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
-        "l"(reinterpret_cast<uint64_t>(m)), "r"(cbar), "r"(x), "r"(y), "l"(policy)
-        : "memory");
-}
-
 __device__ __forceinline__ void bulk_commit_group()
 {
     asm volatile("cp.async.bulk.commit_group;" ::: "memory");
@@ -421,26 +384,11 @@ __device__ __forceinline__ void tc_mma_f16(uint32_t d_tmem, uint64_t a_desc, uin
         : "memory");
 }
 
-// Copy 32 rows x 16 bytes from shared memory into TMEM, replicated into the
-// four 32-lane quarters of the TMEM columns at `taddr`.
-__device__ __forceinline__ void tc_cp_32x128b_warpx4(uint32_t taddr, uint64_t sdesc)
-{
-    asm volatile("tcgen05.cp.cta_group::1.32x128b.warpx4 [%0], %1;" ::"r"(taddr), "l"(sdesc) : "memory");
-}
-
 // Each thread of the warp writes 4 consecutive 32-bit columns of its TMEM lane.
 __device__ __forceinline__ void tmem_st_32x32b_x4(uint32_t taddr, uint32_t r0, uint32_t r1, uint32_t r2, uint32_t r3)
 {
     asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr), "r"(r0), "r"(r1),
                  "r"(r2), "r"(r3)
-                 : "memory");
-}
-
-// Each thread of the warp writes 8 consecutive 32-bit columns of its TMEM lane.
-__device__ __forceinline__ void tmem_st_32x32b_x8(uint32_t taddr, const uint32_t (&r)[8])
-{
-    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"r"(taddr),
-                 "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
                  : "memory");
 }
 
@@ -495,17 +443,6 @@ __device__ __forceinline__ uint64_t sdesc_k_sw64(uint32_t saddr)
     d |= (uint64_t)(512 >> 4) << 32;             // stride byte offset: 8 rows x 64 B
     d |= (uint64_t)1 << 46;
     d |= (uint64_t)4 << 61;                      // 64-byte swizzle
-    return d;
-}
-
-// Descriptor of an unswizzled block of 16-byte rows (8-row core matrices,
-// 128 bytes apart), as read by tcgen05.cp 32x128b.
-__device__ __forceinline__ uint64_t sdesc_rows16(uint32_t saddr)
-{
-    uint64_t d = 0;
-    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
-    d |= (uint64_t)(128 >> 4) << 32;
-    d |= (uint64_t)1 << 46;
     return d;
 }
 
