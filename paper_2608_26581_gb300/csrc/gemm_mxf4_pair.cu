@@ -784,19 +784,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PHI ? THREADS + 32 :
             if (OUT_BF16) {
                 // all 128 columns of this warp into registers as packed bf16
                 uint32_t pk[64];
+                {
+                    // all four 32-column loads in flight, one wait
+                    uint32_t v[4][32];
 #pragma unroll
-                for (int g = 0; g < 2; ++g) {
-                    uint32_t v[2][32];
-                    tmem_ld_32x32b_x32(tcol + 64 * g, v[0]);
-                    tmem_ld_32x32b_x32(tcol + 64 * g + 32, v[1]);
+                    for (int c = 0; c < 4; ++c)
+                        tmem_ld_32x32b_x32(tcol + 32 * c, v[c]);
                     tmem_ld_wait();
 #pragma unroll
-                    for (int c = 0; c < 2; ++c)
+                    for (int c = 0; c < 4; ++c)
 #pragma unroll
                         for (int i = 0; i < 16; ++i) {
                             __nv_bfloat162 b2 = __floats2bfloat162_rn(__uint_as_float(v[c][2 * i]),
                                                                       __uint_as_float(v[c][2 * i + 1]));
-                            pk[32 * g + 16 * c + i] = *reinterpret_cast<uint32_t *>(&b2);
+                            pk[16 * c + i] = *reinterpret_cast<uint32_t *>(&b2);
                         }
                 }
                 release();
