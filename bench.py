@@ -53,6 +53,7 @@ def _peaks():
 # sources they were taken on (the kernel's file plus the shared headers)
 _KERNEL_SRC = {"gemm_mxf4_kernel": "gemm_mxf4.cu", "gemm_mxf4_pair_kernel": "gemm_mxf4_pair.cu",
                "act_quant8_kernel": "quant_mxfp8.cu", "act_quant_rfq8_amax_kernel": "quant_mxfp8.cu",
+               "act_quant_rfq8_kernel": "quant_mxfp8.cu",
                "gemm_mxf4_fused_kernel": "gemm_mxf4_fused.cu",
                "act_quant_mxfp4_kernel": "quant_mxfp4.cu", "act_quant_mxfp4_amax_kernel": "quant_mxfp4.cu",
                "gemm_hif4_kernel": "gemm_hif4.cu", "act_quant_hif4_kernel": "quant_hif4.cu",
@@ -109,7 +110,7 @@ def _src_hash(kernel: str):
     d = os.path.join(HERE, "paper_2608_26581_gb300", "csrc")
     m = hashlib.sha256()
     extra = ("mxfp4_math.cuh",) if kernel in ("act_quant_mxfp4_kernel", "act_quant_mxfp4_amax_kernel",
-                                              "gemm_mxf4_fused_kernel", "act_quant8_kernel",
+                                              "gemm_mxf4_fused_kernel", "act_quant8_kernel", "act_quant_rfq8_kernel",
                                               "act_quant_rfq8_amax_kernel", "gemm_mxf4_pair_kernel") else ()
     for n in (_KERNEL_SRC[kernel], "ptx.cuh", "internal.h") + extra:
         m.update(open(os.path.join(d, n), "rb").read())
@@ -770,7 +771,8 @@ def run_rfq(args):
     elif f8:
         aq_bytes = _act_quant_bytes(Mb, K, "rfq8" if scheme in ("rfq8", "rfq8mix") else "mxfp8",
                                     scheme in ("rfq8", "rfq8mix"), operand=scheme == "rfq8")
-        aq_kernel = "act_quant_rfq8_amax_kernel" if amax_fused else "act_quant8_kernel"
+        aq_kernel = ("act_quant_rfq8_amax_kernel" if amax_fused else
+                     "act_quant_rfq8_kernel" if scheme == "rfq8mix" else "act_quant8_kernel")
     else:
         aq_bytes = _act_quant_bytes(Mb, K, "mxfp4", not no_res)
         # AMAX phi on 128 x 256 tiles: phi and the quantization in one kernel
